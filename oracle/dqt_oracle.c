@@ -1,0 +1,371 @@
+/*
+ * Direct Quantized Training (DQT) -- CPU oracle.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the slow, obviously-correct
+ * statement of what the DQT BitLinear training step computes.  Only the test
+ * suite, the smoke check and the CPU-baseline leg of the benchmark may load
+ * it.  The CUDA library never includes, links or calls it, and it includes
+ * nothing from the CUDA library.
+ *
+ * Paper: "Direct Quantized Training of Language Models with Stochastic
+ * Rounding" (Zhao et al., ACML 2025, arXiv 2412.04787).
+ *
+ *   Eq. 1   stochastic rounding SR(x)                     -> dqt_oracle_sr
+ *   Eq. 2-4 AbsMean grid, scale and initial codes         -> dqt_oracle_absmean_init
+ *   Sec 3.2 8-bit activation quantisation (BitNet style)  -> dqt_oracle_act_quant
+ *   Sec 3.2 BitLinear forward on the quantised operands   -> dqt_oracle_fwd
+ *   Sec 3.2 backward w.r.t. the low-bit weight (no STE)   -> dqt_oracle_bwd_dx / _bwd_dw
+ *   Sec 4.1 AdamW producing the dense target W'           -> dqt_oracle_adamw_x
+ *   Eq. 5   W_hat = SR(W'), kept on the n-bit grid        -> dqt_oracle_update
+ *   Sec 5.1 absmax / round-to-nearest ablation            -> round_mode = 1
+ *
+ * Readings where the paper is silent (each is listed in the design notes):
+ *   - ternary ("1.58 bit") means the grid [-1, 1] with s = 1 / AbsMean;
+ *     integer n uses Q_n = -2^(n-1), Q_p = 2^(n-1) - 1 literally;
+ *   - the scale s is fixed at initialisation and SR acts on the code domain
+ *     x = W' * s, followed by a clamp to [Q_n, Q_p];
+ *   - Round() is round-half-to-even;
+ *   - activations: per-token absmax, s_x = 127 / max(amax, 1e-5),
+ *     q = clamp(rint(x * s_x), -128, 127);
+ *   - the RNG is Philox4x32-10 (Salmon et al., SC'11) keyed by the seed, with
+ *     the counter (element/4, step, tensor id) and word element%4; a uniform
+ *     U = (word >> 8) * 2^-24 rounds up when U < x - floor(x).
+ *
+ * Arithmetic: the reductions of the GEMMs are exact (int64) or fp64; the
+ * AdamW + SR step is a fixed sequence of individually rounded IEEE fp32
+ * operations (build with -ffp-contract=off so that no FMA is formed).
+ *
+ * Parity of every function here is pinned by tests/test_oracle_*.py against
+ * facts fixed by the paper and by mathematics (hand-worked examples, closed
+ * forms, exact enumeration, published Philox known-answer vectors).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <string.h>
+
+/* ------------------------------------------------------------------------ */
+/* bf16 <-> fp32 (IEEE round-to-nearest-even on the dropped 16 bits).        */
+/* ------------------------------------------------------------------------ */
+static float bf16_to_f32(uint16_t h) {
+  uint32_t u = (uint32_t)h << 16;
+  float f;
+  memcpy(&f, &u, 4);
+  return f;
+}
+
+static uint16_t f32_to_bf16_rne(float f) {
+  uint32_t u;
+  memcpy(&u, &f, 4);
+  if ((u & 0x7f800000u) == 0x7f800000u && (u & 0x007fffffu) != 0)
+    return (uint16_t)((u >> 16) | 0x0040u); /* quiet NaN */
+  uint32_t lsb = (u >> 16) & 1u;
+  u += 0x7fffu + lsb;
+  return (uint16_t)(u >> 16);
+}
+
+uint16_t dqt_oracle_f32_to_bf16(float f) { return f32_to_bf16_rne(f); }
+
+/* ------------------------------------------------------------------------ */
+/* Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel random numbers: as   */
+/* easy as 1, 2, 3", SC'11).  One round: two 32x32->64 multiplications of    */
+/* counter words 0 and 2 by the Philox multipliers, then a permutation that  */
+/* xors the high halves with the other counter words and the round key.      */
+/* The key is bumped by the Weyl constants between rounds.                   */
+/* ------------------------------------------------------------------------ */
+#define PHILOX_M0 0xD2511F53u
+#define PHILOX_M1 0xCD9E8D57u
+#define PHILOX_W0 0x9E3779B9u
+#define PHILOX_W1 0xBB67AE85u
+
+void dqt_oracle_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2],
+                              uint32_t out[4]) {
+  uint32_t c0 = ctr[0], c1 = ctr[1], c2 = ctr[2], c3 = ctr[3];
+  uint32_t k0 = key[0], k1 = key[1];
+  for (int round = 0; round < 10; ++round) {
+    if (round > 0) {
+      k0 += PHILOX_W0;
+      k1 += PHILOX_W1;
+    }
+    uint64_t p0 = (uint64_t)PHILOX_M0 * (uint64_t)c0;
+    uint64_t p1 = (uint64_t)PHILOX_M1 * (uint64_t)c2;
+    uint32_t hi0 = (uint32_t)(p0 >> 32), lo0 = (uint32_t)p0;
+    uint32_t hi1 = (uint32_t)(p1 >> 32), lo1 = (uint32_t)p1;
+    uint32_t n0 = hi1 ^ c1 ^ k0;
+    uint32_t n1 = lo1;
+    uint32_t n2 = hi0 ^ c3 ^ k1;
+    uint32_t n3 = lo0;
+    c0 = n0; c1 = n1; c2 = n2; c3 = n3;
+  }
+  out[0] = c0; out[1] = c1; out[2] = c2; out[3] = c3;
+}
+
+/* The uniform variate that drives the rounding of element e (flat row-major
+ * index into the weight tensor) at a given (seed, step, tensor id).  Returns
+ * the raw 32-bit word; the uniform is (word >> 8) * 2^-24. */
+uint32_t dqt_oracle_sr_word(uint64_t seed, int64_t step, uint32_t tensor_id,
+                            int64_t e) {
+  uint64_t blk = (uint64_t)e >> 2;
+  uint32_t ctr[4] = {(uint32_t)blk, (uint32_t)(blk >> 32), (uint32_t)step,
+                     tensor_id};
+  uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+  uint32_t out[4];
+  dqt_oracle_philox4x32_10(ctr, key, out);
+  return out[e & 3];
+}
+
+float dqt_oracle_uniform_from_word(uint32_t w) {
+  return (float)(w >> 8) * (1.0f / 16777216.0f);
+}
+
+/* ------------------------------------------------------------------------ */
+/* Eq. 1: SR(x) = floor(x) with probability ceil(x) - x, otherwise ceil(x).  */
+/* With r = x - floor(x) the value rounds up exactly when the uniform u < r, */
+/* which happens with probability r = 1 - (ceil(x) - x).  An integer x has   */
+/* r = 0 and never moves.                                                    */
+/* ------------------------------------------------------------------------ */
+int32_t dqt_oracle_sr(float x, float u) {
+  float f = floorf(x);
+  float r = x - f;
+  return (int32_t)f + (u < r ? 1 : 0);
+}
+
+void dqt_oracle_sr_batch(const float* x, const float* u, int32_t* out,
+                         int64_t n) {
+  for (int64_t i = 0; i < n; ++i) out[i] = dqt_oracle_sr(x[i], u[i]);
+}
+
+static int32_t clamp_i32(int32_t v, int32_t lo, int32_t hi) {
+  return v < lo ? lo : (v > hi ? hi : v);
+}
+
+/* ------------------------------------------------------------------------ */
+/* Eq. 3 grid.  bits_x100 = 158 selects ternary; otherwise n = bits_x100/100 */
+/* with 2 <= n <= 8 gives Q_n = -2^(n-1), Q_p = 2^(n-1) - 1.                 */
+/* ------------------------------------------------------------------------ */
+int dqt_oracle_grid(int32_t bits_x100, int32_t* qmin, int32_t* qmax) {
+  if (bits_x100 == 158) {
+    *qmin = -1;
+    *qmax = 1;
+    return 0;
+  }
+  if (bits_x100 % 100 != 0) return 1;
+  int32_t n = bits_x100 / 100;
+  if (n < 2 || n > 8) return 1;
+  *qmin = -(1 << (n - 1));
+  *qmax = (1 << (n - 1)) - 1;
+  return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Eq. 2-4: AbsMean(W) = (1/k) sum |w_i|;  s = Q_p / AbsMean(W);             */
+/* codes = Clip[Round(W * s), Q_n, Q_p].  The sum runs in fp64 in index      */
+/* order; s is rounded once to fp32; W * s is one fp32 multiplication and    */
+/* Round() is round-half-to-even.                                            */
+/* ------------------------------------------------------------------------ */
+int dqt_oracle_absmean_init(const float* W0, int64_t numel, int32_t qmin,
+                            int32_t qmax, int8_t* codes, float* s_w,
+                            double* absmean_out) {
+  if (numel <= 0) return 1;
+  double acc = 0.0;
+  for (int64_t i = 0; i < numel; ++i) acc += fabs((double)W0[i]);
+  double absmean = acc / (double)numel;
+  if (absmean_out) *absmean_out = absmean;
+  if (!(absmean > 0.0)) return 2;
+  float s = (float)((double)qmax / absmean);
+  *s_w = s;
+  for (int64_t i = 0; i < numel; ++i) {
+    float p = W0[i] * s;
+    float r = rintf(p);
+    int32_t c;
+    if (r >= (float)qmax) c = qmax;
+    else if (r <= (float)qmin) c = qmin;
+    else c = (int32_t)r;
+    codes[i] = (int8_t)c;
+  }
+  return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Sec 3.2: 8-bit activation quantisation following BitNet: per token t,     */
+/* amax = max_k |x|, s_x = 127 / max(amax, 1e-5), q = Clip[Round(x s_x),     */
+/* -128, 127].  Also returns the two bf16 operand images the GPU path feeds  */
+/* its tensor cores: the codes themselves (exact in bf16) and the            */
+/* dequantised activation bf16(q / s_x).  Either image pointer may be NULL.  */
+/* ------------------------------------------------------------------------ */
+void dqt_oracle_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* q,
+                          float* s_x, uint16_t* q_img, uint16_t* xdq) {
+  for (int64_t t = 0; t < T; ++t) {
+    const uint16_t* row = X + t * K;
+    float amax = 0.0f;
+    for (int64_t k = 0; k < K; ++k) {
+      float a = fabsf(bf16_to_f32(row[k]));
+      if (a > amax) amax = a;
+    }
+    float denom = amax > 1e-5f ? amax : 1e-5f;
+    float s = 127.0f / denom;
+    s_x[t] = s;
+    for (int64_t k = 0; k < K; ++k) {
+      float p = bf16_to_f32(row[k]) * s;
+      float r = rintf(p);
+      int32_t v;
+      if (r >= 127.0f) v = 127;
+      else if (r <= -128.0f) v = -128;
+      else v = (int32_t)r;
+      q[t * K + k] = (int8_t)v;
+      if (q_img) q_img[t * K + k] = f32_to_bf16_rne((float)v);
+      if (xdq) xdq[t * K + k] = f32_to_bf16_rne((float)v / s);
+    }
+  }
+}
+
+/* ------------------------------------------------------------------------ */
+/* Sec 3.2 forward: Y = X_tilde W_tilde^T on the quantised operands.         */
+/* acc[t,n] = sum_k q[t,k] c[n,k]  (exact, int64; must fit int32)            */
+/* Y[t,n]   = bf16( float(acc) * (1 / (s_x[t] * s_w)) )                      */
+/* Returns 1 if an accumulator does not fit int32.                           */
+/* ------------------------------------------------------------------------ */
+int dqt_oracle_fwd(const int8_t* q, const float* s_x, const int8_t* c,
+                   float s_w, int64_t T, int64_t K, int64_t N, uint16_t* Y,
+                   int32_t* acc_out) {
+  int overflow = 0;
+  for (int64_t t = 0; t < T; ++t) {
+    float a_t = 1.0f / (s_x[t] * s_w);
+    for (int64_t n = 0; n < N; ++n) {
+      int64_t acc = 0;
+      for (int64_t k = 0; k < K; ++k)
+        acc += (int64_t)q[t * K + k] * (int64_t)c[n * K + k];
+      if (acc > INT32_MAX || acc < INT32_MIN) overflow = 1;
+      if (acc_out) acc_out[t * N + n] = (int32_t)acc;
+      if (Y) Y[t * N + n] = f32_to_bf16_rne((float)acc * a_t);
+    }
+  }
+  return overflow;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Backward w.r.t. the input (no STE on the weight, straight-through on the  */
+/* activation quantiser): dX[t,k] = sum_n dY[t,n] W_tilde[n,k]               */
+/*                                = (sum_n dY[t,n] c[n,k]) / s_w,  fp64.     */
+/* ------------------------------------------------------------------------ */
+void dqt_oracle_bwd_dx(const uint16_t* dY, const int8_t* c, float s_w,
+                       int64_t T, int64_t N, int64_t K, double* dX) {
+  for (int64_t t = 0; t < T; ++t)
+    for (int64_t k = 0; k < K; ++k) {
+      double acc = 0.0;
+      for (int64_t n = 0; n < N; ++n)
+        acc += (double)bf16_to_f32(dY[t * N + n]) * (double)c[n * K + k];
+      dX[t * K + k] = acc / (double)s_w;
+    }
+}
+
+/* ------------------------------------------------------------------------ */
+/* Backward w.r.t. the low-bit weight W_tilde = c / s_w (Sec 3.2):           */
+/* dW[n,k] = sum_t dY[t,n] X_tilde[t,k],  X_tilde = q / s_x,  fp64.          */
+/* rows (length Nr) selects which output rows n to compute; dW is [Nr, K].   */
+/* ------------------------------------------------------------------------ */
+void dqt_oracle_bwd_dw(const uint16_t* dY, const int8_t* q, const float* s_x,
+                       int64_t T, int64_t N, int64_t K, const int64_t* rows,
+                       int64_t Nr, double* dW) {
+  for (int64_t i = 0; i < Nr; ++i) {
+    int64_t n = rows[i];
+    for (int64_t k = 0; k < K; ++k) dW[i * K + k] = 0.0;
+    for (int64_t t = 0; t < T; ++t) {
+      double g = (double)bf16_to_f32(dY[t * N + n]);
+      double inv = 1.0 / (double)s_x[t];
+      for (int64_t k = 0; k < K; ++k)
+        dW[i * K + k] += g * ((double)q[t * K + k] * inv);
+    }
+  }
+}
+
+/* ------------------------------------------------------------------------ */
+/* AdamW (Loshchilov & Hutter; the optimiser of Sec 4.1) in the code domain. */
+/* The host-side constants follow from the hyper-parameters in fp64, each    */
+/* rounded once to fp32:                                                     */
+/*   omb1 = 1 - b1, omb2 = 1 - b2, bc1 = 1 - b1^step, bc2 = 1 - b2^step,     */
+/*   decay = 1 - lr * wd, lrs = lr * s_w.                                    */
+/* Per element, each a separately rounded fp32 operation:                    */
+/*   m' = b1 m + omb1 g ;  v' = b2 v + omb2 (g g)                            */
+/*   u  = (m' / bc1) / (sqrt(v' / bc2) + eps)                                */
+/*   x  = c decay - lrs u          (= W' s_w, the dense target in codes)     */
+/* ------------------------------------------------------------------------ */
+typedef struct {
+  float b1, b2, eps, omb1, omb2, bc1, bc2, decay, lrs;
+} oracle_adamw_consts;
+
+void dqt_oracle_adamw_consts(float lr, float b1, float b2, float eps, float wd,
+                             int64_t step, float s_w, float* out9) {
+  out9[0] = b1;
+  out9[1] = b2;
+  out9[2] = eps;
+  out9[3] = (float)(1.0 - (double)b1);
+  out9[4] = (float)(1.0 - (double)b2);
+  out9[5] = (float)(1.0 - pow((double)b1, (double)step));
+  out9[6] = (float)(1.0 - pow((double)b2, (double)step));
+  out9[7] = (float)(1.0 - (double)lr * (double)wd);
+  out9[8] = (float)((double)lr * (double)s_w);
+}
+
+static float adamw_x(const oracle_adamw_consts* h, float g, int8_t c, float* m,
+                     float* v) {
+  float m1 = h->b1 * *m;
+  float m2 = h->omb1 * g;
+  float mn = m1 + m2;
+  float v1 = h->b2 * *v;
+  float gg = g * g;
+  float v2 = h->omb2 * gg;
+  float vn = v1 + v2;
+  *m = mn;
+  *v = vn;
+  float mh = mn / h->bc1;
+  float vh = vn / h->bc2;
+  float den = sqrtf(vh) + h->eps;
+  float u = mh / den;
+  float cd = (float)c * h->decay;
+  float du = h->lrs * u;
+  return cd - du;
+}
+
+/* Dense target only (no rounding): x, m', v' for n elements. */
+void dqt_oracle_adamw_x(const float* g, const int8_t* c, float* m, float* v,
+                        const float* consts9, int64_t n, float* x) {
+  oracle_adamw_consts h;
+  memcpy(&h, consts9, sizeof(h));
+  for (int64_t i = 0; i < n; ++i) x[i] = adamw_x(&h, g[i], c[i], &m[i], &v[i]);
+}
+
+/* ------------------------------------------------------------------------ */
+/* Eq. 5: W_hat = SR(W'), clamped to [Q_n, Q_p], written over the codes.     */
+/* g, c, m, v are [Nr, K] row blocks of an [N, K] weight; rows[i] is the      */
+/* global row of block row i, so element (rows[i], k) draws the uniform of   */
+/* flat index rows[i]*K + k.  rows == NULL means rows[i] = i.                */
+/* round_mode 0 = stochastic (Eq. 1); 1 = round-to-nearest (Sec 5.1          */
+/* ablation).  Returns the number of codes that changed.                     */
+/* ------------------------------------------------------------------------ */
+int64_t dqt_oracle_update(const float* g, int8_t* c, float* m, float* v,
+                          const float* consts9, int32_t qmin, int32_t qmax,
+                          uint64_t seed, int64_t step, uint32_t tensor_id,
+                          int32_t round_mode, const int64_t* rows, int64_t Nr,
+                          int64_t K) {
+  oracle_adamw_consts h;
+  memcpy(&h, consts9, sizeof(h));
+  int64_t changed = 0;
+  for (int64_t i = 0; i < Nr; ++i) {
+    int64_t n = rows ? rows[i] : i;
+    for (int64_t k = 0; k < K; ++k) {
+      int64_t j = i * K + k;
+      float x = adamw_x(&h, g[j], c[j], &m[j], &v[j]);
+      int32_t r;
+      if (round_mode == 1) {
+        r = (int32_t)rintf(x);
+      } else {
+        uint32_t w = dqt_oracle_sr_word(seed, step, tensor_id, n * K + k);
+        r = dqt_oracle_sr(x, dqt_oracle_uniform_from_word(w));
+      }
+      r = clamp_i32(r, qmin, qmax);
+      if ((int8_t)r != c[j]) ++changed;
+      c[j] = (int8_t)r;
+    }
+  }
+  return changed;
+}

@@ -1,0 +1,255 @@
+"""ctypes front end of the C oracle (test infrastructure only).
+
+Every function mirrors one step of the DQT BitLinear training step as the
+paper states it (Zhao et al., "Direct Quantized Training of Language Models
+with Stochastic Rounding"):
+
+* ``sr``/``sr_batch``          -- Eq. 1, stochastic rounding
+* ``grid``                     -- Eq. 3, the n-bit grid [Q_n, Q_p]
+* ``absmean_init``             -- Eq. 2-4, AbsMean scale and initial codes
+* ``act_quant``                -- Sec. 3.2, 8-bit per-token absmax activations
+* ``fwd``                      -- Sec. 3.2, BitLinear forward (exact int accumulation)
+* ``bwd_dx`` / ``bwd_dw``      -- Sec. 3.2, backward w.r.t. input and low-bit weight (fp64)
+* ``adamw_consts``/``adamw_x`` -- Sec. 4.1, AdamW producing the dense target W'
+* ``update``                   -- Eq. 5, W_hat = SR(W') clamped onto the grid
+
+bf16 tensors are passed as ``numpy.uint16`` arrays holding the raw bits.
+"""
+import ctypes as C
+import numpy as np
+
+from .build_oracle import build
+
+_lib = None
+
+_f32p = C.POINTER(C.c_float)
+_f64p = C.POINTER(C.c_double)
+_i8p = C.POINTER(C.c_int8)
+_i32p = C.POINTER(C.c_int32)
+_i64p = C.POINTER(C.c_int64)
+_u16p = C.POINTER(C.c_uint16)
+_u32p = C.POINTER(C.c_uint32)
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        L = C.CDLL(build())
+        L.dqt_oracle_f32_to_bf16.argtypes = [C.c_float]
+        L.dqt_oracle_f32_to_bf16.restype = C.c_uint16
+        L.dqt_oracle_philox4x32_10.argtypes = [_u32p, _u32p, _u32p]
+        L.dqt_oracle_philox4x32_10.restype = None
+        L.dqt_oracle_sr_word.argtypes = [C.c_uint64, C.c_int64, C.c_uint32, C.c_int64]
+        L.dqt_oracle_sr_word.restype = C.c_uint32
+        L.dqt_oracle_uniform_from_word.argtypes = [C.c_uint32]
+        L.dqt_oracle_uniform_from_word.restype = C.c_float
+        L.dqt_oracle_sr.argtypes = [C.c_float, C.c_float]
+        L.dqt_oracle_sr.restype = C.c_int32
+        L.dqt_oracle_sr_batch.argtypes = [_f32p, _f32p, _i32p, C.c_int64]
+        L.dqt_oracle_sr_batch.restype = None
+        L.dqt_oracle_grid.argtypes = [C.c_int32, _i32p, _i32p]
+        L.dqt_oracle_grid.restype = C.c_int
+        L.dqt_oracle_absmean_init.argtypes = [_f32p, C.c_int64, C.c_int32, C.c_int32,
+                                              _i8p, _f32p, _f64p]
+        L.dqt_oracle_absmean_init.restype = C.c_int
+        L.dqt_oracle_act_quant.argtypes = [_u16p, C.c_int64, C.c_int64, _i8p, _f32p,
+                                           _u16p, _u16p]
+        L.dqt_oracle_act_quant.restype = None
+        L.dqt_oracle_fwd.argtypes = [_i8p, _f32p, _i8p, C.c_float, C.c_int64, C.c_int64,
+                                     C.c_int64, _u16p, _i32p]
+        L.dqt_oracle_fwd.restype = C.c_int
+        L.dqt_oracle_bwd_dx.argtypes = [_u16p, _i8p, C.c_float, C.c_int64, C.c_int64,
+                                        C.c_int64, _f64p]
+        L.dqt_oracle_bwd_dx.restype = None
+        L.dqt_oracle_bwd_dw.argtypes = [_u16p, _i8p, _f32p, C.c_int64, C.c_int64,
+                                        C.c_int64, _i64p, C.c_int64, _f64p]
+        L.dqt_oracle_bwd_dw.restype = None
+        L.dqt_oracle_adamw_consts.argtypes = [C.c_float, C.c_float, C.c_float, C.c_float,
+                                              C.c_float, C.c_int64, C.c_float, _f32p]
+        L.dqt_oracle_adamw_consts.restype = None
+        L.dqt_oracle_adamw_x.argtypes = [_f32p, _i8p, _f32p, _f32p, _f32p, C.c_int64, _f32p]
+        L.dqt_oracle_adamw_x.restype = None
+        L.dqt_oracle_update.argtypes = [_f32p, _i8p, _f32p, _f32p, _f32p, C.c_int32,
+                                        C.c_int32, C.c_uint64, C.c_int64, C.c_uint32,
+                                        C.c_int32, _i64p, C.c_int64, C.c_int64]
+        L.dqt_oracle_update.restype = C.c_int64
+        _lib = L
+    return _lib
+
+
+def _p(a, ct):
+    assert a.flags["C_CONTIGUOUS"]
+    return a.ctypes.data_as(ct)
+
+
+def _c(a, dt):
+    return np.ascontiguousarray(a, dtype=dt)
+
+
+# --------------------------------------------------------------------------
+# scalars and small helpers
+# --------------------------------------------------------------------------
+def f32_to_bf16_bits(x: float) -> int:
+    return int(lib().dqt_oracle_f32_to_bf16(float(x)))
+
+
+def philox4x32_10(ctr, key):
+    c = _c(ctr, np.uint32)
+    k = _c(key, np.uint32)
+    out = np.zeros(4, np.uint32)
+    lib().dqt_oracle_philox4x32_10(_p(c, _u32p), _p(k, _u32p), _p(out, _u32p))
+    return out
+
+
+def sr_word(seed: int, step: int, tensor_id: int, e: int) -> int:
+    return int(lib().dqt_oracle_sr_word(seed, step, tensor_id, e))
+
+
+def uniform_from_word(w: int) -> float:
+    return float(lib().dqt_oracle_uniform_from_word(w))
+
+
+def sr(x: float, u: float) -> int:
+    return int(lib().dqt_oracle_sr(x, u))
+
+
+def sr_batch(x, u):
+    x = _c(x, np.float32)
+    u = _c(u, np.float32)
+    assert x.shape == u.shape
+    out = np.empty(x.shape, np.int32)
+    lib().dqt_oracle_sr_batch(_p(x, _f32p), _p(u, _f32p), _p(out, _i32p), x.size)
+    return out
+
+
+def grid(bits: float):
+    """Eq. 3 grid for ``bits`` in {1.58, 2, ..., 8}; returns (Q_n, Q_p)."""
+    bx = int(round(bits * 100))
+    qmin = C.c_int32()
+    qmax = C.c_int32()
+    if lib().dqt_oracle_grid(bx, C.byref(qmin), C.byref(qmax)) != 0:
+        raise ValueError("unsupported bit width %r" % bits)
+    return qmin.value, qmax.value
+
+
+# --------------------------------------------------------------------------
+# Eq. 2-4
+# --------------------------------------------------------------------------
+def absmean_init(W0, qmin: int, qmax: int):
+    """Returns (codes int8, s_w float32, absmean float64)."""
+    W = _c(W0, np.float32)
+    codes = np.empty(W.shape, np.int8)
+    s = C.c_float()
+    am = C.c_double()
+    rc = lib().dqt_oracle_absmean_init(_p(W, _f32p), W.size, qmin, qmax,
+                                       _p(codes, _i8p), C.byref(s), C.byref(am))
+    if rc != 0:
+        raise ValueError("absmean_init failed (%d)" % rc)
+    return codes, np.float32(s.value), am.value
+
+
+# --------------------------------------------------------------------------
+# Sec. 3.2 activation quantisation
+# --------------------------------------------------------------------------
+def act_quant(X_bits):
+    """X_bits: uint16 [T, K] raw bf16.  Returns (q int8, s_x f32, q_img u16, xdq u16)."""
+    X = _c(X_bits, np.uint16)
+    T, K = X.shape
+    q = np.empty((T, K), np.int8)
+    s = np.empty(T, np.float32)
+    qi = np.empty((T, K), np.uint16)
+    xd = np.empty((T, K), np.uint16)
+    lib().dqt_oracle_act_quant(_p(X, _u16p), T, K, _p(q, _i8p), _p(s, _f32p),
+                               _p(qi, _u16p), _p(xd, _u16p))
+    return q, s, qi, xd
+
+
+# --------------------------------------------------------------------------
+# Sec. 3.2 forward / backward
+# --------------------------------------------------------------------------
+def fwd(q, s_x, c, s_w):
+    """Returns (Y bf16 bits u16 [T,N], acc int32 [T,N])."""
+    q = _c(q, np.int8)
+    s_x = _c(s_x, np.float32)
+    c = _c(c, np.int8)
+    T, K = q.shape
+    N, K2 = c.shape
+    assert K == K2 and s_x.shape == (T,)
+    Y = np.empty((T, N), np.uint16)
+    acc = np.empty((T, N), np.int32)
+    ov = lib().dqt_oracle_fwd(_p(q, _i8p), _p(s_x, _f32p), _p(c, _i8p), float(s_w),
+                              T, K, N, _p(Y, _u16p), _p(acc, _i32p))
+    if ov:
+        raise OverflowError("int32 accumulator overflow")
+    return Y, acc
+
+
+def bwd_dx(dY_bits, c, s_w):
+    dY = _c(dY_bits, np.uint16)
+    c = _c(c, np.int8)
+    T, N = dY.shape
+    N2, K = c.shape
+    assert N == N2
+    dX = np.empty((T, K), np.float64)
+    lib().dqt_oracle_bwd_dx(_p(dY, _u16p), _p(c, _i8p), float(s_w), T, N, K,
+                            _p(dX, _f64p))
+    return dX
+
+
+def bwd_dw(dY_bits, q, s_x, rows=None):
+    dY = _c(dY_bits, np.uint16)
+    q = _c(q, np.int8)
+    s_x = _c(s_x, np.float32)
+    T, N = dY.shape
+    T2, K = q.shape
+    assert T == T2
+    rows = np.arange(N, dtype=np.int64) if rows is None else _c(rows, np.int64)
+    dW = np.empty((rows.size, K), np.float64)
+    lib().dqt_oracle_bwd_dw(_p(dY, _u16p), _p(q, _i8p), _p(s_x, _f32p), T, N, K,
+                            _p(rows, _i64p), rows.size, _p(dW, _f64p))
+    return dW
+
+
+# --------------------------------------------------------------------------
+# Sec. 4.1 AdamW and Eq. 5 update
+# --------------------------------------------------------------------------
+def adamw_consts(lr, b1, b2, eps, wd, step, s_w):
+    out = np.empty(9, np.float32)
+    lib().dqt_oracle_adamw_consts(lr, b1, b2, eps, wd, step, float(s_w), _p(out, _f32p))
+    return out
+
+
+def adamw_x(g, c, m, v, consts):
+    """Returns (x, m', v'): the dense code-domain target and the new moments."""
+    g = _c(g, np.float32).ravel()
+    c = _c(c, np.int8).ravel()
+    m = _c(m, np.float32).ravel().copy()
+    v = _c(v, np.float32).ravel().copy()
+    x = np.empty_like(g)
+    k = _c(consts, np.float32)
+    lib().dqt_oracle_adamw_x(_p(g, _f32p), _p(c, _i8p), _p(m, _f32p), _p(v, _f32p),
+                             _p(k, _f32p), g.size, _p(x, _f32p))
+    return x, m, v
+
+
+def update(g, c, m, v, consts, qmin, qmax, seed, step, tensor_id, round_mode=0,
+           rows=None):
+    """Eq. 5 over an [Nr, K] block.  Returns (c', m', v', changed)."""
+    g = _c(g, np.float32)
+    if g.ndim == 1:
+        g = g.reshape(1, -1)
+    Nr, K = g.shape
+    c = _c(c, np.int8).reshape(Nr, K).copy()
+    m = _c(m, np.float32).reshape(Nr, K).copy()
+    v = _c(v, np.float32).reshape(Nr, K).copy()
+    k = _c(consts, np.float32)
+    if rows is not None:
+        rows = _c(rows, np.int64)
+        assert rows.size == Nr
+        rp = _p(rows, _i64p)
+    else:
+        rp = None
+    changed = lib().dqt_oracle_update(_p(g, _f32p), _p(c, _i8p), _p(m, _f32p),
+                                      _p(v, _f32p), _p(k, _f32p), qmin, qmax, seed, step,
+                                      tensor_id, round_mode, rp, Nr, K)
+    return c, m, v, int(changed)
