@@ -1,0 +1,434 @@
+"""Benchmark: one DQT training step of a ternary LLaMA MLP GEMM set on GB300.
+
+Workload (the headline configuration): hidden 2048, intermediate 5632,
+tokens 8192 (batch 4 x seq 2048); BitLinear gate and up [2048 -> 5632] and
+down [5632 -> 2048], ternary int8 codes from AbsMean of N(0, 0.02), bf16
+activations ~ N(0, 1), upstream gradients ~ N(0, 1e-2), AdamW moments fp32.
+The down projection's input is a synthetic N(0, 1) activation (no SwiGLU on
+the measured path).  One step runs, through the C ABI:
+
+  act_quant(X)  -> codes image + dequantised X (shared by gate and up)
+  act_quant(H)  -> the same for the down projection's input
+  codes_to_bf16 for the three weights (exact images of the int8 codes)
+  forward GEMM  x3, dX GEMM x3, fused dW GEMM + AdamW + SR update x3
+
+Metric: tokens/s of the whole step (higher is better).  `value` is timed with
+CUDA events on the launching stream with inputs resident in HBM; `e2e` adds,
+every step, the pinned-host -> device copy of that step's activations and
+gradients and the device -> host read of the step's changed-code counts.
+The step's working set (~1.5 GB) is far larger than the 129 MB L2, so no
+flush is needed between steps.
+
+`--impl reference` times the CPU oracle instead (bounded sample of the same
+step, extrapolated).  Under torchrun each rank runs an independent replica
+(weak scaling, no collective on the data path).
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+T_TOK, HID, INTER = 8192, 2048, 5632
+WORKLOAD = "ternary DQT LLaMA MLP GEMM set (gate/up 2048->5632, down 5632->2048), 8192 tokens"
+METRIC = "DQT BitLinear fwd+bwd+SR-update tokens/s"
+PROJ = [("gate", HID, INTER), ("up", HID, INTER), ("down", INTER, HID)]
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return d, "measured"
+    except (OSError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.Q,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self):
+        rows = []
+        for line in (self.out or "").strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) >= 9:
+                rows.append(f)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i] == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+class MLPStep:
+    """Device buffers and the launch sequence of one DQT MLP training step."""
+
+    def __init__(self, dev, seed=1234):
+        from paper_2412_04787_gb300 import dqt, inputs
+
+        self.dqt = dqt
+        self.dev = dev
+        self.grid = dqt.grid(1.58)
+        T = T_TOK
+        self.host = {
+            "X": inputs.normal((T, HID), 1.0, seed=1, dtype=torch.bfloat16),
+            "H": inputs.normal((T, INTER), 1.0, seed=2, dtype=torch.bfloat16),
+        }
+        for i, (name, K, N) in enumerate(PROJ):
+            self.host["dY_" + name] = inputs.normal((T, N), 1e-2, seed=10 + i, dtype=torch.bfloat16)
+        self.d = {k: v.to(dev) for k, v in self.host.items()}
+        self.W, self.s_w, self.m, self.v, self.W_img, self.Y, self.dX, self.Xdq = {}, {}, {}, {}, {}, {}, {}, {}
+        for i, (name, K, N) in enumerate(PROJ):
+            W0 = inputs.normal((N, K), 0.02, seed=20 + i).to(dev)
+            self.W[name], self.s_w[name] = dqt.dqt_absmean_init(W0, self.grid)
+            del W0
+            self.m[name] = torch.zeros((N, K), dtype=torch.float32, device=dev)
+            self.v[name] = torch.zeros((N, K), dtype=torch.float32, device=dev)
+            self.W_img[name] = torch.empty((N, K), dtype=torch.bfloat16, device=dev)
+            self.Y[name] = torch.empty((T, N), dtype=torch.bfloat16, device=dev)
+            self.dX[name] = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
+        self.aq = {}
+        for src, K in (("X", HID), ("H", INTER)):
+            self.aq[src] = (torch.empty(T, dtype=torch.float32, device=dev),
+                            torch.empty((T, K), dtype=torch.bfloat16, device=dev),
+                            torch.empty((T, K), dtype=torch.bfloat16, device=dev))
+        self.changed = torch.zeros(3, dtype=torch.int64, device=dev)
+        self.sr = {name: dqt.sr_stream(seed=seed, tensor_id=i) for i, (name, _, _) in enumerate(PROJ)}
+        self.step_no = 0
+        self.launches_per_step = 2 + 3 + 3 + 3 + 3
+
+    def run(self, timers=None):
+        """Enqueue one step on the current stream.  `timers` maps a kernel kind
+        to a list that receives (start, end) CUDA events around its launches."""
+        dqt = self.dqt
+        self.step_no += 1
+        hp = dqt.adamw(lr=1e-3, step=self.step_no)
+
+        def timed(kind, fn):
+            if timers is not None and kind in timers:
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
+                a.record()
+                fn()
+                b.record()
+                timers[kind].append((a, b))
+            else:
+                fn()
+
+        for src in ("X", "H"):
+            s_x, q_img, xdq = self.aq[src]
+            timed("act_quant", lambda: dqt.dqt_act_quant(self.d[src], None, s_x, q_img, xdq, want=()))
+        for name, K, N in PROJ:
+            timed("codes_to_bf16", lambda: dqt.dqt_codes_to_bf16(self.W[name], self.W_img[name]))
+        for name, K, N in PROJ:
+            s_x, q_img, _ = self.aq["X" if name != "down" else "H"]
+            timed("fwd", lambda: dqt.dqt_bitlinear_fwd(q_img, s_x, self.W_img[name], self.s_w[name],
+                                                      self.grid, Y=self.Y[name]))
+        for i, (name, K, N) in enumerate(PROJ):
+            dY = self.d["dY_" + name]
+            _, _, xdq = self.aq["X" if name != "down" else "H"]
+            timed("bwd_dx", lambda: dqt.dqt_bitlinear_bwd_dx(dY, self.W_img[name], self.s_w[name],
+                                                            dX=self.dX[name]))
+            timed("bwd_dw_update", lambda: dqt.dqt_bitlinear_bwd_dw_update(
+                dY, xdq, self.W[name], self.s_w[name], self.m[name], self.v[name], hp,
+                self.sr[name], self.grid, changed_out=self.changed[i:i + 1]))
+
+    # algorithmic work per launch, per kernel kind
+    def work(self):
+        T = T_TOK
+        flops = {"fwd": [2.0 * T * K * N for _, K, N in PROJ]}
+        flops["bwd_dx"] = list(flops["fwd"])
+        flops["bwd_dw_update"] = list(flops["fwd"])
+        byts = {
+            # bf16 in (2) + bf16 code image (2) + bf16 dequantised image (2) per element, + s_x
+            "act_quant": [T * HID * 6.0 + 4 * T, T * INTER * 6.0 + 4 * T],
+            "codes_to_bf16": [3.0 * K * N for _, K, N in PROJ],
+        }
+        return flops, byts
+
+
+def _elapsed(pairs):
+    return [a.elapsed_time(b) for a, b in pairs]
+
+
+def run_gpu(args):
+    ws, rank, local = _dist()
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if ws > 1 else 0)
+    torch.cuda.set_device(dev)
+    from paper_2412_04787_gb300 import build as dqt_build
+    dqt_build.build()
+    st = MLPStep(dev)
+    dqt = st.dqt
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        if ws > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        st.run()
+    dqt.dqt_check_device_status()
+
+    # ---- device-timed region: inputs resident in HBM ----
+    kinds = ["act_quant", "codes_to_bf16", "fwd", "bwd_dx", "bwd_dw_update"]
+    timers = {k: [] for k in kinds}
+    barrier()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    with ClockSampler(dev.index) as clk:
+        t0.record(stream)
+        for _ in range(args.steps):
+            st.run(timers)
+        t1.record(stream)
+        barrier()
+    dqt.dqt_check_device_status()
+    ms = t0.elapsed_time(t1)
+    if ws > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    ms_step = ms / args.steps
+    value = ws * T_TOK * args.steps / (ms / 1e3)
+
+    # per-kernel live timings
+    flops, byts = st.work()
+    per = {}
+    for k in kinds:
+        ts = _elapsed(timers[k])
+        per[k] = {"launches": len(ts), "total_ms": sum(ts), "avg_ms": sum(ts) / max(1, len(ts))}
+    tot = sum(p["total_ms"] for p in per.values())
+    for k in kinds:
+        per[k]["share"] = per[k]["total_ms"] / tot if tot else None
+    peaks, pk_kind = _peaks()
+    dom = max(["fwd", "bwd_dx", "bwd_dw_update"], key=lambda k: per[k]["total_ms"])
+    nlaunch = len(PROJ)
+    dom_flops = sum(flops[dom]) * args.steps
+    achieved = dom_flops / (per[dom]["total_ms"] / 1e3) / 1e12
+    peak = peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops"))
+    roofline = {"bound": "tensor", "kernel": dom, "achieved": round(achieved, 1),
+                "peak": peak, "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
+                "peak_kind": "bf16 dense sustained, %s" % pk_kind,
+                "traffic": None,
+                "algorithmic_per_launch": "2*T*K*N FLOP (T=8192; K,N = 2048,5632 / 5632,2048)"}
+    kern = {}
+    for k in kinds:
+        d = dict(per[k])
+        if k in flops:
+            d["tflops"] = sum(flops[k]) * args.steps / (per[k]["total_ms"] / 1e3) / 1e12
+            d["frac_of_bf16_sustained"] = d["tflops"] / peak
+        else:
+            d["gbs"] = sum(byts[k]) * args.steps / (per[k]["total_ms"] / 1e3) / 1e9
+            d["frac_of_hbm"] = d["gbs"] / peaks["hbm_gbs"]
+        kern[k] = {kk: (round(vv, 4) if isinstance(vv, float) else vv) for kk, vv in d.items()}
+
+    # ---- e2e: host buffers, H2D inputs + D2H result inside the timed region ----
+    pinned = {k: v.pin_memory() for k, v in st.host.items()}
+    res_host = torch.empty(3, dtype=torch.int64).pin_memory()
+    h2d = sum(v.numel() * v.element_size() for v in pinned.values())
+    d2h = res_host.numel() * res_host.element_size()
+    e_steps = max(1, min(args.steps, 10))
+    barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e_steps):
+        for k, v in pinned.items():
+            st.d[k].copy_(v, non_blocking=True)
+        st.changed.zero_()
+        st.run()
+        res_host.copy_(st.changed, non_blocking=True)
+    e1.record(stream)
+    barrier()
+    e_ms = e0.elapsed_time(e1)
+    if ws > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([e_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e_ms = float(tt.item())
+    dqt.dqt_check_device_status()
+    e2e = {"value": round(ws * T_TOK * e_steps / (e_ms / 1e3), 1), "unit": "tokens/s",
+           "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": e_steps}
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(args.cpu_seconds)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded N(0,1) activations, N(0,1e-2) gradients, AbsMean-ternary codes of N(0,0.02))",
+            "config": {"workload": WORKLOAD, "tokens": T_TOK, "hidden": HID, "intermediate": INTER,
+                       "weights": "ternary int8 codes", "parallelism": "replicas" if ws > 1 else "single GPU",
+                       "l2": "inputs larger than L2 (step working set ~1.5 GB > 129 MB)"},
+            "roofline": roofline, "kernels": kern, "e2e": e2e,
+            "gpu_launches": st.launches_per_step * args.steps,
+            "clocks": clk.summary(), "cpu_baseline": cpu,
+            "changed_codes_last_step": [int(x) for x in res_host.tolist()],
+        }
+        print(json.dumps(line))
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (the reported baseline and the --impl reference arm)
+# ---------------------------------------------------------------------------
+def _oracle_sample(token_rows, weight_rows, seed=7):
+    """Times the oracle on `token_rows` token rows of act-quant + forward + dX
+    and `weight_rows` weight rows of dW + AdamW + SR per projection; returns
+    (seconds measured, seconds extrapolated to the full step)."""
+    import oracle
+    from paper_2412_04787_gb300 import inputs
+
+    qmin, qmax = oracle.grid(1.58)
+    meas = 0.0
+    full = 0.0
+    for i, (name, K, N) in enumerate(PROJ):
+        X = inputs.bf16_bits(inputs.normal((T_TOK, K), 1.0, seed=seed + i, dtype=torch.bfloat16))
+        dY = inputs.bf16_bits(inputs.normal((T_TOK, N), 1e-2, seed=seed + 10 + i, dtype=torch.bfloat16))
+        c, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=seed + 20 + i).numpy(), qmin, qmax)
+        t0 = time.perf_counter()
+        q, s, _, _ = oracle.act_quant(X[:token_rows])
+        oracle.fwd(q, s, c, s_w)
+        oracle.bwd_dx(dY[:token_rows], c, s_w)
+        t1 = time.perf_counter()
+        # dW needs every token's quantised activation
+        qa, sa, _, _ = oracle.act_quant(X)
+        t2 = time.perf_counter()
+        rows = np.arange(weight_rows)
+        g = oracle.bwd_dw(dY, qa, sa, rows=rows).astype(np.float32)
+        k = oracle.adamw_consts(1e-3, 0.9, 0.999, 1e-8, 0.0, 1, s_w)
+        z = np.zeros((weight_rows, K), np.float32)
+        oracle.update(g, c[:weight_rows], z, z, k, qmin, qmax, 1234, 1, i, rows=rows)
+        t3 = time.perf_counter()
+        meas += (t1 - t0) + (t2 - t1) + (t3 - t2)
+        full += (t1 - t0) * T_TOK / token_rows + (t2 - t1) + (t3 - t2) * N / weight_rows
+    return meas, full
+
+
+def cpu_baseline(seconds=15.0):
+    # calibrate on a tiny sample, then size the sample to ~`seconds` of work
+    m0, f0 = _oracle_sample(2, 1)
+    scale = max(1.0, seconds / max(m0, 1e-3))
+    tr = int(min(256, max(2, 2 * scale)))
+    wr = int(min(128, max(1, scale)))
+    meas, full = _oracle_sample(tr, wr)
+    return {"value": round(T_TOK / full, 3), "unit": "tokens/s", "cores": 1, "kind": "oracle",
+            "sample": "%d token rows of act-quant+fwd+dX and %d weight rows of dW+AdamW+SR per "
+                      "projection (plus the full act-quant dW needs), %.1f s measured, "
+                      "extrapolated linearly to the 8192-token step (%.0f s)" % (tr, wr, meas, full)}
+
+
+def run_reference(args):
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return
+    from oracle import build_oracle
+    build_oracle.build()
+    per_step_s = max(5.0, min(30.0, 150.0 / max(1, args.steps + args.warmup)))
+    for _ in range(args.warmup):
+        _oracle_sample(2, 1)
+    vals = []
+    samples = []
+    for _ in range(args.steps):
+        m0, _ = _oracle_sample(2, 1)
+        scale = max(1.0, per_step_s / max(m0, 1e-3))
+        tr, wr = int(min(256, max(2, 2 * scale))), int(min(128, max(1, scale)))
+        meas, full = _oracle_sample(tr, wr)
+        vals.append(full)
+        samples.append((tr, wr, meas))
+    full = statistics.median(vals)
+    value = T_TOK / full
+    tr, wr, meas = samples[-1]
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": "tokens/s",
+        "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(full * 1e3, 1), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64/f32 (oracle)", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "tokens": T_TOK, "hidden": HID, "intermediate": INTER},
+        "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                         "sample": "per step: %d token rows of act-quant+fwd+dX, %d weight rows of "
+                                   "dW+AdamW+SR per projection, extrapolated" % (tr, wr)},
+        "e2e": {"value": round(value, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="dqt", choices=["dqt", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

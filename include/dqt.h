@@ -1,0 +1,183 @@
+/*
+ * dqt.h -- C ABI of the GB300 (sm_103a) Direct Quantized Training library.
+ *
+ * Direct Quantized Training (DQT; Zhao et al., "Direct Quantized Training of
+ * Language Models with Stochastic Rounding", arXiv 2412.04787) trains
+ * BitLinear layers whose weights exist only as n-bit integer codes c with a
+ * fixed per-tensor scale s_w (W_tilde = c / s_w, Eq. 2-4).  One training step
+ * of a layer is:
+ *
+ *   dqt_act_quant                 8-bit per-token absmax activation codes (Sec. 3.2)
+ *   dqt_bitlinear_fwd             Y = X_tilde W_tilde^T, exact integer accumulation (Sec. 3.2)
+ *   dqt_bitlinear_bwd_dx          dX = dY W_tilde (Sec. 3.2; no STE on the weight)
+ *   dqt_bitlinear_bwd_dw_update   dW = dY^T X_tilde, then in the GEMM epilogue the AdamW
+ *                                 step (Sec. 4.1) and W_hat = SR(W') (Eq. 1, Eq. 5),
+ *                                 clamped to the n-bit grid and written over the codes
+ *   dqt_sr_update                 the same AdamW + SR step for a gradient given in memory
+ *
+ * GB300 has no int8 tensor-core MMA for sm_103a, so the integer GEMMs run on
+ * the bf16 tensor cores over exact bf16 images of the integer codes (every
+ * integer in [-256, 256] is exact in bf16; products and partial sums below
+ * 2^24 are exact in the fp32 accumulator).  dqt_act_quant writes those images
+ * next to the int8 codes, and dqt_codes_to_bf16 makes the weight image.
+ *
+ * Conventions for every entry point:
+ *   - All data pointers are DEVICE pointers owned by the caller; the library
+ *     keeps no reference after the call returns and allocates no device memory.
+ *   - Every call is asynchronous on `stream` (a cudaStream_t; NULL selects the
+ *     legacy default stream).  Host-side argument checks run before any launch;
+ *     a non-zero return means nothing was launched (except DQT_ERR_CUDA, which
+ *     reports a launch failure).
+ *   - bf16 tensors are passed as dqt_bf16 (the raw IEEE bfloat16 bits).
+ *   - Matrices are row-major and contiguous.  Device pointers must be 16-byte
+ *     aligned and the row lengths K and N multiples of 8 (the tensor-memory
+ *     accelerator moves 16-byte rows); otherwise DQT_ERR_ALIGN.
+ *   - Device-side waits are bounded.  A kernel whose wait runs out records
+ *     DQT_ERR_TIMEOUT in a device status word and returns early, leaving its
+ *     outputs undefined; dqt_check_device_status() reports and clears it.
+ */
+#ifndef DQT_H_
+#define DQT_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef uint16_t dqt_bf16; /* raw bfloat16 bits */
+
+enum {
+  DQT_OK = 0,
+  DQT_ERR_ARG = 1,     /* null pointer, bad size, bad grid or hyper-parameter   */
+  DQT_ERR_ALIGN = 2,   /* pointer not 16-byte aligned, K or N not a multiple of 8 */
+  DQT_ERR_CUDA = 3,    /* a CUDA runtime or driver call failed                   */
+  DQT_ERR_TIMEOUT = 4, /* a bounded device wait ran out (dqt_check_device_status) */
+  DQT_ERR_RANGE = 5    /* a size exceeds what the kernels index (see each call)  */
+};
+
+/* The n-bit grid [Q_n, Q_p] of Eq. 3.  Ternary ("1.58-bit") is [-1, 1]; an
+ * integer width n in [2, 8] is [-2^(n-1), 2^(n-1) - 1].  Codes are int8. */
+typedef struct {
+  int32_t qmin;
+  int32_t qmax;
+} dqt_grid_t;
+
+/* AdamW hyper-parameters (the optimiser of Sec. 4.1).  step >= 1 is the
+ * 1-based optimiser step used for the bias corrections 1 - beta^step.  The
+ * library derives, in fp64 rounded once to fp32: 1 - beta1, 1 - beta2,
+ * 1 - beta1^step, 1 - beta2^step, 1 - lr * weight_decay and lr * s_w. */
+typedef struct {
+  float lr;
+  float beta1;
+  float beta2;
+  float eps;
+  float weight_decay;
+  int64_t step;
+} dqt_adamw_t;
+
+/* Stochastic rounding stream (Eq. 1).  The uniform for element e (flat
+ * row-major index into the [N, K] weight) is word e % 4 of
+ * Philox4x32-10(counter = (e/4 low 32, e/4 high 32, step low 32, tensor_id),
+ * key = (seed low 32, seed high 32)), U = (word >> 8) * 2^-24; the code rounds
+ * up when U < x - floor(x).  round_mode 0 = stochastic rounding (the paper's
+ * method); 1 = round to nearest (the absmax-without-SR ablation of Sec. 5.1). */
+typedef struct {
+  uint64_t seed;
+  uint32_t tensor_id;
+  int32_t round_mode;
+} dqt_sr_t;
+
+/* Eq. 3: grid for `bits` in {1.58, 2, 3, ..., 8}.  Host only. */
+int dqt_grid_for_bits(float bits, dqt_grid_t* out);
+
+/* Human-readable name of a status code.  Host only; never NULL. */
+const char* dqt_status_string(int status);
+
+/* Synchronises `stream`, then returns DQT_ERR_TIMEOUT if any kernel of this
+ * library recorded a timed-out wait since the last call (and clears the
+ * record), DQT_ERR_CUDA if the stream reports an error, else DQT_OK. */
+int dqt_check_device_status(void* stream);
+
+/* Upper bound, in nanoseconds, on any single device-side wait of this
+ * library's kernels (default 2e9).  Applies to launches made after the call. */
+int dqt_set_wait_limit_ns(uint64_t ns);
+
+/* Eq. 2-4, initialisation (not on the training hot path).
+ *   W0      fp32 [numel] dense initial weight (device)
+ *   codes   int8 [numel] out: Clip[Round(W0 * s_w), qmin, qmax], Round half-to-even
+ *   s_w     HOST float out: qmax / AbsMean(W0), AbsMean = (1/numel) sum |w| in fp64
+ *   ws      device workspace of at least dqt_absmean_workspace_size() bytes
+ * Synchronous: returns after s_w is known and the codes kernel is enqueued. */
+size_t dqt_absmean_workspace_size(void);
+int dqt_absmean_init(const float* W0, int64_t numel, dqt_grid_t grid, int8_t* codes,
+                     float* s_w, void* ws, size_t ws_bytes, void* stream);
+
+/* Sec. 3.2, activation quantisation "following BitNet", 8 bits per token:
+ *   amax[t] = max_k |X[t,k]|,  s_x[t] = 127 / max(amax[t], 1e-5)   (fp32 divide)
+ *   Xq[t,k] = Clip[Round(X[t,k] * s_x[t]), -128, 127]              (fp32 multiply, half-to-even)
+ *   X       bf16 [T, K] in
+ *   Xq      int8 [T, K] out, or NULL
+ *   s_x     fp32 [T] out (required)
+ *   Xq_img  bf16 [T, K] out, or NULL: the codes as exact bf16 values (forward GEMM operand)
+ *   Xdq     bf16 [T, K] out, or NULL: bf16(Xq / s_x), the dequantised activation
+ *           X_tilde that the weight gradient uses (backward GEMM operand)
+ * At least one of Xq, Xq_img, Xdq must be non-NULL. */
+int dqt_act_quant(const dqt_bf16* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
+                  dqt_bf16* Xq_img, dqt_bf16* Xdq, void* stream);
+
+/* Exact bf16 image of int8 codes: W_img[i] = (bf16) W[i].  numel >= 1. */
+int dqt_codes_to_bf16(const int8_t* W, int64_t numel, dqt_bf16* W_img, void* stream);
+
+/* Sec. 3.2 forward, Y = X_tilde W_tilde^T with X_tilde = Xq / s_x, W_tilde = c / s_w:
+ *   acc[t,n] = sum_k Xq[t,k] c[n,k]             exact (int32)
+ *   Y[t,n]   = bf16( float(acc) * (1 / (s_x[t] * s_w)) )
+ *   Xq_img   bf16 [T, K] exact code image from dqt_act_quant (|value| <= 128)
+ *   s_x      fp32 [T]
+ *   W_img    bf16 [N, K] exact code image of the weight (dqt_codes_to_bf16)
+ *   grid     the weight grid; it bounds |c| and so how often the kernel drains its
+ *            fp32 accumulator into int32 to keep every partial sum exact
+ *   Y        bf16 [T, N] out;  acc_out int32 [T, N] out, or NULL
+ * K, N multiples of 8; T >= 1; T, N, K < 2^31. */
+int dqt_bitlinear_fwd(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img,
+                      float s_w, dqt_grid_t grid, int64_t T, int64_t K, int64_t N,
+                      dqt_bf16* Y, int32_t* acc_out, void* stream);
+
+/* Backward w.r.t. the input, no straight-through estimator on the weight
+ * (the gradient is taken w.r.t. W_tilde itself, Sec. 3.2):
+ *   dX[t,k] = bf16( (sum_n dY[t,n] c[n,k]) * (1 / s_w) )   fp32 accumulation
+ *   dY bf16 [T, N];  W_img bf16 [N, K];  dX bf16 [T, K] out. */
+int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, int64_t T,
+                         int64_t N, int64_t K, dqt_bf16* dX, void* stream);
+
+/* Backward w.r.t. the weight fused with the DQT update (Sec. 3.2, Sec. 4.1, Eq. 5):
+ *   g[n,k]  = sum_t dY[t,n] Xdq[t,k]              fp32 accumulation in tensor memory
+ *   m, v    <- AdamW moments (fp32 [N, K], in place)
+ *   x       = c decay - (lr s_w) * (m_hat / (sqrt(v_hat) + eps))     (= W' * s_w)
+ *   c       <- Clip[SR(x), qmin, qmax]  (int8 [N, K], in place; round_mode 1: nearest)
+ * The fp32 gradient never reaches memory unless dW_out (fp32 [N, K]) is given.
+ * With W, m and v all NULL only dW_out is written (gradient only).
+ *   dY bf16 [T, N];  Xdq bf16 [T, K] from dqt_act_quant;  hp, sr: HOST structs.
+ *   changed_out: device int64, or NULL; if given, the number of codes that changed
+ *   is ADDED to it (the weight-update frequency of Sec. 5.2). */
+int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W, float s_w,
+                                float* m, float* v, const dqt_adamw_t* hp, const dqt_sr_t* sr,
+                                dqt_grid_t grid, int64_t T, int64_t N, int64_t K,
+                                float* dW_out, unsigned long long* changed_out, void* stream);
+
+/* The AdamW + SR update of dqt_bitlinear_bwd_dw_update for a gradient already
+ * in memory (Eq. 5 as a bandwidth-bound stream; 22 bytes per weight):
+ *   grad fp32 [numel];  W int8 [numel] in place;  m, v fp32 [numel] in place.
+ * Element i uses the uniform of flat index i, so for an [N, K] weight this
+ * gives exactly the codes of the fused path for the same fp32 gradient.
+ * changed_out as above. */
+int dqt_sr_update(const float* grad, int8_t* W, float s_w, float* m, float* v,
+                  const dqt_adamw_t* hp, const dqt_sr_t* sr, dqt_grid_t grid, int64_t numel,
+                  unsigned long long* changed_out, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DQT_H_ */

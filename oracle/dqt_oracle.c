@@ -15,6 +15,7 @@
  *   Sec 3.2 8-bit activation quantisation (BitNet style)  -> dqt_oracle_act_quant
  *   Sec 3.2 BitLinear forward on the quantised operands   -> dqt_oracle_fwd
  *   Sec 3.2 backward w.r.t. the low-bit weight (no STE)   -> dqt_oracle_bwd_dx / _bwd_dw
+ *   Sec 4.1/4.3 the same with X_tilde held in bf16        -> dqt_oracle_bwd_dw_bf16x
  *   Sec 4.1 AdamW producing the dense target W'           -> dqt_oracle_adamw_x
  *   Eq. 5   W_hat = SR(W'), kept on the n-bit grid        -> dqt_oracle_update
  *   Sec 5.1 absmax / round-to-nearest ablation            -> round_mode = 1
@@ -274,6 +275,25 @@ void dqt_oracle_bwd_dw(const uint16_t* dY, const int8_t* q, const float* s_x,
       double inv = 1.0 / (double)s_x[t];
       for (int64_t k = 0; k < K; ++k)
         dW[i * K + k] += g * ((double)q[t * K + k] * inv);
+    }
+  }
+}
+
+/* ------------------------------------------------------------------------ */
+/* The same weight gradient with X_tilde held in bf16 (the BF16 training     */
+/* environment of Sec 4.1/4.3): dW[n,k] = sum_t dY[t,n] bf16(q/s_x)[t,k],    */
+/* fp64.  xdq is the bf16 image that dqt_oracle_act_quant returns.           */
+/* ------------------------------------------------------------------------ */
+void dqt_oracle_bwd_dw_bf16x(const uint16_t* dY, const uint16_t* xdq, int64_t T,
+                             int64_t N, int64_t K, const int64_t* rows, int64_t Nr,
+                             double* dW) {
+  for (int64_t i = 0; i < Nr; ++i) {
+    int64_t n = rows[i];
+    for (int64_t k = 0; k < K; ++k) dW[i * K + k] = 0.0;
+    for (int64_t t = 0; t < T; ++t) {
+      double g = (double)bf16_to_f32(dY[t * N + n]);
+      for (int64_t k = 0; k < K; ++k)
+        dW[i * K + k] += g * (double)bf16_to_f32(xdq[t * K + k]);
     }
   }
 }

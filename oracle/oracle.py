@@ -10,6 +10,7 @@ with Stochastic Rounding"):
 * ``act_quant``                -- Sec. 3.2, 8-bit per-token absmax activations
 * ``fwd``                      -- Sec. 3.2, BitLinear forward (exact int accumulation)
 * ``bwd_dx`` / ``bwd_dw``      -- Sec. 3.2, backward w.r.t. input and low-bit weight (fp64)
+* ``bwd_dw_bf16x``             -- Sec. 4.1/4.3, the weight gradient with X_tilde in bf16
 * ``adamw_consts``/``adamw_x`` -- Sec. 4.1, AdamW producing the dense target W'
 * ``update``                   -- Eq. 5, W_hat = SR(W') clamped onto the grid
 
@@ -64,6 +65,9 @@ def lib():
         L.dqt_oracle_bwd_dw.argtypes = [_u16p, _i8p, _f32p, C.c_int64, C.c_int64,
                                         C.c_int64, _i64p, C.c_int64, _f64p]
         L.dqt_oracle_bwd_dw.restype = None
+        L.dqt_oracle_bwd_dw_bf16x.argtypes = [_u16p, _u16p, C.c_int64, C.c_int64, C.c_int64,
+                                              _i64p, C.c_int64, _f64p]
+        L.dqt_oracle_bwd_dw_bf16x.restype = None
         L.dqt_oracle_adamw_consts.argtypes = [C.c_float, C.c_float, C.c_float, C.c_float,
                                               C.c_float, C.c_int64, C.c_float, _f32p]
         L.dqt_oracle_adamw_consts.restype = None
@@ -207,6 +211,20 @@ def bwd_dw(dY_bits, q, s_x, rows=None):
     dW = np.empty((rows.size, K), np.float64)
     lib().dqt_oracle_bwd_dw(_p(dY, _u16p), _p(q, _i8p), _p(s_x, _f32p), T, N, K,
                             _p(rows, _i64p), rows.size, _p(dW, _f64p))
+    return dW
+
+
+def bwd_dw_bf16x(dY_bits, xdq_bits, rows=None):
+    """dW with X_tilde held as the bf16 image bf16(q/s_x) (BF16 environment)."""
+    dY = _c(dY_bits, np.uint16)
+    xd = _c(xdq_bits, np.uint16)
+    T, N = dY.shape
+    T2, K = xd.shape
+    assert T == T2
+    rows = np.arange(N, dtype=np.int64) if rows is None else _c(rows, np.int64)
+    dW = np.empty((rows.size, K), np.float64)
+    lib().dqt_oracle_bwd_dw_bf16x(_p(dY, _u16p), _p(xd, _u16p), T, N, K, _p(rows, _i64p),
+                                  rows.size, _p(dW, _f64p))
     return dW
 
 

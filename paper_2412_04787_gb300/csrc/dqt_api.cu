@@ -1,0 +1,268 @@
+// C ABI of the DQT library (declared in include/dqt.h): argument checks,
+// host-side derivation of the AdamW constants, and kernel launches.
+#include <math.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <atomic>
+
+#include "../../include/dqt.h"
+#include "dqt_internal.h"
+
+namespace dqt {
+
+// One status word per device (bounded-wait timeouts, see dqt_device.cuh).
+__device__ unsigned int g_status_word;
+
+namespace {
+std::atomic<uint64_t> g_wait_ns{2000000000ull};
+constexpr int kMaxDevices = 64;
+unsigned int* g_status_ptr[kMaxDevices] = {nullptr};
+}  // namespace
+
+uint64_t wait_limit_ns() { return g_wait_ns.load(); }
+
+unsigned int* status_word() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  if (!g_status_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
+    g_status_ptr[dev] = static_cast<unsigned int*>(p);
+  }
+  return g_status_ptr[dev];
+}
+
+}  // namespace dqt
+
+namespace {
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+inline bool grid_ok(dqt_grid_t g) {
+  return g.qmin <= g.qmax && g.qmin >= -128 && g.qmax <= 127 && g.qmin <= 0 && g.qmax >= 0;
+}
+
+inline cudaStream_t as_stream(void* s) { return static_cast<cudaStream_t>(s); }
+
+// AdamW and SR constants, derived on the host in fp64 and rounded once to fp32.
+int make_update_consts(const dqt_adamw_t* hp, const dqt_sr_t* sr, dqt_grid_t g, float s_w,
+                       dqt::UpdateConsts* uc) {
+  if (!hp || !sr || !grid_ok(g)) return DQT_ERR_ARG;
+  if (hp->step < 1 || !(hp->beta1 >= 0.0f && hp->beta1 < 1.0f) ||
+      !(hp->beta2 >= 0.0f && hp->beta2 < 1.0f) || !(hp->eps >= 0.0f) || !(hp->lr >= 0.0f) ||
+      !isfinite(hp->weight_decay) || !(s_w > 0.0f) || !isfinite(s_w))
+    return DQT_ERR_ARG;
+  if (sr->round_mode != 0 && sr->round_mode != 1) return DQT_ERR_ARG;
+  const double b1 = hp->beta1, b2 = hp->beta2, st = static_cast<double>(hp->step);
+  uc->b1 = hp->beta1;
+  uc->b2 = hp->beta2;
+  uc->eps = hp->eps;
+  uc->omb1 = static_cast<float>(1.0 - b1);
+  uc->omb2 = static_cast<float>(1.0 - b2);
+  uc->bc1 = static_cast<float>(1.0 - pow(b1, st));
+  uc->bc2 = static_cast<float>(1.0 - pow(b2, st));
+  uc->decay = static_cast<float>(1.0 - static_cast<double>(hp->lr) * hp->weight_decay);
+  uc->lrs = static_cast<float>(static_cast<double>(hp->lr) * static_cast<double>(s_w));
+  if (!(uc->bc1 > 0.0f) || !(uc->bc2 > 0.0f)) return DQT_ERR_ARG;
+  uc->qmin = g.qmin;
+  uc->qmax = g.qmax;
+  uc->step_lo = static_cast<uint32_t>(hp->step);
+  uc->tensor_id = sr->tensor_id;
+  uc->key0 = static_cast<uint32_t>(sr->seed);
+  uc->key1 = static_cast<uint32_t>(sr->seed >> 32);
+  uc->round_mode = sr->round_mode;
+  return DQT_OK;
+}
+
+constexpr int64_t kMaxDim = (int64_t(1) << 31) - 1;
+
+}  // namespace
+
+extern "C" {
+
+const char* dqt_status_string(int s) {
+  switch (s) {
+    case DQT_OK: return "DQT_OK";
+    case DQT_ERR_ARG: return "DQT_ERR_ARG: invalid argument";
+    case DQT_ERR_ALIGN: return "DQT_ERR_ALIGN: pointer not 16-byte aligned or K/N not a multiple of 8";
+    case DQT_ERR_CUDA: return "DQT_ERR_CUDA: CUDA call failed";
+    case DQT_ERR_TIMEOUT: return "DQT_ERR_TIMEOUT: a bounded device wait ran out";
+    case DQT_ERR_RANGE: return "DQT_ERR_RANGE: size out of the supported range";
+    default: return "DQT: unknown status";
+  }
+}
+
+int dqt_grid_for_bits(float bits, dqt_grid_t* out) {
+  if (!out) return DQT_ERR_ARG;
+  if (fabsf(bits - 1.58f) < 1e-3f) {
+    out->qmin = -1;
+    out->qmax = 1;
+    return DQT_OK;
+  }
+  const float r = rintf(bits);
+  if (r != bits || r < 2.0f || r > 8.0f) return DQT_ERR_ARG;
+  const int n = static_cast<int>(r);
+  out->qmin = -(1 << (n - 1));
+  out->qmax = (1 << (n - 1)) - 1;
+  return DQT_OK;
+}
+
+int dqt_set_wait_limit_ns(uint64_t ns) {
+  dqt::g_wait_ns.store(ns);
+  return DQT_OK;
+}
+
+int dqt_check_device_status(void* stream) {
+  if (cudaStreamSynchronize(as_stream(stream)) != cudaSuccess) return DQT_ERR_CUDA;
+  unsigned int* p = dqt::status_word();
+  if (!p) return DQT_ERR_CUDA;
+  unsigned int h = 0;
+  if (cudaMemcpy(&h, p, sizeof(h), cudaMemcpyDeviceToHost) != cudaSuccess) return DQT_ERR_CUDA;
+  if (h != 0) {
+    const unsigned int zero = 0;
+    if (cudaMemcpy(p, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess)
+      return DQT_ERR_CUDA;
+    return DQT_ERR_TIMEOUT;
+  }
+  return DQT_OK;
+}
+
+size_t dqt_absmean_workspace_size(void) { return (dqt::kAbsmeanBlocks + 1) * sizeof(double); }
+
+int dqt_absmean_init(const float* W0, int64_t numel, dqt_grid_t grid, int8_t* codes, float* s_w,
+                     void* ws, size_t ws_bytes, void* stream) {
+  if (!W0 || !codes || !s_w || !ws || numel <= 0 || !grid_ok(grid) || grid.qmax <= 0)
+    return DQT_ERR_ARG;
+  if (ws_bytes < dqt_absmean_workspace_size()) return DQT_ERR_ARG;
+  if ((reinterpret_cast<uintptr_t>(ws) & 7u) != 0) return DQT_ERR_ALIGN;
+  cudaStream_t st = as_stream(stream);
+  double* dws = static_cast<double*>(ws);
+  if (dqt::launch_absmean_partial(W0, numel, dws, st)) return DQT_ERR_CUDA;
+  double sum = 0.0;
+  if (cudaMemcpyAsync(&sum, dws + dqt::kAbsmeanBlocks, sizeof(double), cudaMemcpyDeviceToHost,
+                      st) != cudaSuccess)
+    return DQT_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return DQT_ERR_CUDA;
+  const double absmean = sum / static_cast<double>(numel);
+  if (!(absmean > 0.0) || !isfinite(absmean)) return DQT_ERR_ARG;
+  const float s = static_cast<float>(static_cast<double>(grid.qmax) / absmean);
+  *s_w = s;
+  return dqt::launch_absmean_codes(W0, numel, s, grid.qmin, grid.qmax, codes, st) ? DQT_ERR_CUDA
+                                                                                    : DQT_OK;
+}
+
+int dqt_act_quant(const dqt_bf16* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
+                  dqt_bf16* Xq_img, dqt_bf16* Xdq, void* stream) {
+  if (!X || !s_x || (!Xq && !Xq_img && !Xdq) || T <= 0 || K <= 0) return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim) return DQT_ERR_RANGE;
+  if (K % 8 || !aligned16(X) || (Xq && (reinterpret_cast<uintptr_t>(Xq) & 7u)) ||
+      (Xq_img && !aligned16(Xq_img)) || (Xdq && !aligned16(Xdq)))
+    return DQT_ERR_ALIGN;
+  return dqt::launch_act_quant(X, T, K, Xq, s_x, Xq_img, Xdq, as_stream(stream)) ? DQT_ERR_CUDA
+                                                                                 : DQT_OK;
+}
+
+int dqt_codes_to_bf16(const int8_t* W, int64_t numel, dqt_bf16* W_img, void* stream) {
+  if (!W || !W_img || numel <= 0) return DQT_ERR_ARG;
+  if (!aligned16(W) || !aligned16(W_img)) return DQT_ERR_ALIGN;
+  return dqt::launch_codes_to_bf16(W, numel, W_img, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
+int dqt_bitlinear_fwd(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img, float s_w,
+                      dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
+                      int32_t* acc_out, void* stream) {
+  if (!Xq_img || !s_x || !W_img || !Y || T <= 0 || K <= 0 || N <= 0 || !grid_ok(grid) ||
+      !(s_w > 0.0f) || !isfinite(s_w))
+    return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
+  if (K % 8 || N % 8 || !aligned16(Xq_img) || !aligned16(W_img) || !aligned16(Y) ||
+      (acc_out && !aligned16(acc_out)))
+    return DQT_ERR_ALIGN;
+  const int64_t cmax = grid.qmax > -grid.qmin ? grid.qmax : -grid.qmin;
+  const int64_t cm = cmax > 0 ? cmax : 1;
+  // |sum| <= K * 128 * max|c| must fit int32.
+  if (K * 128 * cm > (int64_t(1) << 31) - 1) return DQT_ERR_RANGE;
+  // Largest chunk whose partial sums stay <= 2^24 (exact in fp32), multiple of 64.
+  int64_t chunk = ((int64_t(1) << 24) / (128 * cm)) / 64 * 64;
+  if (chunk < 64) chunk = 64;
+  if (chunk > kMaxDim) chunk = int64_t(1) << 30;
+  dqt::GemmLaunch g{};
+  g.kind = dqt::GEMM_FWD;
+  g.M = static_cast<int>(T);
+  g.N = static_cast<int>(N);
+  g.Kred = static_cast<int>(K);
+  g.A = Xq_img;
+  g.B = W_img;
+  g.chunk_k = static_cast<int>(chunk);
+  g.s_x = s_x;
+  g.scale = s_w;
+  g.out_bf16 = Y;
+  g.acc_out = acc_out;
+  return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
+int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, int64_t T,
+                         int64_t N, int64_t K, dqt_bf16* dX, void* stream) {
+  if (!dY || !W_img || !dX || T <= 0 || N <= 0 || K <= 0 || !(s_w > 0.0f) || !isfinite(s_w))
+    return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
+  if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(W_img) || !aligned16(dX))
+    return DQT_ERR_ALIGN;
+  dqt::GemmLaunch g{};
+  g.kind = dqt::GEMM_DX;
+  g.M = static_cast<int>(T);
+  g.N = static_cast<int>(K);
+  g.Kred = static_cast<int>(N);
+  g.A = dY;
+  g.B = W_img;
+  g.scale = 1.0f / s_w;
+  g.out_bf16 = dX;
+  return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
+int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W, float s_w,
+                                float* m, float* v, const dqt_adamw_t* hp, const dqt_sr_t* sr,
+                                dqt_grid_t grid, int64_t T, int64_t N, int64_t K, float* dW_out,
+                                unsigned long long* changed_out, void* stream) {
+  const bool upd = W || m || v;
+  if (!dY || !Xdq || T <= 0 || N <= 0 || K <= 0) return DQT_ERR_ARG;
+  if (upd && (!W || !m || !v)) return DQT_ERR_ARG;
+  if (!upd && !dW_out) return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
+  if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(Xdq) || (W && !aligned16(W)) ||
+      (m && !aligned16(m)) || (v && !aligned16(v)) || (dW_out && !aligned16(dW_out)))
+    return DQT_ERR_ALIGN;
+  dqt::GemmLaunch g{};
+  if (upd) {
+    const int rc = make_update_consts(hp, sr, grid, s_w, &g.uc);
+    if (rc != DQT_OK) return rc;
+  }
+  g.kind = dqt::GEMM_DW;
+  g.M = static_cast<int>(N);
+  g.N = static_cast<int>(K);
+  g.Kred = static_cast<int>(T);
+  g.A = dY;
+  g.B = Xdq;
+  g.W = upd ? W : nullptr;
+  g.m = m;
+  g.v = v;
+  g.dW_out = dW_out;
+  g.changed = upd ? changed_out : nullptr;
+  return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
+int dqt_sr_update(const float* grad, int8_t* W, float s_w, float* m, float* v,
+                  const dqt_adamw_t* hp, const dqt_sr_t* sr, dqt_grid_t grid, int64_t numel,
+                  unsigned long long* changed_out, void* stream) {
+  if (!grad || !W || !m || !v || numel <= 0) return DQT_ERR_ARG;
+  if (!aligned16(grad) || !aligned16(W) || !aligned16(m) || !aligned16(v)) return DQT_ERR_ALIGN;
+  dqt::UpdateConsts uc;
+  const int rc = make_update_consts(hp, sr, grid, s_w, &uc);
+  if (rc != DQT_OK) return rc;
+  return dqt::launch_sr_update(grad, W, m, v, numel, uc, changed_out, as_stream(stream))
+             ? DQT_ERR_CUDA
+             : DQT_OK;
+}
+
+}  // extern "C"

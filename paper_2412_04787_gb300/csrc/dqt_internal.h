@@ -1,0 +1,56 @@
+// Host-side interfaces between the C ABI (dqt_api.cu) and the kernel files.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "dqt_device.cuh"
+
+namespace dqt {
+
+// Largest wait, in ns, a kernel makes before it records a timeout.
+uint64_t wait_limit_ns();
+
+// Device address of the current device's status word (NULL on failure).
+unsigned int* status_word();
+
+enum GemmKind { GEMM_FWD = 0, GEMM_DX = 1, GEMM_DW = 2 };
+
+struct GemmLaunch {
+  GemmKind kind;
+  // Output is M x N, reduced over Kred.
+  int M, N, Kred;
+  // Operands (bf16, row-major, contiguous):
+  //   FWD: A = Xq_img [M=T, Kred=K],  B = W_img [N, Kred=K]     (both K-major)
+  //   DX : A = dY     [M=T, Kred=N],  B = W_img [Kred=N, N=K]   (B MN-major)
+  //   DW : A = dY     [Kred=T, M=N],  B = Xdq   [Kred=T, N=K]   (both MN-major)
+  const void* A;
+  const void* B;
+  int chunk_k;  // FWD: reduction elements per exact fp32 chunk (multiple of 64)
+  // Epilogue operands.
+  const float* s_x;  // FWD
+  float scale;       // FWD: s_w; DX: 1/s_w
+  void* out_bf16;    // FWD: Y; DX: dX
+  int32_t* acc_out;  // FWD, optional
+  int8_t* W;         // DW (with m, v), optional
+  float* m;
+  float* v;
+  float* dW_out;  // DW, optional
+  unsigned long long* changed;
+  UpdateConsts uc;
+};
+
+int launch_gemm(const GemmLaunch& g, cudaStream_t stream);
+
+int launch_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
+                     uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream);
+int launch_codes_to_bf16(const int8_t* W, int64_t numel, uint16_t* W_img, cudaStream_t stream);
+int launch_absmean_partial(const float* W0, int64_t numel, double* ws, cudaStream_t stream);
+int launch_absmean_codes(const float* W0, int64_t numel, float s_w, int32_t qmin, int32_t qmax,
+                         int8_t* codes, cudaStream_t stream);
+constexpr int kAbsmeanBlocks = 1024;
+
+int launch_sr_update(const float* grad, int8_t* W, float* m, float* v, int64_t numel,
+                     const UpdateConsts& uc, unsigned long long* changed, cudaStream_t stream);
+
+}  // namespace dqt

@@ -1,0 +1,206 @@
+// Bandwidth-bound quantisation kernels of a DQT BitLinear step:
+//   act_quant      8-bit per-token absmax activation codes (Sec. 3.2) plus the
+//                  bf16 operand images the tensor-core GEMMs read
+//   codes_to_bf16  exact bf16 image of the int8 weight codes
+//   absmean_*      Eq. 2-4 initialisation (deterministic fp64 reduction)
+#include "dqt_internal.h"
+
+namespace dqt {
+
+namespace {
+
+__device__ __forceinline__ float bf16_bits_to_f32(uint32_t h) { return __uint_as_float(h << 16); }
+
+__device__ __forceinline__ uint16_t f32_to_bf16_bits(float f) {
+  const __nv_bfloat16 h = __float2bfloat16_rn(f);
+  return *reinterpret_cast<const uint16_t*>(&h);
+}
+
+// One warp per token row; 16-byte (8 x bf16) vector accesses.  Pass 1 finds
+// amax; pass 2 re-reads the row (an L1/L2 hit) and writes the outputs.
+constexpr int kAqWarps = 8;
+
+__global__ void __launch_bounds__(kAqWarps * 32)
+    act_quant_kernel(const uint16_t* __restrict__ X, int T, int K, int8_t* __restrict__ Xq,
+                     float* __restrict__ s_x, uint16_t* __restrict__ Xq_img,
+                     uint16_t* __restrict__ Xdq) {
+  const int row = blockIdx.x * kAqWarps + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= T) return;
+  const int nv = K >> 3;
+  const uint4* xr = reinterpret_cast<const uint4*>(X + static_cast<size_t>(row) * K);
+
+  float amax = 0.0f;
+#pragma unroll 4
+  for (int i = lane; i < nv; i += 32) {
+    const uint4 u = __ldg(xr + i);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      amax = fmaxf(amax, fabsf(bf16_bits_to_f32(w[j] & 0xFFFFu)));
+      amax = fmaxf(amax, fabsf(bf16_bits_to_f32(w[j] >> 16)));
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+  const float s = __fdiv_rn(127.0f, fmaxf(amax, 1e-5f));
+  if (lane == 0) s_x[row] = s;
+
+  const size_t rbase = static_cast<size_t>(row) * K;
+#pragma unroll 4
+  for (int i = lane; i < nv; i += 32) {
+    const uint4 u = __ldg(xr + i);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+    int32_t q[8];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float lo = bf16_bits_to_f32(w[j] & 0xFFFFu);
+      const float hi = bf16_bits_to_f32(w[j] >> 16);
+      q[2 * j] = static_cast<int32_t>(fminf(fmaxf(rintf(__fmul_rn(lo, s)), -128.0f), 127.0f));
+      q[2 * j + 1] = static_cast<int32_t>(fminf(fmaxf(rintf(__fmul_rn(hi, s)), -128.0f), 127.0f));
+    }
+    const size_t e = rbase + static_cast<size_t>(i) * 8;
+    if (Xq) {
+      uint2 pk;
+      pk.x = (q[0] & 0xFF) | ((q[1] & 0xFF) << 8) | ((q[2] & 0xFF) << 16) | ((q[3] & 0xFF) << 24);
+      pk.y = (q[4] & 0xFF) | ((q[5] & 0xFF) << 8) | ((q[6] & 0xFF) << 16) | ((q[7] & 0xFF) << 24);
+      *reinterpret_cast<uint2*>(Xq + e) = pk;
+    }
+    if (Xq_img) {
+      uint4 pk;
+      pk.x = f32_to_bf16_bits(static_cast<float>(q[0])) | (uint32_t(f32_to_bf16_bits(static_cast<float>(q[1]))) << 16);
+      pk.y = f32_to_bf16_bits(static_cast<float>(q[2])) | (uint32_t(f32_to_bf16_bits(static_cast<float>(q[3]))) << 16);
+      pk.z = f32_to_bf16_bits(static_cast<float>(q[4])) | (uint32_t(f32_to_bf16_bits(static_cast<float>(q[5]))) << 16);
+      pk.w = f32_to_bf16_bits(static_cast<float>(q[6])) | (uint32_t(f32_to_bf16_bits(static_cast<float>(q[7]))) << 16);
+      *reinterpret_cast<uint4*>(Xq_img + e) = pk;
+    }
+    if (Xdq) {
+      uint32_t h[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) h[j] = f32_to_bf16_bits(__fdiv_rn(static_cast<float>(q[j]), s));
+      uint4 pk;
+      pk.x = h[0] | (h[1] << 16);
+      pk.y = h[2] | (h[3] << 16);
+      pk.z = h[4] | (h[5] << 16);
+      pk.w = h[6] | (h[7] << 16);
+      *reinterpret_cast<uint4*>(Xdq + e) = pk;
+    }
+  }
+}
+
+// 16 codes per thread per step: one 16-byte load, two 16-byte stores.
+__global__ void codes_to_bf16_kernel(const int8_t* __restrict__ W, int64_t numel,
+                                     uint16_t* __restrict__ img) {
+  const int64_t nvec = numel >> 4;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
+       i += stride) {
+    const uint4 u = __ldg(reinterpret_cast<const uint4*>(W) + i);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+    uint32_t o[8];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int32_t b0 = static_cast<int8_t>(w[j] & 0xFF);
+      const int32_t b1 = static_cast<int8_t>((w[j] >> 8) & 0xFF);
+      const int32_t b2 = static_cast<int8_t>((w[j] >> 16) & 0xFF);
+      const int32_t b3 = static_cast<int8_t>(w[j] >> 24);
+      o[2 * j] = f32_to_bf16_bits(static_cast<float>(b0)) |
+                 (uint32_t(f32_to_bf16_bits(static_cast<float>(b1))) << 16);
+      o[2 * j + 1] = f32_to_bf16_bits(static_cast<float>(b2)) |
+                     (uint32_t(f32_to_bf16_bits(static_cast<float>(b3))) << 16);
+    }
+    uint4* dst = reinterpret_cast<uint4*>(img) + 2 * i;
+    dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
+    dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
+  }
+  // ragged tail (numel % 16 elements), one thread
+  if (blockIdx.x == 0 && threadIdx.x == 0)
+    for (int64_t e = nvec << 4; e < numel; ++e) img[e] = f32_to_bf16_bits(static_cast<float>(W[e]));
+}
+
+// Eq. 2, stage 1: each of kAbsmeanBlocks blocks sums |w| in fp64 over a fixed
+// strided subset and reduces in a fixed tree: the result does not depend on
+// scheduling.
+constexpr int kAbsThreads = 256;
+
+__global__ void __launch_bounds__(kAbsThreads)
+    absmean_partial_kernel(const float* __restrict__ W0, int64_t numel, double* __restrict__ ws) {
+  __shared__ double sh[kAbsThreads];
+  const int64_t stride = static_cast<int64_t>(kAbsmeanBlocks) * kAbsThreads;
+  double acc = 0.0;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * kAbsThreads + threadIdx.x; i < numel;
+       i += stride)
+    acc += fabs(static_cast<double>(W0[i]));
+  sh[threadIdx.x] = acc;
+  __syncthreads();
+  for (int w = kAbsThreads / 2; w > 0; w >>= 1) {
+    if (threadIdx.x < w) sh[threadIdx.x] += sh[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) ws[blockIdx.x] = sh[0];
+}
+
+// Eq. 2, stage 2: one block reduces the kAbsmeanBlocks partials, fixed tree.
+__global__ void __launch_bounds__(kAbsmeanBlocks) absmean_final_kernel(double* ws) {
+  __shared__ double sh[kAbsmeanBlocks];
+  sh[threadIdx.x] = ws[threadIdx.x];
+  __syncthreads();
+  for (int w = kAbsmeanBlocks / 2; w > 0; w >>= 1) {
+    if (threadIdx.x < w) sh[threadIdx.x] += sh[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) ws[kAbsmeanBlocks] = sh[0];
+}
+
+// Eq. 4: codes = Clip[Round(W0 * s_w), qmin, qmax], fp32 multiply, half-to-even.
+__global__ void absmean_codes_kernel(const float* __restrict__ W0, int64_t numel, float s,
+                                     int32_t qmin, int32_t qmax, int8_t* __restrict__ codes) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < numel;
+       i += stride) {
+    const float r = rintf(__fmul_rn(W0[i], s));
+    const float c = fminf(fmaxf(r, static_cast<float>(qmin)), static_cast<float>(qmax));
+    codes[i] = static_cast<int8_t>(static_cast<int32_t>(c));
+  }
+}
+
+int grid_for(int64_t work, int threads) {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t want = (work + threads - 1) / threads;
+  const int64_t cap = static_cast<int64_t>(sms) * 8;
+  return static_cast<int>(want < 1 ? 1 : (want > cap ? cap : want));
+}
+
+}  // namespace
+
+int launch_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
+                     uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream) {
+  const int blocks = static_cast<int>((T + kAqWarps - 1) / kAqWarps);
+  act_quant_kernel<<<blocks, kAqWarps * 32, 0, stream>>>(X, static_cast<int>(T),
+                                                         static_cast<int>(K), Xq, s_x, Xq_img, Xdq);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+int launch_codes_to_bf16(const int8_t* W, int64_t numel, uint16_t* W_img, cudaStream_t stream) {
+  const int threads = 256;
+  codes_to_bf16_kernel<<<grid_for((numel >> 4) + 1, threads), threads, 0, stream>>>(W, numel, W_img);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+int launch_absmean_partial(const float* W0, int64_t numel, double* ws, cudaStream_t stream) {
+  absmean_partial_kernel<<<kAbsmeanBlocks, kAbsThreads, 0, stream>>>(W0, numel, ws);
+  absmean_final_kernel<<<1, kAbsmeanBlocks, 0, stream>>>(ws);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+int launch_absmean_codes(const float* W0, int64_t numel, float s_w, int32_t qmin, int32_t qmax,
+                         int8_t* codes, cudaStream_t stream) {
+  const int threads = 256;
+  absmean_codes_kernel<<<grid_for(numel, threads), threads, 0, stream>>>(W0, numel, s_w, qmin,
+                                                                         qmax, codes);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+}  // namespace dqt

@@ -1,0 +1,84 @@
+// Standalone DQT weight update (Sec. 4.1 AdamW, Eq. 1 stochastic rounding,
+// Eq. 5 W_hat = SR(W')) for a gradient already in memory: a streaming,
+// HBM-bound kernel moving 22 bytes per weight (read g, m, v, c; write m, v, c).
+//
+// Each thread step handles one group of four consecutive weights, which is
+// exactly one Philox4x32-10 block (element e uses word e % 4 of block e / 4),
+// with 16-byte loads and stores of g, m, v and a 4-byte access to the codes.
+#include "dqt_internal.h"
+
+namespace dqt {
+
+namespace {
+
+constexpr int kThreads = 256;
+
+__global__ void __launch_bounds__(kThreads)
+    sr_update_kernel(const float* __restrict__ grad, int8_t* __restrict__ W,
+                     float* __restrict__ m, float* __restrict__ v, int64_t numel,
+                     const UpdateConsts uc, unsigned long long* changed) {
+  const int64_t ngroups = numel >> 2;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * kThreads;
+  uint32_t n_changed = 0;
+  for (int64_t gi = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; gi < ngroups;
+       gi += stride) {
+    const int64_t e = gi << 2;
+    const float4 g4 = __ldcs(reinterpret_cast<const float4*>(grad + e));
+    float4 m4 = __ldcs(reinterpret_cast<const float4*>(m + e));
+    float4 v4 = __ldcs(reinterpret_cast<const float4*>(v + e));
+    const char4 c4 = *reinterpret_cast<const char4*>(W + e);
+    uint4 w = make_uint4(0, 0, 0, 0);
+    if (uc.round_mode == 0) w = sr_words(static_cast<uint64_t>(gi), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
+    const int32_t a = dqt_update_elem(uc, g4.x, c4.x, m4.x, v4.x, w.x);
+    const int32_t b = dqt_update_elem(uc, g4.y, c4.y, m4.y, v4.y, w.y);
+    const int32_t c = dqt_update_elem(uc, g4.z, c4.z, m4.z, v4.z, w.z);
+    const int32_t d = dqt_update_elem(uc, g4.w, c4.w, m4.w, v4.w, w.w);
+    n_changed += (a != c4.x) + (b != c4.y) + (c != c4.z) + (d != c4.w);
+    *reinterpret_cast<char4*>(W + e) =
+        make_char4(static_cast<signed char>(a), static_cast<signed char>(b),
+                   static_cast<signed char>(c), static_cast<signed char>(d));
+    __stcs(reinterpret_cast<float4*>(m + e), m4);
+    __stcs(reinterpret_cast<float4*>(v + e), v4);
+  }
+  // ragged tail: the last numel % 4 elements, one thread, scalar accesses
+  if (blockIdx.x == 0 && threadIdx.x == 0 && (numel & 3)) {
+    const int64_t gi = ngroups;
+    uint4 w = make_uint4(0, 0, 0, 0);
+    if (uc.round_mode == 0) w = sr_words(static_cast<uint64_t>(gi), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
+    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+    for (int64_t e = gi << 2; e < numel; ++e) {
+      float mm = m[e], vv = v[e];
+      const int32_t c0 = W[e];
+      const int32_t r = dqt_update_elem(uc, grad[e], c0, mm, vv, ws[e & 3]);
+      n_changed += (r != c0);
+      W[e] = static_cast<int8_t>(r);
+      m[e] = mm;
+      v[e] = vv;
+    }
+  }
+  if (changed) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) n_changed += __shfl_xor_sync(0xffffffffu, n_changed, off);
+    if ((threadIdx.x & 31) == 0 && n_changed)
+      atomicAdd(changed, static_cast<unsigned long long>(n_changed));
+  }
+}
+
+}  // namespace
+
+int launch_sr_update(const float* grad, int8_t* W, float* m, float* v, int64_t numel,
+                     const UpdateConsts& uc, unsigned long long* changed, cudaStream_t stream) {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t groups = (numel + 3) >> 2;
+  int64_t blocks = (groups + kThreads - 1) / kThreads;
+  const int64_t cap = static_cast<int64_t>(sms) * 8;  // 8 resident 256-thread blocks per SM
+  if (blocks > cap) blocks = cap;
+  if (blocks < 1) blocks = 1;
+  sr_update_kernel<<<static_cast<int>(blocks), kThreads, 0, stream>>>(grad, W, m, v, numel, uc,
+                                                                      changed);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+}  // namespace dqt

@@ -1,0 +1,264 @@
+"""Python binding of the DQT C ABI (``include/dqt.h``), argument marshalling only.
+
+Every function has the name of the C entry point it calls, takes CUDA torch
+tensors, checks dtype / device / contiguity / shape, and passes raw device
+pointers and the current CUDA stream to ``libdqt.so``.  All arithmetic runs in
+the library's CUDA kernels; if the library is missing, loading it raises.
+"""
+import ctypes as C
+import os
+
+import torch
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libdqt.so")
+_lib = None
+
+DQT_OK, DQT_ERR_ARG, DQT_ERR_ALIGN, DQT_ERR_CUDA, DQT_ERR_TIMEOUT, DQT_ERR_RANGE = range(6)
+
+# Every symbol include/dqt.h declares.
+EXPORTED = [
+    "dqt_grid_for_bits", "dqt_status_string", "dqt_check_device_status",
+    "dqt_set_wait_limit_ns", "dqt_absmean_workspace_size", "dqt_absmean_init",
+    "dqt_act_quant", "dqt_codes_to_bf16", "dqt_bitlinear_fwd", "dqt_bitlinear_bwd_dx",
+    "dqt_bitlinear_bwd_dw_update", "dqt_sr_update",
+]
+
+
+class DQTError(RuntimeError):
+    def __init__(self, status, where):
+        self.status = status
+        super().__init__("%s: %s" % (where, lib().dqt_status_string(status).decode()))
+
+
+class dqt_grid_t(C.Structure):
+    _fields_ = [("qmin", C.c_int32), ("qmax", C.c_int32)]
+
+
+class dqt_adamw_t(C.Structure):
+    _fields_ = [("lr", C.c_float), ("beta1", C.c_float), ("beta2", C.c_float),
+                ("eps", C.c_float), ("weight_decay", C.c_float), ("step", C.c_int64)]
+
+
+class dqt_sr_t(C.Structure):
+    _fields_ = [("seed", C.c_uint64), ("tensor_id", C.c_uint32), ("round_mode", C.c_int32)]
+
+
+_vp, _i64, _f32, _sz = C.c_void_p, C.c_int64, C.c_float, C.c_size_t
+
+
+def lib():
+    """Load libdqt.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_LIB_PATH):
+            raise RuntimeError("libdqt.so is not built (run __graft_entry__.build()); "
+                               "the DQT library has no CPU fallback")
+        L = C.CDLL(_LIB_PATH)
+        L.dqt_grid_for_bits.argtypes = [_f32, C.POINTER(dqt_grid_t)]
+        L.dqt_status_string.argtypes = [C.c_int]
+        L.dqt_status_string.restype = C.c_char_p
+        L.dqt_check_device_status.argtypes = [_vp]
+        L.dqt_set_wait_limit_ns.argtypes = [C.c_uint64]
+        L.dqt_absmean_workspace_size.argtypes = []
+        L.dqt_absmean_workspace_size.restype = _sz
+        L.dqt_absmean_init.argtypes = [_vp, _i64, dqt_grid_t, _vp, C.POINTER(C.c_float), _vp,
+                                       _sz, _vp]
+        L.dqt_act_quant.argtypes = [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp]
+        L.dqt_codes_to_bf16.argtypes = [_vp, _i64, _vp, _vp]
+        L.dqt_bitlinear_fwd.argtypes = [_vp, _vp, _vp, _f32, dqt_grid_t, _i64, _i64, _i64, _vp,
+                                        _vp, _vp]
+        L.dqt_bitlinear_bwd_dx.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp]
+        L.dqt_bitlinear_bwd_dw_update.argtypes = [_vp, _vp, _vp, _f32, _vp, _vp,
+                                                  C.POINTER(dqt_adamw_t), C.POINTER(dqt_sr_t),
+                                                  dqt_grid_t, _i64, _i64, _i64, _vp, _vp, _vp]
+        L.dqt_sr_update.argtypes = [_vp, _vp, _f32, _vp, _vp, C.POINTER(dqt_adamw_t),
+                                    C.POINTER(dqt_sr_t), dqt_grid_t, _i64, _vp, _vp]
+        for name in EXPORTED:
+            if name not in ("dqt_status_string", "dqt_absmean_workspace_size"):
+                getattr(L, name).restype = C.c_int
+        _lib = L
+    return _lib
+
+
+def _check(rc, where):
+    if rc != DQT_OK:
+        raise DQTError(rc, where)
+
+
+def _ptr(t):
+    return None if t is None else C.c_void_p(t.data_ptr())
+
+
+def _need(t, name, dtype, shape=None):
+    if t is None:
+        raise ValueError("%s is required" % name)
+    if not t.is_cuda:
+        raise ValueError("%s must be a CUDA tensor" % name)
+    if t.dtype != dtype:
+        raise ValueError("%s must be %s, got %s" % (name, dtype, t.dtype))
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % name)
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError("%s must have shape %s, got %s" % (name, tuple(shape), tuple(t.shape)))
+    return t
+
+
+def _opt(t, name, dtype, shape):
+    return None if t is None else _need(t, name, dtype, shape)
+
+
+def _stream(stream=None):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return C.c_void_p(s.cuda_stream)
+
+
+def grid(bits):
+    """Eq. 3 grid for ``bits`` (1.58 or 2..8) as a dqt_grid_t."""
+    g = dqt_grid_t()
+    _check(lib().dqt_grid_for_bits(float(bits), C.byref(g)), "dqt_grid_for_bits")
+    return g
+
+
+def _grid(g):
+    if isinstance(g, dqt_grid_t):
+        return g
+    if isinstance(g, (tuple, list)):
+        return dqt_grid_t(int(g[0]), int(g[1]))
+    return grid(g)
+
+
+def adamw(lr=1e-3, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.0, step=1):
+    return dqt_adamw_t(lr, beta1, beta2, eps, weight_decay, step)
+
+
+def sr_stream(seed=1234, tensor_id=0, round_mode=0):
+    return dqt_sr_t(seed, tensor_id, round_mode)
+
+
+# ---------------------------------------------------------------------------
+# entry points
+# ---------------------------------------------------------------------------
+def dqt_check_device_status(stream=None):
+    _check(lib().dqt_check_device_status(_stream(stream)), "device status")
+
+
+def dqt_set_wait_limit_ns(ns):
+    _check(lib().dqt_set_wait_limit_ns(int(ns)), "dqt_set_wait_limit_ns")
+
+
+def dqt_absmean_init(W0, bits_or_grid, codes=None, stream=None):
+    """Eq. 2-4.  Returns (codes int8, s_w float)."""
+    _need(W0, "W0", torch.float32)
+    g = _grid(bits_or_grid)
+    codes = torch.empty(W0.shape, dtype=torch.int8, device=W0.device) if codes is None else \
+        _need(codes, "codes", torch.int8, W0.shape)
+    nws = lib().dqt_absmean_workspace_size()
+    ws = torch.empty(nws, dtype=torch.uint8, device=W0.device)
+    s = C.c_float()
+    _check(lib().dqt_absmean_init(_ptr(W0), W0.numel(), g, _ptr(codes), C.byref(s), _ptr(ws),
+                                  nws, _stream(stream)), "dqt_absmean_init")
+    return codes, float(s.value)
+
+
+def dqt_act_quant(X, Xq=None, s_x=None, Xq_img=None, Xdq=None, want=("Xq", "Xq_img", "Xdq"),
+                  stream=None):
+    """Sec. 3.2 activation codes.  Outputs not passed are allocated if named in
+    ``want``.  Returns (Xq, s_x, Xq_img, Xdq), None for outputs not produced."""
+    _need(X, "X", torch.bfloat16)
+    if X.dim() != 2:
+        raise ValueError("X must be [T, K]")
+    T, K = X.shape
+    dev = X.device
+    if Xq is None and "Xq" in want:
+        Xq = torch.empty((T, K), dtype=torch.int8, device=dev)
+    if Xq_img is None and "Xq_img" in want:
+        Xq_img = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
+    if Xdq is None and "Xdq" in want:
+        Xdq = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
+    if s_x is None:
+        s_x = torch.empty(T, dtype=torch.float32, device=dev)
+    _opt(Xq, "Xq", torch.int8, (T, K))
+    _need(s_x, "s_x", torch.float32, (T,))
+    _opt(Xq_img, "Xq_img", torch.bfloat16, (T, K))
+    _opt(Xdq, "Xdq", torch.bfloat16, (T, K))
+    _check(lib().dqt_act_quant(_ptr(X), T, K, _ptr(Xq), _ptr(s_x), _ptr(Xq_img), _ptr(Xdq),
+                               _stream(stream)), "dqt_act_quant")
+    return Xq, s_x, Xq_img, Xdq
+
+
+def dqt_codes_to_bf16(W, W_img=None, stream=None):
+    _need(W, "W", torch.int8)
+    if W_img is None:
+        W_img = torch.empty(W.shape, dtype=torch.bfloat16, device=W.device)
+    _need(W_img, "W_img", torch.bfloat16, W.shape)
+    _check(lib().dqt_codes_to_bf16(_ptr(W), W.numel(), _ptr(W_img), _stream(stream)),
+           "dqt_codes_to_bf16")
+    return W_img
+
+
+def dqt_bitlinear_fwd(Xq_img, s_x, W_img, s_w, bits_or_grid, Y=None, acc_out=None, stream=None):
+    _need(Xq_img, "Xq_img", torch.bfloat16)
+    T, K = Xq_img.shape
+    _need(W_img, "W_img", torch.bfloat16)
+    N = W_img.shape[0]
+    _need(W_img, "W_img", torch.bfloat16, (N, K))
+    _need(s_x, "s_x", torch.float32, (T,))
+    if Y is None:
+        Y = torch.empty((T, N), dtype=torch.bfloat16, device=Xq_img.device)
+    _need(Y, "Y", torch.bfloat16, (T, N))
+    _opt(acc_out, "acc_out", torch.int32, (T, N))
+    _check(lib().dqt_bitlinear_fwd(_ptr(Xq_img), _ptr(s_x), _ptr(W_img), float(s_w),
+                                   _grid(bits_or_grid), T, K, N, _ptr(Y), _ptr(acc_out),
+                                   _stream(stream)), "dqt_bitlinear_fwd")
+    return Y
+
+
+def dqt_bitlinear_bwd_dx(dY, W_img, s_w, dX=None, stream=None):
+    _need(dY, "dY", torch.bfloat16)
+    T, N = dY.shape
+    _need(W_img, "W_img", torch.bfloat16)
+    K = W_img.shape[1]
+    _need(W_img, "W_img", torch.bfloat16, (N, K))
+    if dX is None:
+        dX = torch.empty((T, K), dtype=torch.bfloat16, device=dY.device)
+    _need(dX, "dX", torch.bfloat16, (T, K))
+    _check(lib().dqt_bitlinear_bwd_dx(_ptr(dY), _ptr(W_img), float(s_w), T, N, K, _ptr(dX),
+                                      _stream(stream)), "dqt_bitlinear_bwd_dx")
+    return dX
+
+
+def dqt_bitlinear_bwd_dw_update(dY, Xdq, W, s_w, m, v, hp, sr, bits_or_grid, dW_out=None,
+                                changed_out=None, stream=None):
+    """Fused dW GEMM + AdamW + stochastic rounding; W, m, v updated in place.
+    With W = m = v = None only dW_out is computed."""
+    _need(dY, "dY", torch.bfloat16)
+    T, N = dY.shape
+    _need(Xdq, "Xdq", torch.bfloat16)
+    K = Xdq.shape[1]
+    _need(Xdq, "Xdq", torch.bfloat16, (T, K))
+    _opt(W, "W", torch.int8, (N, K))
+    _opt(m, "m", torch.float32, (N, K))
+    _opt(v, "v", torch.float32, (N, K))
+    _opt(dW_out, "dW_out", torch.float32, (N, K))
+    _opt(changed_out, "changed_out", torch.int64, (1,))
+    _check(lib().dqt_bitlinear_bwd_dw_update(
+        _ptr(dY), _ptr(Xdq), _ptr(W), float(s_w), _ptr(m), _ptr(v),
+        C.byref(hp) if hp is not None else None, C.byref(sr) if sr is not None else None,
+        _grid(bits_or_grid), T, N, K, _ptr(dW_out), _ptr(changed_out), _stream(stream)),
+        "dqt_bitlinear_bwd_dw_update")
+    return W
+
+
+def dqt_sr_update(grad, W, s_w, m, v, hp, sr, bits_or_grid, changed_out=None, stream=None):
+    _need(grad, "grad", torch.float32)
+    n = grad.numel()
+    _need(W, "W", torch.int8)
+    _need(m, "m", torch.float32)
+    _need(v, "v", torch.float32)
+    if W.numel() != n or m.numel() != n or v.numel() != n:
+        raise ValueError("grad, W, m, v must have the same number of elements")
+    _opt(changed_out, "changed_out", torch.int64, (1,))
+    _check(lib().dqt_sr_update(_ptr(grad), _ptr(W), float(s_w), _ptr(m), _ptr(v), C.byref(hp),
+                               C.byref(sr), _grid(bits_or_grid), n, _ptr(changed_out),
+                               _stream(stream)), "dqt_sr_update")
+    return W

@@ -1,0 +1,110 @@
+"""The C-ABI library without a GPU: it builds, loads, exports every symbol that
+include/dqt.h declares, and rejects bad arguments on the host before any CUDA
+call.  No kernel is launched here."""
+import ctypes as C
+import os
+import re
+
+import pytest
+
+from paper_2412_04787_gb300 import build as dqt_build
+from paper_2412_04787_gb300 import dqt
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "dqt.h")
+
+
+@pytest.fixture(scope="module")
+def L():
+    dqt_build.build()
+    return dqt.lib()
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(dqt_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_header_symbols_exported(L):
+    names = _declared()
+    assert len(names) >= 12
+    assert sorted(dqt.EXPORTED) == names
+    for n in names:
+        assert hasattr(L, n), n  # dlsym succeeds
+
+
+def test_north_star_entry_points_present():
+    for n in ["dqt_act_quant", "dqt_bitlinear_fwd", "dqt_bitlinear_bwd_dx",
+              "dqt_bitlinear_bwd_dw_update", "dqt_sr_update"]:
+        assert n in _declared()
+
+
+def test_grid_for_bits(L):
+    g = dqt.dqt_grid_t()
+    assert L.dqt_grid_for_bits(C.c_float(1.58), C.byref(g)) == 0 and (g.qmin, g.qmax) == (-1, 1)
+    for n in range(2, 9):
+        assert L.dqt_grid_for_bits(C.c_float(n), C.byref(g)) == 0
+        assert (g.qmin, g.qmax) == (-(2 ** (n - 1)), 2 ** (n - 1) - 1)
+    for bad in (1.0, 9.0, 2.5):
+        assert L.dqt_grid_for_bits(C.c_float(bad), C.byref(g)) == dqt.DQT_ERR_ARG
+
+
+def test_status_strings(L):
+    for s in range(6):
+        assert L.dqt_status_string(s).startswith(b"DQT")
+    assert L.dqt_status_string(99) == b"DQT: unknown status"
+
+
+def _p(addr):
+    return C.c_void_p(addr)
+
+
+def test_argument_validation_without_launch(L):
+    g = dqt.dqt_grid_t(-1, 1)
+    A = _p(0x10000)  # never dereferenced: validation fails before any CUDA call
+    # null pointers
+    assert L.dqt_bitlinear_fwd(None, A, A, 1.0, g, 4, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_bwd_dx(A, None, 1.0, 4, 8, 8, A, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_act_quant(A, 4, 8, None, A, None, None, None) == dqt.DQT_ERR_ARG
+    # sizes
+    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g, 0, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_act_quant(A, -1, 8, A, A, None, None, None) == dqt.DQT_ERR_ARG
+    # K, N multiples of 8 and 16-byte alignment
+    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g, 4, 12, 8, A, None, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_bitlinear_bwd_dx(A, A, 1.0, 4, 8, 20, A, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_bitlinear_fwd(_p(0x10004), A, A, 1.0, g, 4, 8, 8, A, None, None) == dqt.DQT_ERR_ALIGN
+    # bad grid / scale
+    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, dqt.dqt_grid_t(2, 1), 4, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, dqt.dqt_grid_t(-129, 1), 4, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_fwd(A, A, A, 0.0, g, 4, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
+    # int32 accumulator range: K * 128 * 128 must fit int32
+    g8 = dqt.dqt_grid_t(-128, 127)
+    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g8, 4, 1 << 17, 8, A, None, None) == dqt.DQT_ERR_RANGE
+
+
+def test_update_argument_validation(L):
+    g = dqt.dqt_grid_t(-1, 1)
+    A = _p(0x10000)
+    hp = dqt.adamw()
+    sr = dqt.sr_stream()
+    ok = C.byref(hp), C.byref(sr)
+    # partial state
+    assert L.dqt_bitlinear_bwd_dw_update(A, A, A, 1.0, None, A, *ok, g, 4, 8, 8, None, None, None) == dqt.DQT_ERR_ARG
+    # gradient-only mode needs dW_out
+    assert L.dqt_bitlinear_bwd_dw_update(A, A, None, 1.0, None, None, *ok, g, 4, 8, 8, None, None, None) == dqt.DQT_ERR_ARG
+    bad = dqt.adamw(step=0)
+    assert L.dqt_sr_update(A, A, 1.0, A, A, C.byref(bad), C.byref(sr), g, 16, None, None) == dqt.DQT_ERR_ARG
+    bad = dqt.adamw(beta1=1.0)
+    assert L.dqt_sr_update(A, A, 1.0, A, A, C.byref(bad), C.byref(sr), g, 16, None, None) == dqt.DQT_ERR_ARG
+    badsr = dqt.sr_stream(round_mode=2)
+    assert L.dqt_sr_update(A, A, 1.0, A, A, C.byref(hp), C.byref(badsr), g, 16, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_sr_update(A, A, -1.0, A, A, *ok, g, 16, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_sr_update(_p(0x10008), A, 1.0, A, A, *ok, g, 16, None, None) == dqt.DQT_ERR_ALIGN
+
+
+def test_absmean_workspace(L):
+    assert L.dqt_absmean_workspace_size() >= 8 * 1025
+    s = C.c_float()
+    A = _p(0x10000)
+    assert L.dqt_absmean_init(A, 16, dqt.dqt_grid_t(-1, 1), A, C.byref(s), A, 8, None) == dqt.DQT_ERR_ARG

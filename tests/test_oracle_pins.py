@@ -270,6 +270,12 @@ def test_bwd_dx_dw_are_textbook_matmul():
     assert np.allclose(dW, dYf.T @ Xt, rtol=1e-12, atol=1e-15)
     rows = np.array([31, 0, 7])
     assert np.array_equal(oracle.bwd_dw(inputs.bf16_bits(dY), q, s_x, rows=rows), dW[rows])
+    # BF16 environment: X_tilde held as bf16(q / s_x)
+    _, _, _, xd = oracle.act_quant(inputs.bf16_bits(X))
+    Xb = torch.from_numpy(xd.view(np.int16).copy()).view(torch.bfloat16).double().numpy()
+    dWb = oracle.bwd_dw_bf16x(inputs.bf16_bits(dY), xd)
+    assert np.allclose(dWb, dYf.T @ Xb, rtol=1e-12, atol=1e-15)
+    assert np.abs(dWb - dW).max() <= 2.0**-8 * np.abs(dW).max()
 
 
 # --------------------------------------------------------------------------
