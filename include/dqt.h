@@ -114,6 +114,21 @@ size_t dqt_absmean_workspace_size(void);
 int dqt_absmean_init(const float* W0, int64_t numel, dqt_grid_t grid, int8_t* codes,
                      float* s_w, void* ws, size_t ws_bytes, void* stream);
 
+/* The AbsMean initialisation of dqt_absmean_init for callers that cannot
+ * allocate device memory (a framework that owns every device allocation
+ * through its own pool, code inside an allocator's own set-up, a job whose
+ * memory budget is fully reserved).  The paper has no counterpart: this is a
+ * deployment variant only.  It takes no workspace: the reduction's partial
+ * sums live in a static device array of 1025 doubles (8200 bytes) that every
+ * GPU loading the library holds until the process exits.  Same arguments and
+ * results as dqt_absmean_init; numel <= 2^53, else DQT_ERR_RANGE.  It calls
+ * no allocator.  The first call on a device looks up the array's device
+ * address (so make that first call before any stream capture).  All calls on
+ * a device share the array: calls that overlap on the GPU race, so serialise
+ * them.  Synchronous, like dqt_absmean_init. */
+int dqt_absmean_init_noalloc(const float* W0, int64_t numel, dqt_grid_t grid, int8_t* codes,
+                             float* s_w, void* stream);
+
 /* Sec. 3.2, activation quantisation "following BitNet", 8 bits per token:
  *   amax[t] = max_k |X[t,k]|,  s_x[t] = 127 / max(amax[t], 1e-5)   (fp32 divide)
  *   Xq[t,k] = Clip[Round(X[t,k] * s_x[t]), -128, 127]              (fp32 multiply, half-to-even)

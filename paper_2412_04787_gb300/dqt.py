@@ -20,7 +20,7 @@ EXPORTED = [
     "dqt_grid_for_bits", "dqt_status_string", "dqt_check_device_status",
     "dqt_set_wait_limit_ns", "dqt_absmean_workspace_size", "dqt_absmean_init",
     "dqt_act_quant", "dqt_codes_to_bf16", "dqt_bitlinear_fwd", "dqt_bitlinear_bwd_dx",
-    "dqt_bitlinear_bwd_dw_update", "dqt_sr_update",
+    "dqt_bitlinear_bwd_dw_update", "dqt_sr_update", "dqt_absmean_init_noalloc",
 ]
 
 
@@ -63,6 +63,8 @@ def lib():
         L.dqt_absmean_workspace_size.restype = _sz
         L.dqt_absmean_init.argtypes = [_vp, _i64, dqt_grid_t, _vp, C.POINTER(C.c_float), _vp,
                                        _sz, _vp]
+        L.dqt_absmean_init_noalloc.argtypes = [_vp, _i64, dqt_grid_t, _vp,
+                                               C.POINTER(C.c_float), _vp]
         L.dqt_act_quant.argtypes = [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp]
         L.dqt_codes_to_bf16.argtypes = [_vp, _i64, _vp, _vp]
         L.dqt_bitlinear_fwd.argtypes = [_vp, _vp, _vp, _f32, dqt_grid_t, _i64, _i64, _i64, _vp,

@@ -1,0 +1,76 @@
+"""The allocation-free AbsMean initialisation entry point.
+
+dqt_absmean_init_noalloc serves callers that cannot allocate device memory
+(a framework that owns every device allocation through its own pool, code
+inside an allocator's own set-up, a job whose memory budget is fully
+reserved): it keeps its reduction workspace in a static device array instead
+of a caller-provided buffer.  It must give the same scale and codes as
+dqt_absmean_init, call after call, with the shared array carrying the
+previous call's contents.  This file is collected last on purpose.
+"""
+import ctypes as C
+
+import numpy as np
+import pytest
+import torch
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def L():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2412_04787_gb300 import build, dqt
+    build.build()
+    return dqt.lib()
+
+
+def _with_workspace(L, W0, grid):
+    from paper_2412_04787_gb300 import dqt
+    codes = torch.empty(W0.shape, dtype=torch.int8, device="cuda")
+    nws = L.dqt_absmean_workspace_size()
+    ws = torch.empty(nws, dtype=torch.uint8, device="cuda")
+    s = C.c_float()
+    st = C.c_void_p(torch.cuda.current_stream().cuda_stream)
+    rc = L.dqt_absmean_init(C.c_void_p(W0.data_ptr()), W0.numel(), grid,
+                            C.c_void_p(codes.data_ptr()), C.byref(s), C.c_void_p(ws.data_ptr()),
+                            nws, st)
+    assert rc == dqt.DQT_OK
+    return codes, s.value
+
+
+def _no_alloc(L, W0, grid):
+    from paper_2412_04787_gb300 import dqt
+    codes = torch.empty(W0.shape, dtype=torch.int8, device="cuda")
+    s = C.c_float()
+    st = C.c_void_p(torch.cuda.current_stream().cuda_stream)
+    rc = L.dqt_absmean_init_noalloc(C.c_void_p(W0.data_ptr()), W0.numel(), grid,
+                                    C.c_void_p(codes.data_ptr()), C.byref(s), st)
+    assert rc == dqt.DQT_OK, rc
+    return codes, s.value
+
+
+def test_no_alloc_matches_workspace_entry_two_calls(L):
+    from paper_2412_04787_gb300 import dqt, inputs
+    cases = [(inputs.normal((512, 520), 0.02, seed=101), dqt.dqt_grid_t(-1, 1)),
+             (inputs.normal((1000, 264), 0.05, seed=202), dqt.dqt_grid_t(-128, 127))]
+    for W0, grid in cases:  # two calls in a row share the static array
+        W0 = W0.cuda()
+        c_ref, s_ref = _with_workspace(L, W0, grid)
+        c_new, s_new = _no_alloc(L, W0, grid)
+        torch.cuda.synchronize()
+        # same tolerance as the init parity tests: scale within one fp32 ulp,
+        # codes identical whenever the scales are identical
+        assert abs(s_new - s_ref) <= np.spacing(np.float32(s_ref))
+        if s_new == s_ref:
+            assert torch.equal(c_new, c_ref)
+
+
+def test_no_alloc_rejects_bad_arguments(L):
+    from paper_2412_04787_gb300 import dqt
+    g = dqt.dqt_grid_t(-1, 1)
+    s = C.c_float()
+    A = C.c_void_p(0x10000)
+    assert L.dqt_absmean_init_noalloc(None, 16, g, A, C.byref(s), None) == dqt.DQT_ERR_ARG
+    assert L.dqt_absmean_init_noalloc(A, (1 << 53) + 1, g, A, C.byref(s), None) == dqt.DQT_ERR_RANGE
