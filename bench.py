@@ -413,6 +413,84 @@ def run_reference(args):
     print(json.dumps(line))
 
 
+def run_kernel(args):
+    """One kernel kind alone, repeated: for ncu captures and bandwidth sweeps.
+    GEMMs and act_quant run at the gate projection's shape (T=8192, K=2048,
+    N=5632); sr_update streams --numel weights (fp32 gradient)."""
+    from paper_2412_04787_gb300 import build as dqt_build, dqt, inputs
+    dqt_build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    T, K, N = T_TOK, HID, INTER
+    g = dqt.grid(1.58)
+    k = args.kernel
+    if k == "sr_update":
+        n = args.numel
+        grad = torch.randn(n, device=dev) * 1e-3
+        W = torch.randint(-1, 2, (n,), dtype=torch.int8, device=dev)
+        m = torch.zeros(n, device=dev)
+        v = torch.zeros(n, device=dev)
+        hp = dqt.adamw()
+        sr = dqt.sr_stream()
+        fn = lambda: dqt.dqt_sr_update(grad, W, 62.0, m, v, hp, sr, g)  # noqa: E731
+        work, unit = 22.0 * n, "GB/s"
+    else:
+        X = inputs.normal((T, K), 1.0, seed=1, dtype=torch.bfloat16).to(dev)
+        dY = inputs.normal((T, N), 1e-2, seed=2, dtype=torch.bfloat16).to(dev)
+        W, s_w = dqt.dqt_absmean_init(inputs.normal((N, K), 0.02, seed=3).to(dev), g)
+        _, s_x, q_img, xdq = dqt.dqt_act_quant(X, want=("Xq_img", "Xdq"))
+        W_img = dqt.dqt_codes_to_bf16(W)
+        m = torch.zeros((N, K), device=dev)
+        v = torch.zeros((N, K), device=dev)
+        Y = torch.empty((T, N), dtype=torch.bfloat16, device=dev)
+        dX = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
+        hp = dqt.adamw()
+        sr = dqt.sr_stream()
+        if k == "fwd":
+            fn = lambda: dqt.dqt_bitlinear_fwd(q_img, s_x, W_img, s_w, g, Y=Y)  # noqa: E731
+        elif k == "bwd_dx":
+            fn = lambda: dqt.dqt_bitlinear_bwd_dx(dY, W_img, s_w, dX=dX)  # noqa: E731
+        elif k == "bwd_dw_update":
+            fn = lambda: dqt.dqt_bitlinear_bwd_dw_update(dY, xdq, W, s_w, m, v, hp, sr, g)  # noqa: E731
+        elif k == "act_quant":
+            fn = lambda: dqt.dqt_act_quant(X, None, s_x, q_img, xdq, want=())  # noqa: E731
+        elif k == "codes_to_bf16":
+            fn = lambda: dqt.dqt_codes_to_bf16(W, W_img)  # noqa: E731
+        else:
+            raise SystemExit("unknown kernel %s" % k)
+        if k in ("fwd", "bwd_dx", "bwd_dw_update"):
+            work, unit = 2.0 * T * K * N, "TFLOP/s"
+        elif k == "act_quant":
+            work, unit = 6.0 * T * K + 4 * T, "GB/s"
+        else:
+            work, unit = 3.0 * N * K, "GB/s"
+    for _ in range(args.warmup):
+        fn()
+    torch.cuda.synchronize()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # > L2, between launches
+    times = []
+    for _ in range(args.steps):
+        flush.zero_()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record()
+        fn()
+        b.record()
+        times.append((a, b))
+    torch.cuda.synchronize()
+    dqt.dqt_check_device_status()
+    ms = [a.elapsed_time(b) for a, b in times]
+    med = statistics.median(ms)
+    rate = work / (med / 1e3) / (1e12 if unit == "TFLOP/s" else 1e9)
+    peaks, kind = _peaks()
+    peak = peaks["bf16_tflops"] if unit == "TFLOP/s" else peaks["hbm_gbs"]
+    print(json.dumps({"kernel": k, "numel": args.numel if k == "sr_update" else None,
+                      "median_ms": round(med, 5), "min_ms": round(min(ms), 5),
+                      "rate": round(rate, 1), "unit": unit, "peak": peak,
+                      "frac": round(rate / peak, 4), "peak_kind": "burst, " + kind,
+                      "l2": "256 MiB buffer written between launches"}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -421,10 +499,16 @@ def main():
     ap.add_argument("--impl", default="dqt", choices=["dqt", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--kernel", default=None,
+                    help="time one kernel kind alone (fwd, bwd_dx, bwd_dw_update, act_quant, "
+                         "codes_to_bf16, sr_update)")
+    ap.add_argument("--numel", type=int, default=1 << 26, help="weights for --kernel sr_update")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.impl == "reference":
+    if args.kernel:
+        run_kernel(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_gpu(args)
