@@ -452,13 +452,17 @@ def run_kernel(args):
             fn = lambda: dqt.dqt_bitlinear_bwd_dx(dY, W_img, s_w, dX=dX)  # noqa: E731
         elif k == "bwd_dw_update":
             fn = lambda: dqt.dqt_bitlinear_bwd_dw_update(dY, xdq, W, s_w, m, v, hp, sr, g)  # noqa: E731
+        elif k == "bwd_dw":  # gradient only (fp32 dW written, no update)
+            dW = torch.empty((N, K), dtype=torch.float32, device=dev)
+            fn = lambda: dqt.dqt_bitlinear_bwd_dw_update(dY, xdq, None, s_w, None, None, None,  # noqa: E731
+                                                         None, g, dW_out=dW)
         elif k == "act_quant":
             fn = lambda: dqt.dqt_act_quant(X, None, s_x, q_img, xdq, want=())  # noqa: E731
         elif k == "codes_to_bf16":
             fn = lambda: dqt.dqt_codes_to_bf16(W, W_img)  # noqa: E731
         else:
             raise SystemExit("unknown kernel %s" % k)
-        if k in ("fwd", "bwd_dx", "bwd_dw_update"):
+        if k in ("fwd", "bwd_dx", "bwd_dw_update", "bwd_dw"):
             work, unit = 2.0 * T * K * N, "TFLOP/s"
         elif k == "act_quant":
             work, unit = 6.0 * T * K + 4 * T, "GB/s"

@@ -59,13 +59,19 @@ struct Params {
   UpdateConsts uc;
 };
 
-template <int BN>
+constexpr int kStageLd = 33;  // padded row pitch (floats) of the epilogue transpose buffer
+
+template <int BN, int EPI>
 struct Smem {
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int BAR_OFF = kStages * STAGE_BYTES;
+  // dW: one 32 x 33 fp32 transpose buffer per epilogue warp
+  static constexpr int XPOSE_OFF = kStages * STAGE_BYTES;
+  static constexpr int XPOSE_BYTES = (EPI == GEMM_DW) ? kEpiWarps * 32 * kStageLd * 4 : 0;
+  static constexpr int BAR_OFF = XPOSE_OFF + XPOSE_BYTES;
   static constexpr int BYTES = BAR_OFF + 256 + 1024;  // + barriers + alignment slack
+  static_assert(BYTES <= 232448, "shared memory per CTA");
 };
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
@@ -138,22 +144,34 @@ __device__ __forceinline__ void epi_dx(const Params& p, int gm, int gn0, const u
 }
 
 // dW: gradient -> AdamW -> SR -> codes, in registers, four weights (one
-// Philox block) at a time.  Streaming cache hints keep the optimiser state
-// from evicting the GEMM operands out of L2.
-__device__ __forceinline__ uint32_t epi_dw(const Params& p, int gm, int gn0,
-                                           const uint32_t (&a)[32]) {
+// Philox block) per lane at a time.  The warp's 32 x 32 gradient block (lane
+// i holds row i) is transposed through shared memory so that eight lanes
+// share each row: every optimiser-state access of the warp then covers four
+// full 128-byte row segments instead of 32 scattered ones.  Streaming cache
+// hints keep the optimiser state from evicting the GEMM operands out of L2.
+__device__ __forceinline__ uint32_t epi_dw(const Params& p, int row0, int gn0,
+                                           const uint32_t (&a)[32], float* xp, int lane) {
+#pragma unroll
+  for (int i = 0; i < 32; ++i) xp[lane * kStageLd + i] = __uint_as_float(a[i]);
+  __syncwarp();
+  const int cq = (lane & 7) * 4;  // this lane's four columns within the block
+  const int gk = gn0 + cq;
+  const bool col_ok = gk < p.N;
   uint32_t n_changed = 0;
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
-    float4 m4[4], v4[4];
+    float4 m4[4], v4[4], g4[4];
     char4 c4[4];
     size_t e[4];
     bool in[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      const int gk = gn0 + 16 * h + 4 * j;
-      in[j] = gk < p.N;
+      const int r = (lane >> 3) + 4 * (4 * h + j);
+      const int gm = row0 + r;
+      in[j] = col_ok && gm < p.M;
       e[j] = static_cast<size_t>(gm) * p.N + gk;
+      const float* src = xp + r * kStageLd + cq;
+      g4[j] = make_float4(src[0], src[1], src[2], src[3]);
       if (p.W && in[j]) {
         c4[j] = __ldcs(reinterpret_cast<const char4*>(p.W + e[j]));
         m4[j] = __ldcs(reinterpret_cast<const float4*>(p.m + e[j]));
@@ -163,18 +181,15 @@ __device__ __forceinline__ uint32_t epi_dw(const Params& p, int gm, int gn0,
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       if (!in[j]) continue;
-      const int q = 16 * h + 4 * j;
-      const float4 g4 = make_float4(__uint_as_float(a[q]), __uint_as_float(a[q + 1]),
-                                    __uint_as_float(a[q + 2]), __uint_as_float(a[q + 3]));
-      if (p.dW_out) __stcs(reinterpret_cast<float4*>(p.dW_out + e[j]), g4);
+      if (p.dW_out) __stcs(reinterpret_cast<float4*>(p.dW_out + e[j]), g4[j]);
       if (!p.W) continue;
       uint4 w = make_uint4(0, 0, 0, 0);
       if (p.uc.round_mode == 0)
         w = sr_words(e[j] >> 2, p.uc.step_lo, p.uc.tensor_id, p.uc.key0, p.uc.key1);
-      const int32_t n0c = dqt_update_elem(p.uc, g4.x, c4[j].x, m4[j].x, v4[j].x, w.x);
-      const int32_t n1c = dqt_update_elem(p.uc, g4.y, c4[j].y, m4[j].y, v4[j].y, w.y);
-      const int32_t n2c = dqt_update_elem(p.uc, g4.z, c4[j].z, m4[j].z, v4[j].z, w.z);
-      const int32_t n3c = dqt_update_elem(p.uc, g4.w, c4[j].w, m4[j].w, v4[j].w, w.w);
+      const int32_t n0c = dqt_update_elem(p.uc, g4[j].x, c4[j].x, m4[j].x, v4[j].x, w.x);
+      const int32_t n1c = dqt_update_elem(p.uc, g4[j].y, c4[j].y, m4[j].y, v4[j].y, w.y);
+      const int32_t n2c = dqt_update_elem(p.uc, g4[j].z, c4[j].z, m4[j].z, v4[j].z, w.z);
+      const int32_t n3c = dqt_update_elem(p.uc, g4[j].w, c4[j].w, m4[j].w, v4[j].w, w.w);
       n_changed += (n0c != c4[j].x) + (n1c != c4[j].y) + (n2c != c4[j].z) + (n3c != c4[j].w);
       __stcs(reinterpret_cast<char4*>(p.W + e[j]),
              make_char4(static_cast<signed char>(n0c), static_cast<signed char>(n1c),
@@ -183,6 +198,7 @@ __device__ __forceinline__ uint32_t epi_dw(const Params& p, int gm, int gn0,
       __stcs(reinterpret_cast<float4*>(p.v + e[j]), v4[j]);
     }
   }
+  __syncwarp();  // the transpose buffer is rewritten for the next block
   return n_changed;
 }
 
@@ -190,7 +206,7 @@ template <int BN, bool A_MN, bool B_MN, int EPI, bool DRAIN>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const Params p) {
-  using S = Smem<BN>;
+  using S = Smem<BN, EPI>;
   constexpr uint32_t IDESC = idesc_bf16(BM, BN, A_MN, B_MN);
   constexpr uint32_t TMEM_COLS = 512;  // 2 x 256 accumulators, or 3 x 128 with DRAIN
   static_assert(DRAIN ? 3 * BN <= 512 : 2 * BN <= 512, "tensor memory layout");
@@ -330,6 +346,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int half = (warp - 2) >> 2;        // which half of the tile's columns
     const int row = quad * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    float* xp = reinterpret_cast<float*>(smem + S::XPOSE_OFF) + (warp - 2) * 32 * kStageLd;
     uint32_t n_changed = 0;
     int u = 0;
     bool ok = true;
@@ -363,10 +380,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             continue;
           }
           const int gn0 = nbase + cc * 32;
-          if (!row_ok || gn0 >= p.N) continue;
+          if (gn0 >= p.N) continue;  // warp-uniform
+          if (EPI == GEMM_DW) {
+            n_changed += epi_dw(p, gm - lane, gn0, a, xp, lane);
+            continue;
+          }
+          if (!row_ok) continue;
           if (EPI == GEMM_FWD) epi_fwd(p, gm, gn0, a_t, a, r, DRAIN && c > 0);
-          else if (EPI == GEMM_DX) epi_dx(p, gm, gn0, a);
-          else n_changed += epi_dw(p, gm, gn0, a);
+          else epi_dx(p, gm, gn0, a);
         }
         if (DRAIN && !last) tmem_st_wait();
         tc_fence_before();
@@ -429,7 +450,7 @@ bool make_map(CUtensorMap* map, const void* ptr, uint64_t inner, uint64_t outer,
 template <int BN, bool A_MN, bool B_MN, int EPI, bool DRAIN>
 int launch_tiles(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream) {
   auto kern = gemm_kernel<BN, A_MN, B_MN, EPI, DRAIN>;
-  const int smem = Smem<BN>::BYTES;
+  const int smem = Smem<BN, EPI>::BYTES;
   static bool attr_set = false;  // per template instance
   if (!attr_set) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
