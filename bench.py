@@ -75,7 +75,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.Q,
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "20"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
@@ -144,42 +144,97 @@ class MLPStep:
         self.sr = {name: dqt.sr_stream(seed=seed, tensor_id=i) for i, (name, _, _) in enumerate(PROJ)}
         self.step_no = 0
         self.launches_per_step = 2 + 3 + 3 + 3 + 3
+        self.streams = [torch.cuda.Stream(device=dev) for _ in range(4)]
 
-    def run(self, timers=None):
-        """Enqueue one step on the current stream.  `timers` maps a kernel kind
-        to a list that receives (start, end) CUDA events around its launches."""
+    def run(self, timers=None, serial=False):
+        """Enqueue one step.  The launches follow the dependency graph of a
+        LLaMA MLP (gate and up read the same quantised X; the down projection
+        reads the SwiGLU output H, here a synthetic stand-in that still waits
+        for both forwards; each projection's dX and dW are independent; the
+        gate/up backward waits for the down projection's dX) on four streams
+        joined at the end, so that the persistent kernels fill each other's
+        last-wave idle SMs.  `timers` maps a kernel kind to a list that
+        receives (start, end) CUDA events recorded on the kernel's stream."""
         dqt = self.dqt
         self.step_no += 1
         hp = dqt.adamw(lr=1e-3, step=self.step_no)
+        main = torch.cuda.current_stream()
+        # serial: the same launches, in the same order, all on the current stream
+        s = [main] * 4 if serial else self.streams
 
-        def timed(kind, fn):
-            if timers is not None and kind in timers:
-                a = torch.cuda.Event(enable_timing=True)
-                b = torch.cuda.Event(enable_timing=True)
-                a.record()
-                fn()
-                b.record()
-                timers[kind].append((a, b))
-            else:
-                fn()
+        def timed(kind, stream, fn):
+            with torch.cuda.stream(stream):
+                if timers is not None and kind in timers:
+                    a = torch.cuda.Event(enable_timing=True)
+                    b = torch.cuda.Event(enable_timing=True)
+                    a.record(stream)
+                    fn()
+                    b.record(stream)
+                    timers[kind].append((a, b))
+                else:
+                    fn()
 
-        for src in ("X", "H"):
+        def after(stream, *others):
+            for o in others:
+                if o is stream:
+                    continue
+                e = torch.cuda.Event()
+                e.record(o)
+                stream.wait_event(e)
+
+        def aq(src, stream):
             s_x, q_img, xdq = self.aq[src]
-            timed("act_quant", lambda: dqt.dqt_act_quant(self.d[src], None, s_x, q_img, xdq, want=()))
-        for name, K, N in PROJ:
-            timed("codes_to_bf16", lambda: dqt.dqt_codes_to_bf16(self.W[name], self.W_img[name]))
-        for name, K, N in PROJ:
-            s_x, q_img, _ = self.aq["X" if name != "down" else "H"]
-            timed("fwd", lambda: dqt.dqt_bitlinear_fwd(q_img, s_x, self.W_img[name], self.s_w[name],
-                                                      self.grid, Y=self.Y[name]))
-        for i, (name, K, N) in enumerate(PROJ):
-            dY = self.d["dY_" + name]
-            _, _, xdq = self.aq["X" if name != "down" else "H"]
-            timed("bwd_dx", lambda: dqt.dqt_bitlinear_bwd_dx(dY, self.W_img[name], self.s_w[name],
-                                                            dX=self.dX[name]))
-            timed("bwd_dw_update", lambda: dqt.dqt_bitlinear_bwd_dw_update(
-                dY, xdq, self.W[name], self.s_w[name], self.m[name], self.v[name], hp,
-                self.sr[name], self.grid, changed_out=self.changed[i:i + 1]))
+            timed("act_quant", stream,
+                  lambda: dqt.dqt_act_quant(self.d[src], None, s_x, q_img, xdq, want=()))
+
+        def codes(name, stream):
+            timed("codes_to_bf16", stream,
+                  lambda: dqt.dqt_codes_to_bf16(self.W[name], self.W_img[name]))
+
+        def fwd(name, stream):
+            s_x, q_img, _ = self.aq["H" if name == "down" else "X"]
+            timed("fwd", stream, lambda: dqt.dqt_bitlinear_fwd(
+                q_img, s_x, self.W_img[name], self.s_w[name], self.grid, Y=self.Y[name]))
+
+        def dx(name, stream):
+            timed("bwd_dx", stream, lambda: dqt.dqt_bitlinear_bwd_dx(
+                self.d["dY_" + name], self.W_img[name], self.s_w[name], dX=self.dX[name]))
+
+        def dw(i, name, stream):
+            xdq = self.aq["H" if name == "down" else "X"][2]
+            timed("bwd_dw_update", stream, lambda: dqt.dqt_bitlinear_bwd_dw_update(
+                self.d["dY_" + name], xdq, self.W[name], self.s_w[name], self.m[name],
+                self.v[name], hp, self.sr[name], self.grid, changed_out=self.changed[i:i + 1]))
+
+        for st in s:
+            after(st, main)
+        # forward
+        aq("X", s[0])
+        codes("gate", s[0])
+        after(s[1], s[0])
+        codes("up", s[1])
+        codes("down", s[2])
+        fwd("gate", s[0])
+        fwd("up", s[1])
+        after(s[2], s[0], s[1])
+        aq("H", s[2])
+        fwd("down", s[2])
+        # backward: down projection (dX and dW independent)
+        after(s[3], s[2])
+        dx("down", s[2])
+        dw(2, "down", s[3])
+        # backward: gate and up, after the down projection's dX
+        dx_down = torch.cuda.Event()
+        dx_down.record(s[2])
+        for st in (s[0], s[1], s[3]):
+            if st is not s[2]:
+                st.wait_event(dx_down)
+        dx("gate", s[0])
+        dw(0, "gate", s[1])
+        dx("up", s[2])
+        dw(1, "up", s[3])
+        for st in s:
+            after(main, st)
 
     # algorithmic work per launch, per kernel kind
     def work(self):
@@ -197,6 +252,21 @@ class MLPStep:
 
 def _elapsed(pairs):
     return [a.elapsed_time(b) for a, b in pairs]
+
+
+def max_over_ranks(x, device):
+    """Max of a per-rank float over all ranks (identity when not distributed)."""
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate_tokens_per_s(world_size, tokens_per_step, steps, max_ms):
+    """Whole-job throughput: every rank processed its own tokens in max_ms."""
+    return world_size * tokens_per_step * steps / (max_ms / 1e3)
 
 
 def run_gpu(args):
@@ -224,26 +294,34 @@ def run_gpu(args):
     dqt.dqt_check_device_status()
 
     # ---- device-timed region: inputs resident in HBM ----
-    kinds = ["act_quant", "codes_to_bf16", "fwd", "bwd_dx", "bwd_dw_update"]
-    timers = {k: [] for k in kinds}
     barrier()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     with ClockSampler(dev.index) as clk:
         t0.record(stream)
         for _ in range(args.steps):
-            st.run(timers)
+            st.run()
         t1.record(stream)
         barrier()
     dqt.dqt_check_device_status()
-    ms = t0.elapsed_time(t1)
-    if ws > 1:
-        import torch.distributed as dist
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(t0.elapsed_time(t1), dev)
     ms_step = ms / args.steps
-    value = ws * T_TOK * args.steps / (ms / 1e3)
+    value = aggregate_tokens_per_s(ws, T_TOK, args.steps, ms)
+
+    # ---- per-kernel timing: a second timed region of K steps with the same
+    # launches serialised on one stream, CUDA events around every launch ----
+    kinds = ["act_quant", "codes_to_bf16", "fwd", "bwd_dx", "bwd_dw_update"]
+    timers = {k: [] for k in kinds}
+    barrier()
+    s0 = torch.cuda.Event(enable_timing=True)
+    s1 = torch.cuda.Event(enable_timing=True)
+    s0.record(stream)
+    for _ in range(args.steps):
+        st.run(timers, serial=True)
+    s1.record(stream)
+    barrier()
+    dqt.dqt_check_device_status()
+    serial_ms_step = s0.elapsed_time(s1) / args.steps
 
     # per-kernel live timings
     flops, byts = st.work()
@@ -263,6 +341,8 @@ def run_gpu(args):
     roofline = {"bound": "tensor", "kernel": dom, "achieved": round(achieved, 1),
                 "peak": peak, "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
                 "peak_kind": "bf16 dense sustained, %s" % pk_kind,
+                "timing": "mean CUDA-event duration of its launches over a second timed region "
+                          "of the same K steps run serially on one stream (%.4f ms/step)" % serial_ms_step,
                 "traffic": None,
                 "algorithmic_per_launch": "2*T*K*N FLOP (T=8192; K,N = 2048,5632 / 5632,2048)"}
     kern = {}
@@ -294,14 +374,9 @@ def run_gpu(args):
         res_host.copy_(st.changed, non_blocking=True)
     e1.record(stream)
     barrier()
-    e_ms = e0.elapsed_time(e1)
-    if ws > 1:
-        import torch.distributed as dist
-        tt = torch.tensor([e_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e_ms = float(tt.item())
+    e_ms = max_over_ranks(e0.elapsed_time(e1), dev)
     dqt.dqt_check_device_status()
-    e2e = {"value": round(ws * T_TOK * e_steps / (e_ms / 1e3), 1), "unit": "tokens/s",
+    e2e = {"value": round(aggregate_tokens_per_s(ws, T_TOK, e_steps, e_ms), 1), "unit": "tokens/s",
            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": e_steps}
 
     cpu = None
@@ -498,8 +573,8 @@ def run_kernel(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="dqt", choices=["dqt", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)

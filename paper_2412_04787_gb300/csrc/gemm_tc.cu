@@ -284,12 +284,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      if (!ok) {
-        record_timeout(p.status);
-        // Let the (at most kStages) copies still in flight land before exit.
-        for (int i = (it > kStages ? it - kStages : 0); i < it; ++i)
-          mbar_wait(&full[i % kStages], (i / kStages) & 1u, kDrainNs);
-      }
+      if (!ok) record_timeout(p.status);
+      // Whatever any role did, the (at most kStages) copies still in flight
+      // must land before the CTA exits; in a normal run these are consumed
+      // already and each wait returns at once.
+      for (int i = (it > kStages ? it - kStages : 0); i < it; ++i)
+        mbar_wait(&full[i % kStages], (i / kStages) & 1u, kDrainNs);
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -334,11 +334,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      if (!ok) {
-        record_timeout(p.status);
-        umma_commit(drain_bar);  // every MMA issued so far has finished
-        mbar_wait(drain_bar, 0, kDrainNs);
-      }
+      if (!ok) record_timeout(p.status);
+      // Every MMA issued so far must finish before tensor memory is freed,
+      // also when another role gave up first.
+      umma_commit(drain_bar);
+      mbar_wait(drain_bar, 0, kDrainNs);
     }
   } else {
     // ---------------- epilogue (warps 2..9) ----------------

@@ -88,6 +88,90 @@ __global__ void __launch_bounds__(kAqWarps * 32)
   }
 }
 
+// Single-pass variant for rows of up to NV * 256 elements: each lane keeps
+// its NV 16-byte vectors of the row in registers between the absmax and the
+// quantisation.  The dequantised image needs bf16(q / s_x) for q in
+// [-128, 127] only, so each warp first fills a 256-entry table of those
+// correctly rounded quotients (8 divisions per lane) and then looks them up:
+// bit-identical to dividing per element.
+template <int NV>
+__global__ void __launch_bounds__(kAqWarps * 32)
+    act_quant_rows_kernel(const uint16_t* __restrict__ X, int T, int K, int8_t* __restrict__ Xq,
+                          float* __restrict__ s_x, uint16_t* __restrict__ Xq_img,
+                          uint16_t* __restrict__ Xdq) {
+  __shared__ uint16_t table[kAqWarps][256];
+  const int wid = threadIdx.x >> 5;
+  const int row = blockIdx.x * kAqWarps + wid;
+  const int lane = threadIdx.x & 31;
+  if (row >= T) return;
+  const int nv = K >> 3;
+  const uint4* xr = reinterpret_cast<const uint4*>(X + static_cast<size_t>(row) * K);
+  uint4 u[NV];
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const int vi = lane + 32 * i;
+    u[i] = vi < nv ? __ldcs(xr + vi) : make_uint4(0, 0, 0, 0);
+  }
+  float amax = 0.0f;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const uint32_t w[4] = {u[i].x, u[i].y, u[i].z, u[i].w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      amax = fmaxf(amax, fabsf(bf16_bits_to_f32(w[j] & 0xFFFFu)));
+      amax = fmaxf(amax, fabsf(bf16_bits_to_f32(w[j] >> 16)));
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+  const float s = __fdiv_rn(127.0f, fmaxf(amax, 1e-5f));
+  if (lane == 0) s_x[row] = s;
+  if (Xdq) {
+#pragma unroll
+    for (int j = lane; j < 256; j += 32)
+      table[wid][j] = f32_to_bf16_bits(__fdiv_rn(static_cast<float>(j - 128), s));
+    __syncwarp();
+  }
+  const size_t rbase = static_cast<size_t>(row) * K;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const int vi = lane + 32 * i;
+    if (vi >= nv) break;
+    const uint32_t w[4] = {u[i].x, u[i].y, u[i].z, u[i].w};
+    int32_t q[8];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float lo = bf16_bits_to_f32(w[j] & 0xFFFFu);
+      const float hi = bf16_bits_to_f32(w[j] >> 16);
+      q[2 * j] = static_cast<int32_t>(fminf(fmaxf(rintf(__fmul_rn(lo, s)), -128.0f), 127.0f));
+      q[2 * j + 1] = static_cast<int32_t>(fminf(fmaxf(rintf(__fmul_rn(hi, s)), -128.0f), 127.0f));
+    }
+    const size_t e = rbase + static_cast<size_t>(vi) * 8;
+    if (Xq) {
+      uint2 pk;
+      pk.x = (q[0] & 0xFF) | ((q[1] & 0xFF) << 8) | ((q[2] & 0xFF) << 16) | ((q[3] & 0xFF) << 24);
+      pk.y = (q[4] & 0xFF) | ((q[5] & 0xFF) << 8) | ((q[6] & 0xFF) << 16) | ((q[7] & 0xFF) << 24);
+      __stcs(reinterpret_cast<uint2*>(Xq + e), pk);
+    }
+    if (Xq_img) {
+      uint32_t h[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) h[j] = f32_to_bf16_bits(static_cast<float>(q[j]));
+      __stcs(reinterpret_cast<uint4*>(Xq_img + e),
+             make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
+                        h[6] | (h[7] << 16)));
+    }
+    if (Xdq) {
+      uint32_t h[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) h[j] = table[wid][q[j] + 128];
+      __stcs(reinterpret_cast<uint4*>(Xdq + e),
+             make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
+                        h[6] | (h[7] << 16)));
+    }
+  }
+}
+
 // 16 codes per thread per step: one 16-byte load, two 16-byte stores.
 __global__ void codes_to_bf16_kernel(const int8_t* __restrict__ W, int64_t numel,
                                      uint16_t* __restrict__ img) {
@@ -178,8 +262,17 @@ int grid_for(int64_t work, int threads) {
 int launch_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
                      uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream) {
   const int blocks = static_cast<int>((T + kAqWarps - 1) / kAqWarps);
-  act_quant_kernel<<<blocks, kAqWarps * 32, 0, stream>>>(X, static_cast<int>(T),
-                                                         static_cast<int>(K), Xq, s_x, Xq_img, Xdq);
+  const int t = static_cast<int>(T), k = static_cast<int>(K);
+  const int nvl = static_cast<int>((K / 8 + 31) / 32);  // 16-byte vectors per lane
+#define DQT_AQ(NV) act_quant_rows_kernel<NV><<<blocks, kAqWarps * 32, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq)
+  if (nvl <= 2) DQT_AQ(2);
+  else if (nvl <= 4) DQT_AQ(4);
+  else if (nvl <= 8) DQT_AQ(8);
+  else if (nvl <= 12) DQT_AQ(12);
+  else if (nvl <= 16) DQT_AQ(16);
+  else if (nvl <= 24) DQT_AQ(24);
+  else act_quant_kernel<<<blocks, kAqWarps * 32, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq);
+#undef DQT_AQ
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
