@@ -157,46 +157,45 @@ __device__ __forceinline__ uint32_t epi_dw(const Params& p, int row0, int gn0,
   const int cq = (lane & 7) * 4;  // this lane's four columns within the block
   const int gk = gn0 + cq;
   const bool col_ok = gk < p.N;
+  constexpr int R = 8;  // rows per lane: lane >> 3, +4, +8, ..., +28
+  float4 m4[R], v4[R];
+  char4 c4[R];
+  bool in[R];
+  // all of this lane's optimiser-state loads first: one memory round trip
+#pragma unroll
+  for (int j = 0; j < R; ++j) {
+    const int gm = row0 + (lane >> 3) + 4 * j;
+    in[j] = col_ok && gm < p.M;
+    if (p.W && in[j]) {
+      const size_t e = static_cast<size_t>(gm) * p.N + gk;
+      c4[j] = __ldcs(reinterpret_cast<const char4*>(p.W + e));
+      m4[j] = __ldcs(reinterpret_cast<const float4*>(p.m + e));
+      v4[j] = __ldcs(reinterpret_cast<const float4*>(p.v + e));
+    }
+  }
   uint32_t n_changed = 0;
 #pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    float4 m4[4], v4[4], g4[4];
-    char4 c4[4];
-    size_t e[4];
-    bool in[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int r = (lane >> 3) + 4 * (4 * h + j);
-      const int gm = row0 + r;
-      in[j] = col_ok && gm < p.M;
-      e[j] = static_cast<size_t>(gm) * p.N + gk;
-      const float* src = xp + r * kStageLd + cq;
-      g4[j] = make_float4(src[0], src[1], src[2], src[3]);
-      if (p.W && in[j]) {
-        c4[j] = __ldcs(reinterpret_cast<const char4*>(p.W + e[j]));
-        m4[j] = __ldcs(reinterpret_cast<const float4*>(p.m + e[j]));
-        v4[j] = __ldcs(reinterpret_cast<const float4*>(p.v + e[j]));
-      }
-    }
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      if (!in[j]) continue;
-      if (p.dW_out) __stcs(reinterpret_cast<float4*>(p.dW_out + e[j]), g4[j]);
-      if (!p.W) continue;
-      uint4 w = make_uint4(0, 0, 0, 0);
-      if (p.uc.round_mode == 0)
-        w = sr_words(e[j] >> 2, p.uc.step_lo, p.uc.tensor_id, p.uc.key0, p.uc.key1);
-      const int32_t n0c = dqt_update_elem(p.uc, g4[j].x, c4[j].x, m4[j].x, v4[j].x, w.x);
-      const int32_t n1c = dqt_update_elem(p.uc, g4[j].y, c4[j].y, m4[j].y, v4[j].y, w.y);
-      const int32_t n2c = dqt_update_elem(p.uc, g4[j].z, c4[j].z, m4[j].z, v4[j].z, w.z);
-      const int32_t n3c = dqt_update_elem(p.uc, g4[j].w, c4[j].w, m4[j].w, v4[j].w, w.w);
-      n_changed += (n0c != c4[j].x) + (n1c != c4[j].y) + (n2c != c4[j].z) + (n3c != c4[j].w);
-      __stcs(reinterpret_cast<char4*>(p.W + e[j]),
-             make_char4(static_cast<signed char>(n0c), static_cast<signed char>(n1c),
-                        static_cast<signed char>(n2c), static_cast<signed char>(n3c)));
-      __stcs(reinterpret_cast<float4*>(p.m + e[j]), m4[j]);
-      __stcs(reinterpret_cast<float4*>(p.v + e[j]), v4[j]);
-    }
+  for (int j = 0; j < R; ++j) {
+    if (!in[j]) continue;
+    const int r = (lane >> 3) + 4 * j;
+    const size_t e = static_cast<size_t>(row0 + r) * p.N + gk;
+    const float* src = xp + r * kStageLd + cq;
+    const float4 g4 = make_float4(src[0], src[1], src[2], src[3]);
+    if (p.dW_out) __stcs(reinterpret_cast<float4*>(p.dW_out + e), g4);
+    if (!p.W) continue;
+    uint4 w = make_uint4(0, 0, 0, 0);
+    if (p.uc.round_mode == 0)
+      w = sr_words(e >> 2, p.uc.step_lo, p.uc.tensor_id, p.uc.key0, p.uc.key1);
+    const int32_t n0c = dqt_update_elem(p.uc, g4.x, c4[j].x, m4[j].x, v4[j].x, w.x);
+    const int32_t n1c = dqt_update_elem(p.uc, g4.y, c4[j].y, m4[j].y, v4[j].y, w.y);
+    const int32_t n2c = dqt_update_elem(p.uc, g4.z, c4[j].z, m4[j].z, v4[j].z, w.z);
+    const int32_t n3c = dqt_update_elem(p.uc, g4.w, c4[j].w, m4[j].w, v4[j].w, w.w);
+    n_changed += (n0c != c4[j].x) + (n1c != c4[j].y) + (n2c != c4[j].z) + (n3c != c4[j].w);
+    __stcs(reinterpret_cast<char4*>(p.W + e),
+           make_char4(static_cast<signed char>(n0c), static_cast<signed char>(n1c),
+                      static_cast<signed char>(n2c), static_cast<signed char>(n3c)));
+    __stcs(reinterpret_cast<float4*>(p.m + e), m4[j]);
+    __stcs(reinterpret_cast<float4*>(p.v + e), v4[j]);
   }
   __syncwarp();  // the transpose buffer is rewritten for the next block
   return n_changed;
