@@ -104,6 +104,16 @@ int dqt_check_device_status(void* stream);
  * library's kernels (default 2e9).  Applies to launches made after the call. */
 int dqt_set_wait_limit_ns(uint64_t ns);
 
+/* GEMM tiling for launches made after the call (host setting, all devices):
+ * 0 (default) = 2-SM tiles: a cluster of two CTAs on one TPC computes a
+ *     256 x 256 tile with tcgen05.mma.cta_group::2;
+ * 1 = 1-SM 128 x 256 tiles.
+ * Forward GEMMs whose exact integer accumulation needs fp32 chunks drained
+ * into int32 (codes wider than 4 bits with K > 1024) always use 1-SM tiles.
+ * Results are identical either way (the same per-element arithmetic);
+ * DQT_ERR_ARG for any other mode. */
+int dqt_set_gemm_tiles(int mode);
+
 /* Eq. 2-4, initialisation (not on the training hot path).
  *   W0      fp32 [numel] dense initial weight (device)
  *   codes   int8 [numel] out: Clip[Round(W0 * s_w), qmin, qmax], Round half-to-even

@@ -16,11 +16,13 @@ __device__ unsigned int g_status_word;
 
 namespace {
 std::atomic<uint64_t> g_wait_ns{2000000000ull};
+std::atomic<int> g_gemm_mode{0};
 constexpr int kMaxDevices = 64;
 unsigned int* g_status_ptr[kMaxDevices] = {nullptr};
 }  // namespace
 
 uint64_t wait_limit_ns() { return g_wait_ns.load(); }
+int gemm_mode() { return g_gemm_mode.load(); }
 
 unsigned int* status_word() {
   int dev = 0;
@@ -110,6 +112,12 @@ int dqt_grid_for_bits(float bits, dqt_grid_t* out) {
 
 int dqt_set_wait_limit_ns(uint64_t ns) {
   dqt::g_wait_ns.store(ns);
+  return DQT_OK;
+}
+
+int dqt_set_gemm_tiles(int mode) {
+  if (mode != 0 && mode != 1) return DQT_ERR_ARG;
+  dqt::g_gemm_mode.store(mode);
   return DQT_OK;
 }
 

@@ -14,6 +14,9 @@ uint64_t wait_limit_ns();
 // Device address of the current device's status word (NULL on failure).
 unsigned int* status_word();
 
+// GEMM kernel selection: 0 = 2-SM pair tiles where possible, 1 = 1-SM tiles.
+int gemm_mode();
+
 enum GemmKind { GEMM_FWD = 0, GEMM_DX = 1, GEMM_DW = 2 };
 
 struct GemmLaunch {
@@ -27,6 +30,7 @@ struct GemmLaunch {
   const void* A;
   const void* B;
   int chunk_k;  // FWD: reduction elements per exact fp32 chunk (multiple of 64)
+  bool pair;    // use the 2-SM (cta_group::2) kernel (not with drained chunks)
   // Epilogue operands.
   const float* s_x;  // FWD
   float scale;       // FWD: s_w; DX: 1/s_w

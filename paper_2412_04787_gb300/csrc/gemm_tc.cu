@@ -411,6 +411,230 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ---------------------------------------------------------------------------
+// 2-SM variant (cta_group::2): a cluster of two CTAs on the SM pair of a TPC
+// computes a 256 x 256 output tile.  CTA r stages rows [128 r, 128 r + 128)
+// of A and rows/columns [128 r, 128 r + 128) of B's 256-wide tile: 32 KB per
+// stage instead of 48 KB, so the ring is 7 stages deep (6 for dW, which also
+// holds the transpose buffers) and each SM pulls a third fewer operand bytes
+// through L2 per FLOP.  Both CTAs' copies complete on the leader's `full`
+// barrier; the leader issues the 256 x 256 x 16 MMAs and multicasts its
+// commits to both CTAs' `empty` and `acc_full` barriers; each CTA's epilogue
+// reads its own 128 rows from its own tensor memory and releases the
+// accumulator on the leader's `acc_empty` barrier.
+// ---------------------------------------------------------------------------
+template <int EPI>
+struct SmemPair {
+  static constexpr int A_BYTES = 128 * BK * 2;
+  static constexpr int B_BYTES = 128 * BK * 2;  // this CTA's half of the B tile
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int STAGES = (EPI == GEMM_DW) ? 6 : 7;
+  static constexpr int XPOSE_OFF = STAGES * STAGE_BYTES;
+  static constexpr int XPOSE_BYTES = (EPI == GEMM_DW) ? kEpiWarps * 32 * kStageLd * 4 : 0;
+  static constexpr int BAR_OFF = XPOSE_OFF + XPOSE_BYTES;
+  static constexpr int BYTES = BAR_OFF + 256 + 1024;
+  static_assert(BYTES <= 232448, "shared memory per CTA");
+  static_assert((2 * STAGES + 5) * 8 + 4 <= 256, "barrier area");
+};
+
+template <bool A_MN, bool B_MN, int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA,
+                     const __grid_constant__ CUtensorMap tmB, const Params p) {
+  using S = SmemPair<EPI>;
+  constexpr int ST = S::STAGES;
+  constexpr int BN = 256;    // pair tile width; each CTA holds all 256 columns of its rows
+  constexpr int HALF = 128;  // columns per epilogue warp
+  constexpr uint32_t IDESC = idesc_bf16(256, 256, A_MN, B_MN);
+  constexpr uint32_t TMEM_COLS = 512;
+  constexpr uint32_t MN_CHUNK_BYTES = 64 * BK * 2;
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + ST * S::A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::BAR_OFF);  // used on the leader
+  uint64_t* empty = full + ST;
+  uint64_t* acc_full = empty + ST;     // [2]
+  uint64_t* acc_empty = acc_full + 2;  // [2], used on the leader
+  uint64_t* drain_bar = acc_empty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int cid = static_cast<int>(cluster_id_x());
+  const int ncl = static_cast<int>(num_clusters_x());
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < ST; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 2 * kEpiWarps);
+    }
+    mbar_init(drain_bar, 1);
+    fence_mbarrier_init();
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) tmem_alloc_pair(tmem_slot, TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // both CTAs' barriers initialised, both allocations done
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t full_lead = mapa_shared(smem_u32(full), 0);
+  const uint32_t acc_empty_lead = mapa_shared(smem_u32(acc_empty), 0);
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer (both CTAs) ----------------
+      int it = 0;
+      bool ok = true;
+      for (int t = cid; t < p.num_tiles && ok; t += ncl) {
+        const int m0 = (t / p.num_n) * 256 + static_cast<int>(rank) * 128;
+        const int n0 = (t % p.num_n) * BN + static_cast<int>(rank) * 128;
+        for (int kb = 0; kb < p.num_kb; ++kb, ++it) {
+          const int s = it % ST;
+          const uint32_t ph = (it / ST) & 1u;
+          if (it >= ST && !mbar_wait_cl(&empty[s], ph ^ 1u, p.wait_ns)) {
+            ok = false;
+            break;
+          }
+          if (leader) mbar_arrive_expect_tx(&full[s], 2 * S::STAGE_BYTES);
+          const uint32_t bar = full_lead + 8u * s;
+          uint8_t* a = sA + s * S::A_BYTES;
+          uint8_t* b = sB + s * S::B_BYTES;
+          const int k0 = kb * BK;
+          if (!A_MN) {
+            tma_load_2d_pair(&tmA, bar, a, k0, m0);
+          } else {
+#pragma unroll
+            for (int j = 0; j < 2; ++j)
+              tma_load_2d_pair(&tmA, bar, a + j * MN_CHUNK_BYTES, m0 + 64 * j, k0);
+          }
+          if (!B_MN) {
+            tma_load_2d_pair(&tmB, bar, b, k0, n0);
+          } else {
+#pragma unroll
+            for (int j = 0; j < 2; ++j)
+              tma_load_2d_pair(&tmB, bar, b + j * MN_CHUNK_BYTES, n0 + 64 * j, k0);
+          }
+        }
+      }
+      if (!ok) record_timeout(p.status);
+      // The leader sees every stage's completion (both CTAs' copies land on
+      // its barriers): let the last stages land before the pair exits.
+      if (leader)
+        for (int i = (it > ST ? it - ST : 0); i < it; ++i)
+          mbar_wait_cl(&full[i % ST], (i / ST) & 1u, kDrainNs);
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {
+      // ---------------- MMA issuer (leader CTA) ----------------
+      int it = 0;
+      int u = 0;
+      bool ok = true;
+      for (int t = cid; t < p.num_tiles && ok; t += ncl) {
+        for (int kb = 0; kb < p.num_kb; ++kb, ++it) {
+          const int b = u & 1;
+          if (kb == 0 && u >= 2) {
+            if (!mbar_wait_cl(&acc_empty[b], ((u >> 1) - 1) & 1u, p.wait_ns)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+          }
+          const int s = it % ST;
+          const uint32_t ph = (it / ST) & 1u;
+          if (!mbar_wait_cl(&full[s], ph, p.wait_ns)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_base = smem_u32(sA + s * S::A_BYTES);
+          const uint32_t b_base = smem_u32(sB + s * S::B_BYTES);
+          const uint32_t d = tmem + static_cast<uint32_t>(b * BN);
+#pragma unroll
+          for (int ks = 0; ks < BK / 16; ++ks) {
+            const uint64_t ad = A_MN ? sdesc_sw128(a_base + ks * 2048, MN_CHUNK_BYTES, 1024)
+                                     : sdesc_sw128(a_base + ks * 32, 16, 1024);
+            const uint64_t bd = B_MN ? sdesc_sw128(b_base + ks * 2048, MN_CHUNK_BYTES, 1024)
+                                     : sdesc_sw128(b_base + ks * 32, 16, 1024);
+            umma_bf16_pair(d, ad, bd, IDESC, (kb > 0 || ks > 0) ? 1u : 0u);
+          }
+          umma_commit_pair_mc(&empty[s], 0x3);
+          if (kb == p.num_kb - 1) {
+            umma_commit_pair_mc(&acc_full[b], 0x3);
+            ++u;
+          }
+        }
+      }
+      if (!ok) record_timeout(p.status);
+      umma_commit_pair(drain_bar);
+      mbar_wait_cl(drain_bar, 0, kDrainNs);
+    }
+  } else {
+    // ---------------- epilogue (warps 2..9, both CTAs) ----------------
+    const int quad = warp & 3;
+    const int half = (warp - 2) >> 2;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    float* xp = reinterpret_cast<float*>(smem + S::XPOSE_OFF) + (warp - 2) * 32 * kStageLd;
+    uint32_t n_changed = 0;
+    int u = 0;
+    bool ok = true;
+    for (int t = cid; t < p.num_tiles && ok; t += ncl, ++u) {
+      const int gm = (t / p.num_n) * 256 + static_cast<int>(rank) * 128 + row;
+      const int nbase = (t % p.num_n) * BN + half * HALF;
+      const bool row_ok = gm < p.M;
+      float a_t = 0.0f;
+      if (EPI == GEMM_FWD && row_ok) a_t = __fdiv_rn(1.0f, __fmul_rn(p.s_x[gm], p.scale));
+      const int b = u & 1;
+      ok = __all_sync(0xffffffffu, mbar_wait_cl(&acc_full[b], (u >> 1) & 1u, p.wait_ns));
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(b * BN + half * HALF);
+#pragma unroll 1
+      for (int cc = 0; cc < HALF / 32; ++cc) {
+        uint32_t a[32], r[32];
+        tmem_ld_32x32b_x32(t_acc + cc * 32, a);
+        tmem_ld_wait();
+        const int gn0 = nbase + cc * 32;
+        if (gn0 >= p.N) continue;  // warp-uniform
+        if (EPI == GEMM_DW) {
+          n_changed += epi_dw(p, gm - lane, gn0, a, xp, lane);
+          continue;
+        }
+        if (!row_ok) continue;
+        if (EPI == GEMM_FWD) epi_fwd(p, gm, gn0, a_t, a, r, false);
+        else epi_dx(p, gm, gn0, a);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(acc_empty_lead + 8u * b);
+    }
+    if (!ok && lane == 0) record_timeout(p.status);
+    if (EPI == GEMM_DW && p.changed) {
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) n_changed += __shfl_xor_sync(0xffffffffu, n_changed, off);
+      if (lane == 0 && n_changed) atomicAdd(p.changed, static_cast<unsigned long long>(n_changed));
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // no remote arrive, copy or MMA of either CTA is pending
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Host side: tensor maps and launch.
 // ---------------------------------------------------------------------------
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -467,6 +691,42 @@ int launch_tiles(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStr
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
+template <bool A_MN, bool B_MN, int EPI>
+int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream) {
+  auto kern = gemm_pair_kernel<A_MN, B_MN, EPI>;
+  const int smem = SmemPair<EPI>::BYTES;
+  static int max_clusters = 0;  // per template instance
+  p.num_n = (p.N + 255) / 256;
+  p.num_tiles = ((p.M + 255) / 256) * p.num_n;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (max_clusters == 0) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+        cudaSuccess)
+      return 3;
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    cfg.gridDim = dim3(sms, 1, 1);
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n < 1) return 3;
+    max_clusters = n;
+  }
+  const int clusters = p.num_tiles < max_clusters ? p.num_tiles : max_clusters;
+  cfg.gridDim = dim3(2 * clusters, 1, 1);
+  if (cudaLaunchKernelEx(&cfg, kern, ta, tb, p) != cudaSuccess) return 3;
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
 }  // namespace
 
 int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
@@ -482,6 +742,9 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
     if (ck < p.num_kb) p.chunk_kb = ck;
   }
   const bool drain = p.chunk_kb < p.num_kb;
+  GemmLaunch gl = g;
+  gl.pair = !drain && gemm_mode() == 0;
+  const GemmLaunch& g2 = gl;
   p.wait_ns = wait_limit_ns();
   p.status = status_word();
   if (!p.status) return 3;
@@ -504,15 +767,18 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
         if (!make_map(&tb, g.B, g.Kred, g.N, BK, 128)) return 3;
         return launch_tiles<128, false, false, GEMM_FWD, true>(ta, tb, p, stream);
       }
-      if (!make_map(&tb, g.B, g.Kred, g.N, BK, 256)) return 3;
+      if (!make_map(&tb, g.B, g.Kred, g.N, BK, g2.pair ? 128 : 256)) return 3;
+      if (g2.pair) return launch_pairs<false, false, GEMM_FWD>(ta, tb, p, stream);
       return launch_tiles<256, false, false, GEMM_FWD, false>(ta, tb, p, stream);
     case GEMM_DX:
       if (!make_map(&ta, g.A, g.Kred, g.M, BK, BM)) return 3;
       if (!make_map(&tb, g.B, g.N, g.Kred, 64, BK)) return 3;
+      if (g2.pair) return launch_pairs<false, true, GEMM_DX>(ta, tb, p, stream);
       return launch_tiles<256, false, true, GEMM_DX, false>(ta, tb, p, stream);
     case GEMM_DW:
       if (!make_map(&ta, g.A, g.M, g.Kred, 64, BK)) return 3;
       if (!make_map(&tb, g.B, g.N, g.Kred, 64, BK)) return 3;
+      if (g2.pair) return launch_pairs<true, true, GEMM_DW>(ta, tb, p, stream);
       return launch_tiles<256, true, true, GEMM_DW, false>(ta, tb, p, stream);
   }
   return 1;

@@ -21,6 +21,7 @@ EXPORTED = [
     "dqt_set_wait_limit_ns", "dqt_absmean_workspace_size", "dqt_absmean_init",
     "dqt_act_quant", "dqt_codes_to_bf16", "dqt_bitlinear_fwd", "dqt_bitlinear_bwd_dx",
     "dqt_bitlinear_bwd_dw_update", "dqt_sr_update", "dqt_absmean_init_noalloc",
+    "dqt_set_gemm_tiles",
 ]
 
 
@@ -59,6 +60,7 @@ def lib():
         L.dqt_status_string.restype = C.c_char_p
         L.dqt_check_device_status.argtypes = [_vp]
         L.dqt_set_wait_limit_ns.argtypes = [C.c_uint64]
+        L.dqt_set_gemm_tiles.argtypes = [C.c_int]
         L.dqt_absmean_workspace_size.argtypes = []
         L.dqt_absmean_workspace_size.restype = _sz
         L.dqt_absmean_init.argtypes = [_vp, _i64, dqt_grid_t, _vp, C.POINTER(C.c_float), _vp,
@@ -146,6 +148,11 @@ def dqt_check_device_status(stream=None):
 
 def dqt_set_wait_limit_ns(ns):
     _check(lib().dqt_set_wait_limit_ns(int(ns)), "dqt_set_wait_limit_ns")
+
+
+def dqt_set_gemm_tiles(mode):
+    """0 = 2-SM 256x256 tiles (default), 1 = 1-SM 128x256 tiles."""
+    _check(lib().dqt_set_gemm_tiles(int(mode)), "dqt_set_gemm_tiles")
 
 
 def dqt_absmean_init(W0, bits_or_grid, codes=None, stream=None):

@@ -336,3 +336,47 @@ def test_update_frequency_counter_ternary_step1():
     assert int(changed.item()) == moved
     rate = moved / c.size
     assert 0.2 * 1e-3 * s_w < rate < 1e-3 * s_w * 1.2
+
+
+# ---------------------------------------------------------------------------
+# both GEMM tilings (2-SM pair tiles are the default; 1-SM tiles forced here)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("mode", [0, 1])
+def test_both_tilings_agree_with_oracle(mode):
+    dqt.dqt_set_gemm_tiles(mode)
+    try:
+        _fwd_check(300, 264, 520, 1.58, seed=91)
+        _fwd_check(513, 512, 264, 4, seed=92)
+        X, dY, W0, c, s_w, g = problem(300, 264, 520, 1.58, seed=93)
+        W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
+        dX = dqt.dqt_bitlinear_bwd_dx(dY.cuda(), W_img, s_w)
+        dqt.dqt_check_device_status()
+        ref = oracle.bwd_dx(bits(dY), c, np.float32(s_w))
+        assert elem_err(dX.cpu().double().numpy(), ref) <= REL_TOL
+        _fused(300, 264, 520, 8, 3, seed=94)
+    finally:
+        dqt.dqt_set_gemm_tiles(0)
+
+
+def test_tilings_bit_identical():
+    """Same per-element arithmetic, same reduction order within a tile: the two
+    tilings give bit-identical forward outputs and identical fused updates."""
+    outs = []
+    for mode in (0, 1):
+        dqt.dqt_set_gemm_tiles(mode)
+        try:
+            X, dY, W0, c, s_w, g = problem(520, 512, 776, 1.58, seed=95)
+            _, s_x, q_img, xdq = dqt.dqt_act_quant(X.cuda(), want=("Xq_img", "Xdq"))
+            W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
+            Y = dqt.dqt_bitlinear_fwd(q_img, s_x, W_img, s_w, g)
+            dX = dqt.dqt_bitlinear_bwd_dx(dY.cuda(), W_img, s_w)
+            dW = torch.empty((776, 512), dtype=torch.float32, device="cuda")
+            dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), xdq, None, s_w, None, None, None, None, g,
+                                            dW_out=dW)
+            dqt.dqt_check_device_status()
+            outs.append((Y.cpu(), dX.cpu(), dW.cpu()))
+        finally:
+            dqt.dqt_set_gemm_tiles(0)
+    assert torch.equal(outs[0][0], outs[1][0])
+    assert torch.equal(outs[0][1], outs[1][1])
+    assert torch.equal(outs[0][2], outs[1][2])
