@@ -520,6 +520,8 @@ def run_kernel(args):
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     T, K, N = T_TOK, HID, INTER
+    if args.shape:
+        T, K, N = (int(x) for x in args.shape.split(","))
     g = dqt.grid(1.58)
     k = args.kernel
     if k == "sr_update":
@@ -554,13 +556,20 @@ def run_kernel(args):
             dW = torch.empty((N, K), dtype=torch.float32, device=dev)
             fn = lambda: dqt.dqt_bitlinear_bwd_dw_update(dY, xdq, None, s_w, None, None, None,  # noqa: E731
                                                          None, g, dW_out=dW)
+        elif k == "bwd_dw_unfused":  # gradient to memory, then the standalone update
+            dW = torch.empty((N, K), dtype=torch.float32, device=dev)
+
+            def fn():
+                dqt.dqt_bitlinear_bwd_dw_update(dY, xdq, None, s_w, None, None, None, None, g,
+                                                dW_out=dW)
+                dqt.dqt_sr_update(dW.view(-1), W.view(-1), s_w, m.view(-1), v.view(-1), hp, sr, g)
         elif k == "act_quant":
             fn = lambda: dqt.dqt_act_quant(X, None, s_x, q_img, xdq, want=())  # noqa: E731
         elif k == "codes_to_bf16":
             fn = lambda: dqt.dqt_codes_to_bf16(W, W_img)  # noqa: E731
         else:
             raise SystemExit("unknown kernel %s" % k)
-        if k in ("fwd", "bwd_dx", "bwd_dw_update", "bwd_dw"):
+        if k in ("fwd", "bwd_dx", "bwd_dw_update", "bwd_dw", "bwd_dw_unfused"):
             work, unit = 2.0 * T * K * N, "TFLOP/s"
         elif k == "act_quant":
             work, unit = 6.0 * T * K + 4 * T, "GB/s"
@@ -587,6 +596,7 @@ def run_kernel(args):
     peaks, kind = _peaks()
     peak = peaks["bf16_tflops"] if unit == "TFLOP/s" else peaks["hbm_gbs"]
     print(json.dumps({"kernel": k, "numel": args.numel if k == "sr_update" else None,
+                      "shape": None if k == "sr_update" else [T, K, N],
                       "median_ms": round(med, 5), "min_ms": round(min(ms), 5),
                       "rate": round(rate, 1), "unit": unit, "peak": peak,
                       "frac": round(rate / peak, 4), "peak_kind": "burst, " + kind,
@@ -605,6 +615,7 @@ def main():
                     help="time one kernel kind alone (fwd, bwd_dx, bwd_dw_update, act_quant, "
                          "codes_to_bf16, sr_update)")
     ap.add_argument("--numel", type=int, default=1 << 26, help="weights for --kernel sr_update")
+    ap.add_argument("--shape", default=None, help="T,K,N for --kernel GEMMs (default 8192,2048,5632)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -65,9 +65,11 @@ typedef struct {
 } dqt_grid_t;
 
 /* AdamW hyper-parameters (the optimiser of Sec. 4.1).  step >= 1 is the
- * 1-based optimiser step used for the bias corrections 1 - beta^step.  The
- * library derives, in fp64 rounded once to fp32: 1 - beta1, 1 - beta2,
- * 1 - beta1^step, 1 - beta2^step, 1 - lr * weight_decay and lr * s_w. */
+ * 1-based optimiser step used for the bias corrections bc1 = 1 - beta1^step,
+ * bc2 = 1 - beta2^step; eps > 0.  The library derives, in fp64 rounded once
+ * to fp32: 1 - beta1, 1 - beta2, k1 = bc1 / sqrt(bc2), k2 = bc1 * eps,
+ * 1 - lr * weight_decay and lr * s_w, and evaluates AdamW's
+ * m_hat / (sqrt(v_hat) + eps) as m / (sqrt(v) * k1 + k2). */
 typedef struct {
   float lr;
   float beta1;
@@ -179,7 +181,7 @@ int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, i
 /* Backward w.r.t. the weight fused with the DQT update (Sec. 3.2, Sec. 4.1, Eq. 5):
  *   g[n,k]  = sum_t dY[t,n] Xdq[t,k]              fp32 accumulation in tensor memory
  *   m, v    <- AdamW moments (fp32 [N, K], in place)
- *   x       = c decay - (lr s_w) * (m_hat / (sqrt(v_hat) + eps))     (= W' * s_w)
+ *   x       = c decay - (lr s_w) * m / (sqrt(v) k1 + k2)    (= W' * s_w, see dqt_adamw_t)
  *   c       <- Clip[SR(x), qmin, qmax]  (int8 [N, K], in place; round_mode 1: nearest)
  * The fp32 gradient never reaches memory unless dW_out (fp32 [N, K]) is given.
  * With W, m and v all NULL only dW_out is written (gradient only).

@@ -300,30 +300,36 @@ void dqt_oracle_bwd_dw_bf16x(const uint16_t* dY, const uint16_t* xdq, int64_t T,
 
 /* ------------------------------------------------------------------------ */
 /* AdamW (Loshchilov & Hutter; the optimiser of Sec 4.1) in the code domain. */
-/* The host-side constants follow from the hyper-parameters in fp64, each    */
-/* rounded once to fp32:                                                     */
-/*   omb1 = 1 - b1, omb2 = 1 - b2, bc1 = 1 - b1^step, bc2 = 1 - b2^step,     */
-/*   decay = 1 - lr * wd, lrs = lr * s_w.                                    */
+/* AdamW moves W by -lr * m_hat / (sqrt(v_hat) + eps) - lr * wd * W with     */
+/* m_hat = m'/bc1, v_hat = v'/bc2.  Multiplying through by bc1 gives the same */
+/* step with a single division:                                              */
+/*   m_hat / (sqrt(v_hat) + eps) = m' / (sqrt(v') * k1 + k2),                 */
+/*   k1 = bc1 / sqrt(bc2),  k2 = bc1 * eps.                                  */
+/* Host-side constants, from the hyper-parameters in fp64, each rounded once */
+/* to fp32:  omb1 = 1 - b1, omb2 = 1 - b2, bc = 1 - b^step,                  */
+/*   k1, k2 as above, decay = 1 - lr * wd, lrs = lr * s_w.                   */
 /* Per element, each a separately rounded fp32 operation:                    */
 /*   m' = b1 m + omb1 g ;  v' = b2 v + omb2 (g g)                            */
-/*   u  = (m' / bc1) / (sqrt(v' / bc2) + eps)                                */
+/*   u  = m' / (sqrt(v') k1 + k2)                                            */
 /*   x  = c decay - lrs u          (= W' s_w, the dense target in codes)     */
 /* ------------------------------------------------------------------------ */
 typedef struct {
-  float b1, b2, eps, omb1, omb2, bc1, bc2, decay, lrs;
+  float b1, b2, omb1, omb2, k1, k2, decay, lrs, pad;
 } oracle_adamw_consts;
 
 void dqt_oracle_adamw_consts(float lr, float b1, float b2, float eps, float wd,
                              int64_t step, float s_w, float* out9) {
+  double bc1 = 1.0 - pow((double)b1, (double)step);
+  double bc2 = 1.0 - pow((double)b2, (double)step);
   out9[0] = b1;
   out9[1] = b2;
-  out9[2] = eps;
-  out9[3] = (float)(1.0 - (double)b1);
-  out9[4] = (float)(1.0 - (double)b2);
-  out9[5] = (float)(1.0 - pow((double)b1, (double)step));
-  out9[6] = (float)(1.0 - pow((double)b2, (double)step));
-  out9[7] = (float)(1.0 - (double)lr * (double)wd);
-  out9[8] = (float)((double)lr * (double)s_w);
+  out9[2] = (float)(1.0 - (double)b1);
+  out9[3] = (float)(1.0 - (double)b2);
+  out9[4] = (float)(bc1 / sqrt(bc2));
+  out9[5] = (float)(bc1 * (double)eps);
+  out9[6] = (float)(1.0 - (double)lr * (double)wd);
+  out9[7] = (float)((double)lr * (double)s_w);
+  out9[8] = 0.0f;
 }
 
 static float adamw_x(const oracle_adamw_consts* h, float g, int8_t c, float* m,
@@ -337,10 +343,9 @@ static float adamw_x(const oracle_adamw_consts* h, float g, int8_t c, float* m,
   float vn = v1 + v2;
   *m = mn;
   *v = vn;
-  float mh = mn / h->bc1;
-  float vh = vn / h->bc2;
-  float den = sqrtf(vh) + h->eps;
-  float u = mh / den;
+  float sv = sqrtf(vn);
+  float den = sv * h->k1 + h->k2;
+  float u = mn / den;
   float cd = (float)c * h->decay;
   float du = h->lrs * u;
   return cd - du;

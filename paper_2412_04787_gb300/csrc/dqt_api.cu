@@ -52,21 +52,22 @@ int make_update_consts(const dqt_adamw_t* hp, const dqt_sr_t* sr, dqt_grid_t g, 
                        dqt::UpdateConsts* uc) {
   if (!hp || !sr || !grid_ok(g)) return DQT_ERR_ARG;
   if (hp->step < 1 || !(hp->beta1 >= 0.0f && hp->beta1 < 1.0f) ||
-      !(hp->beta2 >= 0.0f && hp->beta2 < 1.0f) || !(hp->eps >= 0.0f) || !(hp->lr >= 0.0f) ||
+      !(hp->beta2 >= 0.0f && hp->beta2 < 1.0f) || !(hp->eps > 0.0f) || !(hp->lr >= 0.0f) ||
       !isfinite(hp->weight_decay) || !(s_w > 0.0f) || !isfinite(s_w))
     return DQT_ERR_ARG;
   if (sr->round_mode != 0 && sr->round_mode != 1) return DQT_ERR_ARG;
   const double b1 = hp->beta1, b2 = hp->beta2, st = static_cast<double>(hp->step);
+  const double bc1 = 1.0 - pow(b1, st), bc2 = 1.0 - pow(b2, st);
+  if (!(bc1 > 0.0) || !(bc2 > 0.0)) return DQT_ERR_ARG;
   uc->b1 = hp->beta1;
   uc->b2 = hp->beta2;
-  uc->eps = hp->eps;
   uc->omb1 = static_cast<float>(1.0 - b1);
   uc->omb2 = static_cast<float>(1.0 - b2);
-  uc->bc1 = static_cast<float>(1.0 - pow(b1, st));
-  uc->bc2 = static_cast<float>(1.0 - pow(b2, st));
+  uc->k1 = static_cast<float>(bc1 / sqrt(bc2));
+  uc->k2 = static_cast<float>(bc1 * static_cast<double>(hp->eps));
   uc->decay = static_cast<float>(1.0 - static_cast<double>(hp->lr) * hp->weight_decay);
   uc->lrs = static_cast<float>(static_cast<double>(hp->lr) * static_cast<double>(s_w));
-  if (!(uc->bc1 > 0.0f) || !(uc->bc2 > 0.0f)) return DQT_ERR_ARG;
+  if (!(uc->k1 > 0.0f) || !(uc->k2 > 0.0f)) return DQT_ERR_ARG;
   uc->qmin = g.qmin;
   uc->qmax = g.qmax;
   uc->step_lo = static_cast<uint32_t>(hp->step);

@@ -355,11 +355,13 @@ __device__ __forceinline__ uint4 sr_words(uint64_t blk, uint32_t step_lo, uint32
 // ---------------------------------------------------------------------------
 // Per-element DQT update: AdamW (Sec. 4.1) in the code domain, then Eq. 1
 // stochastic rounding and the clamp that keeps the code on the n-bit grid
-// (Eq. 5).  Every operation is an individually rounded IEEE fp32 operation
-// (explicit _rn intrinsics: no contraction into FMA).
+// (Eq. 5).  AdamW's m_hat / (sqrt(v_hat) + eps) is evaluated with a single
+// division as m' / (sqrt(v') * k1 + k2), k1 = bc1 / sqrt(bc2), k2 = bc1 * eps
+// (host constants).  Every operation is an individually rounded IEEE fp32
+// operation (explicit _rn intrinsics: no contraction into FMA).
 // ---------------------------------------------------------------------------
 struct UpdateConsts {
-  float b1, b2, eps, omb1, omb2, bc1, bc2, decay, lrs;
+  float b1, b2, omb1, omb2, k1, k2, decay, lrs;
   int32_t qmin, qmax;
   uint32_t step_lo, tensor_id, key0, key1;
   int32_t round_mode;
@@ -371,9 +373,8 @@ __device__ __forceinline__ int32_t dqt_update_elem(const UpdateConsts& h, float 
   const float vn = __fadd_rn(__fmul_rn(h.b2, v), __fmul_rn(h.omb2, __fmul_rn(g, g)));
   m = mn;
   v = vn;
-  const float mh = __fdiv_rn(mn, h.bc1);
-  const float vh = __fdiv_rn(vn, h.bc2);
-  const float u = __fdiv_rn(mh, __fadd_rn(__fsqrt_rn(vh), h.eps));
+  const float den = __fadd_rn(__fmul_rn(__fsqrt_rn(vn), h.k1), h.k2);
+  const float u = __fdiv_rn(mn, den);
   const float x = __fsub_rn(__fmul_rn(static_cast<float>(c), h.decay), __fmul_rn(h.lrs, u));
   int32_t r;
   if (h.round_mode == 1) {

@@ -144,41 +144,47 @@ __device__ __forceinline__ void epi_dx(const Params& p, int gm, int gn0, const u
 }
 
 // dW: gradient -> AdamW -> SR -> codes, in registers, four weights (one
-// Philox block) per lane at a time.  The warp's 32 x 32 gradient block (lane
-// i holds row i) is transposed through shared memory so that eight lanes
-// share each row: every optimiser-state access of the warp then covers four
-// full 128-byte row segments instead of 32 scattered ones.  Streaming cache
-// hints keep the optimiser state from evicting the GEMM operands out of L2.
-__device__ __forceinline__ uint32_t epi_dw(const Params& p, int row0, int gn0,
-                                           const uint32_t (&a)[32], float* xp, int lane) {
+// Philox block) per lane at a time.  A warp owns 32 rows (its tensor-memory
+// lanes) and a run of 32-column chunks of the tile.  Each chunk's 32 x 32
+// gradient block is transposed through a padded shared buffer so that eight
+// lanes share a row: every optimiser-state access of the warp covers four
+// full 128-byte row segments instead of 32 scattered ones.  The loads are
+// software-pipelined in half-chunks (four rows per lane): the next half's
+// codes, m and v are in flight while the current half is updated.  Streaming
+// cache hints keep the optimiser state from evicting GEMM operands from L2.
+struct DwLoads {
+  float4 m[4], v[4];
+  char4 c[4];
+};
+
+__device__ __forceinline__ void dw_issue(const Params& p, int row0, int gn0, int h, int lane,
+                                         DwLoads& L) {
+  const int gk = gn0 + (lane & 7) * 4;
+  if (!p.W || gn0 >= p.N || gk >= p.N) return;
 #pragma unroll
-  for (int i = 0; i < 32; ++i) xp[lane * kStageLd + i] = __uint_as_float(a[i]);
-  __syncwarp();
-  const int cq = (lane & 7) * 4;  // this lane's four columns within the block
-  const int gk = gn0 + cq;
-  const bool col_ok = gk < p.N;
-  constexpr int R = 8;  // rows per lane: lane >> 3, +4, +8, ..., +28
-  float4 m4[R], v4[R];
-  char4 c4[R];
-  bool in[R];
-  // all of this lane's optimiser-state loads first: one memory round trip
-#pragma unroll
-  for (int j = 0; j < R; ++j) {
-    const int gm = row0 + (lane >> 3) + 4 * j;
-    in[j] = col_ok && gm < p.M;
-    if (p.W && in[j]) {
+  for (int j = 0; j < 4; ++j) {
+    const int gm = row0 + (lane >> 3) + 4 * (4 * h + j);
+    if (gm < p.M) {
       const size_t e = static_cast<size_t>(gm) * p.N + gk;
-      c4[j] = __ldcs(reinterpret_cast<const char4*>(p.W + e));
-      m4[j] = __ldcs(reinterpret_cast<const float4*>(p.m + e));
-      v4[j] = __ldcs(reinterpret_cast<const float4*>(p.v + e));
+      L.c[j] = __ldcs(reinterpret_cast<const char4*>(p.W + e));
+      L.m[j] = __ldcs(reinterpret_cast<const float4*>(p.m + e));
+      L.v[j] = __ldcs(reinterpret_cast<const float4*>(p.v + e));
     }
   }
+}
+
+__device__ __forceinline__ uint32_t dw_update(const Params& p, int row0, int gn0, int h, int lane,
+                                              const float* xp, DwLoads& L) {
+  const int cq = (lane & 7) * 4;
+  const int gk = gn0 + cq;
+  if (gn0 >= p.N || gk >= p.N) return 0;
   uint32_t n_changed = 0;
 #pragma unroll
-  for (int j = 0; j < R; ++j) {
-    if (!in[j]) continue;
-    const int r = (lane >> 3) + 4 * j;
-    const size_t e = static_cast<size_t>(row0 + r) * p.N + gk;
+  for (int j = 0; j < 4; ++j) {
+    const int r = (lane >> 3) + 4 * (4 * h + j);
+    const int gm = row0 + r;
+    if (gm >= p.M) continue;
+    const size_t e = static_cast<size_t>(gm) * p.N + gk;
     const float* src = xp + r * kStageLd + cq;
     const float4 g4 = make_float4(src[0], src[1], src[2], src[3]);
     if (p.dW_out) __stcs(reinterpret_cast<float4*>(p.dW_out + e), g4);
@@ -186,18 +192,54 @@ __device__ __forceinline__ uint32_t epi_dw(const Params& p, int row0, int gn0,
     uint4 w = make_uint4(0, 0, 0, 0);
     if (p.uc.round_mode == 0)
       w = sr_words(e >> 2, p.uc.step_lo, p.uc.tensor_id, p.uc.key0, p.uc.key1);
-    const int32_t n0c = dqt_update_elem(p.uc, g4.x, c4[j].x, m4[j].x, v4[j].x, w.x);
-    const int32_t n1c = dqt_update_elem(p.uc, g4.y, c4[j].y, m4[j].y, v4[j].y, w.y);
-    const int32_t n2c = dqt_update_elem(p.uc, g4.z, c4[j].z, m4[j].z, v4[j].z, w.z);
-    const int32_t n3c = dqt_update_elem(p.uc, g4.w, c4[j].w, m4[j].w, v4[j].w, w.w);
-    n_changed += (n0c != c4[j].x) + (n1c != c4[j].y) + (n2c != c4[j].z) + (n3c != c4[j].w);
+    const int32_t n0c = dqt_update_elem(p.uc, g4.x, L.c[j].x, L.m[j].x, L.v[j].x, w.x);
+    const int32_t n1c = dqt_update_elem(p.uc, g4.y, L.c[j].y, L.m[j].y, L.v[j].y, w.y);
+    const int32_t n2c = dqt_update_elem(p.uc, g4.z, L.c[j].z, L.m[j].z, L.v[j].z, w.z);
+    const int32_t n3c = dqt_update_elem(p.uc, g4.w, L.c[j].w, L.m[j].w, L.v[j].w, w.w);
+    n_changed += (n0c != L.c[j].x) + (n1c != L.c[j].y) + (n2c != L.c[j].z) + (n3c != L.c[j].w);
     __stcs(reinterpret_cast<char4*>(p.W + e),
            make_char4(static_cast<signed char>(n0c), static_cast<signed char>(n1c),
                       static_cast<signed char>(n2c), static_cast<signed char>(n3c)));
-    __stcs(reinterpret_cast<float4*>(p.m + e), m4[j]);
-    __stcs(reinterpret_cast<float4*>(p.v + e), v4[j]);
+    __stcs(reinterpret_cast<float4*>(p.m + e), L.m[j]);
+    __stcs(reinterpret_cast<float4*>(p.v + e), L.v[j]);
   }
-  __syncwarp();  // the transpose buffer is rewritten for the next block
+  return n_changed;
+}
+
+// The whole dW epilogue of one warp for one tile: `nchunk` chunks of 32
+// columns starting at column nbase, rows row0 .. row0 + 31, gradient in
+// tensor memory at t_acc (this warp's lanes, chunk cc at column 32 cc).
+// With PIPE the next half-chunk's loads are in flight while the current one
+// is updated (more registers, for kernels with few epilogue warps).
+template <bool PIPE>
+__device__ __forceinline__ uint32_t epi_dw_tile(const Params& p, int row0, int nbase, int nchunk,
+                                                uint32_t t_acc, float* xp, int lane) {
+  uint32_t n_changed = 0;
+  DwLoads A, B;
+  if (PIPE) dw_issue(p, row0, nbase, 0, lane, A);
+#pragma unroll 1
+  for (int cc = 0; cc < nchunk; ++cc) {
+    const int gn0 = nbase + cc * 32;
+    uint32_t a[32];
+    tmem_ld_32x32b_x32(t_acc + cc * 32, a);
+    tmem_ld_wait();
+#pragma unroll
+    for (int i = 0; i < 32; ++i) xp[lane * kStageLd + i] = __uint_as_float(a[i]);
+    __syncwarp();
+    if (PIPE) {
+      dw_issue(p, row0, gn0, 1, lane, B);
+      n_changed += dw_update(p, row0, gn0, 0, lane, xp, A);
+      if (cc + 1 < nchunk) dw_issue(p, row0, gn0 + 32, 0, lane, A);
+      n_changed += dw_update(p, row0, gn0, 1, lane, xp, B);
+    } else {
+#pragma unroll 1
+      for (int h = 0; h < 2; ++h) {
+        dw_issue(p, row0, gn0, h, lane, A);
+        n_changed += dw_update(p, row0, gn0, h, lane, xp, A);
+      }
+    }
+    __syncwarp();  // the transpose buffer is rewritten for the next chunk
+  }
   return n_changed;
 }
 
@@ -363,6 +405,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(b * BN + half * HALF);
         const uint32_t t_run = tmem + lane_off + RUN_COL + static_cast<uint32_t>(half * HALF);
         const bool last = (c + 1 == nchunks);
+        if (EPI == GEMM_DW) {
+          n_changed += epi_dw_tile<true>(p, gm - lane, nbase, HALF / 32, t_acc, xp, lane);
+        } else
 #pragma unroll 1
         for (int cc = 0; cc < HALF / 32; ++cc) {
           uint32_t a[32], r[32];
@@ -380,10 +425,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           const int gn0 = nbase + cc * 32;
           if (gn0 >= p.N) continue;  // warp-uniform
-          if (EPI == GEMM_DW) {
-            n_changed += epi_dw(p, gm - lane, gn0, a, xp, lane);
-            continue;
-          }
           if (!row_ok) continue;
           if (EPI == GEMM_FWD) epi_fwd(p, gm, gn0, a_t, a, r, DRAIN && c > 0);
           else epi_dx(p, gm, gn0, a);
@@ -422,33 +463,52 @@ __global__ void __launch_bounds__(kThreads, 1)
 // reads its own 128 rows from its own tensor memory and releases the
 // accumulator on the leader's `acc_empty` barrier.
 // ---------------------------------------------------------------------------
+// Epilogue warps of the 2-SM kernels: the dW update is compute-heavy (AdamW,
+// Philox, stochastic rounding per weight) and needs four warps per SM
+// sub-partition to hide its latencies; the forward and dX epilogues are light.
+template <int EPI>
+struct PairCfg {
+  static constexpr int EW = (EPI == GEMM_DW) ? 16 : 8;
+  static constexpr int THREADS = 64 + 32 * EW;
+};
+
 template <int EPI>
 struct SmemPair {
+  static constexpr int EW = PairCfg<EPI>::EW;
   static constexpr int A_BYTES = 128 * BK * 2;
   static constexpr int B_BYTES = 128 * BK * 2;  // this CTA's half of the B tile
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int STAGES = (EPI == GEMM_DW) ? 6 : 7;
+  static constexpr int STAGES = (EPI == GEMM_DW) ? 5 : 7;
   static constexpr int XPOSE_OFF = STAGES * STAGE_BYTES;
-  static constexpr int XPOSE_BYTES = (EPI == GEMM_DW) ? kEpiWarps * 32 * kStageLd * 4 : 0;
+  static constexpr int XPOSE_BYTES = (EPI == GEMM_DW) ? EW * 32 * kStageLd * 4 : 0;
   static constexpr int BAR_OFF = XPOSE_OFF + XPOSE_BYTES;
-  static constexpr int BYTES = BAR_OFF + 256 + 1024;
-  static_assert(BYTES <= 232448, "shared memory per CTA");
+  // alignment slack for the 1024-byte swizzle atoms, as much as fits
+  static constexpr int SLACK = (232448 - (BAR_OFF + 256)) < 1024 ? (232448 - (BAR_OFF + 256)) : 1024;
+  static constexpr int BYTES = BAR_OFF + 256 + SLACK;
+  static_assert(SLACK >= 0, "shared memory per CTA");
   static_assert((2 * STAGES + 5) * 8 + 4 <= 256, "barrier area");
 };
 
 template <bool A_MN, bool B_MN, int EPI>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
     gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA,
                      const __grid_constant__ CUtensorMap tmB, const Params p) {
   using S = SmemPair<EPI>;
   constexpr int ST = S::STAGES;
-  constexpr int BN = 256;    // pair tile width; each CTA holds all 256 columns of its rows
-  constexpr int HALF = 128;  // columns per epilogue warp
+  constexpr int EW = S::EW;
+  constexpr int BN = 256;           // pair tile width; each CTA holds all 256 columns of its rows
+  constexpr int HALF = BN / (EW / 4);  // columns per epilogue warp
   constexpr uint32_t IDESC = idesc_bf16(256, 256, A_MN, B_MN);
   constexpr uint32_t TMEM_COLS = 512;
   constexpr uint32_t MN_CHUNK_BYTES = 64 * BK * 2;
 
   extern __shared__ uint8_t smem_raw[];
+  // The dynamic shared window is 1024-byte aligned in practice; if it is not
+  // and the slack cannot absorb it, every CTA of the grid returns here alike.
+  if (((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u) > static_cast<uint32_t>(S::SLACK)) {
+    if (threadIdx.x == 0) record_timeout(p.status);
+    return;
+  }
   uint8_t* smem = align1024(smem_raw);
   uint8_t* sA = smem;
   uint8_t* sB = smem + ST * S::A_BYTES;
@@ -473,7 +533,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
-      mbar_init(&acc_empty[b], 2 * kEpiWarps);
+      mbar_init(&acc_empty[b], 2 * EW);
     }
     mbar_init(drain_bar, 1);
     fence_mbarrier_init();
@@ -578,9 +638,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_wait_cl(drain_bar, 0, kDrainNs);
     }
   } else {
-    // ---------------- epilogue (warps 2..9, both CTAs) ----------------
-    const int quad = warp & 3;
-    const int half = (warp - 2) >> 2;
+    // ---------------- epilogue (warps 2 .. EW+1, both CTAs) ----------------
+    const int quad = warp & 3;        // tensor-memory lanes this warp may access
+    const int half = (warp - 2) >> 2;  // which run of HALF columns
     const int row = quad * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     float* xp = reinterpret_cast<float*>(smem + S::XPOSE_OFF) + (warp - 2) * 32 * kStageLd;
@@ -598,6 +658,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       tc_fence_after();
       const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(b * BN + half * HALF);
+      if (EPI == GEMM_DW) {
+        n_changed += epi_dw_tile<false>(p, gm - lane, nbase, HALF / 32, t_acc, xp, lane);
+      } else
 #pragma unroll 1
       for (int cc = 0; cc < HALF / 32; ++cc) {
         uint32_t a[32], r[32];
@@ -605,10 +668,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld_wait();
         const int gn0 = nbase + cc * 32;
         if (gn0 >= p.N) continue;  // warp-uniform
-        if (EPI == GEMM_DW) {
-          n_changed += epi_dw(p, gm - lane, gn0, a, xp, lane);
-          continue;
-        }
         if (!row_ok) continue;
         if (EPI == GEMM_FWD) epi_fwd(p, gm, gn0, a_t, a, r, false);
         else epi_dx(p, gm, gn0, a);
@@ -695,6 +754,7 @@ template <bool A_MN, bool B_MN, int EPI>
 int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream) {
   auto kern = gemm_pair_kernel<A_MN, B_MN, EPI>;
   const int smem = SmemPair<EPI>::BYTES;
+  constexpr int threads = PairCfg<EPI>::THREADS;
   static int max_clusters = 0;  // per template instance
   p.num_n = (p.N + 255) / 256;
   p.num_tiles = ((p.M + 255) / 256) * p.num_n;
@@ -704,7 +764,7 @@ int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStr
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.blockDim = dim3(threads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cfg.attrs = attr;
