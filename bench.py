@@ -44,15 +44,18 @@ METRIC = "DQT BitLinear fwd+bwd+SR-update tokens/s"
 PROJ = [("gate", HID, INTER), ("up", HID, INTER), ("down", INTER, HID)]
 
 
-def kernel_fingerprint():
-    """Short hash of the CUDA sources: ncu counters quoted below belong to one build."""
-    import glob
+GEMM_SOURCES = ("gemm_tc.cu", "dqt_device.cuh", "dqt_internal.h")
+
+
+def kernel_fingerprint(files=GEMM_SOURCES):
+    """Short hash of the GEMM kernels' sources: the ncu counters quoted below
+    belong to one version of them."""
     import hashlib
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2412_04787_gb300", "csrc")
-    for f in sorted(glob.glob(os.path.join(csrc, "*"))):
-        with open(f, "rb") as fh:
-            h.update(os.path.basename(f).encode() + b"\0" + fh.read())
+    for f in files:
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(f.encode() + b"\0" + fh.read())
     return h.hexdigest()[:12]
 
 
@@ -61,7 +64,7 @@ def kernel_fingerprint():
 # launches move the same numbers of operand and optimiser-state bytes), keyed
 # by the kernel fingerprint it was taken on (see profiles/).  A stale entry
 # reports null.
-DW_TRAFFIC_BYTES = {"e6c668f9c149": 294566912 + 54456064}
+DW_TRAFFIC_BYTES = {"78cb4d4fdb1b": 294566912 + 54456064}
 
 
 def _dist():
@@ -228,15 +231,17 @@ class MLPStep:
 
         for st in s:
             after(st, main)
-        # forward
+        # forward: the three weight images convert while X is quantised
         aq("X", s[0])
-        codes("gate", s[0])
+        codes("gate", s[1])
+        codes("up", s[2])
+        codes("down", s[3])
         after(s[1], s[0])
-        codes("up", s[1])
-        codes("down", s[2])
-        fwd("gate", s[0])
-        fwd("up", s[1])
-        after(s[2], s[0], s[1])
+        after(s[2], s[0])
+        fwd("gate", s[1])
+        fwd("up", s[2])
+        after(s[0], s[1])
+        after(s[2], s[0], s[1], s[3])
         aq("H", s[2])
         fwd("down", s[2])
         # backward: down projection (dX and dW independent)

@@ -88,29 +88,36 @@ __global__ void __launch_bounds__(kAqWarps * 32)
   }
 }
 
-// Single-pass variant for rows of up to NV * 256 elements: each lane keeps
-// its NV 16-byte vectors of the row in registers between the absmax and the
-// quantisation.  The dequantised image needs bf16(q / s_x) for q in
-// [-128, 127] only, so each warp first fills a 256-entry table of those
-// correctly rounded quotients (8 divisions per lane) and then looks them up:
-// bit-identical to dividing per element.
+// Single-pass variant: WPR warps share a row and each lane keeps its (at
+// most NV) 16-byte vectors of the row in registers between the absmax and the
+// quantisation, so registers stay low and many rows are in flight per SM.
+// The warps of a row combine their partial amax through shared memory.  The
+// dequantised image needs bf16(q / s_x) for q in [-128, 127] only, so the
+// row's threads first fill a 256-entry table of those correctly rounded
+// quotients and then look them up: bit-identical to dividing per element.
 template <int NV>
-__global__ void __launch_bounds__(kAqWarps * 32)
-    act_quant_rows_kernel(const uint16_t* __restrict__ X, int T, int K, int8_t* __restrict__ Xq,
-                          float* __restrict__ s_x, uint16_t* __restrict__ Xq_img,
-                          uint16_t* __restrict__ Xdq) {
-  __shared__ uint16_t table[kAqWarps][256];
-  const int wid = threadIdx.x >> 5;
-  const int row = blockIdx.x * kAqWarps + wid;
+__global__ void __launch_bounds__(256)
+    act_quant_rows_kernel(const uint16_t* __restrict__ X, int T, int K, int wpr,
+                          int8_t* __restrict__ Xq, float* __restrict__ s_x,
+                          uint16_t* __restrict__ Xq_img, uint16_t* __restrict__ Xdq) {
+  __shared__ uint16_t table[8][256];
+  __shared__ float part[8];
+  const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  if (row >= T) return;
+  const int rib = warp / wpr;      // row within the block
+  const int wir = warp - rib * wpr;  // warp within the row
+  const int rpb = blockDim.x / (32 * wpr);
+  const int row = blockIdx.x * rpb + rib;
+  const bool live = row < T;
   const int nv = K >> 3;
-  const uint4* xr = reinterpret_cast<const uint4*>(X + static_cast<size_t>(row) * K);
+  const int tid = wir * 32 + lane;   // thread index within the row
+  const int nth = wpr * 32;
+  const uint4* xr = reinterpret_cast<const uint4*>(X + static_cast<size_t>(live ? row : 0) * K);
   uint4 u[NV];
 #pragma unroll
   for (int i = 0; i < NV; ++i) {
-    const int vi = lane + 32 * i;
-    u[i] = vi < nv ? __ldcs(xr + vi) : make_uint4(0, 0, 0, 0);
+    const int vi = tid + nth * i;
+    u[i] = (live && vi < nv) ? __ldcs(xr + vi) : make_uint4(0, 0, 0, 0);
   }
   float amax = 0.0f;
 #pragma unroll
@@ -124,17 +131,69 @@ __global__ void __launch_bounds__(kAqWarps * 32)
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+  if (lane == 0) part[warp] = amax;
+  __syncthreads();
+  amax = part[rib * wpr];
+  for (int w = 1; w < wpr; ++w) amax = fmaxf(amax, part[rib * wpr + w]);
   const float s = __fdiv_rn(127.0f, fmaxf(amax, 1e-5f));
-  if (lane == 0) s_x[row] = s;
+  if (live && tid == 0) s_x[row] = s;
   if (Xdq) {
-#pragma unroll
-    for (int j = lane; j < 256; j += 32)
-      table[wid][j] = f32_to_bf16_bits(__fdiv_rn(static_cast<float>(j - 128), s));
-    __syncwarp();
+    for (int j = tid; j < 256; j += nth)
+      table[rib][j] = f32_to_bf16_bits(__fdiv_rn(static_cast<float>(j - 128), s));
   }
+  __syncthreads();
+  if (!live) return;
   const size_t rbase = static_cast<size_t>(row) * K;
 #pragma unroll
   for (int i = 0; i < NV; ++i) {
+    const int vi = tid + nth * i;
+    if (vi >= nv) break;
+    const uint32_t w[4] = {u[i].x, u[i].y, u[i].z, u[i].w};
+    int32_t q[8];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float lo = bf16_bits_to_f32(w[j] & 0xFFFFu);
+      const float hi = bf16_bits_to_f32(w[j] >> 16);
+      q[2 * j] = static_cast<int32_t>(fminf(fmaxf(rintf(__fmul_rn(lo, s)), -128.0f), 127.0f));
+      q[2 * j + 1] = static_cast<int32_t>(fminf(fmaxf(rintf(__fmul_rn(hi, s)), -128.0f), 127.0f));
+    }
+    const size_t e = rbase + static_cast<size_t>(vi) * 8;
+    if (Xq) {
+      uint2 pk;
+      pk.x = (q[0] & 0xFF) | ((q[1] & 0xFF) << 8) | ((q[2] & 0xFF) << 16) | ((q[3] & 0xFF) << 24);
+      pk.y = (q[4] & 0xFF) | ((q[5] & 0xFF) << 8) | ((q[6] & 0xFF) << 16) | ((q[7] & 0xFF) << 24);
+      __stcs(reinterpret_cast<uint2*>(Xq + e), pk);
+    }
+    if (Xq_img) {
+      uint32_t h[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) h[j] = f32_to_bf16_bits(static_cast<float>(q[j]));
+      __stcs(reinterpret_cast<uint4*>(Xq_img + e),
+             make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
+                        h[6] | (h[7] << 16)));
+    }
+    if (Xdq) {
+      uint32_t h[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) h[j] = table[rib][q[j] + 128];
+      __stcs(reinterpret_cast<uint4*>(Xdq + e),
+             make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
+                        h[6] | (h[7] << 16)));
+    }
+  }
+}
+
+// Persistent variant for rows of at most 2048 elements (8 vectors per lane):
+// each warp walks rows row0, row0 + stride, ... and loads the next row while
+// it quantises the current one (two register buffers), so every warp keeps
+// two rows in flight and the grid has no wave tail.
+__device__ __forceinline__ void aq_row_store(const uint4 (&u)[8], int nv, int lane, float s,
+                                             size_t rbase, const uint16_t* table,
+                                             int8_t* __restrict__ Xq,
+                                             uint16_t* __restrict__ Xq_img,
+                                             uint16_t* __restrict__ Xdq) {
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
     const int vi = lane + 32 * i;
     if (vi >= nv) break;
     const uint32_t w[4] = {u[i].x, u[i].y, u[i].z, u[i].w};
@@ -164,7 +223,7 @@ __global__ void __launch_bounds__(kAqWarps * 32)
     if (Xdq) {
       uint32_t h[8];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) h[j] = table[wid][q[j] + 128];
+      for (int j = 0; j < 8; ++j) h[j] = table[q[j] + 128];
       __stcs(reinterpret_cast<uint4*>(Xdq + e),
              make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
                         h[6] | (h[7] << 16)));
@@ -172,30 +231,102 @@ __global__ void __launch_bounds__(kAqWarps * 32)
   }
 }
 
-// 16 codes per thread per step: one 16-byte load, two 16-byte stores.
+__device__ __forceinline__ void aq_row_load(const uint16_t* __restrict__ X, int row, int T, int K,
+                                            int nv, int lane, uint4 (&u)[8]) {
+  const uint4* xr = reinterpret_cast<const uint4*>(X + static_cast<size_t>(row) * K);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int vi = lane + 32 * i;
+    u[i] = (row < T && vi < nv) ? __ldcs(xr + vi) : make_uint4(0, 0, 0, 0);
+  }
+}
+
+__global__ void __launch_bounds__(256)
+    act_quant_persist_kernel(const uint16_t* __restrict__ X, int T, int K,
+                             int8_t* __restrict__ Xq, float* __restrict__ s_x,
+                             uint16_t* __restrict__ Xq_img, uint16_t* __restrict__ Xdq) {
+  __shared__ uint16_t table[8][256];
+  const int wid = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int stride = gridDim.x * 8;
+  const int nv = K >> 3;
+  uint4 ua[8], ub[8];
+  int row = blockIdx.x * 8 + wid;
+  aq_row_load(X, row, T, K, nv, lane, ua);
+  for (; row < T; row += stride) {
+    aq_row_load(X, row + stride, T, K, nv, lane, ub);  // next row in flight
+    float amax = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const uint32_t w[4] = {ua[i].x, ua[i].y, ua[i].z, ua[i].w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        amax = fmaxf(amax, fabsf(bf16_bits_to_f32(w[j] & 0xFFFFu)));
+        amax = fmaxf(amax, fabsf(bf16_bits_to_f32(w[j] >> 16)));
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+    const float s = __fdiv_rn(127.0f, fmaxf(amax, 1e-5f));
+    if (lane == 0) s_x[row] = s;
+    if (Xdq) {
+      __syncwarp();  // the previous row's lookups are done
+#pragma unroll
+      for (int j = lane; j < 256; j += 32)
+        table[wid][j] = f32_to_bf16_bits(__fdiv_rn(static_cast<float>(j - 128), s));
+      __syncwarp();
+    }
+    aq_row_store(ua, nv, lane, s, static_cast<size_t>(row) * K, table[wid], Xq, Xq_img, Xdq);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) ua[i] = ub[i];
+  }
+}
+
+// 64 codes per thread per step: four 16-byte loads issued together, then
+// eight 16-byte streaming stores (the image is read by the next kernel only).
+__device__ __forceinline__ void codes16_to_bf16(const uint4 u, uint4& o0, uint4& o1) {
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+  uint32_t o[8];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int32_t b0 = static_cast<int8_t>(w[j] & 0xFF);
+    const int32_t b1 = static_cast<int8_t>((w[j] >> 8) & 0xFF);
+    const int32_t b2 = static_cast<int8_t>((w[j] >> 16) & 0xFF);
+    const int32_t b3 = static_cast<int8_t>(w[j] >> 24);
+    o[2 * j] = f32_to_bf16_bits(static_cast<float>(b0)) |
+               (uint32_t(f32_to_bf16_bits(static_cast<float>(b1))) << 16);
+    o[2 * j + 1] = f32_to_bf16_bits(static_cast<float>(b2)) |
+                   (uint32_t(f32_to_bf16_bits(static_cast<float>(b3))) << 16);
+  }
+  o0 = make_uint4(o[0], o[1], o[2], o[3]);
+  o1 = make_uint4(o[4], o[5], o[6], o[7]);
+}
+
 __global__ void codes_to_bf16_kernel(const int8_t* __restrict__ W, int64_t numel,
                                      uint16_t* __restrict__ img) {
-  const int64_t nvec = numel >> 4;
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
-       i += stride) {
-    const uint4 u = __ldg(reinterpret_cast<const uint4*>(W) + i);
-    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-    uint32_t o[8];
+  const int64_t nvec = numel >> 4;  // 16-code vectors
+  const int64_t nthr = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const uint4* src = reinterpret_cast<const uint4*>(W);
+  uint4* dst = reinterpret_cast<uint4*>(img);
+  const int64_t t0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  // groups of four vectors, consecutive threads on consecutive vectors
+  for (int64_t base = 0; base < nvec; base += 4 * nthr) {
+    uint4 u[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      const int32_t b0 = static_cast<int8_t>(w[j] & 0xFF);
-      const int32_t b1 = static_cast<int8_t>((w[j] >> 8) & 0xFF);
-      const int32_t b2 = static_cast<int8_t>((w[j] >> 16) & 0xFF);
-      const int32_t b3 = static_cast<int8_t>(w[j] >> 24);
-      o[2 * j] = f32_to_bf16_bits(static_cast<float>(b0)) |
-                 (uint32_t(f32_to_bf16_bits(static_cast<float>(b1))) << 16);
-      o[2 * j + 1] = f32_to_bf16_bits(static_cast<float>(b2)) |
-                     (uint32_t(f32_to_bf16_bits(static_cast<float>(b3))) << 16);
+      const int64_t i = base + j * nthr + t0;
+      u[j] = i < nvec ? __ldcs(src + i) : make_uint4(0, 0, 0, 0);
     }
-    uint4* dst = reinterpret_cast<uint4*>(img) + 2 * i;
-    dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
-    dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int64_t i = base + j * nthr + t0;
+      if (i < nvec) {
+        uint4 o0, o1;
+        codes16_to_bf16(u[j], o0, o1);
+        __stcs(dst + 2 * i, o0);
+        __stcs(dst + 2 * i + 1, o1);
+      }
+    }
   }
   // ragged tail (numel % 16 elements), one thread
   if (blockIdx.x == 0 && threadIdx.x == 0)
@@ -261,24 +392,38 @@ int grid_for(int64_t work, int threads) {
 
 int launch_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
                      uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream) {
-  const int blocks = static_cast<int>((T + kAqWarps - 1) / kAqWarps);
   const int t = static_cast<int>(T), k = static_cast<int>(K);
-  const int nvl = static_cast<int>((K / 8 + 31) / 32);  // 16-byte vectors per lane
-#define DQT_AQ(NV) act_quant_rows_kernel<NV><<<blocks, kAqWarps * 32, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq)
-  if (nvl <= 2) DQT_AQ(2);
-  else if (nvl <= 4) DQT_AQ(4);
-  else if (nvl <= 8) DQT_AQ(8);
-  else if (nvl <= 12) DQT_AQ(12);
-  else if (nvl <= 16) DQT_AQ(16);
-  else if (nvl <= 24) DQT_AQ(24);
-  else act_quant_kernel<<<blocks, kAqWarps * 32, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq);
-#undef DQT_AQ
+  const int64_t nv = K / 8;  // 16-byte vectors per row
+  // warps per row: keep at most 4 vectors (32 values) per lane; up to 8 warps
+  const int wpr = static_cast<int>((nv + 127) / 128);
+  if (nv <= 256) {
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t want = (T + 7) / 8;
+    const int blocks = static_cast<int>(want < 2 * sms ? want : 2 * sms);
+    act_quant_persist_kernel<<<blocks, 256, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq);
+  } else if (wpr <= 8) {
+    const int rpb = 8 / wpr;
+    const int threads = 32 * wpr * rpb;
+    const int blocks = static_cast<int>((T + rpb - 1) / rpb);
+    const int per_lane = static_cast<int>((nv + 32 * wpr - 1) / (32 * wpr));
+    if (per_lane <= 2)
+      act_quant_rows_kernel<2><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
+    else if (per_lane <= 4)
+      act_quant_rows_kernel<4><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
+    else
+      act_quant_rows_kernel<8><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
+  } else {
+    const int blocks = static_cast<int>((T + kAqWarps - 1) / kAqWarps);
+    act_quant_kernel<<<blocks, kAqWarps * 32, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq);
+  }
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
 int launch_codes_to_bf16(const int8_t* W, int64_t numel, uint16_t* W_img, cudaStream_t stream) {
   const int threads = 256;
-  codes_to_bf16_kernel<<<grid_for((numel >> 4) + 1, threads), threads, 0, stream>>>(W, numel, W_img);
+  codes_to_bf16_kernel<<<grid_for((numel >> 6) + 1, threads), threads, 0, stream>>>(W, numel, W_img);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
