@@ -141,13 +141,20 @@ class MLPStep:
         self.dev = dev
         self.grid = dqt.grid(1.58)
         T = T_TOK
-        self.host = {
-            "X": inputs.normal((T, HID), 1.0, seed=1, dtype=torch.bfloat16),
-            "H": inputs.normal((T, INTER), 1.0, seed=2, dtype=torch.bfloat16),
-        }
-        for i, (name, K, N) in enumerate(PROJ):
-            self.host["dY_" + name] = inputs.normal((T, N), 1e-2, seed=10 + i, dtype=torch.bfloat16)
-        self.d = {k: v.to(dev) for k, v in self.host.items()}
+        # two seeded input sets, alternated step by step, so that the
+        # optimiser sees changing gradients as in training
+        self.host_sets = []
+        for r in range(2):
+            h = {"X": inputs.normal((T, HID), 1.0, seed=1 + 100 * r, dtype=torch.bfloat16),
+                 "H": inputs.normal((T, INTER), 1.0, seed=2 + 100 * r, dtype=torch.bfloat16)}
+            for i, (name, K, N) in enumerate(PROJ):
+                h["dY_" + name] = inputs.normal((T, N), 1e-2, seed=10 + i + 100 * r,
+                                                dtype=torch.bfloat16)
+            self.host_sets.append(h)
+        self.host = self.host_sets[0]
+        self.dev_sets = [{k: v.to(dev) for k, v in h.items()} for h in self.host_sets]
+        self.d = self.dev_sets[0]
+        self.alternate = True
         self.W, self.s_w, self.m, self.v, self.W_img, self.Y, self.dX, self.Xdq = {}, {}, {}, {}, {}, {}, {}, {}
         for i, (name, K, N) in enumerate(PROJ):
             W0 = inputs.normal((N, K), 0.02, seed=20 + i).to(dev)
@@ -180,6 +187,8 @@ class MLPStep:
         receives (start, end) CUDA events recorded on the kernel's stream."""
         dqt = self.dqt
         self.step_no += 1
+        if self.alternate:
+            self.d = self.dev_sets[self.step_no % 2]
         hp = dqt.adamw(lr=1e-3, step=self.step_no)
         main = torch.cuda.current_stream()
         # serial: the same launches, in the same order, all on the current stream
@@ -387,11 +396,13 @@ def run_gpu(args):
     # memory; the copy of step i+1 runs on a copy stream into the second of
     # two device buffer sets while step i computes (double buffering), and
     # each step's changed-code counts are read back to pinned host memory.
-    pinned = {k: v.pin_memory() for k, v in st.host.items()}
+    pinned_sets = [{k: v.pin_memory() for k, v in h.items()} for h in st.host_sets]
+    pinned = pinned_sets[0]
     res_host = torch.empty((2, 3), dtype=torch.int64).pin_memory()
     h2d = sum(v.numel() * v.element_size() for v in pinned.values())
     d2h = res_host[0].numel() * res_host.element_size()
-    bufs = [st.d, {k: torch.empty_like(v) for k, v in st.d.items()}]
+    st.alternate = False  # here the inputs arrive from the host each step
+    bufs = [st.dev_sets[0], st.dev_sets[1]]
     # the copies are split into 32 MiB pieces spread over several copy
     # streams so that more than one DMA engine drives the host link
     n_copy = 4
@@ -414,9 +425,10 @@ def run_gpu(args):
             if after is not None:
                 cs.wait_event(after)
             with torch.cuda.stream(cs):
+                src_set = pinned_sets[i % 2]
                 for k, off, n in jobs[j::n_copy]:
                     dst = bufs[i % 2][k].view(-1).view(torch.uint8)[off:off + n]
-                    dst.copy_(pinned[k].view(-1).view(torch.uint8)[off:off + n], non_blocking=True)
+                    dst.copy_(src_set[k].view(-1).view(torch.uint8)[off:off + n], non_blocking=True)
                 ev = torch.cuda.Event()
                 ev.record(cs)
                 evs.append(ev)
@@ -438,6 +450,7 @@ def run_gpu(args):
     e1.record(stream)
     barrier()
     st.d = bufs[0]
+    st.alternate = True
     e_ms = max_over_ranks(e0.elapsed_time(e1), dev)
     dqt.dqt_check_device_status()
     e2e = {"value": round(aggregate_tokens_per_s(ws, T_TOK, e_steps, e_ms), 1), "unit": "tokens/s",
@@ -644,6 +657,74 @@ def run_kernel(args):
                       "l2": "256 MiB buffer written between launches"}))
 
 
+def run_decoder(args):
+    """A LLaMA-structured decoder training step with every transformer linear
+    layer a DQT BitLinear (12 layers, hidden 768, 12 heads, FFN 2048, vocab
+    32000, batch 16 x seq 1024, ternary; synthetic uniform token ids).  The
+    BitLinear layers update themselves during backward; the bf16 embedding,
+    norms and head are stepped by torch AdamW inside the timed region."""
+    from paper_2412_04787_gb300 import build as dqt_build
+    from paper_2412_04787_gb300.decoder import DecoderConfig, DQTDecoder
+    dqt_build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    B, S = 16, 1024
+    cfg = DecoderConfig(layers=12, hidden=768, heads=12, ffn=2048, vocab=32000, bits=1.58,
+                        lr=1e-3, seed=1234)
+    model = DQTDecoder(cfg, device=dev)
+    opt = torch.optim.AdamW(model.dense_parameters(), lr=1e-3, fused=True)
+    g = torch.Generator().manual_seed(5)
+    host_ids = [torch.randint(0, cfg.vocab, (B, S + 1), generator=g).pin_memory() for _ in range(2)]
+    ids_dev = [h.to(dev) for h in host_ids]
+    stream = torch.cuda.current_stream()
+
+    def step(ids):
+        loss = model(ids[:, :-1], ids[:, 1:])
+        loss.backward()
+        opt.step()
+        opt.zero_grad(set_to_none=True)
+        return loss
+
+    for i in range(args.warmup):
+        step(ids_dev[i % 2])
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    with ClockSampler(dev.index) as clk:
+        t0.record(stream)
+        for i in range(args.steps):
+            step(ids_dev[i % 2])
+        t1.record(stream)
+        torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1)
+    tokens = B * S
+    # e2e: ids from pinned host memory each step, the loss read back each step
+    loss_host = torch.empty((), dtype=torch.float32).pin_memory()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(args.steps):
+        ids = host_ids[i % 2].to(dev, non_blocking=True)
+        loss = step(ids)
+        loss_host.copy_(loss.detach(), non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e_ms = e0.elapsed_time(e1)
+    bl_flops = model.bitlinear_flops_per_step(tokens)
+    print(json.dumps({
+        "metric": "DQT decoder training step tokens/s", "value": round(tokens * args.steps / (ms / 1e3), 1),
+        "unit": "tokens/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms / args.steps, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic uniform token ids",
+        "config": {"workload": "LLaMA-structured decoder, ternary DQT BitLinear in q,k,v,o,gate,up,down",
+                   "layers": 12, "hidden": 768, "heads": 12, "ffn": 2048, "vocab": 32000,
+                   "batch": B, "seq": S},
+        "bitlinear_tflop_per_step": round(bl_flops / 1e12, 3),
+        "e2e": {"value": round(tokens * args.steps / (e_ms / 1e3), 1), "unit": "tokens/s",
+                "h2d_bytes_per_step": int(host_ids[0].numel() * 8), "d2h_bytes_per_step": 4},
+        "final_loss": float(loss_host), "clocks": clk.summary()}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -657,10 +738,14 @@ def main():
                          "codes_to_bf16, sr_update)")
     ap.add_argument("--numel", type=int, default=1 << 26, help="weights for --kernel sr_update")
     ap.add_argument("--shape", default=None, help="T,K,N for --kernel GEMMs (default 8192,2048,5632)")
+    ap.add_argument("--workload", default="mlp", choices=["mlp", "decoder"],
+                    help="mlp: the headline BitLinear MLP GEMM set; decoder: a 12-layer DQT decoder step")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.kernel:
+    if args.workload == "decoder" and args.impl == "dqt" and not args.kernel:
+        run_decoder(args)
+    elif args.kernel:
         run_kernel(args)
     elif args.impl == "reference":
         run_reference(args)

@@ -1,0 +1,130 @@
+"""DQT BitLinear as a torch module (argument marshalling over the C ABI).
+
+A ``DQTBitLinear`` layer holds only what DQT keeps (Sec. 3.2): the n-bit
+integer codes of its weight (int8), the per-tensor scale s_w fixed at
+initialisation (Eq. 2-4), and AdamW's two moments (Sec. 4.1).  There is no
+high-precision weight and no weight gradient tensor:
+
+* forward: 8-bit per-token activation codes (``dqt_act_quant``), the exact
+  bf16 image of the weight codes (``dqt_codes_to_bf16``) and the integer GEMM
+  (``dqt_bitlinear_fwd``);
+* backward: dX through W_tilde (``dqt_bitlinear_bwd_dx``), then the weight
+  gradient is reduced on the tensor cores and consumed in the same kernel by
+  the AdamW step and stochastic rounding onto the grid
+  (``dqt_bitlinear_bwd_dw_update``, Eq. 1 and Eq. 5): the layer is updated
+  during its own backward.
+
+Consequences: one backward per forward (no gradient accumulation across
+micro-batches, no weight sharing between calls), and ``optimizer.step()`` is
+not needed for these layers.  The state is ordinary module buffers, so
+``state_dict()`` checkpoints it (codes, m, v as buffers; s_w, step, seed and
+tensor id as extra state).
+"""
+import torch
+
+from . import dqt
+
+__all__ = ["DQTBitLinear"]
+
+
+class _BitLinearFn(torch.autograd.Function):
+    @staticmethod
+    def forward(ctx, x, anchor, layer):
+        K, N = layer.in_features, layer.out_features
+        x2 = x.reshape(-1, K)
+        if x2.dtype != torch.bfloat16:
+            x2 = x2.to(torch.bfloat16)
+        x2 = x2.contiguous()
+        _, s_x, q_img, xdq = dqt.dqt_act_quant(x2, want=("Xq_img", "Xdq"))
+        w_img = dqt.dqt_codes_to_bf16(layer.codes)
+        y = dqt.dqt_bitlinear_fwd(q_img, s_x, w_img, float(layer.s_w), layer.grid_tuple)
+        ctx.save_for_backward(xdq)
+        ctx.layer = layer
+        ctx.in_shape = x.shape
+        ctx.in_dtype = x.dtype
+        return y.reshape(*x.shape[:-1], N)
+
+    @staticmethod
+    def backward(ctx, dy):
+        (xdq,) = ctx.saved_tensors
+        layer = ctx.layer
+        N = layer.out_features
+        dy2 = dy.reshape(-1, N)
+        if dy2.dtype != torch.bfloat16:
+            dy2 = dy2.to(torch.bfloat16)
+        dy2 = dy2.contiguous()
+        # the codes have not changed since the forward: the image is rebuilt
+        # instead of being kept alive across the step
+        w_img = dqt.dqt_codes_to_bf16(layer.codes)
+        dx = dqt.dqt_bitlinear_bwd_dx(dy2, w_img, float(layer.s_w))
+        if layer.update_in_backward:
+            layer._dqt_update(dy2, xdq)
+        return dx.reshape(ctx.in_shape).to(ctx.in_dtype), None, None
+
+
+class DQTBitLinear(torch.nn.Module):
+    """y = X_tilde W_tilde^T with W_tilde = codes / s_w, trained by DQT.
+
+    bits: 1.58 (ternary) or an integer width 2..8 (Eq. 3).  The dense initial
+    weight is drawn N(0, init_std) from ``init_seed`` and quantised once with
+    AbsMean (Eq. 2-4) on the device.  ``lr``, ``betas``, ``eps`` and
+    ``weight_decay`` are AdamW's; ``seed`` and ``tensor_id`` key the Philox
+    stream of stochastic rounding (``round_mode`` 1 = round to nearest, the
+    Sec. 5.1 ablation).
+    """
+
+    def __init__(self, in_features, out_features, bits=1.58, lr=1e-3, betas=(0.9, 0.999),
+                 eps=1e-8, weight_decay=0.0, seed=1234, tensor_id=0, init_std=0.02,
+                 init_seed=0, round_mode=0, device="cuda"):
+        super().__init__()
+        if in_features % 8 or out_features % 8:
+            raise ValueError("in_features and out_features must be multiples of 8")
+        self.in_features = in_features
+        self.out_features = out_features
+        g = dqt.grid(bits)
+        self.grid_tuple = (g.qmin, g.qmax)
+        self.lr, self.betas, self.eps, self.weight_decay = lr, tuple(betas), eps, weight_decay
+        self.round_mode = round_mode
+        self.update_in_backward = True
+        gen = torch.Generator(device="cpu")
+        gen.manual_seed(int(init_seed))
+        w0 = (torch.randn(out_features, in_features, generator=gen) * init_std).to(device)
+        codes, s_w = dqt.dqt_absmean_init(w0, self.grid_tuple)
+        del w0
+        self.register_buffer("codes", codes)
+        self.register_buffer("m", torch.zeros(out_features, in_features, device=device))
+        self.register_buffer("v", torch.zeros(out_features, in_features, device=device))
+        # changed-code counter (Sec. 5.2 update frequency), accumulated
+        self.register_buffer("changed", torch.zeros(1, dtype=torch.int64, device=device))
+        self.s_w = float(s_w)
+        self.step = 0
+        self.seed = int(seed)
+        self.tensor_id = int(tensor_id)
+        # anchor: a 0-element tensor that requires grad, so the layer's
+        # backward (and with it the DQT update) runs even if x does not
+        self._anchor = torch.nn.Parameter(torch.zeros(0, device=device), requires_grad=True)
+
+    # host scalars of the DQT state travel in state_dict as extra state
+    def get_extra_state(self):
+        return {"s_w": self.s_w, "step": self.step, "seed": self.seed, "tensor_id": self.tensor_id}
+
+    def set_extra_state(self, state):
+        self.s_w = float(state["s_w"])
+        self.step = int(state["step"])
+        self.seed = int(state["seed"])
+        self.tensor_id = int(state["tensor_id"])
+
+    def forward(self, x):
+        return _BitLinearFn.apply(x, self._anchor, self)
+
+    def _dqt_update(self, dy2, xdq):
+        self.step += 1
+        hp = dqt.adamw(lr=self.lr, beta1=self.betas[0], beta2=self.betas[1], eps=self.eps,
+                       weight_decay=self.weight_decay, step=self.step)
+        sr = dqt.sr_stream(seed=self.seed, tensor_id=self.tensor_id, round_mode=self.round_mode)
+        dqt.dqt_bitlinear_bwd_dw_update(dy2, xdq, self.codes, self.s_w, self.m, self.v, hp, sr,
+                                        self.grid_tuple, changed_out=self.changed)
+
+    def extra_repr(self):
+        return "in_features=%d, out_features=%d, grid=%s" % (self.in_features, self.out_features,
+                                                            self.grid_tuple)

@@ -1,0 +1,126 @@
+"""LLaMA-structured decoder whose linear layers are DQT BitLinear layers.
+
+The paper trains LLaMA-2-structured models (Sec. 4.1) with every weight
+matrix of the transformer blocks kept at n bits and updated by stochastic
+rounding (Sec. 3.2, Eq. 5).  Here q, k, v, o, gate, up and down are
+``DQTBitLinear`` layers running on this library's kernels; the token
+embedding, the RMSNorm gains and the output head stay in bf16 and are trained
+by an ordinary optimiser (which weights the paper keeps in high precision is
+not stated; this is the BitNet convention).  RMSNorm, rotary position
+embedding, causal attention (``scaled_dot_product_attention``), SwiGLU and the
+cross-entropy loss are PyTorch operations around the BitLinear hot path.
+
+A training step is ``loss = model(ids, targets); loss.backward();
+opt.step(); opt.zero_grad()``: each BitLinear applies its DQT update during
+its own backward, the optimiser only sees the bf16 parameters
+(``model.dense_parameters()``).
+"""
+
+import torch
+import torch.nn.functional as F
+
+from .bitlinear import DQTBitLinear
+
+__all__ = ["DecoderConfig", "DQTDecoder"]
+
+
+class DecoderConfig:
+    def __init__(self, layers=12, hidden=768, heads=12, ffn=2048, vocab=32000, bits=1.58,
+                 lr=1e-3, seed=1234, rope_theta=10000.0, norm_eps=1e-6):
+        self.layers, self.hidden, self.heads, self.ffn, self.vocab = layers, hidden, heads, ffn, vocab
+        self.bits, self.lr, self.seed = bits, lr, seed
+        self.rope_theta, self.norm_eps = rope_theta, norm_eps
+
+
+class RMSNorm(torch.nn.Module):
+    def __init__(self, dim, eps, device):
+        super().__init__()
+        self.eps = eps
+        self.weight = torch.nn.Parameter(torch.ones(dim, device=device, dtype=torch.bfloat16))
+
+    def forward(self, x):
+        xf = x.float()
+        y = xf * torch.rsqrt(xf.pow(2).mean(-1, keepdim=True) + self.eps)
+        return (y * self.weight.float()).to(torch.bfloat16)
+
+
+def _rope(x, cos, sin):
+    # x: [B, H, S, D]; rotate pairs (first half, second half)
+    d = x.shape[-1] // 2
+    x1, x2 = x[..., :d], x[..., d:]
+    return torch.cat([x1 * cos - x2 * sin, x1 * sin + x2 * cos], dim=-1)
+
+
+class Block(torch.nn.Module):
+    def __init__(self, cfg, index, device):
+        super().__init__()
+        h, f = cfg.hidden, cfg.ffn
+        self.heads = cfg.heads
+        self.attn_norm = RMSNorm(h, cfg.norm_eps, device)
+        self.mlp_norm = RMSNorm(h, cfg.norm_eps, device)
+
+        def bl(k, n, j):
+            tid = index * 8 + j  # distinct Philox stream and initial draw per weight
+            return DQTBitLinear(k, n, bits=cfg.bits, lr=cfg.lr, seed=cfg.seed, tensor_id=tid,
+                                init_seed=cfg.seed * 1000 + tid, device=device)
+
+        self.q, self.k, self.v, self.o = bl(h, h, 0), bl(h, h, 1), bl(h, h, 2), bl(h, h, 3)
+        self.gate, self.up, self.down = bl(h, f, 4), bl(h, f, 5), bl(f, h, 6)
+
+    def forward(self, x, cos, sin):
+        B, S, Hd = x.shape
+        nh = self.heads
+        hd = Hd // nh
+        a = self.attn_norm(x)
+        q = self.q(a).view(B, S, nh, hd).transpose(1, 2)
+        k = self.k(a).view(B, S, nh, hd).transpose(1, 2)
+        v = self.v(a).view(B, S, nh, hd).transpose(1, 2)
+        q, k = _rope(q, cos, sin), _rope(k, cos, sin)
+        o = F.scaled_dot_product_attention(q, k, v, is_causal=True)
+        x = x + self.o(o.transpose(1, 2).reshape(B, S, Hd))
+        m = self.mlp_norm(x)
+        return x + self.down(F.silu(self.gate(m)) * self.up(m))
+
+
+class DQTDecoder(torch.nn.Module):
+    def __init__(self, cfg, device="cuda"):
+        super().__init__()
+        self.cfg = cfg
+        g = torch.Generator(device="cpu")
+        g.manual_seed(cfg.seed)
+        emb = torch.randn(cfg.vocab, cfg.hidden, generator=g) * 0.02
+        head = torch.randn(cfg.vocab, cfg.hidden, generator=g) * 0.02
+        self.embed = torch.nn.Parameter(emb.to(device=device, dtype=torch.bfloat16))
+        self.blocks = torch.nn.ModuleList([Block(cfg, i, device) for i in range(cfg.layers)])
+        self.norm = RMSNorm(cfg.hidden, cfg.norm_eps, device)
+        self.head = torch.nn.Parameter(head.to(device=device, dtype=torch.bfloat16))
+        hd = cfg.hidden // cfg.heads
+        self.register_buffer("inv_freq", 1.0 / (cfg.rope_theta ** (torch.arange(0, hd, 2, device=device,
+                                                                                  dtype=torch.float32) / hd)),
+                             persistent=False)
+
+    def bitlinear_layers(self):
+        return [m for m in self.modules() if isinstance(m, DQTBitLinear)]
+
+    def dense_parameters(self):
+        """The bf16 parameters an ordinary optimiser trains (not the BitLinear codes)."""
+        return [p for n, p in self.named_parameters() if not n.endswith("_anchor")]
+
+    def forward(self, ids, targets=None):
+        B, S = ids.shape
+        x = F.embedding(ids, self.embed)
+        t = torch.arange(S, device=ids.device, dtype=torch.float32)
+        ang = torch.outer(t, self.inv_freq)
+        cos = ang.cos().to(torch.bfloat16)[None, None]
+        sin = ang.sin().to(torch.bfloat16)[None, None]
+        for blk in self.blocks:
+            x = blk(x, cos, sin)
+        x = self.norm(x)
+        logits = x @ self.head.t()
+        if targets is None:
+            return logits
+        return F.cross_entropy(logits.float().view(-1, logits.shape[-1]), targets.reshape(-1))
+
+    def bitlinear_flops_per_step(self, tokens):
+        """Forward + dX + dW FLOPs of all BitLinear layers for `tokens` tokens."""
+        return sum(6.0 * tokens * m.in_features * m.out_features for m in self.bitlinear_layers())

@@ -1,0 +1,133 @@
+"""DQTBitLinear (the torch module over the C ABI) and the LLaMA-structured DQT
+decoder.
+
+* The module's forward is the oracle's BitLinear forward bit for bit; its
+  backward returns dX within the dX tolerance and leaves the codes where the
+  oracle's DQT update (Eq. 5, fed the bf16-environment weight gradient) puts
+  them, to the fused-update tolerance.
+* state_dict carries the whole DQT state: reload + step == continue.
+* A small decoder trained on a fixed batch lowers its loss with ternary and
+  8-bit weights (Sec. 4.2: training with only low-precision weights
+  converges), and its BitLinear codes move.  With round-to-nearest instead of
+  stochastic rounding (the Sec. 5.1 ablation) and lr * s_w < 1/2, no code can
+  ever move: the update is lost, as the paper observes.
+"""
+import io
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2412_04787_gb300 import inputs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2412_04787_gb300 import build
+    build.build()
+
+
+def bits(t):
+    return t.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+
+
+@pytest.mark.parametrize("bits_w", [1.58, 8])
+def test_bitlinear_module_matches_oracle(bits_w):
+    from paper_2412_04787_gb300.bitlinear import DQTBitLinear
+    T, K, N = 300, 264, 520
+    layer = DQTBitLinear(K, N, bits=bits_w, lr=1e-3, seed=99, tensor_id=4, init_seed=7)
+    qmin, qmax = layer.grid_tuple
+    # the layer starts from the oracle's AbsMean codes of a seeded W0
+    c0, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=7).numpy(), qmin, qmax)
+    layer.codes.copy_(torch.from_numpy(c0))
+    layer.s_w = float(s_w)
+    X = inputs.normal((T, K), 1.0, seed=1, dtype=torch.bfloat16)
+    dY = inputs.normal((T, N), 1e-2, seed=2, dtype=torch.bfloat16)
+    x = X.cuda().requires_grad_(True)
+    y = layer(x)
+    torch.cuda.synchronize()
+    q, s, _, xd = oracle.act_quant(bits(X))
+    Yr, _ = oracle.fwd(q, s, c0, np.float32(layer.s_w))
+    assert np.array_equal(bits(y), Yr)
+    y.backward(dY.cuda())
+    torch.cuda.synchronize()
+    dXr = oracle.bwd_dx(bits(dY), c0, np.float32(layer.s_w))
+    err = np.abs(x.grad.cpu().double().numpy() - dXr).max() / np.abs(dXr).max()
+    assert err <= 2e-2
+    g = oracle.bwd_dw_bf16x(bits(dY), xd).astype(np.float32)
+    k = oracle.adamw_consts(1e-3, 0.9, 0.999, 1e-8, 0.0, 1, layer.s_w)
+    z = np.zeros((N, K), np.float32)
+    c1, m1, _, _ = oracle.update(g, c0, z, z, k, qmin, qmax, 99, 1, 4)
+    cg = layer.codes.cpu().numpy().astype(np.int32)
+    diff = cg != c1
+    assert diff.mean() <= 1e-4 + 1.0 / diff.size
+    assert (np.abs(cg - c1.astype(np.int32))[diff] == 1).all()
+    assert layer.step == 1 and int(layer.changed.item()) == int((cg != c0).sum())
+
+
+def test_bitlinear_state_dict_resume():
+    from paper_2412_04787_gb300.bitlinear import DQTBitLinear
+    K, N = 128, 256
+    a = DQTBitLinear(K, N, bits=4, seed=5, tensor_id=1, init_seed=11)
+    b = DQTBitLinear(K, N, bits=4, seed=5, tensor_id=1, init_seed=12)  # different init
+    xs = [inputs.normal((64, K), 1.0, seed=20 + i, dtype=torch.bfloat16).cuda() for i in range(2)]
+    gs = [inputs.normal((64, N), 1e-2, seed=30 + i, dtype=torch.bfloat16).cuda() for i in range(2)]
+    a(xs[0].requires_grad_(True)).backward(gs[0])
+    buf = io.BytesIO()
+    torch.save(a.state_dict(), buf)
+    buf.seek(0)
+    b.load_state_dict(torch.load(buf, weights_only=False))
+    assert b.step == 1 and b.s_w == a.s_w
+    for layer in (a, b):
+        layer(xs[1].clone().requires_grad_(True)).backward(gs[1])
+    torch.cuda.synchronize()
+    for name in ("codes", "m", "v"):
+        assert torch.equal(getattr(a, name), getattr(b, name)), name
+
+
+def _train(bits_w, round_mode=0, steps=40):
+    from paper_2412_04787_gb300.decoder import DecoderConfig, DQTDecoder
+    torch.manual_seed(0)
+    cfg = DecoderConfig(layers=2, hidden=128, heads=4, ffn=256, vocab=512, bits=bits_w,
+                        lr=2e-3, seed=7)
+    model = DQTDecoder(cfg)
+    for m in model.bitlinear_layers():
+        m.round_mode = round_mode
+    opt = torch.optim.AdamW(model.dense_parameters(), lr=2e-3)
+    g = torch.Generator().manual_seed(3)
+    ids = torch.randint(0, cfg.vocab, (4, 65), generator=g).cuda()
+    codes0 = [m.codes.clone() for m in model.bitlinear_layers()]
+    losses = []
+    for _ in range(steps):
+        loss = model(ids[:, :-1], ids[:, 1:])
+        loss.backward()
+        opt.step()
+        opt.zero_grad(set_to_none=True)
+        losses.append(float(loss.detach()))
+    moved = sum(int((m.codes != c).sum()) for m, c in zip(model.bitlinear_layers(), codes0))
+    return losses, moved, model
+
+
+@pytest.mark.parametrize("bits_w", [1.58, 8])
+def test_decoder_trains_with_low_bit_weights(bits_w):
+    losses, moved, model = _train(bits_w)
+    assert all(np.isfinite(losses))
+    assert losses[-1] < 0.8 * losses[0], (losses[0], losses[-1])
+    assert moved > 0
+    for m in model.bitlinear_layers():
+        lo, hi = m.grid_tuple
+        c = m.codes
+        assert int(c.min()) >= lo and int(c.max()) <= hi
+
+
+def test_round_to_nearest_loses_small_updates():
+    """Ternary, lr * s_w < 1/2: |x - c| <= lr * s_w * |u| with |u| <= ~1 at
+    these steps, so rint(x) == c and no BitLinear code ever moves."""
+    losses, moved, model = _train(1.58, round_mode=1, steps=10)
+    assert max(m.lr * m.s_w for m in model.bitlinear_layers()) < 0.5
+    assert moved == 0
