@@ -662,7 +662,10 @@ def run_decoder(args):
     layer a DQT BitLinear (12 layers, hidden 768, 12 heads, FFN 2048, vocab
     32000, batch 16 x seq 1024, ternary; synthetic uniform token ids).  The
     BitLinear layers update themselves during backward; the bf16 embedding,
-    norms and head are stepped by torch AdamW inside the timed region."""
+    norms and head are stepped by torch AdamW inside the timed region.  By
+    default the whole step is captured once as a CUDA graph and replayed, the
+    per-step DQT constants (step, bias corrections, Philox counter) uploaded
+    from pinned memory before each replay; --no-graph runs it eagerly."""
     from paper_2412_04787_gb300 import build as dqt_build
     from paper_2412_04787_gb300.decoder import DecoderConfig, DQTDecoder
     dqt_build.build()
@@ -672,28 +675,59 @@ def run_decoder(args):
     cfg = DecoderConfig(layers=12, hidden=768, heads=12, ffn=2048, vocab=32000, bits=1.58,
                         lr=1e-3, seed=1234)
     model = DQTDecoder(cfg, device=dev)
-    opt = torch.optim.AdamW(model.dense_parameters(), lr=1e-3, fused=True)
+    use_graph = not args.no_graph
+    model.enable_graph_updates()
+    opt = torch.optim.AdamW(model.dense_parameters(), lr=1e-3, fused=True, capturable=use_graph)
     g = torch.Generator().manual_seed(5)
     host_ids = [torch.randint(0, cfg.vocab, (B, S + 1), generator=g).pin_memory() for _ in range(2)]
     ids_dev = [h.to(dev) for h in host_ids]
-    stream = torch.cuda.current_stream()
+    static_ids = ids_dev[0].clone()
+    state = {"loss": None, "i": 0}
 
-    def step(ids):
-        loss = model(ids[:, :-1], ids[:, 1:])
+    def fwd_bwd_opt():
+        loss = model(static_ids[:, :-1], static_ids[:, 1:])
         loss.backward()
         opt.step()
+        return loss
+
+    def run_step(src):
+        i = state["i"]
+        state["i"] += 1
+        static_ids.copy_(src, non_blocking=True)
+        model.prepare_step(i % 2)
+        model.upload_update_consts(i % 2)
+        if use_graph:
+            graph.replay()
+            return state["loss"]
+        loss = fwd_bwd_opt()
         opt.zero_grad(set_to_none=True)
         return loss
 
-    for i in range(args.warmup):
-        step(ids_dev[i % 2])
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for i in range(args.warmup):
+            static_ids.copy_(ids_dev[i % 2])
+            model.prepare_step(state["i"] % 2)
+            model.upload_update_consts(state["i"] % 2)
+            state["i"] += 1
+            fwd_bwd_opt()
+            opt.zero_grad(set_to_none=True)
+    torch.cuda.current_stream().wait_stream(side)
+    graph = None
+    if use_graph:
+        graph = torch.cuda.CUDAGraph()
+        opt.zero_grad(set_to_none=True)
+        with torch.cuda.graph(graph):
+            state["loss"] = fwd_bwd_opt()
+    stream = torch.cuda.current_stream()
     torch.cuda.synchronize()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     with ClockSampler(dev.index) as clk:
         t0.record(stream)
         for i in range(args.steps):
-            step(ids_dev[i % 2])
+            run_step(ids_dev[i % 2])
         t1.record(stream)
         torch.cuda.synchronize()
     ms = t0.elapsed_time(t1)
@@ -704,8 +738,7 @@ def run_decoder(args):
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for i in range(args.steps):
-        ids = host_ids[i % 2].to(dev, non_blocking=True)
-        loss = step(ids)
+        loss = run_step(host_ids[i % 2])
         loss_host.copy_(loss.detach(), non_blocking=True)
     e1.record(stream)
     torch.cuda.synchronize()
@@ -718,7 +751,7 @@ def run_decoder(args):
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic uniform token ids",
         "config": {"workload": "LLaMA-structured decoder, ternary DQT BitLinear in q,k,v,o,gate,up,down",
                    "layers": 12, "hidden": 768, "heads": 12, "ffn": 2048, "vocab": 32000,
-                   "batch": B, "seq": S},
+                   "batch": B, "seq": S, "cuda_graph": use_graph},
         "bitlinear_tflop_per_step": round(bl_flops / 1e12, 3),
         "e2e": {"value": round(tokens * args.steps / (e_ms / 1e3), 1), "unit": "tokens/s",
                 "h2d_bytes_per_step": int(host_ids[0].numel() * 8), "d2h_bytes_per_step": 4},
@@ -738,6 +771,7 @@ def main():
                          "codes_to_bf16, sr_update)")
     ap.add_argument("--numel", type=int, default=1 << 26, help="weights for --kernel sr_update")
     ap.add_argument("--shape", default=None, help="T,K,N for --kernel GEMMs (default 8192,2048,5632)")
+    ap.add_argument("--no-graph", action="store_true", help="decoder: run the step eagerly")
     ap.add_argument("--workload", default="mlp", choices=["mlp", "decoder"],
                     help="mlp: the headline BitLinear MLP GEMM set; decoder: a 12-layer DQT decoder step")
     args = ap.parse_args()

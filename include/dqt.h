@@ -183,7 +183,8 @@ int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, i
  *   m, v    <- AdamW moments (fp32 [N, K], in place)
  *   x       = c decay - (lr s_w) * m / (sqrt(v) k1 + k2)    (= W' * s_w, see dqt_adamw_t)
  *   c       <- Clip[SR(x), qmin, qmax]  (int8 [N, K], in place; round_mode 1: nearest)
- * The fp32 gradient never reaches memory unless dW_out (fp32 [N, K]) is given.
+ * The fp32 gradient never reaches memory unless dW_out (fp32 [N, K]) is given
+ * (or a split-T workspace is used, see dqt_bwd_dw_workspace_size).
  * With W, m and v all NULL only dW_out is written (gradient only).
  *   dY bf16 [T, N];  Xdq bf16 [T, K] from dqt_act_quant;  hp, sr: HOST structs.
  *   changed_out: device int64, or NULL; if given, the number of codes that changed
@@ -191,7 +192,19 @@ int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, i
 int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W, float s_w,
                                 float* m, float* v, const dqt_adamw_t* hp, const dqt_sr_t* sr,
                                 dqt_grid_t grid, int64_t T, int64_t N, int64_t K,
-                                float* dW_out, unsigned long long* changed_out, void* stream);
+                                float* dW_out, unsigned long long* changed_out, void* ws,
+                                size_t ws_bytes, void* stream);
+
+/* Workspace (bytes, 16-byte aligned device memory) that lets
+ * dqt_bitlinear_bwd_dw_update reduce a weight gradient whose output is too
+ * small to occupy the GPU (few 256 x 256 tiles, long token reduction) in
+ * token slices: each slice's fp32 partial is written to the workspace and one
+ * streaming pass sums the slices in slice order and applies the update.  0 =
+ * no split for this shape on the current device (and under
+ * dqt_set_gemm_tiles(1)).  Passing ws = NULL, or fewer bytes, always runs the
+ * single fused kernel.  The split gives the same update up to the fp32
+ * summation order of the gradient; it is deterministic for a given shape. */
+size_t dqt_bwd_dw_workspace_size(int64_t T, int64_t N, int64_t K);
 
 /* The AdamW + SR update of dqt_bitlinear_bwd_dw_update for a gradient already
  * in memory (Eq. 5 as a bandwidth-bound stream; 22 bytes per weight):
@@ -202,6 +215,28 @@ int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t*
 int dqt_sr_update(const float* grad, int8_t* W, float s_w, float* m, float* v,
                   const dqt_adamw_t* hp, const dqt_sr_t* sr, dqt_grid_t grid, int64_t numel,
                   unsigned long long* changed_out, void* stream);
+
+/* ---- update constants in device memory (CUDA-graph replay) ----------------
+ * The AdamW + SR update depends on the step (bias corrections, Philox counter).
+ * To replay a captured training step with a new step each time, the update
+ * can read its constants from device memory when the kernel runs:
+ *   dqt_update_consts derives, on the host, the block the update kernels use
+ *   (the constants listed at dqt_adamw_t, the grid, s_w and the SR key) into
+ *   `out` (host memory, at least dqt_update_consts_size() bytes); the caller
+ *   copies it to a 16-byte aligned device buffer ordered before the launch
+ *   (e.g. a cudaMemcpyAsync from pinned memory captured in the same graph).
+ * The _dev entry points are dqt_bitlinear_bwd_dw_update and dqt_sr_update
+ * with (hp, sr, grid, s_w) replaced by that device block; results are
+ * identical for identical constants.  W, m, v are required. */
+size_t dqt_update_consts_size(void);
+int dqt_update_consts(const dqt_adamw_t* hp, const dqt_sr_t* sr, dqt_grid_t grid, float s_w,
+                      void* out, size_t out_bytes);
+int dqt_bitlinear_bwd_dw_update_dev(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W, float* m,
+                                    float* v, const void* consts_dev, int64_t T, int64_t N,
+                                    int64_t K, float* dW_out, unsigned long long* changed_out,
+                                    void* ws, size_t ws_bytes, void* stream);
+int dqt_sr_update_dev(const float* grad, int8_t* W, float* m, float* v, const void* consts_dev,
+                      int64_t numel, unsigned long long* changed_out, void* stream);
 
 #ifdef __cplusplus
 }

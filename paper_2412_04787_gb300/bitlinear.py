@@ -100,6 +100,8 @@ class DQTBitLinear(torch.nn.Module):
         self.step = 0
         self.seed = int(seed)
         self.tensor_id = int(tensor_id)
+        # device-resident update constants (CUDA-graph replay), see prepare_step
+        self.uc_dev = None
         # anchor: a 0-element tensor that requires grad, so the layer's
         # backward (and with it the DQT update) runs even if x does not
         self._anchor = torch.nn.Parameter(torch.zeros(0, device=device), requires_grad=True)
@@ -117,11 +119,32 @@ class DQTBitLinear(torch.nn.Module):
     def forward(self, x):
         return _BitLinearFn.apply(x, self._anchor, self)
 
-    def _dqt_update(self, dy2, xdq):
-        self.step += 1
+    def _hyper(self, step):
         hp = dqt.adamw(lr=self.lr, beta1=self.betas[0], beta2=self.betas[1], eps=self.eps,
-                       weight_decay=self.weight_decay, step=self.step)
+                       weight_decay=self.weight_decay, step=step)
         sr = dqt.sr_stream(seed=self.seed, tensor_id=self.tensor_id, round_mode=self.round_mode)
+        return hp, sr
+
+    def use_device_consts(self, dev_row):
+        """Read the update constants from `dev_row` (a 64-byte row of a device
+        block) when the update kernel runs.  The step then advances in
+        prepare_step(), not in backward, so that a captured training step
+        replays with a new step each time."""
+        self.uc_dev = dev_row
+
+    def prepare_step(self, host_row):
+        """Advance the step and write its update constants into `host_row`."""
+        self.step += 1
+        hp, sr = self._hyper(self.step)
+        dqt.dqt_update_consts(hp, sr, self.grid_tuple, self.s_w, out=host_row)
+
+    def _dqt_update(self, dy2, xdq):
+        if self.uc_dev is not None:
+            dqt.dqt_bitlinear_bwd_dw_update_dev(dy2, xdq, self.codes, self.m, self.v, self.uc_dev,
+                                                changed_out=self.changed)
+            return
+        self.step += 1
+        hp, sr = self._hyper(self.step)
         dqt.dqt_bitlinear_bwd_dw_update(dy2, xdq, self.codes, self.s_w, self.m, self.v, hp, sr,
                                         self.grid_tuple, changed_out=self.changed)
 

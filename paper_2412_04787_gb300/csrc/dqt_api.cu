@@ -230,19 +230,30 @@ int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, i
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
+size_t dqt_bwd_dw_workspace_size(int64_t T, int64_t N, int64_t K) {
+  if (T <= 0 || N <= 0 || K <= 0 || T > kMaxDim || N > kMaxDim || K > kMaxDim) return 0;
+  if (dqt::gemm_mode() != 0) return 0;
+  const int s = dqt::dw_splits(static_cast<int>(N), static_cast<int>(K), static_cast<int>(T));
+  return s > 1 ? static_cast<size_t>(s) * static_cast<size_t>(N) * static_cast<size_t>(K) * 4u : 0;
+}
+
 int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W, float s_w,
                                 float* m, float* v, const dqt_adamw_t* hp, const dqt_sr_t* sr,
                                 dqt_grid_t grid, int64_t T, int64_t N, int64_t K, float* dW_out,
-                                unsigned long long* changed_out, void* stream) {
+                                unsigned long long* changed_out, void* ws, size_t ws_bytes,
+                                void* stream) {
   const bool upd = W || m || v;
   if (!dY || !Xdq || T <= 0 || N <= 0 || K <= 0) return DQT_ERR_ARG;
   if (upd && (!W || !m || !v)) return DQT_ERR_ARG;
   if (!upd && !dW_out) return DQT_ERR_ARG;
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
   if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(Xdq) || (W && !aligned16(W)) ||
-      (m && !aligned16(m)) || (v && !aligned16(v)) || (dW_out && !aligned16(dW_out)))
+      (m && !aligned16(m)) || (v && !aligned16(v)) || (dW_out && !aligned16(dW_out)) ||
+      (ws && !aligned16(ws)))
     return DQT_ERR_ALIGN;
   dqt::GemmLaunch g{};
+  g.ws = ws;
+  g.ws_bytes = ws ? ws_bytes : 0;
   if (upd) {
     const int rc = make_update_consts(hp, sr, grid, s_w, &g.uc);
     if (rc != DQT_OK) return rc;
@@ -269,7 +280,61 @@ int dqt_sr_update(const float* grad, int8_t* W, float s_w, float* m, float* v,
   dqt::UpdateConsts uc;
   const int rc = make_update_consts(hp, sr, grid, s_w, &uc);
   if (rc != DQT_OK) return rc;
-  return dqt::launch_sr_update(grad, W, m, v, numel, uc, changed_out, as_stream(stream))
+  return dqt::launch_sr_update(grad, W, m, v, numel, uc, nullptr, changed_out, as_stream(stream))
+             ? DQT_ERR_CUDA
+             : DQT_OK;
+}
+
+size_t dqt_update_consts_size(void) { return sizeof(dqt::UpdateConsts); }
+
+int dqt_update_consts(const dqt_adamw_t* hp, const dqt_sr_t* sr, dqt_grid_t grid, float s_w,
+                      void* out, size_t out_bytes) {
+  if (!out || out_bytes < sizeof(dqt::UpdateConsts)) return DQT_ERR_ARG;
+  dqt::UpdateConsts uc;
+  const int rc = make_update_consts(hp, sr, grid, s_w, &uc);
+  if (rc != DQT_OK) return rc;
+  memcpy(out, &uc, sizeof(uc));
+  return DQT_OK;
+}
+
+int dqt_bitlinear_bwd_dw_update_dev(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W, float* m,
+                                    float* v, const void* consts_dev, int64_t T, int64_t N,
+                                    int64_t K, float* dW_out, unsigned long long* changed_out,
+                                    void* ws, size_t ws_bytes, void* stream) {
+  if (!dY || !Xdq || !W || !m || !v || !consts_dev || T <= 0 || N <= 0 || K <= 0)
+    return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
+  if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(Xdq) || !aligned16(W) || !aligned16(m) ||
+      !aligned16(v) || !aligned16(consts_dev) || (dW_out && !aligned16(dW_out)) ||
+      (ws && !aligned16(ws)))
+    return DQT_ERR_ALIGN;
+  dqt::GemmLaunch g{};
+  g.ws = ws;
+  g.ws_bytes = ws ? ws_bytes : 0;
+  g.kind = dqt::GEMM_DW;
+  g.M = static_cast<int>(N);
+  g.N = static_cast<int>(K);
+  g.Kred = static_cast<int>(T);
+  g.A = dY;
+  g.B = Xdq;
+  g.W = W;
+  g.m = m;
+  g.v = v;
+  g.dW_out = dW_out;
+  g.changed = changed_out;
+  g.uc_dev = static_cast<const dqt::UpdateConsts*>(consts_dev);
+  return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
+int dqt_sr_update_dev(const float* grad, int8_t* W, float* m, float* v, const void* consts_dev,
+                      int64_t numel, unsigned long long* changed_out, void* stream) {
+  if (!grad || !W || !m || !v || !consts_dev || numel <= 0) return DQT_ERR_ARG;
+  if (!aligned16(grad) || !aligned16(W) || !aligned16(m) || !aligned16(v) || !aligned16(consts_dev))
+    return DQT_ERR_ALIGN;
+  dqt::UpdateConsts unused{};
+  return dqt::launch_sr_update(grad, W, m, v, numel, unused,
+                               static_cast<const dqt::UpdateConsts*>(consts_dev), changed_out,
+                               as_stream(stream))
              ? DQT_ERR_CUDA
              : DQT_OK;
 }

@@ -42,7 +42,24 @@ struct GemmLaunch {
   float* dW_out;  // DW, optional
   unsigned long long* changed;
   UpdateConsts uc;
+  const UpdateConsts* uc_dev;  // DW: read the update constants from device memory if set
+  void* ws;                    // DW: split-T workspace (fp32 slabs), or NULL
+  size_t ws_bytes;
 };
+
+// Token slices the 2-SM dW GEMM of an M x N output reduced over Kred uses
+// when given a workspace of dw_splits * M * N floats (1 = no split).
+int dw_splits(int M, int N, int Kred);
+
+// Sum `splits` fp32 slabs (stride `slab` elements) in slice order and apply
+// the update to W, m, v (numel elements); optionally write the sum to g_out.
+int launch_sr_update_slabs(const float* slabs, int splits, long long slab, int8_t* W, float* m,
+                           float* v, int64_t numel, const UpdateConsts& uc,
+                           const UpdateConsts* uc_dev, unsigned long long* changed, float* g_out,
+                           cudaStream_t stream);
+// Sum the slabs into out (gradient only).
+int launch_slab_sum(const float* slabs, int splits, long long slab, float* out,
+                    cudaStream_t stream);
 
 int launch_gemm(const GemmLaunch& g, cudaStream_t stream);
 
@@ -55,6 +72,7 @@ int launch_absmean_codes(const float* W0, int64_t numel, float s_w, int32_t qmin
 constexpr int kAbsmeanBlocks = 1024;
 
 int launch_sr_update(const float* grad, int8_t* W, float* m, float* v, int64_t numel,
-                     const UpdateConsts& uc, unsigned long long* changed, cudaStream_t stream);
+                     const UpdateConsts& uc, const UpdateConsts* uc_dev,
+                     unsigned long long* changed, cudaStream_t stream);
 
 }  // namespace dqt

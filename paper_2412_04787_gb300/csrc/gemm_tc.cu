@@ -33,6 +33,8 @@
 
 namespace dqt {
 
+static_assert(sizeof(UpdateConsts) <= 80, "update constants fit the shared barrier area");
+
 namespace {
 
 constexpr int BM = 128;
@@ -57,6 +59,12 @@ struct Params {
   float* dW_out;
   unsigned long long* changed;
   UpdateConsts uc;
+  const UpdateConsts* uc_dev;  // if set, the update constants are read from here at run time
+  // split-T (2-SM dW only): work unit t covers tile t / splits and the token
+  // slice of k-blocks [s * kb_per_split, ...), s = t % splits; its fp32
+  // partial goes to dW_out + s * slab
+  int splits, kb_per_split;
+  long long slab;
 };
 
 constexpr int kStageLd = 33;  // padded row pitch (floats) of the epilogue transpose buffer
@@ -72,6 +80,7 @@ struct Smem {
   static constexpr int BAR_OFF = XPOSE_OFF + XPOSE_BYTES;
   static constexpr int BYTES = BAR_OFF + 256 + 1024;  // + barriers + alignment slack
   static_assert(BYTES <= 232448, "shared memory per CTA");
+  static_assert((2 * kStages + 5) * 8 + 4 <= 128, "barrier area: barriers, then the update constants");
 };
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
@@ -173,7 +182,8 @@ __device__ __forceinline__ void dw_issue(const Params& p, int row0, int gn0, int
   }
 }
 
-__device__ __forceinline__ uint32_t dw_update(const Params& p, int row0, int gn0, int h, int lane,
+__device__ __forceinline__ uint32_t dw_update(const Params& p, const UpdateConsts& uc,
+                                              float* dw_out, int row0, int gn0, int h, int lane,
                                               const float* xp, DwLoads& L) {
   const int cq = (lane & 7) * 4;
   const int gk = gn0 + cq;
@@ -187,15 +197,15 @@ __device__ __forceinline__ uint32_t dw_update(const Params& p, int row0, int gn0
     const size_t e = static_cast<size_t>(gm) * p.N + gk;
     const float* src = xp + r * kStageLd + cq;
     const float4 g4 = make_float4(src[0], src[1], src[2], src[3]);
-    if (p.dW_out) __stcs(reinterpret_cast<float4*>(p.dW_out + e), g4);
+    if (dw_out) __stcs(reinterpret_cast<float4*>(dw_out + e), g4);
     if (!p.W) continue;
     uint4 w = make_uint4(0, 0, 0, 0);
-    if (p.uc.round_mode == 0)
-      w = sr_words(e >> 2, p.uc.step_lo, p.uc.tensor_id, p.uc.key0, p.uc.key1);
-    const int32_t n0c = dqt_update_elem(p.uc, g4.x, L.c[j].x, L.m[j].x, L.v[j].x, w.x);
-    const int32_t n1c = dqt_update_elem(p.uc, g4.y, L.c[j].y, L.m[j].y, L.v[j].y, w.y);
-    const int32_t n2c = dqt_update_elem(p.uc, g4.z, L.c[j].z, L.m[j].z, L.v[j].z, w.z);
-    const int32_t n3c = dqt_update_elem(p.uc, g4.w, L.c[j].w, L.m[j].w, L.v[j].w, w.w);
+    if (uc.round_mode == 0)
+      w = sr_words(e >> 2, uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
+    const int32_t n0c = dqt_update_elem(uc, g4.x, L.c[j].x, L.m[j].x, L.v[j].x, w.x);
+    const int32_t n1c = dqt_update_elem(uc, g4.y, L.c[j].y, L.m[j].y, L.v[j].y, w.y);
+    const int32_t n2c = dqt_update_elem(uc, g4.z, L.c[j].z, L.m[j].z, L.v[j].z, w.z);
+    const int32_t n3c = dqt_update_elem(uc, g4.w, L.c[j].w, L.m[j].w, L.v[j].w, w.w);
     n_changed += (n0c != L.c[j].x) + (n1c != L.c[j].y) + (n2c != L.c[j].z) + (n3c != L.c[j].w);
     __stcs(reinterpret_cast<char4*>(p.W + e),
            make_char4(static_cast<signed char>(n0c), static_cast<signed char>(n1c),
@@ -212,7 +222,8 @@ __device__ __forceinline__ uint32_t dw_update(const Params& p, int row0, int gn0
 // With PIPE the next half-chunk's loads are in flight while the current one
 // is updated (more registers, for kernels with few epilogue warps).
 template <bool PIPE>
-__device__ __forceinline__ uint32_t epi_dw_tile(const Params& p, int row0, int nbase, int nchunk,
+__device__ __forceinline__ uint32_t epi_dw_tile(const Params& p, const UpdateConsts& uc,
+                                                float* dw_out, int row0, int nbase, int nchunk,
                                                 uint32_t t_acc, float* xp, int lane) {
   uint32_t n_changed = 0;
   DwLoads A, B;
@@ -228,14 +239,14 @@ __device__ __forceinline__ uint32_t epi_dw_tile(const Params& p, int row0, int n
     __syncwarp();
     if (PIPE) {
       dw_issue(p, row0, gn0, 1, lane, B);
-      n_changed += dw_update(p, row0, gn0, 0, lane, xp, A);
+      n_changed += dw_update(p, uc, dw_out, row0, gn0, 0, lane, xp, A);
       if (cc + 1 < nchunk) dw_issue(p, row0, gn0 + 32, 0, lane, A);
-      n_changed += dw_update(p, row0, gn0, 1, lane, xp, B);
+      n_changed += dw_update(p, uc, dw_out, row0, gn0, 1, lane, xp, B);
     } else {
 #pragma unroll 1
       for (int h = 0; h < 2; ++h) {
         dw_issue(p, row0, gn0, h, lane, A);
-        n_changed += dw_update(p, row0, gn0, h, lane, xp, A);
+        n_changed += dw_update(p, uc, dw_out, row0, gn0, h, lane, xp, A);
       }
     }
     __syncwarp();  // the transpose buffer is rewritten for the next chunk
@@ -265,6 +276,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* acc_empty = acc_full + 2;    // [2]
   uint64_t* drain_bar = acc_empty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
+  // update constants, read by the dW epilogue from shared memory
+  UpdateConsts* uc_s = reinterpret_cast<UpdateConsts*>(smem + S::BAR_OFF + 128);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -280,6 +293,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&acc_empty[b], kEpiWarps);
     }
     mbar_init(drain_bar, 1);
+    if (EPI == GEMM_DW) *uc_s = p.uc_dev ? *p.uc_dev : p.uc;
     fence_mbarrier_init();
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
@@ -388,6 +402,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int row = quad * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     float* xp = reinterpret_cast<float*>(smem + S::XPOSE_OFF) + (warp - 2) * 32 * kStageLd;
+    const UpdateConsts& uc = *uc_s;
     uint32_t n_changed = 0;
     int u = 0;
     bool ok = true;
@@ -406,7 +421,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t t_run = tmem + lane_off + RUN_COL + static_cast<uint32_t>(half * HALF);
         const bool last = (c + 1 == nchunks);
         if (EPI == GEMM_DW) {
-          n_changed += epi_dw_tile<true>(p, gm - lane, nbase, HALF / 32, t_acc, xp, lane);
+          n_changed += epi_dw_tile<true>(p, uc, p.dW_out, gm - lane, nbase, HALF / 32, t_acc, xp, lane);
         } else
 #pragma unroll 1
         for (int cc = 0; cc < HALF / 32; ++cc) {
@@ -486,7 +501,7 @@ struct SmemPair {
   static constexpr int SLACK = (232448 - (BAR_OFF + 256)) < 1024 ? (232448 - (BAR_OFF + 256)) : 1024;
   static constexpr int BYTES = BAR_OFF + 256 + SLACK;
   static_assert(SLACK >= 0, "shared memory per CTA");
-  static_assert((2 * STAGES + 5) * 8 + 4 <= 256, "barrier area");
+  static_assert((2 * STAGES + 5) * 8 + 4 <= 176, "barrier area: barriers, then the update constants");
 };
 
 template <bool A_MN, bool B_MN, int EPI>
@@ -518,6 +533,8 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
   uint64_t* acc_empty = acc_full + 2;  // [2], used on the leader
   uint64_t* drain_bar = acc_empty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
+  // update constants, read by the dW epilogue from shared memory
+  UpdateConsts* uc_s = reinterpret_cast<UpdateConsts*>(smem + S::BAR_OFF + 176);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -536,6 +553,7 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
       mbar_init(&acc_empty[b], 2 * EW);
     }
     mbar_init(drain_bar, 1);
+    if (EPI == GEMM_DW) *uc_s = p.uc_dev ? *p.uc_dev : p.uc;
     fence_mbarrier_init();
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
@@ -555,9 +573,12 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
       int it = 0;
       bool ok = true;
       for (int t = cid; t < p.num_tiles && ok; t += ncl) {
-        const int m0 = (t / p.num_n) * 256 + static_cast<int>(rank) * 128;
-        const int n0 = (t % p.num_n) * BN + static_cast<int>(rank) * 128;
-        for (int kb = 0; kb < p.num_kb; ++kb, ++it) {
+        const int tile = t / p.splits;
+        const int kb0 = (t - tile * p.splits) * p.kb_per_split;
+        const int kb1 = min(p.num_kb, kb0 + p.kb_per_split);
+        const int m0 = (tile / p.num_n) * 256 + static_cast<int>(rank) * 128;
+        const int n0 = (tile % p.num_n) * BN + static_cast<int>(rank) * 128;
+        for (int kb = kb0; kb < kb1; ++kb, ++it) {
           const int s = it % ST;
           const uint32_t ph = (it / ST) & 1u;
           if (it >= ST && !mbar_wait_cl(&empty[s], ph ^ 1u, p.wait_ns)) {
@@ -599,9 +620,12 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
       int u = 0;
       bool ok = true;
       for (int t = cid; t < p.num_tiles && ok; t += ncl) {
-        for (int kb = 0; kb < p.num_kb; ++kb, ++it) {
+        const int tile = t / p.splits;
+        const int kb0 = (t - tile * p.splits) * p.kb_per_split;
+        const int kb1 = min(p.num_kb, kb0 + p.kb_per_split);
+        for (int kb = kb0; kb < kb1; ++kb, ++it) {
           const int b = u & 1;
-          if (kb == 0 && u >= 2) {
+          if (kb == kb0 && u >= 2) {
             if (!mbar_wait_cl(&acc_empty[b], ((u >> 1) - 1) & 1u, p.wait_ns)) {
               ok = false;
               break;
@@ -624,10 +648,10 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
                                      : sdesc_sw128(a_base + ks * 32, 16, 1024);
             const uint64_t bd = B_MN ? sdesc_sw128(b_base + ks * 2048, MN_CHUNK_BYTES, 1024)
                                      : sdesc_sw128(b_base + ks * 32, 16, 1024);
-            umma_bf16_pair(d, ad, bd, IDESC, (kb > 0 || ks > 0) ? 1u : 0u);
+            umma_bf16_pair(d, ad, bd, IDESC, (kb > kb0 || ks > 0) ? 1u : 0u);
           }
           umma_commit_pair_mc(&empty[s], 0x3);
-          if (kb == p.num_kb - 1) {
+          if (kb == kb1 - 1) {
             umma_commit_pair_mc(&acc_full[b], 0x3);
             ++u;
           }
@@ -644,12 +668,15 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
     const int row = quad * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     float* xp = reinterpret_cast<float*>(smem + S::XPOSE_OFF) + (warp - 2) * 32 * kStageLd;
+    const UpdateConsts& uc = *uc_s;
     uint32_t n_changed = 0;
     int u = 0;
     bool ok = true;
     for (int t = cid; t < p.num_tiles && ok; t += ncl, ++u) {
-      const int gm = (t / p.num_n) * 256 + static_cast<int>(rank) * 128 + row;
-      const int nbase = (t % p.num_n) * BN + half * HALF;
+      const int tile = t / p.splits;
+      float* dw_out = p.dW_out ? p.dW_out + (t - tile * p.splits) * p.slab : nullptr;
+      const int gm = (tile / p.num_n) * 256 + static_cast<int>(rank) * 128 + row;
+      const int nbase = (tile % p.num_n) * BN + half * HALF;
       const bool row_ok = gm < p.M;
       float a_t = 0.0f;
       if (EPI == GEMM_FWD && row_ok) a_t = __fdiv_rn(1.0f, __fmul_rn(p.s_x[gm], p.scale));
@@ -659,7 +686,7 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
       tc_fence_after();
       const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(b * BN + half * HALF);
       if (EPI == GEMM_DW) {
-        n_changed += epi_dw_tile<false>(p, gm - lane, nbase, HALF / 32, t_acc, xp, lane);
+        n_changed += epi_dw_tile<false>(p, uc, dw_out, gm - lane, nbase, HALF / 32, t_acc, xp, lane);
       } else
 #pragma unroll 1
       for (int cc = 0; cc < HALF / 32; ++cc) {
@@ -751,13 +778,37 @@ int launch_tiles(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStr
 }
 
 template <bool A_MN, bool B_MN, int EPI>
+int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream);
+
+}  // namespace
+
+// Token slices for a 2-SM dW GEMM whose output tiles would leave most SM
+// pairs idle: enough slices to give every pair a unit of work, each slice at
+// least 4 k-blocks (256 tokens) long, at most 32 slices.
+int dw_splits(int M, int N, int Kred) {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int pairs = sms / 2;
+  const long long tiles = static_cast<long long>((M + 255) / 256) * ((N + 255) / 256);
+  const int num_kb = (Kred + BK - 1) / BK;
+  if (tiles * 2 > pairs || num_kb < 8) return 1;
+  long long s = pairs / tiles;
+  if (s > num_kb / 4) s = num_kb / 4;
+  if (s > 32) s = 32;
+  return s < 2 ? 1 : static_cast<int>(s);
+}
+
+namespace {
+
+template <bool A_MN, bool B_MN, int EPI>
 int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream) {
   auto kern = gemm_pair_kernel<A_MN, B_MN, EPI>;
   const int smem = SmemPair<EPI>::BYTES;
   constexpr int threads = PairCfg<EPI>::THREADS;
   static int max_clusters = 0;  // per template instance
   p.num_n = (p.N + 255) / 256;
-  p.num_tiles = ((p.M + 255) / 256) * p.num_n;
+  p.num_tiles = ((p.M + 255) / 256) * p.num_n * p.splits;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -805,6 +856,17 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   GemmLaunch gl = g;
   gl.pair = !drain && gemm_mode() == 0;
   const GemmLaunch& g2 = gl;
+  p.splits = 1;
+  p.kb_per_split = p.num_kb;
+  p.slab = 0;
+  int splits = 1;
+  if (g.kind == GEMM_DW && g2.pair && g.ws)
+    splits = dw_splits(g.M, g.N, g.Kred);
+  if (splits > 1 && g.ws_bytes >= static_cast<size_t>(splits) * g.M * g.N * sizeof(float)) {
+    p.kb_per_split = (p.num_kb + splits - 1) / splits;
+    p.splits = (p.num_kb + p.kb_per_split - 1) / p.kb_per_split;
+    p.slab = static_cast<long long>(g.M) * g.N;
+  }
   p.wait_ns = wait_limit_ns();
   p.status = status_word();
   if (!p.status) return 3;
@@ -818,6 +880,7 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   p.dW_out = g.dW_out;
   p.changed = g.changed;
   p.uc = g.uc;
+  p.uc_dev = g.uc_dev;
 
   CUtensorMap ta, tb;
   switch (g.kind) {
@@ -835,11 +898,31 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
       if (!make_map(&tb, g.B, g.N, g.Kred, 64, BK)) return 3;
       if (g2.pair) return launch_pairs<false, true, GEMM_DX>(ta, tb, p, stream);
       return launch_tiles<256, false, true, GEMM_DX, false>(ta, tb, p, stream);
-    case GEMM_DW:
+    case GEMM_DW: {
       if (!make_map(&ta, g.A, g.M, g.Kred, 64, BK)) return 3;
       if (!make_map(&tb, g.B, g.N, g.Kred, 64, BK)) return 3;
-      if (g2.pair) return launch_pairs<true, true, GEMM_DW>(ta, tb, p, stream);
-      return launch_tiles<256, true, true, GEMM_DW, false>(ta, tb, p, stream);
+      if (!g2.pair) return launch_tiles<256, true, true, GEMM_DW, false>(ta, tb, p, stream);
+      if (p.splits == 1) return launch_pairs<true, true, GEMM_DW>(ta, tb, p, stream);
+      // split-T: fp32 partials of each token slice into the workspace slabs,
+      // then one streaming pass sums the slabs in slice order and applies the
+      // AdamW + stochastic-rounding update (and writes the summed gradient to
+      // dW_out if asked for)
+      Params ps = p;
+      ps.W = nullptr;
+      ps.m = nullptr;
+      ps.v = nullptr;
+      ps.changed = nullptr;
+      ps.dW_out = static_cast<float*>(g.ws);
+      const int rc = launch_pairs<true, true, GEMM_DW>(ta, tb, ps, stream);
+      if (rc) return rc;
+      if (!g.W) {
+        // gradient only: sum the slabs into dW_out
+        return launch_slab_sum(static_cast<const float*>(g.ws), p.splits, p.slab, g.dW_out,
+                               stream);
+      }
+      return launch_sr_update_slabs(static_cast<const float*>(g.ws), p.splits, p.slab, g.W, g.m,
+                                    g.v, p.slab, g.uc, g.uc_dev, g.changed, g.dW_out, stream);
+    }
   }
   return 1;
 }

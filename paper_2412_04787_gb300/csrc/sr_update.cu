@@ -13,17 +13,43 @@ namespace {
 
 constexpr int kThreads = 256;
 
+// The gradient of element e is grad[e], or, with nsplit > 1 partial slabs of
+// `slab` elements each (a split-T weight gradient), their sum taken in slab
+// order; g_out (optional) receives that gradient.
+__device__ __forceinline__ float4 slab_grad4(const float* __restrict__ grad, int nsplit,
+                                             long long slab, int64_t e) {
+  float4 g4 = __ldcs(reinterpret_cast<const float4*>(grad + e));
+  for (int s = 1; s < nsplit; ++s) {
+    const float4 h = __ldcs(reinterpret_cast<const float4*>(grad + s * slab + e));
+    g4.x = __fadd_rn(g4.x, h.x);
+    g4.y = __fadd_rn(g4.y, h.y);
+    g4.z = __fadd_rn(g4.z, h.z);
+    g4.w = __fadd_rn(g4.w, h.w);
+  }
+  return g4;
+}
+
+__device__ __forceinline__ float slab_grad1(const float* __restrict__ grad, int nsplit,
+                                            long long slab, int64_t e) {
+  float g = grad[e];
+  for (int s = 1; s < nsplit; ++s) g = __fadd_rn(g, grad[s * slab + e]);
+  return g;
+}
+
 __global__ void __launch_bounds__(kThreads)
-    sr_update_kernel(const float* __restrict__ grad, int8_t* __restrict__ W,
-                     float* __restrict__ m, float* __restrict__ v, int64_t numel,
-                     const UpdateConsts uc, unsigned long long* changed) {
+    sr_update_kernel(const float* __restrict__ grad, int nsplit, long long slab,
+                     float* __restrict__ g_out, int8_t* __restrict__ W, float* __restrict__ m,
+                     float* __restrict__ v, int64_t numel, const UpdateConsts uc_arg,
+                     const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed) {
+  const UpdateConsts uc = uc_dev ? *uc_dev : uc_arg;
   const int64_t ngroups = numel >> 2;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * kThreads;
   uint32_t n_changed = 0;
   for (int64_t gi = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; gi < ngroups;
        gi += stride) {
     const int64_t e = gi << 2;
-    const float4 g4 = __ldcs(reinterpret_cast<const float4*>(grad + e));
+    const float4 g4 = slab_grad4(grad, nsplit, slab, e);
+    if (g_out) __stcs(reinterpret_cast<float4*>(g_out + e), g4);
     float4 m4 = __ldcs(reinterpret_cast<const float4*>(m + e));
     float4 v4 = __ldcs(reinterpret_cast<const float4*>(v + e));
     const char4 c4 = *reinterpret_cast<const char4*>(W + e);
@@ -49,7 +75,9 @@ __global__ void __launch_bounds__(kThreads)
     for (int64_t e = gi << 2; e < numel; ++e) {
       float mm = m[e], vv = v[e];
       const int32_t c0 = W[e];
-      const int32_t r = dqt_update_elem(uc, grad[e], c0, mm, vv, ws[e & 3]);
+      const float g = slab_grad1(grad, nsplit, slab, e);
+      if (g_out) g_out[e] = g;
+      const int32_t r = dqt_update_elem(uc, g, c0, mm, vv, ws[e & 3]);
       n_changed += (r != c0);
       W[e] = static_cast<int8_t>(r);
       m[e] = mm;
@@ -64,10 +92,19 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
-}  // namespace
+__global__ void __launch_bounds__(kThreads)
+    slab_sum_kernel(const float* __restrict__ slabs, int nsplit, long long slab,
+                    float* __restrict__ out) {
+  const int64_t ngroups = slab >> 2;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * kThreads;
+  for (int64_t gi = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; gi < ngroups;
+       gi += stride)
+    __stcs(reinterpret_cast<float4*>(out + (gi << 2)), slab_grad4(slabs, nsplit, slab, gi << 2));
+  if (blockIdx.x == 0 && threadIdx.x == 0)
+    for (int64_t e = ngroups << 2; e < slab; ++e) out[e] = slab_grad1(slabs, nsplit, slab, e);
+}
 
-int launch_sr_update(const float* grad, int8_t* W, float* m, float* v, int64_t numel,
-                     const UpdateConsts& uc, unsigned long long* changed, cudaStream_t stream) {
+int stream_blocks(int64_t numel) {
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -76,8 +113,31 @@ int launch_sr_update(const float* grad, int8_t* W, float* m, float* v, int64_t n
   const int64_t cap = static_cast<int64_t>(sms) * 8;  // 8 resident 256-thread blocks per SM
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
-  sr_update_kernel<<<static_cast<int>(blocks), kThreads, 0, stream>>>(grad, W, m, v, numel, uc,
-                                                                      changed);
+  return static_cast<int>(blocks);
+}
+
+}  // namespace
+
+int launch_sr_update_slabs(const float* slabs, int splits, long long slab, int8_t* W, float* m,
+                           float* v, int64_t numel, const UpdateConsts& uc,
+                           const UpdateConsts* uc_dev, unsigned long long* changed, float* g_out,
+                           cudaStream_t stream) {
+  sr_update_kernel<<<stream_blocks(numel), kThreads, 0, stream>>>(slabs, splits, slab, g_out, W, m,
+                                                                  v, numel, uc, uc_dev, changed);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+int launch_slab_sum(const float* slabs, int splits, long long slab, float* out,
+                    cudaStream_t stream) {
+  slab_sum_kernel<<<stream_blocks(slab), kThreads, 0, stream>>>(slabs, splits, slab, out);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+int launch_sr_update(const float* grad, int8_t* W, float* m, float* v, int64_t numel,
+                     const UpdateConsts& uc, const UpdateConsts* uc_dev,
+                     unsigned long long* changed, cudaStream_t stream) {
+  sr_update_kernel<<<stream_blocks(numel), kThreads, 0, stream>>>(grad, 1, 0, nullptr, W, m, v,
+                                                                  numel, uc, uc_dev, changed);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 

@@ -13,7 +13,10 @@ cross-entropy loss are PyTorch operations around the BitLinear hot path.
 A training step is ``loss = model(ids, targets); loss.backward();
 opt.step(); opt.zero_grad()``: each BitLinear applies its DQT update during
 its own backward, the optimiser only sees the bf16 parameters
-(``model.dense_parameters()``).
+(``model.dense_parameters()``).  For CUDA-graph replay of whole steps,
+``enable_graph_updates()`` moves the per-step update constants to device
+memory (``prepare_step(slot)`` on the host, ``upload_update_consts(slot)``
+stream-ordered before each replay).
 """
 
 import torch
@@ -101,6 +104,37 @@ class DQTDecoder(torch.nn.Module):
 
     def bitlinear_layers(self):
         return [m for m in self.modules() if isinstance(m, DQTBitLinear)]
+
+    # ---- CUDA-graph replay of whole training steps ----
+    def enable_graph_updates(self):
+        """Move the per-step update constants of every BitLinear to one device
+        block (64-byte rows) fed from two pinned host blocks.  Per step:
+        prepare_step(slot) fills host block `slot` on the host, then
+        upload_update_consts(slot) copies it, stream-ordered, ahead of the
+        step's kernels (e.g. right before replaying a captured step).  Alternate
+        the slots so the host never rewrites a block a pending copy reads."""
+        from . import dqt
+        layers = self.bitlinear_layers()
+        row = (dqt.lib().dqt_update_consts_size() + 63) // 64 * 64
+        dev = layers[0].codes.device
+        self._uc_host = torch.zeros((2, len(layers), row), dtype=torch.uint8).pin_memory()
+        self._uc_dev = torch.zeros((len(layers), row), dtype=torch.uint8, device=dev)
+        self._uc_copied = [None, None]
+        for i, layer in enumerate(layers):
+            layer.use_device_consts(self._uc_dev[i])
+
+    def prepare_step(self, slot=0):
+        ev = self._uc_copied[slot]
+        if ev is not None:
+            ev.synchronize()  # the copy that last read this host block is done
+        for i, layer in enumerate(self.bitlinear_layers()):
+            layer.prepare_step(self._uc_host[slot, i])
+
+    def upload_update_consts(self, slot=0):
+        self._uc_dev.copy_(self._uc_host[slot], non_blocking=True)
+        ev = torch.cuda.Event()
+        ev.record()
+        self._uc_copied[slot] = ev
 
     def dense_parameters(self):
         """The bf16 parameters an ordinary optimiser trains (not the BitLinear codes)."""

@@ -21,7 +21,8 @@ EXPORTED = [
     "dqt_set_wait_limit_ns", "dqt_absmean_workspace_size", "dqt_absmean_init",
     "dqt_act_quant", "dqt_codes_to_bf16", "dqt_bitlinear_fwd", "dqt_bitlinear_bwd_dx",
     "dqt_bitlinear_bwd_dw_update", "dqt_sr_update", "dqt_absmean_init_noalloc",
-    "dqt_set_gemm_tiles",
+    "dqt_set_gemm_tiles", "dqt_update_consts_size", "dqt_update_consts",
+    "dqt_bitlinear_bwd_dw_update_dev", "dqt_sr_update_dev", "dqt_bwd_dw_workspace_size",
 ]
 
 
@@ -74,11 +75,22 @@ def lib():
         L.dqt_bitlinear_bwd_dx.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp]
         L.dqt_bitlinear_bwd_dw_update.argtypes = [_vp, _vp, _vp, _f32, _vp, _vp,
                                                   C.POINTER(dqt_adamw_t), C.POINTER(dqt_sr_t),
-                                                  dqt_grid_t, _i64, _i64, _i64, _vp, _vp, _vp]
+                                                  dqt_grid_t, _i64, _i64, _i64, _vp, _vp, _vp,
+                                                  _sz, _vp]
+        L.dqt_bwd_dw_workspace_size.argtypes = [_i64, _i64, _i64]
+        L.dqt_bwd_dw_workspace_size.restype = _sz
         L.dqt_sr_update.argtypes = [_vp, _vp, _f32, _vp, _vp, C.POINTER(dqt_adamw_t),
                                     C.POINTER(dqt_sr_t), dqt_grid_t, _i64, _vp, _vp]
+        L.dqt_update_consts_size.argtypes = []
+        L.dqt_update_consts_size.restype = _sz
+        L.dqt_update_consts.argtypes = [C.POINTER(dqt_adamw_t), C.POINTER(dqt_sr_t), dqt_grid_t,
+                                        _f32, _vp, _sz]
+        L.dqt_bitlinear_bwd_dw_update_dev.argtypes = [_vp, _vp, _vp, _vp, _vp, _vp, _i64, _i64,
+                                                      _i64, _vp, _vp, _vp, _sz, _vp]
+        L.dqt_sr_update_dev.argtypes = [_vp, _vp, _vp, _vp, _vp, _i64, _vp, _vp]
         for name in EXPORTED:
-            if name not in ("dqt_status_string", "dqt_absmean_workspace_size"):
+            if name not in ("dqt_status_string", "dqt_absmean_workspace_size",
+                            "dqt_update_consts_size", "dqt_bwd_dw_workspace_size"):
                 getattr(L, name).restype = C.c_int
         _lib = L
     return _lib
@@ -236,10 +248,28 @@ def dqt_bitlinear_bwd_dx(dY, W_img, s_w, dX=None, stream=None):
     return dX
 
 
+def _dw_workspace(T, N, K, device, ws):
+    if ws is False:
+        return None, 0
+    need = lib().dqt_bwd_dw_workspace_size(T, N, K)
+    if need == 0:
+        return None, 0
+    if ws is None:
+        ws = torch.empty(need, dtype=torch.uint8, device=device)
+    _need(ws, "ws", torch.uint8)
+    return ws, ws.numel()
+
+
+def dqt_bwd_dw_workspace_size(T, N, K):
+    return int(lib().dqt_bwd_dw_workspace_size(T, N, K))
+
+
 def dqt_bitlinear_bwd_dw_update(dY, Xdq, W, s_w, m, v, hp, sr, bits_or_grid, dW_out=None,
-                                changed_out=None, stream=None):
+                                changed_out=None, ws=None, stream=None):
     """Fused dW GEMM + AdamW + stochastic rounding; W, m, v updated in place.
-    With W = m = v = None only dW_out is computed."""
+    With W = m = v = None only dW_out is computed.  `ws`: split-T workspace
+    (uint8 CUDA tensor of dqt_bwd_dw_workspace_size bytes); None allocates it
+    when the shape benefits, False forces the single fused kernel."""
     _need(dY, "dY", torch.bfloat16)
     T, N = dY.shape
     _need(Xdq, "Xdq", torch.bfloat16)
@@ -250,11 +280,12 @@ def dqt_bitlinear_bwd_dw_update(dY, Xdq, W, s_w, m, v, hp, sr, bits_or_grid, dW_
     _opt(v, "v", torch.float32, (N, K))
     _opt(dW_out, "dW_out", torch.float32, (N, K))
     _opt(changed_out, "changed_out", torch.int64, (1,))
+    ws, nws = _dw_workspace(T, N, K, dY.device, ws)
     _check(lib().dqt_bitlinear_bwd_dw_update(
         _ptr(dY), _ptr(Xdq), _ptr(W), float(s_w), _ptr(m), _ptr(v),
         C.byref(hp) if hp is not None else None, C.byref(sr) if sr is not None else None,
-        _grid(bits_or_grid), T, N, K, _ptr(dW_out), _ptr(changed_out), _stream(stream)),
-        "dqt_bitlinear_bwd_dw_update")
+        _grid(bits_or_grid), T, N, K, _ptr(dW_out), _ptr(changed_out), _ptr(ws), nws,
+        _stream(stream)), "dqt_bitlinear_bwd_dw_update")
     return W
 
 
@@ -270,4 +301,53 @@ def dqt_sr_update(grad, W, s_w, m, v, hp, sr, bits_or_grid, changed_out=None, st
     _check(lib().dqt_sr_update(_ptr(grad), _ptr(W), float(s_w), _ptr(m), _ptr(v), C.byref(hp),
                                C.byref(sr), _grid(bits_or_grid), n, _ptr(changed_out),
                                _stream(stream)), "dqt_sr_update")
+    return W
+
+
+def dqt_update_consts(hp, sr, bits_or_grid, s_w, out=None):
+    """Host block of update constants (a uint8 tensor, pinned if `out` is None)."""
+    n = lib().dqt_update_consts_size()
+    if out is None:
+        out = torch.empty(n, dtype=torch.uint8).pin_memory()
+    if out.device.type != "cpu" or out.numel() < n or not out.is_contiguous():
+        raise ValueError("out must be a contiguous host uint8 tensor of >= %d bytes" % n)
+    _check(lib().dqt_update_consts(C.byref(hp), C.byref(sr), _grid(bits_or_grid), float(s_w),
+                                   C.c_void_p(out.data_ptr()), out.numel()), "dqt_update_consts")
+    return out
+
+
+def dqt_bitlinear_bwd_dw_update_dev(dY, Xdq, W, m, v, consts_dev, dW_out=None, changed_out=None,
+                                    ws=None, stream=None):
+    """As dqt_bitlinear_bwd_dw_update with the update constants read from the
+    device block `consts_dev` (uint8 CUDA tensor) when the kernel runs."""
+    _need(dY, "dY", torch.bfloat16)
+    T, N = dY.shape
+    _need(Xdq, "Xdq", torch.bfloat16)
+    K = Xdq.shape[1]
+    _need(Xdq, "Xdq", torch.bfloat16, (T, K))
+    _need(W, "W", torch.int8, (N, K))
+    _need(m, "m", torch.float32, (N, K))
+    _need(v, "v", torch.float32, (N, K))
+    _need(consts_dev, "consts_dev", torch.uint8)
+    _opt(dW_out, "dW_out", torch.float32, (N, K))
+    _opt(changed_out, "changed_out", torch.int64, (1,))
+    ws, nws = _dw_workspace(T, N, K, dY.device, ws)
+    _check(lib().dqt_bitlinear_bwd_dw_update_dev(
+        _ptr(dY), _ptr(Xdq), _ptr(W), _ptr(m), _ptr(v), _ptr(consts_dev), T, N, K, _ptr(dW_out),
+        _ptr(changed_out), _ptr(ws), nws, _stream(stream)), "dqt_bitlinear_bwd_dw_update_dev")
+    return W
+
+
+def dqt_sr_update_dev(grad, W, m, v, consts_dev, changed_out=None, stream=None):
+    _need(grad, "grad", torch.float32)
+    n = grad.numel()
+    _need(W, "W", torch.int8)
+    _need(m, "m", torch.float32)
+    _need(v, "v", torch.float32)
+    _need(consts_dev, "consts_dev", torch.uint8)
+    if W.numel() != n or m.numel() != n or v.numel() != n:
+        raise ValueError("grad, W, m, v must have the same number of elements")
+    _opt(changed_out, "changed_out", torch.int64, (1,))
+    _check(lib().dqt_sr_update_dev(_ptr(grad), _ptr(W), _ptr(m), _ptr(v), _ptr(consts_dev), n,
+                                   _ptr(changed_out), _stream(stream)), "dqt_sr_update_dev")
     return W

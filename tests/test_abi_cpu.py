@@ -90,9 +90,9 @@ def test_update_argument_validation(L):
     sr = dqt.sr_stream()
     ok = C.byref(hp), C.byref(sr)
     # partial state
-    assert L.dqt_bitlinear_bwd_dw_update(A, A, A, 1.0, None, A, *ok, g, 4, 8, 8, None, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_bwd_dw_update(A, A, A, 1.0, None, A, *ok, g, 4, 8, 8, None, None, None, 0, None) == dqt.DQT_ERR_ARG
     # gradient-only mode needs dW_out
-    assert L.dqt_bitlinear_bwd_dw_update(A, A, None, 1.0, None, None, *ok, g, 4, 8, 8, None, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_bwd_dw_update(A, A, None, 1.0, None, None, *ok, g, 4, 8, 8, None, None, None, 0, None) == dqt.DQT_ERR_ARG
     bad = dqt.adamw(step=0)
     assert L.dqt_sr_update(A, A, 1.0, A, A, C.byref(bad), C.byref(sr), g, 16, None, None) == dqt.DQT_ERR_ARG
     bad = dqt.adamw(beta1=1.0)

@@ -131,3 +131,86 @@ def test_round_to_nearest_loses_small_updates():
     losses, moved, model = _train(1.58, round_mode=1, steps=10)
     assert max(m.lr * m.s_w for m in model.bitlinear_layers()) < 0.5
     assert moved == 0
+
+
+def test_device_consts_update_matches_host_path():
+    """The _dev entry points with the constants block in device memory give
+    exactly the host-constant path's codes and moments (fused and standalone)."""
+    from paper_2412_04787_gb300 import dqt
+    T, K, N = 256, 264, 520
+    qmin, qmax = oracle.grid(8)
+    c0, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=3).numpy(), qmin, qmax)
+    X = inputs.normal((T, K), 1.0, seed=4, dtype=torch.bfloat16).cuda()
+    dY = inputs.normal((T, N), 1e-2, seed=5, dtype=torch.bfloat16).cuda()
+    _, s_x, _, xdq = dqt.dqt_act_quant(X, want=("Xdq",))
+    hp = dqt.adamw(lr=1e-3, weight_decay=0.01, step=3)
+    sr = dqt.sr_stream(seed=11, tensor_id=2)
+    blk = dqt.dqt_update_consts(hp, sr, (qmin, qmax), float(s_w))
+    dev = blk.cuda()
+    m0 = inputs.normal((N, K), 1e-4, seed=6).cuda()
+    v0 = inputs.normal((N, K), 1e-4, seed=7).square().cuda()
+    a = [torch.from_numpy(c0).cuda(), m0.clone(), v0.clone()]
+    b = [torch.from_numpy(c0).cuda(), m0.clone(), v0.clone()]
+    dqt.dqt_bitlinear_bwd_dw_update(dY, xdq, a[0], float(s_w), a[1], a[2], hp, sr, (qmin, qmax))
+    dqt.dqt_bitlinear_bwd_dw_update_dev(dY, xdq, b[0], b[1], b[2], dev)
+    g = inputs.normal((N * K,), 1e-3, seed=8).cuda()
+    dqt.dqt_sr_update(g, a[0].view(-1), float(s_w), a[1].view(-1), a[2].view(-1), hp, sr, (qmin, qmax))
+    dqt.dqt_sr_update_dev(g, b[0].view(-1), b[1].view(-1), b[2].view(-1), dev)
+    dqt.dqt_check_device_status()
+    for x, y in zip(a, b):
+        assert torch.equal(x, y)
+
+
+def test_graph_replayed_decoder_equals_eager():
+    """Whole training steps captured once in a CUDA graph and replayed with a
+    new step each time (constants uploaded from the pinned block) leave the
+    model in exactly the state eager steps do."""
+    from paper_2412_04787_gb300.decoder import DecoderConfig, DQTDecoder
+
+    def make():
+        cfg = DecoderConfig(layers=2, hidden=128, heads=4, ffn=256, vocab=512, bits=1.58,
+                            lr=2e-3, seed=9)
+        model = DQTDecoder(cfg)
+        model.enable_graph_updates()
+        opt = torch.optim.AdamW(model.dense_parameters(), lr=2e-3, capturable=True)
+        return model, opt
+
+    g = torch.Generator().manual_seed(4)
+    batches = [torch.randint(0, 512, (4, 65), generator=g).cuda() for _ in range(6)]
+
+    def eager_step(model, opt, ids, slot):
+        model.prepare_step(slot)
+        model.upload_update_consts(slot)
+        loss = model(ids[:, :-1], ids[:, 1:])
+        loss.backward()
+        opt.step()
+        opt.zero_grad(set_to_none=True)
+
+    ea, oa = make()
+    for i, ids in enumerate(batches):
+        eager_step(ea, oa, ids, i % 2)
+
+    gb, ob = make()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for i, ids in enumerate(batches[:2]):
+            eager_step(gb, ob, ids, i % 2)
+    torch.cuda.current_stream().wait_stream(side)
+    static_ids = batches[2].clone()
+    graph = torch.cuda.CUDAGraph()
+    ob.zero_grad(set_to_none=True)
+    with torch.cuda.graph(graph):
+        loss = gb(static_ids[:, :-1], static_ids[:, 1:])
+        loss.backward()
+        ob.step()
+    for i, ids in enumerate(batches[2:], start=2):
+        static_ids.copy_(ids)
+        gb.prepare_step(i % 2)
+        gb.upload_update_consts(i % 2)
+        graph.replay()
+    torch.cuda.synchronize()
+    for la, lb in zip(ea.bitlinear_layers(), gb.bitlinear_layers()):
+        assert la.step == lb.step == 6
+        assert torch.equal(la.codes, lb.codes)
+        assert torch.equal(la.m, lb.m) and torch.equal(la.v, lb.v)

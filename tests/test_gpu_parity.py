@@ -371,8 +371,9 @@ def test_tilings_bit_identical():
             Y = dqt.dqt_bitlinear_fwd(q_img, s_x, W_img, s_w, g)
             dX = dqt.dqt_bitlinear_bwd_dx(dY.cuda(), W_img, s_w)
             dW = torch.empty((776, 512), dtype=torch.float32, device="cuda")
+            # unsplit on both tilings (the split-T path sums in another order)
             dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), xdq, None, s_w, None, None, None, None, g,
-                                            dW_out=dW)
+                                            dW_out=dW, ws=False)
             dqt.dqt_check_device_status()
             outs.append((Y.cpu(), dX.cpu(), dW.cpu()))
         finally:
@@ -380,3 +381,59 @@ def test_tilings_bit_identical():
     assert torch.equal(outs[0][0], outs[1][0])
     assert torch.equal(outs[0][1], outs[1][1])
     assert torch.equal(outs[0][2], outs[1][2])
+
+
+# ---------------------------------------------------------------------------
+# split-T weight gradient (small outputs, long token reductions)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("T,K,N,bits_w", [(8192, 256, 256, 1.58), (2048, 264, 520, 8),
+                                           (4096, 768, 768, 4)])
+def test_split_t_dw_update(T, K, N, bits_w):
+    assert dqt.dqt_bwd_dw_workspace_size(T, N, K) > 0  # the shape takes the split path
+    X, dY, W0, c, s_w, g = problem(T, K, N, bits_w, seed=T + N)
+    qmin, qmax = g
+    m = inputs.normal((N, K), 1e-4, seed=T + 5)
+    v = inputs.normal((N, K), 1e-4, seed=T + 6).square()
+    hp = dqt.adamw(lr=1e-3, step=2)
+    sr = dqt.sr_stream(seed=1234, tensor_id=6)
+    _, s_x, _, Xdq = dqt.dqt_act_quant(X.cuda(), want=("Xdq",))
+    Wg, mg, vg = torch.from_numpy(c).cuda(), m.clone().cuda(), v.clone().cuda()
+    dW = torch.empty((N, K), dtype=torch.float32, device="cuda")
+    dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), Xdq, Wg, s_w, mg, vg, hp, sr, g, dW_out=dW)
+    dW2 = torch.empty((N, K), dtype=torch.float32, device="cuda")
+    dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=dW2)
+    dqt.dqt_check_device_status()
+    assert torch.equal(dW, dW2)  # the gradient-only split path sums the same slabs
+    q, s, _, xd = oracle.act_quant(bits(X))
+    gref = oracle.bwd_dw_bf16x(bits(dY), xd)
+    assert elem_err(dW.cpu().numpy(), gref) <= REL_TOL
+    assert rel_err(dW.cpu().numpy(), oracle.bwd_dw(bits(dY), q, s)) <= REL_TOL
+    k = oracle.adamw_consts(hp.lr, hp.beta1, hp.beta2, hp.eps, hp.weight_decay, 2, s_w)
+    c1, m1, v1, _ = oracle.update(gref.astype(np.float32), c, m.numpy(), v.numpy(), k, qmin, qmax,
+                                  1234, 2, 6, 0)
+    cg = Wg.cpu().numpy().astype(np.int32)
+    diff = cg != c1.astype(np.int32)
+    assert diff.mean() <= 1e-4 + 1.0 / diff.size, diff.sum()
+    assert (np.abs(cg - c1.astype(np.int32))[diff] == 1).all()
+    assert np.abs(mg.cpu().numpy() - m1).max() <= 1e-3 * np.abs(m1).max()
+    assert np.abs(vg.cpu().numpy() - v1).max() <= 1e-3 * np.abs(v1).max()
+    # and the standalone update on the split path's own summed gradient is the
+    # same update, bit for bit
+    W3, m3, v3 = torch.from_numpy(c).cuda(), m.clone().cuda(), v.clone().cuda()
+    dqt.dqt_sr_update(dW.view(-1), W3.view(-1), s_w, m3.view(-1), v3.view(-1), hp, sr, g)
+    dqt.dqt_check_device_status()
+    assert torch.equal(W3, Wg) and torch.equal(m3, mg) and torch.equal(v3, vg)
+
+
+def test_split_t_matches_unsplit_within_tolerance():
+    T, K, N = 8192, 256, 512
+    X, dY, W0, c, s_w, g = problem(T, K, N, 1.58, seed=77)
+    _, s_x, _, Xdq = dqt.dqt_act_quant(X.cuda(), want=("Xdq",))
+    a = torch.empty((N, K), dtype=torch.float32, device="cuda")
+    b = torch.empty((N, K), dtype=torch.float32, device="cuda")
+    dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=a)
+    dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=b,
+                                    ws=False)
+    dqt.dqt_check_device_status()
+    # fp32 summation order only (a wrong token slice would be an O(1) error)
+    assert elem_err(a.cpu().numpy(), b.cpu().double().numpy()) <= 2e-3
