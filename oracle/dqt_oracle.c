@@ -19,6 +19,8 @@
  *   Sec 4.1 AdamW producing the dense target W'           -> dqt_oracle_adamw_x
  *   Eq. 5   W_hat = SR(W'), kept on the n-bit grid        -> dqt_oracle_update
  *   Sec 5.1 absmax / round-to-nearest ablation            -> round_mode = 1
+ *   Sec 4.1/4.3 FP8 environment: E4M3 activations and      -> dqt_oracle_act_quant_fp8
+ *               the forward on E4M3 operands                -> dqt_oracle_fwd_fp8
  *
  * Readings where the paper is silent (each is listed in the design notes):
  *   - ternary ("1.58 bit") means the grid [-1, 1] with s = 1 / AbsMean;
@@ -30,7 +32,10 @@
  *     q = clamp(rint(x * s_x), -128, 127);
  *   - the RNG is Philox4x32-10 (Salmon et al., SC'11) keyed by the seed, with
  *     the counter (element/4, step, tensor id) and word element%4; a uniform
- *     U = (word >> 8) * 2^-24 rounds up when U < x - floor(x).
+ *     U = (word >> 8) * 2^-24 rounds up when U < x - floor(x);
+ *   - FP8 environment: the 8-bit activation is E4M3 with the per-token scale
+ *     448 / max(amax, 1e-5), rounded to nearest-even with saturation; the
+ *     forward accumulates exactly and rounds Y as the integer path does.
  *
  * Arithmetic: the reductions of the GEMMs are exact (int64) or fp64; the
  * AdamW + SR step is a fixed sequence of individually rounded IEEE fp32
@@ -393,4 +398,95 @@ int64_t dqt_oracle_update(const float* g, int8_t* c, float* m, float* v,
     }
   }
   return changed;
+}
+
+/* ======================================================================== */
+/* FP8 environment (Sec. 4.1 hardware paragraph, Sec. 4.3): the BitLinear    */
+/* forward with 8-bit floating-point operands.  The 8-bit activation is an   */
+/* E4M3 value with a per-token absmax scale instead of an int8 code; the     */
+/* weight codes (integers of magnitude at most 16) are exact E4M3 values.    */
+/* ======================================================================== */
+
+/* E4M3 ("e4m3fn" of the OCP 8-bit floating point format): sign bit, four   */
+/* exponent bits with bias 7, three mantissa bits.  Exponent field 0 holds   */
+/* the subnormals m * 2^-9; every other field is (1 + m/8) * 2^(e-7); the    */
+/* single magnitude pattern 1111.111 is NaN and there are no infinities, so  */
+/* the largest finite magnitude is 1.75 * 2^8 = 448.                          */
+double dqt_oracle_e4m3_value(uint8_t b) {
+  int e = (b >> 3) & 0xF;
+  int m = b & 0x7;
+  double mag;
+  if (e == 0xF && m == 0x7) return NAN;
+  if (e == 0) mag = ldexp((double)m, -9);
+  else mag = ldexp(1.0 + (double)m / 8.0, e - 7);
+  return (b & 0x80) ? -mag : mag;
+}
+
+/* Round-to-nearest-even onto the finite E4M3 values with saturation: the    */
+/* finite magnitude nearest to |p| (all 127 are tried), a tie going to the   */
+/* even code (the code's last bit is the mantissa's), anything beyond 448    */
+/* giving 448.  The sign is p's own, so values that round to zero keep it.   */
+uint8_t dqt_oracle_e4m3_from_f32(float p) {
+  if (isnan(p)) return 0x7F;
+  double a = fabs((double)p);
+  if (a > 448.0) return (uint8_t)(0x7E | (signbit(p) ? 0x80 : 0));
+  int best = 0;
+  double bd = a;
+  for (int b = 1; b < 0x7F; ++b) {
+    double d = fabs(a - dqt_oracle_e4m3_value((uint8_t)b));
+    if (d < bd || (d == bd && (b & 1) == 0 && (best & 1) == 1)) {
+      bd = d;
+      best = b;
+    }
+  }
+  return (uint8_t)(best | (signbit(p) ? 0x80 : 0));
+}
+
+void dqt_oracle_codes_to_e4m3(const int8_t* c, int64_t numel, uint8_t* out) {
+  for (int64_t i = 0; i < numel; ++i) out[i] = dqt_oracle_e4m3_from_f32((float)c[i]);
+}
+
+/* 8-bit activations as E4M3: per token t, amax = max_k |x|,                 */
+/* s8 = 448 / max(amax, 1e-5) (fp32 division), q8 = E4M3(x * s8) with the    */
+/* product one fp32 multiplication.  xdq (optional) is the dequantised       */
+/* activation bf16(value(q8) / s8) that the weight gradient reads.           */
+void dqt_oracle_act_quant_fp8(const uint16_t* X, int64_t T, int64_t K, uint8_t* q8,
+                              float* s8, uint16_t* xdq) {
+  for (int64_t t = 0; t < T; ++t) {
+    const uint16_t* row = X + t * K;
+    float amax = 0.0f;
+    for (int64_t k = 0; k < K; ++k) {
+      float a = fabsf(bf16_to_f32(row[k]));
+      if (a > amax) amax = a;
+    }
+    float s = 448.0f / (amax > 1e-5f ? amax : 1e-5f);
+    s8[t] = s;
+    for (int64_t k = 0; k < K; ++k) {
+      float p = bf16_to_f32(row[k]) * s;
+      uint8_t b = dqt_oracle_e4m3_from_f32(p);
+      q8[t * K + k] = b;
+      if (xdq) xdq[t * K + k] = f32_to_bf16_rne((float)dqt_oracle_e4m3_value(b) / s);
+    }
+  }
+}
+
+/* FP8 forward: acc[t,n] = sum_k value(q8[t,k]) * c[n,k], exact in fp64      */
+/* (every term is a multiple of 2^-9 below 2^13), and                        */
+/* Y[t,n] = bf16( float(acc) * (1 / (s8[t] * s_w)) ).                        */
+/* Returns 1 if a code is outside [-16, 16] (not exact in E4M3).            */
+int dqt_oracle_fwd_fp8(const uint8_t* q8, const float* s8, const int8_t* c, float s_w,
+                       int64_t T, int64_t K, int64_t N, uint16_t* Y, double* acc_out) {
+  for (int64_t i = 0; i < N * K; ++i)
+    if (c[i] < -16 || c[i] > 16) return 1;
+  for (int64_t t = 0; t < T; ++t) {
+    float a_t = 1.0f / (s8[t] * s_w);
+    for (int64_t n = 0; n < N; ++n) {
+      double acc = 0.0;
+      for (int64_t k = 0; k < K; ++k)
+        acc += dqt_oracle_e4m3_value(q8[t * K + k]) * (double)c[n * K + k];
+      if (acc_out) acc_out[t * N + n] = acc;
+      if (Y) Y[t * N + n] = f32_to_bf16_rne((float)acc * a_t);
+    }
+  }
+  return 0;
 }

@@ -13,6 +13,9 @@ with Stochastic Rounding"):
 * ``bwd_dw_bf16x``             -- Sec. 4.1/4.3, the weight gradient with X_tilde in bf16
 * ``adamw_consts``/``adamw_x`` -- Sec. 4.1, AdamW producing the dense target W'
 * ``update``                   -- Eq. 5, W_hat = SR(W') clamped onto the grid
+* ``e4m3_value``/``e4m3_from_f32``/``act_quant_fp8``/``fwd_fp8``
+                               -- Sec. 4.1/4.3 FP8 environment: E4M3 activations
+                                  and the forward on E4M3 operands
 
 bf16 tensors are passed as ``numpy.uint16`` arrays holding the raw bits.
 """
@@ -30,6 +33,7 @@ _i32p = C.POINTER(C.c_int32)
 _i64p = C.POINTER(C.c_int64)
 _u16p = C.POINTER(C.c_uint16)
 _u32p = C.POINTER(C.c_uint32)
+_u8p = C.POINTER(C.c_uint8)
 
 
 def lib():
@@ -77,6 +81,17 @@ def lib():
                                         C.c_int32, C.c_uint64, C.c_int64, C.c_uint32,
                                         C.c_int32, _i64p, C.c_int64, C.c_int64]
         L.dqt_oracle_update.restype = C.c_int64
+        L.dqt_oracle_e4m3_value.argtypes = [C.c_uint8]
+        L.dqt_oracle_e4m3_value.restype = C.c_double
+        L.dqt_oracle_e4m3_from_f32.argtypes = [C.c_float]
+        L.dqt_oracle_e4m3_from_f32.restype = C.c_uint8
+        L.dqt_oracle_codes_to_e4m3.argtypes = [_i8p, C.c_int64, _u8p]
+        L.dqt_oracle_codes_to_e4m3.restype = None
+        L.dqt_oracle_act_quant_fp8.argtypes = [_u16p, C.c_int64, C.c_int64, _u8p, _f32p, _u16p]
+        L.dqt_oracle_act_quant_fp8.restype = None
+        L.dqt_oracle_fwd_fp8.argtypes = [_u8p, _f32p, _i8p, C.c_float, C.c_int64, C.c_int64,
+                                         C.c_int64, _u16p, _f64p]
+        L.dqt_oracle_fwd_fp8.restype = C.c_int
         _lib = L
     return _lib
 
@@ -271,3 +286,52 @@ def update(g, c, m, v, consts, qmin, qmax, seed, step, tensor_id, round_mode=0,
                                       _p(v, _f32p), _p(k, _f32p), qmin, qmax, seed, step,
                                       tensor_id, round_mode, rp, Nr, K)
     return c, m, v, int(changed)
+
+
+# --------------------------------------------------------------------------
+# Sec. 4.1/4.3 FP8 environment
+# --------------------------------------------------------------------------
+def e4m3_value(b: int) -> float:
+    """The real value of the E4M3 byte b (NaN for the NaN patterns)."""
+    return float(lib().dqt_oracle_e4m3_value(int(b) & 0xFF))
+
+
+def e4m3_from_f32(p: float) -> int:
+    """Nearest-even E4M3 byte of the fp32 value p, saturating at +-448."""
+    return int(lib().dqt_oracle_e4m3_from_f32(float(p)))
+
+
+def codes_to_e4m3(c):
+    c = _c(c, np.int8)
+    out = np.empty(c.shape, np.uint8)
+    lib().dqt_oracle_codes_to_e4m3(_p(c, _i8p), c.size, _p(out, _u8p))
+    return out
+
+
+def act_quant_fp8(X_bits):
+    """X_bits: uint16 [T, K] raw bf16.  Returns (q8 u8 E4M3 bytes, s8 f32, xdq u16)."""
+    X = _c(X_bits, np.uint16)
+    T, K = X.shape
+    q8 = np.empty((T, K), np.uint8)
+    s = np.empty(T, np.float32)
+    xd = np.empty((T, K), np.uint16)
+    lib().dqt_oracle_act_quant_fp8(_p(X, _u16p), T, K, _p(q8, _u8p), _p(s, _f32p),
+                                   _p(xd, _u16p))
+    return q8, s, xd
+
+
+def fwd_fp8(q8, s8, c, s_w):
+    """Returns (Y bf16 bits u16 [T,N], acc float64 [T,N], exact)."""
+    q8 = _c(q8, np.uint8)
+    s8 = _c(s8, np.float32)
+    c = _c(c, np.int8)
+    T, K = q8.shape
+    N, K2 = c.shape
+    assert K == K2 and s8.shape == (T,)
+    Y = np.empty((T, N), np.uint16)
+    acc = np.empty((T, N), np.float64)
+    rc = lib().dqt_oracle_fwd_fp8(_p(q8, _u8p), _p(s8, _f32p), _p(c, _i8p), float(s_w),
+                                  T, K, N, _p(Y, _u16p), _p(acc, _f64p))
+    if rc:
+        raise ValueError("weight codes outside [-16, 16] are not exact in E4M3")
+    return Y, acc
