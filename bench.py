@@ -19,6 +19,10 @@ gradients and the device -> host read of the step's changed-code counts.
 The step's working set (~1.5 GB) is far larger than the 129 MB L2, so no
 flush is needed between steps.
 
+`--act fp8` runs the FP8-environment variant of the same step (Sec. 4.3):
+E4M3 activations and weight images, and the forward GEMMs on the 8-bit
+floating-point tensor cores (kind::f8f6f4); the backward is unchanged.
+
 `--impl reference` times the CPU oracle instead (bounded sample of the same
 step, extrapolated).  Under torchrun each rank runs an independent replica
 (weak scaling, no collective on the data path).
@@ -134,11 +138,12 @@ class ClockSampler:
 class MLPStep:
     """Device buffers and the launch sequence of one DQT MLP training step."""
 
-    def __init__(self, dev, seed=1234):
+    def __init__(self, dev, seed=1234, fp8=False):
         from paper_2412_04787_gb300 import dqt, inputs
 
         self.dqt = dqt
         self.dev = dev
+        self.fp8 = fp8
         self.grid = dqt.grid(1.58)
         T = T_TOK
         # two seeded input sets, alternated step by step, so that the
@@ -156,6 +161,7 @@ class MLPStep:
         self.d = self.dev_sets[0]
         self.alternate = True
         self.W, self.s_w, self.m, self.v, self.W_img, self.Y, self.dX, self.Xdq = {}, {}, {}, {}, {}, {}, {}, {}
+        self.W8 = {}
         for i, (name, K, N) in enumerate(PROJ):
             W0 = inputs.normal((N, K), 0.02, seed=20 + i).to(dev)
             self.W[name], self.s_w[name] = dqt.dqt_absmean_init(W0, self.grid)
@@ -163,17 +169,24 @@ class MLPStep:
             self.m[name] = torch.zeros((N, K), dtype=torch.float32, device=dev)
             self.v[name] = torch.zeros((N, K), dtype=torch.float32, device=dev)
             self.W_img[name] = torch.empty((N, K), dtype=torch.bfloat16, device=dev)
+            if fp8:
+                self.W8[name] = torch.empty((N, K), dtype=torch.uint8, device=dev)
             self.Y[name] = torch.empty((T, N), dtype=torch.bfloat16, device=dev)
             self.dX[name] = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
+        # per activation: (scale, forward operand, dequantised bf16 image); the
+        # forward operand is the bf16 code image, or the E4M3 bytes with fp8
         self.aq = {}
         for src, K in (("X", HID), ("H", INTER)):
             self.aq[src] = (torch.empty(T, dtype=torch.float32, device=dev),
-                            torch.empty((T, K), dtype=torch.bfloat16, device=dev),
+                            torch.empty((T, K), dtype=torch.uint8 if fp8 else torch.bfloat16,
+                                        device=dev),
                             torch.empty((T, K), dtype=torch.bfloat16, device=dev))
         self.changed = torch.zeros(3, dtype=torch.int64, device=dev)
         self.sr = {name: dqt.sr_stream(seed=seed, tensor_id=i) for i, (name, _, _) in enumerate(PROJ)}
         self.step_no = 0
-        self.launches_per_step = 2 + 3 + 3 + 3 + 3
+        self.launches_per_step = 2 + 3 + 3 + 3 + 3 + (3 if fp8 else 0)
+        self.kinds = (["act_quant_fp8", "codes_to_fp8", "codes_to_bf16", "fwd_fp8"] if fp8 else
+                      ["act_quant", "codes_to_bf16", "fwd"]) + ["bwd_dx", "bwd_dw_update"]
         self.streams = [torch.cuda.Stream(device=dev) for _ in range(4)]
 
     def run(self, timers=None, serial=False):
@@ -216,17 +229,28 @@ class MLPStep:
 
         def aq(src, stream):
             s_x, q_img, xdq = self.aq[src]
-            timed("act_quant", stream,
-                  lambda: dqt.dqt_act_quant(self.d[src], None, s_x, q_img, xdq, want=()))
+            if self.fp8:
+                timed("act_quant_fp8", stream,
+                      lambda: dqt.dqt_act_quant_fp8(self.d[src], q_img, s_x, xdq))
+            else:
+                timed("act_quant", stream,
+                      lambda: dqt.dqt_act_quant(self.d[src], None, s_x, q_img, xdq, want=()))
 
         def codes(name, stream):
+            if self.fp8:
+                timed("codes_to_fp8", stream,
+                      lambda: dqt.dqt_codes_to_fp8(self.W[name], self.grid, self.W8[name]))
             timed("codes_to_bf16", stream,
                   lambda: dqt.dqt_codes_to_bf16(self.W[name], self.W_img[name]))
 
         def fwd(name, stream):
             s_x, q_img, _ = self.aq["H" if name == "down" else "X"]
-            timed("fwd", stream, lambda: dqt.dqt_bitlinear_fwd(
-                q_img, s_x, self.W_img[name], self.s_w[name], self.grid, Y=self.Y[name]))
+            if self.fp8:
+                timed("fwd_fp8", stream, lambda: dqt.dqt_bitlinear_fwd_fp8(
+                    q_img, s_x, self.W8[name], self.s_w[name], self.grid, Y=self.Y[name]))
+            else:
+                timed("fwd", stream, lambda: dqt.dqt_bitlinear_fwd(
+                    q_img, s_x, self.W_img[name], self.s_w[name], self.grid, Y=self.Y[name]))
 
         def dx(name, stream):
             timed("bwd_dx", stream, lambda: dqt.dqt_bitlinear_bwd_dx(
@@ -276,10 +300,14 @@ class MLPStep:
         flops = {"fwd": [2.0 * T * K * N for _, K, N in PROJ]}
         flops["bwd_dx"] = list(flops["fwd"])
         flops["bwd_dw_update"] = list(flops["fwd"])
+        flops["fwd_fp8"] = list(flops["fwd"])
         byts = {
             # bf16 in (2) + bf16 code image (2) + bf16 dequantised image (2) per element, + s_x
             "act_quant": [T * HID * 6.0 + 4 * T, T * INTER * 6.0 + 4 * T],
+            # bf16 in (2) + E4M3 byte (1) + bf16 dequantised image (2) per element, + s_x8
+            "act_quant_fp8": [T * HID * 5.0 + 4 * T, T * INTER * 5.0 + 4 * T],
             "codes_to_bf16": [3.0 * K * N for _, K, N in PROJ],
+            "codes_to_fp8": [2.0 * K * N for _, K, N in PROJ],
         }
         return flops, byts
 
@@ -313,7 +341,7 @@ def run_gpu(args):
     torch.cuda.set_device(dev)
     from paper_2412_04787_gb300 import build as dqt_build
     dqt_build.build()
-    st = MLPStep(dev)
+    st = MLPStep(dev, fp8=args.act == "fp8")
     dqt = st.dqt
     stream = torch.cuda.current_stream()
 
@@ -344,7 +372,7 @@ def run_gpu(args):
 
     # ---- per-kernel timing: a second timed region of K steps with the same
     # launches serialised on one stream, CUDA events around every launch ----
-    kinds = ["act_quant", "codes_to_bf16", "fwd", "bwd_dx", "bwd_dw_update"]
+    kinds = st.kinds
     timers = {k: [] for k in kinds}
     barrier()
     s0 = torch.cuda.Event(enable_timing=True)
@@ -367,14 +395,17 @@ def run_gpu(args):
     for k in kinds:
         per[k]["share"] = per[k]["total_ms"] / tot if tot else None
     peaks, pk_kind = _peaks()
-    dom = max(["fwd", "bwd_dx", "bwd_dw_update"], key=lambda k: per[k]["total_ms"])
-    nlaunch = len(PROJ)
+    dom = max([k for k in kinds if k in flops], key=lambda k: per[k]["total_ms"])
     dom_flops = sum(flops[dom]) * args.steps
     achieved = dom_flops / (per[dom]["total_ms"] / 1e3) / 1e12
     peak = peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops"))
+    # E4M3 dense tensor rate: the measured bf16 rate times the nominal ratio 4.5 / 2.25
+    peak8 = 2.0 * peak
+    dom_peak = peak8 if dom == "fwd_fp8" else peak
     roofline = {"bound": "tensor", "kernel": dom, "achieved": round(achieved, 1),
-                "peak": peak, "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
-                "peak_kind": "bf16 dense sustained, %s" % pk_kind,
+                "peak": dom_peak, "unit": "TFLOP/s", "frac": round(achieved / dom_peak, 4),
+                "peak_kind": ("e4m3 dense sustained = 2 x measured bf16 sustained (nominal ratio)"
+                              if dom == "fwd_fp8" else "bf16 dense sustained, %s" % pk_kind),
                 "timing": "mean CUDA-event duration of its launches over a second timed region "
                           "of the same K steps run serially on one stream (%.4f ms/step)" % serial_ms_step,
                 "traffic": DW_TRAFFIC_BYTES.get(kernel_fingerprint()) if dom == "bwd_dw_update" else None,
@@ -385,7 +416,10 @@ def run_gpu(args):
         d = dict(per[k])
         if k in flops:
             d["tflops"] = sum(flops[k]) * args.steps / (per[k]["total_ms"] / 1e3) / 1e12
-            d["frac_of_bf16_sustained"] = d["tflops"] / peak
+            if k == "fwd_fp8":
+                d["frac_of_e4m3_sustained"] = d["tflops"] / peak8
+            else:
+                d["frac_of_bf16_sustained"] = d["tflops"] / peak
         else:
             d["gbs"] = sum(byts[k]) * args.steps / (per[k]["total_ms"] / 1e3) / 1e9
             d["frac_of_hbm"] = d["gbs"] / peaks["hbm_gbs"]
@@ -464,9 +498,11 @@ def run_gpu(args):
         line = {
             "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "e4m3 forward, bf16 backward" if st.fp8 else "bf16",
             "data": "synthetic (seeded N(0,1) activations, N(0,1e-2) gradients, AbsMean-ternary codes of N(0,0.02))",
-            "config": {"workload": WORKLOAD, "tokens": T_TOK, "hidden": HID, "intermediate": INTER,
+            "config": {"workload": WORKLOAD + (", FP8 (E4M3) forward" if st.fp8 else ""),
+                       "tokens": T_TOK, "hidden": HID, "intermediate": INTER,
                        "weights": "ternary int8 codes", "parallelism": "replicas" if ws > 1 else "single GPU",
                        "l2": "inputs larger than L2 (step working set ~1.5 GB > 129 MB)"},
             "roofline": roofline, "kernels": kern, "e2e": e2e,
@@ -619,14 +655,27 @@ def run_kernel(args):
                 dqt.dqt_sr_update(dW.view(-1), W.view(-1), s_w, m.view(-1), v.view(-1), hp, sr, g)
         elif k == "act_quant":
             fn = lambda: dqt.dqt_act_quant(X, None, s_x, q_img, xdq, want=())  # noqa: E731
+        elif k in ("act_quant_fp8", "fwd_fp8", "codes_to_fp8"):
+            q8, s8, _ = dqt.dqt_act_quant_fp8(X)
+            W8 = dqt.dqt_codes_to_fp8(W, g)
+            if k == "act_quant_fp8":
+                fn = lambda: dqt.dqt_act_quant_fp8(X, q8, s8, xdq)  # noqa: E731
+            elif k == "codes_to_fp8":
+                fn = lambda: dqt.dqt_codes_to_fp8(W, g, W8)  # noqa: E731
+            else:
+                fn = lambda: dqt.dqt_bitlinear_fwd_fp8(q8, s8, W8, s_w, g, Y=Y)  # noqa: E731
         elif k == "codes_to_bf16":
             fn = lambda: dqt.dqt_codes_to_bf16(W, W_img)  # noqa: E731
         else:
             raise SystemExit("unknown kernel %s" % k)
-        if k in ("fwd", "bwd_dx", "bwd_dw_update", "bwd_dw", "bwd_dw_unfused"):
+        if k in ("fwd", "bwd_dx", "bwd_dw_update", "bwd_dw", "bwd_dw_unfused", "fwd_fp8"):
             work, unit = 2.0 * T * K * N, "TFLOP/s"
         elif k == "act_quant":
             work, unit = 6.0 * T * K + 4 * T, "GB/s"
+        elif k == "act_quant_fp8":
+            work, unit = 5.0 * T * K + 4 * T, "GB/s"
+        elif k == "codes_to_fp8":
+            work, unit = 2.0 * N * K, "GB/s"
         else:
             work, unit = 3.0 * N * K, "GB/s"
     for _ in range(args.warmup):
@@ -649,6 +698,8 @@ def run_kernel(args):
     rate = work / (med / 1e3) / (1e12 if unit == "TFLOP/s" else 1e9)
     peaks, kind = _peaks()
     peak = peaks["bf16_tflops"] if unit == "TFLOP/s" else peaks["hbm_gbs"]
+    if k == "fwd_fp8":
+        peak = 2.0 * peak  # E4M3 dense = bf16 measured x the nominal ratio 4.5 / 2.25
     print(json.dumps({"kernel": k, "numel": args.numel if k == "sr_update" else None,
                       "shape": None if k == "sr_update" else [T, K, N],
                       "median_ms": round(med, 5), "min_ms": round(min(ms), 5),
@@ -657,10 +708,19 @@ def run_kernel(args):
                       "l2": "256 MiB buffer written between launches"}))
 
 
+DECODER_SIZES = {
+    # the paper's LLaMA-structured model sizes (Sec. 4.1): ~130M and ~1B
+    "130m": dict(layers=12, hidden=768, heads=12, ffn=2048, batch=16, seq=1024),
+    "1b": dict(layers=22, hidden=2048, heads=32, ffn=5632, batch=8, seq=2048),
+}
+
+
 def run_decoder(args):
     """A LLaMA-structured decoder training step with every transformer linear
-    layer a DQT BitLinear (12 layers, hidden 768, 12 heads, FFN 2048, vocab
-    32000, batch 16 x seq 1024, ternary; synthetic uniform token ids).  The
+    layer a DQT BitLinear (--decoder-size 130m: 12 layers, hidden 768, 12
+    heads, FFN 2048, batch 16 x seq 1024; 1b: 22 layers, hidden 2048, 32
+    heads, FFN 5632, batch 8 x seq 2048; vocab 32000, ternary; synthetic
+    uniform token ids; --act fp8 for the E4M3 forward).  The
     BitLinear layers update themselves during backward; the bf16 embedding,
     norms and head are stepped by torch AdamW inside the timed region.  By
     default the whole step is captured once as a CUDA graph and replayed, the
@@ -671,9 +731,10 @@ def run_decoder(args):
     dqt_build.build()
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
-    B, S = 16, 1024
-    cfg = DecoderConfig(layers=12, hidden=768, heads=12, ffn=2048, vocab=32000, bits=1.58,
-                        lr=1e-3, seed=1234)
+    sz = DECODER_SIZES[args.decoder_size]
+    B, S = sz["batch"], sz["seq"]
+    cfg = DecoderConfig(layers=sz["layers"], hidden=sz["hidden"], heads=sz["heads"], ffn=sz["ffn"],
+                        vocab=32000, bits=1.58, lr=1e-3, seed=1234, act=args.act)
     model = DQTDecoder(cfg, device=dev)
     use_graph = not args.no_graph
     model.enable_graph_updates()
@@ -748,10 +809,13 @@ def run_decoder(args):
         "metric": "DQT decoder training step tokens/s", "value": round(tokens * args.steps / (ms / 1e3), 1),
         "unit": "tokens/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(ms / args.steps, 3), "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "bf16", "data": "synthetic uniform token ids",
-        "config": {"workload": "LLaMA-structured decoder, ternary DQT BitLinear in q,k,v,o,gate,up,down",
-                   "layers": 12, "hidden": 768, "heads": 12, "ffn": 2048, "vocab": 32000,
-                   "batch": B, "seq": S, "cuda_graph": use_graph},
+        "vs_baseline": None,
+        "dtype": "e4m3 BitLinear forward, bf16 elsewhere" if args.act == "fp8" else "bf16",
+        "data": "synthetic uniform token ids",
+        "config": {"workload": "LLaMA-structured decoder (%s), ternary DQT BitLinear in q,k,v,o,gate,up,down%s"
+                               % (args.decoder_size, ", FP8 (E4M3) forward" if args.act == "fp8" else ""),
+                   "layers": cfg.layers, "hidden": cfg.hidden, "heads": cfg.heads, "ffn": cfg.ffn,
+                   "vocab": cfg.vocab, "batch": B, "seq": S, "cuda_graph": use_graph},
         "bitlinear_tflop_per_step": round(bl_flops / 1e12, 3),
         "e2e": {"value": round(tokens * args.steps / (e_ms / 1e3), 1), "unit": "tokens/s",
                 "h2d_bytes_per_step": int(host_ids[0].numel() * 8), "d2h_bytes_per_step": 4},
@@ -767,11 +831,15 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--kernel", default=None,
-                    help="time one kernel kind alone (fwd, bwd_dx, bwd_dw_update, act_quant, "
-                         "codes_to_bf16, sr_update)")
+                    help="time one kernel kind alone (fwd, bwd_dx, bwd_dw_update, bwd_dw, "
+                         "bwd_dw_unfused, act_quant, codes_to_bf16, sr_update, act_quant_fp8, "
+                         "codes_to_fp8, fwd_fp8)")
     ap.add_argument("--numel", type=int, default=1 << 26, help="weights for --kernel sr_update")
     ap.add_argument("--shape", default=None, help="T,K,N for --kernel GEMMs (default 8192,2048,5632)")
     ap.add_argument("--no-graph", action="store_true", help="decoder: run the step eagerly")
+    ap.add_argument("--act", default="int8", choices=["int8", "fp8"],
+                    help="mlp: 8-bit activations as int8 codes (default) or E4M3 (FP8 environment)")
+    ap.add_argument("--decoder-size", default="130m", choices=sorted(DECODER_SIZES))
     ap.add_argument("--workload", default="mlp", choices=["mlp", "decoder"],
                     help="mlp: the headline BitLinear MLP GEMM set; decoder: a 12-layer DQT decoder step")
     args = ap.parse_args()

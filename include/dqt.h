@@ -14,6 +14,7 @@
  *                                 step (Sec. 4.1) and W_hat = SR(W') (Eq. 1, Eq. 5),
  *                                 clamped to the n-bit grid and written over the codes
  *   dqt_sr_update                 the same AdamW + SR step for a gradient given in memory
+ *   dqt_*_fp8                     the forward with E4M3 operands (FP8 environment, Sec. 4.3)
  *
  * GB300 has no int8 tensor-core MMA for sm_103a, so the integer GEMMs run on
  * the bf16 tensor cores over exact bf16 images of the integer codes (every
@@ -237,6 +238,42 @@ int dqt_bitlinear_bwd_dw_update_dev(const dqt_bf16* dY, const dqt_bf16* Xdq, int
                                     void* ws, size_t ws_bytes, void* stream);
 int dqt_sr_update_dev(const float* grad, int8_t* W, float* m, float* v, const void* consts_dev,
                       int64_t numel, unsigned long long* changed_out, void* stream);
+
+/* ---- FP8 environment (Sec. 4.1 hardware paragraph; Sec. 4.3) ------------------
+ * The paper also trains DQT models with 8-bit floating-point GEMM operands.
+ * These three calls are the forward of that variant; the backward uses the
+ * bf16 calls above (dX with dqt_codes_to_bf16's image, dW + update with the
+ * Xdq image written here).  An E4M3 byte is the OCP 8-bit float "e4m3fn":
+ * sign, 4 exponent bits (bias 7), 3 mantissa bits, largest finite 448.
+ *
+ * Activations, per token t:
+ *   amax[t] = max_k |X[t,k]|,  s_x8[t] = 448 / max(amax[t], 1e-5)   (fp32 divide)
+ *   Xq8[t,k] = E4M3(X[t,k] * s_x8[t])   fp32 multiply, round-to-nearest-even,
+ *                                       saturating at +-448, sign kept for zero
+ *   X    bf16 [T, K] in;  Xq8 uint8 [T, K] out (required);  s_x8 fp32 [T] out
+ *   Xdq  bf16 [T, K] out, or NULL: bf16(value(Xq8) / s_x8), the dequantised
+ *        activation the weight gradient uses
+ * K a multiple of 16 (16-byte E4M3 rows). */
+int dqt_act_quant_fp8(const dqt_bf16* X, int64_t T, int64_t K, uint8_t* Xq8, float* s_x8,
+                      dqt_bf16* Xdq, void* stream);
+
+/* E4M3 image of weight codes: W8[i] = E4M3(W[i]), exact because every integer
+ * of magnitude <= 16 is an E4M3 value.  The grid bounds the codes: grids
+ * with a code beyond 16 in magnitude (6- to 8-bit) return DQT_ERR_RANGE (use
+ * the integer path, dqt_bitlinear_fwd).  numel >= 1. */
+int dqt_codes_to_fp8(const int8_t* W, int64_t numel, dqt_grid_t grid, uint8_t* W8, void* stream);
+
+/* Forward on E4M3 operands (tcgen05 kind::f8f6f4, fp32 accumulation):
+ *   acc[t,n] = sum_k value(Xq8[t,k]) * c[n,k]       fp32 accumulator
+ *   Y[t,n]   = bf16( acc * (1 / (s_x8[t] * s_w)) )
+ * Each product is exact; the sum is rounded by the fp32 accumulation (in an
+ * order the hardware chooses), so Y equals the exact-sum formula up to that
+ * rounding.  Xq8 uint8 [T, K], s_x8 fp32 [T] (dqt_act_quant_fp8); W8 uint8
+ * [N, K] (dqt_codes_to_fp8); grid as for dqt_codes_to_fp8; Y bf16 [T, N] out;
+ * acc_out fp32 [T, N] out, or NULL.  K a multiple of 16, N of 8. */
+int dqt_bitlinear_fwd_fp8(const uint8_t* Xq8, const float* s_x8, const uint8_t* W8, float s_w,
+                          dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
+                          float* acc_out, void* stream);
 
 #ifdef __cplusplus
 }

@@ -14,6 +14,12 @@ high-precision weight and no weight gradient tensor:
   (``dqt_bitlinear_bwd_dw_update``, Eq. 1 and Eq. 5): the layer is updated
   during its own backward.
 
+With ``act="fp8"`` (the FP8 environment of Sec. 4.3) the forward quantises
+activations to E4M3 bytes (``dqt_act_quant_fp8``), converts the codes to their
+exact E4M3 image (``dqt_codes_to_fp8``, grids up to 5 bits) and runs the GEMM
+on the 8-bit floating-point tensor cores (``dqt_bitlinear_fwd_fp8``); the
+backward is the same.
+
 Consequences: one backward per forward (no gradient accumulation across
 micro-batches, no weight sharing between calls), and ``optimizer.step()`` is
 not needed for these layers.  The state is ordinary module buffers, so
@@ -35,9 +41,14 @@ class _BitLinearFn(torch.autograd.Function):
         if x2.dtype != torch.bfloat16:
             x2 = x2.to(torch.bfloat16)
         x2 = x2.contiguous()
-        _, s_x, q_img, xdq = dqt.dqt_act_quant(x2, want=("Xq_img", "Xdq"))
-        w_img = dqt.dqt_codes_to_bf16(layer.codes)
-        y = dqt.dqt_bitlinear_fwd(q_img, s_x, w_img, float(layer.s_w), layer.grid_tuple)
+        if layer.act == "fp8":
+            q8, s_x, xdq = dqt.dqt_act_quant_fp8(x2)
+            w8 = dqt.dqt_codes_to_fp8(layer.codes, layer.grid_tuple)
+            y = dqt.dqt_bitlinear_fwd_fp8(q8, s_x, w8, float(layer.s_w), layer.grid_tuple)
+        else:
+            _, s_x, q_img, xdq = dqt.dqt_act_quant(x2, want=("Xq_img", "Xdq"))
+            w_img = dqt.dqt_codes_to_bf16(layer.codes)
+            y = dqt.dqt_bitlinear_fwd(q_img, s_x, w_img, float(layer.s_w), layer.grid_tuple)
         ctx.save_for_backward(xdq)
         ctx.layer = layer
         ctx.in_shape = x.shape
@@ -70,19 +81,27 @@ class DQTBitLinear(torch.nn.Module):
     AbsMean (Eq. 2-4) on the device.  ``lr``, ``betas``, ``eps`` and
     ``weight_decay`` are AdamW's; ``seed`` and ``tensor_id`` key the Philox
     stream of stochastic rounding (``round_mode`` 1 = round to nearest, the
-    Sec. 5.1 ablation).
+    Sec. 5.1 ablation).  ``act`` is "int8" (8-bit integer activation codes,
+    exact integer forward) or "fp8" (E4M3 activations and weight image).
     """
 
     def __init__(self, in_features, out_features, bits=1.58, lr=1e-3, betas=(0.9, 0.999),
                  eps=1e-8, weight_decay=0.0, seed=1234, tensor_id=0, init_std=0.02,
-                 init_seed=0, round_mode=0, device="cuda"):
+                 init_seed=0, round_mode=0, act="int8", device="cuda"):
         super().__init__()
         if in_features % 8 or out_features % 8:
             raise ValueError("in_features and out_features must be multiples of 8")
+        if act not in ("int8", "fp8"):
+            raise ValueError("act must be 'int8' or 'fp8'")
+        if act == "fp8" and in_features % 16:
+            raise ValueError("the E4M3 forward needs in_features a multiple of 16")
+        self.act = act
         self.in_features = in_features
         self.out_features = out_features
         g = dqt.grid(bits)
         self.grid_tuple = (g.qmin, g.qmax)
+        if act == "fp8" and (g.qmin < -16 or g.qmax > 16):
+            raise ValueError("the E4M3 weight image holds codes up to 16 in magnitude (<= 5 bits)")
         self.lr, self.betas, self.eps, self.weight_decay = lr, tuple(betas), eps, weight_decay
         self.round_mode = round_mode
         self.update_in_backward = True
@@ -149,5 +168,5 @@ class DQTBitLinear(torch.nn.Module):
                                         self.grid_tuple, changed_out=self.changed)
 
     def extra_repr(self):
-        return "in_features=%d, out_features=%d, grid=%s" % (self.in_features, self.out_features,
-                                                            self.grid_tuple)
+        return "in_features=%d, out_features=%d, grid=%s, act=%s" % (
+            self.in_features, self.out_features, self.grid_tuple, self.act)

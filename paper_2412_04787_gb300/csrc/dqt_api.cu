@@ -211,6 +211,49 @@ int dqt_bitlinear_fwd(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* 
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
+int dqt_act_quant_fp8(const dqt_bf16* X, int64_t T, int64_t K, uint8_t* Xq8, float* s_x8,
+                      dqt_bf16* Xdq, void* stream) {
+  if (!X || !Xq8 || !s_x8 || T <= 0 || K <= 0) return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim) return DQT_ERR_RANGE;
+  if (K % 16 || !aligned16(X) || !aligned16(Xq8) || (Xdq && !aligned16(Xdq)))
+    return DQT_ERR_ALIGN;
+  return dqt::launch_act_quant_fp8(X, T, K, Xq8, s_x8, Xdq, as_stream(stream)) ? DQT_ERR_CUDA
+                                                                              : DQT_OK;
+}
+
+int dqt_codes_to_fp8(const int8_t* W, int64_t numel, dqt_grid_t grid, uint8_t* W8, void* stream) {
+  if (!W || !W8 || numel <= 0 || !grid_ok(grid)) return DQT_ERR_ARG;
+  if (grid.qmin < -16 || grid.qmax > 16) return DQT_ERR_RANGE;
+  if (!aligned16(W) || !aligned16(W8)) return DQT_ERR_ALIGN;
+  return dqt::launch_codes_to_fp8(W, numel, W8, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
+int dqt_bitlinear_fwd_fp8(const uint8_t* Xq8, const float* s_x8, const uint8_t* W8, float s_w,
+                          dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
+                          float* acc_out, void* stream) {
+  if (!Xq8 || !s_x8 || !W8 || !Y || T <= 0 || K <= 0 || N <= 0 || !grid_ok(grid) ||
+      !(s_w > 0.0f) || !isfinite(s_w))
+    return DQT_ERR_ARG;
+  if (grid.qmin < -16 || grid.qmax > 16) return DQT_ERR_RANGE;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
+  if (K % 16 || N % 8 || !aligned16(Xq8) || !aligned16(W8) || !aligned16(Y) ||
+      (acc_out && !aligned16(acc_out)))
+    return DQT_ERR_ALIGN;
+  dqt::GemmLaunch g{};
+  g.kind = dqt::GEMM_FWD8;
+  g.M = static_cast<int>(T);
+  g.N = static_cast<int>(N);
+  g.Kred = static_cast<int>(K);
+  g.A = Xq8;
+  g.B = W8;
+  g.pair = true;
+  g.s_x = s_x8;
+  g.scale = s_w;
+  g.out_bf16 = Y;
+  g.acc_f32 = acc_out;
+  return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
 int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, int64_t T,
                          int64_t N, int64_t K, dqt_bf16* dX, void* stream) {
   if (!dY || !W_img || !dX || T <= 0 || N <= 0 || K <= 0 || !(s_w > 0.0f) || !isfinite(s_w))

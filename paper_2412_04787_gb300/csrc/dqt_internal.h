@@ -17,7 +17,7 @@ unsigned int* status_word();
 // GEMM kernel selection: 0 = 2-SM pair tiles where possible, 1 = 1-SM tiles.
 int gemm_mode();
 
-enum GemmKind { GEMM_FWD = 0, GEMM_DX = 1, GEMM_DW = 2 };
+enum GemmKind { GEMM_FWD = 0, GEMM_DX = 1, GEMM_DW = 2, GEMM_FWD8 = 3 };
 
 struct GemmLaunch {
   GemmKind kind;
@@ -27,15 +27,17 @@ struct GemmLaunch {
   //   FWD: A = Xq_img [M=T, Kred=K],  B = W_img [N, Kred=K]     (both K-major)
   //   DX : A = dY     [M=T, Kred=N],  B = W_img [Kred=N, N=K]   (B MN-major)
   //   DW : A = dY     [Kred=T, M=N],  B = Xdq   [Kred=T, N=K]   (both MN-major)
+  //   FWD8: A = Xq8 [M=T, Kred=K], B = W8 [N, Kred=K], E4M3 bytes (both K-major)
   const void* A;
   const void* B;
   int chunk_k;  // FWD: reduction elements per exact fp32 chunk (multiple of 64)
   bool pair;    // use the 2-SM (cta_group::2) kernel (not with drained chunks)
   // Epilogue operands.
-  const float* s_x;  // FWD
+  const float* s_x;  // FWD, FWD8
   float scale;       // FWD: s_w; DX: 1/s_w
   void* out_bf16;    // FWD: Y; DX: dX
   int32_t* acc_out;  // FWD, optional
+  float* acc_f32;    // FWD8, optional
   int8_t* W;         // DW (with m, v), optional
   float* m;
   float* v;
@@ -66,6 +68,11 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream);
 int launch_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
                      uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream);
 int launch_codes_to_bf16(const int8_t* W, int64_t numel, uint16_t* W_img, cudaStream_t stream);
+// FP8 environment: E4M3 activations with per-token scale 448 / max(amax, 1e-5)
+// (and optionally the dequantised bf16 image), and E4M3 images of weight codes.
+int launch_act_quant_fp8(const uint16_t* X, int64_t T, int64_t K, uint8_t* Xq8, float* s8,
+                         uint16_t* Xdq, cudaStream_t stream);
+int launch_codes_to_fp8(const int8_t* W, int64_t numel, uint8_t* W8, cudaStream_t stream);
 int launch_absmean_partial(const float* W0, int64_t numel, double* ws, cudaStream_t stream);
 int launch_absmean_codes(const float* W0, int64_t numel, float s_w, int32_t qmin, int32_t qmax,
                          int8_t* codes, cudaStream_t stream);

@@ -19,6 +19,12 @@
 // tile (for dW: the whole AdamW + stochastic-rounding update) overlaps the
 // MMAs of the next.
 //
+// FP8 environment (Sec. 4.1/4.3): the forward also runs on E4M3 operands
+// (tcgen05.mma kind::f8f6f4, 2-SM tiles only): a 128-byte swizzled row then
+// holds 128 elements of K, so a stage carries twice the reduction of a bf16
+// stage in the same bytes, and Y = bf16(acc * 1/(s_x s_w)) from the fp32
+// accumulator.
+//
 // Integer exactness of the forward GEMM.  The codes are fed as bf16 values
 // (exact for |v| <= 256); each product is exact in fp32 and a sum of integers
 // stays exact while its magnitude is at most 2^24.  The reduction is split into
@@ -53,6 +59,7 @@ struct Params {
   float scale;
   __nv_bfloat16* out_bf16;
   int32_t* acc_out;
+  float* acc_f32;  // FP8 forward: optional fp32 accumulators
   int8_t* W;
   float* m;
   float* v;
@@ -149,6 +156,32 @@ __device__ __forceinline__ void epi_dx(const Params& p, int gm, int gn0, const u
     pk.z = pack_bf16x2(__fmul_rn(f[8 * j + 4], p.scale), __fmul_rn(f[8 * j + 5], p.scale));
     pk.w = pack_bf16x2(__fmul_rn(f[8 * j + 6], p.scale), __fmul_rn(f[8 * j + 7], p.scale));
     *reinterpret_cast<uint4*>(yrow + 8 * j) = pk;
+  }
+}
+
+// FP8 forward: the fp32 accumulators are not integers; Y = bf16(acc * a_t).
+__device__ __forceinline__ void epi_fwd8(const Params& p, int gm, int gn0, float a_t,
+                                         const uint32_t (&a)[32]) {
+  const float* f = reinterpret_cast<const float*>(a);
+  __nv_bfloat16* yrow = p.out_bf16 + static_cast<size_t>(gm) * p.N + gn0;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    if (gn0 + 8 * j >= p.N) break;
+    uint4 pk;
+    pk.x = pack_bf16x2(__fmul_rn(f[8 * j + 0], a_t), __fmul_rn(f[8 * j + 1], a_t));
+    pk.y = pack_bf16x2(__fmul_rn(f[8 * j + 2], a_t), __fmul_rn(f[8 * j + 3], a_t));
+    pk.z = pack_bf16x2(__fmul_rn(f[8 * j + 4], a_t), __fmul_rn(f[8 * j + 5], a_t));
+    pk.w = pack_bf16x2(__fmul_rn(f[8 * j + 6], a_t), __fmul_rn(f[8 * j + 7], a_t));
+    *reinterpret_cast<uint4*>(yrow + 8 * j) = pk;
+  }
+  if (p.acc_f32) {
+    float* arow = p.acc_f32 + static_cast<size_t>(gm) * p.N + gn0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      if (gn0 + 4 * j >= p.N) break;
+      *reinterpret_cast<float4*>(arow + 4 * j) =
+          make_float4(f[4 * j], f[4 * j + 1], f[4 * j + 2], f[4 * j + 3]);
+    }
   }
 }
 
@@ -513,7 +546,10 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
   constexpr int EW = S::EW;
   constexpr int BN = 256;           // pair tile width; each CTA holds all 256 columns of its rows
   constexpr int HALF = BN / (EW / 4);  // columns per epilogue warp
-  constexpr uint32_t IDESC = idesc_bf16(256, 256, A_MN, B_MN);
+  constexpr bool F8 = EPI == GEMM_FWD8;
+  constexpr int KB = F8 ? 128 : BK;  // reduction elements per stage (one 128-byte row)
+  static_assert(!F8 || (!A_MN && !B_MN), "E4M3 operands are read K-major");
+  constexpr uint32_t IDESC = F8 ? idesc_e4m3(256, 256) : idesc_bf16(256, 256, A_MN, B_MN);
   constexpr uint32_t TMEM_COLS = 512;
   constexpr uint32_t MN_CHUNK_BYTES = 64 * BK * 2;
 
@@ -589,7 +625,7 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
           const uint32_t bar = full_lead + 8u * s;
           uint8_t* a = sA + s * S::A_BYTES;
           uint8_t* b = sB + s * S::B_BYTES;
-          const int k0 = kb * BK;
+          const int k0 = kb * KB;
           if (!A_MN) {
             tma_load_2d_pair(&tmA, bar, a, k0, m0);
           } else {
@@ -648,7 +684,8 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
                                      : sdesc_sw128(a_base + ks * 32, 16, 1024);
             const uint64_t bd = B_MN ? sdesc_sw128(b_base + ks * 2048, MN_CHUNK_BYTES, 1024)
                                      : sdesc_sw128(b_base + ks * 32, 16, 1024);
-            umma_bf16_pair(d, ad, bd, IDESC, (kb > kb0 || ks > 0) ? 1u : 0u);
+            if (F8) umma_f8_pair(d, ad, bd, IDESC, (kb > kb0 || ks > 0) ? 1u : 0u);
+            else umma_bf16_pair(d, ad, bd, IDESC, (kb > kb0 || ks > 0) ? 1u : 0u);
           }
           umma_commit_pair_mc(&empty[s], 0x3);
           if (kb == kb1 - 1) {
@@ -679,7 +716,7 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
       const int nbase = (tile % p.num_n) * BN + half * HALF;
       const bool row_ok = gm < p.M;
       float a_t = 0.0f;
-      if (EPI == GEMM_FWD && row_ok) a_t = __fdiv_rn(1.0f, __fmul_rn(p.s_x[gm], p.scale));
+      if ((EPI == GEMM_FWD || F8) && row_ok) a_t = __fdiv_rn(1.0f, __fmul_rn(p.s_x[gm], p.scale));
       const int b = u & 1;
       ok = __all_sync(0xffffffffu, mbar_wait_cl(&acc_full[b], (u >> 1) & 1u, p.wait_ns));
       if (!ok) break;
@@ -697,6 +734,7 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
         if (gn0 >= p.N) continue;  // warp-uniform
         if (!row_ok) continue;
         if (EPI == GEMM_FWD) epi_fwd(p, gm, gn0, a_t, a, r, false);
+        else if (F8) epi_fwd8(p, gm, gn0, a_t, a);
         else epi_dx(p, gm, gn0, a);
       }
       tc_fence_before();
@@ -741,17 +779,19 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 2-D bf16 row-major matrix with `inner` contiguous elements per row and
-// `outer` rows; box of box_inner x box_outer, 128-byte swizzle, zero fill.
+// 2-D row-major matrix of 2-byte (bf16) or 1-byte (E4M3) elements with
+// `inner` contiguous elements per row and `outer` rows; box of box_inner x
+// box_outer, 128-byte swizzle, zero fill.
 bool make_map(CUtensorMap* map, const void* ptr, uint64_t inner, uint64_t outer,
-              uint32_t box_inner, uint32_t box_outer) {
+              uint32_t box_inner, uint32_t box_outer, int elem_bytes = 2) {
   EncodeTiledFn enc = encode_fn();
   if (!enc) return false;
   const cuuint64_t dims[2] = {inner, outer};
-  const cuuint64_t strides[1] = {inner * 2};
+  const cuuint64_t strides[1] = {inner * static_cast<cuuint64_t>(elem_bytes)};
   const cuuint32_t box[2] = {box_inner, box_outer};
   const cuuint32_t estr[2] = {1, 1};
-  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box,
+  return enc(map, elem_bytes == 1 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+             2, const_cast<void*>(ptr), dims, strides, box,
              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -845,7 +885,8 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   p.M = g.M;
   p.N = g.N;
   p.Kred = g.Kred;
-  p.num_kb = (g.Kred + BK - 1) / BK;
+  const int kb_elems = g.kind == GEMM_FWD8 ? 128 : BK;
+  p.num_kb = (g.Kred + kb_elems - 1) / kb_elems;
   p.chunk_kb = p.num_kb;
   if (g.kind == GEMM_FWD) {
     const int ck = g.chunk_k / BK;
@@ -874,6 +915,7 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   p.scale = g.scale;
   p.out_bf16 = static_cast<__nv_bfloat16*>(g.out_bf16);
   p.acc_out = g.acc_out;
+  p.acc_f32 = g.acc_f32;
   p.W = g.W;
   p.m = g.m;
   p.v = g.v;
@@ -893,6 +935,11 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
       if (!make_map(&tb, g.B, g.Kred, g.N, BK, g2.pair ? 128 : 256)) return 3;
       if (g2.pair) return launch_pairs<false, false, GEMM_FWD>(ta, tb, p, stream);
       return launch_tiles<256, false, false, GEMM_FWD, false>(ta, tb, p, stream);
+    case GEMM_FWD8:
+      // 2-SM tiles whatever the tiling mode: E4M3 rows of 128 elements
+      if (!make_map(&ta, g.A, g.Kred, g.M, 128, BM, 1)) return 3;
+      if (!make_map(&tb, g.B, g.Kred, g.N, 128, 128, 1)) return 3;
+      return launch_pairs<false, false, GEMM_FWD8>(ta, tb, p, stream);
     case GEMM_DX:
       if (!make_map(&ta, g.A, g.Kred, g.M, BK, BM)) return 3;
       if (!make_map(&tb, g.B, g.N, g.Kred, 64, BK)) return 3;

@@ -3,6 +3,12 @@
 //                  bf16 operand images the tensor-core GEMMs read
 //   codes_to_bf16  exact bf16 image of the int8 weight codes
 //   absmean_*      Eq. 2-4 initialisation (deterministic fp64 reduction)
+// and, for the FP8 environment (Sec. 4.1/4.3), the same activation kernels
+// emitting E4M3 bytes with the per-token scale 448 / max(amax, 1e-5) (template
+// flag F8), and the E4M3 image of the weight codes.
+#include <cuda_fp16.h>
+#include <cuda_fp8.h>
+
 #include "dqt_internal.h"
 
 namespace dqt {
@@ -16,10 +22,52 @@ __device__ __forceinline__ uint16_t f32_to_bf16_bits(float f) {
   return *reinterpret_cast<const uint16_t*>(&h);
 }
 
+// The 8-bit activation code of eight bf16 values (one 16-byte vector) at
+// scale s: int8 Clip[Round(x s), -128, 127], or (F8) the E4M3 byte of x s,
+// round-to-nearest-even with saturation.  Each product is one fp32 multiply.
+template <bool F8>
+__device__ __forceinline__ void quant8(const uint4 u, float s, int32_t (&q)[8]) {
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float lo = __fmul_rn(bf16_bits_to_f32(w[j] & 0xFFFFu), s);
+    const float hi = __fmul_rn(bf16_bits_to_f32(w[j] >> 16), s);
+    if (F8) {
+      const uint32_t b = __nv_cvt_float2_to_fp8x2(make_float2(lo, hi), __NV_SATFINITE, __NV_E4M3);
+      q[2 * j] = static_cast<int32_t>(b & 0xFFu);
+      q[2 * j + 1] = static_cast<int32_t>((b >> 8) & 0xFFu);
+    } else {
+      q[2 * j] = static_cast<int32_t>(fminf(fmaxf(rintf(lo), -128.0f), 127.0f));
+      q[2 * j + 1] = static_cast<int32_t>(fminf(fmaxf(rintf(hi), -128.0f), 127.0f));
+    }
+  }
+}
+
+template <bool F8>
+__device__ __forceinline__ float code_scale_num() { return F8 ? 448.0f : 127.0f; }
+
+// Entry j of the dequantisation table: bf16(value / s) for the code whose
+// table index is j (int8 code j - 128, or E4M3 byte j).
+template <bool F8>
+__device__ __forceinline__ uint16_t dq_entry(int j, float s) {
+  float v;
+  if (F8) {
+    const __half h(__nv_cvt_fp8_to_halfraw(static_cast<__nv_fp8_storage_t>(j), __NV_E4M3));
+    v = __half2float(h);
+  } else {
+    v = static_cast<float>(j - 128);
+  }
+  return f32_to_bf16_bits(__fdiv_rn(v, s));
+}
+
+template <bool F8>
+__device__ __forceinline__ int dq_index(int32_t q) { return F8 ? q : q + 128; }
+
 // One warp per token row; 16-byte (8 x bf16) vector accesses.  Pass 1 finds
 // amax; pass 2 re-reads the row (an L1/L2 hit) and writes the outputs.
 constexpr int kAqWarps = 8;
 
+template <bool F8>
 __global__ void __launch_bounds__(kAqWarps * 32)
     act_quant_kernel(const uint16_t* __restrict__ X, int T, int K, int8_t* __restrict__ Xq,
                      float* __restrict__ s_x, uint16_t* __restrict__ Xq_img,
@@ -43,22 +91,15 @@ __global__ void __launch_bounds__(kAqWarps * 32)
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
-  const float s = __fdiv_rn(127.0f, fmaxf(amax, 1e-5f));
+  const float s = __fdiv_rn(code_scale_num<F8>(), fmaxf(amax, 1e-5f));
   if (lane == 0) s_x[row] = s;
 
   const size_t rbase = static_cast<size_t>(row) * K;
 #pragma unroll 4
   for (int i = lane; i < nv; i += 32) {
     const uint4 u = __ldg(xr + i);
-    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
     int32_t q[8];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float lo = bf16_bits_to_f32(w[j] & 0xFFFFu);
-      const float hi = bf16_bits_to_f32(w[j] >> 16);
-      q[2 * j] = static_cast<int32_t>(fminf(fmaxf(rintf(__fmul_rn(lo, s)), -128.0f), 127.0f));
-      q[2 * j + 1] = static_cast<int32_t>(fminf(fmaxf(rintf(__fmul_rn(hi, s)), -128.0f), 127.0f));
-    }
+    quant8<F8>(u, s, q);
     const size_t e = rbase + static_cast<size_t>(i) * 8;
     if (Xq) {
       uint2 pk;
@@ -77,7 +118,7 @@ __global__ void __launch_bounds__(kAqWarps * 32)
     if (Xdq) {
       uint32_t h[8];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) h[j] = f32_to_bf16_bits(__fdiv_rn(static_cast<float>(q[j]), s));
+      for (int j = 0; j < 8; ++j) h[j] = dq_entry<F8>(dq_index<F8>(q[j]), s);
       uint4 pk;
       pk.x = h[0] | (h[1] << 16);
       pk.y = h[2] | (h[3] << 16);
@@ -95,7 +136,7 @@ __global__ void __launch_bounds__(kAqWarps * 32)
 // dequantised image needs bf16(q / s_x) for q in [-128, 127] only, so the
 // row's threads first fill a 256-entry table of those correctly rounded
 // quotients and then look them up: bit-identical to dividing per element.
-template <int NV>
+template <int NV, bool F8>
 __global__ void __launch_bounds__(256)
     act_quant_rows_kernel(const uint16_t* __restrict__ X, int T, int K, int wpr,
                           int8_t* __restrict__ Xq, float* __restrict__ s_x,
@@ -135,11 +176,10 @@ __global__ void __launch_bounds__(256)
   __syncthreads();
   amax = part[rib * wpr];
   for (int w = 1; w < wpr; ++w) amax = fmaxf(amax, part[rib * wpr + w]);
-  const float s = __fdiv_rn(127.0f, fmaxf(amax, 1e-5f));
+  const float s = __fdiv_rn(code_scale_num<F8>(), fmaxf(amax, 1e-5f));
   if (live && tid == 0) s_x[row] = s;
   if (Xdq) {
-    for (int j = tid; j < 256; j += nth)
-      table[rib][j] = f32_to_bf16_bits(__fdiv_rn(static_cast<float>(j - 128), s));
+    for (int j = tid; j < 256; j += nth) table[rib][j] = dq_entry<F8>(j, s);
   }
   __syncthreads();
   if (!live) return;
@@ -148,15 +188,8 @@ __global__ void __launch_bounds__(256)
   for (int i = 0; i < NV; ++i) {
     const int vi = tid + nth * i;
     if (vi >= nv) break;
-    const uint32_t w[4] = {u[i].x, u[i].y, u[i].z, u[i].w};
     int32_t q[8];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float lo = bf16_bits_to_f32(w[j] & 0xFFFFu);
-      const float hi = bf16_bits_to_f32(w[j] >> 16);
-      q[2 * j] = static_cast<int32_t>(fminf(fmaxf(rintf(__fmul_rn(lo, s)), -128.0f), 127.0f));
-      q[2 * j + 1] = static_cast<int32_t>(fminf(fmaxf(rintf(__fmul_rn(hi, s)), -128.0f), 127.0f));
-    }
+    quant8<F8>(u[i], s, q);
     const size_t e = rbase + static_cast<size_t>(vi) * 8;
     if (Xq) {
       uint2 pk;
@@ -175,7 +208,7 @@ __global__ void __launch_bounds__(256)
     if (Xdq) {
       uint32_t h[8];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) h[j] = table[rib][q[j] + 128];
+      for (int j = 0; j < 8; ++j) h[j] = table[rib][dq_index<F8>(q[j])];
       __stcs(reinterpret_cast<uint4*>(Xdq + e),
              make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
                         h[6] | (h[7] << 16)));
@@ -187,6 +220,7 @@ __global__ void __launch_bounds__(256)
 // each warp walks rows row0, row0 + stride, ... and loads the next row while
 // it quantises the current one (two register buffers), so every warp keeps
 // two rows in flight and the grid has no wave tail.
+template <bool F8>
 __device__ __forceinline__ void aq_row_store(const uint4 (&u)[8], int nv, int lane, float s,
                                              size_t rbase, const uint16_t* table,
                                              int8_t* __restrict__ Xq,
@@ -196,15 +230,8 @@ __device__ __forceinline__ void aq_row_store(const uint4 (&u)[8], int nv, int la
   for (int i = 0; i < 8; ++i) {
     const int vi = lane + 32 * i;
     if (vi >= nv) break;
-    const uint32_t w[4] = {u[i].x, u[i].y, u[i].z, u[i].w};
     int32_t q[8];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float lo = bf16_bits_to_f32(w[j] & 0xFFFFu);
-      const float hi = bf16_bits_to_f32(w[j] >> 16);
-      q[2 * j] = static_cast<int32_t>(fminf(fmaxf(rintf(__fmul_rn(lo, s)), -128.0f), 127.0f));
-      q[2 * j + 1] = static_cast<int32_t>(fminf(fmaxf(rintf(__fmul_rn(hi, s)), -128.0f), 127.0f));
-    }
+    quant8<F8>(u[i], s, q);
     const size_t e = rbase + static_cast<size_t>(vi) * 8;
     if (Xq) {
       uint2 pk;
@@ -223,7 +250,7 @@ __device__ __forceinline__ void aq_row_store(const uint4 (&u)[8], int nv, int la
     if (Xdq) {
       uint32_t h[8];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) h[j] = table[q[j] + 128];
+      for (int j = 0; j < 8; ++j) h[j] = table[dq_index<F8>(q[j])];
       __stcs(reinterpret_cast<uint4*>(Xdq + e),
              make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
                         h[6] | (h[7] << 16)));
@@ -241,6 +268,7 @@ __device__ __forceinline__ void aq_row_load(const uint16_t* __restrict__ X, int 
   }
 }
 
+template <bool F8>
 __global__ void __launch_bounds__(256)
     act_quant_persist_kernel(const uint16_t* __restrict__ X, int T, int K,
                              int8_t* __restrict__ Xq, float* __restrict__ s_x,
@@ -267,16 +295,15 @@ __global__ void __launch_bounds__(256)
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
-    const float s = __fdiv_rn(127.0f, fmaxf(amax, 1e-5f));
+    const float s = __fdiv_rn(code_scale_num<F8>(), fmaxf(amax, 1e-5f));
     if (lane == 0) s_x[row] = s;
     if (Xdq) {
       __syncwarp();  // the previous row's lookups are done
 #pragma unroll
-      for (int j = lane; j < 256; j += 32)
-        table[wid][j] = f32_to_bf16_bits(__fdiv_rn(static_cast<float>(j - 128), s));
+      for (int j = lane; j < 256; j += 32) table[wid][j] = dq_entry<F8>(j, s);
       __syncwarp();
     }
-    aq_row_store(ua, nv, lane, s, static_cast<size_t>(row) * K, table[wid], Xq, Xq_img, Xdq);
+    aq_row_store<F8>(ua, nv, lane, s, static_cast<size_t>(row) * K, table[wid], Xq, Xq_img, Xdq);
 #pragma unroll
     for (int i = 0; i < 8; ++i) ua[i] = ub[i];
   }
@@ -331,6 +358,34 @@ __global__ void codes_to_bf16_kernel(const int8_t* __restrict__ W, int64_t numel
   // ragged tail (numel % 16 elements), one thread
   if (blockIdx.x == 0 && threadIdx.x == 0)
     for (int64_t e = nvec << 4; e < numel; ++e) img[e] = f32_to_bf16_bits(static_cast<float>(W[e]));
+}
+
+// E4M3 image of weight codes of magnitude <= 16 (exact): 16 codes per thread.
+__device__ __forceinline__ uint32_t codes4_to_e4m3(uint32_t w) {
+  const float c0 = static_cast<float>(static_cast<int8_t>(w & 0xFF));
+  const float c1 = static_cast<float>(static_cast<int8_t>((w >> 8) & 0xFF));
+  const float c2 = static_cast<float>(static_cast<int8_t>((w >> 16) & 0xFF));
+  const float c3 = static_cast<float>(static_cast<int8_t>(w >> 24));
+  const uint32_t lo = __nv_cvt_float2_to_fp8x2(make_float2(c0, c1), __NV_SATFINITE, __NV_E4M3);
+  const uint32_t hi = __nv_cvt_float2_to_fp8x2(make_float2(c2, c3), __NV_SATFINITE, __NV_E4M3);
+  return (lo & 0xFFFFu) | ((hi & 0xFFFFu) << 16);
+}
+
+__global__ void codes_to_fp8_kernel(const int8_t* __restrict__ W, int64_t numel,
+                                    uint8_t* __restrict__ out) {
+  const int64_t nvec = numel >> 4;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const uint4* src = reinterpret_cast<const uint4*>(W);
+  uint4* dst = reinterpret_cast<uint4*>(out);
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
+       i += stride) {
+    const uint4 u = __ldcs(src + i);
+    __stcs(dst + i, make_uint4(codes4_to_e4m3(u.x), codes4_to_e4m3(u.y), codes4_to_e4m3(u.z),
+                               codes4_to_e4m3(u.w)));
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0)
+    for (int64_t e = nvec << 4; e < numel; ++e)
+      out[e] = static_cast<uint8_t>(codes4_to_e4m3(static_cast<uint8_t>(W[e])) & 0xFFu);
 }
 
 // Eq. 2, stage 1: each of kAbsmeanBlocks blocks sums |w| in fp64 over a fixed
@@ -390,8 +445,11 @@ int grid_for(int64_t work, int threads) {
 
 }  // namespace
 
-int launch_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
-                     uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream) {
+namespace {
+
+template <bool F8>
+int launch_aq(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x, uint16_t* Xq_img,
+              uint16_t* Xdq, cudaStream_t stream) {
   const int t = static_cast<int>(T), k = static_cast<int>(K);
   const int64_t nv = K / 8;  // 16-byte vectors per row
   // warps per row: keep at most 4 vectors (32 values) per lane; up to 8 warps
@@ -402,22 +460,40 @@ int launch_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float*
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t want = (T + 7) / 8;
     const int blocks = static_cast<int>(want < 2 * sms ? want : 2 * sms);
-    act_quant_persist_kernel<<<blocks, 256, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq);
+    act_quant_persist_kernel<F8><<<blocks, 256, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq);
   } else if (wpr <= 8) {
     const int rpb = 8 / wpr;
     const int threads = 32 * wpr * rpb;
     const int blocks = static_cast<int>((T + rpb - 1) / rpb);
     const int per_lane = static_cast<int>((nv + 32 * wpr - 1) / (32 * wpr));
     if (per_lane <= 2)
-      act_quant_rows_kernel<2><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
+      act_quant_rows_kernel<2, F8><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
     else if (per_lane <= 4)
-      act_quant_rows_kernel<4><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
+      act_quant_rows_kernel<4, F8><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
     else
-      act_quant_rows_kernel<8><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
+      act_quant_rows_kernel<8, F8><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
   } else {
     const int blocks = static_cast<int>((T + kAqWarps - 1) / kAqWarps);
-    act_quant_kernel<<<blocks, kAqWarps * 32, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq);
+    act_quant_kernel<F8><<<blocks, kAqWarps * 32, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq);
   }
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+}  // namespace
+
+int launch_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
+                     uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream) {
+  return launch_aq<false>(X, T, K, Xq, s_x, Xq_img, Xdq, stream);
+}
+
+int launch_act_quant_fp8(const uint16_t* X, int64_t T, int64_t K, uint8_t* Xq8, float* s8,
+                         uint16_t* Xdq, cudaStream_t stream) {
+  return launch_aq<true>(X, T, K, reinterpret_cast<int8_t*>(Xq8), s8, nullptr, Xdq, stream);
+}
+
+int launch_codes_to_fp8(const int8_t* W, int64_t numel, uint8_t* W8, cudaStream_t stream) {
+  const int threads = 256;
+  codes_to_fp8_kernel<<<grid_for((numel >> 4) + 1, threads), threads, 0, stream>>>(W, numel, W8);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 

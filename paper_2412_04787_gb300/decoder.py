@@ -3,7 +3,8 @@
 The paper trains LLaMA-2-structured models (Sec. 4.1) with every weight
 matrix of the transformer blocks kept at n bits and updated by stochastic
 rounding (Sec. 3.2, Eq. 5).  Here q, k, v, o, gate, up and down are
-``DQTBitLinear`` layers running on this library's kernels; the token
+``DQTBitLinear`` layers running on this library's kernels (``act="fp8"``:
+the FP8-environment forward of Sec. 4.3); the token
 embedding, the RMSNorm gains and the output head stay in bf16 and are trained
 by an ordinary optimiser (which weights the paper keeps in high precision is
 not stated; this is the BitNet convention).  RMSNorm, rotary position
@@ -29,9 +30,9 @@ __all__ = ["DecoderConfig", "DQTDecoder"]
 
 class DecoderConfig:
     def __init__(self, layers=12, hidden=768, heads=12, ffn=2048, vocab=32000, bits=1.58,
-                 lr=1e-3, seed=1234, rope_theta=10000.0, norm_eps=1e-6):
+                 lr=1e-3, seed=1234, rope_theta=10000.0, norm_eps=1e-6, act="int8"):
         self.layers, self.hidden, self.heads, self.ffn, self.vocab = layers, hidden, heads, ffn, vocab
-        self.bits, self.lr, self.seed = bits, lr, seed
+        self.bits, self.lr, self.seed, self.act = bits, lr, seed, act
         self.rope_theta, self.norm_eps = rope_theta, norm_eps
 
 
@@ -65,7 +66,7 @@ class Block(torch.nn.Module):
         def bl(k, n, j):
             tid = index * 8 + j  # distinct Philox stream and initial draw per weight
             return DQTBitLinear(k, n, bits=cfg.bits, lr=cfg.lr, seed=cfg.seed, tensor_id=tid,
-                                init_seed=cfg.seed * 1000 + tid, device=device)
+                                init_seed=cfg.seed * 1000 + tid, act=cfg.act, device=device)
 
         self.q, self.k, self.v, self.o = bl(h, h, 0), bl(h, h, 1), bl(h, h, 2), bl(h, h, 3)
         self.gate, self.up, self.down = bl(h, f, 4), bl(h, f, 5), bl(f, h, 6)

@@ -23,6 +23,7 @@ EXPORTED = [
     "dqt_bitlinear_bwd_dw_update", "dqt_sr_update", "dqt_absmean_init_noalloc",
     "dqt_set_gemm_tiles", "dqt_update_consts_size", "dqt_update_consts",
     "dqt_bitlinear_bwd_dw_update_dev", "dqt_sr_update_dev", "dqt_bwd_dw_workspace_size",
+    "dqt_act_quant_fp8", "dqt_codes_to_fp8", "dqt_bitlinear_fwd_fp8",
 ]
 
 
@@ -88,6 +89,10 @@ def lib():
         L.dqt_bitlinear_bwd_dw_update_dev.argtypes = [_vp, _vp, _vp, _vp, _vp, _vp, _i64, _i64,
                                                       _i64, _vp, _vp, _vp, _sz, _vp]
         L.dqt_sr_update_dev.argtypes = [_vp, _vp, _vp, _vp, _vp, _i64, _vp, _vp]
+        L.dqt_act_quant_fp8.argtypes = [_vp, _i64, _i64, _vp, _vp, _vp, _vp]
+        L.dqt_codes_to_fp8.argtypes = [_vp, _i64, dqt_grid_t, _vp, _vp]
+        L.dqt_bitlinear_fwd_fp8.argtypes = [_vp, _vp, _vp, _f32, dqt_grid_t, _i64, _i64, _i64,
+                                            _vp, _vp, _vp]
         for name in EXPORTED:
             if name not in ("dqt_status_string", "dqt_absmean_workspace_size",
                             "dqt_update_consts_size", "dqt_bwd_dw_workspace_size"):
@@ -351,3 +356,55 @@ def dqt_sr_update_dev(grad, W, m, v, consts_dev, changed_out=None, stream=None):
     _check(lib().dqt_sr_update_dev(_ptr(grad), _ptr(W), _ptr(m), _ptr(v), _ptr(consts_dev), n,
                                    _ptr(changed_out), _stream(stream)), "dqt_sr_update_dev")
     return W
+
+
+# --------------------------------------------------------------------------
+# FP8 environment (Sec. 4.1/4.3): E4M3 bytes travel as torch.uint8 tensors.
+# --------------------------------------------------------------------------
+def dqt_act_quant_fp8(X, Xq8=None, s_x8=None, Xdq=None, want_xdq=True, stream=None):
+    """E4M3 activations with per-token scale 448 / max(amax, 1e-5).  Returns
+    (Xq8 uint8, s_x8 fp32, Xdq bf16 or None)."""
+    _need(X, "X", torch.bfloat16)
+    if X.dim() != 2:
+        raise ValueError("X must be [T, K]")
+    T, K = X.shape
+    dev = X.device
+    if Xq8 is None:
+        Xq8 = torch.empty((T, K), dtype=torch.uint8, device=dev)
+    if s_x8 is None:
+        s_x8 = torch.empty(T, dtype=torch.float32, device=dev)
+    if Xdq is None and want_xdq:
+        Xdq = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
+    _need(Xq8, "Xq8", torch.uint8, (T, K))
+    _need(s_x8, "s_x8", torch.float32, (T,))
+    _opt(Xdq, "Xdq", torch.bfloat16, (T, K))
+    _check(lib().dqt_act_quant_fp8(_ptr(X), T, K, _ptr(Xq8), _ptr(s_x8), _ptr(Xdq),
+                                   _stream(stream)), "dqt_act_quant_fp8")
+    return Xq8, s_x8, Xdq
+
+
+def dqt_codes_to_fp8(W, bits_or_grid, W8=None, stream=None):
+    _need(W, "W", torch.int8)
+    if W8 is None:
+        W8 = torch.empty(W.shape, dtype=torch.uint8, device=W.device)
+    _need(W8, "W8", torch.uint8, W.shape)
+    _check(lib().dqt_codes_to_fp8(_ptr(W), W.numel(), _grid(bits_or_grid), _ptr(W8),
+                                  _stream(stream)), "dqt_codes_to_fp8")
+    return W8
+
+
+def dqt_bitlinear_fwd_fp8(Xq8, s_x8, W8, s_w, bits_or_grid, Y=None, acc_out=None, stream=None):
+    _need(Xq8, "Xq8", torch.uint8)
+    T, K = Xq8.shape
+    _need(W8, "W8", torch.uint8)
+    N = W8.shape[0]
+    _need(W8, "W8", torch.uint8, (N, K))
+    _need(s_x8, "s_x8", torch.float32, (T,))
+    if Y is None:
+        Y = torch.empty((T, N), dtype=torch.bfloat16, device=Xq8.device)
+    _need(Y, "Y", torch.bfloat16, (T, N))
+    _opt(acc_out, "acc_out", torch.float32, (T, N))
+    _check(lib().dqt_bitlinear_fwd_fp8(_ptr(Xq8), _ptr(s_x8), _ptr(W8), float(s_w),
+                                       _grid(bits_or_grid), T, K, N, _ptr(Y), _ptr(acc_out),
+                                       _stream(stream)), "dqt_bitlinear_fwd_fp8")
+    return Y

@@ -108,3 +108,23 @@ def test_absmean_workspace(L):
     s = C.c_float()
     A = _p(0x10000)
     assert L.dqt_absmean_init(A, 16, dqt.dqt_grid_t(-1, 1), A, C.byref(s), A, 8, None) == dqt.DQT_ERR_ARG
+
+
+def test_fp8_argument_validation(L):
+    A = _p(0x10000)
+    t = dqt.dqt_grid_t(-1, 1)
+    g8 = dqt.dqt_grid_t(-128, 127)
+    # activations: K a multiple of 16, outputs required
+    assert L.dqt_act_quant_fp8(A, 4, 24, A, A, None, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_act_quant_fp8(A, 4, 32, None, A, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_act_quant_fp8(A, 0, 32, A, A, None, None) == dqt.DQT_ERR_ARG
+    # weight image: codes beyond 16 in magnitude are not exact in E4M3
+    assert L.dqt_codes_to_fp8(A, 64, g8, A, None) == dqt.DQT_ERR_RANGE
+    assert L.dqt_codes_to_fp8(A, 64, dqt.dqt_grid_t(-32, 31), A, None) == dqt.DQT_ERR_RANGE
+    assert L.dqt_codes_to_fp8(A, 0, t, A, None) == dqt.DQT_ERR_ARG
+    # forward
+    assert L.dqt_bitlinear_fwd_fp8(A, A, A, 1.0, g8, 4, 32, 8, A, None, None) == dqt.DQT_ERR_RANGE
+    assert L.dqt_bitlinear_fwd_fp8(A, A, A, 1.0, t, 4, 24, 8, A, None, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_bitlinear_fwd_fp8(A, A, A, 1.0, t, 4, 32, 12, A, None, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_bitlinear_fwd_fp8(A, A, A, 0.0, t, 4, 32, 8, A, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_fwd_fp8(None, A, A, 1.0, t, 4, 32, 8, A, None, None) == dqt.DQT_ERR_ARG

@@ -90,11 +90,11 @@ def test_bitlinear_state_dict_resume():
         assert torch.equal(getattr(a, name), getattr(b, name)), name
 
 
-def _train(bits_w, round_mode=0, steps=40):
+def _train(bits_w, round_mode=0, steps=40, act="int8"):
     from paper_2412_04787_gb300.decoder import DecoderConfig, DQTDecoder
     torch.manual_seed(0)
     cfg = DecoderConfig(layers=2, hidden=128, heads=4, ffn=256, vocab=512, bits=bits_w,
-                        lr=2e-3, seed=7)
+                        lr=2e-3, seed=7, act=act)
     model = DQTDecoder(cfg)
     for m in model.bitlinear_layers():
         m.round_mode = round_mode
@@ -123,6 +123,53 @@ def test_decoder_trains_with_low_bit_weights(bits_w):
         lo, hi = m.grid_tuple
         c = m.codes
         assert int(c.min()) >= lo and int(c.max()) <= hi
+
+
+def test_decoder_trains_in_fp8_environment():
+    """The same decoder with the E4M3 BitLinear forward (Sec. 4.3: DQT stays
+    robust when moving to the FP8 environment)."""
+    losses, moved, model = _train(1.58, act="fp8")
+    assert all(m.act == "fp8" for m in model.bitlinear_layers())
+    assert all(np.isfinite(losses))
+    assert losses[-1] < 0.8 * losses[0], (losses[0], losses[-1])
+    assert moved > 0
+
+
+def test_bitlinear_module_fp8_matches_oracle():
+    """act="fp8": the forward is the oracle's E4M3 forward (fp32-accumulation
+    bound), and the update is the oracle's DQT update fed the weight gradient
+    of the E4M3 dequantised activation (fused-update tolerance)."""
+    from paper_2412_04787_gb300.bitlinear import DQTBitLinear
+    T, K, N = 300, 272, 520
+    layer = DQTBitLinear(K, N, bits=1.58, lr=1e-3, seed=99, tensor_id=4, init_seed=7, act="fp8")
+    qmin, qmax = layer.grid_tuple
+    c0, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=7).numpy(), qmin, qmax)
+    layer.codes.copy_(torch.from_numpy(c0))
+    layer.s_w = float(s_w)
+    X = inputs.normal((T, K), 1.0, seed=1, dtype=torch.bfloat16)
+    dY = inputs.normal((T, N), 1e-2, seed=2, dtype=torch.bfloat16)
+    x = X.cuda().requires_grad_(True)
+    y = layer(x)
+    torch.cuda.synchronize()
+    q8, s8, xd = oracle.act_quant_fp8(bits(X))
+    Yr, acc = oracle.fwd_fp8(q8, s8, c0, np.float32(layer.s_w))
+    xv = np.vectorize(oracle.e4m3_value)(q8)
+    mag = np.abs(xv) @ np.abs(c0.astype(np.float64)).T
+    a_t = (np.float32(1.0) / (s8 * np.float32(layer.s_w))).astype(np.float64)
+    y_ref = torch.from_numpy(Yr.view(np.int16)).view(torch.bfloat16).double().numpy()
+    y_gpu = y.detach().double().cpu().numpy()
+    ulp = np.exp2(np.floor(np.log2(np.maximum(np.abs(y_ref), 1e-38))) - 7)
+    assert (np.abs(y_gpu - y_ref) <= ulp + a_t[:, None] * (K - 1) * 2.0 ** -24 * mag * 1.01).all()
+    y.backward(dY.cuda())
+    torch.cuda.synchronize()
+    g = oracle.bwd_dw_bf16x(bits(dY), xd).astype(np.float32)
+    k = oracle.adamw_consts(1e-3, 0.9, 0.999, 1e-8, 0.0, 1, layer.s_w)
+    z = np.zeros((N, K), np.float32)
+    c1, _, _, _ = oracle.update(g, c0, z, z, k, qmin, qmax, 99, 1, 4)
+    cg = layer.codes.cpu().numpy().astype(np.int32)
+    diff = cg != c1
+    assert diff.mean() <= 1e-4 + 1.0 / diff.size
+    assert (np.abs(cg - c1.astype(np.int32))[diff] == 1).all()
 
 
 def test_round_to_nearest_loses_small_updates():
