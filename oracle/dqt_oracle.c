@@ -21,6 +21,8 @@
  *   Sec 5.1 absmax / round-to-nearest ablation            -> round_mode = 1
  *   Sec 4.1/4.3 FP8 environment: E4M3 activations and      -> dqt_oracle_act_quant_fp8
  *               the forward on E4M3 operands                -> dqt_oracle_fwd_fp8
+ *   Sec 1       2-bit packed ternary storage                -> dqt_oracle_pack_ternary
+ *   Sec 4.3     Adafactor (factored second moment) + SR     -> dqt_oracle_adafactor_*
  *
  * Readings where the paper is silent (each is listed in the design notes):
  *   - ternary ("1.58 bit") means the grid [-1, 1] with s = 1 / AbsMean;
@@ -489,4 +491,152 @@ int dqt_oracle_fwd_fp8(const uint8_t* q8, const float* s8, const int8_t* c, floa
     }
   }
   return 0;
+}
+
+/* ======================================================================== */
+/* 2-bit packed ternary codes (the ternary storage of Sec. 1: about 0.2 GB    */
+/* for a 1B-parameter model).  Code e of a flat tensor lives in byte e / 4,  */
+/* bits 2 (e % 4) .. 2 (e % 4) + 1, as a 2-bit two's-complement number       */
+/* (-1 = 0b11, 0 = 0b00, +1 = 0b01).  Unused bits of the last byte are 0.    */
+/* ======================================================================== */
+void dqt_oracle_pack_ternary(const int8_t* c, int64_t n, uint8_t* out) {
+  for (int64_t i = 0; i < (n + 3) / 4; ++i) out[i] = 0;
+  for (int64_t e = 0; e < n; ++e)
+    out[e / 4] |= (uint8_t)(((unsigned)c[e] & 3u) << (2 * (e % 4)));
+}
+
+void dqt_oracle_unpack_ternary(const uint8_t* p, int64_t n, int8_t* c) {
+  for (int64_t e = 0; e < n; ++e) {
+    int v = (p[e / 4] >> (2 * (e % 4))) & 3;
+    c[e] = (int8_t)(v >= 2 ? v - 4 : v);
+  }
+}
+
+/* ======================================================================== */
+/* Adafactor with stochastic rounding (Sec. 4.3: DQT trained with the memory- */
+/* efficient Adafactor optimiser).  Adafactor is Shazeer & Stern, "Adafactor:  */
+/* Adaptive Learning Rates with Sublinear Memory Cost" (ICML 2018): the second */
+/* moment of an N x K gradient is kept as its row means R [N] and column      */
+/* means C [K] (factored), updates are clipped to RMS d, and the step size    */
+/* may be relative to the parameter's RMS.  Here without first moment (beta1 */
+/* = 0), the configuration that stores no per-weight state at all.           */
+/*                                                                          */
+/* Per step t (host constants, fp64 -> fp32 once):                          */
+/*   b2 = 1 - t^decay_rate,  omb2 = t^decay_rate                             */
+/*   rho = relative_step ? min(warmup_init ? 1e-6 t : 1e-2, 1/sqrt(t)) : lr  */
+/* Statistics (fp64 sums, state rounded to fp32):                            */
+/*   R[n] <- b2 R[n] + omb2 mean_k(g^2 + eps1)                                */
+/*   C[k] <- b2 C[k] + omb2 mean_n(g^2 + eps1)                                */
+/*   Rbar = mean_n R[n];   V[n,k] = R[n] C[k] / Rbar                         */
+/*   rms_u = sqrt(mean g^2 / V);   rms_x = sqrt(mean (c / s_w)^2)            */
+/*   alpha = rho * (scale_parameter ? max(eps2, rms_x) : 1)                  */
+/*   step  = s_w alpha / max(1, rms_u / d)        (code-domain step, fp32)   */
+/*   decay = 1 - weight_decay alpha                (fp32)                     */
+/* Per element, separately rounded fp32 operations (dqt_oracle_adafactor_    */
+/* apply):  v = (R[n] C[k]) / Rbar;  u = g / sqrt(v);  x = c decay - step u; */
+/* then c' = Clip[SR(x), Q_n, Q_p] with the same Philox stream as AdamW.      */
+/* ======================================================================== */
+void dqt_oracle_adafactor_consts(int64_t t, float lr, float decay_rate, int32_t relative_step,
+                                 int32_t warmup_init, float* b2, float* omb2, float* rho) {
+  double p = pow((double)t, (double)decay_rate);
+  *b2 = (float)(1.0 - p);
+  *omb2 = (float)p;
+  if (relative_step) {
+    double cap = warmup_init ? 1e-6 * (double)t : 1e-2;
+    double inv = 1.0 / sqrt((double)t);
+    *rho = (float)(cap < inv ? cap : inv);
+  } else {
+    *rho = lr;
+  }
+}
+
+/* R, C updated in place.  out4 = {Rbar, rms_u, rms_x, unused}; step and     */
+/* decay as above.                                                          */
+void dqt_oracle_adafactor_stats(const float* g, const int8_t* c, int64_t N, int64_t K,
+                                float s_w, float* R, float* C, float b2, float omb2,
+                                float rho, float eps1, float eps2, float clip_d,
+                                int32_t scale_parameter, float weight_decay, double* out4,
+                                float* step_out, float* decay_out) {
+  for (int64_t n = 0; n < N; ++n) {
+    double acc = 0.0;
+    for (int64_t k = 0; k < K; ++k) {
+      double gv = (double)g[n * K + k];
+      acc += gv * gv + (double)eps1;
+    }
+    R[n] = (float)((double)b2 * (double)R[n] + (double)omb2 * (acc / (double)K));
+  }
+  for (int64_t k = 0; k < K; ++k) {
+    double acc = 0.0;
+    for (int64_t n = 0; n < N; ++n) {
+      double gv = (double)g[n * K + k];
+      acc += gv * gv + (double)eps1;
+    }
+    C[k] = (float)((double)b2 * (double)C[k] + (double)omb2 * (acc / (double)N));
+  }
+  double rsum = 0.0;
+  for (int64_t n = 0; n < N; ++n) rsum += (double)R[n];
+  double rbar = rsum / (double)N;
+  double usq = 0.0, xsq = 0.0;
+  for (int64_t n = 0; n < N; ++n)
+    for (int64_t k = 0; k < K; ++k) {
+      double gv = (double)g[n * K + k];
+      double v = (double)R[n] * (double)C[k] / rbar;
+      usq += gv * gv / v;
+      double w = (double)c[n * K + k] / (double)s_w;
+      xsq += w * w;
+    }
+  double rms_u = sqrt(usq / ((double)N * (double)K));
+  double rms_x = sqrt(xsq / ((double)N * (double)K));
+  double alpha = (double)rho * (scale_parameter ? (rms_x > (double)eps2 ? rms_x : (double)eps2) : 1.0);
+  double div = rms_u / (double)clip_d;
+  if (div < 1.0) div = 1.0;
+  out4[0] = rbar;
+  out4[1] = rms_u;
+  out4[2] = rms_x;
+  out4[3] = alpha;
+  *step_out = (float)((double)s_w * alpha / div);
+  *decay_out = (float)(1.0 - (double)weight_decay * alpha);
+}
+
+static float adafactor_x(float g, int8_t c, float Rn, float Ck, float rbar, float step,
+                         float decay) {
+  float rc = Rn * Ck;
+  float v = rc / rbar;
+  float u = g / sqrtf(v);
+  float cd = (float)c * decay;
+  float du = step * u;
+  return cd - du;
+}
+
+/* Dense code-domain target only (no rounding), N x K. */
+void dqt_oracle_adafactor_x(const float* g, const int8_t* c, const float* R, const float* C,
+                            float rbar, float step, float decay, int64_t N, int64_t K, float* x) {
+  for (int64_t n = 0; n < N; ++n)
+    for (int64_t k = 0; k < K; ++k)
+      x[n * K + k] = adafactor_x(g[n * K + k], c[n * K + k], R[n], C[k], rbar, step, decay);
+}
+
+/* Per-element Adafactor + SR over an N x K weight, given R, C, Rbar (fp32), */
+/* the code-domain step and decay.  Returns the number of codes changed.     */
+int64_t dqt_oracle_adafactor_apply(const float* g, int8_t* c, const float* R, const float* C,
+                                   float rbar, float step, float decay, int64_t N, int64_t K,
+                                   int32_t qmin, int32_t qmax, uint64_t seed, int64_t t,
+                                   uint32_t tensor_id, int32_t round_mode) {
+  int64_t changed = 0;
+  for (int64_t n = 0; n < N; ++n)
+    for (int64_t k = 0; k < K; ++k) {
+      int64_t e = n * K + k;
+      float x = adafactor_x(g[e], c[e], R[n], C[k], rbar, step, decay);
+      int32_t r;
+      if (round_mode == 1) {
+        r = (int32_t)rintf(x);
+      } else {
+        uint32_t w = dqt_oracle_sr_word(seed, t, tensor_id, e);
+        r = dqt_oracle_sr(x, dqt_oracle_uniform_from_word(w));
+      }
+      r = clamp_i32(r, qmin, qmax);
+      if ((int8_t)r != c[e]) ++changed;
+      c[e] = (int8_t)r;
+    }
+  return changed;
 }

@@ -13,6 +13,9 @@ with Stochastic Rounding"):
 * ``bwd_dw_bf16x``             -- Sec. 4.1/4.3, the weight gradient with X_tilde in bf16
 * ``adamw_consts``/``adamw_x`` -- Sec. 4.1, AdamW producing the dense target W'
 * ``update``                   -- Eq. 5, W_hat = SR(W') clamped onto the grid
+* ``pack_ternary``/``unpack_ternary`` -- Sec. 1, 2-bit packed ternary storage
+* ``adafactor_consts``/``adafactor_stats``/``adafactor_x``/``adafactor_apply``
+                               -- Sec. 4.3, Adafactor (factored second moment) + SR
 * ``e4m3_value``/``e4m3_from_f32``/``act_quant_fp8``/``fwd_fp8``
                                -- Sec. 4.1/4.3 FP8 environment: E4M3 activations
                                   and the forward on E4M3 operands
@@ -92,6 +95,26 @@ def lib():
         L.dqt_oracle_fwd_fp8.argtypes = [_u8p, _f32p, _i8p, C.c_float, C.c_int64, C.c_int64,
                                          C.c_int64, _u16p, _f64p]
         L.dqt_oracle_fwd_fp8.restype = C.c_int
+        L.dqt_oracle_pack_ternary.argtypes = [_i8p, C.c_int64, _u8p]
+        L.dqt_oracle_pack_ternary.restype = None
+        L.dqt_oracle_unpack_ternary.argtypes = [_u8p, C.c_int64, _i8p]
+        L.dqt_oracle_unpack_ternary.restype = None
+        L.dqt_oracle_adafactor_consts.argtypes = [C.c_int64, C.c_float, C.c_float, C.c_int32,
+                                                  C.c_int32, _f32p, _f32p, _f32p]
+        L.dqt_oracle_adafactor_consts.restype = None
+        L.dqt_oracle_adafactor_stats.argtypes = [_f32p, _i8p, C.c_int64, C.c_int64, C.c_float,
+                                                 _f32p, _f32p, C.c_float, C.c_float, C.c_float,
+                                                 C.c_float, C.c_float, C.c_float, C.c_int32,
+                                                 C.c_float, _f64p, _f32p, _f32p]
+        L.dqt_oracle_adafactor_stats.restype = None
+        L.dqt_oracle_adafactor_x.argtypes = [_f32p, _i8p, _f32p, _f32p, C.c_float, C.c_float,
+                                             C.c_float, C.c_int64, C.c_int64, _f32p]
+        L.dqt_oracle_adafactor_x.restype = None
+        L.dqt_oracle_adafactor_apply.argtypes = [_f32p, _i8p, _f32p, _f32p, C.c_float,
+                                                 C.c_float, C.c_float, C.c_int64, C.c_int64,
+                                                 C.c_int32, C.c_int32, C.c_uint64, C.c_int64,
+                                                 C.c_uint32, C.c_int32]
+        L.dqt_oracle_adafactor_apply.restype = C.c_int64
         _lib = L
     return _lib
 
@@ -335,3 +358,95 @@ def fwd_fp8(q8, s8, c, s_w):
     if rc:
         raise ValueError("weight codes outside [-16, 16] are not exact in E4M3")
     return Y, acc
+
+
+# --------------------------------------------------------------------------
+# Sec. 1: 2-bit packed ternary storage
+# --------------------------------------------------------------------------
+def pack_ternary(c):
+    """int8 ternary codes -> uint8 [ceil(n/4)], code e in bits 2(e%4)..2(e%4)+1."""
+    c = _c(c, np.int8).ravel()
+    out = np.empty((c.size + 3) // 4, np.uint8)
+    lib().dqt_oracle_pack_ternary(_p(c, _i8p), c.size, _p(out, _u8p))
+    return out
+
+
+def unpack_ternary(p, n):
+    p = _c(p, np.uint8).ravel()
+    assert p.size >= (n + 3) // 4
+    out = np.empty(n, np.int8)
+    lib().dqt_oracle_unpack_ternary(_p(p, _u8p), n, _p(out, _i8p))
+    return out
+
+
+# --------------------------------------------------------------------------
+# Sec. 4.3: Adafactor (Shazeer & Stern 2018) + SR, no first moment
+# --------------------------------------------------------------------------
+class AdafactorHP:
+    """Adafactor hyper-parameters (defaults: a fixed step size lr, no
+    parameter scaling, eps1 = 1e-30 added to g^2, eps2 = 1e-3, update
+    clipping d = 1, beta2_t = 1 - t^-0.8, no weight decay)."""
+
+    def __init__(self, lr=1e-3, eps1=1e-30, eps2=1e-3, clip_d=1.0, decay_rate=-0.8,
+                 weight_decay=0.0, relative_step=False, scale_parameter=False,
+                 warmup_init=False):
+        self.lr, self.eps1, self.eps2, self.clip_d = lr, eps1, eps2, clip_d
+        self.decay_rate, self.weight_decay = decay_rate, weight_decay
+        self.relative_step, self.scale_parameter = relative_step, scale_parameter
+        self.warmup_init = warmup_init
+
+
+def adafactor_consts(t, hp):
+    """(b2, omb2, rho) of step t, each rounded once to fp32."""
+    b2, omb2, rho = C.c_float(), C.c_float(), C.c_float()
+    lib().dqt_oracle_adafactor_consts(int(t), hp.lr, hp.decay_rate, int(hp.relative_step),
+                                      int(hp.warmup_init), C.byref(b2), C.byref(omb2),
+                                      C.byref(rho))
+    return np.float32(b2.value), np.float32(omb2.value), np.float32(rho.value)
+
+
+def adafactor_stats(g, c, s_w, R, C_, t, hp):
+    """Returns (R', C', dict(rbar, rms_u, rms_x, alpha, step, decay)); R', C' fp32."""
+    g = _c(g, np.float32)
+    N, K = g.shape
+    c = _c(c, np.int8).reshape(N, K)
+    R = _c(R, np.float32).copy()
+    Cc = _c(C_, np.float32).copy()
+    assert R.shape == (N,) and Cc.shape == (K,)
+    b2, omb2, rho = adafactor_consts(t, hp)
+    out4 = np.empty(4, np.float64)
+    step, decay = C.c_float(), C.c_float()
+    lib().dqt_oracle_adafactor_stats(_p(g, _f32p), _p(c, _i8p), N, K, float(s_w), _p(R, _f32p),
+                                     _p(Cc, _f32p), b2, omb2, rho, hp.eps1, hp.eps2, hp.clip_d,
+                                     int(hp.scale_parameter), hp.weight_decay, _p(out4, _f64p),
+                                     C.byref(step), C.byref(decay))
+    st = {"rbar": out4[0], "rms_u": out4[1], "rms_x": out4[2], "alpha": out4[3],
+          "step": np.float32(step.value), "decay": np.float32(decay.value)}
+    return R, Cc, st
+
+
+def adafactor_x(g, c, R, C_, rbar, step, decay):
+    g = _c(g, np.float32)
+    N, K = g.shape
+    c = _c(c, np.int8).reshape(N, K)
+    R = _c(R, np.float32)
+    Cc = _c(C_, np.float32)
+    x = np.empty((N, K), np.float32)
+    lib().dqt_oracle_adafactor_x(_p(g, _f32p), _p(c, _i8p), _p(R, _f32p), _p(Cc, _f32p),
+                                 float(np.float32(rbar)), float(step), float(decay), N, K,
+                                 _p(x, _f32p))
+    return x
+
+
+def adafactor_apply(g, c, R, C_, rbar, step, decay, qmin, qmax, seed, t, tensor_id,
+                    round_mode=0):
+    """Returns (c', changed)."""
+    g = _c(g, np.float32)
+    N, K = g.shape
+    c = _c(c, np.int8).reshape(N, K).copy()
+    R = _c(R, np.float32)
+    Cc = _c(C_, np.float32)
+    ch = lib().dqt_oracle_adafactor_apply(_p(g, _f32p), _p(c, _i8p), _p(R, _f32p), _p(Cc, _f32p),
+                                          float(np.float32(rbar)), float(step), float(decay), N,
+                                          K, qmin, qmax, seed, t, tensor_id, round_mode)
+    return c, int(ch)
