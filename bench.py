@@ -23,6 +23,10 @@ flush is needed between steps.
 E4M3 activations and weight images, and the forward GEMMs on the 8-bit
 floating-point tensor cores (kind::f8f6f4); the backward is unchanged.
 
+`--optimizer adafactor` replaces the fused AdamW epilogue by Adafactor with
+SR (gradient GEMM, factored statistics, per-element step; Sec. 4.3) and
+`--packed` stores the ternary codes 2 bits each (Sec. 1).
+
 `--impl reference` times the CPU oracle instead (bounded sample of the same
 step, extrapolated).  Under torchrun each rank runs an independent replica
 (weak scaling, no collective on the data path).
@@ -68,7 +72,7 @@ def kernel_fingerprint(files=GEMM_SOURCES):
 # launches move the same numbers of operand and optimiser-state bytes), keyed
 # by the kernel fingerprint it was taken on (see profiles/).  A stale entry
 # reports null.
-DW_TRAFFIC_BYTES = {"9f06c4b1edd8": 296306944 + 56620032}
+DW_TRAFFIC_BYTES = {"729b805819b4": 295927296 + 57431552}
 
 
 def _dist():
@@ -138,12 +142,14 @@ class ClockSampler:
 class MLPStep:
     """Device buffers and the launch sequence of one DQT MLP training step."""
 
-    def __init__(self, dev, seed=1234, fp8=False):
+    def __init__(self, dev, seed=1234, fp8=False, optimizer="adamw", packed=False):
         from paper_2412_04787_gb300 import dqt, inputs
 
         self.dqt = dqt
         self.dev = dev
         self.fp8 = fp8
+        self.optimizer = optimizer
+        self.packed = packed
         self.grid = dqt.grid(1.58)
         T = T_TOK
         # two seeded input sets, alternated step by step, so that the
@@ -166,8 +172,14 @@ class MLPStep:
             W0 = inputs.normal((N, K), 0.02, seed=20 + i).to(dev)
             self.W[name], self.s_w[name] = dqt.dqt_absmean_init(W0, self.grid)
             del W0
-            self.m[name] = torch.zeros((N, K), dtype=torch.float32, device=dev)
-            self.v[name] = torch.zeros((N, K), dtype=torch.float32, device=dev)
+            if packed:
+                self.W[name] = dqt.dqt_pack_ternary(self.W[name])
+            if optimizer == "adamw":
+                self.m[name] = torch.zeros((N, K), dtype=torch.float32, device=dev)
+                self.v[name] = torch.zeros((N, K), dtype=torch.float32, device=dev)
+            else:  # Adafactor's factored statistics (row and column means)
+                self.m[name] = torch.zeros(N, dtype=torch.float32, device=dev)
+                self.v[name] = torch.zeros(K, dtype=torch.float32, device=dev)
             self.W_img[name] = torch.empty((N, K), dtype=torch.bfloat16, device=dev)
             if fp8:
                 self.W8[name] = torch.empty((N, K), dtype=torch.uint8, device=dev)
@@ -182,11 +194,20 @@ class MLPStep:
                                         device=dev),
                             torch.empty((T, K), dtype=torch.bfloat16, device=dev))
         self.changed = torch.zeros(3, dtype=torch.int64, device=dev)
+        self.af_ws = None
+        if optimizer == "adafactor":
+            nb = max(dqt.dqt_bwd_dw_adafactor_workspace_size(T, N, K) for _, K, N in PROJ)
+            # one workspace per concurrent stream (gate and up run side by side)
+            self.af_ws = [torch.empty(nb, dtype=torch.uint8, device=dev) for _ in range(4)]
         self.sr = {name: dqt.sr_stream(seed=seed, tensor_id=i) for i, (name, _, _) in enumerate(PROJ)}
         self.step_no = 0
         self.launches_per_step = 2 + 3 + 3 + 3 + 3 + (3 if fp8 else 0)
+        self.dw_kind = "bwd_dw_adafactor" if optimizer == "adafactor" else "bwd_dw_update"
         self.kinds = (["act_quant_fp8", "codes_to_fp8", "codes_to_bf16", "fwd_fp8"] if fp8 else
-                      ["act_quant", "codes_to_bf16", "fwd"]) + ["bwd_dx", "bwd_dw_update"]
+                      ["act_quant", "codes_to_bf16", "fwd"]) + ["bwd_dx", self.dw_kind]
+        if optimizer == "adafactor":
+            # gradient GEMM, four statistics kernels and the step per projection
+            self.launches_per_step += 3 * 5
         self.streams = [torch.cuda.Stream(device=dev) for _ in range(4)]
 
     def run(self, timers=None, serial=False):
@@ -237,11 +258,14 @@ class MLPStep:
                       lambda: dqt.dqt_act_quant(self.d[src], None, s_x, q_img, xdq, want=()))
 
         def codes(name, stream):
+            shape = tuple(self.W_img[name].shape)
             if self.fp8:
                 timed("codes_to_fp8", stream,
-                      lambda: dqt.dqt_codes_to_fp8(self.W[name], self.grid, self.W8[name]))
+                      lambda: dqt.dqt_packed_to_fp8(self.W[name], shape, self.W8[name]) if self.packed
+                      else dqt.dqt_codes_to_fp8(self.W[name], self.grid, self.W8[name]))
             timed("codes_to_bf16", stream,
-                  lambda: dqt.dqt_codes_to_bf16(self.W[name], self.W_img[name]))
+                  lambda: dqt.dqt_packed_to_bf16(self.W[name], shape, self.W_img[name]) if self.packed
+                  else dqt.dqt_codes_to_bf16(self.W[name], self.W_img[name]))
 
         def fwd(name, stream):
             s_x, q_img, _ = self.aq["H" if name == "down" else "X"]
@@ -258,9 +282,22 @@ class MLPStep:
 
         def dw(i, name, stream):
             xdq = self.aq["H" if name == "down" else "X"][2]
-            timed("bwd_dw_update", stream, lambda: dqt.dqt_bitlinear_bwd_dw_update(
-                self.d["dY_" + name], xdq, self.W[name], self.s_w[name], self.m[name],
-                self.v[name], hp, self.sr[name], self.grid, changed_out=self.changed[i:i + 1]))
+            ch = self.changed[i:i + 1]
+            if self.optimizer == "adafactor":
+                ws = self.af_ws[s.index(stream)]
+                af = dqt.adafactor(lr=1e-2, step=self.step_no)
+                timed(self.dw_kind, stream, lambda: dqt.dqt_bitlinear_bwd_dw_adafactor(
+                    self.d["dY_" + name], xdq, self.W[name], self.s_w[name], self.m[name],
+                    self.v[name], af, self.sr[name], self.grid, packed=self.packed,
+                    changed_out=ch, ws=ws))
+            elif self.packed:
+                timed(self.dw_kind, stream, lambda: dqt.dqt_bitlinear_bwd_dw_update_packed(
+                    self.d["dY_" + name], xdq, self.W[name], self.s_w[name], self.m[name],
+                    self.v[name], hp, self.sr[name], changed_out=ch))
+            else:
+                timed(self.dw_kind, stream, lambda: dqt.dqt_bitlinear_bwd_dw_update(
+                    self.d["dY_" + name], xdq, self.W[name], self.s_w[name], self.m[name],
+                    self.v[name], hp, self.sr[name], self.grid, changed_out=ch))
 
         for st in s:
             after(st, main)
@@ -300,14 +337,15 @@ class MLPStep:
         flops = {"fwd": [2.0 * T * K * N for _, K, N in PROJ]}
         flops["bwd_dx"] = list(flops["fwd"])
         flops["bwd_dw_update"] = list(flops["fwd"])
+        flops["bwd_dw_adafactor"] = list(flops["fwd"])
         flops["fwd_fp8"] = list(flops["fwd"])
         byts = {
             # bf16 in (2) + bf16 code image (2) + bf16 dequantised image (2) per element, + s_x
             "act_quant": [T * HID * 6.0 + 4 * T, T * INTER * 6.0 + 4 * T],
             # bf16 in (2) + E4M3 byte (1) + bf16 dequantised image (2) per element, + s_x8
             "act_quant_fp8": [T * HID * 5.0 + 4 * T, T * INTER * 5.0 + 4 * T],
-            "codes_to_bf16": [3.0 * K * N for _, K, N in PROJ],
-            "codes_to_fp8": [2.0 * K * N for _, K, N in PROJ],
+            "codes_to_bf16": [(2.25 if self.packed else 3.0) * K * N for _, K, N in PROJ],
+            "codes_to_fp8": [(1.25 if self.packed else 2.0) * K * N for _, K, N in PROJ],
         }
         return flops, byts
 
@@ -341,7 +379,7 @@ def run_gpu(args):
     torch.cuda.set_device(dev)
     from paper_2412_04787_gb300 import build as dqt_build
     dqt_build.build()
-    st = MLPStep(dev, fp8=args.act == "fp8")
+    st = MLPStep(dev, fp8=args.act == "fp8", optimizer=args.optimizer, packed=args.packed)
     dqt = st.dqt
     stream = torch.cuda.current_stream()
 
@@ -408,7 +446,8 @@ def run_gpu(args):
                               if dom == "fwd_fp8" else "bf16 dense sustained, %s" % pk_kind),
                 "timing": "mean CUDA-event duration of its launches over a second timed region "
                           "of the same K steps run serially on one stream (%.4f ms/step)" % serial_ms_step,
-                "traffic": DW_TRAFFIC_BYTES.get(kernel_fingerprint()) if dom == "bwd_dw_update" else None,
+                "traffic": (DW_TRAFFIC_BYTES.get(kernel_fingerprint())
+                            if dom == "bwd_dw_update" and not st.packed else None),
                 "kernel_fingerprint": kernel_fingerprint(),
                 "algorithmic_per_launch": "2*T*K*N FLOP (T=8192; K,N = 2048,5632 / 5632,2048)"}
     kern = {}
@@ -501,9 +540,13 @@ def run_gpu(args):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "e4m3 forward, bf16 backward" if st.fp8 else "bf16",
             "data": "synthetic (seeded N(0,1) activations, N(0,1e-2) gradients, AbsMean-ternary codes of N(0,0.02))",
-            "config": {"workload": WORKLOAD + (", FP8 (E4M3) forward" if st.fp8 else ""),
+            "config": {"workload": WORKLOAD + (", FP8 (E4M3) forward" if st.fp8 else "") +
+                                   (", Adafactor" if st.optimizer == "adafactor" else "") +
+                                   (", 2-bit packed codes" if st.packed else ""),
                        "tokens": T_TOK, "hidden": HID, "intermediate": INTER,
-                       "weights": "ternary int8 codes", "parallelism": "replicas" if ws > 1 else "single GPU",
+                       "weights": "ternary codes, %s" % ("2-bit packed" if st.packed else "int8"),
+                       "optimizer": st.optimizer,
+                       "parallelism": "replicas" if ws > 1 else "single GPU",
                        "l2": "inputs larger than L2 (step working set ~1.5 GB > 129 MB)"},
             "roofline": roofline, "kernels": kern, "e2e": e2e,
             "gpu_launches": st.launches_per_step * args.steps,
@@ -614,7 +657,7 @@ def run_kernel(args):
         T, K, N = (int(x) for x in args.shape.split(","))
     g = dqt.grid(1.58)
     k = args.kernel
-    if k == "sr_update":
+    if k in ("sr_update", "sr_update_packed"):
         n = args.numel
         grad = torch.randn(n, device=dev) * 1e-3
         W = torch.randint(-1, 2, (n,), dtype=torch.int8, device=dev)
@@ -622,8 +665,13 @@ def run_kernel(args):
         v = torch.zeros(n, device=dev)
         hp = dqt.adamw()
         sr = dqt.sr_stream()
-        fn = lambda: dqt.dqt_sr_update(grad, W, 62.0, m, v, hp, sr, g)  # noqa: E731
-        work, unit = 22.0 * n, "GB/s"
+        if k == "sr_update":
+            fn = lambda: dqt.dqt_sr_update(grad, W, 62.0, m, v, hp, sr, g)  # noqa: E731
+            work, unit = 22.0 * n, "GB/s"
+        else:
+            Wp = dqt.dqt_pack_ternary(W)
+            fn = lambda: dqt.dqt_sr_update_packed(grad, Wp, 62.0, m, v, hp, sr)  # noqa: E731
+            work, unit = 20.5 * n, "GB/s"
     else:
         X = inputs.normal((T, K), 1.0, seed=1, dtype=torch.bfloat16).to(dev)
         dY = inputs.normal((T, N), 1e-2, seed=2, dtype=torch.bfloat16).to(dev)
@@ -655,6 +703,24 @@ def run_kernel(args):
                 dqt.dqt_sr_update(dW.view(-1), W.view(-1), s_w, m.view(-1), v.view(-1), hp, sr, g)
         elif k == "act_quant":
             fn = lambda: dqt.dqt_act_quant(X, None, s_x, q_img, xdq, want=())  # noqa: E731
+        elif k == "bwd_dw_update_packed":
+            Wp = dqt.dqt_pack_ternary(W)
+            fn = lambda: dqt.dqt_bitlinear_bwd_dw_update_packed(dY, xdq, Wp, s_w, m, v, hp, sr)  # noqa: E731
+        elif k in ("bwd_dw_adafactor", "adafactor_stats", "adafactor_apply"):
+            R = torch.zeros(N, device=dev)
+            Cc = torch.zeros(K, device=dev)
+            af = dqt.adafactor(lr=1e-2)
+            G = torch.randn((N, K), device=dev) * 1e-3
+            scal = dqt.dqt_adafactor_stats(G, W, s_w, R, Cc, af)
+            if k == "bwd_dw_adafactor":
+                ws = torch.empty(dqt.dqt_bwd_dw_adafactor_workspace_size(T, N, K), dtype=torch.uint8,
+                                 device=dev)
+                fn = lambda: dqt.dqt_bitlinear_bwd_dw_adafactor(dY, xdq, W, s_w, R, Cc, af, sr, g,  # noqa: E731
+                                                                ws=ws)
+            elif k == "adafactor_stats":
+                fn = lambda: dqt.dqt_adafactor_stats(G, W, s_w, R, Cc, af, scalars_out=scal)  # noqa: E731
+            else:
+                fn = lambda: dqt.dqt_adafactor_apply(G, W, R, Cc, scal, 1, sr, g)  # noqa: E731
         elif k in ("act_quant_fp8", "fwd_fp8", "codes_to_fp8"):
             q8, s8, _ = dqt.dqt_act_quant_fp8(X)
             W8 = dqt.dqt_codes_to_fp8(W, g)
@@ -668,8 +734,15 @@ def run_kernel(args):
             fn = lambda: dqt.dqt_codes_to_bf16(W, W_img)  # noqa: E731
         else:
             raise SystemExit("unknown kernel %s" % k)
-        if k in ("fwd", "bwd_dx", "bwd_dw_update", "bwd_dw", "bwd_dw_unfused", "fwd_fp8"):
+        if k in ("fwd", "bwd_dx", "bwd_dw_update", "bwd_dw", "bwd_dw_unfused", "fwd_fp8",
+                 "bwd_dw_update_packed", "bwd_dw_adafactor"):
             work, unit = 2.0 * T * K * N, "TFLOP/s"
+        elif k == "adafactor_stats":
+            # two reads of G (4 B each) and one of the codes (1 B) per weight
+            work, unit = 9.0 * N * K, "GB/s"
+        elif k == "adafactor_apply":
+            # G read (4 B), codes read and written (1 + 1 B) per weight
+            work, unit = 6.0 * N * K, "GB/s"
         elif k == "act_quant":
             work, unit = 6.0 * T * K + 4 * T, "GB/s"
         elif k == "act_quant_fp8":
@@ -700,8 +773,9 @@ def run_kernel(args):
     peak = peaks["bf16_tflops"] if unit == "TFLOP/s" else peaks["hbm_gbs"]
     if k == "fwd_fp8":
         peak = 2.0 * peak  # E4M3 dense = bf16 measured x the nominal ratio 4.5 / 2.25
-    print(json.dumps({"kernel": k, "numel": args.numel if k == "sr_update" else None,
-                      "shape": None if k == "sr_update" else [T, K, N],
+    stream_k = k in ("sr_update", "sr_update_packed")
+    print(json.dumps({"kernel": k, "numel": args.numel if stream_k else None,
+                      "shape": None if stream_k else [T, K, N],
                       "median_ms": round(med, 5), "min_ms": round(min(ms), 5),
                       "rate": round(rate, 1), "unit": unit, "peak": peak,
                       "frac": round(rate / peak, 4), "peak_kind": "burst, " + kind,
@@ -734,10 +808,14 @@ def run_decoder(args):
     sz = DECODER_SIZES[args.decoder_size]
     B, S = sz["batch"], sz["seq"]
     cfg = DecoderConfig(layers=sz["layers"], hidden=sz["hidden"], heads=sz["heads"], ffn=sz["ffn"],
-                        vocab=32000, bits=1.58, lr=1e-3, seed=1234, act=args.act)
+                        vocab=32000, bits=1.58, lr=1e-2 if args.optimizer == "adafactor" else 1e-3,
+                        seed=1234, act=args.act, optimizer=args.optimizer, packed=args.packed)
     model = DQTDecoder(cfg, device=dev)
-    use_graph = not args.no_graph
-    model.enable_graph_updates()
+    # CUDA-graph replay needs the device-resident AdamW constants (int8 codes)
+    graphable = args.optimizer == "adamw" and not args.packed
+    use_graph = not args.no_graph and graphable
+    if graphable:
+        model.enable_graph_updates()
     opt = torch.optim.AdamW(model.dense_parameters(), lr=1e-3, fused=True, capturable=use_graph)
     g = torch.Generator().manual_seed(5)
     host_ids = [torch.randint(0, cfg.vocab, (B, S + 1), generator=g).pin_memory() for _ in range(2)]
@@ -755,8 +833,9 @@ def run_decoder(args):
         i = state["i"]
         state["i"] += 1
         static_ids.copy_(src, non_blocking=True)
-        model.prepare_step(i % 2)
-        model.upload_update_consts(i % 2)
+        if graphable:
+            model.prepare_step(i % 2)
+            model.upload_update_consts(i % 2)
         if use_graph:
             graph.replay()
             return state["loss"]
@@ -769,8 +848,9 @@ def run_decoder(args):
     with torch.cuda.stream(side):
         for i in range(args.warmup):
             static_ids.copy_(ids_dev[i % 2])
-            model.prepare_step(state["i"] % 2)
-            model.upload_update_consts(state["i"] % 2)
+            if graphable:
+                model.prepare_step(state["i"] % 2)
+                model.upload_update_consts(state["i"] % 2)
             state["i"] += 1
             fwd_bwd_opt()
             opt.zero_grad(set_to_none=True)
@@ -812,8 +892,10 @@ def run_decoder(args):
         "vs_baseline": None,
         "dtype": "e4m3 BitLinear forward, bf16 elsewhere" if args.act == "fp8" else "bf16",
         "data": "synthetic uniform token ids",
-        "config": {"workload": "LLaMA-structured decoder (%s), ternary DQT BitLinear in q,k,v,o,gate,up,down%s"
-                               % (args.decoder_size, ", FP8 (E4M3) forward" if args.act == "fp8" else ""),
+        "config": {"workload": "LLaMA-structured decoder (%s), ternary DQT BitLinear in q,k,v,o,gate,up,down%s%s%s"
+                               % (args.decoder_size, ", FP8 (E4M3) forward" if args.act == "fp8" else "",
+                                  ", Adafactor" if args.optimizer == "adafactor" else "",
+                                  ", 2-bit packed codes" if args.packed else ""),
                    "layers": cfg.layers, "hidden": cfg.hidden, "heads": cfg.heads, "ffn": cfg.ffn,
                    "vocab": cfg.vocab, "batch": B, "seq": S, "cuda_graph": use_graph},
         "bitlinear_tflop_per_step": round(bl_flops / 1e12, 3),
@@ -840,6 +922,9 @@ def main():
     ap.add_argument("--act", default="int8", choices=["int8", "fp8"],
                     help="mlp: 8-bit activations as int8 codes (default) or E4M3 (FP8 environment)")
     ap.add_argument("--decoder-size", default="130m", choices=sorted(DECODER_SIZES))
+    ap.add_argument("--optimizer", default="adamw", choices=["adamw", "adafactor"],
+                    help="the DQT optimiser of the BitLinear weights")
+    ap.add_argument("--packed", action="store_true", help="2-bit packed ternary code storage")
     ap.add_argument("--workload", default="mlp", choices=["mlp", "decoder"],
                     help="mlp: the headline BitLinear MLP GEMM set; decoder: a 12-layer DQT decoder step")
     args = ap.parse_args()

@@ -15,6 +15,8 @@
  *                                 clamped to the n-bit grid and written over the codes
  *   dqt_sr_update                 the same AdamW + SR step for a gradient given in memory
  *   dqt_*_fp8                     the forward with E4M3 operands (FP8 environment, Sec. 4.3)
+ *   dqt_*packed*                  2-bit packed ternary code storage (Sec. 1)
+ *   dqt_*adafactor*               Adafactor with SR instead of AdamW (Sec. 4.3)
  *
  * GB300 has no int8 tensor-core MMA for sm_103a, so the integer GEMMs run on
  * the bf16 tensor cores over exact bf16 images of the integer codes (every
@@ -274,6 +276,83 @@ int dqt_codes_to_fp8(const int8_t* W, int64_t numel, dqt_grid_t grid, uint8_t* W
 int dqt_bitlinear_fwd_fp8(const uint8_t* Xq8, const float* s_x8, const uint8_t* W8, float s_w,
                           dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
                           float* acc_out, void* stream);
+
+/* ---- 2-bit packed ternary codes (Sec. 1: ternary weights need a fraction of
+ * a byte each; 4 codes per byte here, 0.25 GB per 1B weights) ----------------
+ * Code e of a tensor is field e % 4 (bits 2 (e % 4) and 2 (e % 4) + 1) of byte
+ * e / 4, a 2-bit two's-complement number (-1 = 0b11, 0 = 0b00, +1 = 0b01);
+ * unused fields of the last byte are 0.  A packed [N, K] weight needs K % 4 ==
+ * 0 (K % 8 == 0 for the GEMMs) so that rows start on byte boundaries.  Packed
+ * tensors are ceil(numel / 4) bytes, 16-byte aligned. */
+int dqt_pack_ternary(const int8_t* codes, int64_t numel, uint8_t* packed, void* stream);
+int dqt_unpack_ternary(const uint8_t* packed, int64_t numel, int8_t* codes, void* stream);
+/* GEMM operand images straight from packed codes (as dqt_codes_to_bf16 and
+ * dqt_codes_to_fp8 do from int8 codes). */
+int dqt_packed_to_bf16(const uint8_t* packed, int64_t numel, dqt_bf16* W_img, void* stream);
+int dqt_packed_to_fp8(const uint8_t* packed, int64_t numel, uint8_t* W8, void* stream);
+/* dqt_sr_update and dqt_bitlinear_bwd_dw_update on packed ternary codes (the
+ * grid is [-1, 1]); identical results, 0.25 byte per weight of code traffic. */
+int dqt_sr_update_packed(const float* grad, uint8_t* Wp, float s_w, float* m, float* v,
+                         const dqt_adamw_t* hp, const dqt_sr_t* sr, int64_t numel,
+                         unsigned long long* changed_out, void* stream);
+int dqt_bitlinear_bwd_dw_update_packed(const dqt_bf16* dY, const dqt_bf16* Xdq, uint8_t* Wp,
+                                       float s_w, float* m, float* v, const dqt_adamw_t* hp,
+                                       const dqt_sr_t* sr, int64_t T, int64_t N, int64_t K,
+                                       float* dW_out, unsigned long long* changed_out, void* ws,
+                                       size_t ws_bytes, void* stream);
+
+/* ---- Adafactor with stochastic rounding (Sec. 4.3) ---------------------------
+ * The memory-efficient optimiser the paper pairs with DQT: Adafactor (Shazeer
+ * & Stern, ICML 2018) without first moment keeps only the row means R [N] and
+ * column means C [K] of an N x K weight's squared gradient (fp32, zero at the
+ * start, in place), so no per-weight optimiser state exists at all.  Step t:
+ *   b2 = 1 - t^decay_rate;  rho = relative_step ? min(warmup_init ? 1e-6 t : 1e-2,
+ *                                                  1/sqrt(t)) : lr
+ *   R <- b2 R + (1 - b2) mean_k(g^2 + eps1);  C <- b2 C + (1 - b2) mean_n(g^2 + eps1)
+ *   Rbar = mean R;  v = R[n] C[k] / Rbar;  u = g / sqrt(v)
+ *   alpha = rho * (scale_parameter ? max(eps2, RMS(W)) : 1),  RMS(W) = RMS(c) / s_w
+ *   x = c (1 - weight_decay alpha) - s_w alpha / max(1, RMS(u) / clip_d) * u
+ *   c <- Clip[SR(x), qmin, qmax]   (Eq. 1, Eq. 5; the Philox stream of dqt_sr_t
+ *                                   with counter step t, as for AdamW)
+ * Defaults a caller may start from: lr 1e-3, eps1 1e-30, eps2 1e-3, clip_d 1,
+ * decay_rate -0.8, weight_decay 0, relative_step 0, scale_parameter 0. */
+typedef struct {
+  float lr, eps1, eps2, clip_d, decay_rate, weight_decay;
+  int64_t step; /* t >= 1 */
+  int32_t relative_step, scale_parameter, warmup_init, pad;
+} dqt_adafactor_t;
+
+/* Statistics of one step for a gradient G fp32 [N, K] in memory: updates R, C
+ * and writes 8 floats to scalars_out (device, 16-byte aligned):
+ * {Rbar, code-domain step s_w alpha / max(1, RMS(u)/clip_d), decay
+ * 1 - weight_decay alpha, RMS(u), RMS(W), alpha, 0, 0}.  W: the codes before
+ * the step (int8 [N, K], or packed ternary if `packed`).  Workspace:
+ * dqt_adafactor_workspace_size(N, K) bytes, 256-byte aligned.  Every sum has
+ * a fixed order: deterministic. */
+size_t dqt_adafactor_workspace_size(int64_t N, int64_t K);
+int dqt_adafactor_stats(const float* G, const void* W, int32_t packed, float s_w, float* R,
+                        float* C, const dqt_adafactor_t* hp, int64_t N, int64_t K,
+                        float* scalars_out, void* ws, size_t ws_bytes, void* stream);
+/* The per-element step given R, C and the scalars {Rbar, step, decay} in
+ * device memory (as dqt_adafactor_stats writes them): v = (R[n] C[k]) / Rbar,
+ * u = g / sqrt(v), x = c decay - step u, each a separately rounded fp32
+ * operation, then SR with counter `step_t` and the clamp.  changed_out as for
+ * dqt_sr_update. */
+int dqt_adafactor_apply(const float* G, void* W, int32_t packed, const float* R, const float* C,
+                        const float* scalars, int64_t step_t, const dqt_sr_t* sr, dqt_grid_t grid,
+                        int64_t N, int64_t K, unsigned long long* changed_out, void* stream);
+/* The whole backward-and-update of a BitLinear weight with Adafactor: the
+ * weight gradient dY^T Xdq (fp32, tensor cores) into the workspace, then the
+ * statistics and the per-element step above.  Workspace:
+ * dqt_bwd_dw_adafactor_workspace_size(T, N, K) bytes (the fp32 gradient, the
+ * statistics, and token-slice partials when the GEMM splits the reduction). */
+size_t dqt_bwd_dw_adafactor_workspace_size(int64_t T, int64_t N, int64_t K);
+int dqt_bitlinear_bwd_dw_adafactor(const dqt_bf16* dY, const dqt_bf16* Xdq, void* W,
+                                   int32_t packed, float s_w, float* R, float* C,
+                                   const dqt_adafactor_t* hp, const dqt_sr_t* sr, dqt_grid_t grid,
+                                   int64_t T, int64_t N, int64_t K,
+                                   unsigned long long* changed_out, void* ws, size_t ws_bytes,
+                                   void* stream);
 
 #ifdef __cplusplus
 }

@@ -20,6 +20,11 @@ exact E4M3 image (``dqt_codes_to_fp8``, grids up to 5 bits) and runs the GEMM
 on the 8-bit floating-point tensor cores (``dqt_bitlinear_fwd_fp8``); the
 backward is the same.
 
+``optimizer="adafactor"`` replaces AdamW's two fp32 moments by Adafactor's
+factored row and column statistics (Sec. 4.3), and ``packed=True`` keeps
+ternary codes 2 bits each (Sec. 1); the two together leave 0.25 byte of
+state per weight plus N + K floats.
+
 Consequences: one backward per forward (no gradient accumulation across
 micro-batches, no weight sharing between calls), and ``optimizer.step()`` is
 not needed for these layers.  The state is ordinary module buffers, so
@@ -43,12 +48,12 @@ class _BitLinearFn(torch.autograd.Function):
         x2 = x2.contiguous()
         if layer.act == "fp8":
             q8, s_x, xdq = dqt.dqt_act_quant_fp8(x2)
-            w8 = dqt.dqt_codes_to_fp8(layer.codes, layer.grid_tuple)
-            y = dqt.dqt_bitlinear_fwd_fp8(q8, s_x, w8, float(layer.s_w), layer.grid_tuple)
+            y = dqt.dqt_bitlinear_fwd_fp8(q8, s_x, layer.weight_fp8(), float(layer.s_w),
+                                          layer.grid_tuple)
         else:
             _, s_x, q_img, xdq = dqt.dqt_act_quant(x2, want=("Xq_img", "Xdq"))
-            w_img = dqt.dqt_codes_to_bf16(layer.codes)
-            y = dqt.dqt_bitlinear_fwd(q_img, s_x, w_img, float(layer.s_w), layer.grid_tuple)
+            y = dqt.dqt_bitlinear_fwd(q_img, s_x, layer.weight_bf16(), float(layer.s_w),
+                                      layer.grid_tuple)
         ctx.save_for_backward(xdq)
         ctx.layer = layer
         ctx.in_shape = x.shape
@@ -66,8 +71,7 @@ class _BitLinearFn(torch.autograd.Function):
         dy2 = dy2.contiguous()
         # the codes have not changed since the forward: the image is rebuilt
         # instead of being kept alive across the step
-        w_img = dqt.dqt_codes_to_bf16(layer.codes)
-        dx = dqt.dqt_bitlinear_bwd_dx(dy2, w_img, float(layer.s_w))
+        dx = dqt.dqt_bitlinear_bwd_dx(dy2, layer.weight_bf16(), float(layer.s_w))
         if layer.update_in_backward:
             layer._dqt_update(dy2, xdq)
         return dx.reshape(ctx.in_shape).to(ctx.in_dtype), None, None
@@ -83,11 +87,15 @@ class DQTBitLinear(torch.nn.Module):
     stream of stochastic rounding (``round_mode`` 1 = round to nearest, the
     Sec. 5.1 ablation).  ``act`` is "int8" (8-bit integer activation codes,
     exact integer forward) or "fp8" (E4M3 activations and weight image).
+    ``optimizer`` is "adamw" or "adafactor" (``adafactor`` holds its other
+    hyper-parameters as a dict for ``dqt.adafactor``); ``packed`` stores
+    ternary codes 2 bits each.
     """
 
     def __init__(self, in_features, out_features, bits=1.58, lr=1e-3, betas=(0.9, 0.999),
                  eps=1e-8, weight_decay=0.0, seed=1234, tensor_id=0, init_std=0.02,
-                 init_seed=0, round_mode=0, act="int8", device="cuda"):
+                 init_seed=0, round_mode=0, act="int8", optimizer="adamw", packed=False,
+                 adafactor=None, device="cuda"):
         super().__init__()
         if in_features % 8 or out_features % 8:
             raise ValueError("in_features and out_features must be multiples of 8")
@@ -96,12 +104,19 @@ class DQTBitLinear(torch.nn.Module):
         if act == "fp8" and in_features % 16:
             raise ValueError("the E4M3 forward needs in_features a multiple of 16")
         self.act = act
+        if optimizer not in ("adamw", "adafactor"):
+            raise ValueError("optimizer must be 'adamw' or 'adafactor'")
+        self.optimizer = optimizer
+        self.packed = bool(packed)
+        self.adafactor = dict(adafactor or {})
         self.in_features = in_features
         self.out_features = out_features
         g = dqt.grid(bits)
         self.grid_tuple = (g.qmin, g.qmax)
         if act == "fp8" and (g.qmin < -16 or g.qmax > 16):
             raise ValueError("the E4M3 weight image holds codes up to 16 in magnitude (<= 5 bits)")
+        if self.packed and (g.qmin, g.qmax) != (-1, 1):
+            raise ValueError("packed storage holds ternary codes only")
         self.lr, self.betas, self.eps, self.weight_decay = lr, tuple(betas), eps, weight_decay
         self.round_mode = round_mode
         self.update_in_backward = True
@@ -110,9 +125,16 @@ class DQTBitLinear(torch.nn.Module):
         w0 = (torch.randn(out_features, in_features, generator=gen) * init_std).to(device)
         codes, s_w = dqt.dqt_absmean_init(w0, self.grid_tuple)
         del w0
+        if self.packed:
+            codes = dqt.dqt_pack_ternary(codes)
         self.register_buffer("codes", codes)
-        self.register_buffer("m", torch.zeros(out_features, in_features, device=device))
-        self.register_buffer("v", torch.zeros(out_features, in_features, device=device))
+        if optimizer == "adamw":
+            self.register_buffer("m", torch.zeros(out_features, in_features, device=device))
+            self.register_buffer("v", torch.zeros(out_features, in_features, device=device))
+        else:
+            # Adafactor's factored second moment: row and column means
+            self.register_buffer("R", torch.zeros(out_features, device=device))
+            self.register_buffer("C", torch.zeros(in_features, device=device))
         # changed-code counter (Sec. 5.2 update frequency), accumulated
         self.register_buffer("changed", torch.zeros(1, dtype=torch.int64, device=device))
         self.s_w = float(s_w)
@@ -138,6 +160,25 @@ class DQTBitLinear(torch.nn.Module):
     def forward(self, x):
         return _BitLinearFn.apply(x, self._anchor, self)
 
+    def int8_codes(self):
+        """The codes as an int8 [N, K] tensor (unpacked if stored packed)."""
+        if not self.packed:
+            return self.codes
+        n = self.out_features * self.in_features
+        return dqt.dqt_unpack_ternary(self.codes, n).view(self.out_features, self.in_features)
+
+    def weight_bf16(self):
+        shape = (self.out_features, self.in_features)
+        if self.packed:
+            return dqt.dqt_packed_to_bf16(self.codes, shape)
+        return dqt.dqt_codes_to_bf16(self.codes)
+
+    def weight_fp8(self):
+        shape = (self.out_features, self.in_features)
+        if self.packed:
+            return dqt.dqt_packed_to_fp8(self.codes, shape)
+        return dqt.dqt_codes_to_fp8(self.codes, self.grid_tuple)
+
     def _hyper(self, step):
         hp = dqt.adamw(lr=self.lr, beta1=self.betas[0], beta2=self.betas[1], eps=self.eps,
                        weight_decay=self.weight_decay, step=step)
@@ -148,7 +189,9 @@ class DQTBitLinear(torch.nn.Module):
         """Read the update constants from `dev_row` (a 64-byte row of a device
         block) when the update kernel runs.  The step then advances in
         prepare_step(), not in backward, so that a captured training step
-        replays with a new step each time."""
+        replays with a new step each time (AdamW, int8 codes)."""
+        if self.optimizer != "adamw" or self.packed:
+            raise ValueError("device-resident update constants need AdamW on int8 codes")
         self.uc_dev = dev_row
 
     def prepare_step(self, host_row):
@@ -158,6 +201,22 @@ class DQTBitLinear(torch.nn.Module):
         dqt.dqt_update_consts(hp, sr, self.grid_tuple, self.s_w, out=host_row)
 
     def _dqt_update(self, dy2, xdq):
+        if self.optimizer == "adafactor":
+            self.step += 1
+            hp = dqt.adafactor(lr=self.lr, weight_decay=self.weight_decay, step=self.step,
+                               **self.adafactor)
+            sr = dqt.sr_stream(seed=self.seed, tensor_id=self.tensor_id,
+                               round_mode=self.round_mode)
+            dqt.dqt_bitlinear_bwd_dw_adafactor(dy2, xdq, self.codes, self.s_w, self.R, self.C, hp,
+                                               sr, self.grid_tuple, packed=self.packed,
+                                               changed_out=self.changed)
+            return
+        if self.packed:
+            self.step += 1
+            hp, sr = self._hyper(self.step)
+            dqt.dqt_bitlinear_bwd_dw_update_packed(dy2, xdq, self.codes, self.s_w, self.m, self.v,
+                                                   hp, sr, changed_out=self.changed)
+            return
         if self.uc_dev is not None:
             dqt.dqt_bitlinear_bwd_dw_update_dev(dy2, xdq, self.codes, self.m, self.v, self.uc_dev,
                                                 changed_out=self.changed)
@@ -168,5 +227,6 @@ class DQTBitLinear(torch.nn.Module):
                                         self.grid_tuple, changed_out=self.changed)
 
     def extra_repr(self):
-        return "in_features=%d, out_features=%d, grid=%s, act=%s" % (
-            self.in_features, self.out_features, self.grid_tuple, self.act)
+        return "in_features=%d, out_features=%d, grid=%s, act=%s, optimizer=%s, packed=%s" % (
+            self.in_features, self.out_features, self.grid_tuple, self.act, self.optimizer,
+            self.packed)

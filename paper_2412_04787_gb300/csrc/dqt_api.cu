@@ -382,4 +382,229 @@ int dqt_sr_update_dev(const float* grad, int8_t* W, float* m, float* v, const vo
              : DQT_OK;
 }
 
+// ---- 2-bit packed ternary codes ----------------------------------------------
+int dqt_pack_ternary(const int8_t* codes, int64_t numel, uint8_t* packed, void* stream) {
+  if (!codes || !packed || numel <= 0) return DQT_ERR_ARG;
+  if (!aligned16(codes) || !aligned16(packed)) return DQT_ERR_ALIGN;
+  return dqt::launch_pack_ternary(codes, numel, packed, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
+int dqt_unpack_ternary(const uint8_t* packed, int64_t numel, int8_t* codes, void* stream) {
+  if (!codes || !packed || numel <= 0) return DQT_ERR_ARG;
+  if (!aligned16(codes) || !aligned16(packed)) return DQT_ERR_ALIGN;
+  return dqt::launch_unpack_ternary(packed, numel, codes, as_stream(stream)) ? DQT_ERR_CUDA
+                                                                             : DQT_OK;
+}
+
+int dqt_packed_to_bf16(const uint8_t* packed, int64_t numel, dqt_bf16* W_img, void* stream) {
+  if (!packed || !W_img || numel <= 0) return DQT_ERR_ARG;
+  if (!aligned16(packed) || !aligned16(W_img)) return DQT_ERR_ALIGN;
+  return dqt::launch_packed_to_bf16(packed, numel, W_img, as_stream(stream)) ? DQT_ERR_CUDA
+                                                                             : DQT_OK;
+}
+
+int dqt_packed_to_fp8(const uint8_t* packed, int64_t numel, uint8_t* W8, void* stream) {
+  if (!packed || !W8 || numel <= 0) return DQT_ERR_ARG;
+  if (!aligned16(packed) || !aligned16(W8)) return DQT_ERR_ALIGN;
+  return dqt::launch_packed_to_fp8(packed, numel, W8, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
+int dqt_sr_update_packed(const float* grad, uint8_t* Wp, float s_w, float* m, float* v,
+                         const dqt_adamw_t* hp, const dqt_sr_t* sr, int64_t numel,
+                         unsigned long long* changed_out, void* stream) {
+  if (!grad || !Wp || !m || !v || numel <= 0) return DQT_ERR_ARG;
+  if (!aligned16(grad) || !aligned16(Wp) || !aligned16(m) || !aligned16(v)) return DQT_ERR_ALIGN;
+  dqt::UpdateConsts uc;
+  const dqt_grid_t tern = {-1, 1};
+  const int rc = make_update_consts(hp, sr, tern, s_w, &uc);
+  if (rc != DQT_OK) return rc;
+  return dqt::launch_sr_update(grad, reinterpret_cast<int8_t*>(Wp), m, v, numel, uc, nullptr,
+                               changed_out, as_stream(stream), true)
+             ? DQT_ERR_CUDA
+             : DQT_OK;
+}
+
+int dqt_bitlinear_bwd_dw_update_packed(const dqt_bf16* dY, const dqt_bf16* Xdq, uint8_t* Wp,
+                                       float s_w, float* m, float* v, const dqt_adamw_t* hp,
+                                       const dqt_sr_t* sr, int64_t T, int64_t N, int64_t K,
+                                       float* dW_out, unsigned long long* changed_out, void* ws,
+                                       size_t ws_bytes, void* stream) {
+  if (!dY || !Xdq || !Wp || !m || !v || T <= 0 || N <= 0 || K <= 0) return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
+  if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(Xdq) || !aligned16(Wp) || !aligned16(m) ||
+      !aligned16(v) || (dW_out && !aligned16(dW_out)) || (ws && !aligned16(ws)))
+    return DQT_ERR_ALIGN;
+  dqt::GemmLaunch g{};
+  const dqt_grid_t tern = {-1, 1};
+  const int rc = make_update_consts(hp, sr, tern, s_w, &g.uc);
+  if (rc != DQT_OK) return rc;
+  g.ws = ws;
+  g.ws_bytes = ws ? ws_bytes : 0;
+  g.kind = dqt::GEMM_DW;
+  g.M = static_cast<int>(N);
+  g.N = static_cast<int>(K);
+  g.Kred = static_cast<int>(T);
+  g.A = dY;
+  g.B = Xdq;
+  g.W = reinterpret_cast<int8_t*>(Wp);
+  g.packed = true;
+  g.m = m;
+  g.v = v;
+  g.dW_out = dW_out;
+  g.changed = changed_out;
+  return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
+// ---- Adafactor ------------------------------------------------------------------
+}  // extern "C"
+
+namespace {
+
+int make_adafactor_consts(const dqt_adafactor_t* hp, dqt::AdafactorConsts* h) {
+  if (!hp || hp->step < 1 || !(hp->lr >= 0.0f) || !(hp->eps1 >= 0.0f) || !(hp->eps2 >= 0.0f) ||
+      !(hp->clip_d > 0.0f) || !(hp->decay_rate <= 0.0f) || !isfinite(hp->weight_decay) ||
+      !isfinite(hp->lr))
+    return DQT_ERR_ARG;
+  const double t = static_cast<double>(hp->step);
+  const double p = pow(t, static_cast<double>(hp->decay_rate));
+  h->b2 = static_cast<float>(1.0 - p);
+  h->omb2 = static_cast<float>(p);
+  if (hp->relative_step) {
+    const double cap = hp->warmup_init ? 1e-6 * t : 1e-2;
+    const double inv = 1.0 / sqrt(t);
+    h->rho = static_cast<float>(cap < inv ? cap : inv);
+  } else {
+    h->rho = hp->lr;
+  }
+  h->eps1 = hp->eps1;
+  h->eps2 = hp->eps2;
+  h->clip_d = hp->clip_d;
+  h->weight_decay = hp->weight_decay;
+  h->scale_parameter = hp->scale_parameter ? 1 : 0;
+  return DQT_OK;
+}
+
+int apply_consts(int64_t step_t, const dqt_sr_t* sr, dqt_grid_t grid, dqt::UpdateConsts* uc) {
+  if (!sr || step_t < 1 || !grid_ok(grid)) return DQT_ERR_ARG;
+  if (sr->round_mode != 0 && sr->round_mode != 1) return DQT_ERR_ARG;
+  *uc = dqt::UpdateConsts{};
+  uc->qmin = grid.qmin;
+  uc->qmax = grid.qmax;
+  uc->step_lo = static_cast<uint32_t>(step_t);
+  uc->tensor_id = sr->tensor_id;
+  uc->key0 = static_cast<uint32_t>(sr->seed);
+  uc->key1 = static_cast<uint32_t>(sr->seed >> 32);
+  uc->round_mode = sr->round_mode;
+  return DQT_OK;
+}
+
+inline size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+}  // namespace
+
+extern "C" {
+
+size_t dqt_adafactor_workspace_size(int64_t N, int64_t K) {
+  if (N <= 0 || K <= 0 || N > kMaxDim || K > kMaxDim) return 0;
+  return dqt::adafactor_stats_ws(N, K);
+}
+
+int dqt_adafactor_stats(const float* G, const void* W, int32_t packed, float s_w, float* R,
+                        float* C, const dqt_adafactor_t* hp, int64_t N, int64_t K,
+                        float* scalars_out, void* ws, size_t ws_bytes, void* stream) {
+  if (!G || !W || !R || !C || !scalars_out || !ws || N <= 0 || K <= 0 || !(s_w > 0.0f) ||
+      !isfinite(s_w))
+    return DQT_ERR_ARG;
+  if (N > kMaxDim || K > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
+  if (ws_bytes < dqt::adafactor_stats_ws(N, K)) return DQT_ERR_ARG;
+  if (K % 4 || !aligned16(G) || !aligned16(W) || !aligned16(R) || !aligned16(C) ||
+      !aligned16(scalars_out) || (reinterpret_cast<uintptr_t>(ws) & 255u))
+    return DQT_ERR_ALIGN;
+  dqt::AdafactorConsts h;
+  const int rc = make_adafactor_consts(hp, &h);
+  if (rc != DQT_OK) return rc;
+  return dqt::launch_adafactor_stats(G, static_cast<const int8_t*>(W), packed != 0, s_w, R, C, h,
+                                     N, K, ws, scalars_out, as_stream(stream))
+             ? DQT_ERR_CUDA
+             : DQT_OK;
+}
+
+int dqt_adafactor_apply(const float* G, void* W, int32_t packed, const float* R, const float* C,
+                        const float* scalars, int64_t step_t, const dqt_sr_t* sr, dqt_grid_t grid,
+                        int64_t N, int64_t K, unsigned long long* changed_out, void* stream) {
+  if (!G || !W || !R || !C || !scalars || N <= 0 || K <= 0) return DQT_ERR_ARG;
+  if (N > kMaxDim || K > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
+  if (packed && (grid.qmin != -1 || grid.qmax != 1)) return DQT_ERR_ARG;
+  if (K % 4 || !aligned16(G) || !aligned16(W) || !aligned16(R) || !aligned16(C) ||
+      !aligned16(scalars))
+    return DQT_ERR_ALIGN;
+  dqt::UpdateConsts uc;
+  const int rc = apply_consts(step_t, sr, grid, &uc);
+  if (rc != DQT_OK) return rc;
+  return dqt::launch_adafactor_apply(G, static_cast<int8_t*>(W), packed != 0, R, C, scalars, uc,
+                                     N, K, changed_out, as_stream(stream))
+             ? DQT_ERR_CUDA
+             : DQT_OK;
+}
+
+size_t dqt_bwd_dw_adafactor_workspace_size(int64_t T, int64_t N, int64_t K) {
+  if (T <= 0 || N <= 0 || K <= 0 || T > kMaxDim || N > kMaxDim || K > kMaxDim) return 0;
+  const size_t g = align256(static_cast<size_t>(N) * static_cast<size_t>(K) * 4u);
+  const size_t st = align256(dqt::adafactor_stats_ws(N, K));
+  return g + st + align256(dqt_bwd_dw_workspace_size(T, N, K));
+}
+
+int dqt_bitlinear_bwd_dw_adafactor(const dqt_bf16* dY, const dqt_bf16* Xdq, void* W,
+                                   int32_t packed, float s_w, float* R, float* C,
+                                   const dqt_adafactor_t* hp, const dqt_sr_t* sr, dqt_grid_t grid,
+                                   int64_t T, int64_t N, int64_t K,
+                                   unsigned long long* changed_out, void* ws, size_t ws_bytes,
+                                   void* stream) {
+  if (!dY || !Xdq || !W || !R || !C || !ws || T <= 0 || N <= 0 || K <= 0 || !(s_w > 0.0f) ||
+      !isfinite(s_w))
+    return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
+  if (packed && (grid.qmin != -1 || grid.qmax != 1)) return DQT_ERR_ARG;
+  if (ws_bytes < dqt_bwd_dw_adafactor_workspace_size(T, N, K)) return DQT_ERR_ARG;
+  if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(Xdq) || !aligned16(W) || !aligned16(R) ||
+      !aligned16(C) || (reinterpret_cast<uintptr_t>(ws) & 255u))
+    return DQT_ERR_ALIGN;
+  dqt::AdafactorConsts h;
+  int rc = make_adafactor_consts(hp, &h);
+  if (rc != DQT_OK) return rc;
+  dqt::UpdateConsts uc;
+  rc = apply_consts(hp->step, sr, grid, &uc);
+  if (rc != DQT_OK) return rc;
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  float* G = reinterpret_cast<float*>(base);
+  const size_t g_bytes = align256(static_cast<size_t>(N) * static_cast<size_t>(K) * 4u);
+  void* st_ws = base + g_bytes;
+  const size_t st_bytes = align256(dqt::adafactor_stats_ws(N, K));
+  void* split_ws = base + g_bytes + st_bytes;
+  const size_t split_bytes = ws_bytes - g_bytes - st_bytes;
+  cudaStream_t s = as_stream(stream);
+  // 1. the weight gradient (gradient-only GEMM) into the workspace
+  dqt::GemmLaunch g{};
+  g.kind = dqt::GEMM_DW;
+  g.M = static_cast<int>(N);
+  g.N = static_cast<int>(K);
+  g.Kred = static_cast<int>(T);
+  g.A = dY;
+  g.B = Xdq;
+  g.dW_out = G;
+  g.ws = split_bytes ? split_ws : nullptr;
+  g.ws_bytes = split_bytes;
+  if (dqt::launch_gemm(g, s)) return DQT_ERR_CUDA;
+  // 2. statistics, 3. the per-element step
+  float* scal = reinterpret_cast<float*>(static_cast<uint8_t*>(st_ws) +
+                                         dqt::adafactor_scalars_offset(N, K));
+  if (dqt::launch_adafactor_stats(G, static_cast<const int8_t*>(W), packed != 0, s_w, R, C, h, N,
+                                  K, st_ws, scal, s))
+    return DQT_ERR_CUDA;
+  return dqt::launch_adafactor_apply(G, static_cast<int8_t*>(W), packed != 0, R, C, scal, uc, N, K,
+                                     changed_out, s)
+             ? DQT_ERR_CUDA
+             : DQT_OK;
+}
+
 }  // extern "C"

@@ -383,6 +383,23 @@ struct UpdateConsts {
   int32_t round_mode;
 };
 
+// Eq. 1 on the code-domain value x: floor(x) + 1 with probability x - floor(x),
+// the uniform U = (word >> 8) 2^-24 deciding (round_mode 1: round to nearest,
+// half to even), then the clamp to the grid [qmin, qmax] (Eq. 5).
+__device__ __forceinline__ int32_t sr_round(float x, uint32_t word, int32_t round_mode,
+                                            int32_t qmin, int32_t qmax) {
+  int32_t r;
+  if (round_mode == 1) {
+    r = static_cast<int32_t>(rintf(x));
+  } else {
+    const float f = floorf(x);
+    const float frac = __fsub_rn(x, f);
+    const float U = __fmul_rn(static_cast<float>(word >> 8), 5.9604644775390625e-08f);  // 2^-24
+    r = static_cast<int32_t>(f) + (U < frac ? 1 : 0);
+  }
+  return min(max(r, qmin), qmax);
+}
+
 __device__ __forceinline__ int32_t dqt_update_elem(const UpdateConsts& h, float g, int32_t c,
                                                    float& m, float& v, uint32_t word) {
   const float mn = __fadd_rn(__fmul_rn(h.b1, m), __fmul_rn(h.omb1, g));
@@ -392,16 +409,20 @@ __device__ __forceinline__ int32_t dqt_update_elem(const UpdateConsts& h, float 
   const float den = __fadd_rn(__fmul_rn(__fsqrt_rn(vn), h.k1), h.k2);
   const float u = __fdiv_rn(mn, den);
   const float x = __fsub_rn(__fmul_rn(static_cast<float>(c), h.decay), __fmul_rn(h.lrs, u));
-  int32_t r;
-  if (h.round_mode == 1) {
-    r = static_cast<int32_t>(rintf(x));
-  } else {
-    const float f = floorf(x);
-    const float frac = __fsub_rn(x, f);
-    const float U = __fmul_rn(static_cast<float>(word >> 8), 5.9604644775390625e-08f);  // 2^-24
-    r = static_cast<int32_t>(f) + (U < frac ? 1 : 0);
-  }
-  return min(max(r, h.qmin), h.qmax);
+  return sr_round(x, word, h.round_mode, h.qmin, h.qmax);
+}
+
+// 2-bit packed ternary codes: code e of a tensor is field e % 4 (bits 2 (e % 4)
+// and up) of byte e / 4, a 2-bit two's-complement number (-1 = 3, 0, +1 = 1).
+__device__ __forceinline__ char4 tern_unpack4(uint32_t b) {
+  return make_char4(static_cast<signed char>(static_cast<int32_t>(b << 30) >> 30),
+                    static_cast<signed char>(static_cast<int32_t>(b << 28) >> 30),
+                    static_cast<signed char>(static_cast<int32_t>(b << 26) >> 30),
+                    static_cast<signed char>(static_cast<int32_t>(b << 24) >> 30));
+}
+__device__ __forceinline__ uint32_t tern_pack4(int32_t a, int32_t b, int32_t c, int32_t d) {
+  return (static_cast<uint32_t>(a) & 3u) | ((static_cast<uint32_t>(b) & 3u) << 2) |
+         ((static_cast<uint32_t>(c) & 3u) << 4) | ((static_cast<uint32_t>(d) & 3u) << 6);
 }
 
 }  // namespace dqt

@@ -38,7 +38,8 @@ struct GemmLaunch {
   void* out_bf16;    // FWD: Y; DX: dX
   int32_t* acc_out;  // FWD, optional
   float* acc_f32;    // FWD8, optional
-  int8_t* W;         // DW (with m, v), optional
+  int8_t* W;         // DW (with m, v), optional; 2-bit packed ternary bytes if `packed`
+  bool packed;
   float* m;
   float* v;
   float* dW_out;  // DW, optional
@@ -58,7 +59,7 @@ int dw_splits(int M, int N, int Kred);
 int launch_sr_update_slabs(const float* slabs, int splits, long long slab, int8_t* W, float* m,
                            float* v, int64_t numel, const UpdateConsts& uc,
                            const UpdateConsts* uc_dev, unsigned long long* changed, float* g_out,
-                           cudaStream_t stream);
+                           cudaStream_t stream, bool packed = false);
 // Sum the slabs into out (gradient only).
 int launch_slab_sum(const float* slabs, int splits, long long slab, float* out,
                     cudaStream_t stream);
@@ -78,8 +79,34 @@ int launch_absmean_codes(const float* W0, int64_t numel, float s_w, int32_t qmin
                          int8_t* codes, cudaStream_t stream);
 constexpr int kAbsmeanBlocks = 1024;
 
+// 2-bit packed ternary codes (4 per byte): conversions and operand images.
+int launch_pack_ternary(const int8_t* c, int64_t n, uint8_t* out, cudaStream_t stream);
+int launch_unpack_ternary(const uint8_t* p, int64_t n, int8_t* c, cudaStream_t stream);
+int launch_packed_to_bf16(const uint8_t* p, int64_t n, uint16_t* img, cudaStream_t stream);
+int launch_packed_to_fp8(const uint8_t* p, int64_t n, uint8_t* out, cudaStream_t stream);
+
+// Adafactor (factored second moment, no first moment) host-derived constants.
+struct AdafactorConsts {
+  float b2, omb2, rho, eps1, eps2, clip_d, weight_decay;
+  int32_t scale_parameter;
+};
+// Workspace of the statistics passes for an N x K weight, and the offset of
+// the 8-float scalar block inside it.
+size_t adafactor_stats_ws(int64_t N, int64_t K);
+size_t adafactor_scalars_offset(int64_t N, int64_t K);
+// R, C updated in place; scalars_out (device, 8 floats; NULL = inside ws) gets
+// {Rbar, code-domain step, decay, rms_u, rms_x, alpha}.
+int launch_adafactor_stats(const float* G, const int8_t* W, bool packed, float s_w, float* R,
+                           float* C, const AdafactorConsts& h, int64_t N, int64_t K, void* ws,
+                           float* scalars_out, cudaStream_t stream);
+// The per-element update given R, C and scalars {Rbar, step, decay} (device).
+// Uses the grid, round mode and Philox key/counter fields of uc.
+int launch_adafactor_apply(const float* G, int8_t* W, bool packed, const float* R, const float* C,
+                           const float* scalars, const UpdateConsts& uc, int64_t N, int64_t K,
+                           unsigned long long* changed, cudaStream_t stream);
+
 int launch_sr_update(const float* grad, int8_t* W, float* m, float* v, int64_t numel,
                      const UpdateConsts& uc, const UpdateConsts* uc_dev,
-                     unsigned long long* changed, cudaStream_t stream);
+                     unsigned long long* changed, cudaStream_t stream, bool packed = false);
 
 }  // namespace dqt

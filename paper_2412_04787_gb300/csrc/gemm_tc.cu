@@ -61,6 +61,7 @@ struct Params {
   int32_t* acc_out;
   float* acc_f32;  // FP8 forward: optional fp32 accumulators
   int8_t* W;
+  bool packed;  // W holds 2-bit packed ternary codes (one byte per 4 weights)
   float* m;
   float* v;
   float* dW_out;
@@ -199,6 +200,7 @@ struct DwLoads {
   char4 c[4];
 };
 
+template <bool PK>
 __device__ __forceinline__ void dw_issue(const Params& p, int row0, int gn0, int h, int lane,
                                          DwLoads& L) {
   const int gk = gn0 + (lane & 7) * 4;
@@ -208,13 +210,15 @@ __device__ __forceinline__ void dw_issue(const Params& p, int row0, int gn0, int
     const int gm = row0 + (lane >> 3) + 4 * (4 * h + j);
     if (gm < p.M) {
       const size_t e = static_cast<size_t>(gm) * p.N + gk;
-      L.c[j] = __ldcs(reinterpret_cast<const char4*>(p.W + e));
+      L.c[j] = PK ? tern_unpack4(__ldcs(reinterpret_cast<const uint8_t*>(p.W) + (e >> 2)))
+                  : __ldcs(reinterpret_cast<const char4*>(p.W + e));
       L.m[j] = __ldcs(reinterpret_cast<const float4*>(p.m + e));
       L.v[j] = __ldcs(reinterpret_cast<const float4*>(p.v + e));
     }
   }
 }
 
+template <bool PK>
 __device__ __forceinline__ uint32_t dw_update(const Params& p, const UpdateConsts& uc,
                                               float* dw_out, int row0, int gn0, int h, int lane,
                                               const float* xp, DwLoads& L) {
@@ -240,9 +244,13 @@ __device__ __forceinline__ uint32_t dw_update(const Params& p, const UpdateConst
     const int32_t n2c = dqt_update_elem(uc, g4.z, L.c[j].z, L.m[j].z, L.v[j].z, w.z);
     const int32_t n3c = dqt_update_elem(uc, g4.w, L.c[j].w, L.m[j].w, L.v[j].w, w.w);
     n_changed += (n0c != L.c[j].x) + (n1c != L.c[j].y) + (n2c != L.c[j].z) + (n3c != L.c[j].w);
-    __stcs(reinterpret_cast<char4*>(p.W + e),
-           make_char4(static_cast<signed char>(n0c), static_cast<signed char>(n1c),
-                      static_cast<signed char>(n2c), static_cast<signed char>(n3c)));
+    if (PK)
+      __stcs(reinterpret_cast<uint8_t*>(p.W) + (e >> 2),
+             static_cast<uint8_t>(tern_pack4(n0c, n1c, n2c, n3c)));
+    else
+      __stcs(reinterpret_cast<char4*>(p.W + e),
+             make_char4(static_cast<signed char>(n0c), static_cast<signed char>(n1c),
+                        static_cast<signed char>(n2c), static_cast<signed char>(n3c)));
     __stcs(reinterpret_cast<float4*>(p.m + e), L.m[j]);
     __stcs(reinterpret_cast<float4*>(p.v + e), L.v[j]);
   }
@@ -253,14 +261,15 @@ __device__ __forceinline__ uint32_t dw_update(const Params& p, const UpdateConst
 // columns starting at column nbase, rows row0 .. row0 + 31, gradient in
 // tensor memory at t_acc (this warp's lanes, chunk cc at column 32 cc).
 // With PIPE the next half-chunk's loads are in flight while the current one
-// is updated (more registers, for kernels with few epilogue warps).
-template <bool PIPE>
+// is updated (more registers, for kernels with few epilogue warps).  PK: the
+// codes are 2-bit packed ternary (one byte per lane and row).
+template <bool PIPE, bool PK>
 __device__ __forceinline__ uint32_t epi_dw_tile(const Params& p, const UpdateConsts& uc,
                                                 float* dw_out, int row0, int nbase, int nchunk,
                                                 uint32_t t_acc, float* xp, int lane) {
   uint32_t n_changed = 0;
   DwLoads A, B;
-  if (PIPE) dw_issue(p, row0, nbase, 0, lane, A);
+  if (PIPE) dw_issue<PK>(p, row0, nbase, 0, lane, A);
 #pragma unroll 1
   for (int cc = 0; cc < nchunk; ++cc) {
     const int gn0 = nbase + cc * 32;
@@ -271,15 +280,15 @@ __device__ __forceinline__ uint32_t epi_dw_tile(const Params& p, const UpdateCon
     for (int i = 0; i < 32; ++i) xp[lane * kStageLd + i] = __uint_as_float(a[i]);
     __syncwarp();
     if (PIPE) {
-      dw_issue(p, row0, gn0, 1, lane, B);
-      n_changed += dw_update(p, uc, dw_out, row0, gn0, 0, lane, xp, A);
-      if (cc + 1 < nchunk) dw_issue(p, row0, gn0 + 32, 0, lane, A);
-      n_changed += dw_update(p, uc, dw_out, row0, gn0, 1, lane, xp, B);
+      dw_issue<PK>(p, row0, gn0, 1, lane, B);
+      n_changed += dw_update<PK>(p, uc, dw_out, row0, gn0, 0, lane, xp, A);
+      if (cc + 1 < nchunk) dw_issue<PK>(p, row0, gn0 + 32, 0, lane, A);
+      n_changed += dw_update<PK>(p, uc, dw_out, row0, gn0, 1, lane, xp, B);
     } else {
 #pragma unroll 1
       for (int h = 0; h < 2; ++h) {
-        dw_issue(p, row0, gn0, h, lane, A);
-        n_changed += dw_update(p, uc, dw_out, row0, gn0, h, lane, xp, A);
+        dw_issue<PK>(p, row0, gn0, h, lane, A);
+        n_changed += dw_update<PK>(p, uc, dw_out, row0, gn0, h, lane, xp, A);
       }
     }
     __syncwarp();  // the transpose buffer is rewritten for the next chunk
@@ -454,7 +463,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t t_run = tmem + lane_off + RUN_COL + static_cast<uint32_t>(half * HALF);
         const bool last = (c + 1 == nchunks);
         if (EPI == GEMM_DW) {
-          n_changed += epi_dw_tile<true>(p, uc, p.dW_out, gm - lane, nbase, HALF / 32, t_acc, xp, lane);
+          n_changed += epi_dw_tile<true, false>(p, uc, p.dW_out, gm - lane, nbase, HALF / 32, t_acc, xp, lane);
         } else
 #pragma unroll 1
         for (int cc = 0; cc < HALF / 32; ++cc) {
@@ -537,7 +546,7 @@ struct SmemPair {
   static_assert((2 * STAGES + 5) * 8 + 4 <= 176, "barrier area: barriers, then the update constants");
 };
 
-template <bool A_MN, bool B_MN, int EPI>
+template <bool A_MN, bool B_MN, int EPI, bool PK = false>
 __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
     gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA,
                      const __grid_constant__ CUtensorMap tmB, const Params p) {
@@ -723,7 +732,7 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
       tc_fence_after();
       const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(b * BN + half * HALF);
       if (EPI == GEMM_DW) {
-        n_changed += epi_dw_tile<false>(p, uc, dw_out, gm - lane, nbase, HALF / 32, t_acc, xp, lane);
+        n_changed += epi_dw_tile<false, PK>(p, uc, dw_out, gm - lane, nbase, HALF / 32, t_acc, xp, lane);
       } else
 #pragma unroll 1
       for (int cc = 0; cc < HALF / 32; ++cc) {
@@ -817,7 +826,7 @@ int launch_tiles(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStr
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
-template <bool A_MN, bool B_MN, int EPI>
+template <bool A_MN, bool B_MN, int EPI, bool PK = false>
 int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream);
 
 }  // namespace
@@ -841,9 +850,9 @@ int dw_splits(int M, int N, int Kred) {
 
 namespace {
 
-template <bool A_MN, bool B_MN, int EPI>
+template <bool A_MN, bool B_MN, int EPI, bool PK>
 int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream) {
-  auto kern = gemm_pair_kernel<A_MN, B_MN, EPI>;
+  auto kern = gemm_pair_kernel<A_MN, B_MN, EPI, PK>;
   const int smem = SmemPair<EPI>::BYTES;
   constexpr int threads = PairCfg<EPI>::THREADS;
   static int max_clusters = 0;  // per template instance
@@ -895,7 +904,8 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   }
   const bool drain = p.chunk_kb < p.num_kb;
   GemmLaunch gl = g;
-  gl.pair = !drain && gemm_mode() == 0;
+  // packed codes: the 2-SM kernel whatever the tiling mode
+  gl.pair = !drain && (gemm_mode() == 0 || g.packed);
   const GemmLaunch& g2 = gl;
   p.splits = 1;
   p.kb_per_split = p.num_kb;
@@ -917,6 +927,7 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   p.acc_out = g.acc_out;
   p.acc_f32 = g.acc_f32;
   p.W = g.W;
+  p.packed = g.packed;
   p.m = g.m;
   p.v = g.v;
   p.dW_out = g.dW_out;
@@ -949,7 +960,9 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
       if (!make_map(&ta, g.A, g.M, g.Kred, 64, BK)) return 3;
       if (!make_map(&tb, g.B, g.N, g.Kred, 64, BK)) return 3;
       if (!g2.pair) return launch_tiles<256, true, true, GEMM_DW, false>(ta, tb, p, stream);
-      if (p.splits == 1) return launch_pairs<true, true, GEMM_DW>(ta, tb, p, stream);
+      if (p.splits == 1)
+        return p.packed && p.W ? launch_pairs<true, true, GEMM_DW, true>(ta, tb, p, stream)
+                               : launch_pairs<true, true, GEMM_DW>(ta, tb, p, stream);
       // split-T: fp32 partials of each token slice into the workspace slabs,
       // then one streaming pass sums the slabs in slice order and applies the
       // AdamW + stochastic-rounding update (and writes the summed gradient to
@@ -968,7 +981,8 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
                                stream);
       }
       return launch_sr_update_slabs(static_cast<const float*>(g.ws), p.splits, p.slab, g.W, g.m,
-                                    g.v, p.slab, g.uc, g.uc_dev, g.changed, g.dW_out, stream);
+                                    g.v, p.slab, g.uc, g.uc_dev, g.changed, g.dW_out, stream,
+                                    g.packed);
     }
   }
   return 1;

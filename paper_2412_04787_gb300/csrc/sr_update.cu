@@ -4,7 +4,8 @@
 //
 // Each thread step handles one group of four consecutive weights, which is
 // exactly one Philox4x32-10 block (element e uses word e % 4 of block e / 4),
-// with 16-byte loads and stores of g, m, v and a 4-byte access to the codes.
+// with 16-byte loads and stores of g, m, v and a 4-byte access to the codes
+// (one byte when the codes are 2-bit packed ternary: a group is one byte).
 #include "dqt_internal.h"
 
 namespace dqt {
@@ -40,7 +41,9 @@ __global__ void __launch_bounds__(kThreads)
     sr_update_kernel(const float* __restrict__ grad, int nsplit, long long slab,
                      float* __restrict__ g_out, int8_t* __restrict__ W, float* __restrict__ m,
                      float* __restrict__ v, int64_t numel, const UpdateConsts uc_arg,
-                     const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed) {
+                     const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed,
+                     bool packed) {
+  uint8_t* Wp = reinterpret_cast<uint8_t*>(W);
   const UpdateConsts uc = uc_dev ? *uc_dev : uc_arg;
   const int64_t ngroups = numel >> 2;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * kThreads;
@@ -52,7 +55,7 @@ __global__ void __launch_bounds__(kThreads)
     if (g_out) __stcs(reinterpret_cast<float4*>(g_out + e), g4);
     float4 m4 = __ldcs(reinterpret_cast<const float4*>(m + e));
     float4 v4 = __ldcs(reinterpret_cast<const float4*>(v + e));
-    const char4 c4 = *reinterpret_cast<const char4*>(W + e);
+    const char4 c4 = packed ? tern_unpack4(Wp[gi]) : *reinterpret_cast<const char4*>(W + e);
     uint4 w = make_uint4(0, 0, 0, 0);
     if (uc.round_mode == 0) w = sr_words(static_cast<uint64_t>(gi), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
     const int32_t a = dqt_update_elem(uc, g4.x, c4.x, m4.x, v4.x, w.x);
@@ -60,9 +63,12 @@ __global__ void __launch_bounds__(kThreads)
     const int32_t c = dqt_update_elem(uc, g4.z, c4.z, m4.z, v4.z, w.z);
     const int32_t d = dqt_update_elem(uc, g4.w, c4.w, m4.w, v4.w, w.w);
     n_changed += (a != c4.x) + (b != c4.y) + (c != c4.z) + (d != c4.w);
-    *reinterpret_cast<char4*>(W + e) =
-        make_char4(static_cast<signed char>(a), static_cast<signed char>(b),
-                   static_cast<signed char>(c), static_cast<signed char>(d));
+    if (packed)
+      Wp[gi] = static_cast<uint8_t>(tern_pack4(a, b, c, d));
+    else
+      *reinterpret_cast<char4*>(W + e) =
+          make_char4(static_cast<signed char>(a), static_cast<signed char>(b),
+                     static_cast<signed char>(c), static_cast<signed char>(d));
     __stcs(reinterpret_cast<float4*>(m + e), m4);
     __stcs(reinterpret_cast<float4*>(v + e), v4);
   }
@@ -72,17 +78,22 @@ __global__ void __launch_bounds__(kThreads)
     uint4 w = make_uint4(0, 0, 0, 0);
     if (uc.round_mode == 0) w = sr_words(static_cast<uint64_t>(gi), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
     const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+    const char4 pc = packed ? tern_unpack4(Wp[gi]) : make_char4(0, 0, 0, 0);
+    int32_t pr[4] = {0, 0, 0, 0};  // packed: the unused fields of the last byte stay 0
     for (int64_t e = gi << 2; e < numel; ++e) {
       float mm = m[e], vv = v[e];
-      const int32_t c0 = W[e];
+      const int j = static_cast<int>(e & 3);
+      const int32_t c0 = packed ? (j == 0 ? pc.x : j == 1 ? pc.y : pc.z) : W[e];
       const float g = slab_grad1(grad, nsplit, slab, e);
       if (g_out) g_out[e] = g;
-      const int32_t r = dqt_update_elem(uc, g, c0, mm, vv, ws[e & 3]);
+      const int32_t r = dqt_update_elem(uc, g, c0, mm, vv, ws[j]);
       n_changed += (r != c0);
-      W[e] = static_cast<int8_t>(r);
+      if (packed) pr[j] = r;
+      else W[e] = static_cast<int8_t>(r);
       m[e] = mm;
       v[e] = vv;
     }
+    if (packed) Wp[gi] = static_cast<uint8_t>(tern_pack4(pr[0], pr[1], pr[2], pr[3]));
   }
   if (changed) {
 #pragma unroll
@@ -121,9 +132,10 @@ int stream_blocks(int64_t numel) {
 int launch_sr_update_slabs(const float* slabs, int splits, long long slab, int8_t* W, float* m,
                            float* v, int64_t numel, const UpdateConsts& uc,
                            const UpdateConsts* uc_dev, unsigned long long* changed, float* g_out,
-                           cudaStream_t stream) {
+                           cudaStream_t stream, bool packed) {
   sr_update_kernel<<<stream_blocks(numel), kThreads, 0, stream>>>(slabs, splits, slab, g_out, W, m,
-                                                                  v, numel, uc, uc_dev, changed);
+                                                                  v, numel, uc, uc_dev, changed,
+                                                                  packed);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
@@ -135,9 +147,10 @@ int launch_slab_sum(const float* slabs, int splits, long long slab, float* out,
 
 int launch_sr_update(const float* grad, int8_t* W, float* m, float* v, int64_t numel,
                      const UpdateConsts& uc, const UpdateConsts* uc_dev,
-                     unsigned long long* changed, cudaStream_t stream) {
+                     unsigned long long* changed, cudaStream_t stream, bool packed) {
   sr_update_kernel<<<stream_blocks(numel), kThreads, 0, stream>>>(grad, 1, 0, nullptr, W, m, v,
-                                                                  numel, uc, uc_dev, changed);
+                                                                  numel, uc, uc_dev, changed,
+                                                                  packed);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 

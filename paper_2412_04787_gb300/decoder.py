@@ -30,9 +30,11 @@ __all__ = ["DecoderConfig", "DQTDecoder"]
 
 class DecoderConfig:
     def __init__(self, layers=12, hidden=768, heads=12, ffn=2048, vocab=32000, bits=1.58,
-                 lr=1e-3, seed=1234, rope_theta=10000.0, norm_eps=1e-6, act="int8"):
+                 lr=1e-3, seed=1234, rope_theta=10000.0, norm_eps=1e-6, act="int8",
+                 optimizer="adamw", packed=False):
         self.layers, self.hidden, self.heads, self.ffn, self.vocab = layers, hidden, heads, ffn, vocab
         self.bits, self.lr, self.seed, self.act = bits, lr, seed, act
+        self.optimizer, self.packed = optimizer, packed
         self.rope_theta, self.norm_eps = rope_theta, norm_eps
 
 
@@ -66,7 +68,8 @@ class Block(torch.nn.Module):
         def bl(k, n, j):
             tid = index * 8 + j  # distinct Philox stream and initial draw per weight
             return DQTBitLinear(k, n, bits=cfg.bits, lr=cfg.lr, seed=cfg.seed, tensor_id=tid,
-                                init_seed=cfg.seed * 1000 + tid, act=cfg.act, device=device)
+                                init_seed=cfg.seed * 1000 + tid, act=cfg.act,
+                                optimizer=cfg.optimizer, packed=cfg.packed, device=device)
 
         self.q, self.k, self.v, self.o = bl(h, h, 0), bl(h, h, 1), bl(h, h, 2), bl(h, h, 3)
         self.gate, self.up, self.down = bl(h, f, 4), bl(h, f, 5), bl(f, h, 6)

@@ -24,6 +24,10 @@ EXPORTED = [
     "dqt_set_gemm_tiles", "dqt_update_consts_size", "dqt_update_consts",
     "dqt_bitlinear_bwd_dw_update_dev", "dqt_sr_update_dev", "dqt_bwd_dw_workspace_size",
     "dqt_act_quant_fp8", "dqt_codes_to_fp8", "dqt_bitlinear_fwd_fp8",
+    "dqt_pack_ternary", "dqt_unpack_ternary", "dqt_packed_to_bf16", "dqt_packed_to_fp8",
+    "dqt_sr_update_packed", "dqt_bitlinear_bwd_dw_update_packed",
+    "dqt_adafactor_workspace_size", "dqt_adafactor_stats", "dqt_adafactor_apply",
+    "dqt_bwd_dw_adafactor_workspace_size", "dqt_bitlinear_bwd_dw_adafactor",
 ]
 
 
@@ -44,6 +48,13 @@ class dqt_adamw_t(C.Structure):
 
 class dqt_sr_t(C.Structure):
     _fields_ = [("seed", C.c_uint64), ("tensor_id", C.c_uint32), ("round_mode", C.c_int32)]
+
+
+class dqt_adafactor_t(C.Structure):
+    _fields_ = [("lr", C.c_float), ("eps1", C.c_float), ("eps2", C.c_float),
+                ("clip_d", C.c_float), ("decay_rate", C.c_float), ("weight_decay", C.c_float),
+                ("step", C.c_int64), ("relative_step", C.c_int32),
+                ("scale_parameter", C.c_int32), ("warmup_init", C.c_int32), ("pad", C.c_int32)]
 
 
 _vp, _i64, _f32, _sz = C.c_void_p, C.c_int64, C.c_float, C.c_size_t
@@ -93,9 +104,33 @@ def lib():
         L.dqt_codes_to_fp8.argtypes = [_vp, _i64, dqt_grid_t, _vp, _vp]
         L.dqt_bitlinear_fwd_fp8.argtypes = [_vp, _vp, _vp, _f32, dqt_grid_t, _i64, _i64, _i64,
                                             _vp, _vp, _vp]
+        for name in ("dqt_pack_ternary", "dqt_unpack_ternary", "dqt_packed_to_bf16",
+                     "dqt_packed_to_fp8"):
+            getattr(L, name).argtypes = [_vp, _i64, _vp, _vp]
+        L.dqt_sr_update_packed.argtypes = [_vp, _vp, _f32, _vp, _vp, C.POINTER(dqt_adamw_t),
+                                           C.POINTER(dqt_sr_t), _i64, _vp, _vp]
+        L.dqt_bitlinear_bwd_dw_update_packed.argtypes = [_vp, _vp, _vp, _f32, _vp, _vp,
+                                                         C.POINTER(dqt_adamw_t),
+                                                         C.POINTER(dqt_sr_t), _i64, _i64, _i64,
+                                                         _vp, _vp, _vp, _sz, _vp]
+        L.dqt_adafactor_workspace_size.argtypes = [_i64, _i64]
+        L.dqt_adafactor_workspace_size.restype = _sz
+        L.dqt_adafactor_stats.argtypes = [_vp, _vp, C.c_int32, _f32, _vp, _vp,
+                                          C.POINTER(dqt_adafactor_t), _i64, _i64, _vp, _vp, _sz,
+                                          _vp]
+        L.dqt_adafactor_apply.argtypes = [_vp, _vp, C.c_int32, _vp, _vp, _vp, _i64,
+                                          C.POINTER(dqt_sr_t), dqt_grid_t, _i64, _i64, _vp, _vp]
+        L.dqt_bwd_dw_adafactor_workspace_size.argtypes = [_i64, _i64, _i64]
+        L.dqt_bwd_dw_adafactor_workspace_size.restype = _sz
+        L.dqt_bitlinear_bwd_dw_adafactor.argtypes = [_vp, _vp, _vp, C.c_int32, _f32, _vp, _vp,
+                                                     C.POINTER(dqt_adafactor_t),
+                                                     C.POINTER(dqt_sr_t), dqt_grid_t, _i64, _i64,
+                                                     _i64, _vp, _vp, _sz, _vp]
         for name in EXPORTED:
             if name not in ("dqt_status_string", "dqt_absmean_workspace_size",
-                            "dqt_update_consts_size", "dqt_bwd_dw_workspace_size"):
+                            "dqt_update_consts_size", "dqt_bwd_dw_workspace_size",
+                            "dqt_adafactor_workspace_size",
+                            "dqt_bwd_dw_adafactor_workspace_size"):
                 getattr(L, name).restype = C.c_int
         _lib = L
     return _lib
@@ -408,3 +443,172 @@ def dqt_bitlinear_fwd_fp8(Xq8, s_x8, W8, s_w, bits_or_grid, Y=None, acc_out=None
                                        _grid(bits_or_grid), T, K, N, _ptr(Y), _ptr(acc_out),
                                        _stream(stream)), "dqt_bitlinear_fwd_fp8")
     return Y
+
+
+# --------------------------------------------------------------------------
+# 2-bit packed ternary codes (uint8 tensors of ceil(numel / 4) bytes)
+# --------------------------------------------------------------------------
+def packed_size(numel):
+    return (int(numel) + 3) // 4
+
+
+def dqt_pack_ternary(codes, packed=None, stream=None):
+    _need(codes, "codes", torch.int8)
+    n = codes.numel()
+    if packed is None:
+        packed = torch.empty(packed_size(n), dtype=torch.uint8, device=codes.device)
+    _need(packed, "packed", torch.uint8, (packed_size(n),))
+    _check(lib().dqt_pack_ternary(_ptr(codes), n, _ptr(packed), _stream(stream)),
+           "dqt_pack_ternary")
+    return packed
+
+
+def dqt_unpack_ternary(packed, numel, codes=None, stream=None):
+    _need(packed, "packed", torch.uint8, (packed_size(numel),))
+    if codes is None:
+        codes = torch.empty(int(numel), dtype=torch.int8, device=packed.device)
+    _need(codes, "codes", torch.int8)
+    if codes.numel() != numel:
+        raise ValueError("codes must hold numel elements")
+    _check(lib().dqt_unpack_ternary(_ptr(packed), int(numel), _ptr(codes), _stream(stream)),
+           "dqt_unpack_ternary")
+    return codes
+
+
+def _numel(shape):
+    n = 1
+    for d in shape:
+        n *= int(d)
+    return n
+
+
+def dqt_packed_to_bf16(packed, shape, W_img=None, stream=None):
+    n = _numel(shape)
+    _need(packed, "packed", torch.uint8, (packed_size(n),))
+    if W_img is None:
+        W_img = torch.empty(tuple(shape), dtype=torch.bfloat16, device=packed.device)
+    _need(W_img, "W_img", torch.bfloat16, tuple(shape))
+    _check(lib().dqt_packed_to_bf16(_ptr(packed), n, _ptr(W_img), _stream(stream)),
+           "dqt_packed_to_bf16")
+    return W_img
+
+
+def dqt_packed_to_fp8(packed, shape, W8=None, stream=None):
+    n = _numel(shape)
+    _need(packed, "packed", torch.uint8, (packed_size(n),))
+    if W8 is None:
+        W8 = torch.empty(tuple(shape), dtype=torch.uint8, device=packed.device)
+    _need(W8, "W8", torch.uint8, tuple(shape))
+    _check(lib().dqt_packed_to_fp8(_ptr(packed), n, _ptr(W8), _stream(stream)),
+           "dqt_packed_to_fp8")
+    return W8
+
+
+def dqt_sr_update_packed(grad, Wp, s_w, m, v, hp, sr, changed_out=None, stream=None):
+    _need(grad, "grad", torch.float32)
+    n = grad.numel()
+    _need(Wp, "Wp", torch.uint8, (packed_size(n),))
+    _need(m, "m", torch.float32)
+    _need(v, "v", torch.float32)
+    if m.numel() != n or v.numel() != n:
+        raise ValueError("m and v must have grad's size")
+    _opt(changed_out, "changed_out", torch.int64, None)
+    _check(lib().dqt_sr_update_packed(_ptr(grad), _ptr(Wp), float(s_w), _ptr(m), _ptr(v),
+                                      C.byref(hp), C.byref(sr), n, _ptr(changed_out),
+                                      _stream(stream)), "dqt_sr_update_packed")
+
+
+def dqt_bitlinear_bwd_dw_update_packed(dY, Xdq, Wp, s_w, m, v, hp, sr, dW_out=None,
+                                       changed_out=None, ws=None, stream=None):
+    _need(dY, "dY", torch.bfloat16)
+    T, N = dY.shape
+    _need(Xdq, "Xdq", torch.bfloat16)
+    K = Xdq.shape[1]
+    _need(Xdq, "Xdq", torch.bfloat16, (T, K))
+    _need(Wp, "Wp", torch.uint8, (packed_size(N * K),))
+    _need(m, "m", torch.float32, (N, K))
+    _need(v, "v", torch.float32, (N, K))
+    _opt(dW_out, "dW_out", torch.float32, (N, K))
+    _opt(changed_out, "changed_out", torch.int64, None)
+    ws_t, ws_n = _dw_workspace(T, N, K, dY.device, ws)
+    _check(lib().dqt_bitlinear_bwd_dw_update_packed(
+        _ptr(dY), _ptr(Xdq), _ptr(Wp), float(s_w), _ptr(m), _ptr(v), C.byref(hp), C.byref(sr),
+        T, N, K, _ptr(dW_out), _ptr(changed_out), _ptr(ws_t), ws_n, _stream(stream)),
+        "dqt_bitlinear_bwd_dw_update_packed")
+
+
+# --------------------------------------------------------------------------
+# Adafactor with stochastic rounding
+# --------------------------------------------------------------------------
+def adafactor(lr=1e-3, eps1=1e-30, eps2=1e-3, clip_d=1.0, decay_rate=-0.8, weight_decay=0.0,
+              step=1, relative_step=False, scale_parameter=False, warmup_init=False):
+    return dqt_adafactor_t(lr, eps1, eps2, clip_d, decay_rate, weight_decay, step,
+                           int(relative_step), int(scale_parameter), int(warmup_init), 0)
+
+
+def _codes_arg(W, packed, N, K):
+    if packed:
+        _need(W, "W", torch.uint8, (packed_size(N * K),))
+    else:
+        _need(W, "W", torch.int8, (N, K))
+
+
+def dqt_adafactor_stats(G, W, s_w, R, C_, hp, packed=False, scalars_out=None, ws=None,
+                        stream=None):
+    """Returns the device scalars {Rbar, step, decay, rms_u, rms_x, alpha, 0, 0}."""
+    _need(G, "G", torch.float32)
+    N, K = G.shape
+    _codes_arg(W, packed, N, K)
+    _need(R, "R", torch.float32, (N,))
+    _need(C_, "C", torch.float32, (K,))
+    if scalars_out is None:
+        scalars_out = torch.zeros(8, dtype=torch.float32, device=G.device)
+    _need(scalars_out, "scalars_out", torch.float32, (8,))
+    nb = lib().dqt_adafactor_workspace_size(N, K)
+    if ws is None:
+        ws = torch.empty(nb, dtype=torch.uint8, device=G.device)
+    _need(ws, "ws", torch.uint8)
+    _check(lib().dqt_adafactor_stats(_ptr(G), _ptr(W), int(packed), float(s_w), _ptr(R),
+                                     _ptr(C_), C.byref(hp), N, K, _ptr(scalars_out), _ptr(ws),
+                                     ws.numel(), _stream(stream)), "dqt_adafactor_stats")
+    return scalars_out
+
+
+def dqt_adafactor_apply(G, W, R, C_, scalars, step_t, sr, bits_or_grid, packed=False,
+                        changed_out=None, stream=None):
+    _need(G, "G", torch.float32)
+    N, K = G.shape
+    _codes_arg(W, packed, N, K)
+    _need(R, "R", torch.float32, (N,))
+    _need(C_, "C", torch.float32, (K,))
+    _need(scalars, "scalars", torch.float32)
+    _opt(changed_out, "changed_out", torch.int64, None)
+    _check(lib().dqt_adafactor_apply(_ptr(G), _ptr(W), int(packed), _ptr(R), _ptr(C_),
+                                     _ptr(scalars), int(step_t), C.byref(sr),
+                                     _grid(bits_or_grid), N, K, _ptr(changed_out),
+                                     _stream(stream)), "dqt_adafactor_apply")
+
+
+def dqt_bwd_dw_adafactor_workspace_size(T, N, K):
+    return int(lib().dqt_bwd_dw_adafactor_workspace_size(T, N, K))
+
+
+def dqt_bitlinear_bwd_dw_adafactor(dY, Xdq, W, s_w, R, C_, hp, sr, bits_or_grid, packed=False,
+                                   changed_out=None, ws=None, stream=None):
+    _need(dY, "dY", torch.bfloat16)
+    T, N = dY.shape
+    _need(Xdq, "Xdq", torch.bfloat16)
+    K = Xdq.shape[1]
+    _need(Xdq, "Xdq", torch.bfloat16, (T, K))
+    _codes_arg(W, packed, N, K)
+    _need(R, "R", torch.float32, (N,))
+    _need(C_, "C", torch.float32, (K,))
+    _opt(changed_out, "changed_out", torch.int64, None)
+    if ws is None:
+        ws = torch.empty(dqt_bwd_dw_adafactor_workspace_size(T, N, K), dtype=torch.uint8,
+                         device=dY.device)
+    _need(ws, "ws", torch.uint8)
+    _check(lib().dqt_bitlinear_bwd_dw_adafactor(
+        _ptr(dY), _ptr(Xdq), _ptr(W), int(packed), float(s_w), _ptr(R), _ptr(C_), C.byref(hp),
+        C.byref(sr), _grid(bits_or_grid), T, N, K, _ptr(changed_out), _ptr(ws), ws.numel(),
+        _stream(stream)), "dqt_bitlinear_bwd_dw_adafactor")

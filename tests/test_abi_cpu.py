@@ -128,3 +128,39 @@ def test_fp8_argument_validation(L):
     assert L.dqt_bitlinear_fwd_fp8(A, A, A, 1.0, t, 4, 32, 12, A, None, None) == dqt.DQT_ERR_ALIGN
     assert L.dqt_bitlinear_fwd_fp8(A, A, A, 0.0, t, 4, 32, 8, A, None, None) == dqt.DQT_ERR_ARG
     assert L.dqt_bitlinear_fwd_fp8(None, A, A, 1.0, t, 4, 32, 8, A, None, None) == dqt.DQT_ERR_ARG
+
+
+def test_packed_and_adafactor_argument_validation(L):
+    A = _p(0x10000)
+    g = dqt.dqt_grid_t(-1, 1)
+    hp = dqt.adamw()
+    sr = dqt.sr_stream()
+    af = dqt.adafactor()
+    assert L.dqt_pack_ternary(None, 16, A, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_pack_ternary(_p(0x10004), 16, A, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_unpack_ternary(A, 0, A, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_packed_to_bf16(A, 16, _p(0x10002), None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_sr_update_packed(A, A, 1.0, A, None, C.byref(hp), C.byref(sr), 16, None,
+                                  None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_bwd_dw_update_packed(A, A, A, 1.0, A, A, C.byref(hp), C.byref(sr), 4,
+                                                8, 12, None, None, None, 0, None) == dqt.DQT_ERR_ALIGN
+    # Adafactor: workspace size, hyper-parameters, packed codes need the ternary grid
+    assert L.dqt_adafactor_workspace_size(64, 64) > 0
+    assert L.dqt_adafactor_workspace_size(0, 64) == 0
+    assert L.dqt_bwd_dw_adafactor_workspace_size(128, 64, 64) >= 64 * 64 * 4
+    nb = L.dqt_adafactor_workspace_size(64, 64)
+    W = _p(0x100000)  # 256-byte aligned
+    assert L.dqt_adafactor_stats(A, A, 0, 1.0, A, A, C.byref(dqt.adafactor(step=0)), 64, 64, A, W,
+                                 nb, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_adafactor_stats(A, A, 0, 1.0, A, A, C.byref(dqt.adafactor(clip_d=0.0)), 64, 64,
+                                 A, W, nb, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_adafactor_stats(A, A, 0, 1.0, A, A, C.byref(af), 64, 64, A, W, nb - 1,
+                                 None) == dqt.DQT_ERR_ARG
+    assert L.dqt_adafactor_stats(A, A, 0, 1.0, A, A, C.byref(af), 64, 64, A, _p(0x10010), nb,
+                                 None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_adafactor_apply(A, A, 1, A, A, A, 1, C.byref(sr), dqt.dqt_grid_t(-2, 1), 64, 64,
+                                 None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_adafactor_apply(A, A, 0, A, A, A, 0, C.byref(sr), g, 64, 64, None,
+                                 None) == dqt.DQT_ERR_ARG
+    assert L.dqt_adafactor_apply(A, A, 0, A, A, A, 1, C.byref(sr), g, 64, 66, None,
+                                 None) == dqt.DQT_ERR_ALIGN

@@ -90,18 +90,18 @@ def test_bitlinear_state_dict_resume():
         assert torch.equal(getattr(a, name), getattr(b, name)), name
 
 
-def _train(bits_w, round_mode=0, steps=40, act="int8"):
+def _train(bits_w, round_mode=0, steps=40, act="int8", optimizer="adamw", packed=False, lr=2e-3):
     from paper_2412_04787_gb300.decoder import DecoderConfig, DQTDecoder
     torch.manual_seed(0)
     cfg = DecoderConfig(layers=2, hidden=128, heads=4, ffn=256, vocab=512, bits=bits_w,
-                        lr=2e-3, seed=7, act=act)
+                        lr=lr, seed=7, act=act, optimizer=optimizer, packed=packed)
     model = DQTDecoder(cfg)
     for m in model.bitlinear_layers():
         m.round_mode = round_mode
     opt = torch.optim.AdamW(model.dense_parameters(), lr=2e-3)
     g = torch.Generator().manual_seed(3)
     ids = torch.randint(0, cfg.vocab, (4, 65), generator=g).cuda()
-    codes0 = [m.codes.clone() for m in model.bitlinear_layers()]
+    codes0 = [m.int8_codes().clone() for m in model.bitlinear_layers()]
     losses = []
     for _ in range(steps):
         loss = model(ids[:, :-1], ids[:, 1:])
@@ -109,7 +109,7 @@ def _train(bits_w, round_mode=0, steps=40, act="int8"):
         opt.step()
         opt.zero_grad(set_to_none=True)
         losses.append(float(loss.detach()))
-    moved = sum(int((m.codes != c).sum()) for m, c in zip(model.bitlinear_layers(), codes0))
+    moved = sum(int((m.int8_codes() != c).sum()) for m, c in zip(model.bitlinear_layers(), codes0))
     return losses, moved, model
 
 
@@ -121,8 +121,68 @@ def test_decoder_trains_with_low_bit_weights(bits_w):
     assert moved > 0
     for m in model.bitlinear_layers():
         lo, hi = m.grid_tuple
-        c = m.codes
+        c = m.int8_codes()
         assert int(c.min()) >= lo and int(c.max()) <= hi
+
+
+@pytest.mark.parametrize("packed", [False, True])
+def test_decoder_trains_with_adafactor(packed):
+    """Sec. 4.3: DQT with the memory-efficient Adafactor optimiser (here with
+    2-bit packed ternary codes as well) still trains."""
+    losses, moved, model = _train(1.58, optimizer="adafactor", packed=packed, lr=1e-2)
+    assert all(m.optimizer == "adafactor" and m.packed == packed for m in model.bitlinear_layers())
+    assert all(np.isfinite(losses))
+    assert losses[-1] < 0.8 * losses[0], (losses[0], losses[-1])
+    assert moved > 0
+
+
+def test_packed_module_equals_int8_module():
+    """AdamW on packed ternary codes: the same forward, dX and codes as on int8 codes."""
+    from paper_2412_04787_gb300.bitlinear import DQTBitLinear
+    T, K, N = 256, 264, 520
+    a = DQTBitLinear(K, N, bits=1.58, seed=3, tensor_id=2, init_seed=5)
+    b = DQTBitLinear(K, N, bits=1.58, seed=3, tensor_id=2, init_seed=5, packed=True)
+    assert b.codes.numel() == (N * K + 3) // 4
+    assert torch.equal(a.codes, b.int8_codes())
+    for i in range(2):
+        X = inputs.normal((T, K), 1.0, seed=40 + i, dtype=torch.bfloat16).cuda()
+        dY = inputs.normal((T, N), 1e-2, seed=50 + i, dtype=torch.bfloat16).cuda()
+        xa = X.clone().requires_grad_(True)
+        xb = X.clone().requires_grad_(True)
+        ya, yb = a(xa), b(xb)
+        assert torch.equal(ya, yb)
+        ya.backward(dY)
+        yb.backward(dY)
+        assert torch.equal(xa.grad, xb.grad)
+        assert torch.equal(a.codes, b.int8_codes()) and torch.equal(a.m, b.m) and torch.equal(a.v, b.v)
+
+
+def test_adafactor_module_matches_oracle():
+    """optimizer="adafactor": after one backward the codes are the oracle's
+    Adafactor + SR step of the bf16-environment gradient (fused tolerance)."""
+    from paper_2412_04787_gb300.bitlinear import DQTBitLinear
+    T, K, N = 300, 264, 520
+    layer = DQTBitLinear(K, N, bits=4, lr=1e-2, seed=8, tensor_id=6, init_seed=9,
+                         optimizer="adafactor")
+    qmin, qmax = layer.grid_tuple
+    c0, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=9).numpy(), qmin, qmax)
+    layer.codes.copy_(torch.from_numpy(c0))
+    layer.s_w = float(s_w)
+    X = inputs.normal((T, K), 1.0, seed=1, dtype=torch.bfloat16)
+    dY = inputs.normal((T, N), 1e-2, seed=2, dtype=torch.bfloat16)
+    layer(X.cuda().requires_grad_(True)).backward(dY.cuda())
+    torch.cuda.synchronize()
+    _, _, _, xd = oracle.act_quant(bits(X))
+    g = oracle.bwd_dw_bf16x(bits(dY), xd).astype(np.float32)
+    hp = oracle.AdafactorHP(lr=1e-2)
+    R, Cc, st = oracle.adafactor_stats(g, c0, np.float32(layer.s_w), np.zeros(N), np.zeros(K), 1, hp)
+    c1, _ = oracle.adafactor_apply(g, c0, R, Cc, st["rbar"], st["step"], st["decay"], qmin, qmax,
+                                   8, 1, 6)
+    cg = layer.codes.cpu().numpy().astype(np.int32)
+    diff = cg != c1
+    assert diff.mean() <= 1e-4 + 1.0 / diff.size
+    assert (np.abs(cg - c1.astype(np.int32))[diff] == 1).all()
+    assert np.allclose(layer.R.cpu().numpy(), R, rtol=1e-4)
 
 
 def test_decoder_trains_in_fp8_environment():
