@@ -527,14 +527,19 @@ void dqt_oracle_unpack_ternary(const uint8_t* p, int64_t n, int8_t* c) {
 /* Statistics (fp64 sums, state rounded to fp32):                            */
 /*   R[n] <- b2 R[n] + omb2 mean_k(g^2 + eps1)                                */
 /*   C[k] <- b2 C[k] + omb2 mean_n(g^2 + eps1)                                */
-/*   Rbar = mean_n R[n];   V[n,k] = R[n] C[k] / Rbar                         */
-/*   rms_u = sqrt(mean g^2 / V);   rms_x = sqrt(mean (c / s_w)^2)            */
+/*   Rbar = mean_n R[n]   (rounded once to fp32)                             */
+/* The estimate V[n,k] = R[n] C[k] / Rbar is rank one, so its inverse square */
+/* root is a row factor times a column factor, each an fp32 value made by    */
+/* two correctly rounded operations:                                         */
+/*   a[n] = 1 / sqrt(R[n] / Rbar),   b[k] = 1 / sqrt(C[k])                   */
+/*   u[n,k] = (g a[n]) b[k]           (two fp32 multiplications)             */
+/*   rms_u = sqrt(mean u^2) (fp64 over the fp32 u);  rms_x = sqrt(mean (c/s_w)^2) */
 /*   alpha = rho * (scale_parameter ? max(eps2, rms_x) : 1)                  */
 /*   step  = s_w alpha / max(1, rms_u / d)        (code-domain step, fp32)   */
 /*   decay = 1 - weight_decay alpha                (fp32)                     */
-/* Per element, separately rounded fp32 operations (dqt_oracle_adafactor_    */
-/* apply):  v = (R[n] C[k]) / Rbar;  u = g / sqrt(v);  x = c decay - step u; */
-/* then c' = Clip[SR(x), Q_n, Q_p] with the same Philox stream as AdamW.      */
+/* Per element (dqt_oracle_adafactor_apply), separately rounded fp32 ops:    */
+/*   u = (g a[n]) b[k];  x = c decay - step u;  c' = Clip[SR(x), Q_n, Q_p]    */
+/* with the same Philox stream as AdamW.                                      */
 /* ======================================================================== */
 void dqt_oracle_adafactor_consts(int64_t t, float lr, float decay_rate, int32_t relative_step,
                                  int32_t warmup_init, float* b2, float* omb2, float* rho) {
@@ -550,13 +555,18 @@ void dqt_oracle_adafactor_consts(int64_t t, float lr, float decay_rate, int32_t 
   }
 }
 
-/* R, C updated in place.  out4 = {Rbar, rms_u, rms_x, unused}; step and     */
-/* decay as above.                                                          */
+static float adafactor_u(float g, float an, float bk) {
+  float ga = g * an;
+  return ga * bk;
+}
+
+/* R, C updated in place; a [N], b [K] the inverse-square-root factors.     */
+/* out4 = {Rbar (fp32 value), rms_u, rms_x, alpha}; step and decay above.   */
 void dqt_oracle_adafactor_stats(const float* g, const int8_t* c, int64_t N, int64_t K,
                                 float s_w, float* R, float* C, float b2, float omb2,
                                 float rho, float eps1, float eps2, float clip_d,
-                                int32_t scale_parameter, float weight_decay, double* out4,
-                                float* step_out, float* decay_out) {
+                                int32_t scale_parameter, float weight_decay, float* a,
+                                float* b, double* out4, float* step_out, float* decay_out) {
   for (int64_t n = 0; n < N; ++n) {
     double acc = 0.0;
     for (int64_t k = 0; k < K; ++k) {
@@ -575,13 +585,14 @@ void dqt_oracle_adafactor_stats(const float* g, const int8_t* c, int64_t N, int6
   }
   double rsum = 0.0;
   for (int64_t n = 0; n < N; ++n) rsum += (double)R[n];
-  double rbar = rsum / (double)N;
+  float rbar = (float)(rsum / (double)N);
+  for (int64_t n = 0; n < N; ++n) a[n] = 1.0f / sqrtf(R[n] / rbar);
+  for (int64_t k = 0; k < K; ++k) b[k] = 1.0f / sqrtf(C[k]);
   double usq = 0.0, xsq = 0.0;
   for (int64_t n = 0; n < N; ++n)
     for (int64_t k = 0; k < K; ++k) {
-      double gv = (double)g[n * K + k];
-      double v = (double)R[n] * (double)C[k] / rbar;
-      usq += gv * gv / v;
+      double u = (double)adafactor_u(g[n * K + k], a[n], b[k]);
+      usq += u * u;
       double w = (double)c[n * K + k] / (double)s_w;
       xsq += w * w;
     }
@@ -590,7 +601,7 @@ void dqt_oracle_adafactor_stats(const float* g, const int8_t* c, int64_t N, int6
   double alpha = (double)rho * (scale_parameter ? (rms_x > (double)eps2 ? rms_x : (double)eps2) : 1.0);
   double div = rms_u / (double)clip_d;
   if (div < 1.0) div = 1.0;
-  out4[0] = rbar;
+  out4[0] = (double)rbar;
   out4[1] = rms_u;
   out4[2] = rms_x;
   out4[3] = alpha;
@@ -598,35 +609,32 @@ void dqt_oracle_adafactor_stats(const float* g, const int8_t* c, int64_t N, int6
   *decay_out = (float)(1.0 - (double)weight_decay * alpha);
 }
 
-static float adafactor_x(float g, int8_t c, float Rn, float Ck, float rbar, float step,
-                         float decay) {
-  float rc = Rn * Ck;
-  float v = rc / rbar;
-  float u = g / sqrtf(v);
+static float adafactor_x(float g, int8_t c, float an, float bk, float step, float decay) {
+  float u = adafactor_u(g, an, bk);
   float cd = (float)c * decay;
   float du = step * u;
   return cd - du;
 }
 
 /* Dense code-domain target only (no rounding), N x K. */
-void dqt_oracle_adafactor_x(const float* g, const int8_t* c, const float* R, const float* C,
-                            float rbar, float step, float decay, int64_t N, int64_t K, float* x) {
+void dqt_oracle_adafactor_x(const float* g, const int8_t* c, const float* a, const float* b,
+                            float step, float decay, int64_t N, int64_t K, float* x) {
   for (int64_t n = 0; n < N; ++n)
     for (int64_t k = 0; k < K; ++k)
-      x[n * K + k] = adafactor_x(g[n * K + k], c[n * K + k], R[n], C[k], rbar, step, decay);
+      x[n * K + k] = adafactor_x(g[n * K + k], c[n * K + k], a[n], b[k], step, decay);
 }
 
-/* Per-element Adafactor + SR over an N x K weight, given R, C, Rbar (fp32), */
+/* Per-element Adafactor + SR over an N x K weight, given the factors a, b,  */
 /* the code-domain step and decay.  Returns the number of codes changed.     */
-int64_t dqt_oracle_adafactor_apply(const float* g, int8_t* c, const float* R, const float* C,
-                                   float rbar, float step, float decay, int64_t N, int64_t K,
-                                   int32_t qmin, int32_t qmax, uint64_t seed, int64_t t,
-                                   uint32_t tensor_id, int32_t round_mode) {
+int64_t dqt_oracle_adafactor_apply(const float* g, int8_t* c, const float* a, const float* b,
+                                   float step, float decay, int64_t N, int64_t K, int32_t qmin,
+                                   int32_t qmax, uint64_t seed, int64_t t, uint32_t tensor_id,
+                                   int32_t round_mode) {
   int64_t changed = 0;
   for (int64_t n = 0; n < N; ++n)
     for (int64_t k = 0; k < K; ++k) {
       int64_t e = n * K + k;
-      float x = adafactor_x(g[e], c[e], R[n], C[k], rbar, step, decay);
+      float x = adafactor_x(g[e], c[e], a[n], b[k], step, decay);
       int32_t r;
       if (round_mode == 1) {
         r = (int32_t)rintf(x);

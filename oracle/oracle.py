@@ -105,15 +105,15 @@ def lib():
         L.dqt_oracle_adafactor_stats.argtypes = [_f32p, _i8p, C.c_int64, C.c_int64, C.c_float,
                                                  _f32p, _f32p, C.c_float, C.c_float, C.c_float,
                                                  C.c_float, C.c_float, C.c_float, C.c_int32,
-                                                 C.c_float, _f64p, _f32p, _f32p]
+                                                 C.c_float, _f32p, _f32p, _f64p, _f32p, _f32p]
         L.dqt_oracle_adafactor_stats.restype = None
         L.dqt_oracle_adafactor_x.argtypes = [_f32p, _i8p, _f32p, _f32p, C.c_float, C.c_float,
-                                             C.c_float, C.c_int64, C.c_int64, _f32p]
+                                             C.c_int64, C.c_int64, _f32p]
         L.dqt_oracle_adafactor_x.restype = None
         L.dqt_oracle_adafactor_apply.argtypes = [_f32p, _i8p, _f32p, _f32p, C.c_float,
-                                                 C.c_float, C.c_float, C.c_int64, C.c_int64,
-                                                 C.c_int32, C.c_int32, C.c_uint64, C.c_int64,
-                                                 C.c_uint32, C.c_int32]
+                                                 C.c_float, C.c_int64, C.c_int64, C.c_int32,
+                                                 C.c_int32, C.c_uint64, C.c_int64, C.c_uint32,
+                                                 C.c_int32]
         L.dqt_oracle_adafactor_apply.restype = C.c_int64
         _lib = L
     return _lib
@@ -406,7 +406,8 @@ def adafactor_consts(t, hp):
 
 
 def adafactor_stats(g, c, s_w, R, C_, t, hp):
-    """Returns (R', C', dict(rbar, rms_u, rms_x, alpha, step, decay)); R', C' fp32."""
+    """Returns (R', C', st) with st = dict(rbar, rms_u, rms_x, alpha, step, decay, a, b):
+    R', C' fp32 state, a [N] and b [K] the fp32 inverse-square-root factors."""
     g = _c(g, np.float32)
     N, K = g.shape
     c = _c(c, np.int8).reshape(N, K)
@@ -414,39 +415,40 @@ def adafactor_stats(g, c, s_w, R, C_, t, hp):
     Cc = _c(C_, np.float32).copy()
     assert R.shape == (N,) and Cc.shape == (K,)
     b2, omb2, rho = adafactor_consts(t, hp)
+    a = np.empty(N, np.float32)
+    b = np.empty(K, np.float32)
     out4 = np.empty(4, np.float64)
     step, decay = C.c_float(), C.c_float()
     lib().dqt_oracle_adafactor_stats(_p(g, _f32p), _p(c, _i8p), N, K, float(s_w), _p(R, _f32p),
                                      _p(Cc, _f32p), b2, omb2, rho, hp.eps1, hp.eps2, hp.clip_d,
-                                     int(hp.scale_parameter), hp.weight_decay, _p(out4, _f64p),
-                                     C.byref(step), C.byref(decay))
+                                     int(hp.scale_parameter), hp.weight_decay, _p(a, _f32p),
+                                     _p(b, _f32p), _p(out4, _f64p), C.byref(step),
+                                     C.byref(decay))
     st = {"rbar": out4[0], "rms_u": out4[1], "rms_x": out4[2], "alpha": out4[3],
-          "step": np.float32(step.value), "decay": np.float32(decay.value)}
+          "step": np.float32(step.value), "decay": np.float32(decay.value), "a": a, "b": b}
     return R, Cc, st
 
 
-def adafactor_x(g, c, R, C_, rbar, step, decay):
+def adafactor_x(g, c, a, b, step, decay):
     g = _c(g, np.float32)
     N, K = g.shape
     c = _c(c, np.int8).reshape(N, K)
-    R = _c(R, np.float32)
-    Cc = _c(C_, np.float32)
+    a = _c(a, np.float32)
+    b = _c(b, np.float32)
     x = np.empty((N, K), np.float32)
-    lib().dqt_oracle_adafactor_x(_p(g, _f32p), _p(c, _i8p), _p(R, _f32p), _p(Cc, _f32p),
-                                 float(np.float32(rbar)), float(step), float(decay), N, K,
-                                 _p(x, _f32p))
+    lib().dqt_oracle_adafactor_x(_p(g, _f32p), _p(c, _i8p), _p(a, _f32p), _p(b, _f32p),
+                                 float(step), float(decay), N, K, _p(x, _f32p))
     return x
 
 
-def adafactor_apply(g, c, R, C_, rbar, step, decay, qmin, qmax, seed, t, tensor_id,
-                    round_mode=0):
+def adafactor_apply(g, c, a, b, step, decay, qmin, qmax, seed, t, tensor_id, round_mode=0):
     """Returns (c', changed)."""
     g = _c(g, np.float32)
     N, K = g.shape
     c = _c(c, np.int8).reshape(N, K).copy()
-    R = _c(R, np.float32)
-    Cc = _c(C_, np.float32)
-    ch = lib().dqt_oracle_adafactor_apply(_p(g, _f32p), _p(c, _i8p), _p(R, _f32p), _p(Cc, _f32p),
-                                          float(np.float32(rbar)), float(step), float(decay), N,
-                                          K, qmin, qmax, seed, t, tensor_id, round_mode)
+    a = _c(a, np.float32)
+    b = _c(b, np.float32)
+    ch = lib().dqt_oracle_adafactor_apply(_p(g, _f32p), _p(c, _i8p), _p(a, _f32p), _p(b, _f32p),
+                                          float(step), float(decay), N, K, qmin, qmax, seed, t,
+                                          tensor_id, round_mode)
     return c, int(ch)

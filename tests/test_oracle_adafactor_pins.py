@@ -92,10 +92,10 @@ def test_rank_one_first_step_is_a_sign_step():
     assert abs(st["rms_u"] - 1.0) < 1e-6
     rho = np.float64(np.float32(1e-2))  # the step size is an fp32 constant
     assert st["alpha"] == rho and st["step"] == np.float32(s_w * rho)
-    x = oracle.adafactor_x(g, c, R, C, st["rbar"], st["step"], st["decay"])
+    x = oracle.adafactor_x(g, c, st["a"], st["b"], st["step"], st["decay"])
     assert np.allclose(x, c - 0.6 * np.sign(g), atol=1e-5)
     # round to nearest moves every code one step against its gradient's sign, where the grid allows
-    c1, _ = oracle.adafactor_apply(g, c, R, C, st["rbar"], st["step"], st["decay"], -1, 1,
+    c1, _ = oracle.adafactor_apply(g, c, st["a"], st["b"], st["step"], st["decay"], -1, 1,
                                    0, 1, 0, round_mode=1)
     want = np.clip(np.rint(c - 0.6 * np.sign(g)), -1, 1)
     assert (c1 == want).all()
@@ -113,6 +113,19 @@ def test_factored_moment_marginals():
     assert np.allclose(V.mean(axis=0), C, rtol=1e-6)
     sq = g.astype(np.float64) ** 2 + 1e-30
     assert np.allclose(R, sq.mean(axis=1), rtol=1e-6) and np.allclose(C, sq.mean(axis=0), rtol=1e-6)
+
+
+def test_factors_are_the_inverse_square_root_of_the_estimate():
+    """a[n] b[k] = 1 / sqrt(R[n] C[k] / Rbar): the rank-one estimate's inverse
+    square root splits into a row and a column factor."""
+    N, K = 40, 24
+    g = inputs.normal((N, K), 1e-3, seed=15).numpy()
+    R, C, st = oracle.adafactor_stats(g, np.zeros((N, K), np.int8), 10.0, np.zeros(N), np.zeros(K),
+                                      1, oracle.AdafactorHP())
+    V = np.outer(R.astype(np.float64), C.astype(np.float64)) / st["rbar"]
+    ab = np.outer(st["a"].astype(np.float64), st["b"].astype(np.float64))
+    assert np.allclose(ab, 1.0 / np.sqrt(V), rtol=1e-6)
+    assert st["rbar"] == np.float32(R.astype(np.float64).mean())
 
 
 def test_moment_ema_over_steps():
@@ -141,8 +154,8 @@ def test_gradient_scale_invariance():
     outs = []
     for scale in (1.0, 4.0):
         R, C, st = oracle.adafactor_stats(g * np.float32(scale), c, 40.0, np.zeros(N), np.zeros(K), 1, hp)
-        x = oracle.adafactor_x(g * np.float32(scale), c, R, C, st["rbar"], st["step"], st["decay"])
-        cc, _ = oracle.adafactor_apply(g * np.float32(scale), c, R, C, st["rbar"], st["step"],
+        x = oracle.adafactor_x(g * np.float32(scale), c, st["a"], st["b"], st["step"], st["decay"])
+        cc, _ = oracle.adafactor_apply(g * np.float32(scale), c, st["a"], st["b"], st["step"],
                                        st["decay"], -1, 1, 1234, 1, 3)
         outs.append((x, cc, st["rms_u"]))
     assert (outs[0][0] == outs[1][0]).all() and (outs[0][1] == outs[1][1]).all()
@@ -160,7 +173,7 @@ def test_update_clipping_to_rms_d():
         hp = oracle.AdafactorHP(lr=1e-2, clip_d=d)
         R, C, st = oracle.adafactor_stats(g, c, 20.0, np.zeros(N), np.zeros(K), 1, hp)
         assert st["rms_u"] > d
-        x = oracle.adafactor_x(g, c, R, C, st["rbar"], st["step"], st["decay"]).astype(np.float64)
+        x = oracle.adafactor_x(g, c, st["a"], st["b"], st["step"], st["decay"]).astype(np.float64)
         upd = -x / (20.0 * 1e-2)  # the normalised update actually applied
         assert math.sqrt((upd ** 2).mean()) == pytest.approx(d, rel=1e-5)
 
@@ -190,7 +203,7 @@ def test_descent_direction():
     g = inputs.normal((N, K), 1e-3, seed=13).numpy()
     c = np.random.default_rng(5).integers(-1, 2, (N, K)).astype(np.int8)
     R, C, st = oracle.adafactor_stats(g, c, 30.0, np.zeros(N), np.zeros(K), 1, oracle.AdafactorHP())
-    x = oracle.adafactor_x(g, c, R, C, st["rbar"], st["step"], st["decay"])
+    x = oracle.adafactor_x(g, c, st["a"], st["b"], st["step"], st["decay"])
     d = x - c
     assert (np.sign(d[g != 0]) == -np.sign(g[g != 0])).all()
 
@@ -219,7 +232,7 @@ def test_matches_torch_adafactor_dense_target():
         opt.step()
         dW = (W.detach() - before).numpy()
         R, C, st = oracle.adafactor_stats(g, cur, s_w, R, C, t, hp)
-        x = oracle.adafactor_x(g, cur, R, C, st["rbar"], st["step"], st["decay"])
+        x = oracle.adafactor_x(g, cur, st["a"], st["b"], st["step"], st["decay"])
         ours = (x.astype(np.float64) - cur) / s_w
         # x is fp32 near the integer c: (x - c) / s_w is exact to 2^-24 |x| / s_w
         assert np.allclose(ours, dW, rtol=1e-5, atol=2.0 ** -23 / s_w), t
