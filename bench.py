@@ -52,7 +52,7 @@ METRIC = "DQT BitLinear fwd+bwd+SR-update tokens/s"
 PROJ = [("gate", HID, INTER), ("up", HID, INTER), ("down", INTER, HID)]
 
 
-GEMM_SOURCES = ("gemm_tc.cu", "dqt_device.cuh", "dqt_internal.h")
+GEMM_SOURCES = ("gemm_tc.cu", "dqt_device.cuh")  # the GEMM kernels' device code
 
 
 def kernel_fingerprint(files=GEMM_SOURCES):
@@ -72,7 +72,7 @@ def kernel_fingerprint(files=GEMM_SOURCES):
 # launches move the same numbers of operand and optimiser-state bytes), keyed
 # by the kernel fingerprint it was taken on (see profiles/).  A stale entry
 # reports null.
-DW_TRAFFIC_BYTES = {"729b805819b4": 295927296 + 57431552}
+DW_TRAFFIC_BYTES = {"5cd93cdc4c54": 295927296 + 57431552}
 
 
 def _dist():
@@ -711,16 +711,17 @@ def run_kernel(args):
             Cc = torch.zeros(K, device=dev)
             af = dqt.adafactor(lr=1e-2)
             G = torch.randn((N, K), device=dev) * 1e-3
-            scal = dqt.dqt_adafactor_stats(G, W, s_w, R, Cc, af)
+            fa, fb, scal = dqt.dqt_adafactor_stats(G, W, s_w, R, Cc, af)
             if k == "bwd_dw_adafactor":
                 ws = torch.empty(dqt.dqt_bwd_dw_adafactor_workspace_size(T, N, K), dtype=torch.uint8,
                                  device=dev)
                 fn = lambda: dqt.dqt_bitlinear_bwd_dw_adafactor(dY, xdq, W, s_w, R, Cc, af, sr, g,  # noqa: E731
                                                                 ws=ws)
             elif k == "adafactor_stats":
-                fn = lambda: dqt.dqt_adafactor_stats(G, W, s_w, R, Cc, af, scalars_out=scal)  # noqa: E731
+                fn = lambda: dqt.dqt_adafactor_stats(G, W, s_w, R, Cc, af, a_out=fa, b_out=fb,  # noqa: E731
+                                                     scalars_out=scal)
             else:
-                fn = lambda: dqt.dqt_adafactor_apply(G, W, R, Cc, scal, 1, sr, g)  # noqa: E731
+                fn = lambda: dqt.dqt_adafactor_apply(G, W, fa, fb, scal, 1, sr, g)  # noqa: E731
         elif k in ("act_quant_fp8", "fwd_fp8", "codes_to_fp8"):
             q8, s8, _ = dqt.dqt_act_quant_fp8(X)
             W8 = dqt.dqt_codes_to_fp8(W, g)

@@ -309,7 +309,10 @@ int dqt_bitlinear_bwd_dw_update_packed(const dqt_bf16* dY, const dqt_bf16* Xdq, 
  *   b2 = 1 - t^decay_rate;  rho = relative_step ? min(warmup_init ? 1e-6 t : 1e-2,
  *                                                  1/sqrt(t)) : lr
  *   R <- b2 R + (1 - b2) mean_k(g^2 + eps1);  C <- b2 C + (1 - b2) mean_n(g^2 + eps1)
- *   Rbar = mean R;  v = R[n] C[k] / Rbar;  u = g / sqrt(v)
+ *   Rbar = mean R; the inverse square root of the rank-one estimate R C / Rbar is
+ *   a row factor a[n] = 1 / sqrt(R[n] / Rbar) times a column factor
+ *   b[k] = 1 / sqrt(C[k]) (each two correctly rounded fp32 operations);
+ *   u = (g a[n]) b[k]
  *   alpha = rho * (scale_parameter ? max(eps2, RMS(W)) : 1),  RMS(W) = RMS(c) / s_w
  *   x = c (1 - weight_decay alpha) - s_w alpha / max(1, RMS(u) / clip_d) * u
  *   c <- Clip[SR(x), qmin, qmax]   (Eq. 1, Eq. 5; the Philox stream of dqt_sr_t
@@ -322,23 +325,24 @@ typedef struct {
   int32_t relative_step, scale_parameter, warmup_init, pad;
 } dqt_adafactor_t;
 
-/* Statistics of one step for a gradient G fp32 [N, K] in memory: updates R, C
- * and writes 8 floats to scalars_out (device, 16-byte aligned):
- * {Rbar, code-domain step s_w alpha / max(1, RMS(u)/clip_d), decay
- * 1 - weight_decay alpha, RMS(u), RMS(W), alpha, 0, 0}.  W: the codes before
- * the step (int8 [N, K], or packed ternary if `packed`).  Workspace:
- * dqt_adafactor_workspace_size(N, K) bytes, 256-byte aligned.  Every sum has
- * a fixed order: deterministic. */
+/* Statistics of one step for a gradient G fp32 [N, K] in memory: updates R, C,
+ * writes the factors a_out fp32 [N] and b_out fp32 [K], and 8 floats to
+ * scalars_out (device, 16-byte aligned): {Rbar, code-domain step
+ * s_w alpha / max(1, RMS(u)/clip_d), decay 1 - weight_decay alpha, RMS(u),
+ * RMS(W) (0 unless scale_parameter: the codes are not read then), alpha, 0, 0}.
+ * W: the codes before the step (int8 [N, K], or packed ternary if `packed`).  Workspace: dqt_adafactor_workspace_size(N, K) bytes,
+ * 256-byte aligned.  Every sum has a fixed order: deterministic. */
 size_t dqt_adafactor_workspace_size(int64_t N, int64_t K);
 int dqt_adafactor_stats(const float* G, const void* W, int32_t packed, float s_w, float* R,
-                        float* C, const dqt_adafactor_t* hp, int64_t N, int64_t K,
-                        float* scalars_out, void* ws, size_t ws_bytes, void* stream);
-/* The per-element step given R, C and the scalars {Rbar, step, decay} in
- * device memory (as dqt_adafactor_stats writes them): v = (R[n] C[k]) / Rbar,
- * u = g / sqrt(v), x = c decay - step u, each a separately rounded fp32
+                        float* C, const dqt_adafactor_t* hp, int64_t N, int64_t K, float* a_out,
+                        float* b_out, float* scalars_out, void* ws, size_t ws_bytes,
+                        void* stream);
+/* The per-element step given the factors a [N], b [K] and the scalars
+ * {., step, decay} in device memory (as dqt_adafactor_stats writes them):
+ * u = (g a[n]) b[k], x = c decay - step u, each a separately rounded fp32
  * operation, then SR with counter `step_t` and the clamp.  changed_out as for
  * dqt_sr_update. */
-int dqt_adafactor_apply(const float* G, void* W, int32_t packed, const float* R, const float* C,
+int dqt_adafactor_apply(const float* G, void* W, int32_t packed, const float* a, const float* b,
                         const float* scalars, int64_t step_t, const dqt_sr_t* sr, dqt_grid_t grid,
                         int64_t N, int64_t K, unsigned long long* changed_out, void* stream);
 /* The whole backward-and-update of a BitLinear weight with Adafactor: the

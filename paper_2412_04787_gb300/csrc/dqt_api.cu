@@ -510,38 +510,40 @@ size_t dqt_adafactor_workspace_size(int64_t N, int64_t K) {
 }
 
 int dqt_adafactor_stats(const float* G, const void* W, int32_t packed, float s_w, float* R,
-                        float* C, const dqt_adafactor_t* hp, int64_t N, int64_t K,
-                        float* scalars_out, void* ws, size_t ws_bytes, void* stream) {
-  if (!G || !W || !R || !C || !scalars_out || !ws || N <= 0 || K <= 0 || !(s_w > 0.0f) ||
-      !isfinite(s_w))
+                        float* C, const dqt_adafactor_t* hp, int64_t N, int64_t K, float* a_out,
+                        float* b_out, float* scalars_out, void* ws, size_t ws_bytes,
+                        void* stream) {
+  if (!G || !W || !R || !C || !a_out || !b_out || !scalars_out || !ws || N <= 0 || K <= 0 ||
+      !(s_w > 0.0f) || !isfinite(s_w))
     return DQT_ERR_ARG;
   if (N > kMaxDim || K > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
   if (ws_bytes < dqt::adafactor_stats_ws(N, K)) return DQT_ERR_ARG;
   if (K % 4 || !aligned16(G) || !aligned16(W) || !aligned16(R) || !aligned16(C) ||
-      !aligned16(scalars_out) || (reinterpret_cast<uintptr_t>(ws) & 255u))
+      !aligned16(a_out) || !aligned16(b_out) || !aligned16(scalars_out) ||
+      (reinterpret_cast<uintptr_t>(ws) & 255u))
     return DQT_ERR_ALIGN;
   dqt::AdafactorConsts h;
   const int rc = make_adafactor_consts(hp, &h);
   if (rc != DQT_OK) return rc;
   return dqt::launch_adafactor_stats(G, static_cast<const int8_t*>(W), packed != 0, s_w, R, C, h,
-                                     N, K, ws, scalars_out, as_stream(stream))
+                                     N, K, ws, a_out, b_out, scalars_out, as_stream(stream))
              ? DQT_ERR_CUDA
              : DQT_OK;
 }
 
-int dqt_adafactor_apply(const float* G, void* W, int32_t packed, const float* R, const float* C,
+int dqt_adafactor_apply(const float* G, void* W, int32_t packed, const float* a, const float* b,
                         const float* scalars, int64_t step_t, const dqt_sr_t* sr, dqt_grid_t grid,
                         int64_t N, int64_t K, unsigned long long* changed_out, void* stream) {
-  if (!G || !W || !R || !C || !scalars || N <= 0 || K <= 0) return DQT_ERR_ARG;
+  if (!G || !W || !a || !b || !scalars || N <= 0 || K <= 0) return DQT_ERR_ARG;
   if (N > kMaxDim || K > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
   if (packed && (grid.qmin != -1 || grid.qmax != 1)) return DQT_ERR_ARG;
-  if (K % 4 || !aligned16(G) || !aligned16(W) || !aligned16(R) || !aligned16(C) ||
+  if (K % 4 || !aligned16(G) || !aligned16(W) || !aligned16(a) || !aligned16(b) ||
       !aligned16(scalars))
     return DQT_ERR_ALIGN;
   dqt::UpdateConsts uc;
   const int rc = apply_consts(step_t, sr, grid, &uc);
   if (rc != DQT_OK) return rc;
-  return dqt::launch_adafactor_apply(G, static_cast<int8_t*>(W), packed != 0, R, C, scalars, uc,
+  return dqt::launch_adafactor_apply(G, static_cast<int8_t*>(W), packed != 0, a, b, scalars, uc,
                                      N, K, changed_out, as_stream(stream))
              ? DQT_ERR_CUDA
              : DQT_OK;
@@ -596,13 +598,12 @@ int dqt_bitlinear_bwd_dw_adafactor(const dqt_bf16* dY, const dqt_bf16* Xdq, void
   g.ws_bytes = split_bytes;
   if (dqt::launch_gemm(g, s)) return DQT_ERR_CUDA;
   // 2. statistics, 3. the per-element step
-  float* scal = reinterpret_cast<float*>(static_cast<uint8_t*>(st_ws) +
-                                         dqt::adafactor_scalars_offset(N, K));
+  const dqt::AdafactorBufs fb = dqt::adafactor_bufs(st_ws, N, K);
   if (dqt::launch_adafactor_stats(G, static_cast<const int8_t*>(W), packed != 0, s_w, R, C, h, N,
-                                  K, st_ws, scal, s))
+                                  K, st_ws, fb.a, fb.b, fb.scalars, s))
     return DQT_ERR_CUDA;
-  return dqt::launch_adafactor_apply(G, static_cast<int8_t*>(W), packed != 0, R, C, scal, uc, N, K,
-                                     changed_out, s)
+  return dqt::launch_adafactor_apply(G, static_cast<int8_t*>(W), packed != 0, fb.a, fb.b,
+                                     fb.scalars, uc, N, K, changed_out, s)
              ? DQT_ERR_CUDA
              : DQT_OK;
 }

@@ -90,20 +90,28 @@ struct AdafactorConsts {
   float b2, omb2, rho, eps1, eps2, clip_d, weight_decay;
   int32_t scale_parameter;
 };
-// Workspace of the statistics passes for an N x K weight, and the offset of
-// the 8-float scalar block inside it.
+// Workspace of the statistics passes for an N x K weight; it also holds a
+// set of factor vectors and a scalar block (adafactor_bufs) for callers that
+// do not keep their own.
 size_t adafactor_stats_ws(int64_t N, int64_t K);
-size_t adafactor_scalars_offset(int64_t N, int64_t K);
-// R, C updated in place; scalars_out (device, 8 floats; NULL = inside ws) gets
-// {Rbar, code-domain step, decay, rms_u, rms_x, alpha}.
+struct AdafactorBufs {
+  float* a;        // [N] row factors
+  float* b;        // [K] column factors
+  float* scalars;  // [8]
+};
+AdafactorBufs adafactor_bufs(void* ws, int64_t N, int64_t K);
+// R, C updated in place; a_out [N], b_out [K] get the inverse-square-root
+// factors, scalars_out (8 floats) {Rbar, code-domain step, decay, rms_u,
+// rms_x, alpha}.
 int launch_adafactor_stats(const float* G, const int8_t* W, bool packed, float s_w, float* R,
                            float* C, const AdafactorConsts& h, int64_t N, int64_t K, void* ws,
-                           float* scalars_out, cudaStream_t stream);
-// The per-element update given R, C and scalars {Rbar, step, decay} (device).
-// Uses the grid, round mode and Philox key/counter fields of uc.
-int launch_adafactor_apply(const float* G, int8_t* W, bool packed, const float* R, const float* C,
-                           const float* scalars, const UpdateConsts& uc, int64_t N, int64_t K,
-                           unsigned long long* changed, cudaStream_t stream);
+                           float* a_out, float* b_out, float* scalars_out, cudaStream_t stream);
+// The per-element update given the factors and scalars {., step, decay}
+// (device).  Uses the grid, round mode and Philox key/counter fields of uc.
+int launch_adafactor_apply(const float* G, int8_t* W, bool packed, const float* fa,
+                           const float* fb, const float* scalars, const UpdateConsts& uc,
+                           int64_t N, int64_t K, unsigned long long* changed,
+                           cudaStream_t stream);
 
 int launch_sr_update(const float* grad, int8_t* W, float* m, float* v, int64_t numel,
                      const UpdateConsts& uc, const UpdateConsts* uc_dev,

@@ -116,8 +116,8 @@ def lib():
         L.dqt_adafactor_workspace_size.argtypes = [_i64, _i64]
         L.dqt_adafactor_workspace_size.restype = _sz
         L.dqt_adafactor_stats.argtypes = [_vp, _vp, C.c_int32, _f32, _vp, _vp,
-                                          C.POINTER(dqt_adafactor_t), _i64, _i64, _vp, _vp, _sz,
-                                          _vp]
+                                          C.POINTER(dqt_adafactor_t), _i64, _i64, _vp, _vp, _vp,
+                                          _vp, _sz, _vp]
         L.dqt_adafactor_apply.argtypes = [_vp, _vp, C.c_int32, _vp, _vp, _vp, _i64,
                                           C.POINTER(dqt_sr_t), dqt_grid_t, _i64, _i64, _vp, _vp]
         L.dqt_bwd_dw_adafactor_workspace_size.argtypes = [_i64, _i64, _i64]
@@ -553,37 +553,44 @@ def _codes_arg(W, packed, N, K):
         _need(W, "W", torch.int8, (N, K))
 
 
-def dqt_adafactor_stats(G, W, s_w, R, C_, hp, packed=False, scalars_out=None, ws=None,
-                        stream=None):
-    """Returns the device scalars {Rbar, step, decay, rms_u, rms_x, alpha, 0, 0}."""
+def dqt_adafactor_stats(G, W, s_w, R, C_, hp, packed=False, a_out=None, b_out=None,
+                        scalars_out=None, ws=None, stream=None):
+    """Returns (a [N], b [K], scalars {Rbar, step, decay, rms_u, rms_x, alpha, 0, 0}),
+    all device fp32."""
     _need(G, "G", torch.float32)
     N, K = G.shape
     _codes_arg(W, packed, N, K)
     _need(R, "R", torch.float32, (N,))
     _need(C_, "C", torch.float32, (K,))
+    dev = G.device
+    a_out = torch.empty(N, dtype=torch.float32, device=dev) if a_out is None else a_out
+    b_out = torch.empty(K, dtype=torch.float32, device=dev) if b_out is None else b_out
     if scalars_out is None:
-        scalars_out = torch.zeros(8, dtype=torch.float32, device=G.device)
+        scalars_out = torch.zeros(8, dtype=torch.float32, device=dev)
+    _need(a_out, "a_out", torch.float32, (N,))
+    _need(b_out, "b_out", torch.float32, (K,))
     _need(scalars_out, "scalars_out", torch.float32, (8,))
     nb = lib().dqt_adafactor_workspace_size(N, K)
     if ws is None:
-        ws = torch.empty(nb, dtype=torch.uint8, device=G.device)
+        ws = torch.empty(nb, dtype=torch.uint8, device=dev)
     _need(ws, "ws", torch.uint8)
     _check(lib().dqt_adafactor_stats(_ptr(G), _ptr(W), int(packed), float(s_w), _ptr(R),
-                                     _ptr(C_), C.byref(hp), N, K, _ptr(scalars_out), _ptr(ws),
-                                     ws.numel(), _stream(stream)), "dqt_adafactor_stats")
-    return scalars_out
+                                     _ptr(C_), C.byref(hp), N, K, _ptr(a_out), _ptr(b_out),
+                                     _ptr(scalars_out), _ptr(ws), ws.numel(), _stream(stream)),
+           "dqt_adafactor_stats")
+    return a_out, b_out, scalars_out
 
 
-def dqt_adafactor_apply(G, W, R, C_, scalars, step_t, sr, bits_or_grid, packed=False,
+def dqt_adafactor_apply(G, W, a, b, scalars, step_t, sr, bits_or_grid, packed=False,
                         changed_out=None, stream=None):
     _need(G, "G", torch.float32)
     N, K = G.shape
     _codes_arg(W, packed, N, K)
-    _need(R, "R", torch.float32, (N,))
-    _need(C_, "C", torch.float32, (K,))
+    _need(a, "a", torch.float32, (N,))
+    _need(b, "b", torch.float32, (K,))
     _need(scalars, "scalars", torch.float32)
     _opt(changed_out, "changed_out", torch.int64, None)
-    _check(lib().dqt_adafactor_apply(_ptr(G), _ptr(W), int(packed), _ptr(R), _ptr(C_),
+    _check(lib().dqt_adafactor_apply(_ptr(G), _ptr(W), int(packed), _ptr(a), _ptr(b),
                                      _ptr(scalars), int(step_t), C.byref(sr),
                                      _grid(bits_or_grid), N, K, _ptr(changed_out),
                                      _stream(stream)), "dqt_adafactor_apply")

@@ -150,14 +150,16 @@ def test_packed_and_adafactor_argument_validation(L):
     assert L.dqt_bwd_dw_adafactor_workspace_size(128, 64, 64) >= 64 * 64 * 4
     nb = L.dqt_adafactor_workspace_size(64, 64)
     W = _p(0x100000)  # 256-byte aligned
-    assert L.dqt_adafactor_stats(A, A, 0, 1.0, A, A, C.byref(dqt.adafactor(step=0)), 64, 64, A, W,
-                                 nb, None) == dqt.DQT_ERR_ARG
-    assert L.dqt_adafactor_stats(A, A, 0, 1.0, A, A, C.byref(dqt.adafactor(clip_d=0.0)), 64, 64,
+    assert L.dqt_adafactor_stats(A, A, 0, 1.0, A, A, C.byref(dqt.adafactor(step=0)), 64, 64, A, A,
                                  A, W, nb, None) == dqt.DQT_ERR_ARG
-    assert L.dqt_adafactor_stats(A, A, 0, 1.0, A, A, C.byref(af), 64, 64, A, W, nb - 1,
+    assert L.dqt_adafactor_stats(A, A, 0, 1.0, A, A, C.byref(dqt.adafactor(clip_d=0.0)), 64, 64,
+                                 A, A, A, W, nb, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_adafactor_stats(A, A, 0, 1.0, A, A, C.byref(af), 64, 64, A, A, A, W, nb - 1,
                                  None) == dqt.DQT_ERR_ARG
-    assert L.dqt_adafactor_stats(A, A, 0, 1.0, A, A, C.byref(af), 64, 64, A, _p(0x10010), nb,
-                                 None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_adafactor_stats(A, A, 0, 1.0, A, A, C.byref(af), 64, 64, None, A, A, W, nb,
+                                 None) == dqt.DQT_ERR_ARG
+    assert L.dqt_adafactor_stats(A, A, 0, 1.0, A, A, C.byref(af), 64, 64, A, A, A, _p(0x10010),
+                                 nb, None) == dqt.DQT_ERR_ALIGN
     assert L.dqt_adafactor_apply(A, A, 1, A, A, A, 1, C.byref(sr), dqt.dqt_grid_t(-2, 1), 64, 64,
                                  None, None) == dqt.DQT_ERR_ARG
     assert L.dqt_adafactor_apply(A, A, 0, A, A, A, 0, C.byref(sr), g, 64, 64, None,

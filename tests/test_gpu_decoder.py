@@ -176,7 +176,7 @@ def test_adafactor_module_matches_oracle():
     g = oracle.bwd_dw_bf16x(bits(dY), xd).astype(np.float32)
     hp = oracle.AdafactorHP(lr=1e-2)
     R, Cc, st = oracle.adafactor_stats(g, c0, np.float32(layer.s_w), np.zeros(N), np.zeros(K), 1, hp)
-    c1, _ = oracle.adafactor_apply(g, c0, R, Cc, st["rbar"], st["step"], st["decay"], qmin, qmax,
+    c1, _ = oracle.adafactor_apply(g, c0, st["a"], st["b"], st["step"], st["decay"], qmin, qmax,
                                    8, 1, 6)
     cg = layer.codes.cpu().numpy().astype(np.int32)
     diff = cg != c1

@@ -143,12 +143,17 @@ def test_adafactor_stats(N, K, hpi):
         if t == 2:
             g[N // 2, K // 3] = 0.5  # an outlier: update clipping is active
         R, Cc, st = oracle.adafactor_stats(g, c, s_w, R, Cc, t, hpo)
-        sc = dqt.dqt_adafactor_stats(torch.from_numpy(g).cuda(), torch.from_numpy(c).cuda(), s_w,
-                                     Rg, Cg, dqt.adafactor(step=t, **HPS[hpi]))
+        ag, bg, sc = dqt.dqt_adafactor_stats(torch.from_numpy(g).cuda(), torch.from_numpy(c).cuda(),
+                                             s_w, Rg, Cg, dqt.adafactor(step=t, **HPS[hpi]))
         assert np.allclose(Rg.cpu().numpy(), R, rtol=1e-5, atol=0)
         assert np.allclose(Cg.cpu().numpy(), Cc, rtol=1e-5, atol=0)
+        assert np.allclose(ag.cpu().numpy(), st["a"], rtol=1e-5, atol=0)
+        assert np.allclose(bg.cpu().numpy(), st["b"], rtol=1e-5, atol=0)
         s = sc.cpu().numpy().astype(np.float64)
         for i, key in enumerate(["rbar", "step", "decay", "rms_u", "rms_x", "alpha"]):
+            if key == "rms_x" and not HPS[hpi].get("scale_parameter"):
+                assert s[i] == 0.0  # the codes are read only for parameter scaling
+                continue
             assert s[i] == pytest.approx(float(st[key]), rel=1e-5), (t, key)
 
 
@@ -161,14 +166,14 @@ def test_adafactor_apply_bit_exact(N, K, bits_w, packed, round_mode):
     g = inputs.normal((N, K), 1e-3, seed=N).numpy()
     hpo = oracle.AdafactorHP(lr=1e-2)
     R, Cc, st = oracle.adafactor_stats(g, c, s_w, np.zeros(N), np.zeros(K), 1, hpo)
-    c1, ch = oracle.adafactor_apply(g, c, R, Cc, st["rbar"], st["step"], st["decay"], qmin, qmax,
+    c1, ch = oracle.adafactor_apply(g, c, st["a"], st["b"], st["step"], st["decay"], qmin, qmax,
                                     77, 1, 9, round_mode)
     scal = torch.tensor([np.float32(st["rbar"]), st["step"], st["decay"], 0, 0, 0, 0, 0],
                         dtype=torch.float32, device="cuda")
     W = torch.from_numpy(oracle.pack_ternary(c) if packed else c).cuda()
     changed = torch.zeros(1, dtype=torch.int64, device="cuda")
-    dqt.dqt_adafactor_apply(torch.from_numpy(g).cuda(), W, torch.from_numpy(R).cuda(),
-                            torch.from_numpy(Cc).cuda(), scal, 1,
+    dqt.dqt_adafactor_apply(torch.from_numpy(g).cuda(), W, torch.from_numpy(st["a"]).cuda(),
+                            torch.from_numpy(st["b"]).cuda(), scal, 1,
                             dqt.sr_stream(seed=77, tensor_id=9, round_mode=round_mode),
                             (qmin, qmax), packed=packed, changed_out=changed)
     got = oracle.unpack_ternary(W.cpu().numpy(), N * K).reshape(N, K) if packed else W.cpu().numpy()
@@ -198,7 +203,7 @@ def test_bwd_dw_adafactor(T, K, N, bits_w, packed):
         dY = inputs.normal((T, N), 1e-2, seed=100 * t + T, dtype=torch.bfloat16)
         g = oracle.bwd_dw_bf16x(bits(dY), xd).astype(np.float32)
         R, Cc, st = oracle.adafactor_stats(g, cur, s_w, R, Cc, t, hpo)
-        cur, _ = oracle.adafactor_apply(g, cur, R, Cc, st["rbar"], st["step"], st["decay"], qmin,
+        cur, _ = oracle.adafactor_apply(g, cur, st["a"], st["b"], st["step"], st["decay"], qmin,
                                         qmax, 4, t, 2)
         dqt.dqt_bitlinear_bwd_dw_adafactor(dY.cuda(), xdq, W, s_w, Rg, Cg,
                                            dqt.adafactor(lr=1e-2, step=t),
