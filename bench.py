@@ -923,6 +923,8 @@ def main():
     ap.add_argument("--act", default="int8", choices=["int8", "fp8"],
                     help="mlp: 8-bit activations as int8 codes (default) or E4M3 (FP8 environment)")
     ap.add_argument("--decoder-size", default="130m", choices=sorted(DECODER_SIZES))
+    ap.add_argument("--tiles", type=int, default=0, choices=[0, 1],
+                    help="GEMM tiling: 0 = 2-SM 256 x 256 tiles (default), 1 = 1-SM 128 x 256 tiles")
     ap.add_argument("--optimizer", default="adamw", choices=["adamw", "adafactor"],
                     help="the DQT optimiser of the BitLinear weights")
     ap.add_argument("--packed", action="store_true", help="2-bit packed ternary code storage")
@@ -931,6 +933,10 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
+    if args.tiles and args.impl == "dqt":
+        from paper_2412_04787_gb300 import build as dqt_build, dqt
+        dqt_build.build()
+        dqt.dqt_set_gemm_tiles(args.tiles)
     if args.workload == "decoder" and args.impl == "dqt" and not args.kernel:
         run_decoder(args)
     elif args.kernel:
