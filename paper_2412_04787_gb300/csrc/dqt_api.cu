@@ -277,7 +277,16 @@ size_t dqt_bwd_dw_workspace_size(int64_t T, int64_t N, int64_t K) {
   if (T <= 0 || N <= 0 || K <= 0 || T > kMaxDim || N > kMaxDim || K > kMaxDim) return 0;
   if (dqt::gemm_mode() != 0) return 0;
   const int s = dqt::dw_splits(static_cast<int>(N), static_cast<int>(K), static_cast<int>(T));
-  return s > 1 ? static_cast<size_t>(s) * static_cast<size_t>(N) * static_cast<size_t>(K) * 4u : 0;
+  if (s > 1) return static_cast<size_t>(s) * static_cast<size_t>(N) * static_cast<size_t>(K) * 4u;
+  // last-wave tail: at most one 256 x 256 fp32 slice partial per cluster (at
+  // most one cluster per SM pair on any launch)
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const dqt::TailPlan tp =
+      dqt::tail_plan(static_cast<int>(N), static_cast<int>(K), static_cast<int>(T), sms / 2);
+  if (tp.splits < 2) return 0;
+  return static_cast<size_t>(sms / 2) * 65536 * sizeof(float);
 }
 
 int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W, float s_w,

@@ -54,6 +54,26 @@ struct GemmLaunch {
 // when given a workspace of dw_splits * M * N floats (1 = no split).
 int dw_splits(int M, int N, int Kred);
 
+// The last-wave tail of a 2-SM dW GEMM on `clusters` clusters: `tail` tiles
+// (tile indices full .. full + tail - 1) each cut into `splits` token slices
+// of `kbps` k-blocks; `bytes` of workspace for their partials (splits 0: no
+// tail split).
+struct TailPlan {
+  int splits, tail, full, kbps;
+  size_t bytes;
+};
+TailPlan tail_plan(int M, int N, int Kred, int clusters);
+
+// Sums the tail slices' partials (slice s of tail tile j at (s * tail + j) *
+// 65536 floats, tile-local row-major 256 x 256; tile full + j of an M x N
+// output with num_n tiles per row) in slice order and applies the update of
+// sr_update_kernel to W, m, v (if W) at the global element indices, and/or
+// writes the summed gradient to dW_out.
+int launch_tail_update(const float* part, int splits, int tail, int full, int num_n, int M, int N,
+                       int8_t* W, bool packed, float* m, float* v, const UpdateConsts& uc,
+                       const UpdateConsts* uc_dev, unsigned long long* changed, float* dW_out,
+                       cudaStream_t stream);
+
 // Sum `splits` fp32 slabs (stride `slab` elements) in slice order and apply
 // the update to W, m, v (numel elements); optionally write the sum to g_out.
 int launch_sr_update_slabs(const float* slabs, int splits, long long slab, int8_t* W, float* m,

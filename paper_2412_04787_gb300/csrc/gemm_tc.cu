@@ -73,7 +73,41 @@ struct Params {
   // partial goes to dW_out + s * slab
   int splits, kb_per_split;
   long long slab;
+  // tail (2-SM dW with splits == 1): units below full_units are whole tiles
+  // with the fused epilogue; the tiles from full_tiles on are each cut into
+  // tail_splits token slices of tail_kbps k-blocks, one unit each, whose fp32
+  // partials go to `part` (slice s of tail tile j at (s * tail_tiles + j) *
+  // 65536 floats, tile-local row-major 256 x 256) for a streaming kernel that
+  // sums them in slice order and applies the update.
+  int full_units, full_tiles, tail_tiles, tail_splits, tail_kbps;
+  float* part;
 };
+
+struct Unit {
+  int tile, kb0, kb1;
+  int slab;   // split-T slab of the unit's partial (0 without split-T)
+  int slice;  // tail slice, -1 for a whole tile
+};
+
+__device__ __forceinline__ Unit decode_unit(const Params& p, int t) {
+  Unit u;
+  if (t < p.full_units) {
+    u.tile = t / p.splits;
+    u.slab = t - u.tile * p.splits;
+    u.kb0 = u.slab * p.kb_per_split;
+    u.kb1 = min(p.num_kb, u.kb0 + p.kb_per_split);
+    u.slice = -1;
+  } else {
+    const int q = t - p.full_units;
+    const int j = q / p.tail_splits;
+    u.tile = p.full_tiles + j;
+    u.slice = q - j * p.tail_splits;
+    u.slab = 0;
+    u.kb0 = u.slice * p.tail_kbps;
+    u.kb1 = min(p.num_kb, u.kb0 + p.tail_kbps);
+  }
+  return u;
+}
 
 constexpr int kStageLd = 33;  // padded row pitch (floats) of the epilogue transpose buffer
 
@@ -618,9 +652,8 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
       int it = 0;
       bool ok = true;
       for (int t = cid; t < p.num_tiles && ok; t += ncl) {
-        const int tile = t / p.splits;
-        const int kb0 = (t - tile * p.splits) * p.kb_per_split;
-        const int kb1 = min(p.num_kb, kb0 + p.kb_per_split);
+        const Unit un = decode_unit(p, t);
+        const int tile = un.tile, kb0 = un.kb0, kb1 = un.kb1;
         const int m0 = (tile / p.num_n) * 256 + static_cast<int>(rank) * 128;
         const int n0 = (tile % p.num_n) * BN + static_cast<int>(rank) * 128;
         for (int kb = kb0; kb < kb1; ++kb, ++it) {
@@ -665,9 +698,8 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
       int u = 0;
       bool ok = true;
       for (int t = cid; t < p.num_tiles && ok; t += ncl) {
-        const int tile = t / p.splits;
-        const int kb0 = (t - tile * p.splits) * p.kb_per_split;
-        const int kb1 = min(p.num_kb, kb0 + p.kb_per_split);
+        const Unit un = decode_unit(p, t);
+        const int kb0 = un.kb0, kb1 = un.kb1;
         for (int kb = kb0; kb < kb1; ++kb, ++it) {
           const int b = u & 1;
           if (kb == kb0 && u >= 2) {
@@ -719,8 +751,9 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
     int u = 0;
     bool ok = true;
     for (int t = cid; t < p.num_tiles && ok; t += ncl, ++u) {
-      const int tile = t / p.splits;
-      float* dw_out = p.dW_out ? p.dW_out + (t - tile * p.splits) * p.slab : nullptr;
+      const Unit un = decode_unit(p, t);
+      const int tile = un.tile;
+      float* dw_out = p.dW_out ? p.dW_out + un.slab * p.slab : nullptr;
       const int gm = (tile / p.num_n) * 256 + static_cast<int>(rank) * 128 + row;
       const int nbase = (tile % p.num_n) * BN + half * HALF;
       const bool row_ok = gm < p.M;
@@ -731,7 +764,25 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
       if (!ok) break;
       tc_fence_after();
       const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(b * BN + half * HALF);
-      if (EPI == GEMM_DW) {
+      if (EPI == GEMM_DW && un.slice >= 0) {
+        // a tail slice: its fp32 partial to the slice buffer, tile-local
+        // row-major (this lane's row, 32 columns per chunk: 128 contiguous bytes)
+        float* dst_tile = p.part + (static_cast<long long>(un.slice) * p.tail_tiles +
+                                    (tile - p.full_tiles)) * 65536LL +
+                          (static_cast<long long>(rank) * 128 + row) * 256 + half * HALF;
+#pragma unroll 1
+        for (int cc = 0; cc < HALF / 32; ++cc) {
+          uint32_t a[32];
+          tmem_ld_32x32b_x32(t_acc + cc * 32, a);
+          tmem_ld_wait();
+          float4* dst = reinterpret_cast<float4*>(dst_tile + cc * 32);
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            __stcg(dst + j, make_float4(__uint_as_float(a[4 * j]), __uint_as_float(a[4 * j + 1]),
+                                        __uint_as_float(a[4 * j + 2]),
+                                        __uint_as_float(a[4 * j + 3])));
+        }
+      } else if (EPI == GEMM_DW) {
         n_changed += epi_dw_tile<false, PK>(p, uc, dw_out, gm - lane, nbase, HALF / 32, t_acc, xp, lane);
       } else
 #pragma unroll 1
@@ -827,9 +878,38 @@ int launch_tiles(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStr
 }
 
 template <bool A_MN, bool B_MN, int EPI, bool PK = false>
-int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream);
+int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream,
+                 void* tail_ws = nullptr, size_t tail_ws_bytes = 0, TailPlan* plan = nullptr);
 
 }  // namespace
+
+// Tail of a 2-SM dW GEMM on `clusters` clusters: the tiles past the last
+// full wave are cut into S token slices (about `clusters` units in the last
+// wave, each slice at least 4 k-blocks long, S <= 16), so that the last wave
+// costs a fraction of a tile's reduction, and their update moves out of the
+// GEMM's epilogue into a streaming kernel.
+TailPlan tail_plan(int M, int N, int Kred, int clusters) {
+  TailPlan t{0, 0, 0, 0, 0};
+  const int tiles = ((M + 255) / 256) * ((N + 255) / 256);
+  const int num_kb = (Kred + BK - 1) / BK;
+  if (clusters < 2) return t;
+  const int full = (tiles / clusters) * clusters;
+  const int tail = tiles - full;
+  if (full == 0 || tail == 0) return t;
+  int S = clusters / tail;
+  if (S > num_kb / 4) S = num_kb / 4;
+  if (S > 16) S = 16;
+  if (S < 2) return t;
+  const int kbps = (num_kb + S - 1) / S;
+  S = (num_kb + kbps - 1) / kbps;  // no empty slice
+  if (S < 2) return t;
+  t.splits = S;
+  t.tail = tail;
+  t.full = full;
+  t.kbps = kbps;
+  t.bytes = static_cast<size_t>(tail) * S * 65536 * sizeof(float);
+  return t;
+}
 
 // Token slices for a 2-SM dW GEMM whose output tiles would leave most SM
 // pairs idle: enough slices to give every pair a unit of work, each slice at
@@ -851,7 +931,8 @@ int dw_splits(int M, int N, int Kred) {
 namespace {
 
 template <bool A_MN, bool B_MN, int EPI, bool PK>
-int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream) {
+int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream,
+                 void* tail_ws, size_t tail_ws_bytes, TailPlan* plan) {
   auto kern = gemm_pair_kernel<A_MN, B_MN, EPI, PK>;
   const int smem = SmemPair<EPI>::BYTES;
   constexpr int threads = PairCfg<EPI>::THREADS;
@@ -880,6 +961,26 @@ int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStr
     int n = 0;
     if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n < 1) return 3;
     max_clusters = n;
+  }
+  p.full_units = p.num_tiles;
+  p.full_tiles = p.num_tiles;
+  p.tail_tiles = 0;
+  p.tail_splits = 1;
+  p.tail_kbps = p.num_kb;
+  p.part = nullptr;
+  if (plan) *plan = TailPlan{0, 0, 0, 0, 0};
+  if (EPI == GEMM_DW && tail_ws && plan && p.splits == 1) {
+    const TailPlan tp = tail_plan(p.M, p.N, p.Kred, max_clusters);
+    if (tp.splits >= 2 && tp.bytes <= tail_ws_bytes) {
+      p.full_units = tp.full;
+      p.full_tiles = tp.full;
+      p.tail_tiles = tp.tail;
+      p.tail_splits = tp.splits;
+      p.tail_kbps = tp.kbps;
+      p.part = static_cast<float*>(tail_ws);
+      p.num_tiles = tp.full + tp.tail * tp.splits;
+      *plan = tp;
+    }
   }
   const int clusters = p.num_tiles < max_clusters ? p.num_tiles : max_clusters;
   cfg.gridDim = dim3(2 * clusters, 1, 1);
@@ -960,9 +1061,19 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
       if (!make_map(&ta, g.A, g.M, g.Kred, 64, BK)) return 3;
       if (!make_map(&tb, g.B, g.N, g.Kred, 64, BK)) return 3;
       if (!g2.pair) return launch_tiles<256, true, true, GEMM_DW, false>(ta, tb, p, stream);
-      if (p.splits == 1)
-        return p.packed && p.W ? launch_pairs<true, true, GEMM_DW, true>(ta, tb, p, stream)
-                               : launch_pairs<true, true, GEMM_DW>(ta, tb, p, stream);
+      if (p.splits == 1) {
+        // the last wave's tiles as token slices, their update in a streaming pass
+        TailPlan tp{0, 0, 0, 0, 0};
+        const int rc = p.packed && p.W
+                           ? launch_pairs<true, true, GEMM_DW, true>(ta, tb, p, stream, g.ws,
+                                                                      g.ws_bytes, &tp)
+                           : launch_pairs<true, true, GEMM_DW>(ta, tb, p, stream, g.ws, g.ws_bytes,
+                                                               &tp);
+        if (rc || tp.splits == 0) return rc;
+        return launch_tail_update(static_cast<const float*>(g.ws), tp.splits, tp.tail, tp.full,
+                                  (g.N + 255) / 256, g.M, g.N, g.W, g.packed, g.m, g.v, g.uc,
+                                  g.uc_dev, g.changed, g.dW_out, stream);
+      }
       // split-T: fp32 partials of each token slice into the workspace slabs,
       // then one streaming pass sums the slabs in slice order and applies the
       // AdamW + stochastic-rounding update (and writes the summed gradient to

@@ -115,6 +115,71 @@ __global__ void __launch_bounds__(kThreads)
     for (int64_t e = ngroups << 2; e < slab; ++e) out[e] = slab_grad1(slabs, nsplit, slab, e);
 }
 
+// The deferred last-wave tail of the fused dW GEMM: each thread step takes
+// four consecutive columns of one row of a tail tile, sums the token slices'
+// partials in slice order, and applies the same update as sr_update_kernel at
+// the global element index (so the Philox words are those of the fused path).
+__global__ void __launch_bounds__(kThreads)
+    tail_update_kernel(const float* __restrict__ part, int splits, int tail, int full, int num_n,
+                       int M, int N, int8_t* __restrict__ W, bool packed, float* __restrict__ m,
+                       float* __restrict__ v, const UpdateConsts uc_arg,
+                       const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed,
+                       float* __restrict__ dW_out) {
+  const UpdateConsts uc = uc_dev ? *uc_dev : uc_arg;
+  uint8_t* Wp = reinterpret_cast<uint8_t*>(W);
+  const int64_t ngroups = static_cast<int64_t>(tail) * 16384;  // 256 x 256 / 4 per tile
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * kThreads;
+  uint32_t n_changed = 0;
+  for (int64_t gi = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; gi < ngroups;
+       gi += stride) {
+    const int j = static_cast<int>(gi >> 14);
+    const int r = static_cast<int>((gi >> 6) & 255);
+    const int c4 = static_cast<int>(gi & 63) * 4;
+    const int tile = full + j;
+    const int row = (tile / num_n) * 256 + r;
+    const int col = (tile % num_n) * 256 + c4;
+    if (row >= M || col >= N) continue;  // N % 4 == 0: the whole group is in range
+    const float* src = part + static_cast<int64_t>(j) * 65536 + r * 256 + c4;
+    float4 g4 = __ldcs(reinterpret_cast<const float4*>(src));
+    for (int s = 1; s < splits; ++s) {
+      const float4 h =
+          __ldcs(reinterpret_cast<const float4*>(src + static_cast<int64_t>(s) * tail * 65536));
+      g4.x = __fadd_rn(g4.x, h.x);
+      g4.y = __fadd_rn(g4.y, h.y);
+      g4.z = __fadd_rn(g4.z, h.z);
+      g4.w = __fadd_rn(g4.w, h.w);
+    }
+    const int64_t e = static_cast<int64_t>(row) * N + col;
+    if (dW_out) __stcs(reinterpret_cast<float4*>(dW_out + e), g4);
+    if (!W) continue;
+    float4 m4 = __ldcs(reinterpret_cast<const float4*>(m + e));
+    float4 v4 = __ldcs(reinterpret_cast<const float4*>(v + e));
+    const char4 c0 = packed ? tern_unpack4(Wp[e >> 2]) : *reinterpret_cast<const char4*>(W + e);
+    uint4 w = make_uint4(0, 0, 0, 0);
+    if (uc.round_mode == 0)
+      w = sr_words(static_cast<uint64_t>(e >> 2), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
+    const int32_t a = dqt_update_elem(uc, g4.x, c0.x, m4.x, v4.x, w.x);
+    const int32_t b = dqt_update_elem(uc, g4.y, c0.y, m4.y, v4.y, w.y);
+    const int32_t c = dqt_update_elem(uc, g4.z, c0.z, m4.z, v4.z, w.z);
+    const int32_t d = dqt_update_elem(uc, g4.w, c0.w, m4.w, v4.w, w.w);
+    n_changed += (a != c0.x) + (b != c0.y) + (c != c0.z) + (d != c0.w);
+    if (packed)
+      Wp[e >> 2] = static_cast<uint8_t>(tern_pack4(a, b, c, d));
+    else
+      *reinterpret_cast<char4*>(W + e) =
+          make_char4(static_cast<signed char>(a), static_cast<signed char>(b),
+                     static_cast<signed char>(c), static_cast<signed char>(d));
+    __stcs(reinterpret_cast<float4*>(m + e), m4);
+    __stcs(reinterpret_cast<float4*>(v + e), v4);
+  }
+  if (changed) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) n_changed += __shfl_xor_sync(0xffffffffu, n_changed, off);
+    if ((threadIdx.x & 31) == 0 && n_changed)
+      atomicAdd(changed, static_cast<unsigned long long>(n_changed));
+  }
+}
+
 int stream_blocks(int64_t numel) {
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
@@ -136,6 +201,15 @@ int launch_sr_update_slabs(const float* slabs, int splits, long long slab, int8_
   sr_update_kernel<<<stream_blocks(numel), kThreads, 0, stream>>>(slabs, splits, slab, g_out, W, m,
                                                                   v, numel, uc, uc_dev, changed,
                                                                   packed);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+int launch_tail_update(const float* part, int splits, int tail, int full, int num_n, int M, int N,
+                       int8_t* W, bool packed, float* m, float* v, const UpdateConsts& uc,
+                       const UpdateConsts* uc_dev, unsigned long long* changed, float* dW_out,
+                       cudaStream_t stream) {
+  tail_update_kernel<<<stream_blocks(static_cast<int64_t>(tail) * 65536), kThreads, 0, stream>>>(
+      part, splits, tail, full, num_n, M, N, W, packed, m, v, uc, uc_dev, changed, dW_out);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 

@@ -312,7 +312,10 @@ def test_fused_update_ragged():
 
 
 def test_fused_update_llama_mlp_sampled_rows():
-    _fused(8192, 2048, 5632, 1.58, 1, seed=51, rows=np.array([0, 127, 128, 3000, 5631]))
+    # rows from the first waves of tiles and from the last, partly idle, wave
+    _fused(8192, 2048, 5632, 1.58, 1, seed=51,
+           rows=np.array([0, 127, 128, 3000, 4864, 5200, 5631]))
+    _fused(8192, 5632, 2048, 1.58, 2, seed=52, rows=np.array([0, 1535, 1536, 1800, 2047]))
 
 
 def test_fused_equals_standalone_on_same_gradient():
