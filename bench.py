@@ -52,7 +52,9 @@ METRIC = "DQT BitLinear fwd+bwd+SR-update tokens/s"
 PROJ = [("gate", HID, INTER), ("up", HID, INTER), ("down", INTER, HID)]
 
 
-GEMM_SOURCES = ("gemm_tc.cu", "dqt_device.cuh")  # the GEMM kernels' device code
+# the device code of the GEMM kernels and of the streaming update that
+# finishes the weight-gradient GEMM's last wave
+GEMM_SOURCES = ("gemm_tc.cu", "dqt_device.cuh", "sr_update.cu")
 
 
 def kernel_fingerprint(files=GEMM_SOURCES):
@@ -67,12 +69,13 @@ def kernel_fingerprint(files=GEMM_SOURCES):
     return h.hexdigest()[:12]
 
 
-# DRAM bytes (read + write) per launch of the fused dW + update GEMM from one
-# ncu capture of the gate-shape launch (T=8192, K=2048, N=5632; the up and down
-# launches move the same numbers of operand and optimiser-state bytes), keyed
-# by the kernel fingerprint it was taken on (see profiles/).  A stale entry
+# DRAM bytes (read + write) of one gate-shape call of the fused dW + update
+# (T=8192, K=2048, N=5632: the 2-SM GEMM and the streaming kernel that
+# finishes its last-wave tiles; the up and down calls move the same numbers
+# of operand and optimiser-state bytes), from one ncu capture, keyed by the
+# GEMM-source fingerprint it was taken on (see profiles/).  A stale entry
 # reports null.
-DW_TRAFFIC_BYTES = {"5cd93cdc4c54": 295927296 + 57431552}
+DW_TRAFFIC_BYTES = {"dc302460ae86": 273493504 + 60064512 + 33048576}
 
 
 def _dist():
