@@ -199,14 +199,20 @@ int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t*
                                 size_t ws_bytes, void* stream);
 
 /* Workspace (bytes, 16-byte aligned device memory) that lets
- * dqt_bitlinear_bwd_dw_update reduce a weight gradient whose output is too
- * small to occupy the GPU (few 256 x 256 tiles, long token reduction) in
- * token slices: each slice's fp32 partial is written to the workspace and one
- * streaming pass sums the slices in slice order and applies the update.  0 =
- * no split for this shape on the current device (and under
- * dqt_set_gemm_tiles(1)).  Passing ws = NULL, or fewer bytes, always runs the
- * single fused kernel.  The split gives the same update up to the fp32
- * summation order of the gradient; it is deterministic for a given shape. */
+ * dqt_bitlinear_bwd_dw_update cut token reductions into slices:
+ *  - a weight gradient whose output is too small to occupy the GPU (few
+ *    256 x 256 tiles, long token reduction) is reduced in token slices
+ *    throughout;
+ *  - otherwise, when the output's tiles do not fill the last wave of SM pairs,
+ *    the tiles of that wave are reduced in token slices, so that the last
+ *    wave is short.
+ * Each slice's fp32 partial goes to the workspace and one streaming pass sums
+ * the slices in slice order and applies the update (bit-identical to
+ * dqt_sr_update on that summed gradient).  0 = neither applies to this shape
+ * on the current device (or under dqt_set_gemm_tiles(1)).  Passing ws = NULL,
+ * or fewer bytes, always runs the single fused kernel.  Slicing gives the same
+ * update up to the fp32 summation order of the gradient; it is deterministic
+ * for a given shape and device. */
 size_t dqt_bwd_dw_workspace_size(int64_t T, int64_t N, int64_t K);
 
 /* The AdamW + SR update of dqt_bitlinear_bwd_dw_update for a gradient already
