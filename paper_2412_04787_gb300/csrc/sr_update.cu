@@ -37,22 +37,26 @@ __device__ __forceinline__ float slab_grad1(const float* __restrict__ grad, int 
   return g;
 }
 
+// DEV: the constants are read from device memory (else the kernel's
+// parameter space); SLABS: the gradient may be split into slabs and the
+// summed gradient written out.  The plain instance is the leanest stream.
+template <bool packed, bool DEV, bool SLABS>
 __global__ void __launch_bounds__(kThreads)
     sr_update_kernel(const float* __restrict__ grad, int nsplit, long long slab,
                      float* __restrict__ g_out, int8_t* __restrict__ W, float* __restrict__ m,
                      float* __restrict__ v, int64_t numel, const UpdateConsts uc_arg,
-                     const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed,
-                     bool packed) {
+                     const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed) {
   uint8_t* Wp = reinterpret_cast<uint8_t*>(W);
-  const UpdateConsts uc = uc_dev ? *uc_dev : uc_arg;
+  const UpdateConsts uc = DEV ? *uc_dev : uc_arg;
   const int64_t ngroups = numel >> 2;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * kThreads;
   uint32_t n_changed = 0;
   for (int64_t gi = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; gi < ngroups;
        gi += stride) {
     const int64_t e = gi << 2;
-    const float4 g4 = slab_grad4(grad, nsplit, slab, e);
-    if (g_out) __stcs(reinterpret_cast<float4*>(g_out + e), g4);
+    const float4 g4 = SLABS ? slab_grad4(grad, nsplit, slab, e)
+                            : __ldcs(reinterpret_cast<const float4*>(grad + e));
+    if (SLABS && g_out) __stcs(reinterpret_cast<float4*>(g_out + e), g4);
     float4 m4 = __ldcs(reinterpret_cast<const float4*>(m + e));
     float4 v4 = __ldcs(reinterpret_cast<const float4*>(v + e));
     const char4 c4 = packed ? tern_unpack4(Wp[gi]) : *reinterpret_cast<const char4*>(W + e);
@@ -84,8 +88,8 @@ __global__ void __launch_bounds__(kThreads)
       float mm = m[e], vv = v[e];
       const int j = static_cast<int>(e & 3);
       const int32_t c0 = packed ? (j == 0 ? pc.x : j == 1 ? pc.y : pc.z) : W[e];
-      const float g = slab_grad1(grad, nsplit, slab, e);
-      if (g_out) g_out[e] = g;
+      const float g = SLABS ? slab_grad1(grad, nsplit, slab, e) : grad[e];
+      if (SLABS && g_out) g_out[e] = g;
       const int32_t r = dqt_update_elem(uc, g, c0, mm, vv, ws[j]);
       n_changed += (r != c0);
       if (packed) pr[j] = r;
@@ -119,13 +123,14 @@ __global__ void __launch_bounds__(kThreads)
 // four consecutive columns of one row of a tail tile, sums the token slices'
 // partials in slice order, and applies the same update as sr_update_kernel at
 // the global element index (so the Philox words are those of the fused path).
+template <bool DEV>
 __global__ void __launch_bounds__(kThreads)
     tail_update_kernel(const float* __restrict__ part, int splits, int tail, int full, int num_n,
                        int M, int N, int8_t* __restrict__ W, bool packed, float* __restrict__ m,
                        float* __restrict__ v, const UpdateConsts uc_arg,
                        const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed,
                        float* __restrict__ dW_out) {
-  const UpdateConsts uc = uc_dev ? *uc_dev : uc_arg;
+  const UpdateConsts uc = DEV ? *uc_dev : uc_arg;
   uint8_t* Wp = reinterpret_cast<uint8_t*>(W);
   const int64_t ngroups = static_cast<int64_t>(tail) * 16384;  // 256 x 256 / 4 per tile
   const int64_t stride = static_cast<int64_t>(gridDim.x) * kThreads;
@@ -194,13 +199,48 @@ int stream_blocks(int64_t numel) {
 
 }  // namespace
 
+namespace {
+
+template <bool packed, bool DEV, bool SLABS>
+void sr_launch(const float* grad, int splits, long long slab, float* g_out, int8_t* W, float* m,
+               float* v, int64_t numel, const UpdateConsts& uc, const UpdateConsts* uc_dev,
+               unsigned long long* changed, cudaStream_t stream) {
+  sr_update_kernel<packed, DEV, SLABS><<<stream_blocks(numel), kThreads, 0, stream>>>(
+      grad, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed);
+}
+
+template <bool packed>
+void sr_dispatch(const float* grad, int splits, long long slab, float* g_out, int8_t* W, float* m,
+                 float* v, int64_t numel, const UpdateConsts& uc, const UpdateConsts* uc_dev,
+                 unsigned long long* changed, cudaStream_t stream) {
+  const bool slabs = splits > 1 || g_out;
+  if (uc_dev) {
+    if (slabs)
+      sr_launch<packed, true, true>(grad, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed,
+                                    stream);
+    else
+      sr_launch<packed, true, false>(grad, 1, 0, nullptr, W, m, v, numel, uc, uc_dev, changed,
+                                     stream);
+  } else {
+    if (slabs)
+      sr_launch<packed, false, true>(grad, splits, slab, g_out, W, m, v, numel, uc, nullptr,
+                                     changed, stream);
+    else
+      sr_launch<packed, false, false>(grad, 1, 0, nullptr, W, m, v, numel, uc, nullptr, changed,
+                                      stream);
+  }
+}
+
+}  // namespace
+
 int launch_sr_update_slabs(const float* slabs, int splits, long long slab, int8_t* W, float* m,
                            float* v, int64_t numel, const UpdateConsts& uc,
                            const UpdateConsts* uc_dev, unsigned long long* changed, float* g_out,
                            cudaStream_t stream, bool packed) {
-  sr_update_kernel<<<stream_blocks(numel), kThreads, 0, stream>>>(slabs, splits, slab, g_out, W, m,
-                                                                  v, numel, uc, uc_dev, changed,
-                                                                  packed);
+  if (packed)
+    sr_dispatch<true>(slabs, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed, stream);
+  else
+    sr_dispatch<false>(slabs, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed, stream);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
@@ -208,8 +248,15 @@ int launch_tail_update(const float* part, int splits, int tail, int full, int nu
                        int8_t* W, bool packed, float* m, float* v, const UpdateConsts& uc,
                        const UpdateConsts* uc_dev, unsigned long long* changed, float* dW_out,
                        cudaStream_t stream) {
-  tail_update_kernel<<<stream_blocks(static_cast<int64_t>(tail) * 65536), kThreads, 0, stream>>>(
-      part, splits, tail, full, num_n, M, N, W, packed, m, v, uc, uc_dev, changed, dW_out);
+  const int blocks = stream_blocks(static_cast<int64_t>(tail) * 65536);
+  if (uc_dev)
+    tail_update_kernel<true><<<blocks, kThreads, 0, stream>>>(part, splits, tail, full, num_n, M, N,
+                                                              W, packed, m, v, uc, uc_dev, changed,
+                                                              dW_out);
+  else
+    tail_update_kernel<false><<<blocks, kThreads, 0, stream>>>(part, splits, tail, full, num_n, M,
+                                                               N, W, packed, m, v, uc, nullptr,
+                                                               changed, dW_out);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
@@ -222,9 +269,10 @@ int launch_slab_sum(const float* slabs, int splits, long long slab, float* out,
 int launch_sr_update(const float* grad, int8_t* W, float* m, float* v, int64_t numel,
                      const UpdateConsts& uc, const UpdateConsts* uc_dev,
                      unsigned long long* changed, cudaStream_t stream, bool packed) {
-  sr_update_kernel<<<stream_blocks(numel), kThreads, 0, stream>>>(grad, 1, 0, nullptr, W, m, v,
-                                                                  numel, uc, uc_dev, changed,
-                                                                  packed);
+  if (packed)
+    sr_dispatch<true>(grad, 1, 0, nullptr, W, m, v, numel, uc, uc_dev, changed, stream);
+  else
+    sr_dispatch<false>(grad, 1, 0, nullptr, W, m, v, numel, uc, uc_dev, changed, stream);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
