@@ -75,7 +75,7 @@ def kernel_fingerprint(files=GEMM_SOURCES):
 # of operand and optimiser-state bytes), from one ncu capture, keyed by the
 # GEMM-source fingerprint it was taken on (see profiles/).  A stale entry
 # reports null.
-DW_TRAFFIC_BYTES = {"dc302460ae86": 273493504 + 60064512 + 33048576}
+DW_TRAFFIC_BYTES = {"d3fc5601e4d7": 273736448 + 60078080 + 33047808}
 
 
 def _dist():
@@ -145,7 +145,7 @@ class ClockSampler:
 class MLPStep:
     """Device buffers and the launch sequence of one DQT MLP training step."""
 
-    def __init__(self, dev, seed=1234, fp8=False, optimizer="adamw", packed=False):
+    def __init__(self, dev, seed=1234, fp8=False, optimizer="adamw", packed=False, bits=1.58):
         from paper_2412_04787_gb300 import dqt, inputs
 
         self.dqt = dqt
@@ -153,7 +153,8 @@ class MLPStep:
         self.fp8 = fp8
         self.optimizer = optimizer
         self.packed = packed
-        self.grid = dqt.grid(1.58)
+        self.bits = bits
+        self.grid = dqt.grid(bits)
         T = T_TOK
         # two seeded input sets, alternated step by step, so that the
         # optimiser sees changing gradients as in training
@@ -382,7 +383,8 @@ def run_gpu(args):
     torch.cuda.set_device(dev)
     from paper_2412_04787_gb300 import build as dqt_build
     dqt_build.build()
-    st = MLPStep(dev, fp8=args.act == "fp8", optimizer=args.optimizer, packed=args.packed)
+    st = MLPStep(dev, fp8=args.act == "fp8", optimizer=args.optimizer, packed=args.packed,
+                 bits=args.bits)
     dqt = st.dqt
     stream = torch.cuda.current_stream()
 
@@ -542,12 +544,16 @@ def run_gpu(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "e4m3 forward, bf16 backward" if st.fp8 else "bf16",
-            "data": "synthetic (seeded N(0,1) activations, N(0,1e-2) gradients, AbsMean-ternary codes of N(0,0.02))",
-            "config": {"workload": WORKLOAD + (", FP8 (E4M3) forward" if st.fp8 else "") +
+            "data": "synthetic (seeded N(0,1) activations, N(0,1e-2) gradients, AbsMean-%s codes of N(0,0.02))"
+                    % ("ternary" if st.bits == 1.58 else "%d-bit" % st.bits),
+            "config": {"workload": (WORKLOAD if st.bits == 1.58 else
+                                    WORKLOAD.replace("ternary", "%d-bit" % st.bits)) +
+                                   (", FP8 (E4M3) forward" if st.fp8 else "") +
                                    (", Adafactor" if st.optimizer == "adafactor" else "") +
                                    (", 2-bit packed codes" if st.packed else ""),
                        "tokens": T_TOK, "hidden": HID, "intermediate": INTER,
-                       "weights": "ternary codes, %s" % ("2-bit packed" if st.packed else "int8"),
+                       "weights": "%s codes, %s" % ("ternary" if st.bits == 1.58 else "%d-bit" % st.bits,
+                                                     "2-bit packed" if st.packed else "int8"),
                        "optimizer": st.optimizer,
                        "parallelism": "replicas" if ws > 1 else "single GPU",
                        "l2": "inputs larger than L2 (step working set ~1.5 GB > 129 MB)"},
@@ -658,7 +664,7 @@ def run_kernel(args):
     T, K, N = T_TOK, HID, INTER
     if args.shape:
         T, K, N = (int(x) for x in args.shape.split(","))
-    g = dqt.grid(1.58)
+    g = dqt.grid(args.bits)
     k = args.kernel
     if k in ("sr_update", "sr_update_packed"):
         n = args.numel
@@ -812,7 +818,8 @@ def run_decoder(args):
     sz = DECODER_SIZES[args.decoder_size]
     B, S = sz["batch"], sz["seq"]
     cfg = DecoderConfig(layers=sz["layers"], hidden=sz["hidden"], heads=sz["heads"], ffn=sz["ffn"],
-                        vocab=32000, bits=1.58, lr=1e-2 if args.optimizer == "adafactor" else 1e-3,
+                        vocab=32000, bits=args.bits,
+                        lr=1e-2 if args.optimizer == "adafactor" else 1e-3,
                         seed=1234, act=args.act, optimizer=args.optimizer, packed=args.packed)
     model = DQTDecoder(cfg, device=dev)
     # CUDA-graph replay needs the device-resident AdamW constants (int8 codes)
@@ -896,8 +903,10 @@ def run_decoder(args):
         "vs_baseline": None,
         "dtype": "e4m3 BitLinear forward, bf16 elsewhere" if args.act == "fp8" else "bf16",
         "data": "synthetic uniform token ids",
-        "config": {"workload": "LLaMA-structured decoder (%s), ternary DQT BitLinear in q,k,v,o,gate,up,down%s%s%s"
-                               % (args.decoder_size, ", FP8 (E4M3) forward" if args.act == "fp8" else "",
+        "config": {"workload": "LLaMA-structured decoder (%s), %s DQT BitLinear in q,k,v,o,gate,up,down%s%s%s"
+                               % (args.decoder_size,
+                                  "ternary" if args.bits == 1.58 else "%d-bit" % args.bits,
+                                  ", FP8 (E4M3) forward" if args.act == "fp8" else "",
                                   ", Adafactor" if args.optimizer == "adafactor" else "",
                                   ", 2-bit packed codes" if args.packed else ""),
                    "layers": cfg.layers, "hidden": cfg.hidden, "heads": cfg.heads, "ffn": cfg.ffn,
@@ -931,6 +940,8 @@ def main():
     ap.add_argument("--optimizer", default="adamw", choices=["adamw", "adafactor"],
                     help="the DQT optimiser of the BitLinear weights")
     ap.add_argument("--packed", action="store_true", help="2-bit packed ternary code storage")
+    ap.add_argument("--bits", type=float, default=1.58,
+                    help="weight grid: 1.58 (ternary, the default) or an integer width 2..8")
     ap.add_argument("--workload", default="mlp", choices=["mlp", "decoder"],
                     help="mlp: the headline BitLinear MLP GEMM set; decoder: a 12-layer DQT decoder step")
     args = ap.parse_args()
