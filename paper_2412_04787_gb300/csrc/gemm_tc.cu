@@ -179,6 +179,35 @@ __device__ __forceinline__ void epi_fwd(const Params& p, int gm, int gn0, float 
   }
 }
 
+// The forward's output from exact int32 accumulators (drained chunks).
+__device__ __forceinline__ void epi_fwd_int(const Params& p, int gm, int gn0, float a_t,
+                                            const int32_t (&acc)[32]) {
+  __nv_bfloat16* yrow = p.out_bf16 + static_cast<size_t>(gm) * p.N + gn0;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    if (gn0 + 8 * j >= p.N) break;
+    uint4 pk;
+    pk.x = pack_bf16x2(__fmul_rn(__int2float_rn(acc[8 * j + 0]), a_t),
+                       __fmul_rn(__int2float_rn(acc[8 * j + 1]), a_t));
+    pk.y = pack_bf16x2(__fmul_rn(__int2float_rn(acc[8 * j + 2]), a_t),
+                       __fmul_rn(__int2float_rn(acc[8 * j + 3]), a_t));
+    pk.z = pack_bf16x2(__fmul_rn(__int2float_rn(acc[8 * j + 4]), a_t),
+                       __fmul_rn(__int2float_rn(acc[8 * j + 5]), a_t));
+    pk.w = pack_bf16x2(__fmul_rn(__int2float_rn(acc[8 * j + 6]), a_t),
+                       __fmul_rn(__int2float_rn(acc[8 * j + 7]), a_t));
+    *reinterpret_cast<uint4*>(yrow + 8 * j) = pk;
+  }
+  if (p.acc_out) {
+    int32_t* arow = p.acc_out + static_cast<size_t>(gm) * p.N + gn0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      if (gn0 + 4 * j >= p.N) break;
+      *reinterpret_cast<int4*>(arow + 4 * j) =
+          make_int4(acc[4 * j], acc[4 * j + 1], acc[4 * j + 2], acc[4 * j + 3]);
+    }
+  }
+}
+
 __device__ __forceinline__ void epi_dx(const Params& p, int gm, int gn0, const uint32_t (&a)[32]) {
   __nv_bfloat16* yrow = p.out_bf16 + static_cast<size_t>(gm) * p.N + gn0;
   const float* f = reinterpret_cast<const float*>(a);
@@ -557,15 +586,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 // Epilogue warps of the 2-SM kernels: the dW update is compute-heavy (AdamW,
 // Philox, stochastic rounding per weight) and needs four warps per SM
 // sub-partition to hide its latencies; the forward and dX epilogues are light.
-template <int EPI>
+template <int EPI, bool DR = false>
 struct PairCfg {
-  static constexpr int EW = (EPI == GEMM_DW) ? 16 : 8;
+  // DR: the exact forward that drains its fp32 accumulator into int32 sums;
+  // its folds stall the MMAs, so they are spread over twice the warps
+  static constexpr int EW = (EPI == GEMM_DW || DR) ? 16 : 8;
   static constexpr int THREADS = 64 + 32 * EW;
 };
 
-template <int EPI>
+template <int EPI, bool DR = false>
 struct SmemPair {
-  static constexpr int EW = PairCfg<EPI>::EW;
+  static constexpr int EW = PairCfg<EPI, DR>::EW;
   static constexpr int A_BYTES = 128 * BK * 2;
   static constexpr int B_BYTES = 128 * BK * 2;  // this CTA's half of the B tile
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
@@ -580,11 +611,17 @@ struct SmemPair {
   static_assert((2 * STAGES + 5) * 8 + 4 <= 176, "barrier area: barriers, then the update constants");
 };
 
-template <bool A_MN, bool B_MN, int EPI, bool PK = false>
-__global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
+// DR (forward only): every chunk of chunk_kb k-blocks is accumulated on its
+// own (an exact fp32 integer sum) in the two alternating accumulators, and
+// the epilogue warps fold each chunk into running int32 sums held in their
+// registers (64 per lane), then write Y from them after the tile's last
+// chunk; the MMAs of the next chunk run meanwhile.
+template <bool A_MN, bool B_MN, int EPI, bool PK = false, bool DR = false>
+__global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
     gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA,
                      const __grid_constant__ CUtensorMap tmB, const Params p) {
-  using S = SmemPair<EPI>;
+  using S = SmemPair<EPI, DR>;
+  static_assert(!DR || EPI == GEMM_FWD, "drained chunks: exact integer forward only");
   constexpr int ST = S::STAGES;
   constexpr int EW = S::EW;
   constexpr int BN = 256;           // pair tile width; each CTA holds all 256 columns of its rows
@@ -701,8 +738,11 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
         const Unit un = decode_unit(p, t);
         const int kb0 = un.kb0, kb1 = un.kb1;
         for (int kb = kb0; kb < kb1; ++kb, ++it) {
+          // two accumulators alternating per unit; DR: a unit is one chunk of
+          // chunk_kb k-blocks, whose exact sum the epilogue folds into int32
+          const int kc = DR ? (kb - kb0) % p.chunk_kb : kb - kb0;
           const int b = u & 1;
-          if (kb == kb0 && u >= 2) {
+          if (kc == 0 && u >= 2) {
             if (!mbar_wait_cl(&acc_empty[b], ((u >> 1) - 1) & 1u, p.wait_ns)) {
               ok = false;
               break;
@@ -725,11 +765,11 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
                                      : sdesc_sw128(a_base + ks * 32, 16, 1024);
             const uint64_t bd = B_MN ? sdesc_sw128(b_base + ks * 2048, MN_CHUNK_BYTES, 1024)
                                      : sdesc_sw128(b_base + ks * 32, 16, 1024);
-            if (F8) umma_f8_pair(d, ad, bd, IDESC, (kb > kb0 || ks > 0) ? 1u : 0u);
-            else umma_bf16_pair(d, ad, bd, IDESC, (kb > kb0 || ks > 0) ? 1u : 0u);
+            if (F8) umma_f8_pair(d, ad, bd, IDESC, (kc > 0 || ks > 0) ? 1u : 0u);
+            else umma_bf16_pair(d, ad, bd, IDESC, (kc > 0 || ks > 0) ? 1u : 0u);
           }
           umma_commit_pair_mc(&empty[s], 0x3);
-          if (kb == kb1 - 1) {
+          if (kb == kb1 - 1 || (DR && kc == p.chunk_kb - 1)) {
             umma_commit_pair_mc(&acc_full[b], 0x3);
             ++u;
           }
@@ -759,6 +799,40 @@ __global__ void __launch_bounds__(PairCfg<EPI>::THREADS, 1)
       const bool row_ok = gm < p.M;
       float a_t = 0.0f;
       if ((EPI == GEMM_FWD || F8) && row_ok) a_t = __fdiv_rn(1.0f, __fmul_rn(p.s_x[gm], p.scale));
+      if (DR) {
+        static_assert(!DR || HALF == 64, "two 32-column chunks of running sums per lane");
+        const int nchunks = (p.num_kb + p.chunk_kb - 1) / p.chunk_kb;
+        int32_t run0[32], run1[32];
+        for (int c = 0; c < nchunks; ++c, ++u) {
+          const int b = u & 1;
+          ok = __all_sync(0xffffffffu, mbar_wait_cl(&acc_full[b], (u >> 1) & 1u, p.wait_ns));
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(b * BN + half * HALF);
+          // 16 columns at a time: 64 running sums + 16 loaded values per lane
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            uint32_t a[16];
+            tmem_ld_32x32b_x16(t_acc + 16 * q, a);
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              int32_t& rr = q < 2 ? run0[16 * q + i] : run1[16 * (q - 2) + i];
+              rr = (c > 0 ? rr : 0) + __float2int_rn(__uint_as_float(a[i]));
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cluster(acc_empty_lead + 8u * b);
+        }
+        if (!ok) break;
+        if (row_ok) {
+          if (nbase < p.N) epi_fwd_int(p, gm, nbase, a_t, run0);
+          if (nbase + 32 < p.N) epi_fwd_int(p, gm, nbase + 32, a_t, run1);
+        }
+        --u;  // the loop header counts one unit per tile
+        continue;
+      }
       const int b = u & 1;
       ok = __all_sync(0xffffffffu, mbar_wait_cl(&acc_full[b], (u >> 1) & 1u, p.wait_ns));
       if (!ok) break;
@@ -877,7 +951,7 @@ int launch_tiles(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStr
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
-template <bool A_MN, bool B_MN, int EPI, bool PK = false>
+template <bool A_MN, bool B_MN, int EPI, bool PK = false, bool DR = false>
 int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream,
                  void* tail_ws = nullptr, size_t tail_ws_bytes = 0, TailPlan* plan = nullptr);
 
@@ -930,12 +1004,12 @@ int dw_splits(int M, int N, int Kred) {
 
 namespace {
 
-template <bool A_MN, bool B_MN, int EPI, bool PK>
+template <bool A_MN, bool B_MN, int EPI, bool PK, bool DR>
 int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream,
                  void* tail_ws, size_t tail_ws_bytes, TailPlan* plan) {
-  auto kern = gemm_pair_kernel<A_MN, B_MN, EPI, PK>;
-  const int smem = SmemPair<EPI>::BYTES;
-  constexpr int threads = PairCfg<EPI>::THREADS;
+  auto kern = gemm_pair_kernel<A_MN, B_MN, EPI, PK, DR>;
+  const int smem = SmemPair<EPI, DR>::BYTES;
+  constexpr int threads = PairCfg<EPI, DR>::THREADS;
   static int max_clusters = 0;  // per template instance
   p.num_n = (p.N + 255) / 256;
   p.num_tiles = ((p.M + 255) / 256) * p.num_n * p.splits;
@@ -1042,6 +1116,8 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
       if (!make_map(&ta, g.A, g.Kred, g.M, BK, BM)) return 3;
       if (drain) {
         if (!make_map(&tb, g.B, g.Kred, g.N, BK, 128)) return 3;
+        if (gemm_mode() == 0)
+          return launch_pairs<false, false, GEMM_FWD, false, true>(ta, tb, p, stream);
         return launch_tiles<128, false, false, GEMM_FWD, true>(ta, tb, p, stream);
       }
       if (!make_map(&tb, g.B, g.Kred, g.N, BK, g2.pair ? 128 : 256)) return 3;
