@@ -75,7 +75,7 @@ def kernel_fingerprint(files=GEMM_SOURCES):
 # of operand and optimiser-state bytes), from one ncu capture, keyed by the
 # GEMM-source fingerprint it was taken on (see profiles/).  A stale entry
 # reports null.
-DW_TRAFFIC_BYTES = {"d3fc5601e4d7": 273736448 + 60078080 + 33047808}
+DW_TRAFFIC_BYTES = {"32d6d013a957": 272136448 + 59985920 + 33047552}
 
 
 def _dist():
@@ -205,13 +205,21 @@ class MLPStep:
             self.af_ws = [torch.empty(nb, dtype=torch.uint8, device=dev) for _ in range(4)]
         self.sr = {name: dqt.sr_stream(seed=seed, tensor_id=i) for i, (name, _, _) in enumerate(PROJ)}
         self.step_no = 0
-        self.launches_per_step = 2 + 3 + 3 + 3 + 3 + (3 if fp8 else 0)
+        # weight-gradient workspace (token-sliced last wave), one per stream
+        nbw = max(dqt.dqt_bwd_dw_workspace_size(T, N, K) for _, K, N in PROJ)
+        self.dw_ws = [torch.empty(max(nbw, 16), dtype=torch.uint8, device=dev) if nbw else False
+                      for _ in range(4)]
+        # kernel launches per step: act_quant 2, weight images 3 (+3 E4M3),
+        # forward 3, dX 3, and per projection the dW GEMM, the streaming
+        # kernel of its sliced last wave (when the shape has one), and for
+        # Adafactor the five statistics kernels and the step
+        dw = [1 + (1 if dqt.dqt_bwd_dw_workspace_size(T, N, K) > 0 else 0) for _, K, N in PROJ]
+        self.launches_per_step = 2 + 3 + 3 + 3 + sum(dw) + (3 if fp8 else 0)
         self.dw_kind = "bwd_dw_adafactor" if optimizer == "adafactor" else "bwd_dw_update"
         self.kinds = (["act_quant_fp8", "codes_to_fp8", "codes_to_bf16", "fwd_fp8"] if fp8 else
                       ["act_quant", "codes_to_bf16", "fwd"]) + ["bwd_dx", self.dw_kind]
         if optimizer == "adafactor":
-            # gradient GEMM, four statistics kernels and the step per projection
-            self.launches_per_step += 3 * 5
+            self.launches_per_step += 3 * 6
         self.streams = [torch.cuda.Stream(device=dev) for _ in range(4)]
 
     def run(self, timers=None, serial=False):
@@ -295,17 +303,22 @@ class MLPStep:
                     self.v[name], af, self.sr[name], self.grid, packed=self.packed,
                     changed_out=ch, ws=ws))
             elif self.packed:
+                ws = self.dw_ws[s.index(stream)]
                 timed(self.dw_kind, stream, lambda: dqt.dqt_bitlinear_bwd_dw_update_packed(
                     self.d["dY_" + name], xdq, self.W[name], self.s_w[name], self.m[name],
-                    self.v[name], hp, self.sr[name], changed_out=ch))
+                    self.v[name], hp, self.sr[name], changed_out=ch, ws=ws))
             else:
+                ws = self.dw_ws[s.index(stream)]
                 timed(self.dw_kind, stream, lambda: dqt.dqt_bitlinear_bwd_dw_update(
                     self.d["dY_" + name], xdq, self.W[name], self.s_w[name], self.m[name],
-                    self.v[name], hp, self.sr[name], self.grid, changed_out=ch))
+                    self.v[name], hp, self.sr[name], self.grid, changed_out=ch, ws=ws))
 
         for st in s:
             after(st, main)
-        # forward: the three weight images convert while X is quantised
+        # forward: the three weight images convert while X is quantised (one
+        # pass writes both the forward's code image and the dequantised image
+        # the weight gradient reads: splitting it into two passes, the second
+        # beside the forward GEMMs, was measured slower)
         aq("X", s[0])
         codes("gate", s[1])
         codes("up", s[2])
