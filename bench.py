@@ -341,10 +341,12 @@ class MLPStep:
         for st in (s[0], s[1], s[3]):
             if st is not s[2]:
                 st.wait_event(dx_down)
-        dx("gate", s[0])
+        # each weight-gradient GEMM is enqueued ahead of its dX: the longer
+        # kernel then takes the SMs first and the dX kernels fill its last wave
         dw(0, "gate", s[1])
-        dx("up", s[2])
+        dx("gate", s[0])
         dw(1, "up", s[3])
+        dx("up", s[2])
         for st in s:
             after(main, st)
 
