@@ -75,7 +75,7 @@ def kernel_fingerprint(files=GEMM_SOURCES):
 # of operand and optimiser-state bytes), from one ncu capture, keyed by the
 # GEMM-source fingerprint it was taken on (see profiles/).  A stale entry
 # reports null.
-DW_TRAFFIC_BYTES = {"32d6d013a957": 272136448 + 59985920 + 33047552}
+DW_TRAFFIC_BYTES = {"c81c5624b6f0": 273583872 + 61053952 + 33047552}
 
 
 def _dist():
@@ -932,6 +932,142 @@ def run_decoder(args):
         "final_loss": float(loss_host), "clocks": clk.summary()}))
 
 
+LAYER_SHAPE = (256, 512, 512)  # T, K, N of the single-layer step
+
+
+def run_layer(args):
+    """One BitLinear layer's training step at T=256, K=512, N=512 (X ~N(0,1),
+    dY ~N(0,1e-2), ternary codes by AbsMean of N(0,0.02), AdamW lr 1e-3, Philox
+    seed 1234): act_quant, the weight's code image, forward, dX and the fused
+    dW + AdamW + SR update.  At this size every kernel is latency-bound, so the
+    K timed steps are captured as one CUDA graph (step i reads its update
+    constants from row i of a device block, uploaded in one copy at the start
+    of the timed region) and the time is the GPU's, not the Python launch
+    path's; the result is quoted in microseconds per step.  e2e: a second
+    graph whose every step also copies X and dY from pinned host memory and
+    reads the changed-code count back."""
+    from paper_2412_04787_gb300 import build as dqt_build
+    from paper_2412_04787_gb300 import dqt, inputs
+    dqt_build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    T, K, N = LAYER_SHAPE
+    KS = args.steps
+    grid = dqt.grid(args.bits)
+    host = [(inputs.normal((T, K), 1.0, seed=1 + 100 * r, dtype=torch.bfloat16).pin_memory(),
+             inputs.normal((T, N), 1e-2, seed=2 + 100 * r, dtype=torch.bfloat16).pin_memory())
+            for r in range(2)]
+    X = host[0][0].to(dev)
+    dY = host[0][1].to(dev)
+    W, s_w = dqt.dqt_absmean_init(inputs.normal((N, K), 0.02, seed=3).to(dev), grid)
+    m = torch.zeros((N, K), dtype=torch.float32, device=dev)
+    v = torch.zeros((N, K), dtype=torch.float32, device=dev)
+    s_x = torch.empty(T, dtype=torch.float32, device=dev)
+    q_img = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
+    xdq = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
+    W_img = torch.empty((N, K), dtype=torch.bfloat16, device=dev)
+    Y = torch.empty((T, N), dtype=torch.bfloat16, device=dev)
+    dX = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
+    changed = torch.zeros(1, dtype=torch.int64, device=dev)
+    nbw = dqt.dqt_bwd_dw_workspace_size(T, N, K)
+    ws = torch.empty(nbw, dtype=torch.uint8, device=dev) if nbw else None
+    row = (dqt.lib().dqt_update_consts_size() + 63) // 64 * 64
+    # the graph of KS steps is replayed R times (about a second of GPU time)
+    # in the timed region; every replay's constants have a host block of
+    # their own, so no block is rewritten while a copy from it may be pending
+    R = max(1, 40000 // KS)
+    uc_host = torch.zeros((R, KS, row), dtype=torch.uint8).pin_memory()
+    uc_host_e2e = torch.zeros((KS, row), dtype=torch.uint8).pin_memory()
+    uc_dev = torch.zeros((KS, row), dtype=torch.uint8, device=dev)
+    sr = dqt.sr_stream(seed=1234, tensor_id=0)
+    state = {"step": 0}
+    ch_host = torch.empty(KS, dtype=torch.int64).pin_memory()
+
+    def kernels(i):
+        dqt.dqt_act_quant(X, None, s_x, q_img, xdq, want=())
+        dqt.dqt_codes_to_bf16(W, W_img)
+        dqt.dqt_bitlinear_fwd(q_img, s_x, W_img, s_w, grid, Y=Y)
+        dqt.dqt_bitlinear_bwd_dx(dY, W_img, s_w, dX=dX)
+        dqt.dqt_bitlinear_bwd_dw_update_dev(dY, xdq, W, m, v, uc_dev[i], changed_out=changed,
+                                            ws=ws)
+
+    def fill(block):
+        for i in range(block.shape[0]):
+            state["step"] += 1
+            dqt.dqt_update_consts(dqt.adamw(lr=1e-3, step=state["step"]), sr, grid, s_w,
+                                  out=block[i])
+
+    # warm-up: eager steps, each with its own constants row
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    warm = torch.zeros((args.warmup, row), dtype=torch.uint8).pin_memory()
+    with torch.cuda.stream(side):
+        for i in range(args.warmup):
+            state["step"] += 1
+            dqt.dqt_update_consts(dqt.adamw(lr=1e-3, step=state["step"]), sr, grid, s_w,
+                                  out=warm[i])
+            uc_dev[i % KS].copy_(warm[i], non_blocking=True)
+            kernels(i % KS)
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        for i in range(KS):
+            kernels(i)
+    graph_e2e = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph_e2e):
+        for i in range(KS):
+            X.copy_(host[i % 2][0], non_blocking=True)
+            dY.copy_(host[i % 2][1], non_blocking=True)
+            kernels(i)
+            ch_host[i:i + 1].copy_(changed, non_blocking=True)
+    torch.cuda.synchronize()
+    dqt.dqt_check_device_status()
+
+    stream = torch.cuda.current_stream()
+    for r in range(R):
+        fill(uc_host[r])
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    with ClockSampler(dev.index) as clk:
+        t0.record(stream)
+        for r in range(R):
+            uc_dev.copy_(uc_host[r], non_blocking=True)
+            graph.replay()
+        t1.record(stream)
+        torch.cuda.synchronize()
+    dqt.dqt_check_device_status()
+    ms = t0.elapsed_time(t1) / (R * KS)
+    fill(uc_host_e2e)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    uc_dev.copy_(uc_host_e2e, non_blocking=True)
+    graph_e2e.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e_ms = e0.elapsed_time(e1) / KS
+    print(json.dumps({
+        "metric": "DQT BitLinear fwd+bwd+SR-update tokens/s", "value": round(T / (ms / 1e3), 1),
+        "unit": "tokens/s", "n_gpus": 1, "steps": R * KS, "warmup": args.warmup,
+        "ms_per_step": round(ms, 5), "us_per_step": round(ms * 1e3, 2),
+        "graph": {"steps_per_graph": KS, "replays": R},
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) activations, N(0,1e-2) gradients, AbsMean-ternary codes of N(0,0.02))",
+        "config": {"workload": "single BitLinear layer training step, 256 tokens, 512 -> 512, "
+                               "ternary codes, AdamW + SR (K steps in one CUDA graph)",
+                   "tokens": T, "in_features": K, "out_features": N,
+                   "l2": "latency-bound: the whole working set (~2 MB) stays in L2"},
+        "roofline": {"bound": "latency", "note": "3 x 0.134 GFLOP and 4.7 MB per step: "
+                     "launch and pipeline latency, not a throughput roofline, bounds this size"},
+        "gpu_launches": (5 + (1 if nbw else 0)) * KS * R,
+        "e2e": {"value": round(T / (e_ms / 1e3), 1), "unit": "tokens/s",
+                "h2d_bytes_per_step": int(X.numel() * 2 + dY.numel() * 2 + row),
+                "d2h_bytes_per_step": 8},
+        "changed_codes_last_step": int(ch_host[KS - 1]),
+        "clocks": clk.summary()}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -957,8 +1093,9 @@ def main():
     ap.add_argument("--packed", action="store_true", help="2-bit packed ternary code storage")
     ap.add_argument("--bits", type=float, default=1.58,
                     help="weight grid: 1.58 (ternary, the default) or an integer width 2..8")
-    ap.add_argument("--workload", default="mlp", choices=["mlp", "decoder"],
-                    help="mlp: the headline BitLinear MLP GEMM set; decoder: a 12-layer DQT decoder step")
+    ap.add_argument("--workload", default="mlp", choices=["mlp", "decoder", "layer"],
+                    help="mlp: the headline BitLinear MLP GEMM set; decoder: a DQT decoder step; "
+                         "layer: one 256 x 512 x 512 BitLinear step")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -968,6 +1105,8 @@ def main():
         dqt.dqt_set_gemm_tiles(args.tiles)
     if args.workload == "decoder" and args.impl == "dqt" and not args.kernel:
         run_decoder(args)
+    elif args.workload == "layer" and args.impl == "dqt" and not args.kernel:
+        run_layer(args)
     elif args.kernel:
         run_kernel(args)
     elif args.impl == "reference":

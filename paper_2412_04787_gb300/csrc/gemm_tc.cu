@@ -616,10 +616,13 @@ struct SmemPair {
 // the epilogue warps fold each chunk into running int32 sums held in their
 // registers (64 per lane), then write Y from them after the tile's last
 // chunk; the MMAs of the next chunk run meanwhile.
-template <bool A_MN, bool B_MN, int EPI, bool PK = false, bool DR = false>
+// UCD: the dW update constants come from device memory (p.uc_dev, copied to
+// shared memory once); otherwise the epilogue reads them straight from the
+// kernel's parameter space, where they take no registers.
+template <bool A_MN, bool B_MN, int EPI, bool PK = false, bool DR = false, bool UCD = false>
 __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
     gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA,
-                     const __grid_constant__ CUtensorMap tmB, const Params p) {
+                     const __grid_constant__ CUtensorMap tmB, const __grid_constant__ Params p) {
   using S = SmemPair<EPI, DR>;
   static_assert(!DR || EPI == GEMM_FWD, "drained chunks: exact integer forward only");
   constexpr int ST = S::STAGES;
@@ -669,7 +672,7 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
       mbar_init(&acc_empty[b], 2 * EW);
     }
     mbar_init(drain_bar, 1);
-    if (EPI == GEMM_DW) *uc_s = p.uc_dev ? *p.uc_dev : p.uc;
+    if (EPI == GEMM_DW && UCD) *uc_s = *p.uc_dev;
     fence_mbarrier_init();
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
@@ -786,7 +789,7 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
     const int row = quad * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     float* xp = reinterpret_cast<float*>(smem + S::XPOSE_OFF) + (warp - 2) * 32 * kStageLd;
-    const UpdateConsts& uc = *uc_s;
+    const UpdateConsts& uc = UCD ? *uc_s : p.uc;
     uint32_t n_changed = 0;
     int u = 0;
     bool ok = true;
@@ -951,7 +954,7 @@ int launch_tiles(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStr
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
-template <bool A_MN, bool B_MN, int EPI, bool PK = false, bool DR = false>
+template <bool A_MN, bool B_MN, int EPI, bool PK = false, bool DR = false, bool UCD = false>
 int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream,
                  void* tail_ws = nullptr, size_t tail_ws_bytes = 0, TailPlan* plan = nullptr);
 
@@ -1004,10 +1007,10 @@ int dw_splits(int M, int N, int Kred) {
 
 namespace {
 
-template <bool A_MN, bool B_MN, int EPI, bool PK, bool DR>
+template <bool A_MN, bool B_MN, int EPI, bool PK, bool DR, bool UCD>
 int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream,
                  void* tail_ws, size_t tail_ws_bytes, TailPlan* plan) {
-  auto kern = gemm_pair_kernel<A_MN, B_MN, EPI, PK, DR>;
+  auto kern = gemm_pair_kernel<A_MN, B_MN, EPI, PK, DR, UCD>;
   const int smem = SmemPair<EPI, DR>::BYTES;
   constexpr int threads = PairCfg<EPI, DR>::THREADS;
   static int max_clusters = 0;  // per template instance
@@ -1140,11 +1143,17 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
       if (p.splits == 1) {
         // the last wave's tiles as token slices, their update in a streaming pass
         TailPlan tp{0, 0, 0, 0, 0};
-        const int rc = p.packed && p.W
-                           ? launch_pairs<true, true, GEMM_DW, true>(ta, tb, p, stream, g.ws,
-                                                                      g.ws_bytes, &tp)
-                           : launch_pairs<true, true, GEMM_DW>(ta, tb, p, stream, g.ws, g.ws_bytes,
-                                                               &tp);
+        const bool pk = p.packed && p.W;
+        const bool ucd = p.uc_dev != nullptr;
+        const int rc =
+            pk ? (ucd ? launch_pairs<true, true, GEMM_DW, true, false, true>(ta, tb, p, stream,
+                                                                             g.ws, g.ws_bytes, &tp)
+                      : launch_pairs<true, true, GEMM_DW, true>(ta, tb, p, stream, g.ws,
+                                                                g.ws_bytes, &tp))
+               : (ucd ? launch_pairs<true, true, GEMM_DW, false, false, true>(
+                            ta, tb, p, stream, g.ws, g.ws_bytes, &tp)
+                      : launch_pairs<true, true, GEMM_DW>(ta, tb, p, stream, g.ws, g.ws_bytes,
+                                                          &tp));
         if (rc || tp.splits == 0) return rc;
         return launch_tail_update(static_cast<const float*>(g.ws), tp.splits, tp.tail, tp.full,
                                   (g.N + 255) / 256, g.M, g.N, g.W, g.packed, g.m, g.v, g.uc,
