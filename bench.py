@@ -75,7 +75,7 @@ def kernel_fingerprint(files=GEMM_SOURCES):
 # of operand and optimiser-state bytes), from one ncu capture, keyed by the
 # GEMM-source fingerprint it was taken on (see profiles/).  A stale entry
 # reports null.
-DW_TRAFFIC_BYTES = {"c81c5624b6f0": 273583872 + 61053952 + 33047552}
+DW_TRAFFIC_BYTES = {"2ec79ec9344c": 274800384 + 61107200 + 33048064}
 
 
 def _dist():
@@ -192,17 +192,11 @@ class MLPStep:
         # per activation: (scale, forward operand, dequantised bf16 image); the
         # forward operand is the bf16 code image, or the E4M3 bytes with fp8
         self.aq = {}
-        # drained exact forwards (8-bit codes): per activation, the row L1
-        # bounds from which the forward plans its chunks
-        self.blk = {}
         for src, K in (("X", HID), ("H", INTER)):
             self.aq[src] = (torch.empty(T, dtype=torch.float32, device=dev),
                             torch.empty((T, K), dtype=torch.uint8 if fp8 else torch.bfloat16,
                                         device=dev),
                             torch.empty((T, K), dtype=torch.bfloat16, device=dev))
-            if not fp8 and dqt.fwd_drains(K, self.grid):
-                self.blk[src] = torch.empty(((T + 127) // 128, (K + 1023) // 1024),
-                                            dtype=torch.int32, device=dev)
         self.changed = torch.zeros(3, dtype=torch.int64, device=dev)
         self.af_ws = None
         if optimizer == "adafactor":
@@ -271,10 +265,6 @@ class MLPStep:
             if self.fp8:
                 timed("act_quant_fp8", stream,
                       lambda: dqt.dqt_act_quant_fp8(self.d[src], q_img, s_x, xdq))
-            elif src in self.blk:
-                timed("act_quant", stream,
-                      lambda: dqt.dqt_act_quant_l1(self.d[src], None, s_x, q_img, xdq,
-                                                   self.blk[src], want=()))
             else:
                 timed("act_quant", stream,
                       lambda: dqt.dqt_act_quant(self.d[src], None, s_x, q_img, xdq, want=()))
@@ -290,15 +280,10 @@ class MLPStep:
                   else dqt.dqt_codes_to_bf16(self.W[name], self.W_img[name]))
 
         def fwd(name, stream):
-            src = "H" if name == "down" else "X"
-            s_x, q_img, _ = self.aq[src]
+            s_x, q_img, _ = self.aq["H" if name == "down" else "X"]
             if self.fp8:
                 timed("fwd_fp8", stream, lambda: dqt.dqt_bitlinear_fwd_fp8(
                     q_img, s_x, self.W8[name], self.s_w[name], self.grid, Y=self.Y[name]))
-            elif src in self.blk:
-                timed("fwd", stream, lambda: dqt.dqt_bitlinear_fwd_l1(
-                    q_img, s_x, self.W_img[name], self.s_w[name], self.grid, self.blk[src],
-                    Y=self.Y[name]))
             else:
                 timed("fwd", stream, lambda: dqt.dqt_bitlinear_fwd(
                     q_img, s_x, self.W_img[name], self.s_w[name], self.grid, Y=self.Y[name]))
@@ -723,11 +708,7 @@ def run_kernel(args):
         dX = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
         hp = dqt.adamw()
         sr = dqt.sr_stream()
-        if k == "fwd" and dqt.fwd_drains(K, g):
-            # drained exact chunks: planned from the row L1 bounds, as in the step
-            _, _, _, _, blk = dqt.dqt_act_quant_l1(X)
-            fn = lambda: dqt.dqt_bitlinear_fwd_l1(q_img, s_x, W_img, s_w, g, blk, Y=Y)  # noqa: E731
-        elif k in ("fwd", "fwd_fixed"):  # fwd_fixed: worst-case chunks even where a plan helps
+        if k == "fwd":
             fn = lambda: dqt.dqt_bitlinear_fwd(q_img, s_x, W_img, s_w, g, Y=Y)  # noqa: E731
         elif k == "bwd_dx":
             fn = lambda: dqt.dqt_bitlinear_bwd_dx(dY, W_img, s_w, dX=dX)  # noqa: E731
@@ -778,7 +759,7 @@ def run_kernel(args):
             fn = lambda: dqt.dqt_codes_to_bf16(W, W_img)  # noqa: E731
         else:
             raise SystemExit("unknown kernel %s" % k)
-        if k in ("fwd", "fwd_fixed", "bwd_dx", "bwd_dw_update", "bwd_dw", "bwd_dw_unfused", "fwd_fp8",
+        if k in ("fwd", "bwd_dx", "bwd_dw_update", "bwd_dw", "bwd_dw_unfused", "fwd_fp8",
                  "bwd_dw_update_packed", "bwd_dw_adafactor"):
             work, unit = 2.0 * T * K * N, "TFLOP/s"
         elif k == "adafactor_stats":

@@ -174,32 +174,6 @@ int dqt_bitlinear_fwd(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* 
                       float s_w, dqt_grid_t grid, int64_t T, int64_t K, int64_t N,
                       dqt_bf16* Y, int32_t* acc_out, void* stream);
 
-/* Row L1 bounds of the activation codes (an implementation device for the
- * exact forward of dqt_bitlinear_fwd; the paper has no counterpart).  As
- * dqt_act_quant, and in addition
- *   blk_l1[b, j] = max over the token rows t of block b (rows 128 b .. 128 b + 127)
- *                  of sum over k in [1024 j, 1024 j + 1024) of |Xq[t,k]|
- *   blk_l1  int32 [ceil(T/128), ceil(K/1024)] out, row-major, device, required
- *           (dqt_act_l1_count(T, K) entries; overwritten, no initialisation needed).
- * The codes and images are those of dqt_act_quant, bit for bit. */
-int64_t dqt_act_l1_count(int64_t T, int64_t K);
-int dqt_act_quant_l1(const dqt_bf16* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
-                     dqt_bf16* Xq_img, dqt_bf16* Xdq, int32_t* blk_l1, void* stream);
-
-/* dqt_bitlinear_fwd given the row bounds blk_l1 that dqt_act_quant_l1 wrote
- * for this Xq_img.  Every partial sum over a run of whole 1024-column blocks
- * is at most (the run's summed bounds) * max|c| in magnitude, so where the
- * grid forces drained chunks (8-bit codes, K > 1024) the 2-SM kernel lets each
- * tile's chunk span as many blocks as keep that product <= 2^24 instead of the
- * worst case 2^24 / (128 max|c|) elements: fewer drains, the same exact int32
- * sums and Y, bit for bit.  Bounds smaller than the true ones void the
- * exactness guarantee.  Without drained chunks, with 1-SM tiles
- * (dqt_set_gemm_tiles(1)) or for K > 32768 the bounds are not used and the
- * call is dqt_bitlinear_fwd. */
-int dqt_bitlinear_fwd_l1(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img,
-                         float s_w, dqt_grid_t grid, int64_t T, int64_t K, int64_t N,
-                         dqt_bf16* Y, int32_t* acc_out, const int32_t* blk_l1, void* stream);
-
 /* Backward w.r.t. the input, no straight-through estimator on the weight
  * (the gradient is taken w.r.t. W_tilde itself, Sec. 3.2):
  *   dX[t,k] = bf16( (sum_n dY[t,n] c[n,k]) * (1 / s_w) )   fp32 accumulation

@@ -50,12 +50,6 @@ class _BitLinearFn(torch.autograd.Function):
             q8, s_x, xdq = dqt.dqt_act_quant_fp8(x2)
             y = dqt.dqt_bitlinear_fwd_fp8(q8, s_x, layer.weight_fp8(), float(layer.s_w),
                                           layer.grid_tuple)
-        elif dqt.fwd_drains(K, layer.grid_tuple):
-            # drained exact chunks (8-bit codes): the row L1 bounds let the
-            # forward take longer ones
-            _, s_x, q_img, xdq, blk = dqt.dqt_act_quant_l1(x2)
-            y = dqt.dqt_bitlinear_fwd_l1(q_img, s_x, layer.weight_bf16(), float(layer.s_w),
-                                         layer.grid_tuple, blk)
         else:
             _, s_x, q_img, xdq = dqt.dqt_act_quant(x2, want=("Xq_img", "Xdq"))
             y = dqt.dqt_bitlinear_fwd(q_img, s_x, layer.weight_bf16(), float(layer.s_w),

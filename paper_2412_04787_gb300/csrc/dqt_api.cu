@@ -172,35 +172,15 @@ int dqt_act_quant(const dqt_bf16* X, int64_t T, int64_t K, int8_t* Xq, float* s_
                                                                                  : DQT_OK;
 }
 
-int64_t dqt_act_l1_count(int64_t T, int64_t K) {
-  if (T <= 0 || K <= 0 || T > kMaxDim || K > kMaxDim) return 0;
-  return dqt::l1_bounds_count(T, K);
-}
-
-int dqt_act_quant_l1(const dqt_bf16* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
-                     dqt_bf16* Xq_img, dqt_bf16* Xdq, int32_t* blk_l1, void* stream) {
-  if (!X || !s_x || !blk_l1 || (!Xq && !Xq_img && !Xdq) || T <= 0 || K <= 0) return DQT_ERR_ARG;
-  if (T > kMaxDim || K > kMaxDim) return DQT_ERR_RANGE;
-  if (K % 8 || !aligned16(X) || (Xq && (reinterpret_cast<uintptr_t>(Xq) & 7u)) ||
-      (Xq_img && !aligned16(Xq_img)) || (Xdq && !aligned16(Xdq)) ||
-      (reinterpret_cast<uintptr_t>(blk_l1) & 3u))
-    return DQT_ERR_ALIGN;
-  return dqt::launch_act_quant(X, T, K, Xq, s_x, Xq_img, Xdq, as_stream(stream), blk_l1)
-             ? DQT_ERR_CUDA
-             : DQT_OK;
-}
-
 int dqt_codes_to_bf16(const int8_t* W, int64_t numel, dqt_bf16* W_img, void* stream) {
   if (!W || !W_img || numel <= 0) return DQT_ERR_ARG;
   if (!aligned16(W) || !aligned16(W_img)) return DQT_ERR_ALIGN;
   return dqt::launch_codes_to_bf16(W, numel, W_img, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
-namespace {
-
-int fwd_impl(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img, float s_w,
-             dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y, int32_t* acc_out,
-             const int32_t* blk_l1, void* stream) {
+int dqt_bitlinear_fwd(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img, float s_w,
+                      dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
+                      int32_t* acc_out, void* stream) {
   if (!Xq_img || !s_x || !W_img || !Y || T <= 0 || K <= 0 || N <= 0 || !grid_ok(grid) ||
       !(s_w > 0.0f) || !isfinite(s_w))
     return DQT_ERR_ARG;
@@ -228,25 +208,7 @@ int fwd_impl(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img, fl
   g.scale = s_w;
   g.out_bf16 = Y;
   g.acc_out = acc_out;
-  g.blk_l1 = blk_l1;
-  g.cmax = static_cast<int>(cm);
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
-}
-
-}  // namespace
-
-int dqt_bitlinear_fwd(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img, float s_w,
-                      dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
-                      int32_t* acc_out, void* stream) {
-  return fwd_impl(Xq_img, s_x, W_img, s_w, grid, T, K, N, Y, acc_out, nullptr, stream);
-}
-
-int dqt_bitlinear_fwd_l1(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img,
-                         float s_w, dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
-                         int32_t* acc_out, const int32_t* blk_l1, void* stream) {
-  if (!blk_l1) return DQT_ERR_ARG;
-  if (reinterpret_cast<uintptr_t>(blk_l1) & 3u) return DQT_ERR_ALIGN;
-  return fwd_impl(Xq_img, s_x, W_img, s_w, grid, T, K, N, Y, acc_out, blk_l1, stream);
 }
 
 int dqt_act_quant_fp8(const dqt_bf16* X, int64_t T, int64_t K, uint8_t* Xq8, float* s_x8,

@@ -31,11 +31,6 @@ struct GemmLaunch {
   const void* A;
   const void* B;
   int chunk_k;  // FWD: reduction elements per exact fp32 chunk (multiple of 64)
-  // FWD with drained chunks, optional: the activations' row L1 bounds
-  // (launch_act_quant's blk_l1) and max|c| of the weight grid, from which the
-  // 2-SM kernel plans longer exact chunks per tile
-  const int32_t* blk_l1;
-  int cmax;
   bool pair;    // use the 2-SM (cta_group::2) kernel (not with drained chunks)
   // Epilogue operands.
   const float* s_x;  // FWD, FWD8
@@ -91,12 +86,8 @@ int launch_slab_sum(const float* slabs, int splits, long long slab, float* out,
 
 int launch_gemm(const GemmLaunch& g, cudaStream_t stream);
 
-// blk_l1 (optional, l1_bounds_count(T, K) int32): per block of 128 rows and
-// 1024 columns, the largest row sum of |q| over the block's columns.
 int launch_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
-                     uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream,
-                     int32_t* blk_l1 = nullptr);
-int64_t l1_bounds_count(int64_t T, int64_t K);
+                     uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream);
 int launch_codes_to_bf16(const int8_t* W, int64_t numel, uint16_t* W_img, cudaStream_t stream);
 // FP8 environment: E4M3 activations with per-token scale 448 / max(amax, 1e-5)
 // (and optionally the dequantised bf16 image), and E4M3 images of weight codes.

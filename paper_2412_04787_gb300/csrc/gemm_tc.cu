@@ -81,12 +81,6 @@ struct Params {
   // sums them in slice order and applies the update.
   int full_units, full_tiles, tail_tiles, tail_splits, tail_kbps;
   float* part;
-  // exact forward with drained chunks (2-SM): the activations' row L1 bounds
-  // (max over each 128-row block of a row's sum of |q| over each 1024-column
-  // block, ncb blocks per row); a tile's chunks then span as many whole
-  // column blocks as keep sum(bound) <= l1_limit = 2^24 / max|c|
-  const int32_t* blk_l1;
-  int ncb, l1_limit;
 };
 
 struct Unit {
@@ -116,97 +110,6 @@ __device__ __forceinline__ Unit decode_unit(const Params& p, int t) {
 }
 
 constexpr int kStageLd = 33;  // padded row pitch (floats) of the epilogue transpose buffer
-
-// Chunk plan of an exact-forward pair tile (rows 256 tm .. 256 tm + 255): bit
-// cb set = a chunk starts at column block cb (k-block 16 cb).  Greedy over the
-// column blocks: a block joins the running chunk while the chunk's summed
-// bound stays within l1_limit; every partial sum of a chunk is then at most
-// l1_limit * max|c| <= 2^24 in magnitude, exact in fp32.  One 1024-column block
-// always fits (1024 * 128 * 128 = 2^24).  The bounds of the first eight column
-// blocks of the tile's two row blocks are loaded ahead (plan_load) and used
-// later (plan_mask), so the load latency overlaps other work.
-struct PlanBounds {
-  int32_t a[8], b[8];
-};
-
-__device__ __forceinline__ void plan_load(const Params& p, int tm, PlanBounds& v) {
-  const int nrb = (p.M + 127) >> 7;
-  const int32_t* r0 = p.blk_l1 + static_cast<size_t>(2 * tm) * p.ncb;
-  const bool has1 = 2 * tm + 1 < nrb;
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    v.a[j] = j < p.ncb ? __ldg(r0 + j) : 0;
-    v.b[j] = (j < p.ncb && has1) ? __ldg(r0 + p.ncb + j) : 0;
-  }
-}
-
-__device__ __forceinline__ uint64_t plan_mask(const Params& p, int tm, const PlanBounds& v) {
-  const int nrb = (p.M + 127) >> 7;
-  const int32_t* r0 = p.blk_l1 + static_cast<size_t>(2 * tm) * p.ncb;
-  const bool has1 = 2 * tm + 1 < nrb;
-  uint64_t mask = 1ull;
-  long long run = 0;
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    if (j < p.ncb) {
-      const int32_t x = max(v.a[j], v.b[j]);
-      if (j > 0 && run + x > p.l1_limit) {
-        mask |= 1ull << j;
-        run = 0;
-      }
-      run += x;
-    }
-  }
-  for (int cb = 8; cb < p.ncb; ++cb) {  // K > 8192: the rest, loaded here (ncb <= 32)
-    const int32_t x = max(__ldg(r0 + cb), has1 ? __ldg(r0 + p.ncb + cb) : 0);
-    if (run + x > p.l1_limit) {
-      mask |= 1ull << cb;
-      run = 0;
-    }
-    run += x;
-  }
-  return mask;
-}
-
-// The chunk count of the same plan formed by a whole warp, lane j holding
-// column block j's two bounds (loaded by plan_load_lane; plans are used for
-// ncb <= 32 only): two registers per lane while the loads are in flight, then
-// a shuffle per column block.
-__device__ __forceinline__ void plan_load_lane(const Params& p, int tm, int lane, int32_t& a,
-                                               int32_t& b) {
-  const int nrb = (p.M + 127) >> 7;
-  const int32_t* r0 = p.blk_l1 + static_cast<size_t>(2 * tm) * p.ncb;
-  a = lane < p.ncb ? __ldg(r0 + lane) : 0;
-  b = (lane < p.ncb && 2 * tm + 1 < nrb) ? __ldg(r0 + p.ncb + lane) : 0;
-}
-
-__device__ __forceinline__ int plan_chunks_warp(const Params& p, int32_t a, int32_t b) {
-  const int32_t x = max(a, b);
-  int n = 1;
-  long long run = 0;
-  for (int cb = 0; cb < p.ncb; ++cb) {
-    const int32_t xc = __shfl_sync(0xffffffffu, x, cb);
-    if (cb > 0 && run + xc > p.l1_limit) {
-      ++n;
-      run = 0;
-    }
-    run += xc;
-  }
-  return n;
-}
-
-// Length in k-blocks of the drained chunk that starts at k-block offset kr of
-// a tile with `rem` k-blocks left: up to the plan's next chunk start, or fixed
-// chunks of chunk_kb k-blocks without a plan.
-__device__ __forceinline__ int chunk_len(const Params& p, uint64_t plan, int kr, int rem) {
-  int len = p.chunk_kb;
-  if (p.blk_l1) {
-    const int cb0 = kr >> 4;
-    const uint64_t rest = cb0 + 1 < 64 ? plan >> (cb0 + 1) : 0ull;
-    len = rest ? 16 * __ffsll(static_cast<long long>(rest)) : rem;
-  }
-  return len < rem ? len : rem;
-}
 
 template <int BN, int EPI>
 struct Smem {
@@ -851,21 +754,15 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
       constexpr uint64_t kAStage = S::A_BYTES >> 4, kBStage = S::B_BYTES >> 4;
       constexpr uint64_t kAStep = A_MN ? (2048 >> 4) : (32 >> 4);  // per 16-element k step
       constexpr uint64_t kBStep = B_MN ? (2048 >> 4) : (32 >> 4);
-      // DR with row bounds: the next tile's bounds are loaded while the current
-      // tile's MMAs run, and its plan is formed when it starts
-      PlanBounds nb;
-      if (DR && p.blk_l1 && cid < p.num_tiles) plan_load(p, cid / p.num_n, nb);
       for (int t = cid; t < p.num_tiles && ok; t += ncl) {
         const Unit un = decode_unit(p, t);
         const int kb0 = un.kb0, kb1 = un.kb1;
-        const uint64_t plan = (DR && p.blk_l1) ? plan_mask(p, un.tile / p.num_n, nb) : 0ull;
         int left = 0;  // DR: k-blocks left in the current chunk
         for (int kb = kb0; kb < kb1; ++kb) {
-          // two accumulators alternating per unit; DR: a unit is one chunk
-          // (fixed chunk_kb k-blocks, or the tile's plan), whose exact sum the
-          // epilogue folds into int32
+          // two accumulators alternating per unit; DR: a unit is one chunk of
+          // chunk_kb k-blocks, whose exact sum the epilogue folds into int32
           const bool cstart = DR ? left == 0 : kb == kb0;
-          if (DR && cstart) left = chunk_len(p, plan, kb - kb0, kb1 - kb);
+          if (DR && cstart) left = min(p.chunk_kb, kb1 - kb);
           const int b = u & 1;
           if (cstart && u >= 2) {
             if (!mbar_wait_cl(&acc_empty[b], ((u >> 1) - 1) & 1u, p.wait_ns)) {
@@ -893,8 +790,6 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
             s = 0;
             ph ^= 1u;
           }
-          if (DR && p.blk_l1 && kb == kb0 && t + ncl < p.num_tiles)
-            plan_load(p, decode_unit(p, t + ncl).tile / p.num_n, nb);
           if (DR) --left;
           if (kb == kb1 - 1 || (DR && left == 0)) {
             umma_commit_pair_mc(&acc_full[b], 0x3);
@@ -928,14 +823,9 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
       if ((EPI == GEMM_FWD || F8) && row_ok) a_t = __fdiv_rn(1.0f, __fmul_rn(p.s_x[gm], p.scale));
       if (DR) {
         static_assert(!DR || HALF == 64, "two 32-column chunks of running sums per lane");
-        int nchunks = (p.num_kb + p.chunk_kb - 1) / p.chunk_kb;
-        if (p.blk_l1) {
-          int32_t la, lb;
-          plan_load_lane(p, tile / p.num_n, lane, la, lb);
-          nchunks = plan_chunks_warp(p, la, lb);
-        }
+        const int nchunks = (p.num_kb + p.chunk_kb - 1) / p.chunk_kb;
         int32_t run0[32], run1[32];
-        for (int c = 0; c == 0 || c < nchunks; ++c, ++u) {  // nchunks >= 1, used late
+        for (int c = 0; c < nchunks; ++c, ++u) {
           const int b = u & 1;
           ok = __all_sync(0xffffffffu, mbar_wait_cl(&acc_full[b], (u >> 1) & 1u, p.wait_ns));
           if (!ok) break;
@@ -1248,15 +1138,8 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
       if (!make_map(&ta, g.A, g.Kred, g.M, BK, BM)) return 3;
       if (drain) {
         if (!make_map(&tb, g.B, g.Kred, g.N, BK, 128)) return 3;
-        if (gemm_mode() == 0) {
-          const int ncb = (g.Kred + 1023) / 1024;
-          if (g.blk_l1 && ncb <= 32 && g.cmax > 0 && g.cmax <= 128) {
-            p.blk_l1 = g.blk_l1;
-            p.ncb = ncb;
-            p.l1_limit = (1 << 24) / g.cmax;
-          }
+        if (gemm_mode() == 0)
           return launch_pairs<false, false, GEMM_FWD, false, true>(ta, tb, p, stream);
-        }
         return launch_tiles<128, false, false, GEMM_FWD, true>(ta, tb, p, stream);
       }
       if (!make_map(&tb, g.B, g.Kred, g.N, BK, g2.pair ? 128 : 256)) return 3;

@@ -63,30 +63,6 @@ __device__ __forceinline__ uint16_t dq_entry(int j, float s) {
 template <bool F8>
 __device__ __forceinline__ int dq_index(int32_t q) { return F8 ? q : q + 128; }
 
-// Row L1 bounds for the exact 8-bit forward: blk_l1[(row / 128) * ncb + cb]
-// becomes the largest sum of |q| over the 1024 columns [1024 cb, 1024 cb +
-// 1024) of any row in the 128-row block (the array is zeroed before the
-// kernel; an 8-element vector never straddles a 1024-column block).
-constexpr int kL1Rows = 128;
-constexpr int kL1Cols = 1024;
-
-__device__ __forceinline__ int32_t l1_8(const int32_t (&q)[8]) {
-  int32_t a = 0;
-#pragma unroll
-  for (int j = 0; j < 8; ++j) a += abs(q[j]);
-  return a;
-}
-
-__device__ __forceinline__ void l1_flush(int32_t* blk_l1, int row, int ncb, int cb, int32_t v) {
-  atomicMax(blk_l1 + static_cast<size_t>(row / kL1Rows) * ncb + cb, v);
-}
-
-__device__ __forceinline__ int32_t warp_sum(int32_t v) {
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-  return v;
-}
-
 // One warp per token row; 16-byte (8 x bf16) vector accesses.  Pass 1 finds
 // amax; pass 2 re-reads the row (an L1/L2 hit) and writes the outputs.
 constexpr int kAqWarps = 8;
@@ -95,7 +71,7 @@ template <bool F8>
 __global__ void __launch_bounds__(kAqWarps * 32)
     act_quant_kernel(const uint16_t* __restrict__ X, int T, int K, int8_t* __restrict__ Xq,
                      float* __restrict__ s_x, uint16_t* __restrict__ Xq_img,
-                     uint16_t* __restrict__ Xdq, int32_t* __restrict__ blk_l1, int ncb) {
+                     uint16_t* __restrict__ Xdq) {
   const int row = blockIdx.x * kAqWarps + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= T) return;
@@ -119,22 +95,11 @@ __global__ void __launch_bounds__(kAqWarps * 32)
   if (lane == 0) s_x[row] = s;
 
   const size_t rbase = static_cast<size_t>(row) * K;
-  // lane + 32 it lies in column block it / 4: every fourth iteration ends one
-  const int niter = (nv + 31) >> 5;
-  int32_t l1 = 0;
 #pragma unroll 4
-  for (int it = 0; it < niter; ++it) {
-    const int i = lane + 32 * it;
-    if (!F8 && blk_l1 && ((it & 3) == 0) && it > 0) {
-      l1 = warp_sum(l1);
-      if (lane == 0) l1_flush(blk_l1, row, ncb, (it >> 2) - 1, l1);
-      l1 = 0;
-    }
-    if (i >= nv) continue;
+  for (int i = lane; i < nv; i += 32) {
     const uint4 u = __ldg(xr + i);
     int32_t q[8];
     quant8<F8>(u, s, q);
-    if (!F8 && blk_l1) l1 += l1_8(q);
     const size_t e = rbase + static_cast<size_t>(i) * 8;
     if (Xq) {
       uint2 pk;
@@ -162,10 +127,6 @@ __global__ void __launch_bounds__(kAqWarps * 32)
       *reinterpret_cast<uint4*>(Xdq + e) = pk;
     }
   }
-  if (!F8 && blk_l1 && niter > 0) {
-    l1 = warp_sum(l1);
-    if (lane == 0) l1_flush(blk_l1, row, ncb, (niter - 1) >> 2, l1);
-  }
 }
 
 // Single-pass variant: WPR warps share a row and each lane keeps its (at
@@ -179,14 +140,9 @@ template <int NV, bool F8>
 __global__ void __launch_bounds__(256)
     act_quant_rows_kernel(const uint16_t* __restrict__ X, int T, int K, int wpr,
                           int8_t* __restrict__ Xq, float* __restrict__ s_x,
-                          uint16_t* __restrict__ Xq_img, uint16_t* __restrict__ Xdq,
-                          int32_t* __restrict__ blk_l1, int ncb) {
+                          uint16_t* __restrict__ Xq_img, uint16_t* __restrict__ Xdq) {
   __shared__ uint16_t table[8][256];
   __shared__ float part[8];
-  __shared__ int32_t l1s[8][16];  // row L1 per 1024-column block (K <= 16384 here)
-  const bool want_l1 = !F8 && blk_l1 != nullptr;
-  if (want_l1)
-    for (int j = threadIdx.x; j < 8 * 16; j += blockDim.x) (&l1s[0][0])[j] = 0;
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int rib = warp / wpr;      // row within the block
@@ -226,14 +182,14 @@ __global__ void __launch_bounds__(256)
     for (int j = tid; j < 256; j += nth) table[rib][j] = dq_entry<F8>(j, s);
   }
   __syncthreads();
+  if (!live) return;
   const size_t rbase = static_cast<size_t>(row) * K;
 #pragma unroll
   for (int i = 0; i < NV; ++i) {
     const int vi = tid + nth * i;
-    if (!live || vi >= nv) break;
+    if (vi >= nv) break;
     int32_t q[8];
     quant8<F8>(u[i], s, q);
-    if (want_l1) atomicAdd(&l1s[rib][vi / (kL1Cols / 8)], l1_8(q));
     const size_t e = rbase + static_cast<size_t>(vi) * 8;
     if (Xq) {
       uint2 pk;
@@ -258,10 +214,6 @@ __global__ void __launch_bounds__(256)
                         h[6] | (h[7] << 16)));
     }
   }
-  if (want_l1) {
-    __syncthreads();
-    if (live && tid < ncb) l1_flush(blk_l1, row, ncb, tid, l1s[rib][tid]);
-  }
 }
 
 // Persistent variant for rows of at most 2048 elements (8 vectors per lane):
@@ -273,15 +225,13 @@ __device__ __forceinline__ void aq_row_store(const uint4 (&u)[8], int nv, int la
                                              size_t rbase, const uint16_t* table,
                                              int8_t* __restrict__ Xq,
                                              uint16_t* __restrict__ Xq_img,
-                                             uint16_t* __restrict__ Xdq, bool want_l1,
-                                             int32_t (&l1)[2]) {
+                                             uint16_t* __restrict__ Xdq) {
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     const int vi = lane + 32 * i;
     if (vi >= nv) break;
     int32_t q[8];
     quant8<F8>(u[i], s, q);
-    if (want_l1) l1[i >> 2] += l1_8(q);  // vector lane + 32 i is in column block i / 4
     const size_t e = rbase + static_cast<size_t>(vi) * 8;
     if (Xq) {
       uint2 pk;
@@ -322,9 +272,7 @@ template <bool F8>
 __global__ void __launch_bounds__(256)
     act_quant_persist_kernel(const uint16_t* __restrict__ X, int T, int K,
                              int8_t* __restrict__ Xq, float* __restrict__ s_x,
-                             uint16_t* __restrict__ Xq_img, uint16_t* __restrict__ Xdq,
-                             int32_t* __restrict__ blk_l1, int ncb) {
-  const bool want_l1 = !F8 && blk_l1 != nullptr;
+                             uint16_t* __restrict__ Xq_img, uint16_t* __restrict__ Xdq) {
   __shared__ uint16_t table[8][256];
   const int wid = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -355,17 +303,7 @@ __global__ void __launch_bounds__(256)
       for (int j = lane; j < 256; j += 32) table[wid][j] = dq_entry<F8>(j, s);
       __syncwarp();
     }
-    int32_t l1[2] = {0, 0};
-    aq_row_store<F8>(ua, nv, lane, s, static_cast<size_t>(row) * K, table[wid], Xq, Xq_img, Xdq,
-                     want_l1, l1);
-    if (want_l1) {
-      l1[0] = warp_sum(l1[0]);
-      l1[1] = warp_sum(l1[1]);
-      if (lane == 0) {
-        l1_flush(blk_l1, row, ncb, 0, l1[0]);
-        if (ncb > 1) l1_flush(blk_l1, row, ncb, 1, l1[1]);
-      }
-    }
+    aq_row_store<F8>(ua, nv, lane, s, static_cast<size_t>(row) * K, table[wid], Xq, Xq_img, Xdq);
 #pragma unroll
     for (int i = 0; i < 8; ++i) ua[i] = ub[i];
   }
@@ -511,12 +449,8 @@ namespace {
 
 template <bool F8>
 int launch_aq(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x, uint16_t* Xq_img,
-              uint16_t* Xdq, cudaStream_t stream, int32_t* blk_l1 = nullptr) {
+              uint16_t* Xdq, cudaStream_t stream) {
   const int t = static_cast<int>(T), k = static_cast<int>(K);
-  const int ncb = static_cast<int>((K + kL1Cols - 1) / kL1Cols);
-  if (blk_l1 &&
-      cudaMemsetAsync(blk_l1, 0, l1_bounds_count(T, K) * sizeof(int32_t), stream) != cudaSuccess)
-    return 3;
   const int64_t nv = K / 8;  // 16-byte vectors per row
   // warps per row: keep at most 4 vectors (32 values) per lane; up to 8 warps
   const int wpr = static_cast<int>((nv + 127) / 128);
@@ -526,26 +460,21 @@ int launch_aq(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x, u
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t want = (T + 7) / 8;
     const int blocks = static_cast<int>(want < 2 * sms ? want : 2 * sms);
-    act_quant_persist_kernel<F8><<<blocks, 256, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq,
-                                                             blk_l1, ncb);
+    act_quant_persist_kernel<F8><<<blocks, 256, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq);
   } else if (wpr <= 8) {
     const int rpb = 8 / wpr;
     const int threads = 32 * wpr * rpb;
     const int blocks = static_cast<int>((T + rpb - 1) / rpb);
     const int per_lane = static_cast<int>((nv + 32 * wpr - 1) / (32 * wpr));
     if (per_lane <= 2)
-      act_quant_rows_kernel<2, F8><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq,
-                                                                    blk_l1, ncb);
+      act_quant_rows_kernel<2, F8><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
     else if (per_lane <= 4)
-      act_quant_rows_kernel<4, F8><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq,
-                                                                    blk_l1, ncb);
+      act_quant_rows_kernel<4, F8><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
     else
-      act_quant_rows_kernel<8, F8><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq,
-                                                                    blk_l1, ncb);
+      act_quant_rows_kernel<8, F8><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
   } else {
     const int blocks = static_cast<int>((T + kAqWarps - 1) / kAqWarps);
-    act_quant_kernel<F8><<<blocks, kAqWarps * 32, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq,
-                                                               blk_l1, ncb);
+    act_quant_kernel<F8><<<blocks, kAqWarps * 32, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq);
   }
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
@@ -553,12 +482,8 @@ int launch_aq(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x, u
 }  // namespace
 
 int launch_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
-                     uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream, int32_t* blk_l1) {
-  return launch_aq<false>(X, T, K, Xq, s_x, Xq_img, Xdq, stream, blk_l1);
-}
-
-int64_t l1_bounds_count(int64_t T, int64_t K) {
-  return ((T + kL1Rows - 1) / kL1Rows) * ((K + kL1Cols - 1) / kL1Cols);
+                     uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream) {
+  return launch_aq<false>(X, T, K, Xq, s_x, Xq_img, Xdq, stream);
 }
 
 int launch_act_quant_fp8(const uint16_t* X, int64_t T, int64_t K, uint8_t* Xq8, float* s8,

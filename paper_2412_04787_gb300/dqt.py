@@ -28,7 +28,6 @@ EXPORTED = [
     "dqt_sr_update_packed", "dqt_bitlinear_bwd_dw_update_packed",
     "dqt_adafactor_workspace_size", "dqt_adafactor_stats", "dqt_adafactor_apply",
     "dqt_bwd_dw_adafactor_workspace_size", "dqt_bitlinear_bwd_dw_adafactor",
-    "dqt_act_l1_count", "dqt_act_quant_l1", "dqt_bitlinear_fwd_l1",
 ]
 
 
@@ -85,11 +84,6 @@ def lib():
         L.dqt_codes_to_bf16.argtypes = [_vp, _i64, _vp, _vp]
         L.dqt_bitlinear_fwd.argtypes = [_vp, _vp, _vp, _f32, dqt_grid_t, _i64, _i64, _i64, _vp,
                                         _vp, _vp]
-        L.dqt_act_l1_count.argtypes = [_i64, _i64]
-        L.dqt_act_l1_count.restype = _i64
-        L.dqt_act_quant_l1.argtypes = [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp, _vp]
-        L.dqt_bitlinear_fwd_l1.argtypes = [_vp, _vp, _vp, _f32, dqt_grid_t, _i64, _i64, _i64,
-                                           _vp, _vp, _vp, _vp]
         L.dqt_bitlinear_bwd_dx.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp]
         L.dqt_bitlinear_bwd_dw_update.argtypes = [_vp, _vp, _vp, _f32, _vp, _vp,
                                                   C.POINTER(dqt_adamw_t), C.POINTER(dqt_sr_t),
@@ -253,52 +247,6 @@ def dqt_act_quant(X, Xq=None, s_x=None, Xq_img=None, Xdq=None, want=("Xq", "Xq_i
     return Xq, s_x, Xq_img, Xdq
 
 
-def fwd_drains(K, bits_or_grid):
-    """Whether the exact forward over K reduction elements with this weight grid
-    splits its fp32 accumulation into drained chunks (where the row L1 bounds of
-    dqt_act_quant_l1 let dqt_bitlinear_fwd_l1 take longer chunks)."""
-    g = _grid(bits_or_grid)
-    cm = max(g.qmax, -g.qmin, 1)
-    chunk = max(64, ((1 << 24) // (128 * cm)) // 64 * 64)
-    return int(K) > chunk
-
-
-def dqt_act_l1_count(T, K):
-    """Entries of the row L1 bounds of a [T, K] activation: ceil(T/128) * ceil(K/1024)."""
-    return int(lib().dqt_act_l1_count(int(T), int(K)))
-
-
-def dqt_act_quant_l1(X, Xq=None, s_x=None, Xq_img=None, Xdq=None, blk_l1=None,
-                     want=("Xq_img", "Xdq"), stream=None):
-    """dqt_act_quant plus the row L1 bounds the exact 8-bit forward plans its
-    fp32 chunks from (int32 [ceil(T/128), ceil(K/1024)]).  Returns (Xq, s_x,
-    Xq_img, Xdq, blk_l1)."""
-    _need(X, "X", torch.bfloat16)
-    if X.dim() != 2:
-        raise ValueError("X must be [T, K]")
-    T, K = X.shape
-    dev = X.device
-    if Xq is None and "Xq" in want:
-        Xq = torch.empty((T, K), dtype=torch.int8, device=dev)
-    if Xq_img is None and "Xq_img" in want:
-        Xq_img = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
-    if Xdq is None and "Xdq" in want:
-        Xdq = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
-    if s_x is None:
-        s_x = torch.empty(T, dtype=torch.float32, device=dev)
-    shape = ((T + 127) // 128, (K + 1023) // 1024)
-    if blk_l1 is None:
-        blk_l1 = torch.empty(shape, dtype=torch.int32, device=dev)
-    _opt(Xq, "Xq", torch.int8, (T, K))
-    _need(s_x, "s_x", torch.float32, (T,))
-    _opt(Xq_img, "Xq_img", torch.bfloat16, (T, K))
-    _opt(Xdq, "Xdq", torch.bfloat16, (T, K))
-    _need(blk_l1, "blk_l1", torch.int32, shape)
-    _check(lib().dqt_act_quant_l1(_ptr(X), T, K, _ptr(Xq), _ptr(s_x), _ptr(Xq_img), _ptr(Xdq),
-                                  _ptr(blk_l1), _stream(stream)), "dqt_act_quant_l1")
-    return Xq, s_x, Xq_img, Xdq, blk_l1
-
-
 def dqt_codes_to_bf16(W, W_img=None, stream=None):
     _need(W, "W", torch.int8)
     if W_img is None:
@@ -323,27 +271,6 @@ def dqt_bitlinear_fwd(Xq_img, s_x, W_img, s_w, bits_or_grid, Y=None, acc_out=Non
     _check(lib().dqt_bitlinear_fwd(_ptr(Xq_img), _ptr(s_x), _ptr(W_img), float(s_w),
                                    _grid(bits_or_grid), T, K, N, _ptr(Y), _ptr(acc_out),
                                    _stream(stream)), "dqt_bitlinear_fwd")
-    return Y
-
-
-def dqt_bitlinear_fwd_l1(Xq_img, s_x, W_img, s_w, bits_or_grid, blk_l1, Y=None, acc_out=None,
-                         stream=None):
-    """dqt_bitlinear_fwd planning its exact fp32 chunks from the row bounds
-    that dqt_act_quant_l1 wrote for this Xq_img (same results, fewer drains)."""
-    _need(Xq_img, "Xq_img", torch.bfloat16)
-    T, K = Xq_img.shape
-    _need(W_img, "W_img", torch.bfloat16)
-    N = W_img.shape[0]
-    _need(W_img, "W_img", torch.bfloat16, (N, K))
-    _need(s_x, "s_x", torch.float32, (T,))
-    _need(blk_l1, "blk_l1", torch.int32, ((T + 127) // 128, (K + 1023) // 1024))
-    if Y is None:
-        Y = torch.empty((T, N), dtype=torch.bfloat16, device=Xq_img.device)
-    _need(Y, "Y", torch.bfloat16, (T, N))
-    _opt(acc_out, "acc_out", torch.int32, (T, N))
-    _check(lib().dqt_bitlinear_fwd_l1(_ptr(Xq_img), _ptr(s_x), _ptr(W_img), float(s_w),
-                                      _grid(bits_or_grid), T, K, N, _ptr(Y), _ptr(acc_out),
-                                      _ptr(blk_l1), _stream(stream)), "dqt_bitlinear_fwd_l1")
     return Y
 
 
