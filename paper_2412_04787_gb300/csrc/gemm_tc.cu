@@ -751,9 +751,12 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
                                     : sdesc_sw128(smem_u32(sA), 16, 1024);
       const uint64_t b_desc0 = B_MN ? sdesc_sw128(smem_u32(sB), MN_CHUNK_BYTES, 1024)
                                     : sdesc_sw128(smem_u32(sB), 16, 1024);
-      constexpr uint64_t kAStage = S::A_BYTES >> 4, kBStage = S::B_BYTES >> 4;
-      constexpr uint64_t kAStep = A_MN ? (2048 >> 4) : (32 >> 4);  // per 16-element k step
-      constexpr uint64_t kBStep = B_MN ? (2048 >> 4) : (32 >> 4);
+      // the offsets only change the low word (no carry out of the 14-bit field)
+      const uint32_t a_lo0 = static_cast<uint32_t>(a_desc0), b_lo0 = static_cast<uint32_t>(b_desc0);
+      const uint64_t a_hi = a_desc0 & 0xFFFFFFFF00000000ull, b_hi = b_desc0 & 0xFFFFFFFF00000000ull;
+      constexpr uint32_t kAStage = S::A_BYTES >> 4, kBStage = S::B_BYTES >> 4;
+      constexpr uint32_t kAStep = A_MN ? (2048 >> 4) : (32 >> 4);  // per 16-element k step
+      constexpr uint32_t kBStep = B_MN ? (2048 >> 4) : (32 >> 4);
       for (int t = cid; t < p.num_tiles && ok; t += ncl) {
         const Unit un = decode_unit(p, t);
         const int kb0 = un.kb0, kb1 = un.kb1;
@@ -776,14 +779,16 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
             break;
           }
           tc_fence_after();
-          const uint64_t ad = a_desc0 + static_cast<uint64_t>(s) * kAStage;
-          const uint64_t bd = b_desc0 + static_cast<uint64_t>(s) * kBStage;
+          const uint32_t alo = a_lo0 + static_cast<uint32_t>(s) * kAStage;
+          const uint32_t blo = b_lo0 + static_cast<uint32_t>(s) * kBStage;
           const uint32_t d = tmem + static_cast<uint32_t>(b * BN);
 #pragma unroll
           for (int ks = 0; ks < BK / 16; ++ks) {
             const uint32_t acc = (!cstart || ks > 0) ? 1u : 0u;
-            if (F8) umma_f8_pair(d, ad + ks * kAStep, bd + ks * kBStep, IDESC, acc);
-            else umma_bf16_pair(d, ad + ks * kAStep, bd + ks * kBStep, IDESC, acc);
+            const uint64_t ad = a_hi | (alo + ks * kAStep);
+            const uint64_t bd = b_hi | (blo + ks * kBStep);
+            if (F8) umma_f8_pair(d, ad, bd, IDESC, acc);
+            else umma_bf16_pair(d, ad, bd, IDESC, acc);
           }
           umma_commit_pair_mc(&empty[s], 0x3);
           if (++s == ST) {
