@@ -75,7 +75,7 @@ def kernel_fingerprint(files=GEMM_SOURCES):
 # of operand and optimiser-state bytes), from one ncu capture, keyed by the
 # GEMM-source fingerprint it was taken on (see profiles/).  A stale entry
 # reports null.
-DW_TRAFFIC_BYTES = {"d1c21e870335": 273578240 + 60980736 + 33048064}
+DW_TRAFFIC_BYTES = {"062901c5c43d": 262199808 + 61180416 + 33049856}
 
 
 def _dist():

@@ -692,6 +692,7 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
       int it = 0, s = 0;  // k-blocks issued; stage it % ST
       uint32_t ph = 0;    // phase (it / ST) & 1
       bool ok = true;
+      const uint64_t pol_b = EPI == GEMM_DW ? l2_policy_evict_last() : 0ull;
       for (int t = cid; t < p.num_tiles && ok; t += ncl) {
         const Unit un = decode_unit(p, t);
         const int tile = un.tile, kb0 = un.kb0, kb1 = un.kb1;
@@ -716,6 +717,12 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
           }
           if (!B_MN) {
             tma_load_2d_pair(&tmB, bar, b, k0, n0);
+          } else if (EPI == GEMM_DW) {
+            // X~ (all K columns) is re-read by every wave of output-row tiles,
+            // while each dY column block is read by one wave: keep X~ in L2
+#pragma unroll
+            for (int j = 0; j < 2; ++j)
+              tma_load_2d_pair_hint(&tmB, bar, b + j * MN_CHUNK_BYTES, n0 + 64 * j, k0, pol_b);
           } else {
 #pragma unroll
             for (int j = 0; j < 2; ++j)
