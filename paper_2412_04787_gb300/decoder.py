@@ -45,9 +45,9 @@ class RMSNorm(torch.nn.Module):
         self.weight = torch.nn.Parameter(torch.ones(dim, device=device, dtype=torch.bfloat16))
 
     def forward(self, x):
-        xf = x.float()
-        y = xf * torch.rsqrt(xf.pow(2).mean(-1, keepdim=True) + self.eps)
-        return (y * self.weight.float()).to(torch.bfloat16)
+        # PyTorch's fused RMSNorm (statistics in fp32 for the bf16 input): one
+        # kernel each way instead of a chain of fp32 elementwise ops
+        return F.rms_norm(x, (x.shape[-1],), self.weight, self.eps)
 
 
 def _rope(x, cos, sin):
