@@ -842,7 +842,9 @@ def run_decoder(args):
     use_graph = not args.no_graph and graphable
     if graphable:
         model.enable_graph_updates()
-    opt = torch.optim.AdamW(model.dense_parameters(), lr=1e-3, fused=True, capturable=use_graph)
+    # the multi-tensor (foreach) AdamW: measured faster than the fused one on
+    # these bf16 parameters (embedding and head 32000 x hidden, norm gains)
+    opt = torch.optim.AdamW(model.dense_parameters(), lr=1e-3, foreach=True, capturable=use_graph)
     g = torch.Generator().manual_seed(5)
     host_ids = [torch.randint(0, cfg.vocab, (B, S + 1), generator=g).pin_memory() for _ in range(2)]
     ids_dev = [h.to(dev) for h in host_ids]
