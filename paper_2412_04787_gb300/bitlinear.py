@@ -31,11 +31,44 @@ not needed for these layers.  The state is ordinary module buffers, so
 ``state_dict()`` checkpoints it (codes, m, v as buffers; s_w, step, seed and
 tensor id as extra state).
 """
+import weakref
+
 import torch
 
 from . import dqt
 
 __all__ = ["DQTBitLinear"]
+
+
+# Sibling layers that read the same activation (q, k and v; gate and up)
+# share its quantisation: the last input quantised is remembered by object
+# identity and version counter, so a new or modified tensor is never mistaken
+# for it (a freed tensor's memory reused by a new one is a different object).
+class _QuantCache:
+    ref = None
+    version = -1
+    act = None
+    result = None
+
+
+def _quantised(x, x2, act):
+    c = _QuantCache
+    try:
+        version = x._version
+    except RuntimeError:  # inference tensors keep no version counter: no sharing
+        version = None
+    if (version is not None and c.ref is not None and c.ref() is x and c.version == version
+            and c.act == act):
+        return c.result
+    if act == "fp8":
+        res = dqt.dqt_act_quant_fp8(x2)
+    else:
+        res = dqt.dqt_act_quant(x2, want=("Xq_img", "Xdq"))
+    if version is not None:
+        c.ref, c.version, c.act, c.result = weakref.ref(x), version, act, res
+    else:
+        c.ref, c.result = None, None
+    return res
 
 
 class _BitLinearFn(torch.autograd.Function):
@@ -47,14 +80,17 @@ class _BitLinearFn(torch.autograd.Function):
             x2 = x2.to(torch.bfloat16)
         x2 = x2.contiguous()
         if layer.act == "fp8":
-            q8, s_x, xdq = dqt.dqt_act_quant_fp8(x2)
+            q8, s_x, xdq = _quantised(x, x2, "fp8")
             y = dqt.dqt_bitlinear_fwd_fp8(q8, s_x, layer.weight_fp8(), float(layer.s_w),
                                           layer.grid_tuple)
+            w_img = None  # dX needs the bf16 image: built in backward
         else:
-            _, s_x, q_img, xdq = dqt.dqt_act_quant(x2, want=("Xq_img", "Xdq"))
-            y = dqt.dqt_bitlinear_fwd(q_img, s_x, layer.weight_bf16(), float(layer.s_w),
-                                      layer.grid_tuple)
-        ctx.save_for_backward(xdq)
+            _, s_x, q_img, xdq = _quantised(x, x2, "int8")
+            # the weight's code image serves the forward and, kept until the
+            # backward, dX (the codes change only after dX, in the update)
+            w_img = layer.weight_bf16()
+            y = dqt.dqt_bitlinear_fwd(q_img, s_x, w_img, float(layer.s_w), layer.grid_tuple)
+        ctx.save_for_backward(xdq, w_img)
         ctx.layer = layer
         ctx.in_shape = x.shape
         ctx.in_dtype = x.dtype
@@ -62,16 +98,17 @@ class _BitLinearFn(torch.autograd.Function):
 
     @staticmethod
     def backward(ctx, dy):
-        (xdq,) = ctx.saved_tensors
+        xdq, w_img = ctx.saved_tensors
         layer = ctx.layer
         N = layer.out_features
         dy2 = dy.reshape(-1, N)
         if dy2.dtype != torch.bfloat16:
             dy2 = dy2.to(torch.bfloat16)
         dy2 = dy2.contiguous()
-        # the codes have not changed since the forward: the image is rebuilt
-        # instead of being kept alive across the step
-        dx = dqt.dqt_bitlinear_bwd_dx(dy2, layer.weight_bf16(), float(layer.s_w))
+        # the codes have not changed since the forward
+        if w_img is None:
+            w_img = layer.weight_bf16()
+        dx = dqt.dqt_bitlinear_bwd_dx(dy2, w_img, float(layer.s_w))
         if layer.update_in_backward:
             layer._dqt_update(dy2, xdq)
         return dx.reshape(ctx.in_shape).to(ctx.in_dtype), None, None

@@ -954,6 +954,15 @@ bool make_map(CUtensorMap* map, const void* ptr, uint64_t inner, uint64_t outer,
               uint32_t box_inner, uint32_t box_outer, int elem_bytes = 2) {
   EncodeTiledFn enc = encode_fn();
   if (!enc) return false;
+  // The encoder is a driver call and needs a context current in the calling
+  // thread.  A thread whose first CUDA work in this process comes through
+  // this library (an autograd worker running a backward, say) may not have
+  // one bound yet: a runtime call binds the device's primary context.
+  thread_local bool bound = false;
+  if (!bound) {
+    if (cudaFree(nullptr) != cudaSuccess) return false;
+    bound = true;
+  }
   const cuuint64_t dims[2] = {inner, outer};
   const cuuint64_t strides[1] = {inner * static_cast<cuuint64_t>(elem_bytes)};
   const cuuint32_t box[2] = {box_inner, box_outer};

@@ -13,6 +13,7 @@ decoder.
   ever move: the update is lost, as the paper observes.
 """
 import io
+import os
 
 import numpy as np
 import pytest
@@ -68,6 +69,28 @@ def test_bitlinear_module_matches_oracle(bits_w):
     assert diff.mean() <= 1e-4 + 1.0 / diff.size
     assert (np.abs(cg - c1.astype(np.int32))[diff] == 1).all()
     assert layer.step == 1 and int(layer.changed.item()) == int((cg != c0).sum())
+
+
+def test_module_backward_in_a_fresh_process():
+    """The first CUDA work of the autograd worker thread of a fresh process is
+    this library's dX GEMM, whose tensor-map encoder (a driver call) needs a
+    context bound in that thread: a process of its own, so that no earlier test
+    has already bound one there."""
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    code = (
+        "import torch\n"
+        "from paper_2412_04787_gb300.bitlinear import DQTBitLinear\n"
+        "layer = DQTBitLinear(264, 520, bits=1.58, seed=3, tensor_id=1, init_seed=5)\n"
+        "x = torch.randn(300, 264, device='cuda', dtype=torch.bfloat16, requires_grad=True)\n"
+        "layer(x).backward(torch.randn(300, 520, device='cuda', dtype=torch.bfloat16))\n"
+        "torch.cuda.synchronize()\n"
+        "assert x.grad is not None and int(layer.step) == 1\n"
+        "print('ok')\n")
+    r = subprocess.run([sys.executable, "-c", code], cwd=root, capture_output=True, text=True,
+                       timeout=600)
+    assert r.returncode == 0 and "ok" in r.stdout, r.stderr[-3000:]
 
 
 def test_bitlinear_state_dict_resume():
