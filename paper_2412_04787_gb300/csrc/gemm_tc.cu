@@ -454,12 +454,24 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       // ---------------- MMA issuer ----------------
-      int it = 0;
+      // (short per-k-block loop, as in the 2-SM kernel: incremental stage and
+      // phase, descriptors from their precomputed 32-bit halves)
+      int s = 0;
+      uint32_t ph = 0;
       int u = 0;  // accumulation units (tile chunks) issued so far
       bool ok = true;
+      const uint64_t a_desc0 = A_MN ? sdesc_sw128(smem_u32(sA), MN_CHUNK_BYTES, 1024)
+                                    : sdesc_sw128(smem_u32(sA), 16, 1024);
+      const uint64_t b_desc0 = B_MN ? sdesc_sw128(smem_u32(sB), MN_CHUNK_BYTES, 1024)
+                                    : sdesc_sw128(smem_u32(sB), 16, 1024);
+      const uint32_t a_lo0 = static_cast<uint32_t>(a_desc0), b_lo0 = static_cast<uint32_t>(b_desc0);
+      const uint64_t a_hi = a_desc0 & 0xFFFFFFFF00000000ull, b_hi = b_desc0 & 0xFFFFFFFF00000000ull;
+      constexpr uint32_t kAStage = S::A_BYTES >> 4, kBStage = S::B_BYTES >> 4;
+      constexpr uint32_t kAStep = A_MN ? (2048 >> 4) : (32 >> 4);
+      constexpr uint32_t kBStep = B_MN ? (2048 >> 4) : (32 >> 4);
       for (int t = blockIdx.x; t < p.num_tiles && ok; t += gridDim.x) {
-        for (int kb = 0; kb < p.num_kb; ++kb, ++it) {
-          const int kc = kb % p.chunk_kb;
+        int kc = 0;  // k-blocks into the current chunk
+        for (int kb = 0; kb < p.num_kb; ++kb) {
           const int b = u & 1;
           if (kc == 0 && u >= 2) {
             // The epilogue must have released this accumulator buffer.
@@ -469,28 +481,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_after();
           }
-          const int s = it % kStages;
-          const uint32_t ph = (it / kStages) & 1u;
           if (!mbar_wait(&full[s], ph, p.wait_ns)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t a_base = smem_u32(sA + s * S::A_BYTES);
-          const uint32_t b_base = smem_u32(sB + s * S::B_BYTES);
+          const uint32_t alo = a_lo0 + static_cast<uint32_t>(s) * kAStage;
+          const uint32_t blo = b_lo0 + static_cast<uint32_t>(s) * kBStage;
           const uint32_t d = tmem + static_cast<uint32_t>(b * BN);
 #pragma unroll
-          for (int ks = 0; ks < BK / 16; ++ks) {
-            const uint64_t ad = A_MN ? sdesc_sw128(a_base + ks * 2048, MN_CHUNK_BYTES, 1024)
-                                     : sdesc_sw128(a_base + ks * 32, 16, 1024);
-            const uint64_t bd = B_MN ? sdesc_sw128(b_base + ks * 2048, MN_CHUNK_BYTES, 1024)
-                                     : sdesc_sw128(b_base + ks * 32, 16, 1024);
-            umma_bf16(d, ad, bd, IDESC, (kc > 0 || ks > 0) ? 1u : 0u);
-          }
+          for (int ks = 0; ks < BK / 16; ++ks)
+            umma_bf16(d, a_hi | (alo + ks * kAStep), b_hi | (blo + ks * kBStep), IDESC,
+                      (kc > 0 || ks > 0) ? 1u : 0u);
           umma_commit(&empty[s]);
-          if (kc == p.chunk_kb - 1 || kb == p.num_kb - 1) {
+          if (++s == kStages) {
+            s = 0;
+            ph ^= 1u;
+          }
+          if (++kc == p.chunk_kb || kb == p.num_kb - 1) {
             umma_commit(&acc_full[b]);
             ++u;
+            kc = 0;
           }
         }
       }
