@@ -7,14 +7,22 @@
 //   dW          = dY^T X_tilde        (Sec. 3.2) fused with AdamW (Sec. 4.1) and
 //                                     W_hat = SR(W') (Eq. 1, Eq. 5) in the epilogue
 //
-// Persistent kernel: one CTA per SM walks output tiles (128 x BN) in a static
-// round-robin order.  Warp roles:
-//   warp 0     TMA producer (one lane): a kStages-deep ring of A/B stages that
-//              runs continuously across tiles
+// Two persistent kernels walk output tiles in a static round-robin order:
+//
+//   gemm_pair_kernel (default): a cluster of two CTAs on one TPC computes a
+//     256 x 256 tile with tcgen05.mma.cta_group::2; each CTA stages its 128
+//     rows of A and its half of B, and the leader's single MMA-issuing lane
+//     drives both SMs' tensor cores.
+//   gemm_kernel (dqt_set_gemm_tiles(1)): one CTA per SM, 128 x 256 tiles.
+//
+// Warp roles (both kernels):
+//   warp 0     TMA producer (one lane): a ring of A/B stages that runs
+//              continuously across tiles
 //   warp 1     tensor-memory allocator and MMA issuer (one lane)
-//   warps 2-9  epilogue: tensor memory -> registers -> global memory; each
-//              tensor-memory lane quadrant is served by two warps, one per
-//              half of the tile's columns
+//   warps 2+   epilogue: tensor memory -> registers -> global memory; each
+//              tensor-memory lane quadrant is served by the same number of
+//              warps (8 epilogue warps, 16 for the dW update and the drained
+//              8-bit forward of the 2-SM kernel)
 // The accumulator is double-buffered in tensor memory, so the epilogue of one
 // tile (for dW: the whole AdamW + stochastic-rounding update) overlaps the
 // MMAs of the next.
@@ -29,10 +37,11 @@
 // (exact for |v| <= 256); each product is exact in fp32 and a sum of integers
 // stays exact while its magnitude is at most 2^24.  The reduction is split into
 // chunks of chunk_k elements with chunk_k * 128 * max|c| <= 2^24.  With more
-// than one chunk (8-bit codes, K > 1024) the kernel runs with BN = 128 and a
-// third tensor-memory region: after each chunk but the last the epilogue
-// converts the fp32 partial to int32 and adds it to the tile's running int32
-// sum there.  Ternary weights (max|c| = 1) need no drain for K <= 131072.
+// than one chunk (8-bit codes, K > 1024) every chunk is its own accumulation
+// unit; the epilogue converts each chunk's exact fp32 sum to int32 and adds it
+// to running sums: in registers (the 2-SM kernel, 16 epilogue warps) or in a
+// third tensor-memory region (the 1-SM kernel, BN = 128).  Ternary weights
+// (max|c| = 1) need no drain for K <= 131072.
 #include <cuda.h>
 
 #include "dqt_internal.h"
