@@ -51,7 +51,8 @@ class RMSNorm(torch.nn.Module):
 
 
 def _rope(x, cos, sin):
-    # x: [B, H, S, D]; rotate pairs (first half, second half)
+    # rotate pairs (first half, second half) of the last dimension; cos and sin
+    # broadcast against x
     d = x.shape[-1] // 2
     x1, x2 = x[..., :d], x[..., d:]
     return torch.cat([x1 * cos - x2 * sin, x1 * sin + x2 * cos], dim=-1)
@@ -79,10 +80,13 @@ class Block(torch.nn.Module):
         nh = self.heads
         hd = Hd // nh
         a = self.attn_norm(x)
-        q = self.q(a).view(B, S, nh, hd).transpose(1, 2)
-        k = self.k(a).view(B, S, nh, hd).transpose(1, 2)
+        # rotary embedding in the [B, S, H, D] layout the projections produce;
+        # attention reads head-major views of it, so no layout copy is made in
+        # either direction (cos, sin: [1, 1, S, D/2] -> [1, S, 1, D/2])
+        c4, s4 = cos.transpose(1, 2), sin.transpose(1, 2)
+        q = _rope(self.q(a).view(B, S, nh, hd), c4, s4).transpose(1, 2)
+        k = _rope(self.k(a).view(B, S, nh, hd), c4, s4).transpose(1, 2)
         v = self.v(a).view(B, S, nh, hd).transpose(1, 2)
-        q, k = _rope(q, cos, sin), _rope(k, cos, sin)
         o = F.scaled_dot_product_attention(q, k, v, is_causal=True)
         x = x + self.o(o.transpose(1, 2).reshape(B, S, Hd))
         m = self.mlp_norm(x)
