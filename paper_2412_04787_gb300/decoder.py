@@ -50,12 +50,12 @@ class RMSNorm(torch.nn.Module):
         return F.rms_norm(x, (x.shape[-1],), self.weight, self.eps)
 
 
-def _rope(x, cos, sin):
-    # rotate pairs (first half, second half) of the last dimension; cos and sin
-    # broadcast against x
-    d = x.shape[-1] // 2
-    x1, x2 = x[..., :d], x[..., d:]
-    return torch.cat([x1 * cos - x2 * sin, x1 * sin + x2 * cos], dim=-1)
+def _rope(x, freqs):
+    # rotary position embedding on interleaved pairs (x[2i], x[2i+1]) of the
+    # last dimension as one complex multiply, in fp32 (the LLaMA formulation);
+    # freqs: unit complex numbers broadcasting against x's pairs
+    xc = torch.view_as_complex(x.float().reshape(*x.shape[:-1], -1, 2))
+    return torch.view_as_real(xc * freqs).flatten(-2).to(x.dtype)
 
 
 class Block(torch.nn.Module):
@@ -75,17 +75,16 @@ class Block(torch.nn.Module):
         self.q, self.k, self.v, self.o = bl(h, h, 0), bl(h, h, 1), bl(h, h, 2), bl(h, h, 3)
         self.gate, self.up, self.down = bl(h, f, 4), bl(h, f, 5), bl(f, h, 6)
 
-    def forward(self, x, cos, sin):
+    def forward(self, x, freqs):
         B, S, Hd = x.shape
         nh = self.heads
         hd = Hd // nh
         a = self.attn_norm(x)
-        # rotary embedding in the [B, S, H, D] layout the projections produce;
-        # attention reads head-major views of it, so no layout copy is made in
-        # either direction (cos, sin: [1, 1, S, D/2] -> [1, S, 1, D/2])
-        c4, s4 = cos.transpose(1, 2), sin.transpose(1, 2)
-        q = _rope(self.q(a).view(B, S, nh, hd), c4, s4).transpose(1, 2)
-        k = _rope(self.k(a).view(B, S, nh, hd), c4, s4).transpose(1, 2)
+        # rotary embedding in the [B, S, H, D] layout the projections produce
+        # (freqs: [1, S, 1, D/2]); attention reads head-major views of it, so
+        # no layout copy is made in either direction
+        q = _rope(self.q(a).view(B, S, nh, hd), freqs).transpose(1, 2)
+        k = _rope(self.k(a).view(B, S, nh, hd), freqs).transpose(1, 2)
         v = self.v(a).view(B, S, nh, hd).transpose(1, 2)
         o = F.scaled_dot_product_attention(q, k, v, is_causal=True)
         x = x + self.o(o.transpose(1, 2).reshape(B, S, Hd))
@@ -153,10 +152,9 @@ class DQTDecoder(torch.nn.Module):
         x = F.embedding(ids, self.embed)
         t = torch.arange(S, device=ids.device, dtype=torch.float32)
         ang = torch.outer(t, self.inv_freq)
-        cos = ang.cos().to(torch.bfloat16)[None, None]
-        sin = ang.sin().to(torch.bfloat16)[None, None]
+        freqs = torch.polar(torch.ones_like(ang), ang)[None, :, None, :]
         for blk in self.blocks:
-            x = blk(x, cos, sin)
+            x = blk(x, freqs)
         x = self.norm(x)
         logits = x @ self.head.t()
         if targets is None:
