@@ -24,7 +24,7 @@
  *   Sec 1       2-bit packed ternary storage                -> dqt_oracle_pack_ternary
  *   Sec 4.3     Adafactor (factored second moment) + SR     -> dqt_oracle_adafactor_*
  *
- * Readings where the paper is silent (each is listed in the design notes):
+ * Readings where the paper is silent, taken here:
  *   - ternary ("1.58 bit") means the grid [-1, 1] with s = 1 / AbsMean;
  *     integer n uses Q_n = -2^(n-1), Q_p = 2^(n-1) - 1 literally;
  *   - the scale s is fixed at initialisation and SR acts on the code domain

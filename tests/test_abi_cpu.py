@@ -34,7 +34,7 @@ def test_header_symbols_exported(L):
         assert hasattr(L, n), n  # dlsym succeeds
 
 
-def test_north_star_entry_points_present():
+def test_hot_path_entry_points_present():
     for n in ["dqt_act_quant", "dqt_bitlinear_fwd", "dqt_bitlinear_bwd_dx",
               "dqt_bitlinear_bwd_dw_update", "dqt_sr_update"]:
         assert n in _declared()
