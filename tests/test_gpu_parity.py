@@ -1,7 +1,7 @@
 """GPU parity: the CUDA path (through the C ABI) against the CPU oracle on the
 same seeded inputs.
 
-Rules (stated here and in the design notes):
+Rules:
   * bit-exact: activation codes, s_x, the bf16 operand images, the int32 forward
     accumulators, the forward output Y (same fp32 formula on both sides), the
     weight image, and the standalone SR update (codes, m, v) given identical
@@ -85,6 +85,22 @@ def test_act_quant_bit_exact(T, K):
     assert np.array_equal(s_x.cpu().numpy().view(np.uint32), s.view(np.uint32))
     assert np.array_equal(bits(Xq_img), qi)
     assert np.array_equal(bits(Xdq), xd)
+
+
+def test_act_quant_beyond_int32_sampled():
+    """T x K = 262147 x 8192 > 2^31 elements (row 262144 starts at element
+    2^31): codes, s_x and both images bit-exact on sampled rows."""
+    T, K = (1 << 18) + 3, 8192
+    X = inputs.normal((T, K), 1.0, seed=45, dtype=torch.bfloat16)
+    Xq, s_x, Xq_img, Xdq = dqt.dqt_act_quant(X.cuda())
+    torch.cuda.synchronize()
+    rows = np.array([0, 1, T // 2, 262143, 262144, T - 1])
+    q, s, qi, xd = oracle.act_quant(bits(X[torch.from_numpy(rows)]))
+    it = torch.from_numpy(rows).cuda()
+    assert np.array_equal(Xq[it].cpu().numpy(), q)
+    assert np.array_equal(s_x[it].cpu().numpy().view(np.uint32), s.view(np.uint32))
+    assert np.array_equal(bits(Xq_img[it]), qi)
+    assert np.array_equal(bits(Xdq[it]), xd)
 
 
 def test_act_quant_partial_outputs():
@@ -174,6 +190,27 @@ def test_fwd_adversarial_magnitudes():
     assert np.array_equal(bits(Y), Yr)
 
 
+def test_fwd_output_beyond_int32_sampled():
+    """Y and the int32 accumulators with T x N = 524293 x 4096 > 2^31 elements
+    (row 524288 starts at element 2^31): sampled rows on both sides of it."""
+    T, K, N = (1 << 19) + 5, 64, 4096
+    X = inputs.normal((T, K), 1.0, seed=41, dtype=torch.bfloat16)
+    W0 = inputs.normal((N, K), 0.02, seed=42)
+    qmin, qmax = oracle.grid(1.58)
+    c, s_w, _ = oracle.absmean_init(W0.numpy(), qmin, qmax)
+    _, s_x, Xq_img, _ = dqt.dqt_act_quant(X.cuda(), want=("Xq_img",))
+    W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
+    acc = torch.empty((T, N), dtype=torch.int32, device="cuda")
+    Y = dqt.dqt_bitlinear_fwd(Xq_img, s_x, W_img, float(s_w), (qmin, qmax), acc_out=acc)
+    dqt.dqt_check_device_status()
+    rows = np.array([0, 1, T // 2, 524287, 524288, T - 2, T - 1])
+    q, s, _, _ = oracle.act_quant(bits(X[torch.from_numpy(rows)]))
+    Yr, accr = oracle.fwd(q, s, c, np.float32(s_w))
+    it = torch.from_numpy(rows).cuda()
+    assert np.array_equal(acc[it].cpu().numpy(), accr)
+    assert np.array_equal(bits(Y[it]), Yr)
+
+
 @pytest.mark.parametrize("which", ["gate_up", "down"])
 def test_fwd_llama_mlp_sampled_rows(which):
     T, H, I = 8192, 2048, 5632
@@ -194,6 +231,24 @@ def test_bwd_dx(T, N, K):
     ref = oracle.bwd_dx(bits(dY), c, np.float32(s_w))
     assert rel_err(dX.cpu().double().numpy(), ref) <= REL_TOL
     assert elem_err(dX.cpu().double().numpy(), ref) <= REL_TOL
+
+
+def test_bwd_dx_output_beyond_int32_sampled():
+    """dX of T x K = 524293 x 4096 > 2^31 elements: sampled rows on both sides
+    of element 2^31, within the fp64 tolerance."""
+    T, N, K = (1 << 19) + 5, 64, 4096
+    dY = inputs.normal((T, N), 1e-2, seed=43, dtype=torch.bfloat16)
+    W0 = inputs.normal((N, K), 0.02, seed=44)
+    qmin, qmax = oracle.grid(1.58)
+    c, s_w, _ = oracle.absmean_init(W0.numpy(), qmin, qmax)
+    W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
+    dX = dqt.dqt_bitlinear_bwd_dx(dY.cuda(), W_img, float(s_w))
+    dqt.dqt_check_device_status()
+    rows = np.array([0, 1, T // 2, 524287, 524288, T - 2, T - 1])
+    ref = oracle.bwd_dx(bits(dY[torch.from_numpy(rows)]), c, np.float32(s_w))
+    got = dX[torch.from_numpy(rows).cuda()].cpu().double().numpy()
+    assert rel_err(got, ref) <= REL_TOL
+    assert elem_err(got, ref) <= REL_TOL
 
 
 @pytest.mark.parametrize("T,N,K", [(256, 512, 512), (300, 520, 264), (77, 24, 200)])
@@ -256,6 +311,47 @@ def test_sr_update_bit_exact(bits_w, numel, step, round_mode):
     assert np.array_equal(mg.cpu().numpy().view(np.uint32), m1.ravel().view(np.uint32))
     assert np.array_equal(vg.cpu().numpy().view(np.uint32), v1.ravel().view(np.uint32))
     assert int(changed.item()) == n_ch
+
+
+def test_sr_update_beyond_int32_sampled():
+    """The largest update size: 2^31 + 6 weights (past the int32 index range,
+    with a ragged tail), ternary codes from the AbsMean init of N(0, 0.02),
+    AdamW step 1.  Bit-exact against the oracle on sampled 4096-element rows
+    (both ends, both sides of element 2^31, random rows) and on the six tail
+    elements, each at its global element index (Philox counter e / 4)."""
+    numel = (1 << 31) + 6
+    qmin, qmax = oracle.grid(1.58)
+    W0 = inputs.normal((numel,), 0.02, seed=31)
+    c, s_w, _ = oracle.absmean_init(W0.numpy(), qmin, qmax)
+    del W0
+    grad = inputs.normal((numel,), 1e-3, seed=32)
+    hp = dqt.adamw(lr=1e-3, step=1)
+    sr = dqt.sr_stream(seed=1234, tensor_id=5)
+    Wg = torch.from_numpy(c).cuda()
+    gg = grad.cuda()
+    mg = torch.zeros(numel, dtype=torch.float32, device="cuda")
+    vg = torch.zeros(numel, dtype=torch.float32, device="cuda")
+    dqt.dqt_sr_update(gg, Wg, s_w, mg, vg, hp, sr, (qmin, qmax))
+    dqt.dqt_check_device_status()
+    del gg
+    k = oracle.adamw_consts(hp.lr, hp.beta1, hp.beta2, hp.eps, hp.weight_decay, 1, s_w)
+    g_np = grad.numpy()
+    K = 4096
+    last_full = numel // K - 1  # row 524287 ends at element 2^31 - 1
+    rng = np.random.default_rng(7)
+    rows = np.unique(np.concatenate([[0, 1, last_full - 1, last_full],
+                                     rng.integers(0, last_full, 28)])).astype(np.int64)
+    cases = [(rows, K), (np.arange(1 << 30, (1 << 30) + 3, dtype=np.int64), 2)]
+    for rws, kk in cases:
+        idx = (rws[:, None] * kk + np.arange(kk)[None, :]).ravel()
+        assert idx.max() < numel
+        zeros = np.zeros(idx.size, np.float32)
+        c1, m1, v1, _ = oracle.update(g_np[idx].reshape(-1, kk), c[idx], zeros, zeros, k,
+                                      qmin, qmax, 1234, 1, 5, 0, rows=rws)
+        it = torch.from_numpy(idx).cuda()
+        assert np.array_equal(Wg[it].cpu().numpy(), c1.ravel())
+        assert np.array_equal(mg[it].cpu().numpy().view(np.uint32), m1.ravel().view(np.uint32))
+        assert np.array_equal(vg[it].cpu().numpy().view(np.uint32), v1.ravel().view(np.uint32))
 
 
 # ---------------------------------------------------------------------------
