@@ -414,6 +414,42 @@ def test_fused_update_llama_mlp_sampled_rows():
     _fused(8192, 5632, 2048, 1.58, 2, seed=52, rows=np.array([0, 1535, 1536, 1800, 2047]))
 
 
+def test_fused_update_beyond_int32_sampled():
+    """The fused dW + AdamW + SR call on N x K = 65544 x 32768 > 2^31 weights
+    (row 65536 starts at element 2^31; the last tile row holds 8 ragged rows),
+    T = 256 tokens: sampled weight rows on both sides of element 2^31, each
+    at its global element index."""
+    T, K, N = 256, 32768, 65544
+    X = inputs.normal((T, K), 1.0, seed=61, dtype=torch.bfloat16)
+    dY = inputs.normal((T, N), 1e-2, seed=62, dtype=torch.bfloat16)
+    qmin, qmax = oracle.grid(1.58)
+    W0 = inputs.normal((N, K), 0.02, seed=63)
+    c, s_w, _ = oracle.absmean_init(W0.numpy(), qmin, qmax)
+    del W0
+    hp = dqt.adamw(lr=1e-3, step=1)
+    sr = dqt.sr_stream(seed=1234, tensor_id=6)
+    _, _, _, Xdq = dqt.dqt_act_quant(X.cuda(), want=("Xdq",))
+    Wg = torch.from_numpy(c).cuda()
+    mg = torch.zeros((N, K), dtype=torch.float32, device="cuda")
+    vg = torch.zeros((N, K), dtype=torch.float32, device="cuda")
+    dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), Xdq, Wg, float(s_w), mg, vg, hp, sr, (qmin, qmax))
+    dqt.dqt_check_device_status()
+    rows = np.array([0, 1, 40000, 65535, 65536, 65543])
+    _, _, _, xd = oracle.act_quant(bits(X))
+    gref = oracle.bwd_dw_bf16x(bits(dY), xd, rows=rows).astype(np.float32)
+    k = oracle.adamw_consts(hp.lr, hp.beta1, hp.beta2, hp.eps, hp.weight_decay, 1, s_w)
+    zeros = np.zeros((rows.size, K), np.float32)
+    c1, m1, _, _ = oracle.update(gref, c[rows], zeros, zeros, k, qmin, qmax, 1234, 1, 6, 0,
+                                 rows=rows)
+    it = torch.from_numpy(rows).cuda()
+    cg = Wg[it].cpu().numpy().astype(np.int32)
+    diff = cg != c1.astype(np.int32)
+    assert diff.mean() <= 1e-4 + 1.0 / diff.size, diff.sum()
+    assert (np.abs(cg - c1.astype(np.int32))[diff] == 1).all()
+    mr = mg[it].cpu().numpy()
+    assert np.abs(mr - m1).max() <= 1e-3 * np.abs(m1).max()
+
+
 def test_fused_equals_standalone_on_same_gradient():
     """Fused epilogue and standalone kernel draw the same uniforms for the same
     element: given the fused kernel's own fp32 gradient, codes are identical."""
