@@ -364,6 +364,40 @@ int dqt_bitlinear_bwd_dw_adafactor(const dqt_bf16* dY, const dqt_bf16* Xdq, void
                                    unsigned long long* changed_out, void* ws, size_t ws_bytes,
                                    void* stream);
 
+/* ---------------------------------------------------------------------------
+ * Decoder support.  Not part of the DQT method: two operations of the
+ * LLaMA-structured decoder built around the BitLinear layers (the model family
+ * of Sec. 4.1), each one pass over bf16 data in HBM with fp32 arithmetic.
+ * ------------------------------------------------------------------------- */
+
+/* Rotary position embedding (LLaMA form) of x, bf16 [rows, H, D] contiguous
+ * with rows = B * S (row r is at position r % S), into y (same shape; y must
+ * not overlap x).  Each interleaved pair (x[2i], x[2i+1]) of a head is a
+ * complex number multiplied by exp(i theta_{pos, i}):
+ *   y[2i] = x[2i] c - x[2i+1] s,   y[2i+1] = x[2i] s + x[2i+1] c
+ * with (c, s) = cos_sin[pos, i, 0..1], fp32 [S, D/2, 2] supplied by the
+ * caller; each product and sum is a separately rounded fp32 operation, the
+ * result rounded to bf16 (nearest-even).  inverse = 1 rotates by -theta (the
+ * backward: the transpose of the rotation).  D a multiple of 8; x, y, cos_sin
+ * 16-byte aligned (DQT_ERR_ALIGN otherwise). */
+int dqt_rope_bf16(const dqt_bf16* x, dqt_bf16* y, const float* cos_sin, int64_t rows, int64_t S,
+                  int64_t H, int64_t D, int32_t inverse, void* stream);
+
+/* Token cross-entropy over bf16 logits [M, V] (row-major, V a multiple of 8,
+ * 16-byte aligned) with int64 targets [M]: per row, in fp32,
+ *   lse[m] = log sum_v exp(logits[m, v]),   row_loss[m] = lse[m] - logits[m, t_m]
+ * (row_loss 0 for a target outside [0, V)).  The mean loss is the caller's sum
+ * of row_loss over the rows with valid targets divided by their count. */
+int dqt_cross_entropy_fwd_bf16(const dqt_bf16* logits, const int64_t* targets, int64_t M,
+                               int64_t V, float* lse, float* row_loss, void* stream);
+/* Its gradient: dlogits[m, v] = bf16((exp(logits[m, v] - lse[m]) - [v == t_m]) * scale[0]),
+ * scale a device fp32 scalar (the upstream gradient divided by the count of
+ * valid rows); rows with a target outside [0, V) get zeros.  dlogits 16-byte
+ * aligned, [M, V] bf16, not overlapping logits. */
+int dqt_cross_entropy_bwd_bf16(const dqt_bf16* logits, const int64_t* targets, const float* lse,
+                               const float* scale, int64_t M, int64_t V, dqt_bf16* dlogits,
+                               void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -1,0 +1,212 @@
+// Decoder support kernels (not part of the DQT method): the rotary position
+// embedding and the token cross-entropy of the LLaMA-structured decoder built
+// around the BitLinear layers, each one HBM-bound pass over bf16 data with
+// fp32 arithmetic, in place of chains of PyTorch elementwise kernels with fp32
+// intermediates in HBM.
+//
+//   rope_kernel      y = x rotated pairwise by the position angle (LLaMA:
+//                    interleaved pairs (x[2i], x[2i+1]) as complex numbers
+//                    times exp(i theta)), or by -theta for the backward
+//   ce_fwd_kernel    per row: lse = log sum_v exp(x_v), loss = lse - x_target
+//   ce_bwd_kernel    dx_v = (exp(x_v - lse) - [v == target]) * scale
+#include <cuda_bf16.h>
+
+#include "dqt_internal.h"
+
+namespace dqt {
+
+namespace {
+
+constexpr int kRopeThreads = 256;
+constexpr int kCeThreads = 256;
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+// One 16-byte vector (four pairs of one head) per thread step.  cs holds
+// (cos, sin) per position and pair: fp32 [S, D/2, 2].
+template <bool INV>
+__global__ void __launch_bounds__(kRopeThreads)
+    rope_kernel(const uint4* __restrict__ x, uint4* __restrict__ y, const float4* __restrict__ cs,
+                int64_t nvec, int64_t row_vecs, int64_t S, int64_t head_vecs) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * kRopeThreads;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * kRopeThreads + threadIdx.x; i < nvec;
+       i += stride) {
+    const int64_t row = i / row_vecs;
+    const int64_t dv = (i - row * row_vecs) % head_vecs;  // vector within the head
+    const int64_t pos = row % S;
+    // four pairs = eight floats = two float4 of the table
+    const float4* t = cs + (pos * head_vecs + dv) * 2;
+    const float4 c01 = __ldg(t), c23 = __ldg(t + 1);
+    const float cth[4] = {c01.x, c01.z, c23.x, c23.z};
+    const float sth[4] = {INV ? -c01.y : c01.y, INV ? -c01.w : c01.w, INV ? -c23.y : c23.y,
+                          INV ? -c23.w : c23.w};
+    const uint4 v = x[i];
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float xe = bf16_lo(w[j]), xo = bf16_hi(w[j]);
+      const float ye = __fsub_rn(__fmul_rn(xe, cth[j]), __fmul_rn(xo, sth[j]));
+      const float yo = __fadd_rn(__fmul_rn(xe, sth[j]), __fmul_rn(xo, cth[j]));
+      o[j] = pack_bf16x2(ye, yo);
+    }
+    y[i] = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+// (max, sum of exp(x - max)) pairs combine associatively
+__device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2) {
+  if (m2 > m) {
+    s = s * expf(m - m2) + s2;
+    m = m2;
+  } else if (m2 != -INFINITY) {
+    s += s2 * expf(m2 - m);
+  }
+}
+
+__device__ __forceinline__ void lse_block(float& m, float& s, float* sh_m, float* sh_s) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1)
+    lse_merge(m, s, __shfl_xor_sync(0xffffffffu, m, off), __shfl_xor_sync(0xffffffffu, s, off));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) {
+    sh_m[warp] = m;
+    sh_s[warp] = s;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    m = lane < kCeThreads / 32 ? sh_m[lane] : -INFINITY;
+    s = lane < kCeThreads / 32 ? sh_s[lane] : 0.0f;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1)
+      lse_merge(m, s, __shfl_xor_sync(0xffffffffu, m, off), __shfl_xor_sync(0xffffffffu, s, off));
+  }
+}
+
+// One block per row; V a multiple of 8 (16-byte vectors of bf16).
+__global__ void __launch_bounds__(kCeThreads)
+    ce_fwd_kernel(const uint4* __restrict__ logits, const int64_t* __restrict__ tgt, int64_t V,
+                  float* __restrict__ lse, float* __restrict__ row_loss) {
+  __shared__ float sh_m[kCeThreads / 32], sh_s[kCeThreads / 32];
+  const int64_t r = blockIdx.x;
+  const int64_t nv = V >> 3;
+  const uint4* row = logits + r * nv;
+  float m = -INFINITY, s = 0.0f;
+  // two vectors in flight per thread step
+  for (int64_t i = threadIdx.x; i < nv; i += 2 * kCeThreads) {
+    const bool two = i + kCeThreads < nv;
+    const uint4 va = __ldcs(row + i);
+    const uint4 vb = two ? __ldcs(row + i + kCeThreads) : va;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      if (h == 1 && !two) break;
+      const uint4 v = h ? vb : va;
+      const float f[8] = {bf16_lo(v.x), bf16_hi(v.x), bf16_lo(v.y), bf16_hi(v.y),
+                          bf16_lo(v.z), bf16_hi(v.z), bf16_lo(v.w), bf16_hi(v.w)};
+      float mv = f[0];
+#pragma unroll
+      for (int j = 1; j < 8; ++j) mv = fmaxf(mv, f[j]);
+      float sv = 0.0f;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) sv += expf(f[j] - mv);
+      lse_merge(m, s, mv, sv);
+    }
+  }
+  lse_block(m, s, sh_m, sh_s);
+  if (threadIdx.x == 0) {
+    const float l = m + logf(s);
+    const int64_t t = tgt[r];
+    const bool ok = t >= 0 && t < V;
+    const uint16_t xt = ok ? reinterpret_cast<const uint16_t*>(row)[t] : 0;
+    lse[r] = l;
+    row_loss[r] = ok ? l - __uint_as_float(static_cast<uint32_t>(xt) << 16) : 0.0f;
+  }
+}
+
+// One block per row; a row whose target is outside [0, V) gets zeros.
+__global__ void __launch_bounds__(kCeThreads)
+    ce_bwd_kernel(const uint4* __restrict__ logits, const int64_t* __restrict__ tgt,
+                  const float* __restrict__ lse, const float* __restrict__ scale, int64_t V,
+                  uint4* __restrict__ dlogits) {
+  const int64_t r = blockIdx.x;
+  const int64_t nv = V >> 3;
+  const int64_t t = tgt[r];
+  const bool ok = t >= 0 && t < V;
+  const float l = lse[r];
+  const float g = ok ? scale[0] : 0.0f;
+  const uint4* row = logits + r * nv;
+  uint4* drow = dlogits + r * nv;
+  // two vectors in flight per thread step
+  for (int64_t i0 = threadIdx.x; i0 < nv; i0 += 2 * kCeThreads) {
+    const bool two = i0 + kCeThreads < nv;
+    const uint4 va = __ldcs(row + i0);
+    const uint4 vb = two ? __ldcs(row + i0 + kCeThreads) : va;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      if (h == 1 && !two) break;
+      const int64_t i = i0 + h * kCeThreads;
+      const uint4 v = h ? vb : va;
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+      uint32_t o[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int64_t c = i * 8 + 2 * j;
+        const float p0 = expf(bf16_lo(w[j]) - l) - (c == t ? 1.0f : 0.0f);
+        const float p1 = expf(bf16_hi(w[j]) - l) - (c + 1 == t ? 1.0f : 0.0f);
+        o[j] = pack_bf16x2(p0 * g, p1 * g);
+      }
+      __stcs(drow + i, make_uint4(o[0], o[1], o[2], o[3]));
+    }
+  }
+}
+
+int grid_cap(int64_t items, int threads) {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int64_t b = (items + threads - 1) / threads;
+  const int64_t cap = static_cast<int64_t>(sms) * 8;
+  if (b > cap) b = cap;
+  return static_cast<int>(b < 1 ? 1 : b);
+}
+
+}  // namespace
+
+int launch_rope(const uint16_t* x, uint16_t* y, const float* cos_sin, int64_t rows, int64_t S,
+                int64_t H, int64_t D, bool inverse, cudaStream_t stream) {
+  const int64_t row_vecs = H * D / 8, head_vecs = D / 8;
+  const int64_t nvec = rows * row_vecs;
+  const int blocks = grid_cap(nvec, kRopeThreads);
+  auto* xv = reinterpret_cast<const uint4*>(x);
+  auto* yv = reinterpret_cast<uint4*>(y);
+  auto* cv = reinterpret_cast<const float4*>(cos_sin);
+  if (inverse)
+    rope_kernel<true><<<blocks, kRopeThreads, 0, stream>>>(xv, yv, cv, nvec, row_vecs, S, head_vecs);
+  else
+    rope_kernel<false><<<blocks, kRopeThreads, 0, stream>>>(xv, yv, cv, nvec, row_vecs, S, head_vecs);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+int launch_ce_fwd(const uint16_t* logits, const int64_t* targets, int64_t M, int64_t V,
+                  float* lse, float* row_loss, cudaStream_t stream) {
+  ce_fwd_kernel<<<static_cast<unsigned>(M), kCeThreads, 0, stream>>>(
+      reinterpret_cast<const uint4*>(logits), targets, V, lse, row_loss);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+int launch_ce_bwd(const uint16_t* logits, const int64_t* targets, const float* lse,
+                  const float* scale, int64_t M, int64_t V, uint16_t* dlogits,
+                  cudaStream_t stream) {
+  ce_bwd_kernel<<<static_cast<unsigned>(M), kCeThreads, 0, stream>>>(
+      reinterpret_cast<const uint4*>(logits), targets, lse, scale, V,
+      reinterpret_cast<uint4*>(dlogits));
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+}  // namespace dqt

@@ -178,6 +178,39 @@ int dqt_codes_to_bf16(const int8_t* W, int64_t numel, dqt_bf16* W_img, void* str
   return dqt::launch_codes_to_bf16(W, numel, W_img, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
+int dqt_rope_bf16(const dqt_bf16* x, dqt_bf16* y, const float* cos_sin, int64_t rows, int64_t S,
+                  int64_t H, int64_t D, int32_t inverse, void* stream) {
+  if (!x || !y || !cos_sin || rows <= 0 || S <= 0 || H <= 0 || D <= 0) return DQT_ERR_ARG;
+  if (inverse != 0 && inverse != 1) return DQT_ERR_ARG;
+  if (D % 8 != 0 || !aligned16(x) || !aligned16(y) || !aligned16(cos_sin)) return DQT_ERR_ALIGN;
+  if (rows > kMaxDim || S > kMaxDim || H > kMaxDim || D > kMaxDim || H * D > kMaxDim)
+    return DQT_ERR_RANGE;
+  return dqt::launch_rope(x, y, cos_sin, rows, S, H, D, inverse == 1, as_stream(stream))
+             ? DQT_ERR_CUDA
+             : DQT_OK;
+}
+
+int dqt_cross_entropy_fwd_bf16(const dqt_bf16* logits, const int64_t* targets, int64_t M,
+                               int64_t V, float* lse, float* row_loss, void* stream) {
+  if (!logits || !targets || !lse || !row_loss || M <= 0 || V <= 0) return DQT_ERR_ARG;
+  if (V % 8 != 0 || !aligned16(logits)) return DQT_ERR_ALIGN;
+  if (M > kMaxDim || V > kMaxDim) return DQT_ERR_RANGE;
+  return dqt::launch_ce_fwd(logits, targets, M, V, lse, row_loss, as_stream(stream))
+             ? DQT_ERR_CUDA
+             : DQT_OK;
+}
+
+int dqt_cross_entropy_bwd_bf16(const dqt_bf16* logits, const int64_t* targets, const float* lse,
+                               const float* scale, int64_t M, int64_t V, dqt_bf16* dlogits,
+                               void* stream) {
+  if (!logits || !targets || !lse || !scale || !dlogits || M <= 0 || V <= 0) return DQT_ERR_ARG;
+  if (V % 8 != 0 || !aligned16(logits) || !aligned16(dlogits)) return DQT_ERR_ALIGN;
+  if (M > kMaxDim || V > kMaxDim) return DQT_ERR_RANGE;
+  return dqt::launch_ce_bwd(logits, targets, lse, scale, M, V, dlogits, as_stream(stream))
+             ? DQT_ERR_CUDA
+             : DQT_OK;
+}
+
 int dqt_bitlinear_fwd(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img, float s_w,
                       dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
                       int32_t* acc_out, void* stream) {

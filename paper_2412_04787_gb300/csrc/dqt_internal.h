@@ -99,6 +99,15 @@ int launch_absmean_codes(const float* W0, int64_t numel, float s_w, int32_t qmin
                          int8_t* codes, cudaStream_t stream);
 constexpr int kAbsmeanBlocks = 1024;
 
+// Decoder support (rotary embedding, token cross-entropy): decoder_ops.cu.
+int launch_rope(const uint16_t* x, uint16_t* y, const float* cos_sin, int64_t rows, int64_t S,
+                int64_t H, int64_t D, bool inverse, cudaStream_t stream);
+int launch_ce_fwd(const uint16_t* logits, const int64_t* targets, int64_t M, int64_t V,
+                  float* lse, float* row_loss, cudaStream_t stream);
+int launch_ce_bwd(const uint16_t* logits, const int64_t* targets, const float* lse,
+                  const float* scale, int64_t M, int64_t V, uint16_t* dlogits,
+                  cudaStream_t stream);
+
 // 2-bit packed ternary codes (4 per byte): conversions and operand images.
 int launch_pack_ternary(const int8_t* c, int64_t n, uint8_t* out, cudaStream_t stream);
 int launch_unpack_ternary(const uint8_t* p, int64_t n, int8_t* c, cudaStream_t stream);

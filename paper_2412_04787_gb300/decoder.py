@@ -7,9 +7,11 @@ rounding (Sec. 3.2, Eq. 5).  Here q, k, v, o, gate, up and down are
 the FP8-environment forward of Sec. 4.3); the token
 embedding, the RMSNorm gains and the output head stay in bf16 and are trained
 by an ordinary optimiser (which weights the paper keeps in high precision is
-not stated; this is the BitNet convention).  RMSNorm, rotary position
-embedding, causal attention (``scaled_dot_product_attention``), SwiGLU and the
-cross-entropy loss are PyTorch operations around the BitLinear hot path.
+not stated; this is the BitNet convention).  RMSNorm, causal attention
+(``scaled_dot_product_attention``) and SwiGLU are PyTorch operations around
+the BitLinear hot path; the rotary position embedding and the token
+cross-entropy run on this library's decoder-support kernels (one bf16 pass
+each way with fp32 arithmetic, no fp32 copies of q, k or the logits).
 
 A training step is ``loss = model(ids, targets); loss.backward();
 opt.step(); opt.zero_grad()``: each BitLinear applies its DQT update during
@@ -23,6 +25,7 @@ stream-ordered before each replay).
 import torch
 import torch.nn.functional as F
 
+from . import dqt
 from .bitlinear import DQTBitLinear
 
 __all__ = ["DecoderConfig", "DQTDecoder"]
@@ -50,12 +53,38 @@ class RMSNorm(torch.nn.Module):
         return F.rms_norm(x, (x.shape[-1],), self.weight, self.eps)
 
 
-def _rope(x, freqs):
-    # rotary position embedding on interleaved pairs (x[2i], x[2i+1]) of the
-    # last dimension as one complex multiply, in fp32 (the LLaMA formulation);
-    # freqs: unit complex numbers broadcasting against x's pairs
-    xc = torch.view_as_complex(x.float().reshape(*x.shape[:-1], -1, 2))
-    return torch.view_as_real(xc * freqs).flatten(-2).to(x.dtype)
+class _Rope(torch.autograd.Function):
+    """Rotary position embedding (LLaMA form: interleaved pairs (x[2i], x[2i+1])
+    of each head times exp(i theta)) of x bf16 [B, S, H, D]; cos_sin fp32
+    [S, D/2, 2].  The backward rotates the gradient by -theta (the transpose)."""
+
+    @staticmethod
+    def forward(ctx, x, cos_sin):
+        ctx.save_for_backward(cos_sin)
+        return dqt.dqt_rope_bf16(x.contiguous(), cos_sin)
+
+    @staticmethod
+    def backward(ctx, g):
+        (cos_sin,) = ctx.saved_tensors
+        return dqt.dqt_rope_bf16(g.contiguous(), cos_sin, inverse=True), None
+
+
+class _TokenCrossEntropy(torch.autograd.Function):
+    """Mean token cross-entropy of bf16 logits [M, V] (log-sum-exp in fp32)
+    over the rows whose target lies in [0, V); the gradient is written in bf16."""
+
+    @staticmethod
+    def forward(ctx, logits, targets):
+        lse, row_loss = dqt.dqt_cross_entropy_fwd_bf16(logits, targets)
+        n = ((targets >= 0) & (targets < logits.shape[1])).sum().to(torch.float32)
+        ctx.save_for_backward(logits, targets, lse, n)
+        return row_loss.sum() / n
+
+    @staticmethod
+    def backward(ctx, g):
+        logits, targets, lse, n = ctx.saved_tensors
+        scale = (g.to(torch.float32) / n).reshape(1)
+        return dqt.dqt_cross_entropy_bwd_bf16(logits, targets, lse, scale), None
 
 
 class Block(torch.nn.Module):
@@ -75,16 +104,16 @@ class Block(torch.nn.Module):
         self.q, self.k, self.v, self.o = bl(h, h, 0), bl(h, h, 1), bl(h, h, 2), bl(h, h, 3)
         self.gate, self.up, self.down = bl(h, f, 4), bl(h, f, 5), bl(f, h, 6)
 
-    def forward(self, x, freqs):
+    def forward(self, x, cos_sin):
         B, S, Hd = x.shape
         nh = self.heads
         hd = Hd // nh
         a = self.attn_norm(x)
         # rotary embedding in the [B, S, H, D] layout the projections produce
-        # (freqs: [1, S, 1, D/2]); attention reads head-major views of it, so
+        # (cos_sin: [S, D/2, 2]); attention reads head-major views of it, so
         # no layout copy is made in either direction
-        q = _rope(self.q(a).view(B, S, nh, hd), freqs).transpose(1, 2)
-        k = _rope(self.k(a).view(B, S, nh, hd), freqs).transpose(1, 2)
+        q = _Rope.apply(self.q(a).view(B, S, nh, hd), cos_sin).transpose(1, 2)
+        k = _Rope.apply(self.k(a).view(B, S, nh, hd), cos_sin).transpose(1, 2)
         v = self.v(a).view(B, S, nh, hd).transpose(1, 2)
         o = F.scaled_dot_product_attention(q, k, v, is_causal=True)
         x = x + self.o(o.transpose(1, 2).reshape(B, S, Hd))
@@ -152,14 +181,15 @@ class DQTDecoder(torch.nn.Module):
         x = F.embedding(ids, self.embed)
         t = torch.arange(S, device=ids.device, dtype=torch.float32)
         ang = torch.outer(t, self.inv_freq)
-        freqs = torch.polar(torch.ones_like(ang), ang)[None, :, None, :]
+        cos_sin = torch.stack((torch.cos(ang), torch.sin(ang)), dim=-1)  # [S, D/2, 2]
         for blk in self.blocks:
-            x = blk(x, freqs)
+            x = blk(x, cos_sin)
         x = self.norm(x)
         logits = x @ self.head.t()
         if targets is None:
             return logits
-        return F.cross_entropy(logits.float().view(-1, logits.shape[-1]), targets.reshape(-1))
+        return _TokenCrossEntropy.apply(logits.view(-1, logits.shape[-1]),
+                                        targets.reshape(-1).to(torch.int64).contiguous())
 
     def bitlinear_flops_per_step(self, tokens):
         """Forward + dX + dW FLOPs of all BitLinear layers for `tokens` tokens."""

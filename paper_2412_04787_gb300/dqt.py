@@ -28,6 +28,7 @@ EXPORTED = [
     "dqt_sr_update_packed", "dqt_bitlinear_bwd_dw_update_packed",
     "dqt_adafactor_workspace_size", "dqt_adafactor_stats", "dqt_adafactor_apply",
     "dqt_bwd_dw_adafactor_workspace_size", "dqt_bitlinear_bwd_dw_adafactor",
+    "dqt_rope_bf16", "dqt_cross_entropy_fwd_bf16", "dqt_cross_entropy_bwd_bf16",
 ]
 
 
@@ -126,6 +127,9 @@ def lib():
                                                      C.POINTER(dqt_adafactor_t),
                                                      C.POINTER(dqt_sr_t), dqt_grid_t, _i64, _i64,
                                                      _i64, _vp, _vp, _sz, _vp]
+        L.dqt_rope_bf16.argtypes = [_vp, _vp, _vp, _i64, _i64, _i64, _i64, C.c_int32, _vp]
+        L.dqt_cross_entropy_fwd_bf16.argtypes = [_vp, _vp, _i64, _i64, _vp, _vp, _vp]
+        L.dqt_cross_entropy_bwd_bf16.argtypes = [_vp, _vp, _vp, _vp, _i64, _i64, _vp, _vp]
         for name in EXPORTED:
             if name not in ("dqt_status_string", "dqt_absmean_workspace_size",
                             "dqt_update_consts_size", "dqt_bwd_dw_workspace_size",
@@ -619,3 +623,50 @@ def dqt_bitlinear_bwd_dw_adafactor(dY, Xdq, W, s_w, R, C_, hp, sr, bits_or_grid,
         _ptr(dY), _ptr(Xdq), _ptr(W), int(packed), float(s_w), _ptr(R), _ptr(C_), C.byref(hp),
         C.byref(sr), _grid(bits_or_grid), T, N, K, _ptr(changed_out), _ptr(ws), ws.numel(),
         _stream(stream)), "dqt_bitlinear_bwd_dw_adafactor")
+
+
+# ---------------------------------------------------------------------------
+# decoder support (not part of the DQT method)
+# ---------------------------------------------------------------------------
+def dqt_rope_bf16(x, cos_sin, inverse=False, y=None, stream=None):
+    """Rotary embedding of x bf16 [B, S, H, D] (contiguous) with the (cos, sin)
+    table fp32 [S, D/2, 2]; inverse rotates by -theta.  Returns y (new unless given)."""
+    _need(x, "x", torch.bfloat16)
+    if x.dim() != 4:
+        raise ValueError("x must be [B, S, H, D]")
+    B, S, H, D = x.shape
+    _need(cos_sin, "cos_sin", torch.float32, (S, D // 2, 2))
+    y = torch.empty_like(x) if y is None else _need(y, "y", torch.bfloat16, x.shape)
+    _check(lib().dqt_rope_bf16(_ptr(x), _ptr(y), _ptr(cos_sin), B * S, S, H, D, int(bool(inverse)),
+                               _stream(stream)), "dqt_rope_bf16")
+    return y
+
+
+def dqt_cross_entropy_fwd_bf16(logits, targets, stream=None):
+    """Per-row log-sum-exp and loss of bf16 logits [M, V] against int64 targets
+    [M].  Returns (lse, row_loss), fp32 [M] each."""
+    _need(logits, "logits", torch.bfloat16)
+    M, V = logits.shape
+    _need(targets, "targets", torch.int64, (M,))
+    lse = torch.empty(M, dtype=torch.float32, device=logits.device)
+    row_loss = torch.empty(M, dtype=torch.float32, device=logits.device)
+    _check(lib().dqt_cross_entropy_fwd_bf16(_ptr(logits), _ptr(targets), M, V, _ptr(lse),
+                                            _ptr(row_loss), _stream(stream)),
+           "dqt_cross_entropy_fwd_bf16")
+    return lse, row_loss
+
+
+def dqt_cross_entropy_bwd_bf16(logits, targets, lse, scale, dlogits=None, stream=None):
+    """Gradient of the loss w.r.t. bf16 logits [M, V]: (softmax - onehot) * scale[0]
+    (scale: fp32 device tensor of one element)."""
+    _need(logits, "logits", torch.bfloat16)
+    M, V = logits.shape
+    _need(targets, "targets", torch.int64, (M,))
+    _need(lse, "lse", torch.float32, (M,))
+    _need(scale, "scale", torch.float32, (1,))
+    dlogits = torch.empty_like(logits) if dlogits is None else \
+        _need(dlogits, "dlogits", torch.bfloat16, (M, V))
+    _check(lib().dqt_cross_entropy_bwd_bf16(_ptr(logits), _ptr(targets), _ptr(lse), _ptr(scale), M,
+                                            V, _ptr(dlogits), _stream(stream)),
+           "dqt_cross_entropy_bwd_bf16")
+    return dlogits

@@ -166,3 +166,19 @@ def test_packed_and_adafactor_argument_validation(L):
                                  None) == dqt.DQT_ERR_ARG
     assert L.dqt_adafactor_apply(A, A, 0, A, A, A, 1, C.byref(sr), g, 64, 66, None,
                                  None) == dqt.DQT_ERR_ALIGN
+
+
+def test_decoder_support_argument_validation(L):
+    A = _p(0x10000)
+    # rotary embedding: D a multiple of 8, aligned pointers, inverse 0 or 1
+    assert L.dqt_rope_bf16(None, A, A, 4, 4, 2, 64, 0, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_rope_bf16(A, A, A, 0, 4, 2, 64, 0, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_rope_bf16(A, A, A, 4, 4, 2, 64, 2, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_rope_bf16(A, A, A, 4, 4, 2, 36, 0, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_rope_bf16(_p(0x10008), A, A, 4, 4, 2, 64, 0, None) == dqt.DQT_ERR_ALIGN
+    # cross-entropy: V a multiple of 8, outputs required
+    assert L.dqt_cross_entropy_fwd_bf16(A, A, 4, 36, A, A, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_cross_entropy_fwd_bf16(A, A, 4, 64, None, A, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_cross_entropy_fwd_bf16(A, A, 0, 64, A, A, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_cross_entropy_bwd_bf16(A, A, A, None, 4, 64, A, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_cross_entropy_bwd_bf16(A, A, A, A, 4, 64, _p(0x10004), None) == dqt.DQT_ERR_ALIGN
