@@ -398,6 +398,15 @@ int dqt_cross_entropy_bwd_bf16(const dqt_bf16* logits, const int64_t* targets, c
                                const float* scale, int64_t M, int64_t V, dqt_bf16* dlogits,
                                void* stream);
 
+/* SwiGLU gate of the decoder's MLP: h = silu(g) u = g sigmoid(g) u per
+ * element of bf16 g, u [n], evaluated in fp32 and rounded once to bf16.  Its
+ * backward, with s = sigmoid(g):  dg = dh u s (1 + g (1 - s)),  du = dh g s
+ * (fp32, each rounded once to bf16).  n a multiple of 8, every pointer 16-byte
+ * aligned, outputs not overlapping inputs. */
+int dqt_swiglu_bf16(const dqt_bf16* g, const dqt_bf16* u, dqt_bf16* h, int64_t n, void* stream);
+int dqt_swiglu_bwd_bf16(const dqt_bf16* g, const dqt_bf16* u, const dqt_bf16* dh, dqt_bf16* dg,
+                        dqt_bf16* du, int64_t n, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -9,6 +9,7 @@
 //                    times exp(i theta)), or by -theta for the backward
 //   ce_fwd_kernel    per row: lse = log sum_v exp(x_v), loss = lse - x_target
 //   ce_bwd_kernel    dx_v = (exp(x_v - lse) - [v == target]) * scale
+//   swiglu_kernel    h = silu(g) u, and its backward dg, du
 #include <cuda_bf16.h>
 
 #include "dqt_internal.h"
@@ -166,6 +167,62 @@ __global__ void __launch_bounds__(kCeThreads)
   }
 }
 
+constexpr int kEwThreads = 256;
+
+// SwiGLU gate: h = g sigmoid(g) u in fp32 per element, one rounding to bf16;
+// 8 elements (one 16-byte vector of each operand) per thread step.
+__global__ void __launch_bounds__(kEwThreads)
+    swiglu_kernel(const uint4* __restrict__ g, const uint4* __restrict__ u, uint4* __restrict__ h,
+                  int64_t nvec) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * kEwThreads;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * kEwThreads + threadIdx.x; i < nvec;
+       i += stride) {
+    const uint4 gv = __ldcs(g + i), uv = __ldcs(u + i);
+    const uint32_t gw[4] = {gv.x, gv.y, gv.z, gv.w}, uw[4] = {uv.x, uv.y, uv.z, uv.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float g0 = bf16_lo(gw[j]), g1 = bf16_hi(gw[j]);
+      const float s0 = 1.0f / (1.0f + expf(-g0)), s1 = 1.0f / (1.0f + expf(-g1));
+      o[j] = pack_bf16x2(g0 * s0 * bf16_lo(uw[j]), g1 * s1 * bf16_hi(uw[j]));
+    }
+    h[i] = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+// Its backward: with s = sigmoid(g),
+//   dg = dh u s (1 + g (1 - s)),   du = dh g s
+__global__ void __launch_bounds__(kEwThreads)
+    swiglu_bwd_kernel(const uint4* __restrict__ g, const uint4* __restrict__ u,
+                      const uint4* __restrict__ dh, uint4* __restrict__ dg,
+                      uint4* __restrict__ du, int64_t nvec) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * kEwThreads;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * kEwThreads + threadIdx.x; i < nvec;
+       i += stride) {
+    const uint4 gv = __ldcs(g + i), uv = __ldcs(u + i), hv = __ldcs(dh + i);
+    const uint32_t gw[4] = {gv.x, gv.y, gv.z, gv.w}, uw[4] = {uv.x, uv.y, uv.z, uv.w},
+                   hw[4] = {hv.x, hv.y, hv.z, hv.w};
+    uint32_t og[4], ou[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      float rg[2], ru[2];
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {
+        const float gg = k ? bf16_hi(gw[j]) : bf16_lo(gw[j]);
+        const float uu = k ? bf16_hi(uw[j]) : bf16_lo(uw[j]);
+        const float d = k ? bf16_hi(hw[j]) : bf16_lo(hw[j]);
+        const float s = 1.0f / (1.0f + expf(-gg));
+        rg[k] = d * uu * s * (1.0f + gg * (1.0f - s));
+        ru[k] = d * gg * s;
+      }
+      og[j] = pack_bf16x2(rg[0], rg[1]);
+      ou[j] = pack_bf16x2(ru[0], ru[1]);
+    }
+    __stcs(dg + i, make_uint4(og[0], og[1], og[2], og[3]));
+    __stcs(du + i, make_uint4(ou[0], ou[1], ou[2], ou[3]));
+  }
+}
+
 int grid_cap(int64_t items, int threads) {
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
@@ -206,6 +263,25 @@ int launch_ce_bwd(const uint16_t* logits, const int64_t* targets, const float* l
   ce_bwd_kernel<<<static_cast<unsigned>(M), kCeThreads, 0, stream>>>(
       reinterpret_cast<const uint4*>(logits), targets, lse, scale, V,
       reinterpret_cast<uint4*>(dlogits));
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+int launch_swiglu(const uint16_t* g, const uint16_t* u, uint16_t* h, int64_t n,
+                  cudaStream_t stream) {
+  const int64_t nvec = n / 8;
+  swiglu_kernel<<<grid_cap(nvec, kEwThreads), kEwThreads, 0, stream>>>(
+      reinterpret_cast<const uint4*>(g), reinterpret_cast<const uint4*>(u),
+      reinterpret_cast<uint4*>(h), nvec);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+int launch_swiglu_bwd(const uint16_t* g, const uint16_t* u, const uint16_t* dh, uint16_t* dg,
+                      uint16_t* du, int64_t n, cudaStream_t stream) {
+  const int64_t nvec = n / 8;
+  swiglu_bwd_kernel<<<grid_cap(nvec, kEwThreads), kEwThreads, 0, stream>>>(
+      reinterpret_cast<const uint4*>(g), reinterpret_cast<const uint4*>(u),
+      reinterpret_cast<const uint4*>(dh), reinterpret_cast<uint4*>(dg),
+      reinterpret_cast<uint4*>(du), nvec);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 

@@ -211,6 +211,21 @@ int dqt_cross_entropy_bwd_bf16(const dqt_bf16* logits, const int64_t* targets, c
              : DQT_OK;
 }
 
+int dqt_swiglu_bf16(const dqt_bf16* g, const dqt_bf16* u, dqt_bf16* h, int64_t n, void* stream) {
+  if (!g || !u || !h || n <= 0) return DQT_ERR_ARG;
+  if (n % 8 != 0 || !aligned16(g) || !aligned16(u) || !aligned16(h)) return DQT_ERR_ALIGN;
+  return dqt::launch_swiglu(g, u, h, n, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
+int dqt_swiglu_bwd_bf16(const dqt_bf16* g, const dqt_bf16* u, const dqt_bf16* dh, dqt_bf16* dg,
+                        dqt_bf16* du, int64_t n, void* stream) {
+  if (!g || !u || !dh || !dg || !du || n <= 0) return DQT_ERR_ARG;
+  if (n % 8 != 0 || !aligned16(g) || !aligned16(u) || !aligned16(dh) || !aligned16(dg) ||
+      !aligned16(du))
+    return DQT_ERR_ALIGN;
+  return dqt::launch_swiglu_bwd(g, u, dh, dg, du, n, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
 int dqt_bitlinear_fwd(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img, float s_w,
                       dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
                       int32_t* acc_out, void* stream) {

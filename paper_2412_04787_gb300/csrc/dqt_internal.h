@@ -107,6 +107,10 @@ int launch_ce_fwd(const uint16_t* logits, const int64_t* targets, int64_t M, int
 int launch_ce_bwd(const uint16_t* logits, const int64_t* targets, const float* lse,
                   const float* scale, int64_t M, int64_t V, uint16_t* dlogits,
                   cudaStream_t stream);
+int launch_swiglu(const uint16_t* g, const uint16_t* u, uint16_t* h, int64_t n,
+                  cudaStream_t stream);
+int launch_swiglu_bwd(const uint16_t* g, const uint16_t* u, const uint16_t* dh, uint16_t* dg,
+                      uint16_t* du, int64_t n, cudaStream_t stream);
 
 // 2-bit packed ternary codes (4 per byte): conversions and operand images.
 int launch_pack_ternary(const int8_t* c, int64_t n, uint8_t* out, cudaStream_t stream);

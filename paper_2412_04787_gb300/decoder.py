@@ -7,9 +7,9 @@ rounding (Sec. 3.2, Eq. 5).  Here q, k, v, o, gate, up and down are
 the FP8-environment forward of Sec. 4.3); the token
 embedding, the RMSNorm gains and the output head stay in bf16 and are trained
 by an ordinary optimiser (which weights the paper keeps in high precision is
-not stated; this is the BitNet convention).  RMSNorm, causal attention
-(``scaled_dot_product_attention``) and SwiGLU are PyTorch operations around
-the BitLinear hot path; the rotary position embedding and the token
+not stated; this is the BitNet convention).  RMSNorm and causal attention
+(``scaled_dot_product_attention``) are PyTorch operations around the BitLinear
+hot path; the rotary position embedding, the SwiGLU gate and the token
 cross-entropy run on this library's decoder-support kernels (one bf16 pass
 each way with fp32 arithmetic, no fp32 copies of q, k or the logits).
 
@@ -69,6 +69,21 @@ class _Rope(torch.autograd.Function):
         return dqt.dqt_rope_bf16(g.contiguous(), cos_sin, inverse=True), None
 
 
+class _SwiGLU(torch.autograd.Function):
+    """h = silu(g) * u of two bf16 tensors of one shape, in one pass each way."""
+
+    @staticmethod
+    def forward(ctx, g, u):
+        g, u = g.contiguous(), u.contiguous()
+        ctx.save_for_backward(g, u)
+        return dqt.dqt_swiglu_bf16(g, u)
+
+    @staticmethod
+    def backward(ctx, dh):
+        g, u = ctx.saved_tensors
+        return dqt.dqt_swiglu_bwd_bf16(g, u, dh.contiguous())
+
+
 class _TokenCrossEntropy(torch.autograd.Function):
     """Mean token cross-entropy of bf16 logits [M, V] (log-sum-exp in fp32)
     over the rows whose target lies in [0, V); the gradient is written in bf16."""
@@ -118,7 +133,7 @@ class Block(torch.nn.Module):
         o = F.scaled_dot_product_attention(q, k, v, is_causal=True)
         x = x + self.o(o.transpose(1, 2).reshape(B, S, Hd))
         m = self.mlp_norm(x)
-        return x + self.down(F.silu(self.gate(m)) * self.up(m))
+        return x + self.down(_SwiGLU.apply(self.gate(m), self.up(m)))
 
 
 class DQTDecoder(torch.nn.Module):

@@ -29,6 +29,7 @@ EXPORTED = [
     "dqt_adafactor_workspace_size", "dqt_adafactor_stats", "dqt_adafactor_apply",
     "dqt_bwd_dw_adafactor_workspace_size", "dqt_bitlinear_bwd_dw_adafactor",
     "dqt_rope_bf16", "dqt_cross_entropy_fwd_bf16", "dqt_cross_entropy_bwd_bf16",
+    "dqt_swiglu_bf16", "dqt_swiglu_bwd_bf16",
 ]
 
 
@@ -130,6 +131,8 @@ def lib():
         L.dqt_rope_bf16.argtypes = [_vp, _vp, _vp, _i64, _i64, _i64, _i64, C.c_int32, _vp]
         L.dqt_cross_entropy_fwd_bf16.argtypes = [_vp, _vp, _i64, _i64, _vp, _vp, _vp]
         L.dqt_cross_entropy_bwd_bf16.argtypes = [_vp, _vp, _vp, _vp, _i64, _i64, _vp, _vp]
+        L.dqt_swiglu_bf16.argtypes = [_vp, _vp, _vp, _i64, _vp]
+        L.dqt_swiglu_bwd_bf16.argtypes = [_vp, _vp, _vp, _vp, _vp, _i64, _vp]
         for name in EXPORTED:
             if name not in ("dqt_status_string", "dqt_absmean_workspace_size",
                             "dqt_update_consts_size", "dqt_bwd_dw_workspace_size",
@@ -670,3 +673,24 @@ def dqt_cross_entropy_bwd_bf16(logits, targets, lse, scale, dlogits=None, stream
                                             V, _ptr(dlogits), _stream(stream)),
            "dqt_cross_entropy_bwd_bf16")
     return dlogits
+
+
+def dqt_swiglu_bf16(g, u, h=None, stream=None):
+    """h = silu(g) * u (fp32 inside, one bf16 rounding); g, u contiguous bf16 of one shape."""
+    _need(g, "g", torch.bfloat16)
+    _need(u, "u", torch.bfloat16, g.shape)
+    h = torch.empty_like(g) if h is None else _need(h, "h", torch.bfloat16, g.shape)
+    _check(lib().dqt_swiglu_bf16(_ptr(g), _ptr(u), _ptr(h), g.numel(), _stream(stream)),
+           "dqt_swiglu_bf16")
+    return h
+
+
+def dqt_swiglu_bwd_bf16(g, u, dh, stream=None):
+    """(dg, du) of h = silu(g) * u for the upstream gradient dh."""
+    _need(g, "g", torch.bfloat16)
+    _need(u, "u", torch.bfloat16, g.shape)
+    _need(dh, "dh", torch.bfloat16, g.shape)
+    dg, du = torch.empty_like(g), torch.empty_like(g)
+    _check(lib().dqt_swiglu_bwd_bf16(_ptr(g), _ptr(u), _ptr(dh), _ptr(dg), _ptr(du), g.numel(),
+                                     _stream(stream)), "dqt_swiglu_bwd_bf16")
+    return dg, du

@@ -182,3 +182,8 @@ def test_decoder_support_argument_validation(L):
     assert L.dqt_cross_entropy_fwd_bf16(A, A, 0, 64, A, A, None) == dqt.DQT_ERR_ARG
     assert L.dqt_cross_entropy_bwd_bf16(A, A, A, None, 4, 64, A, None) == dqt.DQT_ERR_ARG
     assert L.dqt_cross_entropy_bwd_bf16(A, A, A, A, 4, 64, _p(0x10004), None) == dqt.DQT_ERR_ALIGN
+    # SwiGLU: n a multiple of 8, every pointer aligned
+    assert L.dqt_swiglu_bf16(A, A, None, 64, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_swiglu_bf16(A, A, A, 12, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_swiglu_bwd_bf16(A, A, A, A, _p(0x10002), 64, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_swiglu_bwd_bf16(A, A, A, A, A, 0, None) == dqt.DQT_ERR_ARG

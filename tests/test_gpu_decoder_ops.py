@@ -106,3 +106,25 @@ def test_cross_entropy_row_values():
     expect = float(torch.log(torch.tensor(7.0 + torch.exp(torch.tensor(x1)).item())))
     assert abs(lse.item() - expect) <= 1e-6
     assert abs(loss.item() - (expect - x1)) <= 1e-6
+
+
+@pytest.mark.parametrize("shape", [(8,), (3, 40), (64, 5632)])
+def test_swiglu_matches_fp64(shape):
+    from paper_2412_04787_gb300.decoder import _SwiGLU
+    g = inputs.normal(shape, 2.0, seed=1, dtype=torch.bfloat16).cuda().requires_grad_()
+    u = inputs.normal(shape, 1.0, seed=2, dtype=torch.bfloat16).cuda().requires_grad_()
+    dh = inputs.normal(shape, 1.0, seed=3, dtype=torch.bfloat16).cuda()
+    h = _SwiGLU.apply(g, u)
+    h.backward(dh)
+    gd, ud, hd = g.detach().double(), u.detach().double(), dh.double()
+    s = torch.sigmoid(gd)
+    ref_h = gd * s * ud
+    ref_dg = hd * ud * s * (1 + gd * (1 - s))
+    ref_du = hd * gd * s
+    # one rounding of an fp32 evaluation to bf16: within one bf16 ulp
+    for got, ref in ((h, ref_h), (g.grad, ref_dg), (u.grad, ref_du)):
+        err = (got.double() - ref).abs()
+        assert (err <= 2 ** -7 * ref.abs() + 1e-30).all()
+    # and close to PyTorch's own silu(g) * u (which rounds silu(g) to bf16 first)
+    ref_t = F.silu(g.detach()) * u.detach()
+    assert ((h.float() - ref_t.float()).abs() <= 2 ** -6 * ref_t.float().abs() + 1e-30).all()
