@@ -18,6 +18,10 @@
  *   dqt_*packed*                  2-bit packed ternary code storage (Sec. 1)
  *   dqt_*adafactor*               Adafactor with SR instead of AdamW (Sec. 4.3)
  *
+ * and, not part of the method, three operations of the LLaMA-structured decoder
+ * (the model family of Sec. 4.1) built around those layers: dqt_rope_bf16,
+ * dqt_swiglu_bf16 / dqt_swiglu_bwd_bf16, dqt_cross_entropy_fwd_bf16 / _bwd_bf16.
+ *
  * GB300 has no int8 tensor-core MMA for sm_103a, so the integer GEMMs run on
  * the bf16 tensor cores over exact bf16 images of the integer codes (every
  * integer in [-256, 256] is exact in bf16; products and partial sums below
