@@ -18,9 +18,10 @@
  *   dqt_*packed*                  2-bit packed ternary code storage (Sec. 1)
  *   dqt_*adafactor*               Adafactor with SR instead of AdamW (Sec. 4.3)
  *
- * and, not part of the method, three operations of the LLaMA-structured decoder
+ * and, not part of the method, four operations of the LLaMA-structured decoder
  * (the model family of Sec. 4.1) built around those layers: dqt_rope_bf16,
- * dqt_swiglu_bf16 / dqt_swiglu_bwd_bf16, dqt_cross_entropy_fwd_bf16 / _bwd_bf16.
+ * dqt_swiglu_bf16 / dqt_swiglu_bwd_bf16, dqt_rmsnorm_bf16 / dqt_rmsnorm_bwd_bf16,
+ * dqt_cross_entropy_fwd_bf16 / _bwd_bf16.
  *
  * GB300 has no int8 tensor-core MMA for sm_103a, so the integer GEMMs run on
  * the bf16 tensor cores over exact bf16 images of the integer codes (every
@@ -410,6 +411,25 @@ int dqt_cross_entropy_bwd_bf16(const dqt_bf16* logits, const int64_t* targets, c
 int dqt_swiglu_bf16(const dqt_bf16* g, const dqt_bf16* u, dqt_bf16* h, int64_t n, void* stream);
 int dqt_swiglu_bwd_bf16(const dqt_bf16* g, const dqt_bf16* u, const dqt_bf16* dh, dqt_bf16* dg,
                         dqt_bf16* du, int64_t n, void* stream);
+
+/* RMSNorm of the decoder: per row of x bf16 [rows, D],
+ *   rstd = 1 / sqrt(mean_j x_j^2 + eps),   y_j = x_j rstd w_j
+ * in fp32, y rounded once to bf16; rstd fp32 [rows] is kept for the backward.
+ * D a multiple of 8 and at most 2048 (DQT_ERR_RANGE beyond); x, w, y 16-byte
+ * aligned. */
+int dqt_rmsnorm_bf16(const dqt_bf16* x, const dqt_bf16* w, float eps, int64_t rows, int64_t D,
+                     dqt_bf16* y, float* rstd, void* stream);
+/* Its backward for the upstream gradient dy [rows, D]:
+ *   dx_j = rstd w_j dy_j - x_j rstd^3 (1/D) sum_k w_k dy_k x_k   (bf16 [rows, D])
+ *   dw_j = sum over rows of dy_j x_j rstd                        (bf16 [D])
+ * dw is summed in a fixed order (per-warp partial sums in the workspace, then
+ * a column reduction), so it is deterministic.  Workspace:
+ * dqt_rmsnorm_bwd_workspace_size(rows, D) bytes for the current device,
+ * 16-byte aligned. */
+size_t dqt_rmsnorm_bwd_workspace_size(int64_t rows, int64_t D);
+int dqt_rmsnorm_bwd_bf16(const dqt_bf16* x, const dqt_bf16* w, const float* rstd,
+                         const dqt_bf16* dy, int64_t rows, int64_t D, dqt_bf16* dx, dqt_bf16* dw,
+                         void* ws, size_t ws_bytes, void* stream);
 
 #ifdef __cplusplus
 }

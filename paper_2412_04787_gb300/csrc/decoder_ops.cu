@@ -10,6 +10,9 @@
 //   ce_fwd_kernel    per row: lse = log sum_v exp(x_v), loss = lse - x_target
 //   ce_bwd_kernel    dx_v = (exp(x_v - lse) - [v == target]) * scale
 //   swiglu_kernel    h = silu(g) u, and its backward dg, du
+//   rmsnorm_*        y = x rstd w with rstd = 1 / sqrt(mean(x^2) + eps) per
+//                    row, and its backward (dx per row; dw as per-warp partial
+//                    sums reduced in a fixed order)
 #include <cuda_bf16.h>
 
 #include "dqt_internal.h"
@@ -223,6 +226,154 @@ __global__ void __launch_bounds__(kEwThreads)
   }
 }
 
+constexpr int kNormWarps = 8;  // rows per block, one warp per row
+
+// One warp per row; the row's D / 8 vectors are spread over the lanes,
+// VPL = ceil(D / 256) vectors per lane held in registers.
+template <int VPL>
+__global__ void __launch_bounds__(32 * kNormWarps)
+    rmsnorm_fwd_kernel(const uint4* __restrict__ x, const uint4* __restrict__ w, float eps,
+                       int64_t rows, int nv, uint4* __restrict__ y, float* __restrict__ rstd) {
+  const int lane = threadIdx.x & 31;
+  const int64_t row = static_cast<int64_t>(blockIdx.x) * kNormWarps + (threadIdx.x >> 5);
+  if (row >= rows) return;
+  const uint4* xr = x + row * nv;
+  uint4 xv[VPL];
+  float ss = 0.0f;
+#pragma unroll
+  for (int k = 0; k < VPL; ++k) {
+    const int c = lane + 32 * k;
+    xv[k] = c < nv ? __ldcs(xr + c) : make_uint4(0, 0, 0, 0);
+    const uint32_t a[4] = {xv[k].x, xv[k].y, xv[k].z, xv[k].w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float lo = bf16_lo(a[j]), hi = bf16_hi(a[j]);
+      ss += lo * lo + hi * hi;
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+  const float r = 1.0f / sqrtf(ss / static_cast<float>(nv * 8) + eps);
+  if (lane == 0) rstd[row] = r;
+  uint4* yr = y + row * nv;
+#pragma unroll
+  for (int k = 0; k < VPL; ++k) {
+    const int c = lane + 32 * k;
+    if (c >= nv) break;
+    const uint4 wv = __ldg(w + c);
+    const uint32_t a[4] = {xv[k].x, xv[k].y, xv[k].z, xv[k].w};
+    const uint32_t b[4] = {wv.x, wv.y, wv.z, wv.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      o[j] = pack_bf16x2(bf16_lo(a[j]) * r * bf16_lo(b[j]), bf16_hi(a[j]) * r * bf16_hi(b[j]));
+    yr[c] = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+// Backward of y = x r w, r = rstd:
+//   dx_j = r w_j dy_j - x_j r^3 (1/D) sum_k w_k dy_k x_k
+//   dw_j = sum over rows of dy_j x_j r
+// Each warp walks rows warp_id, warp_id + nwarps, ... and keeps its dw
+// partial sums in registers; they go to part[warp_id, :] (fp32) at the end.
+template <int VPL>
+__global__ void __launch_bounds__(32 * kNormWarps)
+    rmsnorm_bwd_kernel(const uint4* __restrict__ x, const uint4* __restrict__ w,
+                       const float* __restrict__ rstd, const uint4* __restrict__ dy, int64_t rows,
+                       int nv, uint4* __restrict__ dx, float* __restrict__ part) {
+  const int lane = threadIdx.x & 31;
+  const int64_t wid = static_cast<int64_t>(blockIdx.x) * kNormWarps + (threadIdx.x >> 5);
+  const int64_t nwarps = static_cast<int64_t>(gridDim.x) * kNormWarps;
+  const float inv_d = 1.0f / static_cast<float>(nv * 8);
+  // the gain vector is re-read per row from L1 (it is D * 2 bytes) rather
+  // than held in registers next to the partial sums
+  float acc[VPL][8];
+#pragma unroll
+  for (int k = 0; k < VPL; ++k)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[k][j] = 0.0f;
+  for (int64_t row = wid; row < rows; row += nwarps) {
+    const float r = rstd[row];
+    uint4 xv[VPL], gv[VPL];
+    float dot = 0.0f;
+#pragma unroll
+    for (int k = 0; k < VPL; ++k) {
+      const int c = lane + 32 * k;
+      xv[k] = c < nv ? __ldcs(x + row * nv + c) : make_uint4(0, 0, 0, 0);
+      gv[k] = c < nv ? __ldcs(dy + row * nv + c) : make_uint4(0, 0, 0, 0);
+      const uint4 wv = c < nv ? __ldg(w + c) : make_uint4(0, 0, 0, 0);
+      const uint32_t a[4] = {xv[k].x, xv[k].y, xv[k].z, xv[k].w};
+      const uint32_t g[4] = {gv[k].x, gv[k].y, gv[k].z, gv[k].w};
+      const uint32_t b[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        dot += bf16_lo(b[j]) * bf16_lo(g[j]) * bf16_lo(a[j]);
+        dot += bf16_hi(b[j]) * bf16_hi(g[j]) * bf16_hi(a[j]);
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+    const float coef = r * r * r * dot * inv_d;
+#pragma unroll
+    for (int k = 0; k < VPL; ++k) {
+      const int c = lane + 32 * k;
+      if (c >= nv) break;
+      const uint4 wv = __ldg(w + c);
+      const uint32_t a[4] = {xv[k].x, xv[k].y, xv[k].z, xv[k].w};
+      const uint32_t g[4] = {gv[k].x, gv[k].y, gv[k].z, gv[k].w};
+      const uint32_t b[4] = {wv.x, wv.y, wv.z, wv.w};
+      uint32_t o[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float x0 = bf16_lo(a[j]), x1 = bf16_hi(a[j]);
+        const float g0 = bf16_lo(g[j]), g1 = bf16_hi(g[j]);
+        o[j] = pack_bf16x2(r * bf16_lo(b[j]) * g0 - x0 * coef, r * bf16_hi(b[j]) * g1 - x1 * coef);
+        acc[k][2 * j] += g0 * x0 * r;
+        acc[k][2 * j + 1] += g1 * x1 * r;
+      }
+      __stcs(dx + row * nv + c, make_uint4(o[0], o[1], o[2], o[3]));
+    }
+  }
+  float* pr = part + wid * static_cast<int64_t>(nv) * 8;
+#pragma unroll
+  for (int k = 0; k < VPL; ++k) {
+    const int c = lane + 32 * k;
+    if (c >= nv) break;
+    float4* d = reinterpret_cast<float4*>(pr + c * 8);
+    d[0] = make_float4(acc[k][0], acc[k][1], acc[k][2], acc[k][3]);
+    d[1] = make_float4(acc[k][4], acc[k][5], acc[k][6], acc[k][7]);
+  }
+}
+
+// dw_j = the sum of the P partial rows, rounded once to bf16, in a fixed
+// order: a block covers 32 columns, warp k sums the partial rows p = k mod 8
+// in increasing p, and the block adds the 8 warp sums in warp order.
+__global__ void __launch_bounds__(256)
+    rmsnorm_dw_kernel(const float* __restrict__ part, int64_t P, int D, uint16_t* __restrict__ dw) {
+  __shared__ float sh[8][33];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int col = blockIdx.x * 32 + lane;
+  float s = 0.0f;
+  if (col < D)
+    for (int64_t p = warp; p < P; p += 8) s += part[p * D + col];
+  sh[warp][lane] = s;
+  __syncthreads();
+  if (warp == 0 && col < D) {
+    float t = 0.0f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) t += sh[k][lane];
+    const __nv_bfloat16 h = __float2bfloat16_rn(t);
+    dw[col] = *reinterpret_cast<const uint16_t*>(&h);
+  }
+}
+
+int norm_blocks_bwd() {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  return sms;  // one block (8 warps) per SM: the partial sums take many registers
+}
+
 int grid_cap(int64_t items, int threads) {
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
@@ -283,6 +434,68 @@ int launch_swiglu_bwd(const uint16_t* g, const uint16_t* u, const uint16_t* dh, 
       reinterpret_cast<const uint4*>(dh), reinterpret_cast<uint4*>(dg),
       reinterpret_cast<uint4*>(du), nvec);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+size_t rmsnorm_bwd_ws(int64_t rows, int64_t D) {
+  const int64_t blocks = norm_blocks_bwd();
+  const int64_t need = (rows + kNormWarps - 1) / kNormWarps;
+  const int64_t b = blocks < need ? blocks : need;
+  return static_cast<size_t>(b * kNormWarps * D) * sizeof(float);
+}
+
+template <int VPL>
+static int rms_launch(const uint16_t* x, const uint16_t* w, float eps, int64_t rows, int64_t D,
+                      uint16_t* y, float* rstd, cudaStream_t stream) {
+  const int nv = static_cast<int>(D / 8);
+  const unsigned blocks = static_cast<unsigned>((rows + kNormWarps - 1) / kNormWarps);
+  rmsnorm_fwd_kernel<VPL><<<blocks, 32 * kNormWarps, 0, stream>>>(
+      reinterpret_cast<const uint4*>(x), reinterpret_cast<const uint4*>(w), eps, rows, nv,
+      reinterpret_cast<uint4*>(y), rstd);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+template <int VPL>
+static int rms_bwd_launch(const uint16_t* x, const uint16_t* w, const float* rstd,
+                          const uint16_t* dy, int64_t rows, int64_t D, uint16_t* dx,
+                          uint16_t* dw, float* part, cudaStream_t stream) {
+  const int nv = static_cast<int>(D / 8);
+  const int64_t need = (rows + kNormWarps - 1) / kNormWarps;
+  const int64_t sms = norm_blocks_bwd();
+  const unsigned blocks = static_cast<unsigned>(sms < need ? sms : need);
+  rmsnorm_bwd_kernel<VPL><<<blocks, 32 * kNormWarps, 0, stream>>>(
+      reinterpret_cast<const uint4*>(x), reinterpret_cast<const uint4*>(w), rstd,
+      reinterpret_cast<const uint4*>(dy), rows, nv, reinterpret_cast<uint4*>(dx), part);
+  const int64_t P = static_cast<int64_t>(blocks) * kNormWarps;
+  rmsnorm_dw_kernel<<<static_cast<unsigned>((D + 31) / 32), 256, 0, stream>>>(
+      part, P, static_cast<int>(D), dw);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+int launch_rmsnorm(const uint16_t* x, const uint16_t* w, float eps, int64_t rows, int64_t D,
+                   uint16_t* y, float* rstd, cudaStream_t stream) {
+  switch ((D / 8 + 31) / 32) {
+    case 1: return rms_launch<1>(x, w, eps, rows, D, y, rstd, stream);
+    case 2: return rms_launch<2>(x, w, eps, rows, D, y, rstd, stream);
+    case 3: return rms_launch<3>(x, w, eps, rows, D, y, rstd, stream);
+    case 4: return rms_launch<4>(x, w, eps, rows, D, y, rstd, stream);
+    case 5: case 6: return rms_launch<6>(x, w, eps, rows, D, y, rstd, stream);
+    case 7: case 8: return rms_launch<8>(x, w, eps, rows, D, y, rstd, stream);
+    default: return 1;
+  }
+}
+
+int launch_rmsnorm_bwd(const uint16_t* x, const uint16_t* w, const float* rstd,
+                       const uint16_t* dy, int64_t rows, int64_t D, uint16_t* dx, uint16_t* dw,
+                       float* part, cudaStream_t stream) {
+  switch ((D / 8 + 31) / 32) {
+    case 1: return rms_bwd_launch<1>(x, w, rstd, dy, rows, D, dx, dw, part, stream);
+    case 2: return rms_bwd_launch<2>(x, w, rstd, dy, rows, D, dx, dw, part, stream);
+    case 3: return rms_bwd_launch<3>(x, w, rstd, dy, rows, D, dx, dw, part, stream);
+    case 4: return rms_bwd_launch<4>(x, w, rstd, dy, rows, D, dx, dw, part, stream);
+    case 5: case 6: return rms_bwd_launch<6>(x, w, rstd, dy, rows, D, dx, dw, part, stream);
+    case 7: case 8: return rms_bwd_launch<8>(x, w, rstd, dy, rows, D, dx, dw, part, stream);
+    default: return 1;
+  }
 }
 
 }  // namespace dqt

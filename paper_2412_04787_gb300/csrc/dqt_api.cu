@@ -226,6 +226,35 @@ int dqt_swiglu_bwd_bf16(const dqt_bf16* g, const dqt_bf16* u, const dqt_bf16* dh
   return dqt::launch_swiglu_bwd(g, u, dh, dg, du, n, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
+int dqt_rmsnorm_bf16(const dqt_bf16* x, const dqt_bf16* w, float eps, int64_t rows, int64_t D,
+                     dqt_bf16* y, float* rstd, void* stream) {
+  if (!x || !w || !y || !rstd || rows <= 0 || D <= 0 || !(eps >= 0.0f)) return DQT_ERR_ARG;
+  if (D % 8 != 0 || !aligned16(x) || !aligned16(w) || !aligned16(y)) return DQT_ERR_ALIGN;
+  if (D > 2048 || rows > kMaxDim) return DQT_ERR_RANGE;
+  return dqt::launch_rmsnorm(x, w, eps, rows, D, y, rstd, as_stream(stream)) ? DQT_ERR_CUDA
+                                                                              : DQT_OK;
+}
+
+size_t dqt_rmsnorm_bwd_workspace_size(int64_t rows, int64_t D) {
+  if (rows <= 0 || D <= 0 || D > 2048 || rows > kMaxDim) return 0;
+  return dqt::rmsnorm_bwd_ws(rows, D);
+}
+
+int dqt_rmsnorm_bwd_bf16(const dqt_bf16* x, const dqt_bf16* w, const float* rstd,
+                         const dqt_bf16* dy, int64_t rows, int64_t D, dqt_bf16* dx, dqt_bf16* dw,
+                         void* ws, size_t ws_bytes, void* stream) {
+  if (!x || !w || !rstd || !dy || !dx || !dw || !ws || rows <= 0 || D <= 0) return DQT_ERR_ARG;
+  if (D % 8 != 0 || !aligned16(x) || !aligned16(w) || !aligned16(dy) || !aligned16(dx) ||
+      !aligned16(ws))
+    return DQT_ERR_ALIGN;
+  if (D > 2048 || rows > kMaxDim) return DQT_ERR_RANGE;
+  if (ws_bytes < dqt::rmsnorm_bwd_ws(rows, D)) return DQT_ERR_ARG;
+  return dqt::launch_rmsnorm_bwd(x, w, rstd, dy, rows, D, dx, dw, static_cast<float*>(ws),
+                                 as_stream(stream))
+             ? DQT_ERR_CUDA
+             : DQT_OK;
+}
+
 int dqt_bitlinear_fwd(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img, float s_w,
                       dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
                       int32_t* acc_out, void* stream) {

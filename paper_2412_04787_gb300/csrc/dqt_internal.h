@@ -111,6 +111,12 @@ int launch_swiglu(const uint16_t* g, const uint16_t* u, uint16_t* h, int64_t n,
                   cudaStream_t stream);
 int launch_swiglu_bwd(const uint16_t* g, const uint16_t* u, const uint16_t* dh, uint16_t* dg,
                       uint16_t* du, int64_t n, cudaStream_t stream);
+int launch_rmsnorm(const uint16_t* x, const uint16_t* w, float eps, int64_t rows, int64_t D,
+                   uint16_t* y, float* rstd, cudaStream_t stream);
+size_t rmsnorm_bwd_ws(int64_t rows, int64_t D);
+int launch_rmsnorm_bwd(const uint16_t* x, const uint16_t* w, const float* rstd,
+                       const uint16_t* dy, int64_t rows, int64_t D, uint16_t* dx, uint16_t* dw,
+                       float* part, cudaStream_t stream);
 
 // 2-bit packed ternary codes (4 per byte): conversions and operand images.
 int launch_pack_ternary(const int8_t* c, int64_t n, uint8_t* out, cudaStream_t stream);

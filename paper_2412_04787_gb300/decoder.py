@@ -7,11 +7,11 @@ rounding (Sec. 3.2, Eq. 5).  Here q, k, v, o, gate, up and down are
 the FP8-environment forward of Sec. 4.3); the token
 embedding, the RMSNorm gains and the output head stay in bf16 and are trained
 by an ordinary optimiser (which weights the paper keeps in high precision is
-not stated; this is the BitNet convention).  RMSNorm and causal attention
-(``scaled_dot_product_attention``) are PyTorch operations around the BitLinear
-hot path; the rotary position embedding, the SwiGLU gate and the token
-cross-entropy run on this library's decoder-support kernels (one bf16 pass
-each way with fp32 arithmetic, no fp32 copies of q, k or the logits).
+not stated; this is the BitNet convention).  Causal attention
+(``scaled_dot_product_attention``) is a PyTorch operation around the BitLinear
+hot path; RMSNorm, the rotary position embedding, the SwiGLU gate and the
+token cross-entropy run on this library's decoder-support kernels (one bf16
+pass each way with fp32 arithmetic, no fp32 copies of q, k or the logits).
 
 A training step is ``loss = model(ids, targets); loss.backward();
 opt.step(); opt.zero_grad()``: each BitLinear applies its DQT update during
@@ -48,9 +48,30 @@ class RMSNorm(torch.nn.Module):
         self.weight = torch.nn.Parameter(torch.ones(dim, device=device, dtype=torch.bfloat16))
 
     def forward(self, x):
-        # PyTorch's fused RMSNorm (statistics in fp32 for the bf16 input): one
-        # kernel each way instead of a chain of fp32 elementwise ops
-        return F.rms_norm(x, (x.shape[-1],), self.weight, self.eps)
+        D = x.shape[-1]
+        if D % 8 == 0 and D <= 2048:
+            return _RMSNorm.apply(x, self.weight, self.eps)
+        # wider rows: PyTorch's fused RMSNorm (statistics in fp32)
+        return F.rms_norm(x, (D,), self.weight, self.eps)
+
+
+class _RMSNorm(torch.autograd.Function):
+    """RMSNorm of bf16 rows (statistics and products in fp32) on the library's
+    kernels: one pass forward; backward one pass for dx plus a fixed-order
+    column reduction for the gain gradient."""
+
+    @staticmethod
+    def forward(ctx, x, w, eps):
+        x2 = x.reshape(-1, x.shape[-1]).contiguous()
+        y, rstd = dqt.dqt_rmsnorm_bf16(x2, w, eps)
+        ctx.save_for_backward(x2, w, rstd)
+        return y.view(x.shape)
+
+    @staticmethod
+    def backward(ctx, dy):
+        x2, w, rstd = ctx.saved_tensors
+        dx, dw = dqt.dqt_rmsnorm_bwd_bf16(x2, w, rstd, dy.reshape(x2.shape).contiguous())
+        return dx.view(dy.shape), dw, None
 
 
 class _Rope(torch.autograd.Function):

@@ -29,7 +29,8 @@ EXPORTED = [
     "dqt_adafactor_workspace_size", "dqt_adafactor_stats", "dqt_adafactor_apply",
     "dqt_bwd_dw_adafactor_workspace_size", "dqt_bitlinear_bwd_dw_adafactor",
     "dqt_rope_bf16", "dqt_cross_entropy_fwd_bf16", "dqt_cross_entropy_bwd_bf16",
-    "dqt_swiglu_bf16", "dqt_swiglu_bwd_bf16",
+    "dqt_swiglu_bf16", "dqt_swiglu_bwd_bf16", "dqt_rmsnorm_bf16",
+    "dqt_rmsnorm_bwd_workspace_size", "dqt_rmsnorm_bwd_bf16",
 ]
 
 
@@ -133,11 +134,17 @@ def lib():
         L.dqt_cross_entropy_bwd_bf16.argtypes = [_vp, _vp, _vp, _vp, _i64, _i64, _vp, _vp]
         L.dqt_swiglu_bf16.argtypes = [_vp, _vp, _vp, _i64, _vp]
         L.dqt_swiglu_bwd_bf16.argtypes = [_vp, _vp, _vp, _vp, _vp, _i64, _vp]
+        L.dqt_rmsnorm_bf16.argtypes = [_vp, _vp, _f32, _i64, _i64, _vp, _vp, _vp]
+        L.dqt_rmsnorm_bwd_workspace_size.argtypes = [_i64, _i64]
+        L.dqt_rmsnorm_bwd_workspace_size.restype = _sz
+        L.dqt_rmsnorm_bwd_bf16.argtypes = [_vp, _vp, _vp, _vp, _i64, _i64, _vp, _vp, _vp, _sz,
+                                           _vp]
         for name in EXPORTED:
             if name not in ("dqt_status_string", "dqt_absmean_workspace_size",
                             "dqt_update_consts_size", "dqt_bwd_dw_workspace_size",
                             "dqt_adafactor_workspace_size",
-                            "dqt_bwd_dw_adafactor_workspace_size"):
+                            "dqt_bwd_dw_adafactor_workspace_size",
+                            "dqt_rmsnorm_bwd_workspace_size"):
                 getattr(L, name).restype = C.c_int
         _lib = L
     return _lib
@@ -694,3 +701,32 @@ def dqt_swiglu_bwd_bf16(g, u, dh, stream=None):
     _check(lib().dqt_swiglu_bwd_bf16(_ptr(g), _ptr(u), _ptr(dh), _ptr(dg), _ptr(du), g.numel(),
                                      _stream(stream)), "dqt_swiglu_bwd_bf16")
     return dg, du
+
+
+def dqt_rmsnorm_bf16(x, w, eps, stream=None):
+    """RMSNorm of x bf16 [rows, D] with gain w bf16 [D].  Returns (y, rstd)."""
+    _need(x, "x", torch.bfloat16)
+    rows, D = x.shape
+    _need(w, "w", torch.bfloat16, (D,))
+    y = torch.empty_like(x)
+    rstd = torch.empty(rows, dtype=torch.float32, device=x.device)
+    _check(lib().dqt_rmsnorm_bf16(_ptr(x), _ptr(w), float(eps), rows, D, _ptr(y), _ptr(rstd),
+                                  _stream(stream)), "dqt_rmsnorm_bf16")
+    return y, rstd
+
+
+def dqt_rmsnorm_bwd_bf16(x, w, rstd, dy, stream=None):
+    """(dx, dw) of the RMSNorm above for the upstream gradient dy [rows, D]."""
+    _need(x, "x", torch.bfloat16)
+    rows, D = x.shape
+    _need(w, "w", torch.bfloat16, (D,))
+    _need(rstd, "rstd", torch.float32, (rows,))
+    _need(dy, "dy", torch.bfloat16, (rows, D))
+    dx = torch.empty_like(x)
+    dw = torch.empty_like(w)
+    nws = lib().dqt_rmsnorm_bwd_workspace_size(rows, D)
+    ws = torch.empty(max(nws, 16), dtype=torch.uint8, device=x.device)
+    _check(lib().dqt_rmsnorm_bwd_bf16(_ptr(x), _ptr(w), _ptr(rstd), _ptr(dy), rows, D, _ptr(dx),
+                                      _ptr(dw), _ptr(ws), nws, _stream(stream)),
+           "dqt_rmsnorm_bwd_bf16")
+    return dx, dw

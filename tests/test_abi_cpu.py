@@ -187,3 +187,9 @@ def test_decoder_support_argument_validation(L):
     assert L.dqt_swiglu_bf16(A, A, A, 12, None) == dqt.DQT_ERR_ALIGN
     assert L.dqt_swiglu_bwd_bf16(A, A, A, A, _p(0x10002), 64, None) == dqt.DQT_ERR_ALIGN
     assert L.dqt_swiglu_bwd_bf16(A, A, A, A, A, 0, None) == dqt.DQT_ERR_ARG
+    # RMSNorm: D a multiple of 8 and at most 2048; the backward needs its workspace
+    assert L.dqt_rmsnorm_bf16(A, A, C.c_float(1e-6), 4, 12, A, A, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_rmsnorm_bf16(A, A, C.c_float(1e-6), 4, 4096, A, A, None) == dqt.DQT_ERR_RANGE
+    assert L.dqt_rmsnorm_bf16(A, A, C.c_float(-1.0), 4, 64, A, A, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_rmsnorm_bwd_workspace_size(4, 4096) == 0
+    assert L.dqt_rmsnorm_bwd_bf16(A, A, A, A, 4, 64, A, A, None, 0, None) == dqt.DQT_ERR_ARG

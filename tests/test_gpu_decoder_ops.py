@@ -128,3 +128,45 @@ def test_swiglu_matches_fp64(shape):
     # and close to PyTorch's own silu(g) * u (which rounds silu(g) to bf16 first)
     ref_t = F.silu(g.detach()) * u.detach()
     assert ((h.float() - ref_t.float()).abs() <= 2 ** -6 * ref_t.float().abs() + 1e-30).all()
+
+
+@pytest.mark.parametrize("rows,D", [(1, 8), (37, 768), (300, 2048), (64, 1288)])
+def test_rmsnorm_matches_fp64(rows, D):
+    from paper_2412_04787_gb300.decoder import _RMSNorm
+    eps = 1e-6
+    x = inputs.normal((rows, D), 1.0, seed=rows + D, dtype=torch.bfloat16).cuda().requires_grad_()
+    w = (1.0 + inputs.normal((D,), 0.1, seed=D, dtype=torch.float32)).to(torch.bfloat16).cuda()
+    w.requires_grad_()
+    dy = inputs.normal((rows, D), 1.0, seed=rows, dtype=torch.bfloat16).cuda()
+    y = _RMSNorm.apply(x, w, eps)
+    y.backward(dy)
+    xd, wd, gd = x.detach().double(), w.detach().double(), dy.double()
+    r = 1.0 / torch.sqrt((xd * xd).mean(dim=1, keepdim=True) + eps)
+    ref_y = xd * r * wd
+    assert ((y.double() - ref_y).abs() <= 2 ** -7 * ref_y.abs() + 1e-30).all()
+    # dx = r w dy - x r^3 mean(w dy x): bounded relative to its two terms
+    t1 = r * wd * gd
+    t2 = xd * r ** 3 * (wd * gd * xd).mean(dim=1, keepdim=True)
+    err = (x.grad.double() - (t1 - t2)).abs()
+    assert (err <= 2 ** -7 * (t1.abs() + t2.abs()) + 1e-6).all()
+    # dw = sum over rows of dy x r (fp32 sums in a fixed order, one bf16 rounding)
+    terms = gd * xd * r
+    ref_dw = terms.sum(dim=0)
+    err = (w.grad.double() - ref_dw).abs()
+    assert (err <= 2 ** -7 * ref_dw.abs() + 1e-5 * terms.abs().sum(dim=0)).all()
+    # the decoder's module agrees with PyTorch's own rms_norm to bf16 rounding
+    ref_t = F.rms_norm(x.detach(), (D,), w.detach(), eps)
+    assert ((y.float() - ref_t.float()).abs() <= 2 ** -6 * ref_t.float().abs() + 1e-6).all()
+
+
+def test_rmsnorm_gain_gradient_is_deterministic():
+    from paper_2412_04787_gb300.decoder import _RMSNorm
+    x = inputs.normal((4096, 768), 1.0, seed=9, dtype=torch.bfloat16).cuda()
+    w = torch.ones(768, dtype=torch.bfloat16, device="cuda")
+    dy = inputs.normal((4096, 768), 1.0, seed=10, dtype=torch.bfloat16).cuda()
+    grads = []
+    for _ in range(2):
+        xi, wi = x.clone().requires_grad_(), w.clone().requires_grad_()
+        _RMSNorm.apply(xi, wi, 1e-6).backward(dy)
+        grads.append((xi.grad, wi.grad))
+    assert torch.equal(grads[0][0], grads[1][0]) and torch.equal(grads[0][1], grads[1][1])
