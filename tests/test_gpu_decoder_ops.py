@@ -1,8 +1,10 @@
-"""Decoder-support kernels (not part of the DQT method) against PyTorch
-references on the same inputs: the rotary embedding bit-exact against the same
-formula in separately rounded fp32 torch operations (and its backward against
-autograd through that formula), the token cross-entropy against
-F.cross_entropy on the fp32 upcast of the same bf16 logits."""
+"""Decoder-support kernels (not part of the DQT method) against references on
+the same inputs: the rotary embedding bit-exact against the same formula in
+separately rounded fp32 torch operations (and its backward against autograd
+through that formula); the token cross-entropy against F.cross_entropy on the
+fp32 upcast of the same bf16 logits; the SwiGLU gate and RMSNorm (outputs and
+all gradients) against fp64 within one bf16 rounding, and close to PyTorch's
+own silu * up and rms_norm."""
 import pytest
 import torch
 import torch.nn.functional as F
