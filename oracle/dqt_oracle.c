@@ -17,12 +17,14 @@
  *   Sec 3.2 backward w.r.t. the low-bit weight (no STE)   -> dqt_oracle_bwd_dx / _bwd_dw
  *   Sec 4.1/4.3 the same with X_tilde held in bf16        -> dqt_oracle_bwd_dw_bf16x
  *   Sec 4.1 AdamW producing the dense target W'           -> dqt_oracle_adamw_x
+ *           (its textbook evaluation order, for the pins)   -> dqt_oracle_adamw_x_textbook
  *   Eq. 5   W_hat = SR(W'), kept on the n-bit grid        -> dqt_oracle_update
  *   Sec 5.1 absmax / round-to-nearest ablation            -> round_mode = 1
  *   Sec 4.1/4.3 FP8 environment: E4M3 activations and      -> dqt_oracle_act_quant_fp8
  *               the forward on E4M3 operands                -> dqt_oracle_fwd_fp8
  *   Sec 1       2-bit packed ternary storage                -> dqt_oracle_pack_ternary
  *   Sec 4.3     Adafactor (factored second moment) + SR     -> dqt_oracle_adafactor_*
+ *               (the printed rank-one form, for the pins)   -> dqt_oracle_adafactor_u_textbook
  *
  * Readings where the paper is silent, taken here:
  *   - ternary ("1.58 bit") means the grid [-1, 1] with s = 1 / AbsMean;
@@ -165,6 +167,23 @@ int dqt_oracle_grid(int32_t bits_x100, int32_t* qmin, int32_t* qmax) {
 }
 
 /* ------------------------------------------------------------------------ */
+/* Eq. 4 alone: codes = Clip[Round(W * s), Q_n, Q_p] for a given fp32 scale  */
+/* s: one fp32 multiplication, Round() half-to-even, then the clip.          */
+/* ------------------------------------------------------------------------ */
+void dqt_oracle_quantize_weights(const float* W, int64_t numel, float s, int32_t qmin,
+                                 int32_t qmax, int8_t* codes) {
+  for (int64_t i = 0; i < numel; ++i) {
+    float p = W[i] * s;
+    float r = rintf(p);
+    int32_t c;
+    if (r >= (float)qmax) c = qmax;
+    else if (r <= (float)qmin) c = qmin;
+    else c = (int32_t)r;
+    codes[i] = (int8_t)c;
+  }
+}
+
+/* ------------------------------------------------------------------------ */
 /* Eq. 2-4: AbsMean(W) = (1/k) sum |w_i|;  s = Q_p / AbsMean(W);             */
 /* codes = Clip[Round(W * s), Q_n, Q_p].  The sum runs in fp64 in index      */
 /* order; s is rounded once to fp32; W * s is one fp32 multiplication and    */
@@ -181,15 +200,7 @@ int dqt_oracle_absmean_init(const float* W0, int64_t numel, int32_t qmin,
   if (!(absmean > 0.0)) return 2;
   float s = (float)((double)qmax / absmean);
   *s_w = s;
-  for (int64_t i = 0; i < numel; ++i) {
-    float p = W0[i] * s;
-    float r = rintf(p);
-    int32_t c;
-    if (r >= (float)qmax) c = qmax;
-    else if (r <= (float)qmin) c = qmin;
-    else c = (int32_t)r;
-    codes[i] = (int8_t)c;
-  }
+  dqt_oracle_quantize_weights(W0, numel, s, qmin, qmax, codes);
   return 0;
 }
 
@@ -367,6 +378,64 @@ void dqt_oracle_adamw_x(const float* g, const int8_t* c, float* m, float* v,
 }
 
 /* ------------------------------------------------------------------------ */
+/* The same AdamW step in the textbook order of Loshchilov & Hutter's         */
+/* algorithm, each a separately rounded fp32 operation:                      */
+/*   m' = b1 m + omb1 g ;  v' = b2 v + omb2 (g g)                            */
+/*   m_hat = m' / bc1 ;  v_hat = v' / bc2                                    */
+/*   u = m_hat / (sqrt(v_hat) + eps)                                         */
+/*   x = c decay - lrs u                                                     */
+/* Host constants, fp64 rounded once to fp32: b1, b2, omb1 = 1 - b1,          */
+/* omb2 = 1 - b2, bc1 = 1 - b1^step, bc2 = 1 - b2^step, eps,                  */
+/* decay = 1 - lr wd, lrs = lr s_w.  The restated one-division form above is  */
+/* the same quantity multiplied through by bc1; the two are compared          */
+/* elementwise by the pins.                                                  */
+/* ------------------------------------------------------------------------ */
+typedef struct {
+  float b1, b2, omb1, omb2, bc1, bc2, eps, decay, lrs;
+} oracle_adamw_textbook_consts;
+
+void dqt_oracle_adamw_textbook_consts(float lr, float b1, float b2, float eps, float wd,
+                                      int64_t step, float s_w, float* out9) {
+  out9[0] = b1;
+  out9[1] = b2;
+  out9[2] = (float)(1.0 - (double)b1);
+  out9[3] = (float)(1.0 - (double)b2);
+  out9[4] = (float)(1.0 - pow((double)b1, (double)step));
+  out9[5] = (float)(1.0 - pow((double)b2, (double)step));
+  out9[6] = eps;
+  out9[7] = (float)(1.0 - (double)lr * (double)wd);
+  out9[8] = (float)((double)lr * (double)s_w);
+}
+
+static float adamw_x_textbook(const oracle_adamw_textbook_consts* h, float g, int8_t c,
+                              float* m, float* v) {
+  float m1 = h->b1 * *m;
+  float m2 = h->omb1 * g;
+  float mn = m1 + m2;
+  float v1 = h->b2 * *v;
+  float gg = g * g;
+  float v2 = h->omb2 * gg;
+  float vn = v1 + v2;
+  *m = mn;
+  *v = vn;
+  float mh = mn / h->bc1;
+  float vh = vn / h->bc2;
+  float sv = sqrtf(vh);
+  float den = sv + h->eps;
+  float u = mh / den;
+  float cd = (float)c * h->decay;
+  float du = h->lrs * u;
+  return cd - du;
+}
+
+void dqt_oracle_adamw_x_textbook(const float* g, const int8_t* c, float* m, float* v,
+                                 const float* tconsts9, int64_t n, float* x) {
+  oracle_adamw_textbook_consts h;
+  memcpy(&h, tconsts9, sizeof(h));
+  for (int64_t i = 0; i < n; ++i) x[i] = adamw_x_textbook(&h, g[i], c[i], &m[i], &v[i]);
+}
+
+/* ------------------------------------------------------------------------ */
 /* Eq. 5: W_hat = SR(W'), clamped to [Q_n, Q_p], written over the codes.     */
 /* g, c, m, v are [Nr, K] row blocks of an [N, K] weight; rows[i] is the      */
 /* global row of block row i, so element (rows[i], k) draws the uniform of   */
@@ -374,19 +443,22 @@ void dqt_oracle_adamw_x(const float* g, const int8_t* c, float* m, float* v,
 /* round_mode 0 = stochastic (Eq. 1); 1 = round-to-nearest (Sec 5.1          */
 /* ablation).  Returns the number of codes that changed.                     */
 /* ------------------------------------------------------------------------ */
-int64_t dqt_oracle_update(const float* g, int8_t* c, float* m, float* v,
-                          const float* consts9, int32_t qmin, int32_t qmax,
-                          uint64_t seed, int64_t step, uint32_t tensor_id,
-                          int32_t round_mode, const int64_t* rows, int64_t Nr,
-                          int64_t K) {
+static int64_t update_impl(int textbook, const float* g, int8_t* c, float* m, float* v,
+                           const float* consts9, int32_t qmin, int32_t qmax,
+                           uint64_t seed, int64_t step, uint32_t tensor_id,
+                           int32_t round_mode, const int64_t* rows, int64_t Nr,
+                           int64_t K) {
   oracle_adamw_consts h;
+  oracle_adamw_textbook_consts ht;
   memcpy(&h, consts9, sizeof(h));
+  memcpy(&ht, consts9, sizeof(ht));
   int64_t changed = 0;
   for (int64_t i = 0; i < Nr; ++i) {
     int64_t n = rows ? rows[i] : i;
     for (int64_t k = 0; k < K; ++k) {
       int64_t j = i * K + k;
-      float x = adamw_x(&h, g[j], c[j], &m[j], &v[j]);
+      float x = textbook ? adamw_x_textbook(&ht, g[j], c[j], &m[j], &v[j])
+                         : adamw_x(&h, g[j], c[j], &m[j], &v[j]);
       int32_t r;
       if (round_mode == 1) {
         r = (int32_t)rintf(x);
@@ -400,6 +472,26 @@ int64_t dqt_oracle_update(const float* g, int8_t* c, float* m, float* v,
     }
   }
   return changed;
+}
+
+int64_t dqt_oracle_update(const float* g, int8_t* c, float* m, float* v,
+                          const float* consts9, int32_t qmin, int32_t qmax,
+                          uint64_t seed, int64_t step, uint32_t tensor_id,
+                          int32_t round_mode, const int64_t* rows, int64_t Nr,
+                          int64_t K) {
+  return update_impl(0, g, c, m, v, consts9, qmin, qmax, seed, step, tensor_id, round_mode,
+                     rows, Nr, K);
+}
+
+/* Eq. 5 with the textbook-order AdamW (tconsts9 from                        */
+/* dqt_oracle_adamw_textbook_consts); otherwise identical to the above.      */
+int64_t dqt_oracle_update_textbook(const float* g, int8_t* c, float* m, float* v,
+                                   const float* tconsts9, int32_t qmin, int32_t qmax,
+                                   uint64_t seed, int64_t step, uint32_t tensor_id,
+                                   int32_t round_mode, const int64_t* rows, int64_t Nr,
+                                   int64_t K) {
+  return update_impl(1, g, c, m, v, tconsts9, qmin, qmax, seed, step, tensor_id, round_mode,
+                     rows, Nr, K);
 }
 
 /* ======================================================================== */
@@ -558,6 +650,30 @@ void dqt_oracle_adafactor_consts(int64_t t, float lr, float decay_rate, int32_t 
 static float adafactor_u(float g, float an, float bk) {
   float ga = g * an;
   return ga * bk;
+}
+
+/* Shazeer & Stern's update in its printed form: the rank-one estimate      */
+/* V[n,k] = R[n] C[k] / Rbar, then u = g / sqrt(V), each a separately        */
+/* rounded fp32 operation.  The factored form above computes the same        */
+/* quantity; the pins compare the two elementwise.  (The printed form         */
+/* underflows fp32 once R[n] C[k] drops below the smallest normal float; the  */
+/* factored form does not.)                                                  */
+void dqt_oracle_adafactor_u_textbook(const float* g, const float* R, const float* C, float rbar,
+                                     int64_t N, int64_t K, float* u) {
+  for (int64_t n = 0; n < N; ++n)
+    for (int64_t k = 0; k < K; ++k) {
+      float rc = R[n] * C[k];
+      float vv = rc / rbar;
+      float sq = sqrtf(vv);
+      u[n * K + k] = g[n * K + k] / sq;
+    }
+}
+
+/* The factored form's u for every element (a, b from the statistics).       */
+void dqt_oracle_adafactor_u(const float* g, const float* a, const float* b, int64_t N, int64_t K,
+                            float* u) {
+  for (int64_t n = 0; n < N; ++n)
+    for (int64_t k = 0; k < K; ++k) u[n * K + k] = adafactor_u(g[n * K + k], a[n], b[k]);
 }
 
 /* R, C updated in place; a [N], b [K] the inverse-square-root factors.     */

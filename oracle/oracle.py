@@ -7,11 +7,13 @@ with Stochastic Rounding"):
 * ``sr``/``sr_batch``          -- Eq. 1, stochastic rounding
 * ``grid``                     -- Eq. 3, the n-bit grid [Q_n, Q_p]
 * ``absmean_init``             -- Eq. 2-4, AbsMean scale and initial codes
+* ``quantize_weights``         -- Eq. 4 alone, for a given scale
 * ``act_quant``                -- Sec. 3.2, 8-bit per-token absmax activations
 * ``fwd``                      -- Sec. 3.2, BitLinear forward (exact int accumulation)
 * ``bwd_dx`` / ``bwd_dw``      -- Sec. 3.2, backward w.r.t. input and low-bit weight (fp64)
 * ``bwd_dw_bf16x``             -- Sec. 4.1/4.3, the weight gradient with X_tilde in bf16
 * ``adamw_consts``/``adamw_x`` -- Sec. 4.1, AdamW producing the dense target W'
+  (``adamw_textbook_consts``/``adamw_x_textbook``: the textbook evaluation order)
 * ``update``                   -- Eq. 5, W_hat = SR(W') clamped onto the grid
 * ``pack_ternary``/``unpack_ternary`` -- Sec. 1, 2-bit packed ternary storage
 * ``adafactor_consts``/``adafactor_stats``/``adafactor_x``/``adafactor_apply``
@@ -84,6 +86,23 @@ def lib():
                                         C.c_int32, C.c_uint64, C.c_int64, C.c_uint32,
                                         C.c_int32, _i64p, C.c_int64, C.c_int64]
         L.dqt_oracle_update.restype = C.c_int64
+        L.dqt_oracle_adamw_textbook_consts.argtypes = [C.c_float, C.c_float, C.c_float,
+                                                       C.c_float, C.c_float, C.c_int64,
+                                                       C.c_float, _f32p]
+        L.dqt_oracle_adamw_textbook_consts.restype = None
+        L.dqt_oracle_adamw_x_textbook.argtypes = [_f32p, _i8p, _f32p, _f32p, _f32p, C.c_int64,
+                                                  _f32p]
+        L.dqt_oracle_adamw_x_textbook.restype = None
+        L.dqt_oracle_update_textbook.argtypes = L.dqt_oracle_update.argtypes
+        L.dqt_oracle_update_textbook.restype = C.c_int64
+        L.dqt_oracle_quantize_weights.argtypes = [_f32p, C.c_int64, C.c_float, C.c_int32,
+                                                  C.c_int32, _i8p]
+        L.dqt_oracle_quantize_weights.restype = None
+        L.dqt_oracle_adafactor_u_textbook.argtypes = [_f32p, _f32p, _f32p, C.c_float,
+                                                      C.c_int64, C.c_int64, _f32p]
+        L.dqt_oracle_adafactor_u_textbook.restype = None
+        L.dqt_oracle_adafactor_u.argtypes = [_f32p, _f32p, _f32p, C.c_int64, C.c_int64, _f32p]
+        L.dqt_oracle_adafactor_u.restype = None
         L.dqt_oracle_e4m3_value.argtypes = [C.c_uint8]
         L.dqt_oracle_e4m3_value.restype = C.c_double
         L.dqt_oracle_e4m3_from_f32.argtypes = [C.c_float]
@@ -190,6 +209,15 @@ def absmean_init(W0, qmin: int, qmax: int):
     return codes, np.float32(s.value), am.value
 
 
+def quantize_weights(W, s_w, qmin: int, qmax: int):
+    """Eq. 4 alone: Clip[Round(W * s_w), qmin, qmax] for a given fp32 scale."""
+    W = _c(W, np.float32)
+    codes = np.empty(W.shape, np.int8)
+    lib().dqt_oracle_quantize_weights(_p(W, _f32p), W.size, float(np.float32(s_w)), qmin, qmax,
+                                      _p(codes, _i8p))
+    return codes
+
+
 # --------------------------------------------------------------------------
 # Sec. 3.2 activation quantisation
 # --------------------------------------------------------------------------
@@ -288,9 +316,33 @@ def adamw_x(g, c, m, v, consts):
     return x, m, v
 
 
+def adamw_textbook_consts(lr, b1, b2, eps, wd, step, s_w):
+    """Constants of the textbook-order AdamW: b1, b2, 1-b1, 1-b2, bc1, bc2, eps,
+    1 - lr wd, lr s_w (each rounded once to fp32)."""
+    out = np.empty(9, np.float32)
+    lib().dqt_oracle_adamw_textbook_consts(lr, b1, b2, eps, wd, step, float(s_w),
+                                           _p(out, _f32p))
+    return out
+
+
+def adamw_x_textbook(g, c, m, v, tconsts):
+    """As adamw_x, with m_hat = m'/bc1, v_hat = v'/bc2, m_hat/(sqrt(v_hat)+eps)."""
+    g = _c(g, np.float32).ravel()
+    c = _c(c, np.int8).ravel()
+    m = _c(m, np.float32).ravel().copy()
+    v = _c(v, np.float32).ravel().copy()
+    x = np.empty_like(g)
+    k = _c(tconsts, np.float32)
+    lib().dqt_oracle_adamw_x_textbook(_p(g, _f32p), _p(c, _i8p), _p(m, _f32p), _p(v, _f32p),
+                                      _p(k, _f32p), g.size, _p(x, _f32p))
+    return x, m, v
+
+
 def update(g, c, m, v, consts, qmin, qmax, seed, step, tensor_id, round_mode=0,
-           rows=None):
-    """Eq. 5 over an [Nr, K] block.  Returns (c', m', v', changed)."""
+           rows=None, textbook=False):
+    """Eq. 5 over an [Nr, K] block.  Returns (c', m', v', changed).  With
+    textbook=True the AdamW step is the textbook-order form and ``consts``
+    come from adamw_textbook_consts."""
     g = _c(g, np.float32)
     if g.ndim == 1:
         g = g.reshape(1, -1)
@@ -305,9 +357,9 @@ def update(g, c, m, v, consts, qmin, qmax, seed, step, tensor_id, round_mode=0,
         rp = _p(rows, _i64p)
     else:
         rp = None
-    changed = lib().dqt_oracle_update(_p(g, _f32p), _p(c, _i8p), _p(m, _f32p),
-                                      _p(v, _f32p), _p(k, _f32p), qmin, qmax, seed, step,
-                                      tensor_id, round_mode, rp, Nr, K)
+    fn = lib().dqt_oracle_update_textbook if textbook else lib().dqt_oracle_update
+    changed = fn(_p(g, _f32p), _p(c, _i8p), _p(m, _f32p), _p(v, _f32p), _p(k, _f32p), qmin,
+                 qmax, seed, step, tensor_id, round_mode, rp, Nr, K)
     return c, m, v, int(changed)
 
 
@@ -427,6 +479,29 @@ def adafactor_stats(g, c, s_w, R, C_, t, hp):
     st = {"rbar": out4[0], "rms_u": out4[1], "rms_x": out4[2], "alpha": out4[3],
           "step": np.float32(step.value), "decay": np.float32(decay.value), "a": a, "b": b}
     return R, Cc, st
+
+
+def adafactor_u(g, a, b):
+    """The factored form's u = (g a[n]) b[k] for every element of g [N, K]."""
+    g = _c(g, np.float32)
+    N, K = g.shape
+    a = _c(a, np.float32)
+    b = _c(b, np.float32)
+    u = np.empty((N, K), np.float32)
+    lib().dqt_oracle_adafactor_u(_p(g, _f32p), _p(a, _f32p), _p(b, _f32p), N, K, _p(u, _f32p))
+    return u
+
+
+def adafactor_u_textbook(g, R, C_, rbar):
+    """The printed form u = g / sqrt(R[n] C[k] / Rbar), fp32 operations."""
+    g = _c(g, np.float32)
+    N, K = g.shape
+    R = _c(R, np.float32)
+    Cc = _c(C_, np.float32)
+    u = np.empty((N, K), np.float32)
+    lib().dqt_oracle_adafactor_u_textbook(_p(g, _f32p), _p(R, _f32p), _p(Cc, _f32p),
+                                          float(np.float32(rbar)), N, K, _p(u, _f32p))
+    return u
 
 
 def adafactor_x(g, c, a, b, step, decay):

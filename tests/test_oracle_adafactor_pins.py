@@ -240,3 +240,89 @@ def test_matches_torch_adafactor_dense_target():
         # oracle's codes do not move (the comparison is of one step's target)
         with torch.no_grad():
             W.copy_(torch.tensor(cur.astype(np.float64) / s_w))
+
+
+# --------------------------------------------------------------------------
+# The factored evaluation u = (g a[n]) b[k] against Shazeer & Stern's printed
+# form u = g / sqrt(R[n] C[k] / Rbar): in fp32 (the same quantity in another
+# order of rounded operations) and in fp64, over edge inputs.
+# --------------------------------------------------------------------------
+# (name, gradient scale, log-spread of row scales, of column scales, steps)
+AF_EDGE_CASES = [
+    ("typical, step 1", 1e-3, 0.0, 0.0, 1),
+    ("rows and columns spread over 2.6 decades", 1e-3, 3.0, 3.0, 1),
+    ("spread, step 5", 1e-3, 3.0, 3.0, 5),
+    ("eps1 dominates (g^2 << 1e-30)", 1e-16, 0.0, 0.0, 1),
+    ("eps1 dominates with spread, step 3", 1e-16, 3.0, 3.0, 3),
+    ("large gradients, wide spread", 1.0, 5.0, 5.0, 2),
+]
+
+
+def _af_edge(case, N=64, K=96):
+    name, gs, rs, cs, steps = case
+    r = np.random.default_rng(len(name) * 1000 + steps)
+    g = (r.normal(0, 1, (N, K)) * gs * np.exp(r.uniform(-rs, rs, (N, 1)))
+         * np.exp(r.uniform(-cs, cs, (1, K)))).astype(np.float32)
+    c = r.integers(-1, 2, (N, K)).astype(np.int8)
+    hp = oracle.AdafactorHP(lr=1e-2)
+    R, Cc = np.zeros(N, np.float32), np.zeros(K, np.float32)
+    for t in range(1, steps + 1):
+        R, Cc, st = oracle.adafactor_stats(g, c, np.float32(62.66), R, Cc, t, hp)
+    return g, c, R, Cc, st, steps
+
+
+@pytest.mark.parametrize("case", AF_EDGE_CASES, ids=[c[0] for c in AF_EDGE_CASES])
+def test_factored_u_equals_printed_form(case):
+    """Relative to the fp64 value of g / sqrt(R C / Rbar) (same fp32 R, C,
+    Rbar): the factored form rounds R/Rbar, two square roots, two
+    reciprocals and two products -- below 7 * 2^-24 of |u| (a square root
+    halves its input's error), bound 8 here; the printed fp32 form rounds the
+    product, the quotient, the square root and the division -- below 4 *
+    2^-24, bound 5, wherever R[n] C[k] is a normal fp32 number (below that
+    the printed form underflows and only the factored one is defined); the
+    two fp32 forms then differ by at most 13 * 2^-24 of |u|."""
+    g, c, R, Cc, st, _ = _af_edge(case)
+    uf = oracle.adafactor_u(g, st["a"], st["b"])
+    ut = oracle.adafactor_u_textbook(g, R, Cc, st["rbar"])
+    rbar = float(np.float32(st["rbar"]))
+    V = R.astype(np.float64)[:, None] * Cc.astype(np.float64)[None, :] / rbar
+    u64 = g.astype(np.float64) / np.sqrt(V)
+    ulp24 = np.abs(u64) * 2.0 ** -24 + 1e-45
+    assert (np.abs(uf - u64) <= 8 * ulp24).all()
+    normal = np.abs(R.astype(np.float64)[:, None] * Cc[None, :]) >= np.finfo(np.float32).tiny
+    assert (np.abs(ut - u64) <= 5 * ulp24)[normal].all()
+    assert (np.abs(uf.astype(np.float64) - ut) <= 13 * ulp24)[normal].all()
+    if case[1] >= 1e-3:
+        assert normal.all()  # the comparison covers every element there
+
+
+def test_factored_and_printed_forms_flip_few_stochastic_roundings():
+    """Under the same Philox stream, codes from x = c decay - step u with the
+    factored u and with the printed-form u (where it is defined) differ in at
+    most 1e-4 of the elements, each by exactly one grid step."""
+    total = flips = 0
+    for case in AF_EDGE_CASES:
+        g, c, R, Cc, st, t = _af_edge(case)
+        N, K = g.shape
+        uf = oracle.adafactor_u(g, st["a"], st["b"])
+        ut = oracle.adafactor_u_textbook(g, R, Cc, st["rbar"])
+        normal = np.abs(R.astype(np.float64)[:, None] * Cc[None, :]) >= np.finfo(np.float32).tiny
+        # x in separately rounded fp32 operations (numpy float32 forms no FMA)
+        cd = c.astype(np.float32) * st["decay"]
+        xf = cd - st["step"] * uf
+        xt = cd - st["step"] * ut
+        # the oracle's own apply reproduces xf's rounding exactly
+        c_apply, _ = oracle.adafactor_apply(g, c, st["a"], st["b"], st["step"], st["decay"],
+                                            -1, 1, 77, t, 9)
+        words = np.array([oracle.sr_word(77, t, 9, e) for e in range(N * K)], np.uint32)
+        U = ((words >> 8).astype(np.float64) * 2.0 ** -24).astype(np.float32)
+        cf = np.clip(oracle.sr_batch(xf.ravel(), U), -1, 1)
+        ctb = np.clip(oracle.sr_batch(xt.ravel(), U), -1, 1)
+        assert np.array_equal(cf, c_apply.ravel())
+        m = normal.ravel()
+        diff = cf[m] != ctb[m]
+        assert (np.abs(cf[m] - ctb[m])[diff] == 1).all()
+        total += int(m.sum())
+        flips += int(diff.sum())
+    assert total > 0
+    assert flips <= int(1e-4 * total), (flips, total)

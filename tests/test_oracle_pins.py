@@ -9,6 +9,7 @@ import ctypes
 import json
 import math
 import os
+import zlib
 
 import numpy as np
 import pytest
@@ -185,6 +186,21 @@ def test_absmean_hand_examples():
         assert abs(am - case["absmean"]) < 1e-7, case
         assert abs(float(s) - case["s"]) < 1e-5 * case["s"], case
         assert codes.tolist() == case["codes"], case
+        # Eq. 4 on its own, at the worked scale, gives the worked codes
+        q = oracle.quantize_weights(np.array(case["W"], np.float32), s, qmin, qmax)
+        assert q.tolist() == case["codes"], case
+
+
+def test_quantize_weights_is_round_half_even_then_clip():
+    """Eq. 4 at a given fp32 scale against numpy's rint (half-to-even) and clip
+    of the fp32 product, over random weights and a scale whose products land
+    on exact .5 ties."""
+    W = np.concatenate([inputs.normal((4096,), 0.02, seed=12).numpy(),
+                        np.arange(-20, 21, dtype=np.float32) * 0.25]).astype(np.float32)
+    for s, (qmin, qmax) in [(np.float32(62.66), (-1, 1)), (np.float32(6.0), (-128, 127)),
+                            (np.float32(2.0), (-8, 7))]:
+        want = np.clip(np.rint(W * s), qmin, qmax).astype(np.int8)
+        assert np.array_equal(oracle.quantize_weights(W, s, qmin, qmax), want)
 
 
 def test_absmean_statistics_gaussian():
@@ -324,6 +340,114 @@ def test_adamw_step1_closed_form():
     assert np.allclose(m, 0.1 * g64, rtol=1e-6)
     assert np.allclose(v, 0.001 * g64 * g64, rtol=1e-6)
     assert np.allclose(x, -0.05 * g64 / (np.abs(g64) + 1e-8), rtol=1e-5)
+
+
+# --------------------------------------------------------------------------
+# Sec. 4.1 AdamW: the one-division form used by the update (m' / (sqrt(v') k1
+# + k2)) against the textbook order (m_hat = m'/bc1, v_hat = v'/bc2,
+# m_hat / (sqrt(v_hat) + eps)), each in separately rounded fp32 operations,
+# and both against the same formula in fp64, over edge inputs.
+# --------------------------------------------------------------------------
+_F32 = lambda a: float(np.float32(a))  # noqa: E731
+# (name, scale of g, scale of m, scale of sqrt(v), step, weight decay, lr)
+ADAMW_EDGE_CASES = [
+    ("zero gradient and moments", 0.0, 0.0, 0.0, 1, 0.0, 1e-3),
+    ("step 1 from zero moments", 1e-3, 0.0, 0.0, 1, 0.0, 1e-3),
+    ("v = 0, m != 0", 0.0, 1e-4, 0.0, 3, 0.0, 1e-3),
+    ("v << eps^2 (eps dominates)", 1e-12, 1e-12, 1e-13, 5, 0.0, 1e-3),
+    ("sqrt(v_hat) ~ eps", 1e-8, 1e-8, 1e-8, 5, 0.0, 1e-3),
+    ("typical, weight decay", 1e-3, 1e-4, 1e-4, 7, 0.01, 1e-3),
+    ("step 100", 1e-3, 1e-4, 1e-4, 100, 0.0, 1e-3),
+    ("step 10^4, wd 0.1, lr 1e-2", 1e-3, 1e-4, 1e-4, 10_000, 0.1, 1e-2),
+    ("large gradients", 1.0, 1.0, 1.0, 2, 0.0, 1e-3),
+    ("subnormal moments", 1e-20, 1e-20, 1e-20, 2, 0.0, 1e-3),
+]
+
+
+def _adamw_edge(case, bits, n=20000):
+    name, gs, ms, vs, step, wd, lr = case
+    r = np.random.default_rng(zlib.crc32(f"{name}/{bits}".encode()))
+    qmin, qmax = oracle.grid(bits)
+    c = r.integers(qmin, qmax + 1, n).astype(np.int8)
+    # s_w of AbsMean-quantised N(0, 0.02) weights: qmax / (0.02 sqrt(2/pi))
+    s_w = np.float32(qmax / (0.02 * math.sqrt(2.0 / math.pi)))
+    g = (r.normal(0, 1, n) * gs).astype(np.float32)
+    m = (r.normal(0, 1, n) * ms).astype(np.float32)
+    v = np.square(r.normal(0, 1, n) * vs).astype(np.float32)
+    k = oracle.adamw_consts(lr, 0.9, 0.999, 1e-8, wd, step, s_w)
+    kt = oracle.adamw_textbook_consts(lr, 0.9, 0.999, 1e-8, wd, step, s_w)
+    return c, s_w, g, m, v, k, kt, (qmin, qmax), (step, wd, lr)
+
+
+def _ulp(x):
+    return np.spacing(np.abs(np.asarray(x, np.float32))).astype(np.float64)
+
+
+@pytest.mark.parametrize("bits", [1.58, 8])
+@pytest.mark.parametrize("case", ADAMW_EDGE_CASES, ids=[c[0] for c in ADAMW_EDGE_CASES])
+def test_adamw_one_division_form_equals_textbook_order(case, bits):
+    """The two orders share m' and v' bit for bit.  Their u differ only by
+    rounding: the textbook order rounds m_hat, v_hat, sqrt, the sum and the
+    quotient; the one-division form rounds sqrt, the product with k1, the sum
+    and the quotient, plus k1 and k2 themselves -- at most 6 roundings each, a
+    relative difference below 12 * 2^-24 of u (a square root halves its
+    input's error).  Through x = c decay - lrs u that is at most
+    (12 + 2 + 2) * 2^-24 of the step |lrs u| (the product and its ulp on
+    either side) plus one ulp of x on either side.  The bound below, 20 ulps
+    of 2^-24 |step| plus 3 ulps of x, holds with margin for every element."""
+    c, s_w, g, m, v, k, kt, _, _ = _adamw_edge(case, bits)
+    xr, mr, vr = oracle.adamw_x(g, c, m, v, k)
+    xt, mt, vt = oracle.adamw_x_textbook(g, c, m, v, kt)
+    assert np.array_equal(mr.view(np.uint32), mt.view(np.uint32))
+    assert np.array_equal(vr.view(np.uint32), vt.view(np.uint32))
+    A = (c.astype(np.float32) * kt[7]).astype(np.float64)  # c decay, rounded alike
+    step_mag = np.abs(A - xt.astype(np.float64))
+    d = np.abs(xr.astype(np.float64) - xt.astype(np.float64))
+    bound = 20 * 2.0 ** -24 * step_mag + 3 * _ulp(xt) + 1e-37
+    assert (d <= bound).all(), float((d / bound).max())
+    # most elements agree bit for bit
+    assert np.mean(d == 0) >= 0.5
+
+
+@pytest.mark.parametrize("bits", [1.58, 8])
+@pytest.mark.parametrize("case", ADAMW_EDGE_CASES, ids=[c[0] for c in ADAMW_EDGE_CASES])
+def test_adamw_both_orders_match_fp64(case, bits):
+    """Both fp32 orders against AdamW's dense target evaluated in fp64 from the
+    same hyper-parameters (as fp32 values) and the same new moments: within
+    8 * 2^-24 of the step, 2^-24 |c| (the rounding of c decay and of its
+    constant) and one ulp of x."""
+    c, s_w, g, m, v, k, kt, _, (step, wd, lr) = _adamw_edge(case, bits)
+    xr, _, _ = oracle.adamw_x(g, c, m, v, k)
+    xt, mt, vt = oracle.adamw_x_textbook(g, c, m, v, kt)
+    b1, b2, eps, lr, wd = _F32(0.9), _F32(0.999), _F32(1e-8), _F32(lr), _F32(wd)
+    bc1 = 1.0 - b1 ** step
+    bc2 = 1.0 - b2 ** step
+    u = (mt.astype(np.float64) / bc1) / (np.sqrt(vt.astype(np.float64) / bc2) + eps)
+    x64 = c.astype(np.float64) * (1.0 - lr * wd) - lr * float(s_w) * u
+    bound = (8 * 2.0 ** -24 * np.abs(lr * float(s_w) * u)
+             + 2.0 ** -24 * np.abs(c.astype(np.float64)) + _ulp(xt) + 1e-37)
+    assert (np.abs(xr - x64) <= bound).all()
+    assert (np.abs(xt - x64) <= bound).all()
+
+
+def test_adamw_orders_flip_few_stochastic_roundings():
+    """Under the same Philox stream, the update with the one-division AdamW and
+    the update with the textbook order round to the same codes except where a
+    uniform falls between their two dense targets: over all edge cases at
+    most 1e-4 of the codes differ, each by exactly one grid step."""
+    total = flips = 0
+    for case in ADAMW_EDGE_CASES:
+        for bits in (1.58, 8):
+            c, s_w, g, m, v, k, kt, (qmin, qmax), (step, _, _) = _adamw_edge(case, bits)
+            cr, mr, vr, _ = oracle.update(g, c, m, v, k, qmin, qmax, 1234, step, 3)
+            ct, mt, vt, _ = oracle.update(g, c, m, v, kt, qmin, qmax, 1234, step, 3,
+                                          textbook=True)
+            assert np.array_equal(mr, mt) and np.array_equal(vr, vt)
+            diff = cr != ct
+            assert (np.abs(cr.astype(np.int32) - ct.astype(np.int32))[diff] == 1).all()
+            total += diff.size
+            flips += int(diff.sum())
+    assert flips <= int(1e-4 * total), (flips, total)
 
 
 # --------------------------------------------------------------------------
