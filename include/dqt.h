@@ -142,10 +142,11 @@ int dqt_absmean_init(const float* W0, int64_t numel, dqt_grid_t grid, int8_t* co
  * sums live in a static device array of 1025 doubles (8200 bytes) that every
  * GPU loading the library holds until the process exits.  Same arguments and
  * results as dqt_absmean_init; numel <= 2^53, else DQT_ERR_RANGE.  It calls
- * no allocator.  The first call on a device looks up the array's device
- * address (so make that first call before any stream capture).  All calls on
- * a device share the array: calls that overlap on the GPU race, so serialise
- * them.  Synchronous, like dqt_absmean_init. */
+ * no allocator.  Each call looks up (and caches) the array's device address
+ * on the current device.  All calls on a device share the array: calls that
+ * overlap on the GPU race, so serialise them.  Synchronous, like
+ * dqt_absmean_init: every call waits for `stream` and copies the mean to the
+ * host, so it must not be called on a stream that is being captured. */
 int dqt_absmean_init_noalloc(const float* W0, int64_t numel, dqt_grid_t grid, int8_t* codes,
                              float* s_w, void* stream);
 

@@ -19,6 +19,8 @@
 // streams, or different host threads) race on the array: serialise them.
 #include <stdint.h>
 
+#include <atomic>
+
 #include "../../include/dqt.h"
 #include "dqt_internal.h"
 
@@ -27,7 +29,9 @@ namespace {
 static __device__ __align__(256) double g_absmean_scratch[dqt::kAbsmeanBlocks + 1];
 
 constexpr int kMaxDevices = 64;
-double* g_scratch_ptr[kMaxDevices] = {nullptr};
+// Per-device address cache.  Host threads may call concurrently: the cache
+// is atomic (every thread that finds it empty stores the same address).
+std::atomic<double*> g_scratch_ptr[kMaxDevices] = {};
 
 // Largest element count whose mean divisor converts to fp64 exactly.
 constexpr int64_t kMaxNumel = int64_t(1) << 53;
@@ -41,26 +45,27 @@ double* scratch_on_current_device(int* status) {
     *status = DQT_ERR_CUDA;
     return nullptr;
   }
-  if (!g_scratch_ptr[dev]) {
+  double* cached = g_scratch_ptr[dev].load(std::memory_order_relaxed);
+  if (!cached) {
     double* p = nullptr;
     if (cudaGetSymbolAddress(reinterpret_cast<void**>(&p), g_absmean_scratch) != cudaSuccess ||
         !p) {
       *status = DQT_ERR_CUDA;
       return nullptr;
     }
-    g_scratch_ptr[dev] = p;
+    cached = p;
+    g_scratch_ptr[dev].store(cached, std::memory_order_relaxed);
   }
   *status = DQT_OK;
-  return g_scratch_ptr[dev];
+  return cached;
 }
 
 }  // namespace
 
 extern "C" int dqt_absmean_init_noalloc(const float* W0, int64_t numel, dqt_grid_t grid,
                                         int8_t* codes, float* s_w, void* stream) {
-  if (!W0 || !codes || !s_w || numel <= 0) return DQT_ERR_ARG;
-  if (grid.qmin > grid.qmax || grid.qmin < -128 || grid.qmax > 127 || grid.qmin > 0 ||
-      grid.qmax <= 0)
+  // the same argument rules as dqt_absmean_init (shared helpers)
+  if (!W0 || !codes || !s_w || numel <= 0 || !dqt::grid_ok(grid) || grid.qmax <= 0)
     return DQT_ERR_ARG;
   if (numel > kMaxNumel) return DQT_ERR_RANGE;
   static_assert(sizeof(g_absmean_scratch) >= (dqt::kAbsmeanBlocks + 1) * sizeof(double),
@@ -76,7 +81,7 @@ extern "C" int dqt_absmean_init_noalloc(const float* W0, int64_t numel, dqt_grid
     return DQT_ERR_CUDA;
   if (cudaStreamSynchronize(st) != cudaSuccess) return DQT_ERR_CUDA;
   const double absmean = sum / static_cast<double>(numel);
-  if (!(absmean > 0.0) || !(absmean < 1e300)) return DQT_ERR_ARG;
+  if (!dqt::absmean_ok(absmean)) return DQT_ERR_ARG;
   const float s = static_cast<float>(static_cast<double>(grid.qmax) / absmean);
   *s_w = s;
   return dqt::launch_absmean_codes(W0, numel, s, grid.qmin, grid.qmax, codes, st) ? DQT_ERR_CUDA

@@ -18,7 +18,8 @@ namespace {
 std::atomic<uint64_t> g_wait_ns{2000000000ull};
 std::atomic<int> g_gemm_mode{0};
 constexpr int kMaxDevices = 64;
-unsigned int* g_status_ptr[kMaxDevices] = {nullptr};
+// Per-device address cache; host threads may look it up concurrently.
+std::atomic<unsigned int*> g_status_ptr[kMaxDevices] = {};
 }  // namespace
 
 uint64_t wait_limit_ns() { return g_wait_ns.load(); }
@@ -27,12 +28,14 @@ int gemm_mode() { return g_gemm_mode.load(); }
 unsigned int* status_word() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
-  if (!g_status_ptr[dev]) {
+  unsigned int* cached = g_status_ptr[dev].load(std::memory_order_relaxed);
+  if (!cached) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
-    g_status_ptr[dev] = static_cast<unsigned int*>(p);
+    cached = static_cast<unsigned int*>(p);
+    g_status_ptr[dev].store(cached, std::memory_order_relaxed);
   }
-  return g_status_ptr[dev];
+  return cached;
 }
 
 }  // namespace dqt
@@ -41,9 +44,7 @@ namespace {
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-inline bool grid_ok(dqt_grid_t g) {
-  return g.qmin <= g.qmax && g.qmin >= -128 && g.qmax <= 127 && g.qmin <= 0 && g.qmax >= 0;
-}
+using dqt::grid_ok;
 
 inline cudaStream_t as_stream(void* s) { return static_cast<cudaStream_t>(s); }
 
@@ -154,7 +155,7 @@ int dqt_absmean_init(const float* W0, int64_t numel, dqt_grid_t grid, int8_t* co
     return DQT_ERR_CUDA;
   if (cudaStreamSynchronize(st) != cudaSuccess) return DQT_ERR_CUDA;
   const double absmean = sum / static_cast<double>(numel);
-  if (!(absmean > 0.0) || !isfinite(absmean)) return DQT_ERR_ARG;
+  if (!dqt::absmean_ok(absmean)) return DQT_ERR_ARG;
   const float s = static_cast<float>(static_cast<double>(grid.qmax) / absmean);
   *s_w = s;
   return dqt::launch_absmean_codes(W0, numel, s, grid.qmin, grid.qmax, codes, st) ? DQT_ERR_CUDA

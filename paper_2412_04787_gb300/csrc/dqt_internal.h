@@ -2,11 +2,21 @@
 #pragma once
 
 #include <cuda_runtime.h>
+#include <math.h>
 #include <stdint.h>
 
+#include "../../include/dqt.h"
 #include "dqt_device.cuh"
 
 namespace dqt {
+
+// Argument rules shared by entry points that must accept and reject alike.
+// A weight grid: Q_n <= 0 <= Q_p, both within int8.
+inline bool grid_ok(dqt_grid_t g) {
+  return g.qmin <= g.qmax && g.qmin >= -128 && g.qmax <= 127 && g.qmin <= 0 && g.qmax >= 0;
+}
+// The AbsMean of Eq. 2 must be positive and finite for s_w = Q_p / AbsMean.
+inline bool absmean_ok(double absmean) { return absmean > 0.0 && isfinite(absmean); }
 
 // Largest wait, in ns, a kernel makes before it records a timeout.
 uint64_t wait_limit_ns();

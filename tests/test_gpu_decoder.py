@@ -20,6 +20,7 @@ import pytest
 import torch
 
 import oracle
+from fused_rule import assert_fused_codes
 from paper_2412_04787_gb300 import inputs
 
 pytestmark = pytest.mark.gpu
@@ -65,9 +66,7 @@ def test_bitlinear_module_matches_oracle(bits_w):
     z = np.zeros((N, K), np.float32)
     c1, m1, _, _ = oracle.update(g, c0, z, z, k, qmin, qmax, 99, 1, 4)
     cg = layer.codes.cpu().numpy().astype(np.int32)
-    diff = cg != c1
-    assert diff.mean() <= 1e-4 + 1.0 / diff.size
-    assert (np.abs(cg - c1.astype(np.int32))[diff] == 1).all()
+    assert_fused_codes(cg, c1)
     assert layer.step == 1 and int(layer.changed.item()) == int((cg != c0).sum())
 
 
@@ -202,9 +201,7 @@ def test_adafactor_module_matches_oracle():
     c1, _ = oracle.adafactor_apply(g, c0, st["a"], st["b"], st["step"], st["decay"], qmin, qmax,
                                    8, 1, 6)
     cg = layer.codes.cpu().numpy().astype(np.int32)
-    diff = cg != c1
-    assert diff.mean() <= 1e-4 + 1.0 / diff.size
-    assert (np.abs(cg - c1.astype(np.int32))[diff] == 1).all()
+    assert_fused_codes(cg, c1)
     assert np.allclose(layer.R.cpu().numpy(), R, rtol=1e-4)
 
 
@@ -250,9 +247,7 @@ def test_bitlinear_module_fp8_matches_oracle():
     z = np.zeros((N, K), np.float32)
     c1, _, _, _ = oracle.update(g, c0, z, z, k, qmin, qmax, 99, 1, 4)
     cg = layer.codes.cpu().numpy().astype(np.int32)
-    diff = cg != c1
-    assert diff.mean() <= 1e-4 + 1.0 / diff.size
-    assert (np.abs(cg - c1.astype(np.int32))[diff] == 1).all()
+    assert_fused_codes(cg, c1)
 
 
 def test_round_to_nearest_loses_small_updates():
