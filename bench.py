@@ -150,7 +150,8 @@ class ClockSampler:
 class MLPStep:
     """Device buffers and the launch sequence of one DQT MLP training step."""
 
-    def __init__(self, dev, seed=1234, fp8=False, optimizer="adamw", packed=False, bits=1.58):
+    def __init__(self, dev, seed=1234, fp8=False, optimizer="adamw", packed=False, bits=1.58,
+                 operands="int8"):
         from paper_2412_04787_gb300 import dqt, inputs
 
         self.dqt = dqt
@@ -159,6 +160,11 @@ class MLPStep:
         self.optimizer = optimizer
         self.packed = packed
         self.bits = bits
+        # int8: the hot-path C ABI on int8 codes (no operand images in HBM for
+        # the forward; dX and dW convert into per-stream workspaces); img: the
+        # *_img calls on images shared between GEMMs (the FP8, packed and
+        # Adafactor variants always take images)
+        self.i8 = operands == "int8" and not fp8 and not packed and optimizer == "adamw"
         self.grid = dqt.grid(bits)
         T = T_TOK
         # two seeded input sets, alternated step by step, so that the
@@ -189,18 +195,22 @@ class MLPStep:
             else:  # Adafactor's factored statistics (row and column means)
                 self.m[name] = torch.zeros(N, dtype=torch.float32, device=dev)
                 self.v[name] = torch.zeros(K, dtype=torch.float32, device=dev)
-            self.W_img[name] = torch.empty((N, K), dtype=torch.bfloat16, device=dev)
+            if not self.i8:  # the int8-operand calls make their images in workspaces
+                self.W_img[name] = torch.empty((N, K), dtype=torch.bfloat16, device=dev)
             if fp8:
                 self.W8[name] = torch.empty((N, K), dtype=torch.uint8, device=dev)
             self.Y[name] = torch.empty((T, N), dtype=torch.bfloat16, device=dev)
             self.dX[name] = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
         # per activation: (scale, forward operand, dequantised bf16 image); the
-        # forward operand is the bf16 code image, or the E4M3 bytes with fp8
+        # forward operand is the int8 codes (no image), the bf16 code image,
+        # or the E4M3 bytes with fp8
         self.aq = {}
         for src, K in (("X", HID), ("H", INTER)):
             self.aq[src] = (torch.empty(T, dtype=torch.float32, device=dev),
-                            torch.empty((T, K), dtype=torch.uint8 if fp8 else torch.bfloat16,
+                            torch.empty((T, K), dtype=(torch.int8 if self.i8 else
+                                                       torch.uint8 if fp8 else torch.bfloat16),
                                         device=dev),
+                            None if self.i8 else
                             torch.empty((T, K), dtype=torch.bfloat16, device=dev))
         self.changed = torch.zeros(3, dtype=torch.int64, device=dev)
         self.af_ws = None
@@ -210,22 +220,54 @@ class MLPStep:
             self.af_ws = [torch.empty(nb, dtype=torch.uint8, device=dev) for _ in range(4)]
         self.sr = {name: dqt.sr_stream(seed=seed, tensor_id=i) for i, (name, _, _) in enumerate(PROJ)}
         self.step_no = 0
-        # weight-gradient workspace (token-sliced last wave), one per stream
-        nbw = max(dqt.dqt_bwd_dw_workspace_size(T, N, K) for _, K, N in PROJ)
-        self.dw_ws = [torch.empty(max(nbw, 16), dtype=torch.uint8, device=dev) if nbw else False
-                      for _ in range(4)]
+        # weight-gradient workspace, one per stream: with int8 operands the
+        # X_tilde image first, then the token-sliced last wave's partials
+        if self.i8:
+            nbw = max(dqt.dqt_bwd_dw_workspace_size(T, N, K) for _, K, N in PROJ)
+            self.dw_ws = [torch.empty(nbw, dtype=torch.uint8, device=dev) for _ in range(4)]
+            nbx = max(dqt.dqt_bwd_dx_workspace_size(N, K) for _, K, N in PROJ)
+            self.dx_ws = [torch.empty(nbx, dtype=torch.uint8, device=dev) for _ in range(4)]
+        else:
+            nbw = max(dqt.dqt_bwd_dw_img_workspace_size(T, N, K) for _, K, N in PROJ)
+            self.dw_ws = [torch.empty(max(nbw, 16), dtype=torch.uint8, device=dev) if nbw else False
+                          for _ in range(4)]
         # kernel launches per step: act_quant 2, weight images 3 (+3 E4M3),
         # forward 3, dX 3, and per projection the dW GEMM, the streaming
         # kernel of its sliced last wave (when the shape has one), and for
-        # Adafactor the five statistics kernels and the step
-        dw = [1 + (1 if dqt.dqt_bwd_dw_workspace_size(T, N, K) > 0 else 0) for _, K, N in PROJ]
-        self.launches_per_step = 2 + 3 + 3 + 3 + sum(dw) + (3 if fp8 else 0)
+        # Adafactor the five statistics kernels and the step; with int8
+        # operands the weight image is made inside each dX call and the
+        # X_tilde image inside each dW call (3 + 3)
+        dw = [1 + (1 if dqt.dqt_bwd_dw_img_workspace_size(T, N, K) > 0 else 0) for _, K, N in PROJ]
+        self.launches_per_step = 2 + 3 + 3 + 3 + sum(dw) + (3 if fp8 else 0) + (3 if self.i8 else 0)
         self.dw_kind = "bwd_dw_adafactor" if optimizer == "adafactor" else "bwd_dw_update"
-        self.kinds = (["act_quant_fp8", "codes_to_fp8", "codes_to_bf16", "fwd_fp8"] if fp8 else
-                      ["act_quant", "codes_to_bf16", "fwd"]) + ["bwd_dx", self.dw_kind]
+        if self.i8:
+            self.kinds = ["act_quant", "fwd", "codes_to_bf16", "bwd_dx", "codes_to_xdq",
+                          self.dw_kind]
+        else:
+            self.kinds = (["act_quant_fp8", "codes_to_fp8", "codes_to_bf16", "fwd_fp8"] if fp8 else
+                          ["act_quant", "codes_to_bf16", "fwd"]) + ["bwd_dx", self.dw_kind]
         if optimizer == "adafactor":
             self.launches_per_step += 3 * 6
         self.streams = [torch.cuda.Stream(device=dev) for _ in range(4)]
+        self.dp = None
+
+    def enable_dp(self):
+        """Data-parallel exchange per weight (one rank per GPU): the dW GEMM
+        writes the rank's fp32 gradient; then a reduce-scatter, the AdamW + SR
+        update of this rank's shard (its moments only, ZeRO-1) and an
+        all-gather of the int8 codes (paper_2412_04787_gb300/dp.py)."""
+        from paper_2412_04787_gb300 import dp
+        if not self.i8:
+            raise SystemExit("the data-parallel exchange runs on the int8-operand AdamW step")
+        self.dp = {}
+        for name, _, _ in PROJ:
+            upd = dp.DataParallelUpdater(self.W[name])
+            self.dp[name] = upd
+            self.W[name] = upd.codes_view()  # the GEMMs read the gathered codes
+            self.m[name] = self.v[name] = None
+        # per projection: the shard's update kernel (the collectives are NCCL's)
+        self.launches_per_step += len(PROJ)
+        self.kinds = [k for k in self.kinds if k != self.dw_kind] + ["bwd_dw", "dp_exchange"]
 
     def run(self, timers=None, serial=False):
         """Enqueue one step.  The launches follow the dependency graph of a
@@ -265,14 +307,21 @@ class MLPStep:
                 e.record(o)
                 stream.wait_event(e)
 
+        # per-kernel timing (timers given) runs the conversion inside each
+        # int8 dX / dW call as its own launch, on the same workspace slices,
+        # so that each kernel is timed alone; the launches are the same
+        parts = timers is not None
+
         def aq(src, stream):
             s_x, q_img, xdq = self.aq[src]
-            if self.fp8:
+            if self.i8:
+                timed("act_quant", stream, lambda: dqt.dqt_act_quant(self.d[src], q_img, s_x))
+            elif self.fp8:
                 timed("act_quant_fp8", stream,
                       lambda: dqt.dqt_act_quant_fp8(self.d[src], q_img, s_x, xdq))
             else:
                 timed("act_quant", stream,
-                      lambda: dqt.dqt_act_quant(self.d[src], None, s_x, q_img, xdq, want=()))
+                      lambda: dqt.dqt_act_quant_images(self.d[src], None, s_x, q_img, xdq, want=()))
 
         def codes(name, stream):
             shape = tuple(self.W_img[name].shape)
@@ -286,20 +335,62 @@ class MLPStep:
 
         def fwd(name, stream):
             s_x, q_img, _ = self.aq["H" if name == "down" else "X"]
-            if self.fp8:
+            if self.i8:
+                timed("fwd", stream, lambda: dqt.dqt_bitlinear_fwd(
+                    q_img, s_x, self.W[name], self.s_w[name], self.grid, Y=self.Y[name]))
+            elif self.fp8:
                 timed("fwd_fp8", stream, lambda: dqt.dqt_bitlinear_fwd_fp8(
                     q_img, s_x, self.W8[name], self.s_w[name], self.grid, Y=self.Y[name]))
             else:
-                timed("fwd", stream, lambda: dqt.dqt_bitlinear_fwd(
+                timed("fwd", stream, lambda: dqt.dqt_bitlinear_fwd_img(
                     q_img, s_x, self.W_img[name], self.s_w[name], self.grid, Y=self.Y[name]))
 
         def dx(name, stream):
-            timed("bwd_dx", stream, lambda: dqt.dqt_bitlinear_bwd_dx(
+            if self.i8:
+                ws = self.dx_ws[s.index(stream)]
+                if parts:
+                    img = ws[: 2 * self.W[name].numel()].view(torch.bfloat16).view(self.W[name].shape)
+                    timed("codes_to_bf16", stream,
+                          lambda: dqt.dqt_codes_to_bf16(self.W[name], img))
+                    timed("bwd_dx", stream, lambda: dqt.dqt_bitlinear_bwd_dx_img(
+                        self.d["dY_" + name], img, self.s_w[name], dX=self.dX[name]))
+                else:
+                    dqt.dqt_bitlinear_bwd_dx(self.d["dY_" + name], self.W[name], self.s_w[name],
+                                             dX=self.dX[name], ws=ws)
+                return
+            timed("bwd_dx", stream, lambda: dqt.dqt_bitlinear_bwd_dx_img(
                 self.d["dY_" + name], self.W_img[name], self.s_w[name], dX=self.dX[name]))
 
         def dw(i, name, stream):
             xdq = self.aq["H" if name == "down" else "X"][2]
             ch = self.changed[i:i + 1]
+            if self.i8 and self.dp:
+                s_x, q, _ = self.aq["H" if name == "down" else "X"]
+                upd = self.dp[name]
+                timed("bwd_dw", stream, lambda: dqt.dqt_bitlinear_bwd_dw_update(
+                    self.d["dY_" + name], q, s_x, None, self.s_w[name], None, None, None, None,
+                    self.grid, dW_out=upd.grad_view(), ws=self.dw_ws[s.index(stream)]))
+                timed("dp_exchange", stream, lambda: upd.step(
+                    self.s_w[name], hp, self.sr[name], self.grid, changed_out=ch))
+                return
+            if self.i8:
+                s_x, q, _ = self.aq["H" if name == "down" else "X"]
+                ws = self.dw_ws[s.index(stream)]
+                if parts:
+                    T_, K_ = q.shape
+                    img_bytes = (T_ * K_ * 2 + 255) // 256 * 256
+                    img = ws[: T_ * K_ * 2].view(torch.bfloat16).view(T_, K_)
+                    rest = ws[img_bytes:]
+                    timed("codes_to_xdq", stream, lambda: dqt.dqt_codes_to_xdq(q, s_x, img))
+                    timed(self.dw_kind, stream, lambda: dqt.dqt_bitlinear_bwd_dw_update_img(
+                        self.d["dY_" + name], img, self.W[name], self.s_w[name], self.m[name],
+                        self.v[name], hp, self.sr[name], self.grid, changed_out=ch,
+                        ws=rest if rest.numel() else False))
+                else:
+                    dqt.dqt_bitlinear_bwd_dw_update(
+                        self.d["dY_" + name], q, s_x, self.W[name], self.s_w[name], self.m[name],
+                        self.v[name], hp, self.sr[name], self.grid, changed_out=ch, ws=ws)
+                return
             if self.optimizer == "adafactor":
                 ws = self.af_ws[s.index(stream)]
                 af = dqt.adafactor(lr=1e-2, step=self.step_no)
@@ -314,7 +405,7 @@ class MLPStep:
                     self.v[name], hp, self.sr[name], changed_out=ch, ws=ws))
             else:
                 ws = self.dw_ws[s.index(stream)]
-                timed(self.dw_kind, stream, lambda: dqt.dqt_bitlinear_bwd_dw_update(
+                timed(self.dw_kind, stream, lambda: dqt.dqt_bitlinear_bwd_dw_update_img(
                     self.d["dY_" + name], xdq, self.W[name], self.s_w[name], self.m[name],
                     self.v[name], hp, self.sr[name], self.grid, changed_out=ch, ws=ws))
 
@@ -325,9 +416,10 @@ class MLPStep:
         # the weight gradient reads: splitting it into two passes, the second
         # beside the forward GEMMs, was measured slower)
         aq("X", s[0])
-        codes("gate", s[1])
-        codes("up", s[2])
-        codes("down", s[3])
+        if not self.i8:
+            codes("gate", s[1])
+            codes("up", s[2])
+            codes("down", s[3])
         after(s[1], s[0])
         after(s[2], s[0])
         fwd("gate", s[1])
@@ -362,16 +454,31 @@ class MLPStep:
         flops["bwd_dx"] = list(flops["fwd"])
         flops["bwd_dw_update"] = list(flops["fwd"])
         flops["bwd_dw_adafactor"] = list(flops["fwd"])
+        flops["bwd_dw"] = list(flops["fwd"])  # gradient only (data-parallel exchange)
         flops["fwd_fp8"] = list(flops["fwd"])
+        # Algorithmic bytes of the method (the a1 quantiser: 2 B read + 1 B
+        # written per element + 4 B per row) and, apart, the bytes of the
+        # operand images the method does not have (the tensor cores' exact
+        # 16-bit copies of integer codes)
         byts = {
-            # bf16 in (2) + bf16 code image (2) + bf16 dequantised image (2) per element, + s_x
-            "act_quant": [T * HID * 6.0 + 4 * T, T * INTER * 6.0 + 4 * T],
-            # bf16 in (2) + E4M3 byte (1) + bf16 dequantised image (2) per element, + s_x8
-            "act_quant_fp8": [T * HID * 5.0 + 4 * T, T * INTER * 5.0 + 4 * T],
+            "act_quant": [T * HID * 3.0 + 4 * T, T * INTER * 3.0 + 4 * T],
+            # bf16 in (2) + E4M3 byte (1) per element, + s_x8
+            "act_quant_fp8": [T * HID * 3.0 + 4 * T, T * INTER * 3.0 + 4 * T],
+            "codes_to_bf16": [0.0 for _ in PROJ],
+            "codes_to_fp8": [0.0 for _ in PROJ],
+            "codes_to_xdq": [0.0 for _ in PROJ],
+        }
+        overhead = {
+            # the bf16 code image and the bf16 dequantised image (2 + 2 B per element)
+            "act_quant": [0.0, 0.0] if self.i8 else [T * HID * 4.0, T * INTER * 4.0],
+            # the bf16 dequantised image (2 B per element)
+            "act_quant_fp8": [T * HID * 2.0, T * INTER * 2.0],
             "codes_to_bf16": [(2.25 if self.packed else 3.0) * K * N for _, K, N in PROJ],
             "codes_to_fp8": [(1.25 if self.packed else 2.0) * K * N for _, K, N in PROJ],
+            # int8 codes read, bf16 image written, s_x read (gate, up: X; down: H)
+            "codes_to_xdq": [3.0 * T * K + 4 * T for _, K, N in PROJ],
         }
-        return flops, byts
+        return flops, byts, overhead
 
 
 def _elapsed(pairs):
@@ -393,24 +500,39 @@ def aggregate_tokens_per_s(world_size, tokens_per_step, steps, max_ms):
     return world_size * tokens_per_step * steps / (max_ms / 1e3)
 
 
+def _free_port():
+    import socket
+    with socket.socket() as so:
+        so.bind(("127.0.0.1", 0))
+        return so.getsockname()[1]
+
+
 def run_gpu(args):
     ws, rank, local = _dist()
-    if ws > 1:
-        import torch.distributed as dist
+    # several ranks: the data-parallel exchange (default) or independent
+    # replicas; --dp exchange on one GPU runs the exchange over a one-rank group
+    dp_mode = args.dp if args.dp != "auto" else ("exchange" if ws > 1 else "none")
+    import torch.distributed as dist
+    if ws > 1 or dp_mode == "exchange":
         torch.cuda.set_device(local)
-        dist.init_process_group("nccl")
+        if "MASTER_ADDR" in os.environ:
+            dist.init_process_group("nccl")
+        else:
+            dist.init_process_group("nccl", init_method="tcp://127.0.0.1:%d" % _free_port(),
+                                    rank=0, world_size=1)
     dev = torch.device("cuda", local if ws > 1 else 0)
     torch.cuda.set_device(dev)
     from paper_2412_04787_gb300 import build as dqt_build
     dqt_build.build()
     st = MLPStep(dev, fp8=args.act == "fp8", optimizer=args.optimizer, packed=args.packed,
-                 bits=args.bits)
+                 bits=args.bits, operands=args.operands)
+    if dp_mode == "exchange":
+        st.enable_dp()
     dqt = st.dqt
     stream = torch.cuda.current_stream()
 
     def barrier():
-        if ws > 1:
-            import torch.distributed as dist
+        if dist.is_initialized():
             dist.barrier()
         torch.cuda.synchronize()
 
@@ -449,7 +571,7 @@ def run_gpu(args):
     serial_ms_step = s0.elapsed_time(s1) / args.steps
 
     # per-kernel live timings
-    flops, byts = st.work()
+    flops, byts, overhead = st.work()
     per = {}
     for k in kinds:
         ts = _elapsed(timers[k])
@@ -458,17 +580,26 @@ def run_gpu(args):
     for k in kinds:
         per[k]["share"] = per[k]["total_ms"] / tot if tot else None
     peaks, pk_kind = _peaks()
+    # The per-kernel region lasts K serial steps (well under a second at the
+    # default K): its kernels run at the burst clock, so the burst peak (a
+    # cuBLAS GEMM timed alone) is the denominator; a region of a second or
+    # more is measured against the sustained (power-capped) peak.
+    serial_ms_total = serial_ms_step * args.steps
+    burst = serial_ms_total < 1000.0
+    peak = peaks["bf16_tflops"] if burst else peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
+    which = "burst" if burst else "sustained"
     dom = max([k for k in kinds if k in flops], key=lambda k: per[k]["total_ms"])
     dom_flops = sum(flops[dom]) * args.steps
     achieved = dom_flops / (per[dom]["total_ms"] / 1e3) / 1e12
-    peak = peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops"))
     # E4M3 dense tensor rate: the measured bf16 rate times the nominal ratio 4.5 / 2.25
     peak8 = 2.0 * peak
     dom_peak = peak8 if dom == "fwd_fp8" else peak
     roofline = {"bound": "tensor", "kernel": dom, "achieved": round(achieved, 1),
                 "peak": dom_peak, "unit": "TFLOP/s", "frac": round(achieved / dom_peak, 4),
-                "peak_kind": ("e4m3 dense sustained = 2 x measured bf16 sustained (nominal ratio)"
-                              if dom == "fwd_fp8" else "bf16 dense sustained, %s" % pk_kind),
+                "peak_kind": ("e4m3 dense %s = 2 x measured bf16 %s (nominal ratio)" % (which, which)
+                              if dom == "fwd_fp8" else
+                              "bf16 dense %s, %s (the per-kernel region lasted %.1f ms)"
+                              % (which, pk_kind, serial_ms_total)),
                 "timing": "mean CUDA-event duration of its launches over a second timed region "
                           "of the same K steps run serially on one stream (%.4f ms/step)" % serial_ms_step,
                 "traffic": (DW_TRAFFIC_BYTES.get(kernel_fingerprint())
@@ -478,15 +609,27 @@ def run_gpu(args):
     kern = {}
     for k in kinds:
         d = dict(per[k])
-        if k in flops:
-            d["tflops"] = sum(flops[k]) * args.steps / (per[k]["total_ms"] / 1e3) / 1e12
+        sec = per[k]["total_ms"] / 1e3
+        if k == "dp_exchange":
+            pass  # reduce-scatter + shard update + all-gather: time only
+        elif k in flops:
+            d["tflops"] = sum(flops[k]) * args.steps / sec / 1e12
             if k == "fwd_fp8":
-                d["frac_of_e4m3_sustained"] = d["tflops"] / peak8
+                d["frac_of_e4m3_" + which] = d["tflops"] / peak8
             else:
-                d["frac_of_bf16_sustained"] = d["tflops"] / peak
+                d["frac_of_bf16_" + which] = d["tflops"] / peak
         else:
-            d["gbs"] = sum(byts[k]) * args.steps / (per[k]["total_ms"] / 1e3) / 1e9
-            d["frac_of_hbm"] = d["gbs"] / peaks["hbm_gbs"]
+            alg = sum(byts[k]) * args.steps
+            ovh = sum(overhead.get(k, [0.0])) * args.steps
+            # frac_of_hbm on the method's own bytes; the operand images'
+            # bytes (overhead) are reported apart
+            d["algorithmic_bytes_per_launch"] = alg / max(1, len(timers[k]))
+            d["overhead_bytes_per_launch"] = ovh / max(1, len(timers[k]))
+            if alg > 0:
+                d["gbs"] = alg / sec / 1e9
+                d["frac_of_hbm"] = d["gbs"] / peaks["hbm_gbs"]
+            d["moved_gbs"] = (alg + ovh) / sec / 1e9
+            d["moved_frac_of_hbm"] = d["moved_gbs"] / peaks["hbm_gbs"]
         kern[k] = {kk: (round(vv, 4) if isinstance(vv, float) else vv) for kk, vv in d.items()}
 
     # ---- e2e: host buffers, H2D inputs + D2H result inside the timed region ----
@@ -575,7 +718,12 @@ def run_gpu(args):
                        "weights": "%s codes, %s" % ("ternary" if st.bits == 1.58 else "%d-bit" % st.bits,
                                                      "2-bit packed" if st.packed else "int8"),
                        "optimizer": st.optimizer,
-                       "parallelism": "replicas" if ws > 1 else "single GPU",
+                       "operands": ("int8 codes through the C ABI" if st.i8 else
+                                    "bf16 / E4M3 operand images"),
+                       "parallelism": (("data parallel over %d GPU(s): reduce-scatter of fp32 dW, "
+                                        "ZeRO-1 sharded AdamW + SR update, all-gather of int8 "
+                                        "codes" % ws) if dp_mode == "exchange" else
+                                       "replicas" if ws > 1 else "single GPU"),
                        "l2": "inputs larger than L2 (step working set ~1.5 GB > 129 MB)"},
             "roofline": roofline, "kernels": kern, "e2e": e2e,
             "gpu_launches": st.launches_per_step * args.steps,
@@ -583,8 +731,7 @@ def run_gpu(args):
             "changed_codes_last_step": [int(x) for x in res_host[(e_steps - 1) % 2].tolist()],
         }
         print(json.dumps(line))
-    if ws > 1:
-        import torch.distributed as dist
+    if dist.is_initialized():
         dist.destroy_process_group()
 
 
@@ -705,7 +852,7 @@ def run_kernel(args):
         X = inputs.normal((T, K), 1.0, seed=1, dtype=torch.bfloat16).to(dev)
         dY = inputs.normal((T, N), 1e-2, seed=2, dtype=torch.bfloat16).to(dev)
         W, s_w = dqt.dqt_absmean_init(inputs.normal((N, K), 0.02, seed=3).to(dev), g)
-        _, s_x, q_img, xdq = dqt.dqt_act_quant(X, want=("Xq_img", "Xdq"))
+        _, s_x, q_img, xdq = dqt.dqt_act_quant_images(X, want=("Xq_img", "Xdq"))
         W_img = dqt.dqt_codes_to_bf16(W)
         m = torch.zeros((N, K), device=dev)
         v = torch.zeros((N, K), device=dev)
@@ -714,24 +861,24 @@ def run_kernel(args):
         hp = dqt.adamw()
         sr = dqt.sr_stream()
         if k == "fwd":
-            fn = lambda: dqt.dqt_bitlinear_fwd(q_img, s_x, W_img, s_w, g, Y=Y)  # noqa: E731
+            fn = lambda: dqt.dqt_bitlinear_fwd_img(q_img, s_x, W_img, s_w, g, Y=Y)  # noqa: E731
         elif k == "bwd_dx":
-            fn = lambda: dqt.dqt_bitlinear_bwd_dx(dY, W_img, s_w, dX=dX)  # noqa: E731
+            fn = lambda: dqt.dqt_bitlinear_bwd_dx_img(dY, W_img, s_w, dX=dX)  # noqa: E731
         elif k == "bwd_dw_update":
-            fn = lambda: dqt.dqt_bitlinear_bwd_dw_update(dY, xdq, W, s_w, m, v, hp, sr, g)  # noqa: E731
+            fn = lambda: dqt.dqt_bitlinear_bwd_dw_update_img(dY, xdq, W, s_w, m, v, hp, sr, g)  # noqa: E731
         elif k == "bwd_dw":  # gradient only (fp32 dW written, no update)
             dW = torch.empty((N, K), dtype=torch.float32, device=dev)
-            fn = lambda: dqt.dqt_bitlinear_bwd_dw_update(dY, xdq, None, s_w, None, None, None,  # noqa: E731
+            fn = lambda: dqt.dqt_bitlinear_bwd_dw_update_img(dY, xdq, None, s_w, None, None, None,  # noqa: E731
                                                          None, g, dW_out=dW)
         elif k == "bwd_dw_unfused":  # gradient to memory, then the standalone update
             dW = torch.empty((N, K), dtype=torch.float32, device=dev)
 
             def fn():
-                dqt.dqt_bitlinear_bwd_dw_update(dY, xdq, None, s_w, None, None, None, None, g,
+                dqt.dqt_bitlinear_bwd_dw_update_img(dY, xdq, None, s_w, None, None, None, None, g,
                                                 dW_out=dW)
                 dqt.dqt_sr_update(dW.view(-1), W.view(-1), s_w, m.view(-1), v.view(-1), hp, sr, g)
         elif k == "act_quant":
-            fn = lambda: dqt.dqt_act_quant(X, None, s_x, q_img, xdq, want=())  # noqa: E731
+            fn = lambda: dqt.dqt_act_quant_images(X, None, s_x, q_img, xdq, want=())  # noqa: E731
         elif k == "bwd_dw_update_packed":
             Wp = dqt.dqt_pack_ternary(W)
             fn = lambda: dqt.dqt_bitlinear_bwd_dw_update_packed(dY, xdq, Wp, s_w, m, v, hp, sr)  # noqa: E731
@@ -982,7 +1129,7 @@ def run_layer(args):
     Y = torch.empty((T, N), dtype=torch.bfloat16, device=dev)
     dX = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
     changed = torch.zeros(1, dtype=torch.int64, device=dev)
-    nbw = dqt.dqt_bwd_dw_workspace_size(T, N, K)
+    nbw = dqt.dqt_bwd_dw_img_workspace_size(T, N, K)
     ws = torch.empty(nbw, dtype=torch.uint8, device=dev) if nbw else None
     row = (dqt.lib().dqt_update_consts_size() + 63) // 64 * 64
     # the graph of KS steps is replayed R times (about a second of GPU time)
@@ -997,10 +1144,10 @@ def run_layer(args):
     ch_host = torch.empty(KS, dtype=torch.int64).pin_memory()
 
     def kernels(i):
-        dqt.dqt_act_quant(X, None, s_x, q_img, xdq, want=())
+        dqt.dqt_act_quant_images(X, None, s_x, q_img, xdq, want=())
         dqt.dqt_codes_to_bf16(W, W_img)
-        dqt.dqt_bitlinear_fwd(q_img, s_x, W_img, s_w, grid, Y=Y)
-        dqt.dqt_bitlinear_bwd_dx(dY, W_img, s_w, dX=dX)
+        dqt.dqt_bitlinear_fwd_img(q_img, s_x, W_img, s_w, grid, Y=Y)
+        dqt.dqt_bitlinear_bwd_dx_img(dY, W_img, s_w, dX=dX)
         dqt.dqt_bitlinear_bwd_dw_update_dev(dY, xdq, W, m, v, uc_dev[i], changed_out=changed,
                                             ws=ws)
 
@@ -1104,6 +1251,12 @@ def main():
     ap.add_argument("--optimizer", default="adamw", choices=["adamw", "adafactor"],
                     help="the DQT optimiser of the BitLinear weights")
     ap.add_argument("--packed", action="store_true", help="2-bit packed ternary code storage")
+    ap.add_argument("--operands", default="int8", choices=["int8", "img"],
+                    help="mlp: the hot-path C ABI on int8 codes (default) or the *_img calls on "
+                         "shared bf16 operand images")
+    ap.add_argument("--dp", default="auto", choices=["auto", "exchange", "replicas"],
+                    help="several ranks: the data-parallel exchange (auto, the default) or "
+                         "independent replicas; exchange on one GPU uses a one-rank group")
     ap.add_argument("--bits", type=float, default=1.58,
                     help="weight grid: 1.58 (ternary, the default) or an integer width 2..8")
     ap.add_argument("--workload", default="mlp", choices=["mlp", "decoder", "layer"],

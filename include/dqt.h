@@ -24,10 +24,14 @@
  * dqt_cross_entropy_fwd_bf16 / _bwd_bf16.
  *
  * GB300 has no int8 tensor-core MMA for sm_103a, so the integer GEMMs run on
- * the bf16 tensor cores over exact bf16 images of the integer codes (every
- * integer in [-256, 256] is exact in bf16; products and partial sums below
- * 2^24 are exact in the fp32 accumulator).  dqt_act_quant writes those images
- * next to the int8 codes, and dqt_codes_to_bf16 makes the weight image.
+ * the 16-bit tensor cores over exact 16-bit images of the integer codes
+ * (every integer in [-256, 256] is exact in bf16 and fp16; products and
+ * partial sums below 2^24 are exact in the fp32 accumulator).  The hot-path
+ * calls take the int8 codes themselves: the forward converts both operands
+ * to fp16 in shared memory inside the GEMM; dX and dW make the bf16 operand
+ * they need in a caller-provided workspace.  The *_img calls take those
+ * images directly (dqt_act_quant_images, dqt_codes_to_bf16) for callers that
+ * share one image between several GEMMs.
  *
  * Conventions for every entry point:
  *   - All data pointers are DEVICE pointers owned by the caller; the library
@@ -87,16 +91,25 @@ typedef struct {
   int64_t step;
 } dqt_adamw_t;
 
-/* Stochastic rounding stream (Eq. 1).  The uniform for element e (flat
- * row-major index into the [N, K] weight) is word e % 4 of
+/* Stochastic rounding stream (Eq. 1).  The uniform for element e (global
+ * flat row-major index into the weight tensor) is word e % 4 of
  * Philox4x32-10(counter = (e/4 low 32, e/4 high 32, step low 32, tensor_id),
  * key = (seed low 32, seed high 32)), U = (word >> 8) * 2^-24; the code rounds
  * up when U < x - floor(x).  round_mode 0 = stochastic rounding (the paper's
- * method); 1 = round to nearest (the absmax-without-SR ablation of Sec. 5.1). */
+ * method); 1 = round to nearest (the absmax-without-SR ablation of Sec. 5.1).
+ * elem0: the global index of the first element a call updates (element i of
+ * the call is global element elem0 + i; for a weight-gradient call, element
+ * (n, k) is elem0 + n K + k).  0 for a whole tensor; a data-parallel rank
+ * that updates the shard [a, b) of a flat weight passes elem0 = a, so the
+ * codes do not depend on how the tensor is sharded.  elem0 >= 0 and a
+ * multiple of 4 (one Philox block per four elements), else DQT_ERR_ARG /
+ * DQT_ERR_ALIGN.  The Adafactor calls need elem0 = 0 (their factored
+ * statistics span the whole matrix). */
 typedef struct {
   uint64_t seed;
   uint32_t tensor_id;
   int32_t round_mode;
+  int64_t elem0;
 } dqt_sr_t;
 
 /* Eq. 3: grid for `bits` in {1.58, 2, 3, ..., 8}.  Host only. */
@@ -153,59 +166,108 @@ int dqt_absmean_init_noalloc(const float* W0, int64_t numel, dqt_grid_t grid, in
 /* Sec. 3.2, activation quantisation "following BitNet", 8 bits per token:
  *   amax[t] = max_k |X[t,k]|,  s_x[t] = 127 / max(amax[t], 1e-5)   (fp32 divide)
  *   Xq[t,k] = Clip[Round(X[t,k] * s_x[t]), -128, 127]              (fp32 multiply, half-to-even)
- *   X       bf16 [T, K] in
- *   Xq      int8 [T, K] out, or NULL
- *   s_x     fp32 [T] out (required)
- *   Xq_img  bf16 [T, K] out, or NULL: the codes as exact bf16 values (forward GEMM operand)
- *   Xdq     bf16 [T, K] out, or NULL: bf16(Xq / s_x), the dequantised activation
- *           X_tilde that the weight gradient uses (backward GEMM operand)
- * At least one of Xq, Xq_img, Xdq must be non-NULL. */
+ *   X       bf16 [T, K] in (16-byte aligned, K a multiple of 8)
+ *   Xq      int8 [T, K] out (8-byte aligned)
+ *   s_x     fp32 [T] out
+ * One pass: 2 bytes read and 1 byte written per element, 4 bytes per row. */
 int dqt_act_quant(const dqt_bf16* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
-                  dqt_bf16* Xq_img, dqt_bf16* Xdq, void* stream);
+                  void* stream);
 
-/* Exact bf16 image of int8 codes: W_img[i] = (bf16) W[i].  numel >= 1. */
+/* dqt_act_quant that can also write the 16-bit GEMM operand images in the
+ * same pass (for the *_img calls):
+ *   Xq      int8 [T, K] out, or NULL
+ *   Xq_img  bf16 [T, K] out, or NULL: the codes as exact bf16 values (forward operand)
+ *   Xdq     bf16 [T, K] out, or NULL: bf16(Xq / s_x), the dequantised activation
+ *           X_tilde that the weight gradient uses (weight-gradient operand)
+ * At least one of Xq, Xq_img, Xdq must be non-NULL; s_x is required. */
+int dqt_act_quant_images(const dqt_bf16* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
+                         dqt_bf16* Xq_img, dqt_bf16* Xdq, void* stream);
+
+/* Exact bf16 image of int8 codes: W_img[i] = (bf16) W[i].  numel >= 1.
+ * (dqt_bitlinear_bwd_dx runs this into its workspace.) */
 int dqt_codes_to_bf16(const int8_t* W, int64_t numel, dqt_bf16* W_img, void* stream);
+
+/* The dequantised activation image from int8 codes: Xdq[t,k] = bf16(Xq[t,k] /
+ * s_x[t]) (correctly rounded fp32 division, then bf16), bit-identical to the
+ * Xdq of dqt_act_quant_images.  (dqt_bitlinear_bwd_dw_update runs this into
+ * its workspace.)  Xq int8 [T, K], s_x fp32 [T], Xdq bf16 [T, K]; K a multiple
+ * of 16; Xq, Xdq 16-byte aligned. */
+int dqt_codes_to_xdq(const int8_t* Xq, const float* s_x, int64_t T, int64_t K, dqt_bf16* Xdq,
+                     void* stream);
 
 /* Sec. 3.2 forward, Y = X_tilde W_tilde^T with X_tilde = Xq / s_x, W_tilde = c / s_w:
  *   acc[t,n] = sum_k Xq[t,k] c[n,k]             exact (int32)
  *   Y[t,n]   = bf16( float(acc) * (1 / (s_x[t] * s_w)) )
- *   Xq_img   bf16 [T, K] exact code image from dqt_act_quant (|value| <= 128)
+ *   Xq       int8 [T, K] activation codes from dqt_act_quant
  *   s_x      fp32 [T]
- *   W_img    bf16 [N, K] exact code image of the weight (dqt_codes_to_bf16)
+ *   W        int8 [N, K] weight codes c
  *   grid     the weight grid; it bounds |c| and so how often the kernel drains its
  *            fp32 accumulator into int32 to keep every partial sum exact
  *   Y        bf16 [T, N] out;  acc_out int32 [T, N] out, or NULL
- * K, N multiples of 8; T >= 1; T, N, K < 2^31. */
-int dqt_bitlinear_fwd(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img,
-                      float s_w, dqt_grid_t grid, int64_t T, int64_t K, int64_t N,
-                      dqt_bf16* Y, int32_t* acc_out, void* stream);
+ * Both operands are converted to exact fp16 values in shared memory inside
+ * the GEMM (2-SM tiles whatever dqt_set_gemm_tiles says); no workspace.
+ * K a multiple of 16 (16-byte int8 rows), N of 8; Xq, W, Y, acc_out 16-byte
+ * aligned; T >= 1; T, N, K < 2^31. */
+int dqt_bitlinear_fwd(const int8_t* Xq, const float* s_x, const int8_t* W, float s_w,
+                      dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
+                      int32_t* acc_out, void* stream);
+
+/* The same forward on the bf16 operand images (dqt_act_quant_images' Xq_img
+ * and dqt_codes_to_bf16's W_img); K, N multiples of 8.  Identical Y and acc. */
+int dqt_bitlinear_fwd_img(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img,
+                          float s_w, dqt_grid_t grid, int64_t T, int64_t K, int64_t N,
+                          dqt_bf16* Y, int32_t* acc_out, void* stream);
 
 /* Backward w.r.t. the input, no straight-through estimator on the weight
  * (the gradient is taken w.r.t. W_tilde itself, Sec. 3.2):
  *   dX[t,k] = bf16( (sum_n dY[t,n] c[n,k]) * (1 / s_w) )   fp32 accumulation
- *   dY bf16 [T, N];  W_img bf16 [N, K];  dX bf16 [T, K] out. */
-int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, int64_t T,
-                         int64_t N, int64_t K, dqt_bf16* dX, void* stream);
+ *   dY bf16 [T, N];  W int8 [N, K] codes;  dX bf16 [T, K] out.
+ * ws: device workspace of at least dqt_bwd_dx_workspace_size(N, K) bytes
+ * (16-byte aligned; it receives the exact bf16 image of the codes, 3 bytes
+ * moved per weight, before the GEMM reads it).  K, N multiples of 8. */
+size_t dqt_bwd_dx_workspace_size(int64_t N, int64_t K);
+int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const int8_t* W, float s_w, int64_t T, int64_t N,
+                         int64_t K, dqt_bf16* dX, void* ws, size_t ws_bytes, void* stream);
+
+/* The same on the weight's bf16 image W_img [N, K] (dqt_codes_to_bf16). */
+int dqt_bitlinear_bwd_dx_img(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, int64_t T,
+                             int64_t N, int64_t K, dqt_bf16* dX, void* stream);
 
 /* Backward w.r.t. the weight fused with the DQT update (Sec. 3.2, Sec. 4.1, Eq. 5):
- *   g[n,k]  = sum_t dY[t,n] Xdq[t,k]              fp32 accumulation in tensor memory
+ *   X_tilde = bf16(Xq / s_x)                       the dequantised activation
+ *   g[n,k]  = sum_t dY[t,n] X_tilde[t,k]           fp32 accumulation in tensor memory
  *   m, v    <- AdamW moments (fp32 [N, K], in place)
  *   x       = c decay - (lr s_w) * m / (sqrt(v) k1 + k2)    (= W' * s_w, see dqt_adamw_t)
  *   c       <- Clip[SR(x), qmin, qmax]  (int8 [N, K], in place; round_mode 1: nearest)
  * The fp32 gradient never reaches memory unless dW_out (fp32 [N, K]) is given
- * (or a split-T workspace is used, see dqt_bwd_dw_workspace_size).
+ * (or the workspace holds token-sliced partials, see below).
  * With W, m and v all NULL only dW_out is written (gradient only).
- *   dY bf16 [T, N];  Xdq bf16 [T, K] from dqt_act_quant;  hp, sr: HOST structs.
+ *   dY bf16 [T, N];  Xq int8 [T, K] and s_x fp32 [T] from dqt_act_quant;
+ *   hp, sr: HOST structs.
  *   changed_out: device int64, or NULL; if given, the number of codes that changed
- *   is ADDED to it (the weight-update frequency of Sec. 5.2). */
-int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W, float s_w,
-                                float* m, float* v, const dqt_adamw_t* hp, const dqt_sr_t* sr,
-                                dqt_grid_t grid, int64_t T, int64_t N, int64_t K,
-                                float* dW_out, unsigned long long* changed_out, void* ws,
-                                size_t ws_bytes, void* stream);
+ *   is ADDED to it (the weight-update frequency of Sec. 5.2).
+ *   ws: device workspace, 16-byte aligned, of at least the bf16 image of X_tilde
+ *   (T K 2 bytes rounded up to 256); dqt_bwd_dw_workspace_size(T, N, K) bytes
+ *   also let the GEMM cut token reductions into slices (as for the _img call).
+ * K a multiple of 16, N of 8. */
+int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const int8_t* Xq, const float* s_x,
+                                int8_t* W, float s_w, float* m, float* v, const dqt_adamw_t* hp,
+                                const dqt_sr_t* sr, dqt_grid_t grid, int64_t T, int64_t N,
+                                int64_t K, float* dW_out, unsigned long long* changed_out,
+                                void* ws, size_t ws_bytes, void* stream);
+size_t dqt_bwd_dw_workspace_size(int64_t T, int64_t N, int64_t K);
+
+/* The same weight gradient + update on the X_tilde image Xdq bf16 [T, K]
+ * (dqt_act_quant_images); ws: the token-slice workspace below, or NULL. */
+int dqt_bitlinear_bwd_dw_update_img(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W,
+                                    float s_w, float* m, float* v, const dqt_adamw_t* hp,
+                                    const dqt_sr_t* sr, dqt_grid_t grid, int64_t T, int64_t N,
+                                    int64_t K, float* dW_out, unsigned long long* changed_out,
+                                    void* ws, size_t ws_bytes, void* stream);
 
 /* Workspace (bytes, 16-byte aligned device memory) that lets
- * dqt_bitlinear_bwd_dw_update cut token reductions into slices:
+ * dqt_bitlinear_bwd_dw_update_img (and the rest of dqt_bitlinear_bwd_dw_update's
+ * workspace) cut token reductions into slices:
  *  - a weight gradient whose output is too small to occupy the GPU (few
  *    256 x 256 tiles, long token reduction) is reduced in token slices
  *    throughout;
@@ -219,7 +281,7 @@ int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t*
  * or fewer bytes, always runs the single fused kernel.  Slicing gives the same
  * update up to the fp32 summation order of the gradient; it is deterministic
  * for a given shape and device. */
-size_t dqt_bwd_dw_workspace_size(int64_t T, int64_t N, int64_t K);
+size_t dqt_bwd_dw_img_workspace_size(int64_t T, int64_t N, int64_t K);
 
 /* The AdamW + SR update of dqt_bitlinear_bwd_dw_update for a gradient already
  * in memory (Eq. 5 as a bandwidth-bound stream; 22 bytes per weight):
@@ -240,9 +302,11 @@ int dqt_sr_update(const float* grad, int8_t* W, float s_w, float* m, float* v,
  *   `out` (host memory, at least dqt_update_consts_size() bytes); the caller
  *   copies it to a 16-byte aligned device buffer ordered before the launch
  *   (e.g. a cudaMemcpyAsync from pinned memory captured in the same graph).
- * The _dev entry points are dqt_bitlinear_bwd_dw_update and dqt_sr_update
+ * The _dev entry points are dqt_bitlinear_bwd_dw_update_img and dqt_sr_update
  * with (hp, sr, grid, s_w) replaced by that device block; results are
- * identical for identical constants.  W, m, v are required. */
+ * identical for identical constants.  W, m, v are required; the weight
+ * gradient takes the X_tilde image Xdq and the token-slice workspace of
+ * dqt_bitlinear_bwd_dw_update_img. */
 size_t dqt_update_consts_size(void);
 int dqt_update_consts(const dqt_adamw_t* hp, const dqt_sr_t* sr, dqt_grid_t grid, float s_w,
                       void* out, size_t out_bytes);
@@ -302,8 +366,9 @@ int dqt_unpack_ternary(const uint8_t* packed, int64_t numel, int8_t* codes, void
  * dqt_codes_to_fp8 do from int8 codes). */
 int dqt_packed_to_bf16(const uint8_t* packed, int64_t numel, dqt_bf16* W_img, void* stream);
 int dqt_packed_to_fp8(const uint8_t* packed, int64_t numel, uint8_t* W8, void* stream);
-/* dqt_sr_update and dqt_bitlinear_bwd_dw_update on packed ternary codes (the
- * grid is [-1, 1]); identical results, 0.25 byte per weight of code traffic. */
+/* dqt_sr_update and dqt_bitlinear_bwd_dw_update_img (X_tilde image Xdq,
+ * token-slice workspace) on packed ternary codes (the grid is [-1, 1]);
+ * identical results, 0.25 byte per weight of code traffic. */
 int dqt_sr_update_packed(const float* grad, uint8_t* Wp, float s_w, float* m, float* v,
                          const dqt_adamw_t* hp, const dqt_sr_t* sr, int64_t numel,
                          unsigned long long* changed_out, void* stream);
@@ -358,7 +423,8 @@ int dqt_adafactor_apply(const float* G, void* W, int32_t packed, const float* a,
                         const float* scalars, int64_t step_t, const dqt_sr_t* sr, dqt_grid_t grid,
                         int64_t N, int64_t K, unsigned long long* changed_out, void* stream);
 /* The whole backward-and-update of a BitLinear weight with Adafactor: the
- * weight gradient dY^T Xdq (fp32, tensor cores) into the workspace, then the
+ * weight gradient dY^T Xdq (fp32, tensor cores; Xdq the X_tilde image of
+ * dqt_act_quant_images) into the workspace, then the
  * statistics and the per-element step above.  Workspace:
  * dqt_bwd_dw_adafactor_workspace_size(T, N, K) bytes (the fp32 gradient, the
  * statistics, and token-slice partials when the GEMM splits the reduction). */

@@ -19,6 +19,7 @@
  *   Sec 4.1 AdamW producing the dense target W'           -> dqt_oracle_adamw_x
  *           (its textbook evaluation order, for the pins)   -> dqt_oracle_adamw_x_textbook
  *   Eq. 5   W_hat = SR(W'), kept on the n-bit grid        -> dqt_oracle_update
+ *           on one data-parallel shard of the weight        -> dqt_oracle_update_shard
  *   Sec 5.1 absmax / round-to-nearest ablation            -> round_mode = 1
  *   Sec 4.1/4.3 FP8 environment: E4M3 activations and      -> dqt_oracle_act_quant_fp8
  *               the forward on E4M3 operands                -> dqt_oracle_fwd_fp8
@@ -447,7 +448,7 @@ static int64_t update_impl(int textbook, const float* g, int8_t* c, float* m, fl
                            const float* consts9, int32_t qmin, int32_t qmax,
                            uint64_t seed, int64_t step, uint32_t tensor_id,
                            int32_t round_mode, const int64_t* rows, int64_t Nr,
-                           int64_t K) {
+                           int64_t K, int64_t elem0) {
   oracle_adamw_consts h;
   oracle_adamw_textbook_consts ht;
   memcpy(&h, consts9, sizeof(h));
@@ -463,7 +464,7 @@ static int64_t update_impl(int textbook, const float* g, int8_t* c, float* m, fl
       if (round_mode == 1) {
         r = (int32_t)rintf(x);
       } else {
-        uint32_t w = dqt_oracle_sr_word(seed, step, tensor_id, n * K + k);
+        uint32_t w = dqt_oracle_sr_word(seed, step, tensor_id, elem0 + n * K + k);
         r = dqt_oracle_sr(x, dqt_oracle_uniform_from_word(w));
       }
       r = clamp_i32(r, qmin, qmax);
@@ -480,7 +481,19 @@ int64_t dqt_oracle_update(const float* g, int8_t* c, float* m, float* v,
                           int32_t round_mode, const int64_t* rows, int64_t Nr,
                           int64_t K) {
   return update_impl(0, g, c, m, v, consts9, qmin, qmax, seed, step, tensor_id, round_mode,
-                     rows, Nr, K);
+                     rows, Nr, K, 0);
+}
+
+/* Eq. 5 on a flat shard of a weight tensor: element i of the n given is    */
+/* global element elem0 + i and draws that element's uniform, so updating  */
+/* the shards of a partition one by one gives the codes of the whole-tensor */
+/* update (the data-parallel form: each rank updates its shard).           */
+int64_t dqt_oracle_update_shard(const float* g, int8_t* c, float* m, float* v,
+                                const float* consts9, int32_t qmin, int32_t qmax,
+                                uint64_t seed, int64_t step, uint32_t tensor_id,
+                                int32_t round_mode, int64_t elem0, int64_t n) {
+  return update_impl(0, g, c, m, v, consts9, qmin, qmax, seed, step, tensor_id, round_mode,
+                     NULL, 1, n, elem0);
 }
 
 /* Eq. 5 with the textbook-order AdamW (tconsts9 from                        */
@@ -491,7 +504,7 @@ int64_t dqt_oracle_update_textbook(const float* g, int8_t* c, float* m, float* v
                                    int32_t round_mode, const int64_t* rows, int64_t Nr,
                                    int64_t K) {
   return update_impl(1, g, c, m, v, tconsts9, qmin, qmax, seed, step, tensor_id, round_mode,
-                     rows, Nr, K);
+                     rows, Nr, K, 0);
 }
 
 /* ======================================================================== */

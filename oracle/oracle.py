@@ -15,6 +15,7 @@ with Stochastic Rounding"):
 * ``adamw_consts``/``adamw_x`` -- Sec. 4.1, AdamW producing the dense target W'
   (``adamw_textbook_consts``/``adamw_x_textbook``: the textbook evaluation order)
 * ``update``                   -- Eq. 5, W_hat = SR(W') clamped onto the grid
+* ``update_shard``             -- Eq. 5 on a flat shard at a global element offset
 * ``pack_ternary``/``unpack_ternary`` -- Sec. 1, 2-bit packed ternary storage
 * ``adafactor_consts``/``adafactor_stats``/``adafactor_x``/``adafactor_apply``
                                -- Sec. 4.3, Adafactor (factored second moment) + SR
@@ -93,6 +94,10 @@ def lib():
         L.dqt_oracle_adamw_x_textbook.argtypes = [_f32p, _i8p, _f32p, _f32p, _f32p, C.c_int64,
                                                   _f32p]
         L.dqt_oracle_adamw_x_textbook.restype = None
+        L.dqt_oracle_update_shard.argtypes = [_f32p, _i8p, _f32p, _f32p, _f32p, C.c_int32,
+                                              C.c_int32, C.c_uint64, C.c_int64, C.c_uint32,
+                                              C.c_int32, C.c_int64, C.c_int64]
+        L.dqt_oracle_update_shard.restype = C.c_int64
         L.dqt_oracle_update_textbook.argtypes = L.dqt_oracle_update.argtypes
         L.dqt_oracle_update_textbook.restype = C.c_int64
         L.dqt_oracle_quantize_weights.argtypes = [_f32p, C.c_int64, C.c_float, C.c_int32,
@@ -360,6 +365,23 @@ def update(g, c, m, v, consts, qmin, qmax, seed, step, tensor_id, round_mode=0,
     fn = lib().dqt_oracle_update_textbook if textbook else lib().dqt_oracle_update
     changed = fn(_p(g, _f32p), _p(c, _i8p), _p(m, _f32p), _p(v, _f32p), _p(k, _f32p), qmin,
                  qmax, seed, step, tensor_id, round_mode, rp, Nr, K)
+    return c, m, v, int(changed)
+
+
+def update_shard(g, c, m, v, consts, qmin, qmax, seed, step, tensor_id, elem0,
+                 round_mode=0):
+    """Eq. 5 on a flat shard: element i is global element elem0 + i of the
+    weight tensor.  Returns (c', m', v', changed) as flat arrays."""
+    g = _c(g, np.float32).ravel()
+    n = g.size
+    c = _c(c, np.int8).ravel().copy()
+    m = _c(m, np.float32).ravel().copy()
+    v = _c(v, np.float32).ravel().copy()
+    assert c.size == n and m.size == n and v.size == n
+    k = _c(consts, np.float32)
+    changed = lib().dqt_oracle_update_shard(_p(g, _f32p), _p(c, _i8p), _p(m, _f32p),
+                                            _p(v, _f32p), _p(k, _f32p), qmin, qmax, seed, step,
+                                            tensor_id, round_mode, int(elem0), n)
     return c, m, v, int(changed)
 
 

@@ -63,7 +63,7 @@ def _quantised(x, x2, act):
     if act == "fp8":
         res = dqt.dqt_act_quant_fp8(x2)
     else:
-        res = dqt.dqt_act_quant(x2, want=("Xq_img", "Xdq"))
+        res = dqt.dqt_act_quant_images(x2, want=("Xq_img", "Xdq"))
     if version is not None:
         c.ref, c.version, c.act, c.result = weakref.ref(x), version, act, res
     else:
@@ -89,7 +89,7 @@ class _BitLinearFn(torch.autograd.Function):
             # the weight's code image serves the forward and, kept until the
             # backward, dX (the codes change only after dX, in the update)
             w_img = layer.weight_bf16()
-            y = dqt.dqt_bitlinear_fwd(q_img, s_x, w_img, float(layer.s_w), layer.grid_tuple)
+            y = dqt.dqt_bitlinear_fwd_img(q_img, s_x, w_img, float(layer.s_w), layer.grid_tuple)
         ctx.save_for_backward(xdq, w_img)
         ctx.layer = layer
         ctx.in_shape = x.shape
@@ -108,7 +108,7 @@ class _BitLinearFn(torch.autograd.Function):
         # the codes have not changed since the forward
         if w_img is None:
             w_img = layer.weight_bf16()
-        dx = dqt.dqt_bitlinear_bwd_dx(dy2, w_img, float(layer.s_w))
+        dx = dqt.dqt_bitlinear_bwd_dx_img(dy2, w_img, float(layer.s_w))
         if layer.update_in_backward:
             layer._dqt_update(dy2, xdq)
         return dx.reshape(ctx.in_shape).to(ctx.in_dtype), None, None
@@ -223,7 +223,7 @@ class DQTBitLinear(torch.nn.Module):
         return hp, sr
 
     def use_device_consts(self, dev_row):
-        """Read the update constants from `dev_row` (a 64-byte row of a device
+        """Read the update constants from `dev_row` (a 16-byte aligned row of a device
         block) when the update kernel runs.  The step then advances in
         prepare_step(), not in backward, so that a captured training step
         replays with a new step each time (AdamW, int8 codes)."""
@@ -260,7 +260,7 @@ class DQTBitLinear(torch.nn.Module):
             return
         self.step += 1
         hp, sr = self._hyper(self.step)
-        dqt.dqt_bitlinear_bwd_dw_update(dy2, xdq, self.codes, self.s_w, self.m, self.v, hp, sr,
+        dqt.dqt_bitlinear_bwd_dw_update_img(dy2, xdq, self.codes, self.s_w, self.m, self.v, hp, sr,
                                         self.grid_tuple, changed_out=self.changed)
 
     def extra_repr(self):

@@ -57,6 +57,8 @@ int make_update_consts(const dqt_adamw_t* hp, const dqt_sr_t* sr, dqt_grid_t g, 
       !isfinite(hp->weight_decay) || !(s_w > 0.0f) || !isfinite(s_w))
     return DQT_ERR_ARG;
   if (sr->round_mode != 0 && sr->round_mode != 1) return DQT_ERR_ARG;
+  if (sr->elem0 < 0) return DQT_ERR_ARG;
+  if (sr->elem0 & 3) return DQT_ERR_ALIGN;
   const double b1 = hp->beta1, b2 = hp->beta2, st = static_cast<double>(hp->step);
   const double bc1 = 1.0 - pow(b1, st), bc2 = 1.0 - pow(b2, st);
   if (!(bc1 > 0.0) || !(bc2 > 0.0)) return DQT_ERR_ARG;
@@ -76,6 +78,9 @@ int make_update_consts(const dqt_adamw_t* hp, const dqt_sr_t* sr, dqt_grid_t g, 
   uc->key0 = static_cast<uint32_t>(sr->seed);
   uc->key1 = static_cast<uint32_t>(sr->seed >> 32);
   uc->round_mode = sr->round_mode;
+  const uint64_t blk0 = static_cast<uint64_t>(sr->elem0) >> 2;
+  uc->blk0_lo = static_cast<uint32_t>(blk0);
+  uc->blk0_hi = static_cast<uint32_t>(blk0 >> 32);
   return DQT_OK;
 }
 
@@ -163,7 +168,17 @@ int dqt_absmean_init(const float* W0, int64_t numel, dqt_grid_t grid, int8_t* co
 }
 
 int dqt_act_quant(const dqt_bf16* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
-                  dqt_bf16* Xq_img, dqt_bf16* Xdq, void* stream) {
+                  void* stream) {
+  if (!X || !Xq || !s_x || T <= 0 || K <= 0) return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim) return DQT_ERR_RANGE;
+  if (K % 8 || !aligned16(X) || (reinterpret_cast<uintptr_t>(Xq) & 7u)) return DQT_ERR_ALIGN;
+  return dqt::launch_act_quant(X, T, K, Xq, s_x, nullptr, nullptr, as_stream(stream))
+             ? DQT_ERR_CUDA
+             : DQT_OK;
+}
+
+int dqt_act_quant_images(const dqt_bf16* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
+                         dqt_bf16* Xq_img, dqt_bf16* Xdq, void* stream) {
   if (!X || !s_x || (!Xq && !Xq_img && !Xdq) || T <= 0 || K <= 0) return DQT_ERR_ARG;
   if (T > kMaxDim || K > kMaxDim) return DQT_ERR_RANGE;
   if (K % 8 || !aligned16(X) || (Xq && (reinterpret_cast<uintptr_t>(Xq) & 7u)) ||
@@ -171,6 +186,14 @@ int dqt_act_quant(const dqt_bf16* X, int64_t T, int64_t K, int8_t* Xq, float* s_
     return DQT_ERR_ALIGN;
   return dqt::launch_act_quant(X, T, K, Xq, s_x, Xq_img, Xdq, as_stream(stream)) ? DQT_ERR_CUDA
                                                                                  : DQT_OK;
+}
+
+int dqt_codes_to_xdq(const int8_t* Xq, const float* s_x, int64_t T, int64_t K, dqt_bf16* Xdq,
+                     void* stream) {
+  if (!Xq || !s_x || !Xdq || T <= 0 || K <= 0) return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim) return DQT_ERR_RANGE;
+  if (K % 16 || !aligned16(Xq) || !aligned16(Xdq)) return DQT_ERR_ALIGN;
+  return dqt::launch_codes_to_xdq(Xq, s_x, T, K, Xdq, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
 int dqt_codes_to_bf16(const int8_t* W, int64_t numel, dqt_bf16* W_img, void* stream) {
@@ -256,16 +279,11 @@ int dqt_rmsnorm_bwd_bf16(const dqt_bf16* x, const dqt_bf16* w, const float* rstd
              : DQT_OK;
 }
 
-int dqt_bitlinear_fwd(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img, float s_w,
-                      dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
-                      int32_t* acc_out, void* stream) {
-  if (!Xq_img || !s_x || !W_img || !Y || T <= 0 || K <= 0 || N <= 0 || !grid_ok(grid) ||
-      !(s_w > 0.0f) || !isfinite(s_w))
-    return DQT_ERR_ARG;
-  if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
-  if (K % 8 || N % 8 || !aligned16(Xq_img) || !aligned16(W_img) || !aligned16(Y) ||
-      (acc_out && !aligned16(acc_out)))
-    return DQT_ERR_ALIGN;
+// The exact integer forward (both operand forms): the reduction is cut into
+// chunks whose partial sums stay <= 2^24 (exact in fp32).
+static int fwd_launch(const void* A, const float* s_x, const void* B, bool i8, float s_w,
+               dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y, int32_t* acc_out,
+               void* stream) {
   const int64_t cmax = grid.qmax > -grid.qmin ? grid.qmax : -grid.qmin;
   const int64_t cm = cmax > 0 ? cmax : 1;
   // |sum| <= K * 128 * max|c| must fit int32.
@@ -279,14 +297,41 @@ int dqt_bitlinear_fwd(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* 
   g.M = static_cast<int>(T);
   g.N = static_cast<int>(N);
   g.Kred = static_cast<int>(K);
-  g.A = Xq_img;
-  g.B = W_img;
+  g.A = A;
+  g.B = B;
+  g.i8 = i8;
   g.chunk_k = static_cast<int>(chunk);
   g.s_x = s_x;
   g.scale = s_w;
   g.out_bf16 = Y;
   g.acc_out = acc_out;
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
+int dqt_bitlinear_fwd(const int8_t* Xq, const float* s_x, const int8_t* W, float s_w,
+                      dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
+                      int32_t* acc_out, void* stream) {
+  if (!Xq || !s_x || !W || !Y || T <= 0 || K <= 0 || N <= 0 || !grid_ok(grid) ||
+      !(s_w > 0.0f) || !isfinite(s_w))
+    return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
+  if (K % 16 || N % 8 || !aligned16(Xq) || !aligned16(W) || !aligned16(Y) ||
+      (acc_out && !aligned16(acc_out)))
+    return DQT_ERR_ALIGN;
+  return fwd_launch(Xq, s_x, W, true, s_w, grid, T, K, N, Y, acc_out, stream);
+}
+
+int dqt_bitlinear_fwd_img(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img,
+                          float s_w, dqt_grid_t grid, int64_t T, int64_t K, int64_t N,
+                          dqt_bf16* Y, int32_t* acc_out, void* stream) {
+  if (!Xq_img || !s_x || !W_img || !Y || T <= 0 || K <= 0 || N <= 0 || !grid_ok(grid) ||
+      !(s_w > 0.0f) || !isfinite(s_w))
+    return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
+  if (K % 8 || N % 8 || !aligned16(Xq_img) || !aligned16(W_img) || !aligned16(Y) ||
+      (acc_out && !aligned16(acc_out)))
+    return DQT_ERR_ALIGN;
+  return fwd_launch(Xq_img, s_x, W_img, false, s_w, grid, T, K, N, Y, acc_out, stream);
 }
 
 int dqt_act_quant_fp8(const dqt_bf16* X, int64_t T, int64_t K, uint8_t* Xq8, float* s_x8,
@@ -332,8 +377,29 @@ int dqt_bitlinear_fwd_fp8(const uint8_t* Xq8, const float* s_x8, const uint8_t* 
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
-int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, int64_t T,
-                         int64_t N, int64_t K, dqt_bf16* dX, void* stream) {
+static inline size_t ws_align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+size_t dqt_bwd_dx_workspace_size(int64_t N, int64_t K) {
+  if (N <= 0 || K <= 0 || N > kMaxDim || K > kMaxDim) return 0;
+  return ws_align256(static_cast<size_t>(N) * static_cast<size_t>(K) * 2u);
+}
+
+int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const int8_t* W, float s_w, int64_t T, int64_t N,
+                         int64_t K, dqt_bf16* dX, void* ws, size_t ws_bytes, void* stream) {
+  if (!dY || !W || !dX || !ws || T <= 0 || N <= 0 || K <= 0 || !(s_w > 0.0f) || !isfinite(s_w))
+    return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
+  if (ws_bytes < dqt_bwd_dx_workspace_size(N, K)) return DQT_ERR_ARG;
+  if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(W) || !aligned16(dX) || !aligned16(ws))
+    return DQT_ERR_ALIGN;
+  // the exact bf16 image of the codes, then the GEMM on it
+  dqt_bf16* W_img = static_cast<dqt_bf16*>(ws);
+  if (dqt::launch_codes_to_bf16(W, N * K, W_img, as_stream(stream))) return DQT_ERR_CUDA;
+  return dqt_bitlinear_bwd_dx_img(dY, W_img, s_w, T, N, K, dX, stream);
+}
+
+int dqt_bitlinear_bwd_dx_img(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, int64_t T,
+                             int64_t N, int64_t K, dqt_bf16* dX, void* stream) {
   if (!dY || !W_img || !dX || T <= 0 || N <= 0 || K <= 0 || !(s_w > 0.0f) || !isfinite(s_w))
     return DQT_ERR_ARG;
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
@@ -353,6 +419,12 @@ int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, i
 
 size_t dqt_bwd_dw_workspace_size(int64_t T, int64_t N, int64_t K) {
   if (T <= 0 || N <= 0 || K <= 0 || T > kMaxDim || N > kMaxDim || K > kMaxDim) return 0;
+  return ws_align256(static_cast<size_t>(T) * static_cast<size_t>(K) * 2u) +
+         dqt_bwd_dw_img_workspace_size(T, N, K);
+}
+
+size_t dqt_bwd_dw_img_workspace_size(int64_t T, int64_t N, int64_t K) {
+  if (T <= 0 || N <= 0 || K <= 0 || T > kMaxDim || N > kMaxDim || K > kMaxDim) return 0;
   if (dqt::gemm_mode() != 0) return 0;
   const int s = dqt::dw_splits(static_cast<int>(N), static_cast<int>(K), static_cast<int>(T));
   if (s > 1) return static_cast<size_t>(s) * static_cast<size_t>(N) * static_cast<size_t>(K) * 4u;
@@ -367,11 +439,41 @@ size_t dqt_bwd_dw_workspace_size(int64_t T, int64_t N, int64_t K) {
   return static_cast<size_t>(sms / 2) * 65536 * sizeof(float);
 }
 
-int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W, float s_w,
-                                float* m, float* v, const dqt_adamw_t* hp, const dqt_sr_t* sr,
-                                dqt_grid_t grid, int64_t T, int64_t N, int64_t K, float* dW_out,
-                                unsigned long long* changed_out, void* ws, size_t ws_bytes,
-                                void* stream) {
+int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const int8_t* Xq, const float* s_x,
+                                int8_t* W, float s_w, float* m, float* v, const dqt_adamw_t* hp,
+                                const dqt_sr_t* sr, dqt_grid_t grid, int64_t T, int64_t N,
+                                int64_t K, float* dW_out, unsigned long long* changed_out,
+                                void* ws, size_t ws_bytes, void* stream) {
+  if (!dY || !Xq || !s_x || !ws || T <= 0 || N <= 0 || K <= 0) return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
+  const size_t img = ws_align256(static_cast<size_t>(T) * static_cast<size_t>(K) * 2u);
+  if (ws_bytes < img) return DQT_ERR_ARG;
+  if (K % 16 || !aligned16(Xq) || !aligned16(ws)) return DQT_ERR_ALIGN;
+  // the argument checks of the GEMM call before anything is launched
+  const bool upd = W || m || v;
+  if (upd && (!W || !m || !v)) return DQT_ERR_ARG;
+  if (!upd && !dW_out) return DQT_ERR_ARG;
+  if (upd) {
+    dqt::UpdateConsts uc;
+    const int rc = make_update_consts(hp, sr, grid, s_w, &uc);
+    if (rc != DQT_OK) return rc;
+  }
+  // X_tilde = bf16(q / s_x) into the workspace, then the GEMM + update on it;
+  // the rest of the workspace serves the token-sliced reduction
+  dqt_bf16* Xdq = static_cast<dqt_bf16*>(ws);
+  if (dqt::launch_codes_to_xdq(Xq, s_x, T, K, Xdq, as_stream(stream))) return DQT_ERR_CUDA;
+  uint8_t* rest = static_cast<uint8_t*>(ws) + img;
+  const size_t rest_bytes = ws_bytes - img;
+  return dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, s_w, m, v, hp, sr, grid, T, N, K, dW_out,
+                                         changed_out, rest_bytes ? rest : nullptr, rest_bytes,
+                                         stream);
+}
+
+int dqt_bitlinear_bwd_dw_update_img(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W,
+                                    float s_w, float* m, float* v, const dqt_adamw_t* hp,
+                                    const dqt_sr_t* sr, dqt_grid_t grid, int64_t T, int64_t N,
+                                    int64_t K, float* dW_out, unsigned long long* changed_out,
+                                    void* ws, size_t ws_bytes, void* stream) {
   const bool upd = W || m || v;
   if (!dY || !Xdq || T <= 0 || N <= 0 || K <= 0) return DQT_ERR_ARG;
   if (upd && (!W || !m || !v)) return DQT_ERR_ARG;
@@ -574,6 +676,7 @@ int make_adafactor_consts(const dqt_adafactor_t* hp, dqt::AdafactorConsts* h) {
 int apply_consts(int64_t step_t, const dqt_sr_t* sr, dqt_grid_t grid, dqt::UpdateConsts* uc) {
   if (!sr || step_t < 1 || !grid_ok(grid)) return DQT_ERR_ARG;
   if (sr->round_mode != 0 && sr->round_mode != 1) return DQT_ERR_ARG;
+  if (sr->elem0 != 0) return DQT_ERR_ARG;  // the statistics span the whole matrix
   *uc = dqt::UpdateConsts{};
   uc->qmin = grid.qmin;
   uc->qmax = grid.qmax;
@@ -640,7 +743,7 @@ size_t dqt_bwd_dw_adafactor_workspace_size(int64_t T, int64_t N, int64_t K) {
   if (T <= 0 || N <= 0 || K <= 0 || T > kMaxDim || N > kMaxDim || K > kMaxDim) return 0;
   const size_t g = align256(static_cast<size_t>(N) * static_cast<size_t>(K) * 4u);
   const size_t st = align256(dqt::adafactor_stats_ws(N, K));
-  return g + st + align256(dqt_bwd_dw_workspace_size(T, N, K));
+  return g + st + align256(dqt_bwd_dw_img_workspace_size(T, N, K));
 }
 
 int dqt_bitlinear_bwd_dw_adafactor(const dqt_bf16* dY, const dqt_bf16* Xdq, void* W,

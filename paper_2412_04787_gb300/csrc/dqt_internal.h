@@ -34,12 +34,14 @@ struct GemmLaunch {
   // Output is M x N, reduced over Kred.
   int M, N, Kred;
   // Operands (bf16, row-major, contiguous):
-  //   FWD: A = Xq_img [M=T, Kred=K],  B = W_img [N, Kred=K]     (both K-major)
+  //   FWD: A = Xq_img [M=T, Kred=K],  B = W_img [N, Kred=K]     (both K-major);
+  //        with i8, A = Xq and B = W, the int8 codes themselves
   //   DX : A = dY     [M=T, Kred=N],  B = W_img [Kred=N, N=K]   (B MN-major)
   //   DW : A = dY     [Kred=T, M=N],  B = Xdq   [Kred=T, N=K]   (both MN-major)
   //   FWD8: A = Xq8 [M=T, Kred=K], B = W8 [N, Kred=K], E4M3 bytes (both K-major)
   const void* A;
   const void* B;
+  bool i8;      // FWD: A and B are int8 codes (converted to fp16 in shared memory)
   int chunk_k;  // FWD: reduction elements per exact fp32 chunk (multiple of 64)
   bool pair;    // use the 2-SM (cta_group::2) kernel (not with drained chunks)
   // Epilogue operands.
@@ -99,6 +101,9 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream);
 int launch_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
                      uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream);
 int launch_codes_to_bf16(const int8_t* W, int64_t numel, uint16_t* W_img, cudaStream_t stream);
+// Xdq[t,k] = bf16(Xq[t,k] / s_x[t]) (the image dqt_act_quant writes); K % 16 == 0.
+int launch_codes_to_xdq(const int8_t* Xq, const float* s_x, int64_t T, int64_t K, uint16_t* Xdq,
+                        cudaStream_t stream);
 // FP8 environment: E4M3 activations with per-token scale 448 / max(amax, 1e-5)
 // (and optionally the dequantised bf16 image), and E4M3 images of weight codes.
 int launch_act_quant_fp8(const uint16_t* X, int64_t T, int64_t K, uint8_t* Xq8, float* s8,

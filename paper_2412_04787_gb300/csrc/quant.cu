@@ -309,6 +309,44 @@ __global__ void __launch_bounds__(256)
   }
 }
 
+// X_tilde = bf16(q / s_x) from int8 activation codes: the operand the
+// weight-gradient GEMM reads.  One warp per token row; the row's 256 possible
+// values come from a per-warp table of correctly rounded fp32 divisions (the
+// table dqt_act_quant uses), so the image is bit-identical to the one it
+// writes.  16 codes (one 16-byte load, two 16-byte stores) per lane step;
+// K % 16 == 0.
+__global__ void __launch_bounds__(256)
+    codes_to_xdq_kernel(const int8_t* __restrict__ Xq, const float* __restrict__ s_x, int T,
+                        int K, uint16_t* __restrict__ Xdq) {
+  __shared__ uint16_t table[8][256];
+  const int wid = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int nv = K >> 4;
+  for (int row = blockIdx.x * 8 + wid; row < T; row += gridDim.x * 8) {
+    const float s = s_x[row];
+    __syncwarp();  // the previous row's lookups are done
+#pragma unroll
+    for (int j = lane; j < 256; j += 32) table[wid][j] = dq_entry<false>(j, s);
+    __syncwarp();
+    const uint4* src = reinterpret_cast<const uint4*>(Xq + static_cast<size_t>(row) * K);
+    uint4* dst = reinterpret_cast<uint4*>(Xdq + static_cast<size_t>(row) * K);
+    for (int v = lane; v < nv; v += 32) {
+      const uint4 u = __ldcs(src + v);
+      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+      uint32_t h[8];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint16_t* t = table[wid];
+        h[2 * j] = t[((w[j] & 0xFFu) ^ 0x80u)] | (uint32_t(t[((w[j] >> 8) & 0xFFu) ^ 0x80u]) << 16);
+        h[2 * j + 1] =
+            t[((w[j] >> 16) & 0xFFu) ^ 0x80u] | (uint32_t(t[(w[j] >> 24) ^ 0x80u]) << 16);
+      }
+      __stcs(dst + 2 * v, make_uint4(h[0], h[1], h[2], h[3]));
+      __stcs(dst + 2 * v + 1, make_uint4(h[4], h[5], h[6], h[7]));
+    }
+  }
+}
+
 // 64 codes per thread per step: four 16-byte loads issued together, then
 // eight 16-byte streaming stores (the image is read by the next kernel only).
 __device__ __forceinline__ void codes16_to_bf16(const uint4 u, uint4& o0, uint4& o1) {
@@ -484,6 +522,18 @@ int launch_aq(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x, u
 int launch_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
                      uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream) {
   return launch_aq<false>(X, T, K, Xq, s_x, Xq_img, Xdq, stream);
+}
+
+int launch_codes_to_xdq(const int8_t* Xq, const float* s_x, int64_t T, int64_t K, uint16_t* Xdq,
+                        cudaStream_t stream) {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t want = (T + 7) / 8;
+  const int blocks = static_cast<int>(want < 4 * sms ? want : 4 * sms);
+  codes_to_xdq_kernel<<<blocks, 256, 0, stream>>>(Xq, s_x, static_cast<int>(T),
+                                                  static_cast<int>(K), Xdq);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
 int launch_act_quant_fp8(const uint16_t* X, int64_t T, int64_t K, uint8_t* Xq8, float* s8,

@@ -61,7 +61,9 @@ __global__ void __launch_bounds__(kThreads)
     float4 v4 = __ldcs(reinterpret_cast<const float4*>(v + e));
     const char4 c4 = packed ? tern_unpack4(Wp[gi]) : *reinterpret_cast<const char4*>(W + e);
     uint4 w = make_uint4(0, 0, 0, 0);
-    if (uc.round_mode == 0) w = sr_words(static_cast<uint64_t>(gi), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
+    if (uc.round_mode == 0)
+      w = sr_words(global_blk(uc, static_cast<uint64_t>(gi)), uc.step_lo, uc.tensor_id, uc.key0,
+                   uc.key1);
     const int32_t a = dqt_update_elem(uc, g4.x, c4.x, m4.x, v4.x, w.x);
     const int32_t b = dqt_update_elem(uc, g4.y, c4.y, m4.y, v4.y, w.y);
     const int32_t c = dqt_update_elem(uc, g4.z, c4.z, m4.z, v4.z, w.z);
@@ -80,7 +82,9 @@ __global__ void __launch_bounds__(kThreads)
   if (blockIdx.x == 0 && threadIdx.x == 0 && (numel & 3)) {
     const int64_t gi = ngroups;
     uint4 w = make_uint4(0, 0, 0, 0);
-    if (uc.round_mode == 0) w = sr_words(static_cast<uint64_t>(gi), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
+    if (uc.round_mode == 0)
+      w = sr_words(global_blk(uc, static_cast<uint64_t>(gi)), uc.step_lo, uc.tensor_id, uc.key0,
+                   uc.key1);
     const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
     const char4 pc = packed ? tern_unpack4(Wp[gi]) : make_char4(0, 0, 0, 0);
     int32_t pr[4] = {0, 0, 0, 0};  // packed: the unused fields of the last byte stay 0
@@ -162,7 +166,8 @@ __global__ void __launch_bounds__(kThreads)
     const char4 c0 = packed ? tern_unpack4(Wp[e >> 2]) : *reinterpret_cast<const char4*>(W + e);
     uint4 w = make_uint4(0, 0, 0, 0);
     if (uc.round_mode == 0)
-      w = sr_words(static_cast<uint64_t>(e >> 2), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
+      w = sr_words(global_blk(uc, static_cast<uint64_t>(e >> 2)), uc.step_lo, uc.tensor_id, uc.key0,
+                   uc.key1);
     const int32_t a = dqt_update_elem(uc, g4.x, c0.x, m4.x, v4.x, w.x);
     const int32_t b = dqt_update_elem(uc, g4.y, c0.y, m4.y, v4.y, w.y);
     const int32_t c = dqt_update_elem(uc, g4.z, c0.z, m4.z, v4.z, w.z);

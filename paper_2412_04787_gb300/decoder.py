@@ -180,7 +180,8 @@ class DQTDecoder(torch.nn.Module):
     # ---- CUDA-graph replay of whole training steps ----
     def enable_graph_updates(self):
         """Move the per-step update constants of every BitLinear to one device
-        block (64-byte rows) fed from two pinned host blocks.  Per step:
+        block (one row per layer, dqt_update_consts_size() bytes rounded up to a
+        multiple of 64) fed from two pinned host blocks.  Per step:
         prepare_step(slot) fills host block `slot` on the host, then
         upload_update_consts(slot) copies it, stream-ordered, ahead of the
         step's kernels (e.g. right before replaying a captured step).  Alternate

@@ -31,6 +31,9 @@ EXPORTED = [
     "dqt_rope_bf16", "dqt_cross_entropy_fwd_bf16", "dqt_cross_entropy_bwd_bf16",
     "dqt_swiglu_bf16", "dqt_swiglu_bwd_bf16", "dqt_rmsnorm_bf16",
     "dqt_rmsnorm_bwd_workspace_size", "dqt_rmsnorm_bwd_bf16",
+    "dqt_act_quant_images", "dqt_bitlinear_fwd_img", "dqt_bitlinear_bwd_dx_img",
+    "dqt_bwd_dx_workspace_size", "dqt_bitlinear_bwd_dw_update_img",
+    "dqt_bwd_dw_img_workspace_size", "dqt_codes_to_xdq",
 ]
 
 
@@ -50,7 +53,8 @@ class dqt_adamw_t(C.Structure):
 
 
 class dqt_sr_t(C.Structure):
-    _fields_ = [("seed", C.c_uint64), ("tensor_id", C.c_uint32), ("round_mode", C.c_int32)]
+    _fields_ = [("seed", C.c_uint64), ("tensor_id", C.c_uint32), ("round_mode", C.c_int32),
+                ("elem0", C.c_int64)]
 
 
 class dqt_adafactor_t(C.Structure):
@@ -83,17 +87,29 @@ def lib():
                                        _sz, _vp]
         L.dqt_absmean_init_noalloc.argtypes = [_vp, _i64, dqt_grid_t, _vp,
                                                C.POINTER(C.c_float), _vp]
-        L.dqt_act_quant.argtypes = [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp]
+        L.dqt_act_quant.argtypes = [_vp, _i64, _i64, _vp, _vp, _vp]
+        L.dqt_act_quant_images.argtypes = [_vp, _i64, _i64, _vp, _vp, _vp, _vp, _vp]
         L.dqt_codes_to_bf16.argtypes = [_vp, _i64, _vp, _vp]
+        L.dqt_codes_to_xdq.argtypes = [_vp, _vp, _i64, _i64, _vp, _vp]
         L.dqt_bitlinear_fwd.argtypes = [_vp, _vp, _vp, _f32, dqt_grid_t, _i64, _i64, _i64, _vp,
                                         _vp, _vp]
-        L.dqt_bitlinear_bwd_dx.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp]
-        L.dqt_bitlinear_bwd_dw_update.argtypes = [_vp, _vp, _vp, _f32, _vp, _vp,
+        L.dqt_bitlinear_fwd_img.argtypes = L.dqt_bitlinear_fwd.argtypes
+        L.dqt_bitlinear_bwd_dx.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp, _sz, _vp]
+        L.dqt_bitlinear_bwd_dx_img.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp]
+        L.dqt_bwd_dx_workspace_size.argtypes = [_i64, _i64]
+        L.dqt_bwd_dx_workspace_size.restype = _sz
+        L.dqt_bitlinear_bwd_dw_update.argtypes = [_vp, _vp, _vp, _vp, _f32, _vp, _vp,
                                                   C.POINTER(dqt_adamw_t), C.POINTER(dqt_sr_t),
                                                   dqt_grid_t, _i64, _i64, _i64, _vp, _vp, _vp,
                                                   _sz, _vp]
+        L.dqt_bitlinear_bwd_dw_update_img.argtypes = [_vp, _vp, _vp, _f32, _vp, _vp,
+                                                      C.POINTER(dqt_adamw_t),
+                                                      C.POINTER(dqt_sr_t), dqt_grid_t, _i64,
+                                                      _i64, _i64, _vp, _vp, _vp, _sz, _vp]
         L.dqt_bwd_dw_workspace_size.argtypes = [_i64, _i64, _i64]
         L.dqt_bwd_dw_workspace_size.restype = _sz
+        L.dqt_bwd_dw_img_workspace_size.argtypes = [_i64, _i64, _i64]
+        L.dqt_bwd_dw_img_workspace_size.restype = _sz
         L.dqt_sr_update.argtypes = [_vp, _vp, _f32, _vp, _vp, C.POINTER(dqt_adamw_t),
                                     C.POINTER(dqt_sr_t), dqt_grid_t, _i64, _vp, _vp]
         L.dqt_update_consts_size.argtypes = []
@@ -142,6 +158,7 @@ def lib():
         for name in EXPORTED:
             if name not in ("dqt_status_string", "dqt_absmean_workspace_size",
                             "dqt_update_consts_size", "dqt_bwd_dw_workspace_size",
+                            "dqt_bwd_dw_img_workspace_size", "dqt_bwd_dx_workspace_size",
                             "dqt_adafactor_workspace_size",
                             "dqt_bwd_dw_adafactor_workspace_size",
                             "dqt_rmsnorm_bwd_workspace_size"):
@@ -201,8 +218,10 @@ def adamw(lr=1e-3, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.0, step=1):
     return dqt_adamw_t(lr, beta1, beta2, eps, weight_decay, step)
 
 
-def sr_stream(seed=1234, tensor_id=0, round_mode=0):
-    return dqt_sr_t(seed, tensor_id, round_mode)
+def sr_stream(seed=1234, tensor_id=0, round_mode=0, elem0=0):
+    """The SR stream of a tensor; elem0 = global index of the call's first
+    element (a data-parallel shard's offset into the flat weight)."""
+    return dqt_sr_t(seed, tensor_id, round_mode, elem0)
 
 
 # ---------------------------------------------------------------------------
@@ -235,10 +254,28 @@ def dqt_absmean_init(W0, bits_or_grid, codes=None, stream=None):
     return codes, float(s.value)
 
 
-def dqt_act_quant(X, Xq=None, s_x=None, Xq_img=None, Xdq=None, want=("Xq", "Xq_img", "Xdq"),
-                  stream=None):
-    """Sec. 3.2 activation codes.  Outputs not passed are allocated if named in
-    ``want``.  Returns (Xq, s_x, Xq_img, Xdq), None for outputs not produced."""
+def dqt_act_quant(X, Xq=None, s_x=None, stream=None):
+    """Sec. 3.2 activation codes: returns (Xq int8 [T, K], s_x fp32 [T])."""
+    _need(X, "X", torch.bfloat16)
+    if X.dim() != 2:
+        raise ValueError("X must be [T, K]")
+    T, K = X.shape
+    if Xq is None:
+        Xq = torch.empty((T, K), dtype=torch.int8, device=X.device)
+    if s_x is None:
+        s_x = torch.empty(T, dtype=torch.float32, device=X.device)
+    _need(Xq, "Xq", torch.int8, (T, K))
+    _need(s_x, "s_x", torch.float32, (T,))
+    _check(lib().dqt_act_quant(_ptr(X), T, K, _ptr(Xq), _ptr(s_x), _stream(stream)),
+           "dqt_act_quant")
+    return Xq, s_x
+
+
+def dqt_act_quant_images(X, Xq=None, s_x=None, Xq_img=None, Xdq=None,
+                         want=("Xq", "Xq_img", "Xdq"), stream=None):
+    """Activation codes and the bf16 operand images of the *_img calls.
+    Outputs not passed are allocated if named in ``want``.  Returns (Xq, s_x,
+    Xq_img, Xdq), None for outputs not produced."""
     _need(X, "X", torch.bfloat16)
     if X.dim() != 2:
         raise ValueError("X must be [T, K]")
@@ -256,8 +293,8 @@ def dqt_act_quant(X, Xq=None, s_x=None, Xq_img=None, Xdq=None, want=("Xq", "Xq_i
     _need(s_x, "s_x", torch.float32, (T,))
     _opt(Xq_img, "Xq_img", torch.bfloat16, (T, K))
     _opt(Xdq, "Xdq", torch.bfloat16, (T, K))
-    _check(lib().dqt_act_quant(_ptr(X), T, K, _ptr(Xq), _ptr(s_x), _ptr(Xq_img), _ptr(Xdq),
-                               _stream(stream)), "dqt_act_quant")
+    _check(lib().dqt_act_quant_images(_ptr(X), T, K, _ptr(Xq), _ptr(s_x), _ptr(Xq_img),
+                                      _ptr(Xdq), _stream(stream)), "dqt_act_quant_images")
     return Xq, s_x, Xq_img, Xdq
 
 
@@ -271,7 +308,39 @@ def dqt_codes_to_bf16(W, W_img=None, stream=None):
     return W_img
 
 
-def dqt_bitlinear_fwd(Xq_img, s_x, W_img, s_w, bits_or_grid, Y=None, acc_out=None, stream=None):
+def dqt_codes_to_xdq(Xq, s_x, Xdq=None, stream=None):
+    """X_tilde = bf16(Xq / s_x), the weight-gradient operand image."""
+    _need(Xq, "Xq", torch.int8)
+    T, K = Xq.shape
+    _need(s_x, "s_x", torch.float32, (T,))
+    if Xdq is None:
+        Xdq = torch.empty((T, K), dtype=torch.bfloat16, device=Xq.device)
+    _need(Xdq, "Xdq", torch.bfloat16, (T, K))
+    _check(lib().dqt_codes_to_xdq(_ptr(Xq), _ptr(s_x), T, K, _ptr(Xdq), _stream(stream)),
+           "dqt_codes_to_xdq")
+    return Xdq
+
+
+def dqt_bitlinear_fwd(Xq, s_x, W, s_w, bits_or_grid, Y=None, acc_out=None, stream=None):
+    """Sec. 3.2 forward on the int8 codes (converted to fp16 inside the GEMM)."""
+    _need(Xq, "Xq", torch.int8)
+    T, K = Xq.shape
+    _need(W, "W", torch.int8)
+    N = W.shape[0]
+    _need(W, "W", torch.int8, (N, K))
+    _need(s_x, "s_x", torch.float32, (T,))
+    if Y is None:
+        Y = torch.empty((T, N), dtype=torch.bfloat16, device=Xq.device)
+    _need(Y, "Y", torch.bfloat16, (T, N))
+    _opt(acc_out, "acc_out", torch.int32, (T, N))
+    _check(lib().dqt_bitlinear_fwd(_ptr(Xq), _ptr(s_x), _ptr(W), float(s_w),
+                                   _grid(bits_or_grid), T, K, N, _ptr(Y), _ptr(acc_out),
+                                   _stream(stream)), "dqt_bitlinear_fwd")
+    return Y
+
+
+def dqt_bitlinear_fwd_img(Xq_img, s_x, W_img, s_w, bits_or_grid, Y=None, acc_out=None,
+                          stream=None):
     _need(Xq_img, "Xq_img", torch.bfloat16)
     T, K = Xq_img.shape
     _need(W_img, "W_img", torch.bfloat16)
@@ -282,13 +351,39 @@ def dqt_bitlinear_fwd(Xq_img, s_x, W_img, s_w, bits_or_grid, Y=None, acc_out=Non
         Y = torch.empty((T, N), dtype=torch.bfloat16, device=Xq_img.device)
     _need(Y, "Y", torch.bfloat16, (T, N))
     _opt(acc_out, "acc_out", torch.int32, (T, N))
-    _check(lib().dqt_bitlinear_fwd(_ptr(Xq_img), _ptr(s_x), _ptr(W_img), float(s_w),
-                                   _grid(bits_or_grid), T, K, N, _ptr(Y), _ptr(acc_out),
-                                   _stream(stream)), "dqt_bitlinear_fwd")
+    _check(lib().dqt_bitlinear_fwd_img(_ptr(Xq_img), _ptr(s_x), _ptr(W_img), float(s_w),
+                                       _grid(bits_or_grid), T, K, N, _ptr(Y), _ptr(acc_out),
+                                       _stream(stream)), "dqt_bitlinear_fwd_img")
     return Y
 
 
-def dqt_bitlinear_bwd_dx(dY, W_img, s_w, dX=None, stream=None):
+def dqt_bwd_dx_workspace_size(N, K):
+    return int(lib().dqt_bwd_dx_workspace_size(N, K))
+
+
+def dqt_bitlinear_bwd_dx(dY, W, s_w, dX=None, ws=None, stream=None):
+    """dX = dY W_tilde from the int8 codes; `ws` (uint8 CUDA tensor of
+    dqt_bwd_dx_workspace_size bytes) receives their bf16 image, allocated if
+    None."""
+    _need(dY, "dY", torch.bfloat16)
+    T, N = dY.shape
+    _need(W, "W", torch.int8)
+    K = W.shape[1]
+    _need(W, "W", torch.int8, (N, K))
+    if dX is None:
+        dX = torch.empty((T, K), dtype=torch.bfloat16, device=dY.device)
+    _need(dX, "dX", torch.bfloat16, (T, K))
+    nws = lib().dqt_bwd_dx_workspace_size(N, K)
+    if ws is None:
+        ws = torch.empty(nws, dtype=torch.uint8, device=dY.device)
+    _need(ws, "ws", torch.uint8)
+    _check(lib().dqt_bitlinear_bwd_dx(_ptr(dY), _ptr(W), float(s_w), T, N, K, _ptr(dX),
+                                      _ptr(ws), ws.numel(), _stream(stream)),
+           "dqt_bitlinear_bwd_dx")
+    return dX
+
+
+def dqt_bitlinear_bwd_dx_img(dY, W_img, s_w, dX=None, stream=None):
     _need(dY, "dY", torch.bfloat16)
     T, N = dY.shape
     _need(W_img, "W_img", torch.bfloat16)
@@ -297,15 +392,15 @@ def dqt_bitlinear_bwd_dx(dY, W_img, s_w, dX=None, stream=None):
     if dX is None:
         dX = torch.empty((T, K), dtype=torch.bfloat16, device=dY.device)
     _need(dX, "dX", torch.bfloat16, (T, K))
-    _check(lib().dqt_bitlinear_bwd_dx(_ptr(dY), _ptr(W_img), float(s_w), T, N, K, _ptr(dX),
-                                      _stream(stream)), "dqt_bitlinear_bwd_dx")
+    _check(lib().dqt_bitlinear_bwd_dx_img(_ptr(dY), _ptr(W_img), float(s_w), T, N, K,
+                                          _ptr(dX), _stream(stream)), "dqt_bitlinear_bwd_dx_img")
     return dX
 
 
 def _dw_workspace(T, N, K, device, ws):
     if ws is False:
         return None, 0
-    need = lib().dqt_bwd_dw_workspace_size(T, N, K)
+    need = lib().dqt_bwd_dw_img_workspace_size(T, N, K)
     if need == 0:
         return None, 0
     if ws is None:
@@ -318,12 +413,49 @@ def dqt_bwd_dw_workspace_size(T, N, K):
     return int(lib().dqt_bwd_dw_workspace_size(T, N, K))
 
 
-def dqt_bitlinear_bwd_dw_update(dY, Xdq, W, s_w, m, v, hp, sr, bits_or_grid, dW_out=None,
+def dqt_bwd_dw_img_workspace_size(T, N, K):
+    return int(lib().dqt_bwd_dw_img_workspace_size(T, N, K))
+
+
+def dqt_bitlinear_bwd_dw_update(dY, Xq, s_x, W, s_w, m, v, hp, sr, bits_or_grid, dW_out=None,
                                 changed_out=None, ws=None, stream=None):
-    """Fused dW GEMM + AdamW + stochastic rounding; W, m, v updated in place.
-    With W = m = v = None only dW_out is computed.  `ws`: split-T workspace
-    (uint8 CUDA tensor of dqt_bwd_dw_workspace_size bytes); None allocates it
-    when the shape benefits, False forces the single fused kernel."""
+    """Weight gradient from the int8 activation codes + AdamW + stochastic
+    rounding; W, m, v updated in place (W = m = v = None: dW_out only).
+    `ws`: uint8 CUDA tensor of at least the X_tilde image (T K 2 bytes,
+    rounded up to 256) -- dqt_bwd_dw_workspace_size bytes also enable the
+    token-sliced reduction; None allocates the full size, False only the
+    image (the single fused kernel)."""
+    _need(dY, "dY", torch.bfloat16)
+    T, N = dY.shape
+    _need(Xq, "Xq", torch.int8)
+    K = Xq.shape[1]
+    _need(Xq, "Xq", torch.int8, (T, K))
+    _need(s_x, "s_x", torch.float32, (T,))
+    _opt(W, "W", torch.int8, (N, K))
+    _opt(m, "m", torch.float32, (N, K))
+    _opt(v, "v", torch.float32, (N, K))
+    _opt(dW_out, "dW_out", torch.float32, (N, K))
+    _opt(changed_out, "changed_out", torch.int64, (1,))
+    if ws is None or ws is False:
+        n = (lib().dqt_bwd_dw_workspace_size(T, N, K) if ws is None
+             else (T * K * 2 + 255) // 256 * 256)
+        ws = torch.empty(n, dtype=torch.uint8, device=dY.device)
+    _need(ws, "ws", torch.uint8)
+    _check(lib().dqt_bitlinear_bwd_dw_update(
+        _ptr(dY), _ptr(Xq), _ptr(s_x), _ptr(W), float(s_w), _ptr(m), _ptr(v),
+        C.byref(hp) if hp is not None else None, C.byref(sr) if sr is not None else None,
+        _grid(bits_or_grid), T, N, K, _ptr(dW_out), _ptr(changed_out), _ptr(ws), ws.numel(),
+        _stream(stream)), "dqt_bitlinear_bwd_dw_update")
+    return W
+
+
+def dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, s_w, m, v, hp, sr, bits_or_grid, dW_out=None,
+                                    changed_out=None, ws=None, stream=None):
+    """Fused dW GEMM + AdamW + stochastic rounding on the X_tilde image Xdq;
+    W, m, v updated in place.  With W = m = v = None only dW_out is computed.
+    `ws`: split-T workspace (uint8 CUDA tensor of dqt_bwd_dw_img_workspace_size
+    bytes); None allocates it when the shape benefits, False forces the single
+    fused kernel."""
     _need(dY, "dY", torch.bfloat16)
     T, N = dY.shape
     _need(Xdq, "Xdq", torch.bfloat16)
@@ -335,11 +467,11 @@ def dqt_bitlinear_bwd_dw_update(dY, Xdq, W, s_w, m, v, hp, sr, bits_or_grid, dW_
     _opt(dW_out, "dW_out", torch.float32, (N, K))
     _opt(changed_out, "changed_out", torch.int64, (1,))
     ws, nws = _dw_workspace(T, N, K, dY.device, ws)
-    _check(lib().dqt_bitlinear_bwd_dw_update(
+    _check(lib().dqt_bitlinear_bwd_dw_update_img(
         _ptr(dY), _ptr(Xdq), _ptr(W), float(s_w), _ptr(m), _ptr(v),
         C.byref(hp) if hp is not None else None, C.byref(sr) if sr is not None else None,
         _grid(bits_or_grid), T, N, K, _ptr(dW_out), _ptr(changed_out), _ptr(ws), nws,
-        _stream(stream)), "dqt_bitlinear_bwd_dw_update")
+        _stream(stream)), "dqt_bitlinear_bwd_dw_update_img")
     return W
 
 

@@ -65,15 +65,24 @@ def test_argument_validation_without_launch(L):
     A = _p(0x10000)  # never dereferenced: validation fails before any CUDA call
     # null pointers
     assert L.dqt_bitlinear_fwd(None, A, A, 1.0, g, 4, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
-    assert L.dqt_bitlinear_bwd_dx(A, None, 1.0, 4, 8, 8, A, None) == dqt.DQT_ERR_ARG
-    assert L.dqt_act_quant(A, 4, 8, None, A, None, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_bwd_dx(A, None, 1.0, 4, 8, 8, A, A, 1 << 20, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_bwd_dx(A, A, 1.0, 4, 8, 8, A, None, 1 << 20, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_act_quant(A, 4, 8, None, A, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_act_quant_images(A, 4, 8, None, A, None, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_fwd_img(None, A, A, 1.0, g, 4, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
     # sizes
     assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g, 0, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
-    assert L.dqt_act_quant(A, -1, 8, A, A, None, None, None) == dqt.DQT_ERR_ARG
-    # K, N multiples of 8 and 16-byte alignment
-    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g, 4, 12, 8, A, None, None) == dqt.DQT_ERR_ALIGN
-    assert L.dqt_bitlinear_bwd_dx(A, A, 1.0, 4, 8, 20, A, None) == dqt.DQT_ERR_ALIGN
-    assert L.dqt_bitlinear_fwd(_p(0x10004), A, A, 1.0, g, 4, 8, 8, A, None, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_act_quant(A, -1, 8, A, A, None) == dqt.DQT_ERR_ARG
+    # the dX workspace must hold the weight's bf16 image
+    assert L.dqt_bwd_dx_workspace_size(8, 8) >= 8 * 8 * 2
+    assert L.dqt_bitlinear_bwd_dx(A, A, 1.0, 4, 8, 8, A, A, 64, None) == dqt.DQT_ERR_ARG
+    # int8 rows of the forward: K a multiple of 16; bf16 rows: K, N multiples
+    # of 8; 16-byte alignment
+    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g, 4, 24, 8, A, None, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_bitlinear_fwd_img(A, A, A, 1.0, g, 4, 12, 8, A, None, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_bitlinear_bwd_dx(A, A, 1.0, 4, 8, 20, A, A, 1 << 20, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_bitlinear_bwd_dx_img(A, A, 1.0, 4, 8, 20, A, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_bitlinear_fwd(_p(0x10004), A, A, 1.0, g, 4, 16, 8, A, None, None) == dqt.DQT_ERR_ALIGN
     # bad grid / scale
     assert L.dqt_bitlinear_fwd(A, A, A, 1.0, dqt.dqt_grid_t(2, 1), 4, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
     assert L.dqt_bitlinear_fwd(A, A, A, 1.0, dqt.dqt_grid_t(-129, 1), 4, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
@@ -90,9 +99,15 @@ def test_update_argument_validation(L):
     sr = dqt.sr_stream()
     ok = C.byref(hp), C.byref(sr)
     # partial state
-    assert L.dqt_bitlinear_bwd_dw_update(A, A, A, 1.0, None, A, *ok, g, 4, 8, 8, None, None, None, 0, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_bwd_dw_update_img(A, A, A, 1.0, None, A, *ok, g, 4, 8, 8, None, None, None, 0, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_bwd_dw_update(A, A, A, A, 1.0, None, A, *ok, g, 4, 8, 16, None, None, A, 1 << 20, None) == dqt.DQT_ERR_ARG
     # gradient-only mode needs dW_out
-    assert L.dqt_bitlinear_bwd_dw_update(A, A, None, 1.0, None, None, *ok, g, 4, 8, 8, None, None, None, 0, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_bwd_dw_update_img(A, A, None, 1.0, None, None, *ok, g, 4, 8, 8, None, None, None, 0, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_bwd_dw_update(A, A, A, None, 1.0, None, None, *ok, g, 4, 8, 16, None, None, A, 1 << 20, None) == dqt.DQT_ERR_ARG
+    # the int8 call needs the X_tilde image in its workspace, 16-byte int8 rows
+    assert L.dqt_bwd_dw_workspace_size(4, 8, 16) >= 4 * 16 * 2
+    assert L.dqt_bitlinear_bwd_dw_update(A, A, A, A, 1.0, A, A, *ok, g, 4, 8, 16, None, None, A, 64, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_bwd_dw_update(A, A, A, A, 1.0, A, A, *ok, g, 4, 8, 24, None, None, A, 1 << 20, None) == dqt.DQT_ERR_ALIGN
     bad = dqt.adamw(step=0)
     assert L.dqt_sr_update(A, A, 1.0, A, A, C.byref(bad), C.byref(sr), g, 16, None, None) == dqt.DQT_ERR_ARG
     bad = dqt.adamw(beta1=1.0)
@@ -193,3 +208,28 @@ def test_decoder_support_argument_validation(L):
     assert L.dqt_rmsnorm_bf16(A, A, C.c_float(-1.0), 4, 64, A, A, None) == dqt.DQT_ERR_ARG
     assert L.dqt_rmsnorm_bwd_workspace_size(4, 4096) == 0
     assert L.dqt_rmsnorm_bwd_bf16(A, A, A, A, 4, 64, A, A, None, 0, None) == dqt.DQT_ERR_ARG
+
+
+def test_sr_stream_offset_validation(L):
+    """elem0 of the SR stream: negative -> DQT_ERR_ARG, not a multiple of 4 ->
+    DQT_ERR_ALIGN (one Philox block per four elements); Adafactor's calls need
+    elem0 = 0.  The host block of constants records elem0 / 4."""
+    g = dqt.dqt_grid_t(-1, 1)
+    hp = dqt.adamw(lr=1e-3, step=1)
+    out = (C.c_uint8 * 256)()
+    n = L.dqt_update_consts_size()
+    assert n <= 80  # fits the shared-memory slot the GEMM kernels copy it to
+    ok = dqt.sr_stream(seed=1, tensor_id=2, elem0=1 << 36)
+    assert L.dqt_update_consts(C.byref(hp), C.byref(ok), g, C.c_float(10.0), out, 256) == dqt.DQT_OK
+    blk0 = int.from_bytes(bytes(out[n - 8: n]), "little")
+    assert blk0 == (1 << 36) // 4
+    for bad, rc in [(-4, dqt.DQT_ERR_ARG), (2, dqt.DQT_ERR_ALIGN), (6, dqt.DQT_ERR_ALIGN)]:
+        sr = dqt.sr_stream(seed=1, tensor_id=2, elem0=bad)
+        assert L.dqt_update_consts(C.byref(hp), C.byref(sr), g, C.c_float(10.0), out, 256) == rc
+        A = _p(0x10000)
+        assert L.dqt_sr_update(A, A, C.c_float(10.0), A, A, C.byref(hp), C.byref(sr), g, 64,
+                               None, None) == rc
+    sr = dqt.sr_stream(seed=1, tensor_id=2, elem0=16)
+    A = _p(0x10000)
+    assert L.dqt_adafactor_apply(A, A, 0, A, A, A, 1, C.byref(sr), g, 8, 8, None,
+                                 None) == dqt.DQT_ERR_ARG

@@ -267,7 +267,7 @@ def test_device_consts_update_matches_host_path():
     c0, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=3).numpy(), qmin, qmax)
     X = inputs.normal((T, K), 1.0, seed=4, dtype=torch.bfloat16).cuda()
     dY = inputs.normal((T, N), 1e-2, seed=5, dtype=torch.bfloat16).cuda()
-    _, s_x, _, xdq = dqt.dqt_act_quant(X, want=("Xdq",))
+    _, s_x, _, xdq = dqt.dqt_act_quant_images(X, want=("Xdq",))
     hp = dqt.adamw(lr=1e-3, weight_decay=0.01, step=3)
     sr = dqt.sr_stream(seed=11, tensor_id=2)
     blk = dqt.dqt_update_consts(hp, sr, (qmin, qmax), float(s_w))
@@ -276,7 +276,7 @@ def test_device_consts_update_matches_host_path():
     v0 = inputs.normal((N, K), 1e-4, seed=7).square().cuda()
     a = [torch.from_numpy(c0).cuda(), m0.clone(), v0.clone()]
     b = [torch.from_numpy(c0).cuda(), m0.clone(), v0.clone()]
-    dqt.dqt_bitlinear_bwd_dw_update(dY, xdq, a[0], float(s_w), a[1], a[2], hp, sr, (qmin, qmax))
+    dqt.dqt_bitlinear_bwd_dw_update_img(dY, xdq, a[0], float(s_w), a[1], a[2], hp, sr, (qmin, qmax))
     dqt.dqt_bitlinear_bwd_dw_update_dev(dY, xdq, b[0], b[1], b[2], dev)
     g = inputs.normal((N * K,), 1e-3, seed=8).cuda()
     dqt.dqt_sr_update(g, a[0].view(-1), float(s_w), a[1].view(-1), a[2].view(-1), hp, sr, (qmin, qmax))

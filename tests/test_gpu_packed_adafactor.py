@@ -99,13 +99,13 @@ def test_fused_dw_update_packed_equals_int8(T, K, N, ws):
     X = inputs.normal((T, K), 1.0, seed=T, dtype=torch.bfloat16).cuda()
     dY = inputs.normal((T, N), 1e-2, seed=T + 1, dtype=torch.bfloat16).cuda()
     c0, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=T + 2).numpy(), -1, 1)
-    _, s_x, _, xdq = dqt.dqt_act_quant(X, want=("Xdq",))
+    _, s_x, _, xdq = dqt.dqt_act_quant_images(X, want=("Xdq",))
     hp = dqt.adamw(lr=1e-3, step=1)
     sr = dqt.sr_stream(seed=5, tensor_id=1)
     W = torch.from_numpy(c0).cuda()
     m = torch.zeros((N, K), device="cuda")
     v = torch.zeros((N, K), device="cuda")
-    dqt.dqt_bitlinear_bwd_dw_update(dY, xdq, W, float(s_w), m, v, hp, sr, (-1, 1), ws=ws)
+    dqt.dqt_bitlinear_bwd_dw_update_img(dY, xdq, W, float(s_w), m, v, hp, sr, (-1, 1), ws=ws)
     Wp = torch.from_numpy(oracle.pack_ternary(c0)).cuda()
     m2 = torch.zeros((N, K), device="cuda")
     v2 = torch.zeros((N, K), device="cuda")
@@ -194,7 +194,7 @@ def test_bwd_dw_adafactor(T, K, N, bits_w, packed):
     X = inputs.normal((T, K), 1.0, seed=T, dtype=torch.bfloat16)
     c, s_w, (qmin, qmax) = _af_problem(N, K, bits_w, seed=N)
     Xg = X.cuda()
-    _, s_x, _, xdq = dqt.dqt_act_quant(Xg, want=("Xdq",))
+    _, s_x, _, xdq = dqt.dqt_act_quant_images(Xg, want=("Xdq",))
     xd = bits(xdq)
     Rg = torch.zeros(N, device="cuda")
     Cg = torch.zeros(K, device="cuda")

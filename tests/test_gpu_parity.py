@@ -80,7 +80,7 @@ def test_act_quant_bit_exact(T, K):
         X[1] = 0.0  # all-zero row: amax floor
         X[2, : K // 2] = 0.5  # ties at .5 after scaling
     q, s, qi, xd = oracle.act_quant(bits(X))
-    Xq, s_x, Xq_img, Xdq = dqt.dqt_act_quant(X.cuda())
+    Xq, s_x, Xq_img, Xdq = dqt.dqt_act_quant_images(X.cuda())
     torch.cuda.synchronize()
     assert np.array_equal(Xq.cpu().numpy(), q)
     assert np.array_equal(s_x.cpu().numpy().view(np.uint32), s.view(np.uint32))
@@ -93,7 +93,7 @@ def test_act_quant_beyond_int32_sampled():
     2^31): codes, s_x and both images bit-exact on sampled rows."""
     T, K = (1 << 18) + 3, 8192
     X = inputs.normal((T, K), 1.0, seed=45, dtype=torch.bfloat16)
-    Xq, s_x, Xq_img, Xdq = dqt.dqt_act_quant(X.cuda())
+    Xq, s_x, Xq_img, Xdq = dqt.dqt_act_quant_images(X.cuda())
     torch.cuda.synchronize()
     rows = np.array([0, 1, T // 2, 262143, 262144, T - 1])
     q, s, qi, xd = oracle.act_quant(bits(X[torch.from_numpy(rows)]))
@@ -107,7 +107,7 @@ def test_act_quant_beyond_int32_sampled():
 def test_act_quant_partial_outputs():
     X = inputs.normal((64, 128), 1.0, seed=3, dtype=torch.bfloat16)
     q, s, qi, xd = oracle.act_quant(bits(X))
-    _, s_x, Xq_img, _ = dqt.dqt_act_quant(X.cuda(), want=("Xq_img",))
+    _, s_x, Xq_img, _ = dqt.dqt_act_quant_images(X.cuda(), want=("Xq_img",))
     torch.cuda.synchronize()
     assert np.array_equal(bits(Xq_img), qi)
     assert np.array_equal(s_x.cpu().numpy(), s)
@@ -146,10 +146,10 @@ def test_absmean_init_matches_oracle(bits_w):
 def _fwd_check(T, K, N, bits_w, rows=None, seed=1):
     X, dY, W0, c, s_w, g = problem(T, K, N, bits_w, seed)
     Xg = X.cuda()
-    _, s_x, Xq_img, _ = dqt.dqt_act_quant(Xg, want=("Xq_img",))
+    _, s_x, Xq_img, _ = dqt.dqt_act_quant_images(Xg, want=("Xq_img",))
     W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
     acc = torch.empty((T, N), dtype=torch.int32, device="cuda")
-    Y = dqt.dqt_bitlinear_fwd(Xq_img, s_x, W_img, s_w, g, acc_out=acc)
+    Y = dqt.dqt_bitlinear_fwd_img(Xq_img, s_x, W_img, s_w, g, acc_out=acc)
     dqt.dqt_check_device_status()
     q, s, _, _ = oracle.act_quant(bits(X))
     if rows is None:
@@ -184,7 +184,7 @@ def test_fwd_adversarial_magnitudes():
     c = -torch.randint(120, 129, (N, K), dtype=torch.int32, generator=g)
     s_x = torch.full((T,), 1.0, dtype=torch.float32)
     acc = torch.empty((T, N), dtype=torch.int32, device="cuda")
-    Y = dqt.dqt_bitlinear_fwd(q.to(torch.bfloat16).cuda(), s_x.cuda(), c.to(torch.bfloat16).cuda(),
+    Y = dqt.dqt_bitlinear_fwd_img(q.to(torch.bfloat16).cuda(), s_x.cuda(), c.to(torch.bfloat16).cuda(),
                               1.0, (-128, 127), acc_out=acc)
     dqt.dqt_check_device_status()
     ref = q.to(torch.int64) @ c.to(torch.int64).T
@@ -202,10 +202,10 @@ def test_fwd_output_beyond_int32_sampled():
     W0 = inputs.normal((N, K), 0.02, seed=42)
     qmin, qmax = oracle.grid(1.58)
     c, s_w, _ = oracle.absmean_init(W0.numpy(), qmin, qmax)
-    _, s_x, Xq_img, _ = dqt.dqt_act_quant(X.cuda(), want=("Xq_img",))
+    _, s_x, Xq_img, _ = dqt.dqt_act_quant_images(X.cuda(), want=("Xq_img",))
     W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
     acc = torch.empty((T, N), dtype=torch.int32, device="cuda")
-    Y = dqt.dqt_bitlinear_fwd(Xq_img, s_x, W_img, float(s_w), (qmin, qmax), acc_out=acc)
+    Y = dqt.dqt_bitlinear_fwd_img(Xq_img, s_x, W_img, float(s_w), (qmin, qmax), acc_out=acc)
     dqt.dqt_check_device_status()
     rows = np.array([0, 1, T // 2, 524287, 524288, T - 2, T - 1])
     q, s, _, _ = oracle.act_quant(bits(X[torch.from_numpy(rows)]))
@@ -230,7 +230,7 @@ def test_fwd_llama_mlp_sampled_rows(which):
 def test_bwd_dx(T, N, K):
     X, dY, W0, c, s_w, g = problem(T, K, N, 1.58, seed=N)
     W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
-    dX = dqt.dqt_bitlinear_bwd_dx(dY.cuda(), W_img, s_w)
+    dX = dqt.dqt_bitlinear_bwd_dx_img(dY.cuda(), W_img, s_w)
     dqt.dqt_check_device_status()
     ref = oracle.bwd_dx(bits(dY), c, np.float32(s_w))
     assert rel_err(dX.cpu().double().numpy(), ref) <= REL_TOL
@@ -246,7 +246,7 @@ def test_bwd_dx_output_beyond_int32_sampled():
     qmin, qmax = oracle.grid(1.58)
     c, s_w, _ = oracle.absmean_init(W0.numpy(), qmin, qmax)
     W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
-    dX = dqt.dqt_bitlinear_bwd_dx(dY.cuda(), W_img, float(s_w))
+    dX = dqt.dqt_bitlinear_bwd_dx_img(dY.cuda(), W_img, float(s_w))
     dqt.dqt_check_device_status()
     rows = np.array([0, 1, T // 2, 524287, 524288, T - 2, T - 1])
     ref = oracle.bwd_dx(bits(dY[torch.from_numpy(rows)]), c, np.float32(s_w))
@@ -258,9 +258,9 @@ def test_bwd_dx_output_beyond_int32_sampled():
 @pytest.mark.parametrize("T,N,K", [(256, 512, 512), (300, 520, 264), (77, 24, 200)])
 def test_bwd_dw_gradient(T, N, K):
     X, dY, W0, c, s_w, g = problem(T, K, N, 1.58, seed=K)
-    _, s_x, _, Xdq = dqt.dqt_act_quant(X.cuda(), want=("Xdq",))
+    _, s_x, _, Xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xdq",))
     dW = torch.empty((N, K), dtype=torch.float32, device="cuda")
-    dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=dW)
+    dqt.dqt_bitlinear_bwd_dw_update_img(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=dW)
     dqt.dqt_check_device_status()
     q, s, _, xd = oracle.act_quant(bits(X))
     ref = oracle.bwd_dw(bits(dY), q, s)
@@ -273,10 +273,10 @@ def test_bwd_llama_mlp_sampled_rows():
     T, H, I = 8192, 2048, 5632
     X, dY, W0, c, s_w, g = problem(T, H, I, 1.58, seed=21)
     W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
-    dX = dqt.dqt_bitlinear_bwd_dx(dY.cuda(), W_img, s_w)
-    _, s_x, _, Xdq = dqt.dqt_act_quant(X.cuda(), want=("Xdq",))
+    dX = dqt.dqt_bitlinear_bwd_dx_img(dY.cuda(), W_img, s_w)
+    _, s_x, _, Xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xdq",))
     dW = torch.empty((I, H), dtype=torch.float32, device="cuda")
-    dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=dW)
+    dqt.dqt_bitlinear_bwd_dw_update_img(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=dW)
     dqt.dqt_check_device_status()
     trows = np.array([0, 129, 4097, 8191])
     ref = oracle.bwd_dx(bits(dY)[trows], c, np.float32(s_w))
@@ -372,11 +372,11 @@ def _fused(T, K, N, bits_w, step, seed, rows=None):
         v = torch.zeros((N, K))
     hp = dqt.adamw(lr=1e-3, step=step)
     sr = dqt.sr_stream(seed=1234, tensor_id=1)
-    _, s_x, _, Xdq = dqt.dqt_act_quant(X.cuda(), want=("Xdq",))
+    _, s_x, _, Xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xdq",))
     Wg, mg, vg = torch.from_numpy(c).cuda(), m.clone().cuda(), v.clone().cuda()
     dW = torch.empty((N, K), dtype=torch.float32, device="cuda")
     changed = torch.zeros(1, dtype=torch.int64, device="cuda")
-    dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), Xdq, Wg, s_w, mg, vg, hp, sr, g, dW_out=dW,
+    dqt.dqt_bitlinear_bwd_dw_update_img(dY.cuda(), Xdq, Wg, s_w, mg, vg, hp, sr, g, dW_out=dW,
                                     changed_out=changed)
     dqt.dqt_check_device_status()
     q, s, _, xd = oracle.act_quant(bits(X))
@@ -429,11 +429,11 @@ def test_fused_update_beyond_int32_sampled():
     del W0
     hp = dqt.adamw(lr=1e-3, step=1)
     sr = dqt.sr_stream(seed=1234, tensor_id=6)
-    _, _, _, Xdq = dqt.dqt_act_quant(X.cuda(), want=("Xdq",))
+    _, _, _, Xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xdq",))
     Wg = torch.from_numpy(c).cuda()
     mg = torch.zeros((N, K), dtype=torch.float32, device="cuda")
     vg = torch.zeros((N, K), dtype=torch.float32, device="cuda")
-    dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), Xdq, Wg, float(s_w), mg, vg, hp, sr, (qmin, qmax))
+    dqt.dqt_bitlinear_bwd_dw_update_img(dY.cuda(), Xdq, Wg, float(s_w), mg, vg, hp, sr, (qmin, qmax))
     dqt.dqt_check_device_status()
     rows = np.array([0, 1, 40000, 65535, 65536, 65543])
     _, _, _, xd = oracle.act_quant(bits(X))
@@ -482,7 +482,7 @@ def test_both_tilings_agree_with_oracle(mode):
         _fwd_check(513, 512, 264, 4, seed=92)
         X, dY, W0, c, s_w, g = problem(300, 264, 520, 1.58, seed=93)
         W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
-        dX = dqt.dqt_bitlinear_bwd_dx(dY.cuda(), W_img, s_w)
+        dX = dqt.dqt_bitlinear_bwd_dx_img(dY.cuda(), W_img, s_w)
         dqt.dqt_check_device_status()
         ref = oracle.bwd_dx(bits(dY), c, np.float32(s_w))
         assert elem_err(dX.cpu().double().numpy(), ref) <= REL_TOL
@@ -499,13 +499,13 @@ def test_tilings_bit_identical():
         dqt.dqt_set_gemm_tiles(mode)
         try:
             X, dY, W0, c, s_w, g = problem(520, 512, 776, 1.58, seed=95)
-            _, s_x, q_img, xdq = dqt.dqt_act_quant(X.cuda(), want=("Xq_img", "Xdq"))
+            _, s_x, q_img, xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xq_img", "Xdq"))
             W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
-            Y = dqt.dqt_bitlinear_fwd(q_img, s_x, W_img, s_w, g)
-            dX = dqt.dqt_bitlinear_bwd_dx(dY.cuda(), W_img, s_w)
+            Y = dqt.dqt_bitlinear_fwd_img(q_img, s_x, W_img, s_w, g)
+            dX = dqt.dqt_bitlinear_bwd_dx_img(dY.cuda(), W_img, s_w)
             dW = torch.empty((776, 512), dtype=torch.float32, device="cuda")
             # unsplit on both tilings (the split-T path sums in another order)
-            dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), xdq, None, s_w, None, None, None, None, g,
+            dqt.dqt_bitlinear_bwd_dw_update_img(dY.cuda(), xdq, None, s_w, None, None, None, None, g,
                                             dW_out=dW, ws=False)
             dqt.dqt_check_device_status()
             outs.append((Y.cpu(), dX.cpu(), dW.cpu()))
@@ -522,19 +522,19 @@ def test_tilings_bit_identical():
 @pytest.mark.parametrize("T,K,N,bits_w", [(8192, 256, 256, 1.58), (2048, 264, 520, 8),
                                            (4096, 768, 768, 4)])
 def test_split_t_dw_update(T, K, N, bits_w):
-    assert dqt.dqt_bwd_dw_workspace_size(T, N, K) > 0  # the shape takes the split path
+    assert dqt.dqt_bwd_dw_img_workspace_size(T, N, K) > 0  # the shape takes the split path
     X, dY, W0, c, s_w, g = problem(T, K, N, bits_w, seed=T + N)
     qmin, qmax = g
     m = inputs.normal((N, K), 1e-4, seed=T + 5)
     v = inputs.normal((N, K), 1e-4, seed=T + 6).square()
     hp = dqt.adamw(lr=1e-3, step=2)
     sr = dqt.sr_stream(seed=1234, tensor_id=6)
-    _, s_x, _, Xdq = dqt.dqt_act_quant(X.cuda(), want=("Xdq",))
+    _, s_x, _, Xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xdq",))
     Wg, mg, vg = torch.from_numpy(c).cuda(), m.clone().cuda(), v.clone().cuda()
     dW = torch.empty((N, K), dtype=torch.float32, device="cuda")
-    dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), Xdq, Wg, s_w, mg, vg, hp, sr, g, dW_out=dW)
+    dqt.dqt_bitlinear_bwd_dw_update_img(dY.cuda(), Xdq, Wg, s_w, mg, vg, hp, sr, g, dW_out=dW)
     dW2 = torch.empty((N, K), dtype=torch.float32, device="cuda")
-    dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=dW2)
+    dqt.dqt_bitlinear_bwd_dw_update_img(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=dW2)
     dqt.dqt_check_device_status()
     assert torch.equal(dW, dW2)  # the gradient-only split path sums the same slabs
     q, s, _, xd = oracle.act_quant(bits(X))
@@ -558,11 +558,11 @@ def test_split_t_dw_update(T, K, N, bits_w):
 def test_split_t_matches_unsplit_within_tolerance():
     T, K, N = 8192, 256, 512
     X, dY, W0, c, s_w, g = problem(T, K, N, 1.58, seed=77)
-    _, s_x, _, Xdq = dqt.dqt_act_quant(X.cuda(), want=("Xdq",))
+    _, s_x, _, Xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xdq",))
     a = torch.empty((N, K), dtype=torch.float32, device="cuda")
     b = torch.empty((N, K), dtype=torch.float32, device="cuda")
-    dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=a)
-    dqt.dqt_bitlinear_bwd_dw_update(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=b,
+    dqt.dqt_bitlinear_bwd_dw_update_img(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=a)
+    dqt.dqt_bitlinear_bwd_dw_update_img(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=b,
                                     ws=False)
     dqt.dqt_check_device_status()
     # fp32 summation order only (a wrong token slice would be an O(1) error)

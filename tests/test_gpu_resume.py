@@ -36,11 +36,11 @@ def _layer(bits_w, T=320, K=264, N=520, seed=3):
 
 
 def _step(g, s_w, X, dY, state, step):
-    _, s_x, q_img, xdq = dqt.dqt_act_quant(X, want=("Xq_img", "Xdq"))
+    _, s_x, q_img, xdq = dqt.dqt_act_quant_images(X, want=("Xq_img", "Xdq"))
     W_img = dqt.dqt_codes_to_bf16(state["W"])
-    dqt.dqt_bitlinear_fwd(q_img, s_x, W_img, s_w, g)
-    dqt.dqt_bitlinear_bwd_dx(dY, W_img, s_w)
-    dqt.dqt_bitlinear_bwd_dw_update(dY, xdq, state["W"], s_w, state["m"], state["v"],
+    dqt.dqt_bitlinear_fwd_img(q_img, s_x, W_img, s_w, g)
+    dqt.dqt_bitlinear_bwd_dx_img(dY, W_img, s_w)
+    dqt.dqt_bitlinear_bwd_dw_update_img(dY, xdq, state["W"], s_w, state["m"], state["v"],
                                     dqt.adamw(lr=1e-3, step=step),
                                     dqt.sr_stream(seed=77, tensor_id=5), g)
     dqt.dqt_check_device_status()

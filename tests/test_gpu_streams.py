@@ -48,7 +48,7 @@ def _state():
         st["aq_" + src] = (torch.empty(T, dtype=torch.float32, device=dev),
                            torch.empty((T, K), dtype=torch.bfloat16, device=dev),
                            torch.empty((T, K), dtype=torch.bfloat16, device=dev))
-    nbw = max(dqt.dqt_bwd_dw_workspace_size(T, N, K) for _, K, N in PROJ)
+    nbw = max(dqt.dqt_bwd_dw_img_workspace_size(T, N, K) for _, K, N in PROJ)
     st["ws"] = [torch.empty(max(nbw, 16), dtype=torch.uint8, device=dev) for _ in range(4)]
     return st
 
@@ -72,7 +72,7 @@ def _step(st, streams, step_no=1):
 
     def aq(src, stream):
         s_x, img, xdq = st["aq_" + src]
-        on(stream, lambda: dqt.dqt_act_quant(st[src], None, s_x, img, xdq, want=()))
+        on(stream, lambda: dqt.dqt_act_quant_images(st[src], None, s_x, img, xdq, want=()))
 
     def codes(name, stream):
         p = st[name]
@@ -81,17 +81,17 @@ def _step(st, streams, step_no=1):
     def fwd(name, stream):
         p = st[name]
         s_x, img, _ = st["aq_H" if name == "down" else "aq_X"]
-        on(stream, lambda: dqt.dqt_bitlinear_fwd(img, s_x, p["img"], p["s_w"], grid, Y=p["Y"]))
+        on(stream, lambda: dqt.dqt_bitlinear_fwd_img(img, s_x, p["img"], p["s_w"], grid, Y=p["Y"]))
 
     def dx(name, stream):
         p = st[name]
-        on(stream, lambda: dqt.dqt_bitlinear_bwd_dx(p["dY"], p["img"], p["s_w"], dX=p["dX"]))
+        on(stream, lambda: dqt.dqt_bitlinear_bwd_dx_img(p["dY"], p["img"], p["s_w"], dX=p["dX"]))
 
     def dw(i, name, stream):
         p = st[name]
         xdq = st["aq_H" if name == "down" else "aq_X"][2]
         ws = st["ws"][s.index(stream)]
-        on(stream, lambda: dqt.dqt_bitlinear_bwd_dw_update(
+        on(stream, lambda: dqt.dqt_bitlinear_bwd_dw_update_img(
             p["dY"], xdq, p["W"], p["s_w"], p["m"], p["v"], hp, dqt.sr_stream(seed=7, tensor_id=i),
             grid, changed_out=p["changed"], ws=ws))
 

@@ -34,13 +34,13 @@ def test_timeout_reported_and_context_survives():
     X = inputs.normal((T, K), 1.0, seed=5, dtype=torch.bfloat16)
     W0 = inputs.normal((N, K), 0.02, seed=6)
     c, s_w, _ = oracle.absmean_init(W0.numpy(), -1, 1)
-    _, s_x, q_img, _ = dqt.dqt_act_quant(X.cuda(), want=("Xq_img",))
+    _, s_x, q_img, _ = dqt.dqt_act_quant_images(X.cuda(), want=("Xq_img",))
     W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
     dqt.dqt_check_device_status()
 
     dqt.dqt_set_wait_limit_ns(0)
     try:
-        dqt.dqt_bitlinear_fwd(q_img, s_x, W_img, float(s_w), (-1, 1))
+        dqt.dqt_bitlinear_fwd_img(q_img, s_x, W_img, float(s_w), (-1, 1))
         with pytest.raises(dqt.DQTError) as err:
             dqt.dqt_check_device_status()
         assert err.value.status == dqt.DQT_ERR_TIMEOUT
@@ -49,7 +49,7 @@ def test_timeout_reported_and_context_survives():
 
     # the record is cleared and the context is usable: a normal launch is exact
     acc = torch.empty((T, N), dtype=torch.int32, device="cuda")
-    dqt.dqt_bitlinear_fwd(q_img, s_x, W_img, float(s_w), (-1, 1), acc_out=acc)
+    dqt.dqt_bitlinear_fwd_img(q_img, s_x, W_img, float(s_w), (-1, 1), acc_out=acc)
     dqt.dqt_check_device_status()
     q, s, _, _ = oracle.act_quant(_bits(X))
     rows = np.array([0, 511, 1023])

@@ -17,7 +17,7 @@ def test_entry_points_refuse_cpu_tensors(built):
     x = torch.zeros(8, 64, dtype=torch.bfloat16)
     w = torch.zeros(64, 64, dtype=torch.int8)
     with pytest.raises(ValueError, match="CUDA"):
-        dqt.dqt_act_quant(x)
+        dqt.dqt_act_quant_images(x)
     with pytest.raises(ValueError, match="CUDA"):
         dqt.dqt_codes_to_bf16(w)
     with pytest.raises(ValueError, match="CUDA"):
