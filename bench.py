@@ -227,6 +227,8 @@ class MLPStep:
             self.dw_ws = [torch.empty(nbw, dtype=torch.uint8, device=dev) for _ in range(4)]
             nbx = max(dqt.dqt_bwd_dx_workspace_size(N, K) for _, K, N in PROJ)
             self.dx_ws = [torch.empty(nbx, dtype=torch.uint8, device=dev) for _ in range(4)]
+            nbf = max(dqt.dqt_fwd_workspace_size(T, K, N) for _, K, N in PROJ)
+            self.fwd_ws = [torch.empty(nbf, dtype=torch.uint8, device=dev) for _ in range(4)]
         else:
             nbw = max(dqt.dqt_bwd_dw_img_workspace_size(T, N, K) for _, K, N in PROJ)
             self.dw_ws = [torch.empty(max(nbw, 16), dtype=torch.uint8, device=dev) if nbw else False
@@ -235,13 +237,14 @@ class MLPStep:
         # forward 3, dX 3, and per projection the dW GEMM, the streaming
         # kernel of its sliced last wave (when the shape has one), and for
         # Adafactor the five statistics kernels and the step; with int8
-        # operands the weight image is made inside each dX call and the
-        # X_tilde image inside each dW call (3 + 3)
+        # operands each forward call converts both operands (3 x 2 images
+        # instead of the 3 shared weight images), each dX call the weight
+        # and each dW call X_tilde (3 + 3)
         dw = [1 + (1 if dqt.dqt_bwd_dw_img_workspace_size(T, N, K) > 0 else 0) for _, K, N in PROJ]
-        self.launches_per_step = 2 + 3 + 3 + 3 + sum(dw) + (3 if fp8 else 0) + (3 if self.i8 else 0)
+        self.launches_per_step = 2 + 3 + 3 + 3 + sum(dw) + (3 if fp8 else 0) + (6 if self.i8 else 0)
         self.dw_kind = "bwd_dw_adafactor" if optimizer == "adafactor" else "bwd_dw_update"
         if self.i8:
-            self.kinds = ["act_quant", "fwd", "codes_to_bf16", "bwd_dx", "codes_to_xdq",
+            self.kinds = ["act_quant", "codes_to_bf16", "fwd", "bwd_dx", "codes_to_xdq",
                           self.dw_kind]
         else:
             self.kinds = (["act_quant_fp8", "codes_to_fp8", "codes_to_bf16", "fwd_fp8"] if fp8 else
@@ -336,8 +339,20 @@ class MLPStep:
         def fwd(name, stream):
             s_x, q_img, _ = self.aq["H" if name == "down" else "X"]
             if self.i8:
-                timed("fwd", stream, lambda: dqt.dqt_bitlinear_fwd(
-                    q_img, s_x, self.W[name], self.s_w[name], self.grid, Y=self.Y[name]))
+                ws = self.fwd_ws[s.index(stream)]
+                if parts:
+                    W = self.W[name]
+                    (T_, K_), N_ = q_img.shape, W.shape[0]
+                    a_bytes = (T_ * K_ * 2 + 255) // 256 * 256
+                    qi = ws[: T_ * K_ * 2].view(torch.bfloat16).view(T_, K_)
+                    wi = ws[a_bytes: a_bytes + N_ * K_ * 2].view(torch.bfloat16).view(N_, K_)
+                    timed("codes_to_bf16", stream, lambda: dqt.dqt_codes_to_bf16(q_img, qi))
+                    timed("codes_to_bf16", stream, lambda: dqt.dqt_codes_to_bf16(W, wi))
+                    timed("fwd", stream, lambda: dqt.dqt_bitlinear_fwd_img(
+                        qi, s_x, wi, self.s_w[name], self.grid, Y=self.Y[name]))
+                else:
+                    dqt.dqt_bitlinear_fwd(q_img, s_x, self.W[name], self.s_w[name], self.grid,
+                                          Y=self.Y[name], ws=ws)
             elif self.fp8:
                 timed("fwd_fp8", stream, lambda: dqt.dqt_bitlinear_fwd_fp8(
                     q_img, s_x, self.W8[name], self.s_w[name], self.grid, Y=self.Y[name]))
@@ -464,7 +479,7 @@ class MLPStep:
             "act_quant": [T * HID * 3.0 + 4 * T, T * INTER * 3.0 + 4 * T],
             # bf16 in (2) + E4M3 byte (1) per element, + s_x8
             "act_quant_fp8": [T * HID * 3.0 + 4 * T, T * INTER * 3.0 + 4 * T],
-            "codes_to_bf16": [0.0 for _ in PROJ],
+            "codes_to_bf16": [0.0],
             "codes_to_fp8": [0.0 for _ in PROJ],
             "codes_to_xdq": [0.0 for _ in PROJ],
         }
@@ -473,7 +488,11 @@ class MLPStep:
             "act_quant": [0.0, 0.0] if self.i8 else [T * HID * 4.0, T * INTER * 4.0],
             # the bf16 dequantised image (2 B per element)
             "act_quant_fp8": [T * HID * 2.0, T * INTER * 2.0],
-            "codes_to_bf16": [(2.25 if self.packed else 3.0) * K * N for _, K, N in PROJ],
+            # per step: the weight images (with int8 operands, each weight twice:
+            # forward and dX), and with int8 operands each forward's activation image
+            "codes_to_bf16": ([3.0 * K * N for _, K, N in PROJ] * 2 +
+                              [3.0 * T * K for _, K, N in PROJ]) if self.i8 else
+                             [(2.25 if self.packed else 3.0) * K * N for _, K, N in PROJ],
             "codes_to_fp8": [(1.25 if self.packed else 2.0) * K * N for _, K, N in PROJ],
             # int8 codes read, bf16 image written, s_x read (gate, up: X; down: H)
             "codes_to_xdq": [3.0 * T * K + 4 * T for _, K, N in PROJ],
@@ -697,6 +716,16 @@ def run_gpu(args):
     e2e = {"value": round(aggregate_tokens_per_s(ws, T_TOK, e_steps, e_ms), 1), "unit": "tokens/s",
            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": e_steps}
 
+    # the other configurations' sub-results, on rank 0 at N = 1: the
+    # single-layer step (256 x 512 x 512) and the standalone update's
+    # bandwidth sweep of the 8-bit configuration
+    extra = {}
+    if rank == 0 and ws == 1 and not args.no_extras and st.i8 and dp_mode != "exchange":
+        lay = layer_step(1.58, 200, 10)
+        extra["layer_256x512x512"] = {k: lay[k] for k in (
+            "value", "unit", "us_per_step", "graph", "e2e", "changed_codes_last_step", "clocks")}
+        extra["sr_update_sweep"] = sr_sweep()
+
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = cpu_baseline(args.cpu_seconds)
@@ -709,27 +738,15 @@ def run_gpu(args):
             "dtype": "e4m3 forward, bf16 backward" if st.fp8 else "bf16",
             "data": "synthetic (seeded N(0,1) activations, N(0,1e-2) gradients, AbsMean-%s codes of N(0,0.02))"
                     % ("ternary" if st.bits == 1.58 else "%d-bit" % st.bits),
-            "config": {"workload": (WORKLOAD if st.bits == 1.58 else
-                                    WORKLOAD.replace("ternary", "%d-bit" % st.bits)) +
-                                   (", FP8 (E4M3) forward" if st.fp8 else "") +
-                                   (", Adafactor" if st.optimizer == "adafactor" else "") +
-                                   (", 2-bit packed codes" if st.packed else ""),
-                       "tokens": T_TOK, "hidden": HID, "intermediate": INTER,
-                       "weights": "%s codes, %s" % ("ternary" if st.bits == 1.58 else "%d-bit" % st.bits,
-                                                     "2-bit packed" if st.packed else "int8"),
-                       "optimizer": st.optimizer,
-                       "operands": ("int8 codes through the C ABI" if st.i8 else
-                                    "bf16 / E4M3 operand images"),
-                       "parallelism": (("data parallel over %d GPU(s): reduce-scatter of fp32 dW, "
-                                        "ZeRO-1 sharded AdamW + SR update, all-gather of int8 "
-                                        "codes" % ws) if dp_mode == "exchange" else
-                                       "replicas" if ws > 1 else "single GPU"),
-                       "l2": "inputs larger than L2 (step working set ~1.5 GB > 129 MB)"},
+            "config": mlp_config(bits=st.bits, fp8=st.fp8, optimizer=st.optimizer,
+                                 packed=st.packed, i8=st.i8,
+                                 parallelism=_parallelism(ws, dp_mode)),
             "roofline": roofline, "kernels": kern, "e2e": e2e,
             "gpu_launches": st.launches_per_step * args.steps,
             "clocks": clk.summary(), "cpu_baseline": cpu,
             "changed_codes_last_step": [int(x) for x in res_host[(e_steps - 1) % 2].tolist()],
         }
+        line.update(extra)
         print(json.dumps(line))
     if dist.is_initialized():
         dist.destroy_process_group()
@@ -738,27 +755,42 @@ def run_gpu(args):
 # ---------------------------------------------------------------------------
 # CPU oracle timing (the reported baseline and the --impl reference arm)
 # ---------------------------------------------------------------------------
-def _oracle_sample(token_rows, weight_rows, seed=7):
-    """Times the oracle on `token_rows` token rows of act-quant + forward + dX
-    and `weight_rows` weight rows of dW + AdamW + SR per projection; returns
-    (seconds measured, seconds extrapolated to the full step)."""
+_SAMPLE_INPUTS = {}  # per process: the generated inputs of each (seed, projection)
+
+
+def _sample_inputs(seed, i, K, N):
     import oracle
     from paper_2412_04787_gb300 import inputs
+    key = (seed, i)
+    if key not in _SAMPLE_INPUTS:
+        qmin, qmax = oracle.grid(1.58)
+        X = inputs.bf16_bits(inputs.normal((T_TOK, K), 1.0, seed=seed + i, dtype=torch.bfloat16))
+        dY = inputs.bf16_bits(inputs.normal((T_TOK, N), 1e-2, seed=seed + 10 + i,
+                                            dtype=torch.bfloat16))
+        c, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=seed + 20 + i).numpy(),
+                                        qmin, qmax)
+        _SAMPLE_INPUTS[key] = (X, dY, c, s_w)
+    return _SAMPLE_INPUTS[key]
+
+
+def _oracle_sample(token_rows, weight_rows, seed=7):
+    """Times the oracle, per projection, on the act-quant of all tokens (the
+    weight gradient needs every token's code), the forward and dX of
+    `token_rows` token rows, and dW + AdamW + SR of `weight_rows` weight rows;
+    returns (seconds measured, seconds extrapolated to the full step: the
+    row parts scaled by T / token_rows and N / weight_rows)."""
+    import oracle
 
     qmin, qmax = oracle.grid(1.58)
     meas = 0.0
     full = 0.0
     for i, (name, K, N) in enumerate(PROJ):
-        X = inputs.bf16_bits(inputs.normal((T_TOK, K), 1.0, seed=seed + i, dtype=torch.bfloat16))
-        dY = inputs.bf16_bits(inputs.normal((T_TOK, N), 1e-2, seed=seed + 10 + i, dtype=torch.bfloat16))
-        c, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=seed + 20 + i).numpy(), qmin, qmax)
+        X, dY, c, s_w = _sample_inputs(seed, i, K, N)
         t0 = time.perf_counter()
-        q, s, _, _ = oracle.act_quant(X[:token_rows])
-        oracle.fwd(q, s, c, s_w)
-        oracle.bwd_dx(dY[:token_rows], c, s_w)
-        t1 = time.perf_counter()
-        # dW needs every token's quantised activation
         qa, sa, _, _ = oracle.act_quant(X)
+        t1 = time.perf_counter()
+        oracle.fwd(qa[:token_rows], sa[:token_rows], c, s_w)
+        oracle.bwd_dx(dY[:token_rows], c, s_w)
         t2 = time.perf_counter()
         rows = np.arange(weight_rows)
         g = oracle.bwd_dw(dY, qa, sa, rows=rows).astype(np.float32)
@@ -766,58 +798,210 @@ def _oracle_sample(token_rows, weight_rows, seed=7):
         z = np.zeros((weight_rows, K), np.float32)
         oracle.update(g, c[:weight_rows], z, z, k, qmin, qmax, 1234, 1, i, rows=rows)
         t3 = time.perf_counter()
-        meas += (t1 - t0) + (t2 - t1) + (t3 - t2)
-        full += (t1 - t0) * T_TOK / token_rows + (t2 - t1) + (t3 - t2) * N / weight_rows
+        meas += t3 - t0
+        full += (t1 - t0) + (t2 - t1) * T_TOK / token_rows + (t3 - t2) * N / weight_rows
     return meas, full
 
 
-def cpu_baseline(seconds=15.0):
-    # calibrate on a tiny sample, then size the sample to ~`seconds` of work
-    m0, f0 = _oracle_sample(2, 1)
+def _oracle_layer_full():
+    """The single-layer configuration (T=256, K=512, N=512, ternary, AdamW
+    step 1) through the oracle in full: act-quant, forward, dX, dW and the
+    update.  Returns the seconds it took."""
+    import oracle
+    from paper_2412_04787_gb300 import inputs
+
+    T, K, N = LAYER_SHAPE
+    qmin, qmax = oracle.grid(1.58)
+    X = inputs.bf16_bits(inputs.normal((T, K), 1.0, seed=1, dtype=torch.bfloat16))
+    dY = inputs.bf16_bits(inputs.normal((T, N), 1e-2, seed=2, dtype=torch.bfloat16))
+    c, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=3).numpy(), qmin, qmax)
+    t0 = time.perf_counter()
+    q, s, _, _ = oracle.act_quant(X)
+    oracle.fwd(q, s, c, s_w)
+    oracle.bwd_dx(dY, c, s_w)
+    g = oracle.bwd_dw(dY, q, s).astype(np.float32)
+    k = oracle.adamw_consts(1e-3, 0.9, 0.999, 1e-8, 0.0, 1, s_w)
+    z = np.zeros((N, K), np.float32)
+    oracle.update(g, c, z, z, k, qmin, qmax, 1234, 1, 0)
+    return time.perf_counter() - t0
+
+
+def _oracle_sample_worker(job):
+    """One host core's share of the sampled MLP step (spawned process)."""
+    tr, wr, seed = job
+    from oracle import build_oracle
+    build_oracle.build()
+    return _oracle_sample(tr, wr, seed=seed)
+
+
+class OraclePool:
+    """The oracle on every host core: `cores` spawned processes (never forked
+    from a process that has touched the GPU), each timing the same bounded
+    sample of the MLP step at once, so that memory contention between cores is
+    in every measurement.  A step of the full workload on `cores` cores then
+    takes mean(extrapolated single-core step) / cores."""
+
+    def __init__(self, cores=None):
+        import concurrent.futures
+        import multiprocessing
+        self.cores = cores or os.cpu_count() or 1
+        self.ex = concurrent.futures.ProcessPoolExecutor(
+            max_workers=self.cores, mp_context=multiprocessing.get_context("spawn"))
+        # start every worker, build the oracle there and generate its inputs
+        list(self.ex.map(_oracle_sample_worker, [(2, 1, 7 + i) for i in range(self.cores)]))
+
+    def sample(self, tr, wr):
+        """Returns (wall seconds of the sample on all cores, extrapolated
+        seconds of one full step on all cores)."""
+        t0 = time.perf_counter()
+        res = list(self.ex.map(_oracle_sample_worker, [(tr, wr, 7 + i) for i in range(self.cores)]))
+        wall = time.perf_counter() - t0
+        full_1core = statistics.mean(f for _, f in res)
+        return wall, full_1core / self.cores
+
+    def close(self):
+        self.ex.shutdown()
+
+
+def _sample_size(seconds):
+    m0, _ = _oracle_sample(2, 1)
     scale = max(1.0, seconds / max(m0, 1e-3))
-    tr = int(min(256, max(2, 2 * scale)))
-    wr = int(min(128, max(1, scale)))
-    meas, full = _oracle_sample(tr, wr)
-    return {"value": round(T_TOK / full, 3), "unit": "tokens/s", "cores": 1, "kind": "oracle",
-            "sample": "%d token rows of act-quant+fwd+dX and %d weight rows of dW+AdamW+SR per "
-                      "projection (plus the full act-quant dW needs), %.1f s measured, "
-                      "extrapolated linearly to the 8192-token step (%.0f s)" % (tr, wr, meas, full)}
+    return int(min(256, max(2, 2 * scale))), int(min(128, max(1, scale)))
+
+
+def cpu_baseline(seconds=15.0):
+    """The oracle as it stands on the GPU machine's host: the single-layer
+    configuration in full on one core, and a bounded sample of the MLP step
+    on every core, extrapolated to the full step."""
+    t1 = _oracle_layer_full()
+    tr, wr = _sample_size(seconds)
+    pool = OraclePool()
+    try:
+        wall, full = pool.sample(tr, wr)
+    finally:
+        pool.close()
+    frac = wall / full  # the share of the full step's work the cores did in `wall`
+    return {"value": round(T_TOK / full, 3), "unit": "tokens/s", "cores": pool.cores,
+            "nproc": os.cpu_count(), "kind": "oracle",
+            "sample": "%d processes at once, each %d token rows of act-quant+fwd+dX and %d weight "
+                      "rows of dW+AdamW+SR per projection (plus the full act-quant dW needs), "
+                      "%.1f s wall: %.4f of the 8192-token step's work; extrapolated step "
+                      "%.1f s on %d cores" % (pool.cores, tr, wr, wall, frac, full, pool.cores),
+            "layer_256x512x512": {"value": round(LAYER_SHAPE[0] / t1, 2), "unit": "tokens/s",
+                                  "cores": 1, "seconds": round(t1, 3),
+                                  "sample": "the whole single-layer step, not sampled"}}
+
+
+def mlp_config(bits=1.58, fp8=False, optimizer="adamw", packed=False, i8=True, parallelism=None):
+    """The `config` of the MLP step's JSON line (both arms)."""
+    wname = "ternary" if bits == 1.58 else "%d-bit" % bits
+    return {"workload": (WORKLOAD if bits == 1.58 else WORKLOAD.replace("ternary", wname)) +
+                        (", FP8 (E4M3) forward" if fp8 else "") +
+                        (", Adafactor" if optimizer == "adafactor" else "") +
+                        (", 2-bit packed codes" if packed else ""),
+            "tokens": T_TOK, "hidden": HID, "intermediate": INTER,
+            "weights": "%s codes, %s" % (wname, "2-bit packed" if packed else "int8"),
+            "optimizer": optimizer,
+            "operands": "int8 codes through the C ABI" if i8 else "bf16 / E4M3 operand images",
+            "parallelism": parallelism or "single GPU",
+            "l2": "inputs larger than L2 (step working set ~1.5 GB > 129 MB)"}
+
+
+def _parallelism(ws, dp_mode):
+    if dp_mode == "exchange":
+        return ("data parallel over %d GPU(s): reduce-scatter of fp32 dW, ZeRO-1 sharded "
+                "AdamW + SR update, all-gather of int8 codes" % ws)
+    return "replicas" if ws > 1 else "single GPU"
 
 
 def run_reference(args):
+    """The oracle as it stands on the host cores: each step is one bounded
+    sample of the MLP step run on every core at once (OraclePool); the step's
+    time is that sample's wall time and `value` the throughput it implies."""
     ws, rank, _ = _dist()
     if rank != 0:
         return
     from oracle import build_oracle
     build_oracle.build()
     per_step_s = max(5.0, min(30.0, 150.0 / max(1, args.steps + args.warmup)))
-    for _ in range(args.warmup):
-        _oracle_sample(2, 1)
-    vals = []
-    samples = []
-    for _ in range(args.steps):
-        m0, _ = _oracle_sample(2, 1)
-        scale = max(1.0, per_step_s / max(m0, 1e-3))
-        tr, wr = int(min(256, max(2, 2 * scale))), int(min(128, max(1, scale)))
-        meas, full = _oracle_sample(tr, wr)
-        vals.append(full)
-        samples.append((tr, wr, meas))
-    full = statistics.median(vals)
+    tr, wr = _sample_size(per_step_s)
+    pool = OraclePool()
+    try:
+        for _ in range(args.warmup):
+            pool.sample(2, 1)
+        walls, fulls = [], []
+        for _ in range(args.steps):
+            wall, full = pool.sample(tr, wr)
+            walls.append(wall)
+            fulls.append(full)
+    finally:
+        pool.close()
+    full = statistics.median(fulls)
+    wall = statistics.median(walls)
     value = T_TOK / full
-    tr, wr, meas = samples[-1]
+    dp_mode = args.dp if args.dp != "auto" else ("exchange" if ws > 1 else "none")
     line = {
         "impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": "tokens/s",
         "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": round(full * 1e3, 1), "higher_is_better": True, "scaling": "weak",
+        "ms_per_step": round(wall * 1e3, 1), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64/f32 (oracle)", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "tokens": T_TOK, "hidden": HID, "intermediate": INTER},
-        "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": 1, "kind": "oracle",
-                         "sample": "per step: %d token rows of act-quant+fwd+dX, %d weight rows of "
-                                   "dW+AdamW+SR per projection, extrapolated" % (tr, wr)},
+        "config": mlp_config(bits=args.bits, fp8=args.act == "fp8", optimizer=args.optimizer,
+                             packed=args.packed, i8=args.operands == "int8",
+                             parallelism=_parallelism(ws, dp_mode)),
+        "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": pool.cores,
+                         "nproc": os.cpu_count(), "kind": "oracle",
+                         "sample": "each step: %d processes at once, each %d token rows of "
+                                   "act-quant+fwd+dX and %d weight rows of dW+AdamW+SR per "
+                                   "projection (plus the full act-quant dW needs): %.4f of the "
+                                   "8192-token step's work in %.1f s" % (
+                                       pool.cores, tr, wr, wall / full, wall)},
         "e2e": {"value": round(value, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line))
+
+
+def sr_sweep(sizes=(1 << 24, 1 << 26, 1 << 28), reps=10):
+    """The 8-bit standalone AdamW + SR update (22 bytes per weight: g 4, c
+    1 + 1, m 4 + 4, v 4 + 4) at each size: median CUDA-event time of `reps`
+    launches, each after an L2 flush (256 MiB written, then 256 MiB read)."""
+    from paper_2412_04787_gb300 import dqt
+    dev = torch.device("cuda", torch.cuda.current_device())
+    peaks, kind = _peaks()
+    g8 = dqt.grid(8)
+    hp = dqt.adamw(step=3)
+    sr = dqt.sr_stream()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    flush_r = torch.ones(32 << 20, dtype=torch.int64, device=dev)
+    out = []
+    for n in sizes:
+        gen = torch.Generator(device=dev).manual_seed(n)
+        grad = torch.randn(n, device=dev, generator=gen) * 1e-3
+        W = torch.randint(-128, 128, (n,), dtype=torch.int8, device=dev, generator=gen)
+        m = torch.randn(n, device=dev, generator=gen) * 1e-4
+        v = (torch.randn(n, device=dev, generator=gen) * 1e-4).square()
+        for _ in range(3):
+            dqt.dqt_sr_update(grad, W, 7958.0, m, v, hp, sr, g8)
+        times = []
+        for _ in range(reps):
+            flush.zero_()
+            flush_r.sum()
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record()
+            dqt.dqt_sr_update(grad, W, 7958.0, m, v, hp, sr, g8)
+            b.record()
+            times.append((a, b))
+        torch.cuda.synchronize()
+        ms = statistics.median(a.elapsed_time(b) for a, b in times)
+        gbs = 22.0 * n / (ms / 1e3) / 1e9
+        out.append({"numel": n, "median_ms": round(ms, 4), "gbs": round(gbs, 1),
+                    "frac_of_hbm": round(gbs / peaks["hbm_gbs"], 4)})
+        del grad, W, m, v
+    dqt.dqt_check_device_status()
+    return {"kernel": "sr_update (8-bit grid, fp32 gradient in memory)", "points": out,
+            "peak_gbs": peaks["hbm_gbs"], "peak_kind": "copy bandwidth, %s" % kind,
+            "bytes_per_weight": 22, "l2": "flushed before every launch"}
 
 
 def run_kernel(args):
@@ -1096,6 +1280,10 @@ LAYER_SHAPE = (256, 512, 512)  # T, K, N of the single-layer step
 
 
 def run_layer(args):
+    print(json.dumps(layer_step(args.bits, args.steps, args.warmup)))
+
+
+def layer_step(bits=1.58, steps=200, warmup=10):
     """One BitLinear layer's training step at T=256, K=512, N=512 (X ~N(0,1),
     dY ~N(0,1e-2), ternary codes by AbsMean of N(0,0.02), AdamW lr 1e-3, Philox
     seed 1234): act_quant, the weight's code image, forward, dX and the fused
@@ -1112,8 +1300,8 @@ def run_layer(args):
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     T, K, N = LAYER_SHAPE
-    KS = args.steps
-    grid = dqt.grid(args.bits)
+    KS = steps
+    grid = dqt.grid(bits)
     host = [(inputs.normal((T, K), 1.0, seed=1 + 100 * r, dtype=torch.bfloat16).pin_memory(),
              inputs.normal((T, N), 1e-2, seed=2 + 100 * r, dtype=torch.bfloat16).pin_memory())
             for r in range(2)]
@@ -1160,9 +1348,9 @@ def run_layer(args):
     # warm-up: eager steps, each with its own constants row
     side = torch.cuda.Stream()
     side.wait_stream(torch.cuda.current_stream())
-    warm = torch.zeros((args.warmup, row), dtype=torch.uint8).pin_memory()
+    warm = torch.zeros((warmup, row), dtype=torch.uint8).pin_memory()
     with torch.cuda.stream(side):
-        for i in range(args.warmup):
+        for i in range(warmup):
             state["step"] += 1
             dqt.dqt_update_consts(dqt.adamw(lr=1e-3, step=state["step"]), sr, grid, s_w,
                                   out=warm[i])
@@ -1207,9 +1395,9 @@ def run_layer(args):
     e1.record(stream)
     torch.cuda.synchronize()
     e_ms = e0.elapsed_time(e1) / KS
-    print(json.dumps({
+    return {
         "metric": "DQT BitLinear fwd+bwd+SR-update tokens/s", "value": round(T / (ms / 1e3), 1),
-        "unit": "tokens/s", "n_gpus": 1, "steps": R * KS, "warmup": args.warmup,
+        "unit": "tokens/s", "n_gpus": 1, "steps": R * KS, "warmup": warmup,
         "ms_per_step": round(ms, 5), "us_per_step": round(ms * 1e3, 2),
         "graph": {"steps_per_graph": KS, "replays": R},
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
@@ -1225,7 +1413,7 @@ def run_layer(args):
                 "h2d_bytes_per_step": int(X.numel() * 2 + dY.numel() * 2 + row),
                 "d2h_bytes_per_step": 8},
         "changed_codes_last_step": int(ch_host[KS - 1]),
-        "clocks": clk.summary()}))
+        "clocks": clk.summary()}
 
 
 def main():
@@ -1236,6 +1424,8 @@ def main():
     ap.add_argument("--impl", default="dqt", choices=["dqt", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-extras", action="store_true",
+                    help="mlp: skip the single-layer step and the SR-update sweep keys")
     ap.add_argument("--kernel", default=None,
                     help="time one kernel kind alone (fwd, bwd_dx, bwd_dw_update, bwd_dw, "
                          "bwd_dw_unfused, act_quant, codes_to_bf16, sr_update, act_quant_fp8, "

@@ -27,11 +27,11 @@
  * the 16-bit tensor cores over exact 16-bit images of the integer codes
  * (every integer in [-256, 256] is exact in bf16 and fp16; products and
  * partial sums below 2^24 are exact in the fp32 accumulator).  The hot-path
- * calls take the int8 codes themselves: the forward converts both operands
- * to fp16 in shared memory inside the GEMM; dX and dW make the bf16 operand
- * they need in a caller-provided workspace.  The *_img calls take those
- * images directly (dqt_act_quant_images, dqt_codes_to_bf16) for callers that
- * share one image between several GEMMs.
+ * calls take the int8 codes themselves and make the bf16 operands they need
+ * in a caller-provided workspace (dqt_codes_to_bf16, dqt_codes_to_xdq) before
+ * the GEMM.  The *_img calls take those images directly
+ * (dqt_act_quant_images, dqt_codes_to_bf16) for callers that share one image
+ * between several GEMMs.
  *
  * Conventions for every entry point:
  *   - All data pointers are DEVICE pointers owned by the caller; the library
@@ -204,13 +204,14 @@ int dqt_codes_to_xdq(const int8_t* Xq, const float* s_x, int64_t T, int64_t K, d
  *   grid     the weight grid; it bounds |c| and so how often the kernel drains its
  *            fp32 accumulator into int32 to keep every partial sum exact
  *   Y        bf16 [T, N] out;  acc_out int32 [T, N] out, or NULL
- * Both operands are converted to exact fp16 values in shared memory inside
- * the GEMM (2-SM tiles whatever dqt_set_gemm_tiles says); no workspace.
- * K a multiple of 16 (16-byte int8 rows), N of 8; Xq, W, Y, acc_out 16-byte
- * aligned; T >= 1; T, N, K < 2^31. */
+ *   ws       device workspace of at least dqt_fwd_workspace_size(T, K, N) bytes
+ *            (16-byte aligned): it receives the exact bf16 images of Xq and W
+ *            (3 bytes moved per element of each), which the GEMM then reads
+ * K, N multiples of 8; Xq, W, Y, acc_out 16-byte aligned; T >= 1; T, N, K < 2^31. */
+size_t dqt_fwd_workspace_size(int64_t T, int64_t K, int64_t N);
 int dqt_bitlinear_fwd(const int8_t* Xq, const float* s_x, const int8_t* W, float s_w,
                       dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
-                      int32_t* acc_out, void* stream);
+                      int32_t* acc_out, void* ws, size_t ws_bytes, void* stream);
 
 /* The same forward on the bf16 operand images (dqt_act_quant_images' Xq_img
  * and dqt_codes_to_bf16's W_img); K, N multiples of 8.  Identical Y and acc. */

@@ -279,15 +279,20 @@ int dqt_rmsnorm_bwd_bf16(const dqt_bf16* x, const dqt_bf16* w, const float* rstd
              : DQT_OK;
 }
 
+// |sum| <= K * 128 * max|c| must fit int32 (checked before any launch).
+static bool fwd_range_ok(dqt_grid_t grid, int64_t K) {
+  const int64_t cmax = grid.qmax > -grid.qmin ? grid.qmax : -grid.qmin;
+  const int64_t cm = cmax > 0 ? cmax : 1;
+  return K * 128 * cm <= (int64_t(1) << 31) - 1;
+}
+
 // The exact integer forward (both operand forms): the reduction is cut into
 // chunks whose partial sums stay <= 2^24 (exact in fp32).
-static int fwd_launch(const void* A, const float* s_x, const void* B, bool i8, float s_w,
+static int fwd_launch(const void* A, const float* s_x, const void* B, float s_w,
                dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y, int32_t* acc_out,
                void* stream) {
   const int64_t cmax = grid.qmax > -grid.qmin ? grid.qmax : -grid.qmin;
   const int64_t cm = cmax > 0 ? cmax : 1;
-  // |sum| <= K * 128 * max|c| must fit int32.
-  if (K * 128 * cm > (int64_t(1) << 31) - 1) return DQT_ERR_RANGE;
   // Largest chunk whose partial sums stay <= 2^24 (exact in fp32), multiple of 64.
   int64_t chunk = ((int64_t(1) << 24) / (128 * cm)) / 64 * 64;
   if (chunk < 64) chunk = 64;
@@ -299,7 +304,6 @@ static int fwd_launch(const void* A, const float* s_x, const void* B, bool i8, f
   g.Kred = static_cast<int>(K);
   g.A = A;
   g.B = B;
-  g.i8 = i8;
   g.chunk_k = static_cast<int>(chunk);
   g.s_x = s_x;
   g.scale = s_w;
@@ -308,17 +312,34 @@ static int fwd_launch(const void* A, const float* s_x, const void* B, bool i8, f
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
+static inline size_t fwd_ws_align(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+size_t dqt_fwd_workspace_size(int64_t T, int64_t K, int64_t N) {
+  if (T <= 0 || K <= 0 || N <= 0 || T > kMaxDim || K > kMaxDim || N > kMaxDim) return 0;
+  return fwd_ws_align(static_cast<size_t>(T) * static_cast<size_t>(K) * 2u) +
+         fwd_ws_align(static_cast<size_t>(N) * static_cast<size_t>(K) * 2u);
+}
+
 int dqt_bitlinear_fwd(const int8_t* Xq, const float* s_x, const int8_t* W, float s_w,
                       dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
-                      int32_t* acc_out, void* stream) {
-  if (!Xq || !s_x || !W || !Y || T <= 0 || K <= 0 || N <= 0 || !grid_ok(grid) ||
+                      int32_t* acc_out, void* ws, size_t ws_bytes, void* stream) {
+  if (!Xq || !s_x || !W || !Y || !ws || T <= 0 || K <= 0 || N <= 0 || !grid_ok(grid) ||
       !(s_w > 0.0f) || !isfinite(s_w))
     return DQT_ERR_ARG;
-  if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
-  if (K % 16 || N % 8 || !aligned16(Xq) || !aligned16(W) || !aligned16(Y) ||
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim || !fwd_range_ok(grid, K)) return DQT_ERR_RANGE;
+  if (ws_bytes < dqt_fwd_workspace_size(T, K, N)) return DQT_ERR_ARG;
+  if (K % 8 || N % 8 || !aligned16(Xq) || !aligned16(W) || !aligned16(Y) || !aligned16(ws) ||
       (acc_out && !aligned16(acc_out)))
     return DQT_ERR_ALIGN;
-  return fwd_launch(Xq, s_x, W, true, s_w, grid, T, K, N, Y, acc_out, stream);
+  // the exact bf16 images of both operands' codes, then the GEMM on them
+  cudaStream_t st = as_stream(stream);
+  dqt_bf16* Xq_img = static_cast<dqt_bf16*>(ws);
+  dqt_bf16* W_img = reinterpret_cast<dqt_bf16*>(
+      static_cast<uint8_t*>(ws) + fwd_ws_align(static_cast<size_t>(T) * static_cast<size_t>(K) * 2u));
+  if (dqt::launch_codes_to_bf16(Xq, T * K, Xq_img, st) ||
+      dqt::launch_codes_to_bf16(W, N * K, W_img, st))
+    return DQT_ERR_CUDA;
+  return fwd_launch(Xq_img, s_x, W_img, s_w, grid, T, K, N, Y, acc_out, stream);
 }
 
 int dqt_bitlinear_fwd_img(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img,
@@ -331,7 +352,8 @@ int dqt_bitlinear_fwd_img(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf
   if (K % 8 || N % 8 || !aligned16(Xq_img) || !aligned16(W_img) || !aligned16(Y) ||
       (acc_out && !aligned16(acc_out)))
     return DQT_ERR_ALIGN;
-  return fwd_launch(Xq_img, s_x, W_img, false, s_w, grid, T, K, N, Y, acc_out, stream);
+  if (!fwd_range_ok(grid, K)) return DQT_ERR_RANGE;
+  return fwd_launch(Xq_img, s_x, W_img, s_w, grid, T, K, N, Y, acc_out, stream);
 }
 
 int dqt_act_quant_fp8(const dqt_bf16* X, int64_t T, int64_t K, uint8_t* Xq8, float* s_x8,
@@ -445,10 +467,13 @@ int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const int8_t* Xq, const floa
                                 int64_t K, float* dW_out, unsigned long long* changed_out,
                                 void* ws, size_t ws_bytes, void* stream) {
   if (!dY || !Xq || !s_x || !ws || T <= 0 || N <= 0 || K <= 0) return DQT_ERR_ARG;
-  if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
   const size_t img = ws_align256(static_cast<size_t>(T) * static_cast<size_t>(K) * 2u);
   if (ws_bytes < img) return DQT_ERR_ARG;
-  if (K % 16 || !aligned16(Xq) || !aligned16(ws)) return DQT_ERR_ALIGN;
+  if (K % 16 || N % 8 || !aligned16(Xq) || !aligned16(ws) || !aligned16(dY) ||
+      (W && !aligned16(W)) || (m && !aligned16(m)) || (v && !aligned16(v)) ||
+      (dW_out && !aligned16(dW_out)))
+    return DQT_ERR_ALIGN;
   // the argument checks of the GEMM call before anything is launched
   const bool upd = W || m || v;
   if (upd && (!W || !m || !v)) return DQT_ERR_ARG;

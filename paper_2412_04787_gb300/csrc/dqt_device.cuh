@@ -7,7 +7,6 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
-#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -193,36 +192,6 @@ __device__ __forceinline__ uint64_t l2_policy_evict_last() {
   return pol;
 }
 
-// Orders this thread's earlier generic-proxy writes to shared memory before
-// later async-proxy accesses (TMA, tcgen05.mma operand reads) that are
-// ordered after it through an mbarrier.
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
-// Sixteen int8 codes (one 16-byte vector) as sixteen exact fp16 values (two
-// 16-byte vectors).  For a signed byte b, u = b XOR 0x80 = b + 128 in
-// [0, 255]; the fp16 bit pattern 0x6400 | u is 1024 + u exactly (fp16 holds
-// every integer up to 2048), and 1024 + u - 1152 = b, exact again.  One
-// byte permute builds two such halves, one packed subtraction finishes them.
-__device__ __forceinline__ void i8x16_to_f16(const uint4 in, uint4& lo, uint4& hi) {
-  const uint32_t w[4] = {in.x ^ 0x80808080u, in.y ^ 0x80808080u, in.z ^ 0x80808080u,
-                         in.w ^ 0x80808080u};
-  const __half2 bias = __halves2half2(__ushort_as_half(0x6480), __ushort_as_half(0x6480));
-  uint32_t o[8];
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    const uint32_t a = __byte_perm(w[j], 0x64646464u, 0x4140);  // bytes 0, 1
-    const uint32_t b = __byte_perm(w[j], 0x64646464u, 0x4342);  // bytes 2, 3
-    const __half2 ha = __hsub2(*reinterpret_cast<const __half2*>(&a), bias);
-    const __half2 hb = __hsub2(*reinterpret_cast<const __half2*>(&b), bias);
-    o[2 * j] = *reinterpret_cast<const uint32_t*>(&ha);
-    o[2 * j + 1] = *reinterpret_cast<const uint32_t*>(&hb);
-  }
-  lo = make_uint4(o[0], o[1], o[2], o[3]);
-  hi = make_uint4(o[4], o[5], o[6], o[7]);
-}
-
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
@@ -395,11 +364,6 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool a_mn, bool 
   return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn ? 1u : 0u) << 15) |
          ((b_mn ? 1u : 0u) << 16) | (static_cast<uint32_t>(N >> 3) << 17) |
          (static_cast<uint32_t>(M >> 4) << 24);
-}
-// The same for fp16 A and B (type code 0 in both operand-type fields).
-__host__ __device__ constexpr uint32_t idesc_f16(int M, int N, bool a_mn, bool b_mn) {
-  return (1u << 4) | ((a_mn ? 1u : 0u) << 15) | ((b_mn ? 1u : 0u) << 16) |
-         (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
 }
 // kind::f8f6f4 with both operands E4M3 (format code 0 in the A and B type
 // fields), fp32 accumulator, both K-major.

@@ -34,14 +34,12 @@ struct GemmLaunch {
   // Output is M x N, reduced over Kred.
   int M, N, Kred;
   // Operands (bf16, row-major, contiguous):
-  //   FWD: A = Xq_img [M=T, Kred=K],  B = W_img [N, Kred=K]     (both K-major);
-  //        with i8, A = Xq and B = W, the int8 codes themselves
+  //   FWD: A = Xq_img [M=T, Kred=K],  B = W_img [N, Kred=K]     (both K-major)
   //   DX : A = dY     [M=T, Kred=N],  B = W_img [Kred=N, N=K]   (B MN-major)
   //   DW : A = dY     [Kred=T, M=N],  B = Xdq   [Kred=T, N=K]   (both MN-major)
   //   FWD8: A = Xq8 [M=T, Kred=K], B = W8 [N, Kred=K], E4M3 bytes (both K-major)
   const void* A;
   const void* B;
-  bool i8;      // FWD: A and B are int8 codes (converted to fp16 in shared memory)
   int chunk_k;  // FWD: reduction elements per exact fp32 chunk (multiple of 64)
   bool pair;    // use the 2-SM (cta_group::2) kernel (not with drained chunks)
   // Epilogue operands.

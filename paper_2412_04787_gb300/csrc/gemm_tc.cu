@@ -606,46 +606,29 @@ __global__ void __launch_bounds__(kThreads, 1)
 // Epilogue warps of the 2-SM kernels: the dW update is compute-heavy (AdamW,
 // Philox, stochastic rounding per weight) and needs four warps per SM
 // sub-partition to hide its latencies; the forward and dX epilogues are light.
-// I8 (forward only): the operands arrive as int8 codes.  TMA stages each
-// CTA's 128 rows of A and of B (64 bytes of the reduction per row, unswizzled)
-// in a ring of int8 stages; CW converter warps turn every stage into exact
-// fp16 values written in the 128-byte-swizzled K-major layout the MMA reads
-// (i8x16_to_f16), then signal the leader.  The MMAs run on fp16 operands.
-template <int EPI, bool DR = false, bool I8 = false>
+template <int EPI, bool DR = false>
 struct PairCfg {
   // DR: the exact forward that drains its fp32 accumulator into int32 sums;
   // its folds stall the MMAs, so they are spread over twice the warps
   static constexpr int EW = (EPI == GEMM_DW || DR) ? 16 : 8;
-  // converter warps (warps 2 .. 2 + CW - 1); two beside the drained
-  // forward's sixteen epilogue warps, whose int32 running sums need the
-  // registers
-  static constexpr int CW = I8 ? (DR ? 2 : 4) : 0;
-  static constexpr int THREADS = 64 + 32 * (CW + EW);
+  static constexpr int THREADS = 64 + 32 * EW;
 };
 
-template <int EPI, bool DR = false, bool I8 = false>
+template <int EPI, bool DR = false>
 struct SmemPair {
-  static constexpr int EW = PairCfg<EPI, DR, I8>::EW;
+  static constexpr int EW = PairCfg<EPI, DR>::EW;
   static constexpr int A_BYTES = 128 * BK * 2;
   static constexpr int B_BYTES = 128 * BK * 2;  // this CTA's half of the B tile
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int STAGES = I8 ? 5 : ((EPI == GEMM_DW) ? 5 : 7);
-  // I8: int8 staging ring (this CTA's A rows, then its B rows, 64 B each)
-  static constexpr int A8_BYTES = I8 ? 128 * BK : 0;
-  static constexpr int STAGE8_BYTES = 2 * A8_BYTES;
-  static constexpr int STAGES8 = I8 ? 4 : 0;
-  static constexpr int I8_OFF = STAGES * STAGE_BYTES;
-  static constexpr int XPOSE_OFF = I8_OFF + STAGES8 * STAGE8_BYTES;
+  static constexpr int STAGES = (EPI == GEMM_DW) ? 5 : 7;
+  static constexpr int XPOSE_OFF = STAGES * STAGE_BYTES;
   static constexpr int XPOSE_BYTES = (EPI == GEMM_DW) ? EW * 32 * kStageLd * 4 : 0;
   static constexpr int BAR_OFF = XPOSE_OFF + XPOSE_BYTES;
   // alignment slack for the 1024-byte swizzle atoms, as much as fits
   static constexpr int SLACK = (232448 - (BAR_OFF + 256)) < 1024 ? (232448 - (BAR_OFF + 256)) : 1024;
   static constexpr int BYTES = BAR_OFF + 256 + SLACK;
   static_assert(SLACK >= 0, "shared memory per CTA");
-  // barriers: full, empty [STAGES]; acc_full, acc_empty [2]; drain; the
-  // tensor-memory slot; I8: full8, empty8 [STAGES8]; dW: update constants at 176
-  static constexpr int BAR_END = (2 * STAGES + 5) * 8 + 8 + 16 * STAGES8;
-  static_assert(EPI == GEMM_DW ? BAR_END <= 176 : BAR_END <= 256, "barrier area");
+  static_assert((2 * STAGES + 5) * 8 + 4 <= 176, "barrier area: barriers, then the update constants");
 };
 
 // DR (forward only): every chunk of chunk_kb k-blocks is accumulated on its
@@ -656,26 +639,20 @@ struct SmemPair {
 // UCD: the dW update constants come from device memory (p.uc_dev, copied to
 // shared memory once); otherwise the epilogue reads them straight from the
 // kernel's parameter space, where they take no registers.
-template <bool A_MN, bool B_MN, int EPI, bool PK = false, bool DR = false, bool UCD = false,
-          bool I8 = false>
-__global__ void __launch_bounds__(PairCfg<EPI, DR, I8>::THREADS, 1)
+template <bool A_MN, bool B_MN, int EPI, bool PK = false, bool DR = false, bool UCD = false>
+__global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
     gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA,
                      const __grid_constant__ CUtensorMap tmB, const __grid_constant__ Params p) {
-  using S = SmemPair<EPI, DR, I8>;
+  using S = SmemPair<EPI, DR>;
   static_assert(!DR || EPI == GEMM_FWD, "drained chunks: exact integer forward only");
-  static_assert(!I8 || (EPI == GEMM_FWD && !A_MN && !B_MN), "int8 operands: K-major forward");
   constexpr int ST = S::STAGES;
   constexpr int EW = S::EW;
-  constexpr int CW = PairCfg<EPI, DR, I8>::CW;
-  constexpr int EPI0 = 2 + CW;         // first epilogue warp
   constexpr int BN = 256;           // pair tile width; each CTA holds all 256 columns of its rows
   constexpr int HALF = BN / (EW / 4);  // columns per epilogue warp
   constexpr bool F8 = EPI == GEMM_FWD8;
   constexpr int KB = F8 ? 128 : BK;  // reduction elements per stage (one 128-byte row)
   static_assert(!F8 || (!A_MN && !B_MN), "E4M3 operands are read K-major");
-  constexpr uint32_t IDESC = F8   ? idesc_e4m3(256, 256)
-                             : I8 ? idesc_f16(256, 256, false, false)
-                                  : idesc_bf16(256, 256, A_MN, B_MN);
+  constexpr uint32_t IDESC = F8 ? idesc_e4m3(256, 256) : idesc_bf16(256, 256, A_MN, B_MN);
   constexpr uint32_t TMEM_COLS = 512;
   constexpr uint32_t MN_CHUNK_BYTES = 64 * BK * 2;
 
@@ -695,9 +672,6 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR, I8>::THREADS, 1)
   uint64_t* acc_empty = acc_full + 2;  // [2], used on the leader
   uint64_t* drain_bar = acc_empty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
-  uint64_t* full8 = drain_bar + 2;        // I8: int8 stage landed (this CTA's TMA)
-  uint64_t* empty8 = full8 + S::STAGES8;  // I8: int8 stage converted (this CTA)
-  uint8_t* s8 = smem + S::I8_OFF;
   // update constants, read by the dW epilogue from shared memory
   UpdateConsts* uc_s = reinterpret_cast<UpdateConsts*>(smem + S::BAR_OFF + 176);
 
@@ -710,14 +684,8 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR, I8>::THREADS, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < ST; ++s) {
-      // I8: an operand stage is full once every converter warp of both CTAs
-      // has written its share
-      mbar_init(&full[s], I8 ? 2 * CW : 1);
+      mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
-    }
-    for (int s = 0; s < S::STAGES8; ++s) {
-      mbar_init(&full8[s], 1);
-      mbar_init(&empty8[s], CW);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
@@ -738,86 +706,7 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR, I8>::THREADS, 1)
   const uint32_t full_lead = mapa_shared(smem_u32(full), 0);
   const uint32_t acc_empty_lead = mapa_shared(smem_u32(acc_empty), 0);
 
-  if (I8 && warp == 0) {
-    if (lane == 0) {
-      // ---------------- TMA producer of int8 stages (each CTA its own) ----
-      int it = 0, s = 0;
-      uint32_t ph = 0;
-      bool ok = true;
-      for (int t = cid; t < p.num_tiles && ok; t += ncl) {
-        const Unit un = decode_unit(p, t);
-        const int m0 = (un.tile / p.num_n) * 256 + static_cast<int>(rank) * 128;
-        const int n0 = (un.tile % p.num_n) * BN + static_cast<int>(rank) * 128;
-        for (int kb = un.kb0; kb < un.kb1; ++kb, ++it) {
-          if (it >= S::STAGES8 && !mbar_wait(&empty8[s], ph ^ 1u, p.wait_ns)) {
-            ok = false;
-            break;
-          }
-          uint8_t* a8 = s8 + s * S::STAGE8_BYTES;
-          mbar_arrive_expect_tx(&full8[s], S::STAGE8_BYTES);
-          tma_load_2d(&tmA, &full8[s], a8, kb * BK, m0);
-          tma_load_2d(&tmB, &full8[s], a8 + S::A8_BYTES, kb * BK, n0);
-          if (++s == S::STAGES8) {
-            s = 0;
-            ph ^= 1u;
-          }
-        }
-      }
-      if (!ok) record_timeout(p.status);
-      // let this CTA's last copies land before it exits
-      for (int i = (it > S::STAGES8 ? it - S::STAGES8 : 0); i < it; ++i)
-        mbar_wait(&full8[i % S::STAGES8], (i / S::STAGES8) & 1u, kDrainNs);
-    }
-  } else if (I8 && warp >= 2 && warp < EPI0) {
-    // ---------------- converters (warps 2 .. 2 + CW - 1, both CTAs) ----------
-    // Per k-block this CTA stages 2 x 128 rows of 64 codes: 1024 16-byte
-    // vectors, 1024 / (32 CW) per converter thread.  Vector c covers row c / 4 of A
-    // (c < 512) or of B, codes 16 (c % 4) .. +15, which land as two 16-byte
-    // fp16 chunks 2 (c % 4) and 2 (c % 4) + 1 of that row, XOR-swizzled with
-    // the row index mod 8 (the 128-byte swizzle TMA would have written).
-    const int tid = (warp - 2) * 32 + lane;
-    int it = 0, s = 0, q = 0;  // k-blocks converted; fp16 stage, int8 stage
-    uint32_t ph = 0, ph8 = 0;
-    bool ok = true;
-    for (int t = cid; t < p.num_tiles && ok; t += ncl) {
-      const Unit un = decode_unit(p, t);
-      for (int kb = un.kb0; kb < un.kb1; ++kb, ++it) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&full8[q], ph8, p.wait_ns));
-        if (ok && it >= ST) ok = __all_sync(0xffffffffu, mbar_wait_cl(&empty[s], ph ^ 1u, p.wait_ns));
-        if (!ok) break;
-        const uint8_t* src = s8 + q * S::STAGE8_BYTES;
-        uint8_t* dA = sA + s * S::A_BYTES;
-        uint8_t* dB = sB + s * S::B_BYTES;
-#pragma unroll
-        for (int i = 0; i < 1024 / (32 * CW); ++i) {
-          const int c = tid + 32 * CW * i;
-          const int cc = c & 511;
-          const int r = cc >> 2, j = cc & 3;
-          const uint4 v = *reinterpret_cast<const uint4*>(src + c * 16);
-          uint4 lo, hi;
-          i8x16_to_f16(v, lo, hi);
-          uint8_t* row = (c < 512 ? dA : dB) + r * 128;
-          *reinterpret_cast<uint4*>(row + (((2 * j) ^ (r & 7)) << 4)) = lo;
-          *reinterpret_cast<uint4*>(row + (((2 * j + 1) ^ (r & 7)) << 4)) = hi;
-        }
-        fence_proxy_async_smem();  // the MMA reads these through the async proxy
-        __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(&empty8[q]);
-          mbar_arrive_cluster(full_lead + 8u * s);
-        }
-        if (++s == ST) {
-          s = 0;
-          ph ^= 1u;
-        }
-        if (++q == S::STAGES8) {
-          q = 0;
-          ph8 ^= 1u;
-        }
-      }
-    }
-    if (!ok && lane == 0) record_timeout(p.status);
-  } else if (warp == 0) {
+  if (warp == 0) {
     if (lane == 0) {
       // ---------------- TMA producer (both CTAs) ----------------
       int it = 0, s = 0;  // k-blocks issued; stage it % ST
@@ -945,12 +834,12 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR, I8>::THREADS, 1)
       mbar_wait_cl(drain_bar, 0, kDrainNs);
     }
   } else {
-    // ---------------- epilogue (warps EPI0 .. EPI0+EW-1, both CTAs) --------
+    // ---------------- epilogue (warps 2 .. EW+1, both CTAs) ----------------
     const int quad = warp & 3;        // tensor-memory lanes this warp may access
-    const int half = (warp - EPI0) >> 2;  // which run of HALF columns
+    const int half = (warp - 2) >> 2;  // which run of HALF columns
     const int row = quad * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
-    float* xp = reinterpret_cast<float*>(smem + S::XPOSE_OFF) + (warp - EPI0) * 32 * kStageLd;
+    float* xp = reinterpret_cast<float*>(smem + S::XPOSE_OFF) + (warp - 2) * 32 * kStageLd;
     const UpdateConsts& uc = UCD ? *uc_s : p.uc;
     uint32_t n_changed = 0;
     int u = 0;
@@ -1078,11 +967,11 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 2-D row-major matrix of 2-byte (bf16) or 1-byte (E4M3, int8) elements with
+// 2-D row-major matrix of 2-byte (bf16) or 1-byte (E4M3) elements with
 // `inner` contiguous elements per row and `outer` rows; box of box_inner x
-// box_outer, 128-byte swizzle (or none), zero fill.
+// box_outer, 128-byte swizzle, zero fill.
 bool make_map(CUtensorMap* map, const void* ptr, uint64_t inner, uint64_t outer,
-              uint32_t box_inner, uint32_t box_outer, int elem_bytes = 2, bool swizzle = true) {
+              uint32_t box_inner, uint32_t box_outer, int elem_bytes = 2) {
   EncodeTiledFn enc = encode_fn();
   if (!enc) return false;
   // The encoder is a driver call and needs a context current in the calling
@@ -1100,8 +989,7 @@ bool make_map(CUtensorMap* map, const void* ptr, uint64_t inner, uint64_t outer,
   const cuuint32_t estr[2] = {1, 1};
   return enc(map, elem_bytes == 1 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
              2, const_cast<void*>(ptr), dims, strides, box,
-             estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-             swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -1126,8 +1014,7 @@ int launch_tiles(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStr
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
-template <bool A_MN, bool B_MN, int EPI, bool PK = false, bool DR = false, bool UCD = false,
-          bool I8 = false>
+template <bool A_MN, bool B_MN, int EPI, bool PK = false, bool DR = false, bool UCD = false>
 int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream,
                  void* tail_ws = nullptr, size_t tail_ws_bytes = 0, TailPlan* plan = nullptr);
 
@@ -1180,12 +1067,12 @@ int dw_splits(int M, int N, int Kred) {
 
 namespace {
 
-template <bool A_MN, bool B_MN, int EPI, bool PK, bool DR, bool UCD, bool I8>
+template <bool A_MN, bool B_MN, int EPI, bool PK, bool DR, bool UCD>
 int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream,
                  void* tail_ws, size_t tail_ws_bytes, TailPlan* plan) {
-  auto kern = gemm_pair_kernel<A_MN, B_MN, EPI, PK, DR, UCD, I8>;
-  const int smem = SmemPair<EPI, DR, I8>::BYTES;
-  constexpr int threads = PairCfg<EPI, DR, I8>::THREADS;
+  auto kern = gemm_pair_kernel<A_MN, B_MN, EPI, PK, DR, UCD>;
+  const int smem = SmemPair<EPI, DR>::BYTES;
+  constexpr int threads = PairCfg<EPI, DR>::THREADS;
   static int max_clusters = 0;  // per template instance
   p.num_n = (p.N + 255) / 256;
   p.num_tiles = ((p.M + 255) / 256) * p.num_n * p.splits;
@@ -1289,15 +1176,6 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   CUtensorMap ta, tb;
   switch (g.kind) {
     case GEMM_FWD:
-      if (g.i8) {
-        // int8 codes, converted to fp16 in shared memory: 2-SM tiles whatever
-        // the tiling mode; 64-byte unswizzled rows of this CTA's 128 rows
-        if (!make_map(&ta, g.A, g.Kred, g.M, BK, 128, 1, false)) return 3;
-        if (!make_map(&tb, g.B, g.Kred, g.N, BK, 128, 1, false)) return 3;
-        if (drain)
-          return launch_pairs<false, false, GEMM_FWD, false, true, false, true>(ta, tb, p, stream);
-        return launch_pairs<false, false, GEMM_FWD, false, false, false, true>(ta, tb, p, stream);
-      }
       if (!make_map(&ta, g.A, g.Kred, g.M, BK, BM)) return 3;
       if (drain) {
         if (!make_map(&tb, g.B, g.Kred, g.N, BK, 128)) return 3;

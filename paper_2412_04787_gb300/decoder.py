@@ -24,9 +24,17 @@ stream-ordered before each replay).
 
 import torch
 import torch.nn.functional as F
+from torch.nn.attention import SDPBackend, sdpa_kernel
 
 from . import dqt
 from .bitlinear import DQTBitLinear
+
+# Attention runs on PyTorch's FlashAttention kernels (memory-efficient
+# attention where FlashAttention does not apply), never on cuDNN's fused
+# attention: a CUDA-graph replay of this decoder raised an illegal memory
+# access with the cuDNN backend selected, and a PyTorch default that changes
+# between versions must not route back onto it.
+_SDPA_BACKENDS = [SDPBackend.FLASH_ATTENTION, SDPBackend.EFFICIENT_ATTENTION]
 
 __all__ = ["DecoderConfig", "DQTDecoder"]
 
@@ -151,7 +159,8 @@ class Block(torch.nn.Module):
         q = _Rope.apply(self.q(a).view(B, S, nh, hd), cos_sin).transpose(1, 2)
         k = _Rope.apply(self.k(a).view(B, S, nh, hd), cos_sin).transpose(1, 2)
         v = self.v(a).view(B, S, nh, hd).transpose(1, 2)
-        o = F.scaled_dot_product_attention(q, k, v, is_causal=True)
+        with sdpa_kernel(_SDPA_BACKENDS):
+            o = F.scaled_dot_product_attention(q, k, v, is_causal=True)
         x = x + self.o(o.transpose(1, 2).reshape(B, S, Hd))
         m = self.mlp_norm(x)
         return x + self.down(_SwiGLU.apply(self.gate(m), self.up(m)))

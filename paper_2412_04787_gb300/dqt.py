@@ -33,7 +33,7 @@ EXPORTED = [
     "dqt_rmsnorm_bwd_workspace_size", "dqt_rmsnorm_bwd_bf16",
     "dqt_act_quant_images", "dqt_bitlinear_fwd_img", "dqt_bitlinear_bwd_dx_img",
     "dqt_bwd_dx_workspace_size", "dqt_bitlinear_bwd_dw_update_img",
-    "dqt_bwd_dw_img_workspace_size", "dqt_codes_to_xdq",
+    "dqt_bwd_dw_img_workspace_size", "dqt_codes_to_xdq", "dqt_fwd_workspace_size",
 ]
 
 
@@ -92,8 +92,11 @@ def lib():
         L.dqt_codes_to_bf16.argtypes = [_vp, _i64, _vp, _vp]
         L.dqt_codes_to_xdq.argtypes = [_vp, _vp, _i64, _i64, _vp, _vp]
         L.dqt_bitlinear_fwd.argtypes = [_vp, _vp, _vp, _f32, dqt_grid_t, _i64, _i64, _i64, _vp,
-                                        _vp, _vp]
-        L.dqt_bitlinear_fwd_img.argtypes = L.dqt_bitlinear_fwd.argtypes
+                                        _vp, _vp, _sz, _vp]
+        L.dqt_fwd_workspace_size.argtypes = [_i64, _i64, _i64]
+        L.dqt_fwd_workspace_size.restype = _sz
+        L.dqt_bitlinear_fwd_img.argtypes = [_vp, _vp, _vp, _f32, dqt_grid_t, _i64, _i64, _i64,
+                                            _vp, _vp, _vp]
         L.dqt_bitlinear_bwd_dx.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp, _sz, _vp]
         L.dqt_bitlinear_bwd_dx_img.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp]
         L.dqt_bwd_dx_workspace_size.argtypes = [_i64, _i64]
@@ -159,6 +162,7 @@ def lib():
             if name not in ("dqt_status_string", "dqt_absmean_workspace_size",
                             "dqt_update_consts_size", "dqt_bwd_dw_workspace_size",
                             "dqt_bwd_dw_img_workspace_size", "dqt_bwd_dx_workspace_size",
+                            "dqt_fwd_workspace_size",
                             "dqt_adafactor_workspace_size",
                             "dqt_bwd_dw_adafactor_workspace_size",
                             "dqt_rmsnorm_bwd_workspace_size"):
@@ -321,8 +325,13 @@ def dqt_codes_to_xdq(Xq, s_x, Xdq=None, stream=None):
     return Xdq
 
 
-def dqt_bitlinear_fwd(Xq, s_x, W, s_w, bits_or_grid, Y=None, acc_out=None, stream=None):
-    """Sec. 3.2 forward on the int8 codes (converted to fp16 inside the GEMM)."""
+def dqt_fwd_workspace_size(T, K, N):
+    return int(lib().dqt_fwd_workspace_size(T, K, N))
+
+
+def dqt_bitlinear_fwd(Xq, s_x, W, s_w, bits_or_grid, Y=None, acc_out=None, ws=None, stream=None):
+    """Sec. 3.2 forward from the int8 codes; `ws` (uint8 CUDA tensor of
+    dqt_fwd_workspace_size bytes) receives their bf16 images, allocated if None."""
     _need(Xq, "Xq", torch.int8)
     T, K = Xq.shape
     _need(W, "W", torch.int8)
@@ -333,9 +342,13 @@ def dqt_bitlinear_fwd(Xq, s_x, W, s_w, bits_or_grid, Y=None, acc_out=None, strea
         Y = torch.empty((T, N), dtype=torch.bfloat16, device=Xq.device)
     _need(Y, "Y", torch.bfloat16, (T, N))
     _opt(acc_out, "acc_out", torch.int32, (T, N))
+    if ws is None:
+        ws = torch.empty(lib().dqt_fwd_workspace_size(T, K, N), dtype=torch.uint8,
+                         device=Xq.device)
+    _need(ws, "ws", torch.uint8)
     _check(lib().dqt_bitlinear_fwd(_ptr(Xq), _ptr(s_x), _ptr(W), float(s_w),
                                    _grid(bits_or_grid), T, K, N, _ptr(Y), _ptr(acc_out),
-                                   _stream(stream)), "dqt_bitlinear_fwd")
+                                   _ptr(ws), ws.numel(), _stream(stream)), "dqt_bitlinear_fwd")
     return Y
 
 

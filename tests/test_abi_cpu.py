@@ -64,32 +64,34 @@ def test_argument_validation_without_launch(L):
     g = dqt.dqt_grid_t(-1, 1)
     A = _p(0x10000)  # never dereferenced: validation fails before any CUDA call
     # null pointers
-    assert L.dqt_bitlinear_fwd(None, A, A, 1.0, g, 4, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_fwd(None, A, A, 1.0, g, 4, 8, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ARG
     assert L.dqt_bitlinear_bwd_dx(A, None, 1.0, 4, 8, 8, A, A, 1 << 20, None) == dqt.DQT_ERR_ARG
     assert L.dqt_bitlinear_bwd_dx(A, A, 1.0, 4, 8, 8, A, None, 1 << 20, None) == dqt.DQT_ERR_ARG
     assert L.dqt_act_quant(A, 4, 8, None, A, None) == dqt.DQT_ERR_ARG
     assert L.dqt_act_quant_images(A, 4, 8, None, A, None, None, None) == dqt.DQT_ERR_ARG
     assert L.dqt_bitlinear_fwd_img(None, A, A, 1.0, g, 4, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
     # sizes
-    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g, 0, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g, 0, 8, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ARG
     assert L.dqt_act_quant(A, -1, 8, A, A, None) == dqt.DQT_ERR_ARG
     # the dX workspace must hold the weight's bf16 image
     assert L.dqt_bwd_dx_workspace_size(8, 8) >= 8 * 8 * 2
     assert L.dqt_bitlinear_bwd_dx(A, A, 1.0, 4, 8, 8, A, A, 64, None) == dqt.DQT_ERR_ARG
-    # int8 rows of the forward: K a multiple of 16; bf16 rows: K, N multiples
-    # of 8; 16-byte alignment
-    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g, 4, 24, 8, A, None, None) == dqt.DQT_ERR_ALIGN
+    # K, N multiples of 8 and 16-byte alignment; the forward's workspace holds
+    # both operands' bf16 images
+    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g, 4, 12, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_fwd_workspace_size(4, 8, 8) >= (4 + 8) * 8 * 2
+    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g, 4, 8, 8, A, None, A, 16, None) == dqt.DQT_ERR_ARG
     assert L.dqt_bitlinear_fwd_img(A, A, A, 1.0, g, 4, 12, 8, A, None, None) == dqt.DQT_ERR_ALIGN
     assert L.dqt_bitlinear_bwd_dx(A, A, 1.0, 4, 8, 20, A, A, 1 << 20, None) == dqt.DQT_ERR_ALIGN
     assert L.dqt_bitlinear_bwd_dx_img(A, A, 1.0, 4, 8, 20, A, None) == dqt.DQT_ERR_ALIGN
-    assert L.dqt_bitlinear_fwd(_p(0x10004), A, A, 1.0, g, 4, 16, 8, A, None, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_bitlinear_fwd(_p(0x10004), A, A, 1.0, g, 4, 8, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ALIGN
     # bad grid / scale
-    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, dqt.dqt_grid_t(2, 1), 4, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
-    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, dqt.dqt_grid_t(-129, 1), 4, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
-    assert L.dqt_bitlinear_fwd(A, A, A, 0.0, g, 4, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, dqt.dqt_grid_t(2, 1), 4, 8, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, dqt.dqt_grid_t(-129, 1), 4, 8, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_fwd(A, A, A, 0.0, g, 4, 8, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ARG
     # int32 accumulator range: K * 128 * 128 must fit int32
     g8 = dqt.dqt_grid_t(-128, 127)
-    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g8, 4, 1 << 17, 8, A, None, None) == dqt.DQT_ERR_RANGE
+    assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g8, 4, 1 << 17, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_RANGE
 
 
 def test_update_argument_validation(L):

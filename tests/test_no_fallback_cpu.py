@@ -47,3 +47,14 @@ def test_missing_library_raises(monkeypatch):
     monkeypatch.setattr(dqt, "_lib", None)
     with pytest.raises(RuntimeError, match="no CPU fallback"):
         dqt.lib()
+
+
+def test_decoder_attention_is_pinned_off_cudnn():
+    """The decoder's attention is pinned to FlashAttention / memory-efficient
+    attention: cuDNN's fused attention is never selected, whatever PyTorch's
+    default priority."""
+    from torch.nn.attention import SDPBackend
+
+    from paper_2412_04787_gb300 import decoder
+    assert SDPBackend.CUDNN_ATTENTION not in decoder._SDPA_BACKENDS
+    assert decoder._SDPA_BACKENDS[0] == SDPBackend.FLASH_ATTENTION
