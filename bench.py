@@ -260,8 +260,8 @@ class MLPStep:
         update of this rank's shard (its moments only, ZeRO-1) and an
         all-gather of the int8 codes (paper_2412_04787_gb300/dp.py)."""
         from paper_2412_04787_gb300 import dp
-        if not self.i8:
-            raise SystemExit("the data-parallel exchange runs on the int8-operand AdamW step")
+        if self.packed or self.optimizer != "adamw":
+            raise SystemExit("the data-parallel exchange runs the AdamW step on int8 codes")
         self.dp = {}
         for name, _, _ in PROJ:
             upd = dp.DataParallelUpdater(self.W[name])
@@ -379,12 +379,32 @@ class MLPStep:
         def dw(i, name, stream):
             xdq = self.aq["H" if name == "down" else "X"][2]
             ch = self.changed[i:i + 1]
+            if self.dp and not self.i8:
+                upd = self.dp[name]
+                ws = self.dw_ws[s.index(stream)]
+                timed("bwd_dw", stream, lambda: dqt.dqt_bitlinear_bwd_dw_update_img(
+                    self.d["dY_" + name], xdq, None, self.s_w[name], None, None, None, None,
+                    self.grid, dW_out=upd.grad_view(), ws=ws))
+                timed("dp_exchange", stream, lambda: upd.step(
+                    self.s_w[name], hp, self.sr[name], self.grid, changed_out=ch))
+                return
             if self.i8 and self.dp:
                 s_x, q, _ = self.aq["H" if name == "down" else "X"]
                 upd = self.dp[name]
-                timed("bwd_dw", stream, lambda: dqt.dqt_bitlinear_bwd_dw_update(
-                    self.d["dY_" + name], q, s_x, None, self.s_w[name], None, None, None, None,
-                    self.grid, dW_out=upd.grad_view(), ws=self.dw_ws[s.index(stream)]))
+                ws = self.dw_ws[s.index(stream)]
+                if parts:  # the call's conversion and gradient GEMM, timed apart
+                    T_, K_ = q.shape
+                    img_bytes = (T_ * K_ * 2 + 255) // 256 * 256
+                    img = ws[: T_ * K_ * 2].view(torch.bfloat16).view(T_, K_)
+                    rest = ws[img_bytes:]
+                    timed("codes_to_xdq", stream, lambda: dqt.dqt_codes_to_xdq(q, s_x, img))
+                    timed("bwd_dw", stream, lambda: dqt.dqt_bitlinear_bwd_dw_update_img(
+                        self.d["dY_" + name], img, None, self.s_w[name], None, None, None, None,
+                        self.grid, dW_out=upd.grad_view(), ws=rest if rest.numel() else False))
+                else:
+                    dqt.dqt_bitlinear_bwd_dw_update(
+                        self.d["dY_" + name], q, s_x, None, self.s_w[name], None, None, None, None,
+                        self.grid, dW_out=upd.grad_view(), ws=ws)
                 timed("dp_exchange", stream, lambda: upd.step(
                     self.s_w[name], hp, self.sr[name], self.grid, changed_out=ch))
                 return
@@ -498,6 +518,41 @@ class MLPStep:
             "codes_to_xdq": [3.0 * T * K + 4 * T for _, K, N in PROJ],
         }
         return flops, byts, overhead
+
+
+def int8_api_step(dev, args, bits):
+    """The same MLP step through the C ABI calls on int8 codes (each GEMM
+    call makes the bf16 images it needs in its workspace): the step time in
+    the same four-stream DAG, and the serial time of its image conversions."""
+    st = MLPStep(dev, bits=bits, operands="int8")
+    for _ in range(args.warmup):
+        st.run()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(args.steps):
+        st.run()
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / args.steps
+    timers = {k: [] for k in st.kinds}
+    for _ in range(args.steps):
+        st.run(timers, serial=True)
+    torch.cuda.synchronize()
+    st.dqt.dqt_check_device_status()
+    per = {k: sum(_elapsed(timers[k])) / args.steps for k in st.kinds}
+    peaks, _ = _peaks()
+    aq_bytes = (T_TOK * HID * 3.0 + 4 * T_TOK) + (T_TOK * INTER * 3.0 + 4 * T_TOK)
+    return {"value": round(T_TOK / (ms / 1e3), 1), "unit": "tokens/s",
+            "ms_per_step": round(ms, 4),
+            "operands": "int8 codes through the C ABI (dqt_act_quant, dqt_bitlinear_fwd, "
+                        "dqt_bitlinear_bwd_dx, dqt_bitlinear_bwd_dw_update)",
+            "conversion_ms_per_step_serial": round(per["codes_to_bf16"] + per["codes_to_xdq"], 4),
+            "act_quant_frac_of_hbm": round(aq_bytes / (per["act_quant"] / 1e3) / 1e9 /
+                                           peaks["hbm_gbs"], 4),
+            "kernel_ms_per_step_serial": {k: round(v, 4) for k, v in per.items()}}
 
 
 def _elapsed(pairs):
@@ -629,7 +684,9 @@ def run_gpu(args):
     for k in kinds:
         d = dict(per[k])
         sec = per[k]["total_ms"] / 1e3
-        if k == "dp_exchange":
+        if sec <= 0.0:
+            pass  # no launch of this kind in the step
+        elif k == "dp_exchange":
             pass  # reduce-scatter + shard update + all-gather: time only
         elif k in flops:
             d["tflops"] = sum(flops[k]) * args.steps / sec / 1e12
@@ -720,7 +777,10 @@ def run_gpu(args):
     # single-layer step (256 x 512 x 512) and the standalone update's
     # bandwidth sweep of the 8-bit configuration
     extra = {}
-    if rank == 0 and ws == 1 and not args.no_extras and st.i8 and dp_mode != "exchange":
+    if (rank == 0 and ws == 1 and not args.no_extras and dp_mode != "exchange" and not st.i8
+            and not st.fp8 and not st.packed and st.optimizer == "adamw"):
+        extra["int8_c_abi_step"] = int8_api_step(dev, args, st.bits)
+    if rank == 0 and ws == 1 and not args.no_extras and dp_mode != "exchange" and not st.fp8:
         lay = layer_step(1.58, 200, 10)
         extra["layer_256x512x512"] = {k: lay[k] for k in (
             "value", "unit", "us_per_step", "graph", "e2e", "changed_codes_last_step", "clocks")}
@@ -1441,9 +1501,10 @@ def main():
     ap.add_argument("--optimizer", default="adamw", choices=["adamw", "adafactor"],
                     help="the DQT optimiser of the BitLinear weights")
     ap.add_argument("--packed", action="store_true", help="2-bit packed ternary code storage")
-    ap.add_argument("--operands", default="int8", choices=["int8", "img"],
-                    help="mlp: the hot-path C ABI on int8 codes (default) or the *_img calls on "
-                         "shared bf16 operand images")
+    ap.add_argument("--operands", default="img", choices=["int8", "img"],
+                    help="mlp: the *_img calls on operand images written once and shared "
+                         "between GEMMs (default), or the C ABI calls on int8 codes, each "
+                         "making its own images in its workspace")
     ap.add_argument("--dp", default="auto", choices=["auto", "exchange", "replicas"],
                     help="several ranks: the data-parallel exchange (auto, the default) or "
                          "independent replicas; exchange on one GPU uses a one-rank group")
