@@ -80,7 +80,8 @@ def kernel_fingerprint(files=GEMM_SOURCES):
 # of operand and optimiser-state bytes), from one ncu capture, keyed by the
 # GEMM-source fingerprint it was taken on (see profiles/).  A stale entry
 # reports null.
-DW_TRAFFIC_BYTES = {"82d12725fdfa": 262571008 + 61169152 + 33047808}
+DW_TRAFFIC_BYTES = {"82d12725fdfa": 262571008 + 61169152 + 33047808,
+                    "a25cf8632190": 261430272 + 59386112 + 33048064}
 
 
 def _dist():
