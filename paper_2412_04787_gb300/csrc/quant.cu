@@ -129,163 +129,51 @@ __global__ void __launch_bounds__(kAqWarps * 32)
   }
 }
 
-// Single-pass variant: WPR warps share a row and each lane keeps its (at
-// most NV) 16-byte vectors of the row in registers between the absmax and the
-// quantisation, so registers stay low and many rows are in flight per SM.
-// The warps of a row combine their partial amax through shared memory.  The
-// dequantised image needs bf16(q / s_x) for q in [-128, 127] only, so the
-// row's threads first fill a 256-entry table of those correctly rounded
-// quotients and then look them up: bit-identical to dividing per element.
+// Activation quantisation, persistent: each group of `wpr` warps walks
+// rows row0, row0 + stride, ... of the grid and keeps the next row's vectors
+// in flight (a second register buffer) while it reduces and quantises the
+// current one, so the loads of one row overlap the reduction and the stores
+// of the previous one.  The grid is sized from the kernel's occupancy.  The
+// row's amax is combined through shared memory (two buffers, alternating per
+// row, so one barrier per row suffices); with Xdq a second barrier orders
+// the 256-entry table of correctly rounded quotients before its lookups.
 template <int NV, bool F8>
-__global__ void __launch_bounds__(256)
-    act_quant_rows_kernel(const uint16_t* __restrict__ X, int T, int K, int wpr,
-                          int8_t* __restrict__ Xq, float* __restrict__ s_x,
-                          uint16_t* __restrict__ Xq_img, uint16_t* __restrict__ Xdq) {
-  __shared__ uint16_t table[8][256];
-  __shared__ float part[8];
-  const int warp = threadIdx.x >> 5;
-  const int lane = threadIdx.x & 31;
-  const int rib = warp / wpr;      // row within the block
-  const int wir = warp - rib * wpr;  // warp within the row
-  const int rpb = blockDim.x / (32 * wpr);
-  const int row = blockIdx.x * rpb + rib;
-  const bool live = row < T;
+__device__ __forceinline__ void aq_load_row(const uint16_t* __restrict__ X, int row, int T, int K,
+                                            int tid, int nth, uint4 (&u)[NV]) {
   const int nv = K >> 3;
-  const int tid = wir * 32 + lane;   // thread index within the row
-  const int nth = wpr * 32;
-  const uint4* xr = reinterpret_cast<const uint4*>(X + static_cast<size_t>(live ? row : 0) * K);
-  uint4 u[NV];
+  const uint4* xr = reinterpret_cast<const uint4*>(X + static_cast<size_t>(row < T ? row : 0) * K);
 #pragma unroll
   for (int i = 0; i < NV; ++i) {
     const int vi = tid + nth * i;
-    u[i] = (live && vi < nv) ? __ldcs(xr + vi) : make_uint4(0, 0, 0, 0);
-  }
-  float amax = 0.0f;
-#pragma unroll
-  for (int i = 0; i < NV; ++i) {
-    const uint32_t w[4] = {u[i].x, u[i].y, u[i].z, u[i].w};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      amax = fmaxf(amax, fabsf(bf16_bits_to_f32(w[j] & 0xFFFFu)));
-      amax = fmaxf(amax, fabsf(bf16_bits_to_f32(w[j] >> 16)));
-    }
-  }
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
-  if (lane == 0) part[warp] = amax;
-  __syncthreads();
-  amax = part[rib * wpr];
-  for (int w = 1; w < wpr; ++w) amax = fmaxf(amax, part[rib * wpr + w]);
-  const float s = __fdiv_rn(code_scale_num<F8>(), fmaxf(amax, 1e-5f));
-  if (live && tid == 0) s_x[row] = s;
-  if (Xdq) {
-    for (int j = tid; j < 256; j += nth) table[rib][j] = dq_entry<F8>(j, s);
-  }
-  __syncthreads();
-  if (!live) return;
-  const size_t rbase = static_cast<size_t>(row) * K;
-#pragma unroll
-  for (int i = 0; i < NV; ++i) {
-    const int vi = tid + nth * i;
-    if (vi >= nv) break;
-    int32_t q[8];
-    quant8<F8>(u[i], s, q);
-    const size_t e = rbase + static_cast<size_t>(vi) * 8;
-    if (Xq) {
-      uint2 pk;
-      pk.x = (q[0] & 0xFF) | ((q[1] & 0xFF) << 8) | ((q[2] & 0xFF) << 16) | ((q[3] & 0xFF) << 24);
-      pk.y = (q[4] & 0xFF) | ((q[5] & 0xFF) << 8) | ((q[6] & 0xFF) << 16) | ((q[7] & 0xFF) << 24);
-      __stcs(reinterpret_cast<uint2*>(Xq + e), pk);
-    }
-    if (Xq_img) {
-      uint32_t h[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) h[j] = f32_to_bf16_bits(static_cast<float>(q[j]));
-      __stcs(reinterpret_cast<uint4*>(Xq_img + e),
-             make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
-                        h[6] | (h[7] << 16)));
-    }
-    if (Xdq) {
-      uint32_t h[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) h[j] = table[rib][dq_index<F8>(q[j])];
-      __stcs(reinterpret_cast<uint4*>(Xdq + e),
-             make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
-                        h[6] | (h[7] << 16)));
-    }
-  }
-}
-
-// Persistent variant for rows of at most 2048 elements (8 vectors per lane):
-// each warp walks rows row0, row0 + stride, ... and loads the next row while
-// it quantises the current one (two register buffers), so every warp keeps
-// two rows in flight and the grid has no wave tail.
-template <bool F8>
-__device__ __forceinline__ void aq_row_store(const uint4 (&u)[8], int nv, int lane, float s,
-                                             size_t rbase, const uint16_t* table,
-                                             int8_t* __restrict__ Xq,
-                                             uint16_t* __restrict__ Xq_img,
-                                             uint16_t* __restrict__ Xdq) {
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int vi = lane + 32 * i;
-    if (vi >= nv) break;
-    int32_t q[8];
-    quant8<F8>(u[i], s, q);
-    const size_t e = rbase + static_cast<size_t>(vi) * 8;
-    if (Xq) {
-      uint2 pk;
-      pk.x = (q[0] & 0xFF) | ((q[1] & 0xFF) << 8) | ((q[2] & 0xFF) << 16) | ((q[3] & 0xFF) << 24);
-      pk.y = (q[4] & 0xFF) | ((q[5] & 0xFF) << 8) | ((q[6] & 0xFF) << 16) | ((q[7] & 0xFF) << 24);
-      __stcs(reinterpret_cast<uint2*>(Xq + e), pk);
-    }
-    if (Xq_img) {
-      uint32_t h[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) h[j] = f32_to_bf16_bits(static_cast<float>(q[j]));
-      __stcs(reinterpret_cast<uint4*>(Xq_img + e),
-             make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
-                        h[6] | (h[7] << 16)));
-    }
-    if (Xdq) {
-      uint32_t h[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) h[j] = table[dq_index<F8>(q[j])];
-      __stcs(reinterpret_cast<uint4*>(Xdq + e),
-             make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
-                        h[6] | (h[7] << 16)));
-    }
-  }
-}
-
-__device__ __forceinline__ void aq_row_load(const uint16_t* __restrict__ X, int row, int T, int K,
-                                            int nv, int lane, uint4 (&u)[8]) {
-  const uint4* xr = reinterpret_cast<const uint4*>(X + static_cast<size_t>(row) * K);
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int vi = lane + 32 * i;
     u[i] = (row < T && vi < nv) ? __ldcs(xr + vi) : make_uint4(0, 0, 0, 0);
   }
 }
 
-template <bool F8>
+template <int NV, bool F8>
 __global__ void __launch_bounds__(256)
-    act_quant_persist_kernel(const uint16_t* __restrict__ X, int T, int K,
-                             int8_t* __restrict__ Xq, float* __restrict__ s_x,
-                             uint16_t* __restrict__ Xq_img, uint16_t* __restrict__ Xdq) {
+    act_quant_stream_kernel(const uint16_t* __restrict__ X, int T, int K, int wpr,
+                            int8_t* __restrict__ Xq, float* __restrict__ s_x,
+                            uint16_t* __restrict__ Xq_img, uint16_t* __restrict__ Xdq) {
   __shared__ uint16_t table[8][256];
-  const int wid = threadIdx.x >> 5;
+  __shared__ float part[2][8];
+  const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int stride = gridDim.x * 8;
+  const int rib = warp / wpr;        // row within the block
+  const int wir = warp - rib * wpr;  // warp within the row
+  const int rpb = blockDim.x / (32 * wpr);
   const int nv = K >> 3;
-  uint4 ua[8], ub[8];
-  int row = blockIdx.x * 8 + wid;
-  aq_row_load(X, row, T, K, nv, lane, ua);
-  for (; row < T; row += stride) {
-    aq_row_load(X, row + stride, T, K, nv, lane, ub);  // next row in flight
+  const int tid = wir * 32 + lane;
+  const int nth = wpr * 32;
+  const int stride = gridDim.x * rpb;
+  uint4 ua[NV], ub[NV];
+  int row = blockIdx.x * rpb + rib;
+  aq_load_row<NV, F8>(X, row, T, K, tid, nth, ua);
+  int par = 0;
+  for (int base = blockIdx.x * rpb; base < T; base += stride, row += stride, par ^= 1) {
+    aq_load_row<NV, F8>(X, row + stride, T, K, tid, nth, ub);  // next row in flight
     float amax = 0.0f;
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
+    for (int i = 0; i < NV; ++i) {
       const uint32_t w[4] = {ua[i].x, ua[i].y, ua[i].z, ua[i].w};
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
@@ -295,17 +183,52 @@ __global__ void __launch_bounds__(256)
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+    if (lane == 0) part[par][warp] = amax;
+    __syncthreads();
+    amax = part[par][rib * wpr];
+    for (int w = 1; w < wpr; ++w) amax = fmaxf(amax, part[par][rib * wpr + w]);
     const float s = __fdiv_rn(code_scale_num<F8>(), fmaxf(amax, 1e-5f));
-    if (lane == 0) s_x[row] = s;
+    const bool live = row < T;
+    if (live && tid == 0) s_x[row] = s;
     if (Xdq) {
-      __syncwarp();  // the previous row's lookups are done
-#pragma unroll
-      for (int j = lane; j < 256; j += 32) table[wid][j] = dq_entry<F8>(j, s);
-      __syncwarp();
+      for (int j = tid; j < 256; j += nth) table[rib][j] = dq_entry<F8>(j, s);
+      __syncthreads();
     }
-    aq_row_store<F8>(ua, nv, lane, s, static_cast<size_t>(row) * K, table[wid], Xq, Xq_img, Xdq);
+    if (live) {
+      const size_t rbase = static_cast<size_t>(row) * K;
 #pragma unroll
-    for (int i = 0; i < 8; ++i) ua[i] = ub[i];
+      for (int i = 0; i < NV; ++i) {
+        const int vi = tid + nth * i;
+        if (vi >= nv) break;
+        int32_t q[8];
+        quant8<F8>(ua[i], s, q);
+        const size_t e = rbase + static_cast<size_t>(vi) * 8;
+        if (Xq) {
+          uint2 pk;
+          pk.x = (q[0] & 0xFF) | ((q[1] & 0xFF) << 8) | ((q[2] & 0xFF) << 16) | ((q[3] & 0xFF) << 24);
+          pk.y = (q[4] & 0xFF) | ((q[5] & 0xFF) << 8) | ((q[6] & 0xFF) << 16) | ((q[7] & 0xFF) << 24);
+          __stcs(reinterpret_cast<uint2*>(Xq + e), pk);
+        }
+        if (Xq_img) {
+          uint32_t h[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) h[j] = f32_to_bf16_bits(static_cast<float>(q[j]));
+          __stcs(reinterpret_cast<uint4*>(Xq_img + e),
+                 make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
+                            h[6] | (h[7] << 16)));
+        }
+        if (Xdq) {
+          uint32_t h[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) h[j] = table[rib][dq_index<F8>(q[j])];
+          __stcs(reinterpret_cast<uint4*>(Xdq + e),
+                 make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
+                            h[6] | (h[7] << 16)));
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < NV; ++i) ua[i] = ub[i];
   }
 }
 
@@ -490,30 +413,35 @@ int launch_aq(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x, u
               uint16_t* Xdq, cudaStream_t stream) {
   const int t = static_cast<int>(T), k = static_cast<int>(K);
   const int64_t nv = K / 8;  // 16-byte vectors per row
-  // warps per row: keep at most 4 vectors (32 values) per lane; up to 8 warps
-  const int wpr = static_cast<int>((nv + 127) / 128);
-  if (nv <= 256) {
-    int dev = 0, sms = 148;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int64_t want = (T + 7) / 8;
-    const int blocks = static_cast<int>(want < 2 * sms ? want : 2 * sms);
-    act_quant_persist_kernel<F8><<<blocks, 256, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq);
-  } else if (wpr <= 8) {
-    const int rpb = 8 / wpr;
-    const int threads = 32 * wpr * rpb;
-    const int blocks = static_cast<int>((T + rpb - 1) / rpb);
-    const int per_lane = static_cast<int>((nv + 32 * wpr - 1) / (32 * wpr));
-    if (per_lane <= 2)
-      act_quant_rows_kernel<2, F8><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
-    else if (per_lane <= 4)
-      act_quant_rows_kernel<4, F8><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
-    else
-      act_quant_rows_kernel<8, F8><<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
-  } else {
-    const int blocks = static_cast<int>((T + kAqWarps - 1) / kAqWarps);
-    act_quant_kernel<F8><<<blocks, kAqWarps * 32, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq);
+  // persistent rows: warps per row so that each lane holds at most 4 vectors
+  // (8 above 4096 vectors), rows per 256-thread block 8 / wpr
+  {
+    const int wpr4 = static_cast<int>((nv + 127) / 128);
+    const int wpr8 = static_cast<int>((nv + 255) / 256);
+    if (wpr4 <= 8 || wpr8 <= 8) {
+      const bool four = wpr4 <= 8;
+      const int wpr = four ? wpr4 : wpr8;
+      const int rpb = 8 / wpr;
+      const int threads = 32 * wpr * rpb;
+      auto kern = four ? act_quant_stream_kernel<4, F8> : act_quant_stream_kernel<8, F8>;
+      static int occ[2][9] = {};  // resident blocks per SM, per NV and wpr
+      int& o = occ[four ? 0 : 1][wpr];
+      int dev = 0, sms = 148;
+      cudaGetDevice(&dev);
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+      if (o == 0 && (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, kern, threads, 0) !=
+                         cudaSuccess || o < 1))
+        o = 1;
+      const int64_t want = (T + rpb - 1) / rpb;
+      const int64_t cap = static_cast<int64_t>(sms) * o;
+      const int blocks = static_cast<int>(want < cap ? want : cap);
+      kern<<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
+      return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+    }
   }
+  // longer rows (more than 16384 elements): one warp per row, two passes
+  const int blocks = static_cast<int>((T + kAqWarps - 1) / kAqWarps);
+  act_quant_kernel<F8><<<blocks, kAqWarps * 32, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
