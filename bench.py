@@ -107,8 +107,9 @@ class ClockSampler:
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, index):
+    def __init__(self, index, window="the timed region"):
         self.index = index
+        self.window = window
         self.proc = None
 
     def __enter__(self):
@@ -138,14 +139,15 @@ class ClockSampler:
             if len(f) >= 9:
                 rows.append(f)
         if not rows:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"],
+                    "window": self.window}
         sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
         mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i] == "Active"})
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
-                "samples": len(rows)}
+                "samples": len(rows), "window": self.window}
 
 
 class MLPStep:
@@ -611,6 +613,9 @@ def run_gpu(args):
             dist.barrier()
         torch.cuda.synchronize()
 
+    # the clock sampler (one nvidia-smi sample per 20 ms) covers the warm-up
+    # and the timed steps: the timed region alone lasts only ~20-30 ms
+    clk = ClockSampler(dev.index, "the warm-up and the timed steps").__enter__()
     for _ in range(args.warmup):
         st.run()
     dqt.dqt_check_device_status()
@@ -619,12 +624,12 @@ def run_gpu(args):
     barrier()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
-    with ClockSampler(dev.index) as clk:
-        t0.record(stream)
-        for _ in range(args.steps):
-            st.run()
-        t1.record(stream)
-        barrier()
+    t0.record(stream)
+    for _ in range(args.steps):
+        st.run()
+    t1.record(stream)
+    barrier()
+    clk.__exit__(None, None, None)
     dqt.dqt_check_device_status()
     ms = max_over_ranks(t0.elapsed_time(t1), dev)
     ms_step = ms / args.steps
@@ -1114,16 +1119,22 @@ def run_kernel(args):
         elif k == "bwd_dw":  # gradient only (fp32 dW written, no update)
             dW = torch.empty((N, K), dtype=torch.float32, device=dev)
             fn = lambda: dqt.dqt_bitlinear_bwd_dw_update_img(dY, xdq, None, s_w, None, None, None,  # noqa: E731
-                                                         None, g, dW_out=dW)
+                                                             None, g, dW_out=dW)
         elif k == "bwd_dw_unfused":  # gradient to memory, then the standalone update
             dW = torch.empty((N, K), dtype=torch.float32, device=dev)
 
             def fn():
                 dqt.dqt_bitlinear_bwd_dw_update_img(dY, xdq, None, s_w, None, None, None, None, g,
-                                                dW_out=dW)
+                                                    dW_out=dW)
                 dqt.dqt_sr_update(dW.view(-1), W.view(-1), s_w, m.view(-1), v.view(-1), hp, sr, g)
         elif k == "act_quant":
             fn = lambda: dqt.dqt_act_quant_images(X, None, s_x, q_img, xdq, want=())  # noqa: E731
+        elif k == "act_quant_codes":  # the int8 call: codes and scales only
+            Xq = torch.empty((T, K), dtype=torch.int8, device=dev)
+            fn = lambda: dqt.dqt_act_quant(X, Xq, s_x)  # noqa: E731
+        elif k == "codes_to_xdq":
+            Xq, _ = dqt.dqt_act_quant(X)
+            fn = lambda: dqt.dqt_codes_to_xdq(Xq, s_x, xdq)  # noqa: E731
         elif k == "bwd_dw_update_packed":
             Wp = dqt.dqt_pack_ternary(W)
             fn = lambda: dqt.dqt_bitlinear_bwd_dw_update_packed(dY, xdq, Wp, s_w, m, v, hp, sr)  # noqa: E731
@@ -1167,6 +1178,8 @@ def run_kernel(args):
             work, unit = 6.0 * N * K, "GB/s"
         elif k == "act_quant":
             work, unit = 6.0 * T * K + 4 * T, "GB/s"
+        elif k in ("act_quant_codes", "codes_to_xdq"):
+            work, unit = 3.0 * T * K + 4 * T, "GB/s"
         elif k == "act_quant_fp8":
             work, unit = 5.0 * T * K + 4 * T, "GB/s"
         elif k == "codes_to_fp8":
@@ -1489,8 +1502,9 @@ def main():
                     help="mlp: skip the single-layer step and the SR-update sweep keys")
     ap.add_argument("--kernel", default=None,
                     help="time one kernel kind alone (fwd, bwd_dx, bwd_dw_update, bwd_dw, "
-                         "bwd_dw_unfused, act_quant, codes_to_bf16, sr_update, act_quant_fp8, "
-                         "codes_to_fp8, fwd_fp8)")
+                         "bwd_dw_unfused, act_quant (with both images), act_quant_codes, "
+                         "codes_to_xdq, codes_to_bf16, sr_update, act_quant_fp8, codes_to_fp8, "
+                         "fwd_fp8)")
     ap.add_argument("--numel", type=int, default=1 << 26, help="weights for --kernel sr_update")
     ap.add_argument("--shape", default=None, help="T,K,N for --kernel GEMMs (default 8192,2048,5632)")
     ap.add_argument("--no-graph", action="store_true", help="decoder: run the step eagerly")

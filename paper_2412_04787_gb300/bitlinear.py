@@ -261,7 +261,7 @@ class DQTBitLinear(torch.nn.Module):
         self.step += 1
         hp, sr = self._hyper(self.step)
         dqt.dqt_bitlinear_bwd_dw_update_img(dy2, xdq, self.codes, self.s_w, self.m, self.v, hp, sr,
-                                        self.grid_tuple, changed_out=self.changed)
+                                            self.grid_tuple, changed_out=self.changed)
 
     def extra_repr(self):
         return "in_features=%d, out_features=%d, grid=%s, act=%s, optimizer=%s, packed=%s" % (

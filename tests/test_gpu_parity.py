@@ -185,7 +185,7 @@ def test_fwd_adversarial_magnitudes():
     s_x = torch.full((T,), 1.0, dtype=torch.float32)
     acc = torch.empty((T, N), dtype=torch.int32, device="cuda")
     Y = dqt.dqt_bitlinear_fwd_img(q.to(torch.bfloat16).cuda(), s_x.cuda(), c.to(torch.bfloat16).cuda(),
-                              1.0, (-128, 127), acc_out=acc)
+                                  1.0, (-128, 127), acc_out=acc)
     dqt.dqt_check_device_status()
     ref = q.to(torch.int64) @ c.to(torch.int64).T
     assert ref.abs().max() > 2**24
@@ -377,7 +377,7 @@ def _fused(T, K, N, bits_w, step, seed, rows=None):
     dW = torch.empty((N, K), dtype=torch.float32, device="cuda")
     changed = torch.zeros(1, dtype=torch.int64, device="cuda")
     dqt.dqt_bitlinear_bwd_dw_update_img(dY.cuda(), Xdq, Wg, s_w, mg, vg, hp, sr, g, dW_out=dW,
-                                    changed_out=changed)
+                                        changed_out=changed)
     dqt.dqt_check_device_status()
     q, s, _, xd = oracle.act_quant(bits(X))
     if rows is None:
@@ -506,7 +506,7 @@ def test_tilings_bit_identical():
             dW = torch.empty((776, 512), dtype=torch.float32, device="cuda")
             # unsplit on both tilings (the split-T path sums in another order)
             dqt.dqt_bitlinear_bwd_dw_update_img(dY.cuda(), xdq, None, s_w, None, None, None, None, g,
-                                            dW_out=dW, ws=False)
+                                                dW_out=dW, ws=False)
             dqt.dqt_check_device_status()
             outs.append((Y.cpu(), dX.cpu(), dW.cpu()))
         finally:
@@ -563,7 +563,7 @@ def test_split_t_matches_unsplit_within_tolerance():
     b = torch.empty((N, K), dtype=torch.float32, device="cuda")
     dqt.dqt_bitlinear_bwd_dw_update_img(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=a)
     dqt.dqt_bitlinear_bwd_dw_update_img(dY.cuda(), Xdq, None, s_w, None, None, None, None, g, dW_out=b,
-                                    ws=False)
+                                        ws=False)
     dqt.dqt_check_device_status()
     # fp32 summation order only (a wrong token slice would be an O(1) error)
     assert elem_err(a.cpu().numpy(), b.cpu().double().numpy()) <= 2e-3

@@ -41,8 +41,8 @@ def _step(g, s_w, X, dY, state, step):
     dqt.dqt_bitlinear_fwd_img(q_img, s_x, W_img, s_w, g)
     dqt.dqt_bitlinear_bwd_dx_img(dY, W_img, s_w)
     dqt.dqt_bitlinear_bwd_dw_update_img(dY, xdq, state["W"], s_w, state["m"], state["v"],
-                                    dqt.adamw(lr=1e-3, step=step),
-                                    dqt.sr_stream(seed=77, tensor_id=5), g)
+                                        dqt.adamw(lr=1e-3, step=step),
+                                        dqt.sr_stream(seed=77, tensor_id=5), g)
     dqt.dqt_check_device_status()
 
 

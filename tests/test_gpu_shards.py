@@ -114,7 +114,7 @@ def test_fused_update_with_offset_equals_standalone():
     v1 = torch.zeros((N, K), device="cuda")
     dW = torch.empty((N, K), device="cuda")
     dqt.dqt_bitlinear_bwd_dw_update_img(dY.cuda(), Xdq, W1, s_w, m1, v1, hp, sr, (qmin, qmax),
-                                    dW_out=dW, ws=False)
+                                        dW_out=dW, ws=False)
     W2 = torch.from_numpy(c).cuda()
     m2 = torch.zeros((N, K), device="cuda")
     v2 = torch.zeros((N, K), device="cuda")
