@@ -14,6 +14,7 @@
  *                                 step (Sec. 4.1) and W_hat = SR(W') (Eq. 1, Eq. 5),
  *                                 clamped to the n-bit grid and written over the codes
  *   dqt_sr_update                 the same AdamW + SR step for a gradient given in memory
+ *                                 (dqt_sr_t.elem0: a data-parallel shard's global offset)
  *   dqt_*_fp8                     the forward with E4M3 operands (FP8 environment, Sec. 4.3)
  *   dqt_*packed*                  2-bit packed ternary code storage (Sec. 1)
  *   dqt_*adafactor*               Adafactor with SR instead of AdamW (Sec. 4.3)
@@ -24,9 +25,9 @@
  * dqt_cross_entropy_fwd_bf16 / _bwd_bf16.
  *
  * GB300 has no int8 tensor-core MMA for sm_103a, so the integer GEMMs run on
- * the 16-bit tensor cores over exact 16-bit images of the integer codes
- * (every integer in [-256, 256] is exact in bf16 and fp16; products and
- * partial sums below 2^24 are exact in the fp32 accumulator).  The hot-path
+ * the bf16 tensor cores over exact bf16 images of the integer codes (every
+ * integer in [-256, 256] is exact in bf16; products and partial sums below
+ * 2^24 are exact in the fp32 accumulator).  The hot-path
  * calls take the int8 codes themselves and make the bf16 operands they need
  * in a caller-provided workspace (dqt_codes_to_bf16, dqt_codes_to_xdq) before
  * the GEMM.  The *_img calls take those images directly
