@@ -613,9 +613,11 @@ def run_gpu(args):
             dist.barrier()
         torch.cuda.synchronize()
 
-    # the clock sampler (one nvidia-smi sample per 20 ms) covers the warm-up
-    # and the timed steps: the timed region alone lasts only ~20-30 ms
-    clk = ClockSampler(dev.index, "the warm-up and the timed steps").__enter__()
+    # the clock sampler (one nvidia-smi sample per 20 ms) covers the warm-up,
+    # the timed steps, the per-kernel region and the e2e steps: the timed
+    # region alone lasts only ~20-30 ms
+    clk = ClockSampler(dev.index, "the warm-up, the timed steps, the per-kernel region and "
+                                  "the e2e steps").__enter__()
     for _ in range(args.warmup):
         st.run()
     dqt.dqt_check_device_status()
@@ -629,7 +631,6 @@ def run_gpu(args):
         st.run()
     t1.record(stream)
     barrier()
-    clk.__exit__(None, None, None)
     dqt.dqt_check_device_status()
     ms = max_over_ranks(t0.elapsed_time(t1), dev)
     ms_step = ms / args.steps
@@ -774,6 +775,7 @@ def run_gpu(args):
     barrier()
     st.d = bufs[0]
     st.alternate = True
+    clk.__exit__(None, None, None)
     e_ms = max_over_ranks(e0.elapsed_time(e1), dev)
     dqt.dqt_check_device_status()
     e2e = {"value": round(aggregate_tokens_per_s(ws, T_TOK, e_steps, e_ms), 1), "unit": "tokens/s",
