@@ -329,6 +329,110 @@ __device__ __forceinline__ uint32_t dw_update(const Params& p, const UpdateConst
   return n_changed;
 }
 
+// Optimiser state of one lane for one row of a half-chunk (4 weights): the
+// moments and the codes as loaded (four int8 codes, or one byte of 2-bit
+// packed codes, unpacked where they are used).
+struct DwRow {
+  float4 m, v;
+  uint32_t c;
+};
+
+template <bool PK>
+__device__ __forceinline__ void dw_load_row(const Params& p, int gm, int gk, DwRow& L) {
+  if (!p.W || gk >= p.N || gm >= p.M) return;
+  const size_t e = static_cast<size_t>(gm) * p.N + gk;
+  L.c = PK ? static_cast<uint32_t>(__ldcs(reinterpret_cast<const uint8_t*>(p.W) + (e >> 2)))
+           : __ldcs(reinterpret_cast<const unsigned int*>(p.W + e));
+  L.m = __ldcs(reinterpret_cast<const float4*>(p.m + e));
+  L.v = __ldcs(reinterpret_cast<const float4*>(p.v + e));
+}
+
+template <bool PK>
+__device__ __forceinline__ uint32_t dw_update_row(const Params& p, const UpdateConsts& uc,
+                                                  float* dw_out, int gm, int gk, const float* src,
+                                                  DwRow& L) {
+  if (gk >= p.N || gm >= p.M) return 0;
+  const size_t e = static_cast<size_t>(gm) * p.N + gk;
+  const float4 g4 = make_float4(src[0], src[1], src[2], src[3]);
+  if (dw_out) __stcs(reinterpret_cast<float4*>(dw_out + e), g4);
+  if (!p.W) return 0;
+  const char4 c = PK ? tern_unpack4(L.c)
+                     : make_char4(static_cast<signed char>(L.c & 0xFFu),
+                                  static_cast<signed char>((L.c >> 8) & 0xFFu),
+                                  static_cast<signed char>((L.c >> 16) & 0xFFu),
+                                  static_cast<signed char>(L.c >> 24));
+  uint4 w = make_uint4(0, 0, 0, 0);
+  if (uc.round_mode == 0)
+    w = sr_words(global_blk(uc, e >> 2), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
+  const int32_t n0c = dqt_update_elem(uc, g4.x, c.x, L.m.x, L.v.x, w.x);
+  const int32_t n1c = dqt_update_elem(uc, g4.y, c.y, L.m.y, L.v.y, w.y);
+  const int32_t n2c = dqt_update_elem(uc, g4.z, c.z, L.m.z, L.v.z, w.z);
+  const int32_t n3c = dqt_update_elem(uc, g4.w, c.w, L.m.w, L.v.w, w.w);
+  if (PK)
+    __stcs(reinterpret_cast<uint8_t*>(p.W) + (e >> 2),
+           static_cast<uint8_t>(tern_pack4(n0c, n1c, n2c, n3c)));
+  else
+    __stcs(reinterpret_cast<char4*>(p.W + e),
+           make_char4(static_cast<signed char>(n0c), static_cast<signed char>(n1c),
+                      static_cast<signed char>(n2c), static_cast<signed char>(n3c)));
+  __stcs(reinterpret_cast<float4*>(p.m + e), L.m);
+  __stcs(reinterpret_cast<float4*>(p.v + e), L.v);
+  return (n0c != c.x) + (n1c != c.y) + (n2c != c.z) + (n3c != c.w);
+}
+
+// The first half-chunk's state loads of a tile (rows row0 + (lane >> 3) +
+// 4 j, columns nbase + 4 (lane & 7) .. + 3).
+template <bool PK>
+__device__ __forceinline__ void dw_load_first(const Params& p, int row0, int nbase, int lane,
+                                              DwRow (&L)[4]) {
+#pragma unroll
+  for (int j = 0; j < 4; ++j) dw_load_row<PK>(p, row0 + (lane >> 3) + 4 * j, nbase + (lane & 7) * 4, L[j]);
+}
+
+// The dW epilogue of one warp for one tile, with the optimiser state loads
+// rotated through the registers that hold them: as soon as row j of a
+// half-chunk is updated, the loads of row j of the next half-chunk (this
+// tile's, or the first of the tile at row0n, nbasen when row0n >= 0) go into
+// the same registers, so each load has most of a half-chunk's update to
+// arrive in.  On entry L holds the tile's first half-chunk.  Half-chunk q
+// covers chunk q / 2 (32 columns at nbase + 32 (q / 2)), rows
+// (lane >> 3) + 4 (4 (q % 2) + j), j = 0..3, and columns 4 (lane & 7) .. + 3.
+template <bool PK>
+__device__ __forceinline__ uint32_t epi_dw_tile_roll(const Params& p, const UpdateConsts& uc,
+                                                     float* dw_out, int row0, int nbase,
+                                                     int nchunk, uint32_t t_acc, float* xp,
+                                                     int lane, DwRow (&L)[4], int row0n,
+                                                     int nbasen) {
+  const int cq = (lane & 7) * 4;
+  const int nq = 2 * nchunk;
+  uint32_t n_changed = 0;
+#pragma unroll 1
+  for (int q = 0; q < nq; ++q) {
+    const int h = q & 1;
+    const int gn0 = nbase + (q >> 1) * 32;
+    if (h == 0) {
+      uint32_t a[32];
+      tmem_ld_32x32b_x32(t_acc + (q >> 1) * 32, a);
+      tmem_ld_wait();
+#pragma unroll
+      for (int i = 0; i < 32; ++i) xp[lane * kStageLd + i] = __uint_as_float(a[i]);
+      __syncwarp();
+    }
+    const bool in_tile = q + 1 < nq;
+    const int nrow0 = in_tile ? row0 : row0n;
+    const int ngk = (in_tile ? nbase + ((q + 1) >> 1) * 32 : nbasen) + cq;
+    const int nh = in_tile ? (q + 1) & 1 : 0;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int r = (lane >> 3) + 4 * (4 * h + j);
+      n_changed += dw_update_row<PK>(p, uc, dw_out, row0 + r, gn0 + cq, xp + r * kStageLd + cq, L[j]);
+      if (nrow0 >= 0) dw_load_row<PK>(p, nrow0 + (lane >> 3) + 4 * (4 * nh + j), ngk, L[j]);
+    }
+    if (h == 1) __syncwarp();  // the transpose buffer is rewritten for the next chunk
+  }
+  return n_changed;
+}
+
 // The whole dW epilogue of one warp for one tile: `nchunk` chunks of 32
 // columns starting at column nbase, rows row0 .. row0 + 31, gradient in
 // tensor memory at t_acc (this warp's lanes, chunk cc at column 32 cc).
@@ -844,6 +948,8 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
     uint32_t n_changed = 0;
     int u = 0;
     bool ok = true;
+    DwRow st[4];            // dW: optimiser state of the half-chunk being updated
+    bool st_loaded = false;  // st already holds this unit's first half-chunk
     for (int t = cid; t < p.num_tiles && ok; t += ncl, ++u) {
       const Unit un = decode_unit(p, t);
       const int tile = un.tile;
@@ -851,6 +957,8 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
       const int gm = (tile / p.num_n) * 256 + static_cast<int>(rank) * 128 + row;
       const int nbase = (tile % p.num_n) * BN + half * HALF;
       const bool row_ok = gm < p.M;
+      if (EPI == GEMM_DW && un.slice < 0 && !st_loaded)
+        dw_load_first<PK>(p, gm - lane, nbase, lane, st);  // in flight during the wait below
       float a_t = 0.0f;
       if ((EPI == GEMM_FWD || F8) && row_ok) a_t = __fdiv_rn(1.0f, __fmul_rn(p.s_x[gm], p.scale));
       if (DR) {
@@ -911,7 +1019,19 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
                                         __uint_as_float(a[4 * j + 3])));
         }
       } else if (EPI == GEMM_DW) {
-        n_changed += epi_dw_tile<false, PK>(p, uc, dw_out, gm - lane, nbase, HALF / 32, t_acc, xp, lane);
+        // the first half-chunk of this warp's next unit, if a whole tile,
+        // is loaded during this tile's last half-chunk
+        int row0n = -1, nbasen = 0;
+        if (t + ncl < p.num_tiles) {
+          const Unit nu = decode_unit(p, t + ncl);
+          if (nu.slice < 0) {
+            row0n = (nu.tile / p.num_n) * 256 + static_cast<int>(rank) * 128 + quad * 32;
+            nbasen = (nu.tile % p.num_n) * BN + half * HALF;
+          }
+        }
+        n_changed += epi_dw_tile_roll<PK>(p, uc, dw_out, gm - lane, nbase, HALF / 32, t_acc, xp,
+                                          lane, st, row0n, nbasen);
+        st_loaded = row0n >= 0;
       } else
 #pragma unroll 1
       for (int cc = 0; cc < HALF / 32; ++cc) {

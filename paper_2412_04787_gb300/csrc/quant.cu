@@ -129,106 +129,286 @@ __global__ void __launch_bounds__(kAqWarps * 32)
   }
 }
 
-// Activation quantisation, persistent: each group of `wpr` warps walks
-// rows row0, row0 + stride, ... of the grid and keeps the next row's vectors
-// in flight (a second register buffer) while it reduces and quantises the
-// current one, so the loads of one row overlap the reduction and the stores
-// of the previous one.  The grid is sized from the kernel's occupancy.  The
-// row's amax is combined through shared memory (two buffers, alternating per
-// row, so one barrier per row suffices); with Xdq a second barrier orders
-// the 256-entry table of correctly rounded quotients before its lookups.
-template <int NV, bool F8>
-__device__ __forceinline__ void aq_load_row(const uint16_t* __restrict__ X, int row, int T, int K,
-                                            int tid, int nth, uint4 (&u)[NV]) {
-  const int nv = K >> 3;
-  const uint4* xr = reinterpret_cast<const uint4*>(X + static_cast<size_t>(row < T ? row : 0) * K);
-#pragma unroll
-  for (int i = 0; i < NV; ++i) {
-    const int vi = tid + nth * i;
-    u[i] = (row < T && vi < nv) ? __ldcs(xr + vi) : make_uint4(0, 0, 0, 0);
-  }
+// Activation quantisation with whole rows staged in shared memory: one CTA
+// per SM, a producer lane that streams the CTA's rows (blockIdx.x,
+// blockIdx.x + gridDim.x, ...) with linear bulk copies into a ring of S row
+// slots, and W consumer warps, warp w owning slots w, w + W, ... (S a
+// multiple of W, at least two slots per warp).  The j-th row of the CTA goes
+// to slot j % S and is processed by one warp: pass 1 reduces amax over the
+// row in shared memory, pass 2 re-reads it and writes the outputs.  Every
+// slot carries a `full` barrier (the copy's bytes) and an `empty` barrier
+// (one arrive by its consumer warp); the ring keeps up to S rows in flight
+// per SM, which a register-held design cannot.
+//
+// amax is reduced on pairs of bf16 magnitudes (max.bf16x2 returns the
+// non-NaN operand, as fmaxf does, and is exact).  Round(y) for the int8
+// codes is taken with the fp32 add y + 1.5 * 2^23, which rounds to the
+// nearest integer, half to even, for |y| < 2^22; the code is then the low
+// byte of the sum's bit pattern.  Here y = RN(x s) with |x| <= a and
+// s = RN(127 / a), a = max(amax, 1e-5), so |y| <= RN(127 (1 + 2^-24)) <=
+// 127 + 2^-17 and the sum never exceeds 1.5 * 2^23 + 127: only the lower
+// clamp is needed, and it maps a NaN product (an infinite input) to -128, as
+// act_quant_kernel does.
+constexpr int kAqbRing = 192 * 1024;  // shared-memory bytes of the row ring
+
+// Linear bulk copy (no tensor map) of `bytes` from global memory into this
+// CTA's shared memory, completing on `bar`, whose expected byte count the
+// caller has raised by `bytes`.  Both addresses 16-byte aligned; `bytes` a
+// multiple of 16.
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes,
+                                          uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
 }
 
-template <int NV, bool F8>
-__global__ void __launch_bounds__(256)
-    act_quant_stream_kernel(const uint16_t* __restrict__ X, int T, int K, int wpr,
-                            int8_t* __restrict__ Xq, float* __restrict__ s_x,
-                            uint16_t* __restrict__ Xq_img, uint16_t* __restrict__ Xdq) {
-  __shared__ uint16_t table[8][256];
-  __shared__ float part[2][8];
+// The ring of row chunks in dynamic shared memory: S slots of rpc rows of
+// row_bytes, then S `full` and S `empty` mbarriers.  CTA b owns the rows
+// [b T / G, (b + 1) T / G) (G = gridDim.x <= T, so at least one), cut into
+// chunks of rpc rows (the last one shorter); chunk j is one linear bulk copy
+// into slot j % S and is processed by consumer warp j % W (S a multiple of W).
+struct RowRing {
+  uint8_t* base;
+  uint64_t* full;
+  uint64_t* empty;
+  uint32_t row_bytes;
+  int S, rpc;
+  int64_t lo, hi;  // this CTA's rows
+  int nchunks;
+
+  __device__ __forceinline__ RowRing(uint8_t* smem, int slots, uint32_t rb, int rows_per_chunk,
+                                     int64_t T)
+      : base(smem),
+        full(reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(slots) * rows_per_chunk * rb)),
+        empty(full + slots),
+        row_bytes(rb),
+        S(slots),
+        rpc(rows_per_chunk),
+        lo(static_cast<int64_t>(blockIdx.x) * T / gridDim.x),
+        hi(static_cast<int64_t>(blockIdx.x + 1) * T / gridDim.x) {
+    nchunks = static_cast<int>((hi - lo + rpc - 1) / rpc);
+  }
+  // shared memory after the ring and its barriers
+  __device__ __forceinline__ uint8_t* end() const { return reinterpret_cast<uint8_t*>(empty + S); }
+
+  // every thread, followed by __syncthreads()
+  __device__ __forceinline__ void init_barriers() const {
+    if (static_cast<int>(threadIdx.x) < S) {
+      mbar_init(&full[threadIdx.x], 1);
+      mbar_init(&empty[threadIdx.x], 1);
+      fence_mbarrier_init();
+    }
+  }
+
+  __device__ __forceinline__ int64_t row0(int j) const { return lo + static_cast<int64_t>(j) * rpc; }
+  __device__ __forceinline__ int rows(int j) const {
+    const int64_t r = hi - row0(j);
+    return r < rpc ? static_cast<int>(r) : rpc;
+  }
+
+  // One thread: the chunks of this CTA from `src` (rows of row_bytes bytes),
+  // each slot refilled once its consumer has released it; returns when every
+  // copy it issued has landed (the CTA must not retire before).
+  __device__ void produce(const uint8_t* src, unsigned int* status, uint64_t limit_ns) const {
+    int issued = 0;
+    for (; issued < nchunks; ++issued) {
+      const int slot = issued % S, use = issued / S;
+      if (use > 0 && !mbar_wait(&empty[slot], (use - 1) & 1, limit_ns)) {
+        record_timeout(status);
+        break;
+      }
+      const uint32_t bytes = static_cast<uint32_t>(rows(issued)) * row_bytes;
+      mbar_arrive_expect_tx(&full[slot], bytes);
+      bulk_load(base + static_cast<size_t>(slot) * rpc * row_bytes,
+                src + static_cast<size_t>(row0(issued)) * row_bytes, bytes, &full[slot]);
+    }
+    for (int j = issued > S ? issued - S : 0; j < issued; ++j)
+      if (!mbar_wait(&full[j % S], (j / S) & 1, limit_ns)) {
+        record_timeout(status);
+        break;
+      }
+  }
+
+  // All lanes of the consumer warp: waits for chunk j; false (warp-uniform,
+  // timeout recorded) if it did not arrive in time.
+  __device__ __forceinline__ bool acquire(int j, int lane, unsigned int* status,
+                                          uint64_t limit_ns) const {
+    const bool ok = __all_sync(0xffffffffu, mbar_wait(&full[j % S], (j / S) & 1, limit_ns));
+    if (!ok && lane == 0) record_timeout(status);
+    return ok;
+  }
+  // row r of chunk j
+  __device__ __forceinline__ const uint8_t* row(int j, int r) const {
+    return base + (static_cast<size_t>(j % S) * rpc + r) * row_bytes;
+  }
+  // All lanes, after their last read of the slot.
+  __device__ __forceinline__ void release(int j, int lane) const {
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&empty[j % S]);
+  }
+};
+
+template <bool F8>
+__global__ void __launch_bounds__(32 * 17, 1)
+    act_quant_bulk_kernel(const uint16_t* __restrict__ X, int T, int K,
+                          int8_t* __restrict__ Xq, float* __restrict__ s_x,
+                          uint16_t* __restrict__ Xq_img, uint16_t* __restrict__ Xdq, int S, int W,
+                          int rpc, unsigned int* status, uint64_t limit_ns) {
+  extern __shared__ __align__(128) uint8_t aqb_smem[];
+  const RowRing ring(aqb_smem, S, static_cast<uint32_t>(K) * 2u, rpc, T);
+  uint16_t* tables = reinterpret_cast<uint16_t*>(ring.end());
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int rib = warp / wpr;        // row within the block
-  const int wir = warp - rib * wpr;  // warp within the row
-  const int rpb = blockDim.x / (32 * wpr);
-  const int nv = K >> 3;
-  const int tid = wir * 32 + lane;
-  const int nth = wpr * 32;
-  const int stride = gridDim.x * rpb;
-  uint4 ua[NV], ub[NV];
-  int row = blockIdx.x * rpb + rib;
-  aq_load_row<NV, F8>(X, row, T, K, tid, nth, ua);
-  int par = 0;
-  for (int base = blockIdx.x * rpb; base < T; base += stride, row += stride, par ^= 1) {
-    aq_load_row<NV, F8>(X, row + stride, T, K, tid, nth, ub);  // next row in flight
-    float amax = 0.0f;
+  ring.init_barriers();
+  __syncthreads();
+  if (warp == 0) {
+    if (lane == 0) ring.produce(reinterpret_cast<const uint8_t*>(X), status, limit_ns);
+    return;
+  }
+
+  const int cw = warp - 1;
+  uint16_t* table = tables + cw * 256;
+  const int nv = K >> 3;  // 16-byte vectors per row
+  constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23
+  for (int j = cw; j < ring.nchunks; j += W) {
+    if (!ring.acquire(j, lane, status, limit_ns)) return;
+    const int nr = ring.rows(j);
+#pragma unroll 1
+    for (int r = 0; r < nr; ++r) {
+      const int64_t row = ring.row0(j) + r;
+      const uint4* xr = reinterpret_cast<const uint4*>(ring.row(j, r));
+      __nv_bfloat162 am2 = __floats2bfloat162_rn(0.0f, 0.0f);
+#pragma unroll 4
+      for (int v = lane; v < nv; v += 32) {
+        const uint4 u = xr[v];
+        const uint32_t w[4] = {u.x & 0x7FFF7FFFu, u.y & 0x7FFF7FFFu, u.z & 0x7FFF7FFFu,
+                               u.w & 0x7FFF7FFFu};
 #pragma unroll
-    for (int i = 0; i < NV; ++i) {
-      const uint32_t w[4] = {ua[i].x, ua[i].y, ua[i].z, ua[i].w};
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        amax = fmaxf(amax, fabsf(bf16_bits_to_f32(w[j] & 0xFFFFu)));
-        amax = fmaxf(amax, fabsf(bf16_bits_to_f32(w[j] >> 16)));
+        for (int i = 0; i < 4; ++i) am2 = __hmax2(am2, *reinterpret_cast<const __nv_bfloat162*>(&w[i]));
       }
-    }
+      float amax = fmaxf(__low2float(am2), __high2float(am2));
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
-    if (lane == 0) part[par][warp] = amax;
-    __syncthreads();
-    amax = part[par][rib * wpr];
-    for (int w = 1; w < wpr; ++w) amax = fmaxf(amax, part[par][rib * wpr + w]);
-    const float s = __fdiv_rn(code_scale_num<F8>(), fmaxf(amax, 1e-5f));
-    const bool live = row < T;
-    if (live && tid == 0) s_x[row] = s;
-    if (Xdq) {
-      for (int j = tid; j < 256; j += nth) table[rib][j] = dq_entry<F8>(j, s);
-      __syncthreads();
-    }
-    if (live) {
+      for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+      const float s = __fdiv_rn(code_scale_num<F8>(), fmaxf(amax, 1e-5f));
+      if (lane == 0) s_x[row] = s;
+      if (Xdq) {
+        for (int i = lane; i < 256; i += 32) table[i] = dq_entry<F8>(i, s);
+        __syncwarp();
+      }
       const size_t rbase = static_cast<size_t>(row) * K;
+#pragma unroll 4
+      for (int v = lane; v < nv; v += 32) {
+        const uint4 u = xr[v];
+        const size_t e = rbase + static_cast<size_t>(v) * 8;
+        uint32_t b[8];  // per element: the code's table index in the low byte
+        if (F8) {
+          int32_t q[8];
+          quant8<true>(u, s, q);
 #pragma unroll
-      for (int i = 0; i < NV; ++i) {
-        const int vi = tid + nth * i;
-        if (vi >= nv) break;
-        int32_t q[8];
-        quant8<F8>(ua[i], s, q);
-        const size_t e = rbase + static_cast<size_t>(vi) * 8;
+          for (int i = 0; i < 8; ++i) b[i] = static_cast<uint32_t>(q[i]);
+        } else {
+          const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+          float z[8];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            z[2 * i] = __fadd_rn(__fmul_rn(bf16_bits_to_f32(w[i] & 0xFFFFu), s), kMagic);
+            z[2 * i + 1] = __fadd_rn(__fmul_rn(bf16_bits_to_f32(w[i] >> 16), s), kMagic);
+          }
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            z[i] = fmaxf(z[i], kMagic - 128.0f);
+            b[i] = __float_as_uint(z[i]);
+          }
+          if (Xq_img) {
+            uint32_t h[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const __nv_bfloat162 p =
+                  __floats2bfloat162_rn(__fsub_rn(z[2 * i], kMagic), __fsub_rn(z[2 * i + 1], kMagic));
+              h[i] = *reinterpret_cast<const uint32_t*>(&p);
+            }
+            __stcs(reinterpret_cast<uint4*>(Xq_img + e), make_uint4(h[0], h[1], h[2], h[3]));
+          }
+        }
         if (Xq) {
           uint2 pk;
-          pk.x = (q[0] & 0xFF) | ((q[1] & 0xFF) << 8) | ((q[2] & 0xFF) << 16) | ((q[3] & 0xFF) << 24);
-          pk.y = (q[4] & 0xFF) | ((q[5] & 0xFF) << 8) | ((q[6] & 0xFF) << 16) | ((q[7] & 0xFF) << 24);
+          pk.x = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
+          pk.y = __byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410);
           __stcs(reinterpret_cast<uint2*>(Xq + e), pk);
-        }
-        if (Xq_img) {
-          uint32_t h[8];
-#pragma unroll
-          for (int j = 0; j < 8; ++j) h[j] = f32_to_bf16_bits(static_cast<float>(q[j]));
-          __stcs(reinterpret_cast<uint4*>(Xq_img + e),
-                 make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
-                            h[6] | (h[7] << 16)));
         }
         if (Xdq) {
           uint32_t h[8];
 #pragma unroll
-          for (int j = 0; j < 8; ++j) h[j] = table[rib][dq_index<F8>(q[j])];
+          for (int i = 0; i < 8; ++i) h[i] = table[F8 ? (b[i] & 0xFFu) : ((b[i] & 0xFFu) ^ 0x80u)];
           __stcs(reinterpret_cast<uint4*>(Xdq + e),
                  make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
                             h[6] | (h[7] << 16)));
         }
       }
+      __syncwarp();  // the table is rewritten for the next row
     }
+    ring.release(j, lane);  // the slot is read for the last time
+  }
+}
+
+// X_tilde = bf16(q / s_x) from int8 activation codes (the dW operand of the
+// int8 call), rows staged as in act_quant_bulk_kernel: each consumer warp
+// builds its row's 256-entry table of correctly rounded quotients (the table
+// dqt_act_quant uses), then maps the row's codes through it, 16 codes (one
+// 16-byte shared load, two 16-byte stores) per lane step.  K % 16 == 0.
+__global__ void __launch_bounds__(32 * 17, 1)
+    codes_to_xdq_bulk_kernel(const int8_t* __restrict__ Xq, const float* __restrict__ s_x, int T,
+                             int K, uint16_t* __restrict__ Xdq, int S, int W, int rpc,
+                             unsigned int* status, uint64_t limit_ns) {
+  extern __shared__ __align__(128) uint8_t cxb_smem[];
+  const RowRing ring(cxb_smem, S, static_cast<uint32_t>(K), rpc, T);
+  uint16_t* tables = reinterpret_cast<uint16_t*>(ring.end());
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  ring.init_barriers();
+  __syncthreads();
+  if (warp == 0) {
+    if (lane == 0) ring.produce(reinterpret_cast<const uint8_t*>(Xq), status, limit_ns);
+    return;
+  }
+  const int cw = warp - 1;
+  uint16_t* t = tables + cw * 256;
+  const int nv = K >> 4;
+  for (int j = cw; j < ring.nchunks; j += W) {
+    const int nr = ring.rows(j);
+    bool acquired = false;
+#pragma unroll 1
+    for (int r = 0; r < nr; ++r) {
+      const int64_t row = ring.row0(j) + r;
+      const float s = s_x[row];
 #pragma unroll
-    for (int i = 0; i < NV; ++i) ua[i] = ub[i];
+      for (int i = lane; i < 256; i += 32) t[i] = dq_entry<false>(i, s);
+      __syncwarp();
+      if (!acquired) {
+        if (!ring.acquire(j, lane, status, limit_ns)) return;
+        acquired = true;
+      }
+      const uint4* src = reinterpret_cast<const uint4*>(ring.row(j, r));
+      uint4* dst = reinterpret_cast<uint4*>(Xdq + static_cast<size_t>(row) * K);
+#pragma unroll 4
+      for (int v = lane; v < nv; v += 32) {
+        const uint4 u = src[v];
+        const uint32_t w[4] = {u.x ^ 0x80808080u, u.y ^ 0x80808080u, u.z ^ 0x80808080u,
+                               u.w ^ 0x80808080u};  // table indices q + 128
+        uint32_t h[8];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          h[2 * i] = t[w[i] & 0xFFu] | (uint32_t(t[(w[i] >> 8) & 0xFFu]) << 16);
+          h[2 * i + 1] = t[(w[i] >> 16) & 0xFFu] | (uint32_t(t[w[i] >> 24]) << 16);
+        }
+        __stcs(dst + 2 * v, make_uint4(h[0], h[1], h[2], h[3]));
+        __stcs(dst + 2 * v + 1, make_uint4(h[4], h[5], h[6], h[7]));
+      }
+      __syncwarp();  // the table is rewritten for the next row
+    }
+    ring.release(j, lane);  // the slot is read for the last time
   }
 }
 
@@ -408,40 +588,67 @@ int grid_for(int64_t work, int threads) {
 
 namespace {
 
+// Geometry of a row ring (act_quant_bulk_kernel, codes_to_xdq_bulk_kernel):
+// chunks of about 8 KB (rows of up to 8 KB are copied one per chunk), then up
+// to 16 consumer warps and as many slots per warp as fit in kAqbRing bytes
+// (48 slots at most); false when fewer than four chunks fit.  One producer
+// thread issues a bulk copy about every 0.2 us whatever its size, so copies
+// below ~8 KB leave the ring short of bytes in flight.
+bool ring_geometry(int64_t row_bytes, int& rpc, int& W, int& S) {
+  rpc = row_bytes >= 8192 ? 1 : static_cast<int>(8192 / row_bytes);
+  const int64_t smax = kAqbRing / (rpc * row_bytes);
+  if (smax < 4) return false;
+  W = static_cast<int>(smax < 16 ? smax : 16);
+  S = static_cast<int>(smax < 48 ? smax : 48) / W * W;
+  return true;
+}
+constexpr int kRingMaxSmem = kAqbRing + 16 * 48 + 16 * 512;  // ring, barriers, tables
+
+// Launches a row-ring kernel: one CTA per SM (at most T), 32 (W + 1) threads.
+template <typename Kern, typename... Args>
+int launch_ring(Kern kern, bool& attr_set, int64_t T, int rpc, int W, int S, int64_t row_bytes,
+                cudaStream_t stream, Args... args) {
+  if (!attr_set) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingMaxSmem) !=
+        cudaSuccess)
+      return 3;
+    attr_set = true;
+  }
+  unsigned int* status = status_word();
+  if (!status) return 3;
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int blocks = static_cast<int>(T < sms ? T : sms);
+  const size_t smem =
+      static_cast<size_t>(S) * rpc * row_bytes + 16 * static_cast<size_t>(S) + 512 * W;
+  kern<<<blocks, 32 * (W + 1), smem, stream>>>(args..., S, W, rpc, status, wait_limit_ns());
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+// Rows staged in shared memory when at least four fit in the ring; -1 when
+// the rows are too long.
+template <bool F8>
+int launch_aq_bulk(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
+                   uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream) {
+  int rpc, W, S;
+  if (!ring_geometry(2 * K, rpc, W, S)) return -1;
+  static bool attr_set = false;  // per template instance
+  return launch_ring(act_quant_bulk_kernel<F8>, attr_set, T, rpc, W, S, 2 * K, stream, X,
+                     static_cast<int>(T), static_cast<int>(K), Xq, s_x, Xq_img, Xdq);
+}
+
 template <bool F8>
 int launch_aq(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x, uint16_t* Xq_img,
               uint16_t* Xdq, cudaStream_t stream) {
-  const int t = static_cast<int>(T), k = static_cast<int>(K);
-  const int64_t nv = K / 8;  // 16-byte vectors per row
-  // persistent rows: warps per row so that each lane holds at most 4 vectors
-  // (8 above 4096 vectors), rows per 256-thread block 8 / wpr
   {
-    const int wpr4 = static_cast<int>((nv + 127) / 128);
-    const int wpr8 = static_cast<int>((nv + 255) / 256);
-    if (wpr4 <= 8 || wpr8 <= 8) {
-      const bool four = wpr4 <= 8;
-      const int wpr = four ? wpr4 : wpr8;
-      const int rpb = 8 / wpr;
-      const int threads = 32 * wpr * rpb;
-      auto kern = four ? act_quant_stream_kernel<4, F8> : act_quant_stream_kernel<8, F8>;
-      static int occ[2][9] = {};  // resident blocks per SM, per NV and wpr
-      int& o = occ[four ? 0 : 1][wpr];
-      int dev = 0, sms = 148;
-      cudaGetDevice(&dev);
-      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-      if (o == 0 && (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, kern, threads, 0) !=
-                         cudaSuccess || o < 1))
-        o = 1;
-      const int64_t want = (T + rpb - 1) / rpb;
-      const int64_t cap = static_cast<int64_t>(sms) * o;
-      const int blocks = static_cast<int>(want < cap ? want : cap);
-      kern<<<blocks, threads, 0, stream>>>(X, t, k, wpr, Xq, s_x, Xq_img, Xdq);
-      return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
-    }
+    const int r = launch_aq_bulk<F8>(X, T, K, Xq, s_x, Xq_img, Xdq, stream);
+    if (r >= 0) return r;
   }
-  // longer rows (more than 16384 elements): one warp per row, two passes
+  // rows longer than 48 KB (K > 24576): one warp per row, two passes
   const int blocks = static_cast<int>((T + kAqWarps - 1) / kAqWarps);
-  act_quant_kernel<F8><<<blocks, kAqWarps * 32, 0, stream>>>(X, t, k, Xq, s_x, Xq_img, Xdq);
+  act_quant_kernel<F8><<<blocks, kAqWarps * 32, 0, stream>>>(X, static_cast<int>(T),
+                                                            static_cast<int>(K), Xq, s_x, Xq_img, Xdq);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
@@ -454,6 +661,14 @@ int launch_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float*
 
 int launch_codes_to_xdq(const int8_t* Xq, const float* s_x, int64_t T, int64_t K, uint16_t* Xdq,
                         cudaStream_t stream) {
+  {
+    int rpc, W, S;
+    if (ring_geometry(K, rpc, W, S)) {
+      static bool attr_set = false;
+      return launch_ring(codes_to_xdq_bulk_kernel, attr_set, T, rpc, W, S, K, stream, Xq, s_x,
+                         static_cast<int>(T), static_cast<int>(K), Xdq);
+    }
+  }
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);

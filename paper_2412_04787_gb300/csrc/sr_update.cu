@@ -127,8 +127,46 @@ __global__ void __launch_bounds__(kThreads)
 // four consecutive columns of one row of a tail tile, sums the token slices'
 // partials in slice order, and applies the same update as sr_update_kernel at
 // the global element index (so the Philox words are those of the fused path).
+// The grid is sized to the blocks that fit at once, and each thread's loads
+// for its next group (the optimiser state and the first four slices'
+// partials) are issued before it updates the current one.
+struct TailGroup {
+  float4 p[4];  // partials of slices 0..3
+  float4 m, v;
+  uint32_t c;   // four int8 codes, or one byte of 2-bit packed codes
+  int64_t e;    // first element, or -1 outside the weight
+  const float* src;
+};
+
+__device__ __forceinline__ void tail_load(int64_t gi, const float* __restrict__ part, int splits,
+                                          int tail, int full, int num_n, int M, int N,
+                                          const int8_t* __restrict__ W, bool packed,
+                                          const float* __restrict__ m, const float* __restrict__ v,
+                                          TailGroup& g) {
+  const int j = static_cast<int>(gi >> 14);
+  const int r = static_cast<int>((gi >> 6) & 255);
+  const int c4 = static_cast<int>(gi & 63) * 4;
+  const int tile = full + j;
+  const int row = (tile / num_n) * 256 + r;
+  const int col = (tile % num_n) * 256 + c4;
+  g.e = -1;
+  if (row >= M || col >= N) return;  // N % 4 == 0: the whole group is in range
+  g.e = static_cast<int64_t>(row) * N + col;
+  if (W) {
+    g.m = __ldcs(reinterpret_cast<const float4*>(m + g.e));
+    g.v = __ldcs(reinterpret_cast<const float4*>(v + g.e));
+    g.c = packed ? static_cast<uint32_t>(reinterpret_cast<const uint8_t*>(W)[g.e >> 2])
+                 : *reinterpret_cast<const uint32_t*>(W + g.e);
+  }
+  g.src = part + static_cast<int64_t>(j) * 65536 + r * 256 + c4;
+  const int64_t sstride = static_cast<int64_t>(tail) * 65536;
+#pragma unroll
+  for (int s = 0; s < 4; ++s)
+    if (s < splits) g.p[s] = __ldcs(reinterpret_cast<const float4*>(g.src + s * sstride));
+}
+
 template <bool DEV>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 3)
     tail_update_kernel(const float* __restrict__ part, int splits, int tail, int full, int num_n,
                        int M, int N, int8_t* __restrict__ W, bool packed, float* __restrict__ m,
                        float* __restrict__ v, const UpdateConsts uc_arg,
@@ -138,49 +176,63 @@ __global__ void __launch_bounds__(kThreads)
   uint8_t* Wp = reinterpret_cast<uint8_t*>(W);
   const int64_t ngroups = static_cast<int64_t>(tail) * 16384;  // 256 x 256 / 4 per tile
   const int64_t stride = static_cast<int64_t>(gridDim.x) * kThreads;
+  const int64_t sstride = static_cast<int64_t>(tail) * 65536;
   uint32_t n_changed = 0;
-  for (int64_t gi = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; gi < ngroups;
-       gi += stride) {
-    const int j = static_cast<int>(gi >> 14);
-    const int r = static_cast<int>((gi >> 6) & 255);
-    const int c4 = static_cast<int>(gi & 63) * 4;
-    const int tile = full + j;
-    const int row = (tile / num_n) * 256 + r;
-    const int col = (tile % num_n) * 256 + c4;
-    if (row >= M || col >= N) continue;  // N % 4 == 0: the whole group is in range
-    const float* src = part + static_cast<int64_t>(j) * 65536 + r * 256 + c4;
-    float4 g4 = __ldcs(reinterpret_cast<const float4*>(src));
-    for (int s = 1; s < splits; ++s) {
-      const float4 h =
-          __ldcs(reinterpret_cast<const float4*>(src + static_cast<int64_t>(s) * tail * 65536));
-      g4.x = __fadd_rn(g4.x, h.x);
-      g4.y = __fadd_rn(g4.y, h.y);
-      g4.z = __fadd_rn(g4.z, h.z);
-      g4.w = __fadd_rn(g4.w, h.w);
+  int64_t gi = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x;
+  TailGroup cur;
+  if (gi < ngroups) tail_load(gi, part, splits, tail, full, num_n, M, N, W, packed, m, v, cur);
+  for (; gi < ngroups; gi += stride) {
+    TailGroup nxt;
+    nxt.e = -1;
+    if (gi + stride < ngroups)
+      tail_load(gi + stride, part, splits, tail, full, num_n, M, N, W, packed, m, v, nxt);
+    if (cur.e >= 0) {
+      const int64_t e = cur.e;
+      float4 g4 = cur.p[0];
+#pragma unroll
+      for (int s = 1; s < 4; ++s)
+        if (s < splits) {
+          g4.x = __fadd_rn(g4.x, cur.p[s].x);
+          g4.y = __fadd_rn(g4.y, cur.p[s].y);
+          g4.z = __fadd_rn(g4.z, cur.p[s].z);
+          g4.w = __fadd_rn(g4.w, cur.p[s].w);
+        }
+      for (int s = 4; s < splits; ++s) {  // slices beyond the fourth, in order
+        const float4 h = __ldcs(reinterpret_cast<const float4*>(cur.src + s * sstride));
+        g4.x = __fadd_rn(g4.x, h.x);
+        g4.y = __fadd_rn(g4.y, h.y);
+        g4.z = __fadd_rn(g4.z, h.z);
+        g4.w = __fadd_rn(g4.w, h.w);
+      }
+      if (dW_out) __stcs(reinterpret_cast<float4*>(dW_out + e), g4);
+      if (W) {
+        const uint32_t craw = cur.c;
+        const char4 c0 = packed ? tern_unpack4(craw)
+                                : make_char4(static_cast<signed char>(craw & 0xFFu),
+                                             static_cast<signed char>((craw >> 8) & 0xFFu),
+                                             static_cast<signed char>((craw >> 16) & 0xFFu),
+                                             static_cast<signed char>(craw >> 24));
+        float4 m4 = cur.m, v4 = cur.v;
+        uint4 w = make_uint4(0, 0, 0, 0);
+        if (uc.round_mode == 0)
+          w = sr_words(global_blk(uc, static_cast<uint64_t>(e >> 2)), uc.step_lo, uc.tensor_id,
+                       uc.key0, uc.key1);
+        const int32_t a = dqt_update_elem(uc, g4.x, c0.x, m4.x, v4.x, w.x);
+        const int32_t b = dqt_update_elem(uc, g4.y, c0.y, m4.y, v4.y, w.y);
+        const int32_t c = dqt_update_elem(uc, g4.z, c0.z, m4.z, v4.z, w.z);
+        const int32_t d = dqt_update_elem(uc, g4.w, c0.w, m4.w, v4.w, w.w);
+        n_changed += (a != c0.x) + (b != c0.y) + (c != c0.z) + (d != c0.w);
+        if (packed)
+          Wp[e >> 2] = static_cast<uint8_t>(tern_pack4(a, b, c, d));
+        else
+          *reinterpret_cast<char4*>(W + e) =
+              make_char4(static_cast<signed char>(a), static_cast<signed char>(b),
+                         static_cast<signed char>(c), static_cast<signed char>(d));
+        __stcs(reinterpret_cast<float4*>(m + e), m4);
+        __stcs(reinterpret_cast<float4*>(v + e), v4);
+      }
     }
-    const int64_t e = static_cast<int64_t>(row) * N + col;
-    if (dW_out) __stcs(reinterpret_cast<float4*>(dW_out + e), g4);
-    if (!W) continue;
-    float4 m4 = __ldcs(reinterpret_cast<const float4*>(m + e));
-    float4 v4 = __ldcs(reinterpret_cast<const float4*>(v + e));
-    const char4 c0 = packed ? tern_unpack4(Wp[e >> 2]) : *reinterpret_cast<const char4*>(W + e);
-    uint4 w = make_uint4(0, 0, 0, 0);
-    if (uc.round_mode == 0)
-      w = sr_words(global_blk(uc, static_cast<uint64_t>(e >> 2)), uc.step_lo, uc.tensor_id, uc.key0,
-                   uc.key1);
-    const int32_t a = dqt_update_elem(uc, g4.x, c0.x, m4.x, v4.x, w.x);
-    const int32_t b = dqt_update_elem(uc, g4.y, c0.y, m4.y, v4.y, w.y);
-    const int32_t c = dqt_update_elem(uc, g4.z, c0.z, m4.z, v4.z, w.z);
-    const int32_t d = dqt_update_elem(uc, g4.w, c0.w, m4.w, v4.w, w.w);
-    n_changed += (a != c0.x) + (b != c0.y) + (c != c0.z) + (d != c0.w);
-    if (packed)
-      Wp[e >> 2] = static_cast<uint8_t>(tern_pack4(a, b, c, d));
-    else
-      *reinterpret_cast<char4*>(W + e) =
-          make_char4(static_cast<signed char>(a), static_cast<signed char>(b),
-                     static_cast<signed char>(c), static_cast<signed char>(d));
-    __stcs(reinterpret_cast<float4*>(m + e), m4);
-    __stcs(reinterpret_cast<float4*>(v + e), v4);
+    cur = nxt;
   }
   if (changed) {
 #pragma unroll
@@ -253,7 +305,22 @@ int launch_tail_update(const float* part, int splits, int tail, int full, int nu
                        int8_t* W, bool packed, float* m, float* v, const UpdateConsts& uc,
                        const UpdateConsts* uc_dev, unsigned long long* changed, float* dW_out,
                        cudaStream_t stream) {
-  const int blocks = stream_blocks(static_cast<int64_t>(tail) * 65536);
+  // the blocks that fit at once: each thread walks several groups, its next
+  // group's loads in flight
+  static int occ[2] = {0, 0};  // resident blocks per SM, per template instance
+  int& o = occ[uc_dev ? 1 : 0];
+  if (o == 0) {
+    const void* k = uc_dev ? reinterpret_cast<const void*>(tail_update_kernel<true>)
+                           : reinterpret_cast<const void*>(tail_update_kernel<false>);
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, k, kThreads, 0) != cudaSuccess || o < 1)
+      o = 1;
+  }
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t want = (static_cast<int64_t>(tail) * 16384 + kThreads - 1) / kThreads;
+  const int64_t cap = static_cast<int64_t>(sms) * o;
+  const int blocks = static_cast<int>(want < cap ? want : cap);
   if (uc_dev)
     tail_update_kernel<true><<<blocks, kThreads, 0, stream>>>(part, splits, tail, full, num_n, M, N,
                                                               W, packed, m, v, uc, uc_dev, changed,

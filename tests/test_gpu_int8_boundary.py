@@ -58,7 +58,8 @@ def problem(T, K, N, bits_w, seed=1):
 # ---------------------------------------------------------------------------
 # activation codes: 2 bytes read, 1 byte written per element
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("T,K", [(256, 512), (37, 264), (1, 8), (8192, 2048), (300, 5632)])
+@pytest.mark.parametrize("T,K", [(256, 512), (37, 264), (1, 8), (8192, 2048), (300, 5632),
+                                 (1000, 1088), (3, 24584)])
 def test_act_quant_codes_only(T, K):
     X = inputs.normal((T, K), 1.0, seed=T * 7 + K, dtype=torch.bfloat16)
     if T > 2:
@@ -71,7 +72,7 @@ def test_act_quant_codes_only(T, K):
     assert np.array_equal(s_x.cpu().numpy().view(np.uint32), s.view(np.uint32))
 
 
-@pytest.mark.parametrize("T,K", [(256, 512), (37, 272), (8192, 5632)])
+@pytest.mark.parametrize("T,K", [(256, 512), (37, 272), (8192, 5632), (300, 2048), (3, 49168)])
 def test_codes_to_xdq_is_the_act_quant_image(T, K):
     """The X_tilde conversion the weight-gradient call runs: bf16(q / s_x),
     bit for bit the oracle's image."""

@@ -73,7 +73,8 @@ def problem(T, K, N, bits_w, seed=1):
 # ---------------------------------------------------------------------------
 # act_quant (bit-exact)
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("T,K", [(256, 512), (37, 264), (1, 8), (300, 5632), (8192, 2048)])
+@pytest.mark.parametrize("T,K", [(256, 512), (37, 264), (1, 8), (300, 5632), (8192, 2048),
+                                 (129, 72), (5, 16384), (3, 24584)])
 def test_act_quant_bit_exact(T, K):
     X = inputs.normal((T, K), 1.0, seed=T + K, dtype=torch.bfloat16)
     if T > 2:
