@@ -80,7 +80,8 @@ def kernel_fingerprint(files=GEMM_SOURCES):
 # of operand and optimiser-state bytes), from one ncu capture, keyed by the
 # GEMM-source fingerprint it was taken on (see profiles/).  A stale entry
 # reports null.
-DW_TRAFFIC_BYTES = {"82d12725fdfa": 262571008 + 61169152 + 33047808,
+DW_TRAFFIC_BYTES = {"ac36c0aa63c5": 261135360 + 57050112 + 33049600,
+                    "82d12725fdfa": 262571008 + 61169152 + 33047808,
                     "a25cf8632190": 261430272 + 59386112 + 33048064}
 
 
@@ -154,7 +155,7 @@ class MLPStep:
     """Device buffers and the launch sequence of one DQT MLP training step."""
 
     def __init__(self, dev, seed=1234, fp8=False, optimizer="adamw", packed=False, bits=1.58,
-                 operands="int8"):
+                 operands="int8", tail_slices=True):
         from paper_2412_04787_gb300 import dqt, inputs
 
         self.dqt = dqt
@@ -228,7 +229,7 @@ class MLPStep:
         if self.i8:
             nbw = max(dqt.dqt_bwd_dw_workspace_size(T, N, K) for _, K, N in PROJ)
             self.dw_ws = [torch.empty(nbw, dtype=torch.uint8, device=dev) for _ in range(4)]
-            nbx = max(dqt.dqt_bwd_dx_workspace_size(N, K) for _, K, N in PROJ)
+            nbx = max(dqt.dqt_bwd_dx_workspace_size(T, N, K) for _, K, N in PROJ)
             self.dx_ws = [torch.empty(nbx, dtype=torch.uint8, device=dev) for _ in range(4)]
             nbf = max(dqt.dqt_fwd_workspace_size(T, K, N) for _, K, N in PROJ)
             self.fwd_ws = [torch.empty(nbf, dtype=torch.uint8, device=dev) for _ in range(4)]
@@ -236,6 +237,12 @@ class MLPStep:
             nbw = max(dqt.dqt_bwd_dw_img_workspace_size(T, N, K) for _, K, N in PROJ)
             self.dw_ws = [torch.empty(max(nbw, 16), dtype=torch.uint8, device=dev) if nbw else False
                           for _ in range(4)]
+        # forward and dX workspace for the partials of their sliced last wave,
+        # one per stream (the GEMMs of one stream run one after the other)
+        nbt = max(max(dqt.dqt_fwd_img_workspace_size(T, K, N),
+                      dqt.dqt_bwd_dx_img_workspace_size(T, N, K)) for _, K, N in PROJ)
+        self.tail_ws = [torch.empty(max(nbt, 16), dtype=torch.uint8, device=dev)
+                        if nbt and tail_slices else False for _ in range(4)]
         # kernel launches per step: act_quant 2, weight images 3 (+3 E4M3),
         # forward 3, dX 3, and per projection the dW GEMM, the streaming
         # kernel of its sliced last wave (when the shape has one), and for
@@ -244,6 +251,8 @@ class MLPStep:
         # instead of the 3 shared weight images), each dX call the weight
         # and each dW call X_tilde (3 + 3)
         dw = [1 + (1 if dqt.dqt_bwd_dw_img_workspace_size(T, N, K) > 0 else 0) for _, K, N in PROJ]
+        # (the forward's and dX's cut last wave is summed inside the GEMM: no
+        # launch of its own)
         self.launches_per_step = 2 + 3 + 3 + 3 + sum(dw) + (3 if fp8 else 0) + (6 if self.i8 else 0)
         self.dw_kind = "bwd_dw_adafactor" if optimizer == "adafactor" else "bwd_dw_update"
         if self.i8:
@@ -347,12 +356,15 @@ class MLPStep:
                     W = self.W[name]
                     (T_, K_), N_ = q_img.shape, W.shape[0]
                     a_bytes = (T_ * K_ * 2 + 255) // 256 * 256
+                    w_bytes = (N_ * K_ * 2 + 255) // 256 * 256
                     qi = ws[: T_ * K_ * 2].view(torch.bfloat16).view(T_, K_)
                     wi = ws[a_bytes: a_bytes + N_ * K_ * 2].view(torch.bfloat16).view(N_, K_)
+                    tail = ws[a_bytes + w_bytes:]
                     timed("codes_to_bf16", stream, lambda: dqt.dqt_codes_to_bf16(q_img, qi))
                     timed("codes_to_bf16", stream, lambda: dqt.dqt_codes_to_bf16(W, wi))
                     timed("fwd", stream, lambda: dqt.dqt_bitlinear_fwd_img(
-                        qi, s_x, wi, self.s_w[name], self.grid, Y=self.Y[name]))
+                        qi, s_x, wi, self.s_w[name], self.grid, Y=self.Y[name],
+                        ws=tail if tail.numel() else False))
                 else:
                     dqt.dqt_bitlinear_fwd(q_img, s_x, self.W[name], self.s_w[name], self.grid,
                                           Y=self.Y[name], ws=ws)
@@ -361,23 +373,28 @@ class MLPStep:
                     q_img, s_x, self.W8[name], self.s_w[name], self.grid, Y=self.Y[name]))
             else:
                 timed("fwd", stream, lambda: dqt.dqt_bitlinear_fwd_img(
-                    q_img, s_x, self.W_img[name], self.s_w[name], self.grid, Y=self.Y[name]))
+                    q_img, s_x, self.W_img[name], self.s_w[name], self.grid, Y=self.Y[name],
+                    ws=self.tail_ws[s.index(stream)]))
 
         def dx(name, stream):
             if self.i8:
                 ws = self.dx_ws[s.index(stream)]
                 if parts:
-                    img = ws[: 2 * self.W[name].numel()].view(torch.bfloat16).view(self.W[name].shape)
+                    nb = 2 * self.W[name].numel()
+                    img = ws[: nb].view(torch.bfloat16).view(self.W[name].shape)
+                    tail = ws[(nb + 255) // 256 * 256:]
                     timed("codes_to_bf16", stream,
                           lambda: dqt.dqt_codes_to_bf16(self.W[name], img))
                     timed("bwd_dx", stream, lambda: dqt.dqt_bitlinear_bwd_dx_img(
-                        self.d["dY_" + name], img, self.s_w[name], dX=self.dX[name]))
+                        self.d["dY_" + name], img, self.s_w[name], dX=self.dX[name],
+                        ws=tail if tail.numel() else False))
                 else:
                     dqt.dqt_bitlinear_bwd_dx(self.d["dY_" + name], self.W[name], self.s_w[name],
                                              dX=self.dX[name], ws=ws)
                 return
             timed("bwd_dx", stream, lambda: dqt.dqt_bitlinear_bwd_dx_img(
-                self.d["dY_" + name], self.W_img[name], self.s_w[name], dX=self.dX[name]))
+                self.d["dY_" + name], self.W_img[name], self.s_w[name], dX=self.dX[name],
+                ws=self.tail_ws[s.index(stream)]))
 
         def dw(i, name, stream):
             xdq = self.aq["H" if name == "down" else "X"][2]
@@ -602,7 +619,7 @@ def run_gpu(args):
     from paper_2412_04787_gb300 import build as dqt_build
     dqt_build.build()
     st = MLPStep(dev, fp8=args.act == "fp8", optimizer=args.optimizer, packed=args.packed,
-                 bits=args.bits, operands=args.operands)
+                 bits=args.bits, operands=args.operands, tail_slices=not args.no_tail_slices)
     if dp_mode == "exchange":
         st.enable_dp()
     dqt = st.dqt
@@ -1112,10 +1129,14 @@ def run_kernel(args):
         dX = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
         hp = dqt.adamw()
         sr = dqt.sr_stream()
+        nbt = max(dqt.dqt_fwd_img_workspace_size(T, K, N), dqt.dqt_bwd_dx_img_workspace_size(T, N, K))
+        tws = torch.empty(nbt, dtype=torch.uint8, device=dev) if nbt else False
+        if args.no_tail_slices:
+            tws = False
         if k == "fwd":
-            fn = lambda: dqt.dqt_bitlinear_fwd_img(q_img, s_x, W_img, s_w, g, Y=Y)  # noqa: E731
+            fn = lambda: dqt.dqt_bitlinear_fwd_img(q_img, s_x, W_img, s_w, g, Y=Y, ws=tws)  # noqa: E731
         elif k == "bwd_dx":
-            fn = lambda: dqt.dqt_bitlinear_bwd_dx_img(dY, W_img, s_w, dX=dX)  # noqa: E731
+            fn = lambda: dqt.dqt_bitlinear_bwd_dx_img(dY, W_img, s_w, dX=dX, ws=tws)  # noqa: E731
         elif k == "bwd_dw_update":
             fn = lambda: dqt.dqt_bitlinear_bwd_dw_update_img(dY, xdq, W, s_w, m, v, hp, sr, g)  # noqa: E731
         elif k == "bwd_dw":  # gradient only (fp32 dW written, no update)
@@ -1500,6 +1521,9 @@ def main():
     ap.add_argument("--impl", default="dqt", choices=["dqt", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-tail-slices", action="store_true",
+                    help="the forward and dX GEMMs without a workspace, so their last wave is "
+                         "not cut into reduction slices (A/B of that schedule; image operands)")
     ap.add_argument("--no-extras", action="store_true",
                     help="mlp: skip the single-layer step and the SR-update sweep keys")
     ap.add_argument("--kernel", default=None,

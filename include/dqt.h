@@ -207,7 +207,8 @@ int dqt_codes_to_xdq(const int8_t* Xq, const float* s_x, int64_t T, int64_t K, d
  *   Y        bf16 [T, N] out;  acc_out int32 [T, N] out, or NULL
  *   ws       device workspace of at least dqt_fwd_workspace_size(T, K, N) bytes
  *            (16-byte aligned): it receives the exact bf16 images of Xq and W
- *            (3 bytes moved per element of each), which the GEMM then reads
+ *            (3 bytes moved per element of each), which the GEMM then reads,
+ *            and the partials of the last-wave slices (dqt_bitlinear_fwd_img)
  * K, N multiples of 8; Xq, W, Y, acc_out 16-byte aligned; T >= 1; T, N, K < 2^31. */
 size_t dqt_fwd_workspace_size(int64_t T, int64_t K, int64_t N);
 int dqt_bitlinear_fwd(const int8_t* Xq, const float* s_x, const int8_t* W, float s_w,
@@ -215,25 +216,43 @@ int dqt_bitlinear_fwd(const int8_t* Xq, const float* s_x, const int8_t* W, float
                       int32_t* acc_out, void* ws, size_t ws_bytes, void* stream);
 
 /* The same forward on the bf16 operand images (dqt_act_quant_images' Xq_img
- * and dqt_codes_to_bf16's W_img); K, N multiples of 8.  Identical Y and acc. */
+ * and dqt_codes_to_bf16's W_img); K, N multiples of 8.  Identical Y and acc.
+ * ws: NULL, or a device workspace of at least dqt_fwd_img_workspace_size(T, K,
+ * N) bytes (16-byte aligned; DQT_ERR_ARG if smaller).  With it, when the
+ * output's 256 x 256 tiles leave the last wave of the 2-SM kernel short, the
+ * tiles of that wave are cut into reduction slices whose fp32 partials go to
+ * the workspace, and the last slice to finish a region adds them in slice
+ * order and applies the epilogue; every partial is an exact integer, so Y and
+ * acc are those of the uncut kernel bit for bit.  The size is 0 (any ws) when
+ * no cut is planned.  A workspace serves one call at a time. */
+size_t dqt_fwd_img_workspace_size(int64_t T, int64_t K, int64_t N);
 int dqt_bitlinear_fwd_img(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img,
                           float s_w, dqt_grid_t grid, int64_t T, int64_t K, int64_t N,
-                          dqt_bf16* Y, int32_t* acc_out, void* stream);
+                          dqt_bf16* Y, int32_t* acc_out, void* ws, size_t ws_bytes,
+                          void* stream);
 
 /* Backward w.r.t. the input, no straight-through estimator on the weight
  * (the gradient is taken w.r.t. W_tilde itself, Sec. 3.2):
  *   dX[t,k] = bf16( (sum_n dY[t,n] c[n,k]) * (1 / s_w) )   fp32 accumulation
  *   dY bf16 [T, N];  W int8 [N, K] codes;  dX bf16 [T, K] out.
- * ws: device workspace of at least dqt_bwd_dx_workspace_size(N, K) bytes
+ * ws: device workspace of at least dqt_bwd_dx_workspace_size(T, N, K) bytes
  * (16-byte aligned; it receives the exact bf16 image of the codes, 3 bytes
- * moved per weight, before the GEMM reads it).  K, N multiples of 8. */
-size_t dqt_bwd_dx_workspace_size(int64_t N, int64_t K);
+ * moved per weight, before the GEMM reads it, and the partials of the
+ * last-wave slices, see dqt_bitlinear_bwd_dx_img).  K, N multiples of 8. */
+size_t dqt_bwd_dx_workspace_size(int64_t T, int64_t N, int64_t K);
 int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const int8_t* W, float s_w, int64_t T, int64_t N,
                          int64_t K, dqt_bf16* dX, void* ws, size_t ws_bytes, void* stream);
 
-/* The same on the weight's bf16 image W_img [N, K] (dqt_codes_to_bf16). */
+/* The same on the weight's bf16 image W_img [N, K] (dqt_codes_to_bf16).
+ * ws: NULL, or at least dqt_bwd_dx_img_workspace_size(T, N, K) bytes
+ * (16-byte aligned; DQT_ERR_ARG if smaller): with it the last wave's output
+ * tiles may be cut into reduction slices as in dqt_bitlinear_fwd_img, their
+ * partials added in slice order (a fixed fp32 summation order, so the result
+ * is reproducible; it may differ in the last bits from the uncut kernel's). */
+size_t dqt_bwd_dx_img_workspace_size(int64_t T, int64_t N, int64_t K);
 int dqt_bitlinear_bwd_dx_img(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, int64_t T,
-                             int64_t N, int64_t K, dqt_bf16* dX, void* stream);
+                             int64_t N, int64_t K, dqt_bf16* dX, void* ws, size_t ws_bytes,
+                             void* stream);
 
 /* Backward w.r.t. the weight fused with the DQT update (Sec. 3.2, Sec. 4.1, Eq. 5):
  *   X_tilde = bf16(Xq / s_x)                       the dequantised activation

@@ -290,7 +290,7 @@ static bool fwd_range_ok(dqt_grid_t grid, int64_t K) {
 // chunks whose partial sums stay <= 2^24 (exact in fp32).
 static int fwd_launch(const void* A, const float* s_x, const void* B, float s_w,
                dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y, int32_t* acc_out,
-               void* stream) {
+               void* tail_ws, size_t tail_bytes, void* stream) {
   const int64_t cmax = grid.qmax > -grid.qmin ? grid.qmax : -grid.qmin;
   const int64_t cm = cmax > 0 ? cmax : 1;
   // Largest chunk whose partial sums stay <= 2^24 (exact in fp32), multiple of 64.
@@ -309,15 +309,30 @@ static int fwd_launch(const void* A, const float* s_x, const void* B, float s_w,
   g.scale = s_w;
   g.out_bf16 = Y;
   g.acc_out = acc_out;
+  g.ws = tail_ws;
+  g.ws_bytes = tail_ws ? tail_bytes : 0;
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
 static inline size_t fwd_ws_align(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
+// Workspace of the last-wave reduction slices of a 2-SM forward or dX GEMM
+// (M x N output reduced over Kred); 0 with 1-SM tiles.
+static size_t gemm_tail_ws(int64_t M, int64_t N, int64_t Kred) {
+  if (dqt::gemm_mode() != 0) return 0;
+  return dqt::gemm_tail_bytes(static_cast<int>(M), static_cast<int>(N), static_cast<int>(Kred));
+}
+
 size_t dqt_fwd_workspace_size(int64_t T, int64_t K, int64_t N) {
   if (T <= 0 || K <= 0 || N <= 0 || T > kMaxDim || K > kMaxDim || N > kMaxDim) return 0;
   return fwd_ws_align(static_cast<size_t>(T) * static_cast<size_t>(K) * 2u) +
-         fwd_ws_align(static_cast<size_t>(N) * static_cast<size_t>(K) * 2u);
+         fwd_ws_align(static_cast<size_t>(N) * static_cast<size_t>(K) * 2u) +
+         dqt_fwd_img_workspace_size(T, K, N);
+}
+
+size_t dqt_fwd_img_workspace_size(int64_t T, int64_t K, int64_t N) {
+  if (T <= 0 || K <= 0 || N <= 0 || T > kMaxDim || K > kMaxDim || N > kMaxDim) return 0;
+  return gemm_tail_ws(T, N, K);
 }
 
 int dqt_bitlinear_fwd(const int8_t* Xq, const float* s_x, const int8_t* W, float s_w,
@@ -333,27 +348,32 @@ int dqt_bitlinear_fwd(const int8_t* Xq, const float* s_x, const int8_t* W, float
     return DQT_ERR_ALIGN;
   // the exact bf16 images of both operands' codes, then the GEMM on them
   cudaStream_t st = as_stream(stream);
+  const size_t x_bytes = fwd_ws_align(static_cast<size_t>(T) * static_cast<size_t>(K) * 2u);
+  const size_t w_bytes = fwd_ws_align(static_cast<size_t>(N) * static_cast<size_t>(K) * 2u);
   dqt_bf16* Xq_img = static_cast<dqt_bf16*>(ws);
-  dqt_bf16* W_img = reinterpret_cast<dqt_bf16*>(
-      static_cast<uint8_t*>(ws) + fwd_ws_align(static_cast<size_t>(T) * static_cast<size_t>(K) * 2u));
+  dqt_bf16* W_img = reinterpret_cast<dqt_bf16*>(static_cast<uint8_t*>(ws) + x_bytes);
   if (dqt::launch_codes_to_bf16(Xq, T * K, Xq_img, st) ||
       dqt::launch_codes_to_bf16(W, N * K, W_img, st))
     return DQT_ERR_CUDA;
-  return fwd_launch(Xq_img, s_x, W_img, s_w, grid, T, K, N, Y, acc_out, stream);
+  return fwd_launch(Xq_img, s_x, W_img, s_w, grid, T, K, N, Y, acc_out,
+                    static_cast<uint8_t*>(ws) + x_bytes + w_bytes, ws_bytes - x_bytes - w_bytes,
+                    stream);
 }
 
 int dqt_bitlinear_fwd_img(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img,
                           float s_w, dqt_grid_t grid, int64_t T, int64_t K, int64_t N,
-                          dqt_bf16* Y, int32_t* acc_out, void* stream) {
+                          dqt_bf16* Y, int32_t* acc_out, void* ws, size_t ws_bytes,
+                          void* stream) {
   if (!Xq_img || !s_x || !W_img || !Y || T <= 0 || K <= 0 || N <= 0 || !grid_ok(grid) ||
       !(s_w > 0.0f) || !isfinite(s_w))
     return DQT_ERR_ARG;
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
+  if (ws && ws_bytes < dqt_fwd_img_workspace_size(T, K, N)) return DQT_ERR_ARG;
   if (K % 8 || N % 8 || !aligned16(Xq_img) || !aligned16(W_img) || !aligned16(Y) ||
-      (acc_out && !aligned16(acc_out)))
+      (acc_out && !aligned16(acc_out)) || (ws && !aligned16(ws)))
     return DQT_ERR_ALIGN;
   if (!fwd_range_ok(grid, K)) return DQT_ERR_RANGE;
-  return fwd_launch(Xq_img, s_x, W_img, s_w, grid, T, K, N, Y, acc_out, stream);
+  return fwd_launch(Xq_img, s_x, W_img, s_w, grid, T, K, N, Y, acc_out, ws, ws_bytes, stream);
 }
 
 int dqt_act_quant_fp8(const dqt_bf16* X, int64_t T, int64_t K, uint8_t* Xq8, float* s_x8,
@@ -401,9 +421,15 @@ int dqt_bitlinear_fwd_fp8(const uint8_t* Xq8, const float* s_x8, const uint8_t* 
 
 static inline size_t ws_align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
-size_t dqt_bwd_dx_workspace_size(int64_t N, int64_t K) {
-  if (N <= 0 || K <= 0 || N > kMaxDim || K > kMaxDim) return 0;
-  return ws_align256(static_cast<size_t>(N) * static_cast<size_t>(K) * 2u);
+size_t dqt_bwd_dx_workspace_size(int64_t T, int64_t N, int64_t K) {
+  if (T <= 0 || N <= 0 || K <= 0 || T > kMaxDim || N > kMaxDim || K > kMaxDim) return 0;
+  return ws_align256(static_cast<size_t>(N) * static_cast<size_t>(K) * 2u) +
+         dqt_bwd_dx_img_workspace_size(T, N, K);
+}
+
+size_t dqt_bwd_dx_img_workspace_size(int64_t T, int64_t N, int64_t K) {
+  if (T <= 0 || N <= 0 || K <= 0 || T > kMaxDim || N > kMaxDim || K > kMaxDim) return 0;
+  return gemm_tail_ws(T, K, N);
 }
 
 int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const int8_t* W, float s_w, int64_t T, int64_t N,
@@ -411,21 +437,27 @@ int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const int8_t* W, float s_w, int64_t
   if (!dY || !W || !dX || !ws || T <= 0 || N <= 0 || K <= 0 || !(s_w > 0.0f) || !isfinite(s_w))
     return DQT_ERR_ARG;
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
-  if (ws_bytes < dqt_bwd_dx_workspace_size(N, K)) return DQT_ERR_ARG;
+  if (ws_bytes < dqt_bwd_dx_workspace_size(T, N, K)) return DQT_ERR_ARG;
   if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(W) || !aligned16(dX) || !aligned16(ws))
     return DQT_ERR_ALIGN;
-  // the exact bf16 image of the codes, then the GEMM on it
+  // the exact bf16 image of the codes, then the GEMM on it (the rest of the
+  // workspace holds its last-wave slice partials)
+  const size_t w_bytes = ws_align256(static_cast<size_t>(N) * static_cast<size_t>(K) * 2u);
   dqt_bf16* W_img = static_cast<dqt_bf16*>(ws);
   if (dqt::launch_codes_to_bf16(W, N * K, W_img, as_stream(stream))) return DQT_ERR_CUDA;
-  return dqt_bitlinear_bwd_dx_img(dY, W_img, s_w, T, N, K, dX, stream);
+  return dqt_bitlinear_bwd_dx_img(dY, W_img, s_w, T, N, K, dX, static_cast<uint8_t*>(ws) + w_bytes,
+                                  ws_bytes - w_bytes, stream);
 }
 
 int dqt_bitlinear_bwd_dx_img(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, int64_t T,
-                             int64_t N, int64_t K, dqt_bf16* dX, void* stream) {
+                             int64_t N, int64_t K, dqt_bf16* dX, void* ws, size_t ws_bytes,
+                             void* stream) {
   if (!dY || !W_img || !dX || T <= 0 || N <= 0 || K <= 0 || !(s_w > 0.0f) || !isfinite(s_w))
     return DQT_ERR_ARG;
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
-  if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(W_img) || !aligned16(dX))
+  if (ws && ws_bytes < dqt_bwd_dx_img_workspace_size(T, N, K)) return DQT_ERR_ARG;
+  if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(W_img) || !aligned16(dX) ||
+      (ws && !aligned16(ws)))
     return DQT_ERR_ALIGN;
   dqt::GemmLaunch g{};
   g.kind = dqt::GEMM_DX;
@@ -436,6 +468,8 @@ int dqt_bitlinear_bwd_dx_img(const dqt_bf16* dY, const dqt_bf16* W_img, float s_
   g.B = W_img;
   g.scale = 1.0f / s_w;
   g.out_bf16 = dX;
+  g.ws = ws;
+  g.ws_bytes = ws ? ws_bytes : 0;
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
@@ -458,7 +492,7 @@ size_t dqt_bwd_dw_img_workspace_size(int64_t T, int64_t N, int64_t K) {
   const dqt::TailPlan tp =
       dqt::tail_plan(static_cast<int>(N), static_cast<int>(K), static_cast<int>(T), sms / 2);
   if (tp.splits < 2) return 0;
-  return static_cast<size_t>(sms / 2) * 65536 * sizeof(float);
+  return 256 + static_cast<size_t>(sms / 2) * 65536 * sizeof(float);  // + 256: alignment
 }
 
 int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const int8_t* Xq, const float* s_x,

@@ -74,6 +74,12 @@ struct TailPlan {
 };
 TailPlan tail_plan(int M, int N, int Kred, int clusters);
 
+// Workspace bytes for the last-wave token (or reduction) slices of a 2-SM
+// GEMM with an M x N output reduced over Kred on this device: the slices'
+// fp32 partials, or 0 when the output's tiles fill the waves closely enough
+// that no slicing is planned.
+size_t gemm_tail_bytes(int M, int N, int Kred);
+
 // Sums the tail slices' partials (slice s of tail tile j at (s * tail + j) *
 // 65536 floats, tile-local row-major 256 x 256; tile full + j of an M x N
 // output with num_n tiles per row) in slice order and applies the update of

@@ -44,6 +44,8 @@
 // (max|c| = 1) need no drain for K <= 131072.
 #include <cuda.h>
 
+#include <atomic>
+
 #include "dqt_internal.h"
 
 namespace dqt {
@@ -90,6 +92,12 @@ struct Params {
   // sums them in slice order and applies the update.
   int full_units, full_tiles, tail_tiles, tail_splits, tail_kbps;
   float* part;
+  // forward / dX tail: the slices of a tile region are added by the last of
+  // them to finish, found with one counter per (tail tile, CTA rank,
+  // epilogue warp): (tag << 16) | slices done, tag unique per launch, so a
+  // counter left by an earlier launch counts as zero
+  unsigned long long* tail_ctr;
+  unsigned long long tail_tag;
 };
 
 struct Unit {
@@ -137,6 +145,12 @@ struct Smem {
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   const uint32_t s = smem_u32(p);
   return p + ((1024u - (s & 1023u)) & 1023u);
+}
+
+// Invalidate the 128-byte L2 line at p (128-byte aligned) without writing it
+// back: for data that is dead once read (slice partials).
+__device__ __forceinline__ void l2_discard_line(const void* p) {
+  asm volatile("discard.global.L2 [%0], 128;" ::"l"(p) : "memory");
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
@@ -1000,23 +1014,98 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
       if (!ok) break;
       tc_fence_after();
       const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(b * BN + half * HALF);
-      if (EPI == GEMM_DW && un.slice >= 0) {
+      if ((EPI == GEMM_DW || EPI == GEMM_FWD || EPI == GEMM_DX) && un.slice >= 0) {
         // a tail slice: its fp32 partial to the slice buffer, tile-local
         // row-major (this lane's row, 32 columns per chunk: 128 contiguous bytes)
-        float* dst_tile = p.part + (static_cast<long long>(un.slice) * p.tail_tiles +
-                                    (tile - p.full_tiles)) * 65536LL +
-                          (static_cast<long long>(rank) * 128 + row) * 256 + half * HALF;
+        // dW: tile-local row-major (this lane's row, 32 columns per chunk:
+        // 128 contiguous bytes), the layout the streaming update reads.
+        // Forward / dX: 32 x 32 blocks (block (row / 32, column / 32) at
+        // 1024 (8 (row / 32) + column / 32) floats), each stored as [column
+        // quad][row][4]: a warp's store of one column quad of its 32 rows is
+        // 512 contiguous bytes, and so is the fix-up's load below.
+        const int jt = tile - p.full_tiles;
+        const long long roff = (static_cast<long long>(rank) * 128 + row) * 256 + half * HALF;
+        const long long tile_off = (static_cast<long long>(un.slice) * p.tail_tiles + jt) * 65536LL;
+        const int blk0 = ((static_cast<int>(rank) * 4 + quad) * 8 + half * (HALF / 32)) * 1024;
 #pragma unroll 1
         for (int cc = 0; cc < HALF / 32; ++cc) {
           uint32_t a[32];
           tmem_ld_32x32b_x32(t_acc + cc * 32, a);
           tmem_ld_wait();
-          float4* dst = reinterpret_cast<float4*>(dst_tile + cc * 32);
+          float4* dst = EPI == GEMM_DW
+                            ? reinterpret_cast<float4*>(p.part + tile_off + roff + cc * 32)
+                            : reinterpret_cast<float4*>(p.part + tile_off + blk0 + cc * 1024) + lane;
 #pragma unroll
           for (int j = 0; j < 8; ++j)
-            __stcg(dst + j, make_float4(__uint_as_float(a[4 * j]), __uint_as_float(a[4 * j + 1]),
-                                        __uint_as_float(a[4 * j + 2]),
-                                        __uint_as_float(a[4 * j + 3])));
+            __stcg(dst + (EPI == GEMM_DW ? j : 32 * j),
+                   make_float4(__uint_as_float(a[4 * j]), __uint_as_float(a[4 * j + 1]),
+                               __uint_as_float(a[4 * j + 2]), __uint_as_float(a[4 * j + 3])));
+        }
+        if (EPI == GEMM_FWD || EPI == GEMM_DX) {
+          // the last of the tile's slices to finish this warp's region adds
+          // the partials in slice order and applies the epilogue
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cluster(acc_empty_lead + 8u * b);  // accumulator released
+          __threadfence();
+          __syncwarp();
+          unsigned long long done = 0;
+          if (lane == 0) {
+            unsigned long long* ctr =
+                p.tail_ctr + (static_cast<long long>(jt) * 2 + rank) * EW + (warp - 2);
+            unsigned long long assumed = 0ull, nv;
+            while (true) {  // at most tail_splits + 1 tries: each failure sees another slice's count
+              nv = (assumed >> 16) == p.tail_tag ? assumed + 1ull : ((p.tail_tag << 16) | 1ull);
+              const unsigned long long prev = atomicCAS(ctr, assumed, nv);
+              if (prev == assumed) break;
+              assumed = prev;
+            }
+            done = nv & 0xFFFFull;
+          }
+          done = __shfl_sync(0xffffffffu, done, 0);
+          if (done == static_cast<unsigned long long>(p.tail_splits)) {
+            __threadfence();
+            const float* src0 = p.part + static_cast<long long>(jt) * 65536LL + blk0;
+            const long long sstride = static_cast<long long>(p.tail_tiles) * 65536LL;
+#pragma unroll 1
+            for (int cc = 0; cc < HALF / 32; ++cc) {
+              const int gn0 = nbase + cc * 32;
+              float f[32];
+#pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                const float4 v = __ldcg(reinterpret_cast<const float4*>(src0 + cc * 1024) + 32 * j + lane);
+                f[4 * j] = v.x;
+                f[4 * j + 1] = v.y;
+                f[4 * j + 2] = v.z;
+                f[4 * j + 3] = v.w;
+              }
+#pragma unroll 1
+              for (int sl = 1; sl < p.tail_splits; ++sl) {
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                  const float4 v = __ldcg(
+                      reinterpret_cast<const float4*>(src0 + sl * sstride + cc * 1024) + 32 * j + lane);
+                  f[4 * j] = __fadd_rn(f[4 * j], v.x);
+                  f[4 * j + 1] = __fadd_rn(f[4 * j + 1], v.y);
+                  f[4 * j + 2] = __fadd_rn(f[4 * j + 2], v.z);
+                  f[4 * j + 3] = __fadd_rn(f[4 * j + 3], v.w);
+                }
+              }
+              // every slice's block of this chunk is read: drop its lines
+              // from L2 so that they are never written back
+              __syncwarp();
+#pragma unroll 1
+              for (int sl = 0; sl < p.tail_splits; ++sl)
+                l2_discard_line(src0 + sl * sstride + cc * 1024 + lane * 32);
+              if (gn0 >= p.N || !row_ok) continue;
+              uint32_t a[32];
+#pragma unroll
+              for (int i = 0; i < 32; ++i) a[i] = __float_as_uint(f[i]);
+              if (EPI == GEMM_FWD) epi_fwd(p, gm, gn0, a_t, a, a, false);  // no running sums
+              else epi_dx(p, gm, gn0, a);
+            }
+          }
+          continue;  // the accumulator is already released
         }
       } else if (EPI == GEMM_DW) {
         // the first half-chunk of this warp's next unit, if a whole tile,
@@ -1168,6 +1257,36 @@ TailPlan tail_plan(int M, int N, int Kred, int clusters) {
   return t;
 }
 
+// Forward / dX tail workspace: the slice counters (2 CTA ranks x 8 epilogue
+// warps per tail tile, tail <= clusters) in the first kTailCtrBytes, then the
+// partials (tail * splits <= clusters tiles of 256 x 256 floats).
+constexpr size_t kTailCtrBytes = 16384;
+
+// The tail partials start on a 256-byte boundary inside the workspace (the
+// consumers discard each 128-byte line from L2 once read, which must not
+// touch a neighbour's bytes); the size functions leave 256 bytes for it.
+static float* tail_partials(void* ws, size_t ctr) {
+  const uintptr_t a = reinterpret_cast<uintptr_t>(ws) + ctr;
+  return reinterpret_cast<float*>((a + 255) & ~static_cast<uintptr_t>(255));
+}
+
+// A forward or dX GEMM cuts its last wave only when the reduction is at
+// least 4096 long: a slice's fixed costs (its pipeline fill, the partials'
+// round trip through L2, the fix-up) are ~10 us, which a cut of a 2048-long
+// reduction (~12 us of tile) does not win back.
+constexpr int kTailMinKb = 4096 / BK;
+
+size_t gemm_tail_bytes(int M, int N, int Kred) {
+  if ((Kred + BK - 1) / BK < kTailMinKb) return 0;
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const TailPlan tp = tail_plan(M, N, Kred, sms / 2);
+  // any launch's plan has tail * splits <= its clusters <= sms / 2
+  return tp.splits >= 2 ? kTailCtrBytes + 256 + static_cast<size_t>(sms / 2) * 65536 * sizeof(float)
+                        : 0;
+}
+
 // Token slices for a 2-SM dW GEMM whose output tiles would leave most SM
 // pairs idle: enough slices to give every pair a unit of work, each slice at
 // least 4 k-blocks (256 tokens) long, at most 32 slices.
@@ -1226,16 +1345,28 @@ int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStr
   p.tail_kbps = p.num_kb;
   p.part = nullptr;
   if (plan) *plan = TailPlan{0, 0, 0, 0, 0};
-  if (EPI == GEMM_DW && tail_ws && plan && p.splits == 1) {
+  if ((EPI == GEMM_DW || ((EPI == GEMM_FWD || EPI == GEMM_DX) && !DR && p.num_kb >= kTailMinKb)) &&
+      tail_ws && plan && p.splits == 1) {
     const TailPlan tp = tail_plan(p.M, p.N, p.Kred, max_clusters);
-    if (tp.splits >= 2 && tp.bytes <= tail_ws_bytes) {
+    const size_t ctr = EPI == GEMM_DW ? 0 : kTailCtrBytes;
+    static_assert(2 * 8 * 8 * 128 <= kTailCtrBytes, "slice counters: 128 tail tiles");
+    float* part = tail_partials(tail_ws, ctr);
+    const size_t used = static_cast<size_t>(reinterpret_cast<uint8_t*>(part) -
+                                            static_cast<uint8_t*>(tail_ws)) + tp.bytes;
+    if (tp.splits >= 2 && tp.tail <= 128 && used <= tail_ws_bytes) {
       p.full_units = tp.full;
       p.full_tiles = tp.full;
       p.tail_tiles = tp.tail;
       p.tail_splits = tp.splits;
       p.tail_kbps = tp.kbps;
-      p.part = static_cast<float*>(tail_ws);
+      p.part = part;
       p.num_tiles = tp.full + tp.tail * tp.splits;
+      if (EPI != GEMM_DW) {
+        static std::atomic<unsigned long long> tag{0};
+        p.tail_ctr = static_cast<unsigned long long*>(tail_ws);
+        p.tail_tag = (tag.fetch_add(1) + 1) & 0xFFFFFFFFFFFFull;  // 48 bits, never 0
+        if (p.tail_tag == 0) p.tail_tag = 1;
+      }
       *plan = tp;
     }
   }
@@ -1304,7 +1435,12 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
         return launch_tiles<128, false, false, GEMM_FWD, true>(ta, tb, p, stream);
       }
       if (!make_map(&tb, g.B, g.Kred, g.N, BK, g2.pair ? 128 : 256)) return 3;
-      if (g2.pair) return launch_pairs<false, false, GEMM_FWD>(ta, tb, p, stream);
+      if (g2.pair) {
+        // with a workspace, the last wave's tiles as reduction slices
+        TailPlan tp{0, 0, 0, 0, 0};
+        return launch_pairs<false, false, GEMM_FWD>(ta, tb, p, stream, g.ws, g.ws_bytes,
+                                                    g.ws ? &tp : nullptr);
+      }
       return launch_tiles<256, false, false, GEMM_FWD, false>(ta, tb, p, stream);
     case GEMM_FWD8:
       // 2-SM tiles whatever the tiling mode: E4M3 rows of 128 elements
@@ -1314,7 +1450,11 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
     case GEMM_DX:
       if (!make_map(&ta, g.A, g.Kred, g.M, BK, BM)) return 3;
       if (!make_map(&tb, g.B, g.N, g.Kred, 64, BK)) return 3;
-      if (g2.pair) return launch_pairs<false, true, GEMM_DX>(ta, tb, p, stream);
+      if (g2.pair) {
+        TailPlan tp{0, 0, 0, 0, 0};
+        return launch_pairs<false, true, GEMM_DX>(ta, tb, p, stream, g.ws, g.ws_bytes,
+                                                  g.ws ? &tp : nullptr);
+      }
       return launch_tiles<256, false, true, GEMM_DX, false>(ta, tb, p, stream);
     case GEMM_DW: {
       if (!make_map(&ta, g.A, g.M, g.Kred, 64, BK)) return 3;
@@ -1335,7 +1475,7 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
                       : launch_pairs<true, true, GEMM_DW>(ta, tb, p, stream, g.ws, g.ws_bytes,
                                                           &tp));
         if (rc || tp.splits == 0) return rc;
-        return launch_tail_update(static_cast<const float*>(g.ws), tp.splits, tp.tail, tp.full,
+        return launch_tail_update(tail_partials(g.ws, 0), tp.splits, tp.tail, tp.full,
                                   (g.N + 255) / 256, g.M, g.N, g.W, g.packed, g.m, g.v, g.uc,
                                   g.uc_dev, g.changed, g.dW_out, stream);
       }

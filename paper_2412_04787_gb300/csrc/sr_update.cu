@@ -232,6 +232,12 @@ __global__ void __launch_bounds__(kThreads, 3)
         __stcs(reinterpret_cast<float4*>(v + e), v4);
       }
     }
+    // the slices' 128-byte lines of these 32 columns (eight lanes' groups)
+    // are read: drop them from L2 so that they are never written back
+    __syncwarp();
+    if ((threadIdx.x & 7) == 0 && cur.e >= 0)
+      for (int s = 0; s < splits; ++s)
+        asm volatile("discard.global.L2 [%0], 128;" ::"l"(cur.src + s * sstride) : "memory");
     cur = nxt;
   }
   if (changed) {

@@ -34,6 +34,7 @@ EXPORTED = [
     "dqt_act_quant_images", "dqt_bitlinear_fwd_img", "dqt_bitlinear_bwd_dx_img",
     "dqt_bwd_dx_workspace_size", "dqt_bitlinear_bwd_dw_update_img",
     "dqt_bwd_dw_img_workspace_size", "dqt_codes_to_xdq", "dqt_fwd_workspace_size",
+    "dqt_fwd_img_workspace_size", "dqt_bwd_dx_img_workspace_size",
 ]
 
 
@@ -96,11 +97,16 @@ def lib():
         L.dqt_fwd_workspace_size.argtypes = [_i64, _i64, _i64]
         L.dqt_fwd_workspace_size.restype = _sz
         L.dqt_bitlinear_fwd_img.argtypes = [_vp, _vp, _vp, _f32, dqt_grid_t, _i64, _i64, _i64,
-                                            _vp, _vp, _vp]
+                                            _vp, _vp, _vp, _sz, _vp]
+        L.dqt_fwd_img_workspace_size.argtypes = [_i64, _i64, _i64]
+        L.dqt_fwd_img_workspace_size.restype = _sz
         L.dqt_bitlinear_bwd_dx.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp, _sz, _vp]
-        L.dqt_bitlinear_bwd_dx_img.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp]
-        L.dqt_bwd_dx_workspace_size.argtypes = [_i64, _i64]
+        L.dqt_bitlinear_bwd_dx_img.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp, _sz,
+                                               _vp]
+        L.dqt_bwd_dx_workspace_size.argtypes = [_i64, _i64, _i64]
         L.dqt_bwd_dx_workspace_size.restype = _sz
+        L.dqt_bwd_dx_img_workspace_size.argtypes = [_i64, _i64, _i64]
+        L.dqt_bwd_dx_img_workspace_size.restype = _sz
         L.dqt_bitlinear_bwd_dw_update.argtypes = [_vp, _vp, _vp, _vp, _f32, _vp, _vp,
                                                   C.POINTER(dqt_adamw_t), C.POINTER(dqt_sr_t),
                                                   dqt_grid_t, _i64, _i64, _i64, _vp, _vp, _vp,
@@ -162,7 +168,8 @@ def lib():
             if name not in ("dqt_status_string", "dqt_absmean_workspace_size",
                             "dqt_update_consts_size", "dqt_bwd_dw_workspace_size",
                             "dqt_bwd_dw_img_workspace_size", "dqt_bwd_dx_workspace_size",
-                            "dqt_fwd_workspace_size",
+                            "dqt_fwd_workspace_size", "dqt_fwd_img_workspace_size",
+                            "dqt_bwd_dx_img_workspace_size",
                             "dqt_adafactor_workspace_size",
                             "dqt_bwd_dw_adafactor_workspace_size",
                             "dqt_rmsnorm_bwd_workspace_size"):
@@ -352,8 +359,26 @@ def dqt_bitlinear_fwd(Xq, s_x, W, s_w, bits_or_grid, Y=None, acc_out=None, ws=No
     return Y
 
 
+def _tail_workspace(need, device, ws):
+    """Optional workspace of the GEMM calls whose last wave may be cut into
+    slices: None allocates the `need` bytes, False passes none."""
+    if ws is False or need == 0:
+        return None, 0
+    if ws is None:
+        ws = torch.empty(need, dtype=torch.uint8, device=device)
+    _need(ws, "ws", torch.uint8)
+    return ws, ws.numel()
+
+
+def dqt_fwd_img_workspace_size(T, K, N):
+    return int(lib().dqt_fwd_img_workspace_size(T, K, N))
+
+
 def dqt_bitlinear_fwd_img(Xq_img, s_x, W_img, s_w, bits_or_grid, Y=None, acc_out=None,
-                          stream=None):
+                          ws=None, stream=None):
+    """The forward on the bf16 operand images; `ws` (uint8 CUDA tensor of
+    dqt_fwd_img_workspace_size bytes) holds last-wave slice partials:
+    allocated if None, none if False."""
     _need(Xq_img, "Xq_img", torch.bfloat16)
     T, K = Xq_img.shape
     _need(W_img, "W_img", torch.bfloat16)
@@ -364,14 +389,19 @@ def dqt_bitlinear_fwd_img(Xq_img, s_x, W_img, s_w, bits_or_grid, Y=None, acc_out
         Y = torch.empty((T, N), dtype=torch.bfloat16, device=Xq_img.device)
     _need(Y, "Y", torch.bfloat16, (T, N))
     _opt(acc_out, "acc_out", torch.int32, (T, N))
+    ws, nws = _tail_workspace(lib().dqt_fwd_img_workspace_size(T, K, N), Xq_img.device, ws)
     _check(lib().dqt_bitlinear_fwd_img(_ptr(Xq_img), _ptr(s_x), _ptr(W_img), float(s_w),
                                        _grid(bits_or_grid), T, K, N, _ptr(Y), _ptr(acc_out),
-                                       _stream(stream)), "dqt_bitlinear_fwd_img")
+                                       _ptr(ws), nws, _stream(stream)), "dqt_bitlinear_fwd_img")
     return Y
 
 
-def dqt_bwd_dx_workspace_size(N, K):
-    return int(lib().dqt_bwd_dx_workspace_size(N, K))
+def dqt_bwd_dx_workspace_size(T, N, K):
+    return int(lib().dqt_bwd_dx_workspace_size(T, N, K))
+
+
+def dqt_bwd_dx_img_workspace_size(T, N, K):
+    return int(lib().dqt_bwd_dx_img_workspace_size(T, N, K))
 
 
 def dqt_bitlinear_bwd_dx(dY, W, s_w, dX=None, ws=None, stream=None):
@@ -386,7 +416,7 @@ def dqt_bitlinear_bwd_dx(dY, W, s_w, dX=None, ws=None, stream=None):
     if dX is None:
         dX = torch.empty((T, K), dtype=torch.bfloat16, device=dY.device)
     _need(dX, "dX", torch.bfloat16, (T, K))
-    nws = lib().dqt_bwd_dx_workspace_size(N, K)
+    nws = lib().dqt_bwd_dx_workspace_size(T, N, K)
     if ws is None:
         ws = torch.empty(nws, dtype=torch.uint8, device=dY.device)
     _need(ws, "ws", torch.uint8)
@@ -396,7 +426,9 @@ def dqt_bitlinear_bwd_dx(dY, W, s_w, dX=None, ws=None, stream=None):
     return dX
 
 
-def dqt_bitlinear_bwd_dx_img(dY, W_img, s_w, dX=None, stream=None):
+def dqt_bitlinear_bwd_dx_img(dY, W_img, s_w, dX=None, ws=None, stream=None):
+    """dX on the weight's bf16 image; `ws` as for dqt_bitlinear_fwd_img
+    (dqt_bwd_dx_img_workspace_size bytes)."""
     _need(dY, "dY", torch.bfloat16)
     T, N = dY.shape
     _need(W_img, "W_img", torch.bfloat16)
@@ -405,8 +437,10 @@ def dqt_bitlinear_bwd_dx_img(dY, W_img, s_w, dX=None, stream=None):
     if dX is None:
         dX = torch.empty((T, K), dtype=torch.bfloat16, device=dY.device)
     _need(dX, "dX", torch.bfloat16, (T, K))
+    ws, nws = _tail_workspace(lib().dqt_bwd_dx_img_workspace_size(T, N, K), dY.device, ws)
     _check(lib().dqt_bitlinear_bwd_dx_img(_ptr(dY), _ptr(W_img), float(s_w), T, N, K,
-                                          _ptr(dX), _stream(stream)), "dqt_bitlinear_bwd_dx_img")
+                                          _ptr(dX), _ptr(ws), nws, _stream(stream)),
+           "dqt_bitlinear_bwd_dx_img")
     return dX
 
 

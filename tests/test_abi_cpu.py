@@ -69,22 +69,41 @@ def test_argument_validation_without_launch(L):
     assert L.dqt_bitlinear_bwd_dx(A, A, 1.0, 4, 8, 8, A, None, 1 << 20, None) == dqt.DQT_ERR_ARG
     assert L.dqt_act_quant(A, 4, 8, None, A, None) == dqt.DQT_ERR_ARG
     assert L.dqt_act_quant_images(A, 4, 8, None, A, None, None, None) == dqt.DQT_ERR_ARG
-    assert L.dqt_bitlinear_fwd_img(None, A, A, 1.0, g, 4, 8, 8, A, None, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_fwd_img(None, A, A, 1.0, g, 4, 8, 8, A, None, None, 0, None) == dqt.DQT_ERR_ARG
     # sizes
     assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g, 0, 8, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ARG
     assert L.dqt_act_quant(A, -1, 8, A, A, None) == dqt.DQT_ERR_ARG
     # the dX workspace must hold the weight's bf16 image
-    assert L.dqt_bwd_dx_workspace_size(8, 8) >= 8 * 8 * 2
+    assert L.dqt_bwd_dx_workspace_size(4, 8, 8) >= 8 * 8 * 2
     assert L.dqt_bitlinear_bwd_dx(A, A, 1.0, 4, 8, 8, A, A, 64, None) == dqt.DQT_ERR_ARG
     # K, N multiples of 8 and 16-byte alignment; the forward's workspace holds
     # both operands' bf16 images
     assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g, 4, 12, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ALIGN
     assert L.dqt_fwd_workspace_size(4, 8, 8) >= (4 + 8) * 8 * 2
     assert L.dqt_bitlinear_fwd(A, A, A, 1.0, g, 4, 8, 8, A, None, A, 16, None) == dqt.DQT_ERR_ARG
-    assert L.dqt_bitlinear_fwd_img(A, A, A, 1.0, g, 4, 12, 8, A, None, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_bitlinear_fwd_img(A, A, A, 1.0, g, 4, 12, 8, A, None, None, 0, None) == dqt.DQT_ERR_ALIGN
     assert L.dqt_bitlinear_bwd_dx(A, A, 1.0, 4, 8, 20, A, A, 1 << 20, None) == dqt.DQT_ERR_ALIGN
-    assert L.dqt_bitlinear_bwd_dx_img(A, A, 1.0, 4, 8, 20, A, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_bitlinear_bwd_dx_img(A, A, 1.0, 4, 8, 20, A, None, 0, None) == dqt.DQT_ERR_ALIGN
     assert L.dqt_bitlinear_fwd(_p(0x10004), A, A, 1.0, g, 4, 8, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ALIGN
+    # the forward's and dX's optional workspace for last-wave slice partials:
+    # when a cut is planned (a shape whose tiles leave the last wave short),
+    # a workspace below the size, or misaligned, is refused before any launch
+    # (8192 x 2048 outputs: 256 pair tiles, 3.4 waves on 74 or 76 SM pairs)
+    T, K, N = 8192, 5632, 2048
+    need = L.dqt_fwd_img_workspace_size(T, K, N)
+    assert need > 0
+    assert L.dqt_bitlinear_fwd_img(A, A, A, 1.0, g, T, K, N, A, None, A, need - 16, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_fwd_img(A, A, A, 1.0, g, T, K, N, A, None, _p(0x10008), need, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_fwd_workspace_size(T, K, N) >= (T + N) * K * 2 + need
+    T, N, K = 8192, 5632, 2048
+    need = L.dqt_bwd_dx_img_workspace_size(T, N, K)
+    assert need > 0
+    assert L.dqt_bitlinear_bwd_dx_img(A, A, 1.0, T, N, K, A, A, need - 16, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bwd_dx_workspace_size(T, N, K) >= N * K * 2 + need
+    # one pair tile, or a reduction shorter than 4096: nothing to cut
+    assert L.dqt_fwd_img_workspace_size(256, 512, 256) == 0
+    assert L.dqt_fwd_img_workspace_size(8192, 2048, 5632) == 0
+    assert L.dqt_bwd_dx_img_workspace_size(8192, 2048, 5632) == 0
     # bad grid / scale
     assert L.dqt_bitlinear_fwd(A, A, A, 1.0, dqt.dqt_grid_t(2, 1), 4, 8, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ARG
     assert L.dqt_bitlinear_fwd(A, A, A, 1.0, dqt.dqt_grid_t(-129, 1), 4, 8, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ARG
