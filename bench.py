@@ -80,6 +80,9 @@ def kernel_fingerprint(files=GEMM_SOURCES):
 # of operand and optimiser-state bytes), from one ncu capture, keyed by the
 # GEMM-source fingerprint it was taken on (see profiles/).  A stale entry
 # reports null.
+# With gate and up stacked, the mean over the step's two dW launches (the
+# stacked gate/up call and the down call, each its GEMM and streaming kernel).
+DW_TRAFFIC_STACKED = {}
 DW_TRAFFIC_BYTES = {"ac36c0aa63c5": 261135360 + 57050112 + 33049600,
                     "82d12725fdfa": 262571008 + 61169152 + 33047808,
                     "a25cf8632190": 261430272 + 59386112 + 33048064}
@@ -155,7 +158,7 @@ class MLPStep:
     """Device buffers and the launch sequence of one DQT MLP training step."""
 
     def __init__(self, dev, seed=1234, fp8=False, optimizer="adamw", packed=False, bits=1.58,
-                 operands="int8", tail_slices=True):
+                 operands="int8", tail_slices=True, stack_gate_up=False):
         from paper_2412_04787_gb300 import dqt, inputs
 
         self.dqt = dqt
@@ -169,6 +172,11 @@ class MLPStep:
         # *_img calls on images shared between GEMMs (the FP8, packed and
         # Adafactor variants always take images)
         self.i8 = operands == "int8" and not fp8 and not packed and optimizer == "adamw"
+        # gate and up as two stacked weights of one call (the forward and the
+        # fused dW + update; dX stays per weight): image operands, AdamW, int8
+        # codes
+        self.stack = (stack_gate_up and not self.i8 and not fp8 and not packed
+                      and optimizer == "adamw")
         self.grid = dqt.grid(bits)
         T = T_TOK
         # two seeded input sets, alternated step by step, so that the
@@ -180,17 +188,41 @@ class MLPStep:
             for i, (name, K, N) in enumerate(PROJ):
                 h["dY_" + name] = inputs.normal((T, N), 1e-2, seed=10 + i + 100 * r,
                                                 dtype=torch.bfloat16)
+            if self.stack:
+                # the gradient of the stacked output [gate | up] as a SwiGLU
+                # backward writes it; the dX GEMMs read each half in place
+                h["dY_gu"] = torch.cat([h.pop("dY_gate"), h.pop("dY_up")], dim=1)
             self.host_sets.append(h)
         self.host = self.host_sets[0]
         self.dev_sets = [{k: v.to(dev) for k, v in h.items()} for h in self.host_sets]
+        if self.stack:
+            for d in self.dev_sets:
+                d["dY_gate"], d["dY_up"] = d["dY_gu"][:, :INTER], d["dY_gu"][:, INTER:]
         self.d = self.dev_sets[0]
         self.alternate = True
         self.W, self.s_w, self.m, self.v, self.W_img, self.Y, self.dX, self.Xdq = {}, {}, {}, {}, {}, {}, {}, {}
         self.W8 = {}
+        if self.stack:
+            # one buffer of codes, moments and image for both weights; each
+            # weight's own per-tensor scale
+            self.W_gu = torch.empty((2 * INTER, HID), dtype=torch.int8, device=dev)
+            self.m_gu = torch.zeros((2 * INTER, HID), dtype=torch.float32, device=dev)
+            self.v_gu = torch.zeros((2 * INTER, HID), dtype=torch.float32, device=dev)
+            self.W_img_gu = torch.empty((2 * INTER, HID), dtype=torch.bfloat16, device=dev)
+            self.Y_gu = torch.empty((T, 2 * INTER), dtype=torch.bfloat16, device=dev)
         for i, (name, K, N) in enumerate(PROJ):
             W0 = inputs.normal((N, K), 0.02, seed=20 + i).to(dev)
             self.W[name], self.s_w[name] = dqt.dqt_absmean_init(W0, self.grid)
             del W0
+            if self.stack and name in ("gate", "up"):
+                half = slice(0, INTER) if name == "gate" else slice(INTER, 2 * INTER)
+                self.W_gu[half].copy_(self.W[name])
+                self.W[name] = self.W_gu[half]
+                self.m[name], self.v[name] = self.m_gu[half], self.v_gu[half]
+                self.W_img[name] = self.W_img_gu[half]
+                self.Y[name] = self.Y_gu[:, half]
+                self.dX[name] = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
+                continue
             if packed:
                 self.W[name] = dqt.dqt_pack_ternary(self.W[name])
             if optimizer == "adamw":
@@ -254,6 +286,15 @@ class MLPStep:
         # (the forward's and dX's cut last wave is summed inside the GEMM: no
         # launch of its own)
         self.launches_per_step = 2 + 3 + 3 + 3 + sum(dw) + (3 if fp8 else 0) + (6 if self.i8 else 0)
+        if self.stack:
+            # one weight image, one forward and one dW call for gate and up
+            nbp = dqt.dqt_bwd_dw_img_workspace_size(T, 2 * INTER, HID)
+            self.launches_per_step = (2 + 2 + 2 + 3 + (1 + (1 if nbp > 0 else 0)) + dw[2])
+            if nbp > max(nbw, 16):
+                self.dw_ws = [torch.empty(nbp, dtype=torch.uint8, device=dev) for _ in range(4)]
+            nbt = max(nbt, dqt.dqt_fwd_img_workspace_size(T, HID, 2 * INTER))
+            self.tail_ws = [torch.empty(max(nbt, 16), dtype=torch.uint8, device=dev)
+                            if nbt and tail_slices else False for _ in range(4)]
         self.dw_kind = "bwd_dw_adafactor" if optimizer == "adafactor" else "bwd_dw_update"
         if self.i8:
             self.kinds = ["act_quant", "codes_to_bf16", "fwd", "bwd_dx", "codes_to_xdq",
@@ -339,6 +380,10 @@ class MLPStep:
                       lambda: dqt.dqt_act_quant_images(self.d[src], None, s_x, q_img, xdq, want=()))
 
         def codes(name, stream):
+            if name == "gate_up":  # both stacked weights' image in one launch
+                timed("codes_to_bf16", stream,
+                      lambda: dqt.dqt_codes_to_bf16(self.W_gu, self.W_img_gu))
+                return
             shape = tuple(self.W_img[name].shape)
             if self.fp8:
                 timed("codes_to_fp8", stream,
@@ -350,6 +395,11 @@ class MLPStep:
 
         def fwd(name, stream):
             s_x, q_img, _ = self.aq["H" if name == "down" else "X"]
+            if name == "gate_up":  # the stacked weights, [gate | up] in one output
+                timed("fwd", stream, lambda: dqt.dqt_bitlinear_fwd_img_pair(
+                    q_img, s_x, self.W_img_gu, INTER, self.s_w["gate"], self.s_w["up"], self.grid,
+                    Y=self.Y_gu, ws=self.tail_ws[s.index(stream)]))
+                return
             if self.i8:
                 ws = self.fwd_ws[s.index(stream)]
                 if parts:
@@ -399,6 +449,13 @@ class MLPStep:
         def dw(i, name, stream):
             xdq = self.aq["H" if name == "down" else "X"][2]
             ch = self.changed[i:i + 1]
+            if name == "gate_up":  # the stacked weights, each with its scale and stream
+                ws = self.dw_ws[s.index(stream)]
+                timed(self.dw_kind, stream, lambda: dqt.dqt_bitlinear_bwd_dw_update_img_pair(
+                    self.d["dY_gu"], xdq, self.W_gu, INTER, self.s_w["gate"], self.s_w["up"],
+                    self.m_gu, self.v_gu, hp, self.sr["gate"], self.sr["up"], self.grid,
+                    changed_out=ch, ws=ws))
+                return
             if self.dp and not self.i8:
                 upd = self.dp[name]
                 ws = self.dw_ws[s.index(stream)]
@@ -471,14 +528,20 @@ class MLPStep:
         # the weight gradient reads: splitting it into two passes, the second
         # beside the forward GEMMs, was measured slower)
         aq("X", s[0])
-        if not self.i8:
-            codes("gate", s[1])
-            codes("up", s[2])
+        if self.stack:
+            codes("gate_up", s[1])
             codes("down", s[3])
-        after(s[1], s[0])
-        after(s[2], s[0])
-        fwd("gate", s[1])
-        fwd("up", s[2])
+            after(s[1], s[0])
+            fwd("gate_up", s[1])
+        else:
+            if not self.i8:
+                codes("gate", s[1])
+                codes("up", s[2])
+                codes("down", s[3])
+            after(s[1], s[0])
+            after(s[2], s[0])
+            fwd("gate", s[1])
+            fwd("up", s[2])
         after(s[0], s[1])
         after(s[2], s[0], s[1], s[3])
         aq("H", s[2])
@@ -495,10 +558,15 @@ class MLPStep:
                 st.wait_event(dx_down)
         # each weight-gradient GEMM is enqueued ahead of its dX: the longer
         # kernel then takes the SMs first and the dX kernels fill its last wave
-        dw(0, "gate", s[1])
-        dx("gate", s[0])
-        dw(1, "up", s[3])
-        dx("up", s[2])
+        if self.stack:
+            dw(0, "gate_up", s[1])
+            dx("gate", s[0])
+            dx("up", s[2])
+        else:
+            dw(0, "gate", s[1])
+            dx("gate", s[0])
+            dw(1, "up", s[3])
+            dx("up", s[2])
         for st in s:
             after(main, st)
 
@@ -508,6 +576,9 @@ class MLPStep:
         flops = {"fwd": [2.0 * T * K * N for _, K, N in PROJ]}
         flops["bwd_dx"] = list(flops["fwd"])
         flops["bwd_dw_update"] = list(flops["fwd"])
+        if self.stack:  # gate and up in one forward and one dW call
+            flops["fwd"] = [2.0 * T * HID * 2 * INTER, 2.0 * T * INTER * HID]
+            flops["bwd_dw_update"] = list(flops["fwd"])
         flops["bwd_dw_adafactor"] = list(flops["fwd"])
         flops["bwd_dw"] = list(flops["fwd"])  # gradient only (data-parallel exchange)
         flops["fwd_fp8"] = list(flops["fwd"])
@@ -532,6 +603,7 @@ class MLPStep:
             # forward and dX), and with int8 operands each forward's activation image
             "codes_to_bf16": ([3.0 * K * N for _, K, N in PROJ] * 2 +
                               [3.0 * T * K for _, K, N in PROJ]) if self.i8 else
+                             [3.0 * HID * 2 * INTER, 3.0 * INTER * HID] if self.stack else
                              [(2.25 if self.packed else 3.0) * K * N for _, K, N in PROJ],
             "codes_to_fp8": [(1.25 if self.packed else 2.0) * K * N for _, K, N in PROJ],
             # int8 codes read, bf16 image written, s_x read (gate, up: X; down: H)
@@ -619,7 +691,8 @@ def run_gpu(args):
     from paper_2412_04787_gb300 import build as dqt_build
     dqt_build.build()
     st = MLPStep(dev, fp8=args.act == "fp8", optimizer=args.optimizer, packed=args.packed,
-                 bits=args.bits, operands=args.operands, tail_slices=not args.no_tail_slices)
+                 bits=args.bits, operands=args.operands, tail_slices=not args.no_tail_slices,
+                 stack_gate_up=stacked_gate_up(args, dp_mode))
     if dp_mode == "exchange":
         st.enable_dp()
     dqt = st.dqt
@@ -700,10 +773,13 @@ def run_gpu(args):
                               % (which, pk_kind, serial_ms_total)),
                 "timing": "mean CUDA-event duration of its launches over a second timed region "
                           "of the same K steps run serially on one stream (%.4f ms/step)" % serial_ms_step,
-                "traffic": (DW_TRAFFIC_BYTES.get(kernel_fingerprint())
+                "traffic": ((DW_TRAFFIC_STACKED if st.stack else DW_TRAFFIC_BYTES)
+                            .get(kernel_fingerprint())
                             if dom == "bwd_dw_update" and not st.packed else None),
                 "kernel_fingerprint": kernel_fingerprint(),
-                "algorithmic_per_launch": "2*T*K*N FLOP (T=8192; K,N = 2048,5632 / 5632,2048)"}
+                "algorithmic_per_launch": ("2*T*K*N FLOP (T=8192; gate and up stacked: K,N = "
+                                           "2048,11264; down: 5632,2048)" if st.stack else
+                                           "2*T*K*N FLOP (T=8192; K,N = 2048,5632 / 5632,2048)")}
     kern = {}
     for k in kinds:
         d = dict(per[k])
@@ -825,7 +901,7 @@ def run_gpu(args):
                     % ("ternary" if st.bits == 1.58 else "%d-bit" % st.bits),
             "config": mlp_config(bits=st.bits, fp8=st.fp8, optimizer=st.optimizer,
                                  packed=st.packed, i8=st.i8,
-                                 parallelism=_parallelism(ws, dp_mode)),
+                                 parallelism=_parallelism(ws, dp_mode), stacked=st.stack),
             "roofline": roofline, "kernels": kern, "e2e": e2e,
             "gpu_launches": st.launches_per_step * args.steps,
             "clocks": clk.summary(), "cpu_baseline": cpu,
@@ -977,7 +1053,16 @@ def cpu_baseline(seconds=15.0):
                                   "sample": "the whole single-layer step, not sampled"}}
 
 
-def mlp_config(bits=1.58, fp8=False, optimizer="adamw", packed=False, i8=True, parallelism=None):
+def stacked_gate_up(args, dp_mode="replicas"):
+    """Whether the MLP step runs gate and up as two stacked weights (one
+    forward call, one dW + update call; MLPStep's condition; the data-parallel
+    exchange keeps one weight per exchange)."""
+    return (not args.separate_gate_up and args.operands == "img" and args.act != "fp8"
+            and not args.packed and args.optimizer == "adamw" and dp_mode != "exchange")
+
+
+def mlp_config(bits=1.58, fp8=False, optimizer="adamw", packed=False, i8=True, parallelism=None,
+               stacked=False):
     """The `config` of the MLP step's JSON line (both arms)."""
     wname = "ternary" if bits == 1.58 else "%d-bit" % bits
     return {"workload": (WORKLOAD if bits == 1.58 else WORKLOAD.replace("ternary", wname)) +
@@ -989,6 +1074,9 @@ def mlp_config(bits=1.58, fp8=False, optimizer="adamw", packed=False, i8=True, p
             "optimizer": optimizer,
             "operands": "int8 codes through the C ABI" if i8 else "bf16 / E4M3 operand images",
             "parallelism": parallelism or "single GPU",
+            "gate_up": ("two weights stacked in one forward call and one dW + update call, each "
+                        "with its own scale and SR stream; dX per weight" if stacked else
+                        "separate calls"),
             "l2": "inputs larger than L2 (step working set ~1.5 GB > 129 MB)"}
 
 
@@ -1032,7 +1120,8 @@ def run_reference(args):
         "vs_baseline": None, "dtype": "f64/f32 (oracle)", "data": "synthetic",
         "config": mlp_config(bits=args.bits, fp8=args.act == "fp8", optimizer=args.optimizer,
                              packed=args.packed, i8=args.operands == "int8",
-                             parallelism=_parallelism(ws, dp_mode)),
+                             parallelism=_parallelism(ws, dp_mode),
+                             stacked=stacked_gate_up(args, dp_mode)),
         "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": pool.cores,
                          "nproc": os.cpu_count(), "kind": "oracle",
                          "sample": "each step: %d processes at once, each %d token rows of "
@@ -1521,6 +1610,11 @@ def main():
     ap.add_argument("--impl", default="dqt", choices=["dqt", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--separate-gate-up", action="store_true",
+                    help="mlp: gate and up as two separate calls each (by default, with image "
+                         "operands and AdamW on int8 codes, they are two stacked weights of one "
+                         "forward call and one dW + update call, each weight with its own scale "
+                         "and SR stream; dX per weight)")
     ap.add_argument("--no-tail-slices", action="store_true",
                     help="the forward and dX GEMMs without a workspace, so their last wave is "
                          "not cut into reduction slices (A/B of that schedule; image operands)")

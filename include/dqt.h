@@ -231,6 +231,19 @@ int dqt_bitlinear_fwd_img(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf
                           dqt_bf16* Y, int32_t* acc_out, void* ws, size_t ws_bytes,
                           void* stream);
 
+/* Two BitLinear weights that read the same input (a LLaMA MLP's gate and up
+ * projections), stacked along N in one call: W_img [N, K] holds the first
+ * weight's code image in rows [0, N0) and the second's in rows [N0, N), each
+ * with its own per-tensor scale (s_w0, s_w1; Eq. 2-3 apply to each weight
+ * alone).  Y [T, N] receives both outputs side by side: columns [0, N0) are
+ * the first weight's Y and [N0, N) the second's, bit for bit what two
+ * dqt_bitlinear_fwd_img calls write.  N0 a multiple of 256 (whole output
+ * tiles), 0 < N0 < N; ws and everything else as dqt_bitlinear_fwd_img. */
+int dqt_bitlinear_fwd_img_pair(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img,
+                               int64_t N0, float s_w0, float s_w1, dqt_grid_t grid, int64_t T,
+                               int64_t K, int64_t N, dqt_bf16* Y, int32_t* acc_out, void* ws,
+                               size_t ws_bytes, void* stream);
+
 /* Backward w.r.t. the input, no straight-through estimator on the weight
  * (the gradient is taken w.r.t. W_tilde itself, Sec. 3.2):
  *   dX[t,k] = bf16( (sum_n dY[t,n] c[n,k]) * (1 / s_w) )   fp32 accumulation
@@ -253,6 +266,13 @@ size_t dqt_bwd_dx_img_workspace_size(int64_t T, int64_t N, int64_t K);
 int dqt_bitlinear_bwd_dx_img(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, int64_t T,
                              int64_t N, int64_t K, dqt_bf16* dX, void* ws, size_t ws_bytes,
                              void* stream);
+
+/* The same with dY's rows ldy elements apart (ldy >= N, a multiple of 8):
+ * dY may be one weight's columns of a stacked output's gradient (see
+ * dqt_bitlinear_bwd_dw_update_img_pair), read in place. */
+int dqt_bitlinear_bwd_dx_img_ld(const dqt_bf16* dY, int64_t ldy, const dqt_bf16* W_img, float s_w,
+                                int64_t T, int64_t N, int64_t K, dqt_bf16* dX, void* ws,
+                                size_t ws_bytes, void* stream);
 
 /* Backward w.r.t. the weight fused with the DQT update (Sec. 3.2, Sec. 4.1, Eq. 5):
  *   X_tilde = bf16(Xq / s_x)                       the dequantised activation
@@ -303,6 +323,24 @@ int dqt_bitlinear_bwd_dw_update_img(const dqt_bf16* dY, const dqt_bf16* Xdq, int
  * update up to the fp32 summation order of the gradient; it is deterministic
  * for a given shape and device. */
 size_t dqt_bwd_dw_img_workspace_size(int64_t T, int64_t N, int64_t K);
+
+/* The fused weight gradient and update of two stacked weights that read the
+ * same input (see dqt_bitlinear_fwd_img_pair): dY [T, N] holds both outputs'
+ * gradients side by side (columns [0, N0) the first weight's), W, m, v [N, K]
+ * both weights' codes and moments (rows [0, N0) the first's).  Each weight is
+ * updated with its own scale and stochastic-rounding stream: the first with
+ * (s_w0, sr0), the second with (s_w1, sr1), its Philox elements counted from
+ * its own first element, so codes, m and v equal those of two
+ * dqt_bitlinear_bwd_dw_update_img calls computing the same gradients.  N0 a
+ * multiple of 256, 0 < N0 < N; ws of dqt_bwd_dw_img_workspace_size(T, N, K)
+ * bytes or NULL; changed_out counts both weights' changed codes. */
+int dqt_bitlinear_bwd_dw_update_img_pair(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W,
+                                         int64_t N0, float s_w0, float s_w1, float* m, float* v,
+                                         const dqt_adamw_t* hp, const dqt_sr_t* sr0,
+                                         const dqt_sr_t* sr1, dqt_grid_t grid, int64_t T,
+                                         int64_t N, int64_t K, float* dW_out,
+                                         unsigned long long* changed_out, void* ws,
+                                         size_t ws_bytes, void* stream);
 
 /* The AdamW + SR update of dqt_bitlinear_bwd_dw_update for a gradient already
  * in memory (Eq. 5 as a bandwidth-bound stream; 22 bytes per weight):

@@ -290,7 +290,8 @@ static bool fwd_range_ok(dqt_grid_t grid, int64_t K) {
 // chunks whose partial sums stay <= 2^24 (exact in fp32).
 static int fwd_launch(const void* A, const float* s_x, const void* B, float s_w,
                dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y, int32_t* acc_out,
-               void* tail_ws, size_t tail_bytes, void* stream) {
+               void* tail_ws, size_t tail_bytes, void* stream, int split = 0,
+               float s_w1 = 0.0f) {
   const int64_t cmax = grid.qmax > -grid.qmin ? grid.qmax : -grid.qmin;
   const int64_t cm = cmax > 0 ? cmax : 1;
   // Largest chunk whose partial sums stay <= 2^24 (exact in fp32), multiple of 64.
@@ -311,6 +312,8 @@ static int fwd_launch(const void* A, const float* s_x, const void* B, float s_w,
   g.acc_out = acc_out;
   g.ws = tail_ws;
   g.ws_bytes = tail_ws ? tail_bytes : 0;
+  g.split = split;
+  g.scale1 = s_w1;
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
@@ -374,6 +377,28 @@ int dqt_bitlinear_fwd_img(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf
     return DQT_ERR_ALIGN;
   if (!fwd_range_ok(grid, K)) return DQT_ERR_RANGE;
   return fwd_launch(Xq_img, s_x, W_img, s_w, grid, T, K, N, Y, acc_out, ws, ws_bytes, stream);
+}
+
+// Two weights stacked along N that read the same input (rows [0, N0) the
+// first weight's codes with scale s_w0, rows [N0, N) the second's with s_w1).
+static bool pair_split_ok(int64_t N0, int64_t N) { return N0 > 0 && N0 < N && N0 % 256 == 0; }
+
+int dqt_bitlinear_fwd_img_pair(const dqt_bf16* Xq_img, const float* s_x, const dqt_bf16* W_img,
+                               int64_t N0, float s_w0, float s_w1, dqt_grid_t grid, int64_t T,
+                               int64_t K, int64_t N, dqt_bf16* Y, int32_t* acc_out, void* ws,
+                               size_t ws_bytes, void* stream) {
+  if (!Xq_img || !s_x || !W_img || !Y || T <= 0 || K <= 0 || N <= 0 || !grid_ok(grid) ||
+      !(s_w0 > 0.0f) || !isfinite(s_w0) || !(s_w1 > 0.0f) || !isfinite(s_w1) ||
+      !pair_split_ok(N0, N))
+    return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
+  if (ws && ws_bytes < dqt_fwd_img_workspace_size(T, K, N)) return DQT_ERR_ARG;
+  if (K % 8 || N % 8 || !aligned16(Xq_img) || !aligned16(W_img) || !aligned16(Y) ||
+      (acc_out && !aligned16(acc_out)) || (ws && !aligned16(ws)))
+    return DQT_ERR_ALIGN;
+  if (!fwd_range_ok(grid, K)) return DQT_ERR_RANGE;
+  return fwd_launch(Xq_img, s_x, W_img, s_w0, grid, T, K, N, Y, acc_out, ws, ws_bytes, stream,
+                    static_cast<int>(N0), s_w1);
 }
 
 int dqt_act_quant_fp8(const dqt_bf16* X, int64_t T, int64_t K, uint8_t* Xq8, float* s_x8,
@@ -452,8 +477,17 @@ int dqt_bitlinear_bwd_dx(const dqt_bf16* dY, const int8_t* W, float s_w, int64_t
 int dqt_bitlinear_bwd_dx_img(const dqt_bf16* dY, const dqt_bf16* W_img, float s_w, int64_t T,
                              int64_t N, int64_t K, dqt_bf16* dX, void* ws, size_t ws_bytes,
                              void* stream) {
-  if (!dY || !W_img || !dX || T <= 0 || N <= 0 || K <= 0 || !(s_w > 0.0f) || !isfinite(s_w))
+  return dqt_bitlinear_bwd_dx_img_ld(dY, N, W_img, s_w, T, N, K, dX, ws, ws_bytes, stream);
+}
+
+int dqt_bitlinear_bwd_dx_img_ld(const dqt_bf16* dY, int64_t ldy, const dqt_bf16* W_img, float s_w,
+                                int64_t T, int64_t N, int64_t K, dqt_bf16* dX, void* ws,
+                                size_t ws_bytes, void* stream) {
+  if (!dY || !W_img || !dX || T <= 0 || N <= 0 || K <= 0 || !(s_w > 0.0f) || !isfinite(s_w) ||
+      ldy < N)
     return DQT_ERR_ARG;
+  if (ldy > kMaxDim) return DQT_ERR_RANGE;
+  if (ldy % 8) return DQT_ERR_ALIGN;
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
   if (ws && ws_bytes < dqt_bwd_dx_img_workspace_size(T, N, K)) return DQT_ERR_ARG;
   if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(W_img) || !aligned16(dX) ||
@@ -470,6 +504,7 @@ int dqt_bitlinear_bwd_dx_img(const dqt_bf16* dY, const dqt_bf16* W_img, float s_
   g.out_bf16 = dX;
   g.ws = ws;
   g.ws_bytes = ws ? ws_bytes : 0;
+  g.lda = ldy;
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
@@ -560,6 +595,40 @@ int dqt_bitlinear_bwd_dw_update_img(const dqt_bf16* dY, const dqt_bf16* Xdq, int
   g.v = v;
   g.dW_out = dW_out;
   g.changed = upd ? changed_out : nullptr;
+  return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
+int dqt_bitlinear_bwd_dw_update_img_pair(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W,
+                                         int64_t N0, float s_w0, float s_w1, float* m, float* v,
+                                         const dqt_adamw_t* hp, const dqt_sr_t* sr0,
+                                         const dqt_sr_t* sr1, dqt_grid_t grid, int64_t T,
+                                         int64_t N, int64_t K, float* dW_out,
+                                         unsigned long long* changed_out, void* ws,
+                                         size_t ws_bytes, void* stream) {
+  if (!dY || !Xdq || !W || !m || !v || T <= 0 || N <= 0 || K <= 0 || !pair_split_ok(N0, N))
+    return DQT_ERR_ARG;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
+  if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(Xdq) || !aligned16(W) || !aligned16(m) ||
+      !aligned16(v) || (dW_out && !aligned16(dW_out)) || (ws && !aligned16(ws)))
+    return DQT_ERR_ALIGN;
+  dqt::GemmLaunch g{};
+  g.ws = ws;
+  g.ws_bytes = ws ? ws_bytes : 0;
+  int rc = make_update_consts(hp, sr0, grid, s_w0, &g.uc);
+  if (rc == DQT_OK) rc = make_update_consts(hp, sr1, grid, s_w1, &g.uc1);
+  if (rc != DQT_OK) return rc;
+  g.split = static_cast<int>(N0);
+  g.kind = dqt::GEMM_DW;
+  g.M = static_cast<int>(N);
+  g.N = static_cast<int>(K);
+  g.Kred = static_cast<int>(T);
+  g.A = dY;
+  g.B = Xdq;
+  g.W = W;
+  g.m = m;
+  g.v = v;
+  g.dW_out = dW_out;
+  g.changed = changed_out;
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 

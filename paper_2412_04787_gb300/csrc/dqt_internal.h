@@ -58,6 +58,13 @@ struct GemmLaunch {
   const UpdateConsts* uc_dev;  // DW: read the update constants from device memory if set
   void* ws;                    // DW: split-T workspace (fp32 slabs), or NULL
   size_t ws_bytes;
+  // two stacked weights (2-SM kernels only): from output column (FWD) or
+  // output row (DW) `split` on (a multiple of 256) the second weight, with
+  // scale scale1 (FWD) or constants uc1 (DW); 0: one weight
+  int split;
+  float scale1;
+  UpdateConsts uc1;
+  int64_t lda;  // DX: elements between rows of A (dY); 0: packed rows
 };
 
 // Token slices the 2-SM dW GEMM of an M x N output reduced over Kred uses
@@ -88,7 +95,7 @@ size_t gemm_tail_bytes(int M, int N, int Kred);
 int launch_tail_update(const float* part, int splits, int tail, int full, int num_n, int M, int N,
                        int8_t* W, bool packed, float* m, float* v, const UpdateConsts& uc,
                        const UpdateConsts* uc_dev, unsigned long long* changed, float* dW_out,
-                       cudaStream_t stream);
+                       cudaStream_t stream, const UpdateConsts* uc1 = nullptr, int split = 0);
 
 // Sum `splits` fp32 slabs (stride `slab` elements) in slice order and apply
 // the update to W, m, v (numel elements); optionally write the sum to g_out.

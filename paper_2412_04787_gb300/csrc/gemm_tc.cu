@@ -98,6 +98,15 @@ struct Params {
   // counter left by an earlier launch counts as zero
   unsigned long long* tail_ctr;
   unsigned long long tail_tag;
+  // two weights stacked in one call (e.g. a LLaMA MLP's gate and up
+  // projections, which read the same input): output columns (forward) or
+  // output rows (dW) from `split` on, a multiple of 256 (whole tiles), belong
+  // to the second weight, with its own scale (scale1) and update constants
+  // (uc1), and its Philox elements counted from its own first element; 0: one
+  // weight
+  int split;
+  float scale1;
+  UpdateConsts uc1;
 };
 
 struct Unit {
@@ -305,7 +314,7 @@ __device__ __forceinline__ void dw_issue(const Params& p, int row0, int gn0, int
 }
 
 template <bool PK>
-__device__ __forceinline__ uint32_t dw_update(const Params& p, const UpdateConsts& uc,
+__device__ __forceinline__ uint32_t dw_update(const Params& p, const UpdateConsts& uc, size_t e_off,
                                               float* dw_out, int row0, int gn0, int h, int lane,
                                               const float* xp, DwLoads& L) {
   const int cq = (lane & 7) * 4;
@@ -324,7 +333,7 @@ __device__ __forceinline__ uint32_t dw_update(const Params& p, const UpdateConst
     if (!p.W) continue;
     uint4 w = make_uint4(0, 0, 0, 0);
     if (uc.round_mode == 0)
-      w = sr_words(global_blk(uc, e >> 2), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
+      w = sr_words(global_blk(uc, (e - e_off) >> 2), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
     const int32_t n0c = dqt_update_elem(uc, g4.x, L.c[j].x, L.m[j].x, L.v[j].x, w.x);
     const int32_t n1c = dqt_update_elem(uc, g4.y, L.c[j].y, L.m[j].y, L.v[j].y, w.y);
     const int32_t n2c = dqt_update_elem(uc, g4.z, L.c[j].z, L.m[j].z, L.v[j].z, w.z);
@@ -363,8 +372,8 @@ __device__ __forceinline__ void dw_load_row(const Params& p, int gm, int gk, DwR
 
 template <bool PK>
 __device__ __forceinline__ uint32_t dw_update_row(const Params& p, const UpdateConsts& uc,
-                                                  float* dw_out, int gm, int gk, const float* src,
-                                                  DwRow& L) {
+                                                  size_t e_off, float* dw_out, int gm, int gk,
+                                                  const float* src, DwRow& L) {
   if (gk >= p.N || gm >= p.M) return 0;
   const size_t e = static_cast<size_t>(gm) * p.N + gk;
   const float4 g4 = make_float4(src[0], src[1], src[2], src[3]);
@@ -377,7 +386,7 @@ __device__ __forceinline__ uint32_t dw_update_row(const Params& p, const UpdateC
                                   static_cast<signed char>(L.c >> 24));
   uint4 w = make_uint4(0, 0, 0, 0);
   if (uc.round_mode == 0)
-    w = sr_words(global_blk(uc, e >> 2), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
+    w = sr_words(global_blk(uc, (e - e_off) >> 2), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
   const int32_t n0c = dqt_update_elem(uc, g4.x, c.x, L.m.x, L.v.x, w.x);
   const int32_t n1c = dqt_update_elem(uc, g4.y, c.y, L.m.y, L.v.y, w.y);
   const int32_t n2c = dqt_update_elem(uc, g4.z, c.z, L.m.z, L.v.z, w.z);
@@ -413,7 +422,7 @@ __device__ __forceinline__ void dw_load_first(const Params& p, int row0, int nba
 // (lane >> 3) + 4 (4 (q % 2) + j), j = 0..3, and columns 4 (lane & 7) .. + 3.
 template <bool PK>
 __device__ __forceinline__ uint32_t epi_dw_tile_roll(const Params& p, const UpdateConsts& uc,
-                                                     float* dw_out, int row0, int nbase,
+                                                     size_t e_off, float* dw_out, int row0, int nbase,
                                                      int nchunk, uint32_t t_acc, float* xp,
                                                      int lane, DwRow (&L)[4], int row0n,
                                                      int nbasen) {
@@ -439,7 +448,8 @@ __device__ __forceinline__ uint32_t epi_dw_tile_roll(const Params& p, const Upda
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const int r = (lane >> 3) + 4 * (4 * h + j);
-      n_changed += dw_update_row<PK>(p, uc, dw_out, row0 + r, gn0 + cq, xp + r * kStageLd + cq, L[j]);
+      n_changed += dw_update_row<PK>(p, uc, e_off, dw_out, row0 + r, gn0 + cq,
+                                     xp + r * kStageLd + cq, L[j]);
       if (nrow0 >= 0) dw_load_row<PK>(p, nrow0 + (lane >> 3) + 4 * (4 * nh + j), ngk, L[j]);
     }
     if (h == 1) __syncwarp();  // the transpose buffer is rewritten for the next chunk
@@ -455,8 +465,8 @@ __device__ __forceinline__ uint32_t epi_dw_tile_roll(const Params& p, const Upda
 // codes are 2-bit packed ternary (one byte per lane and row).
 template <bool PIPE, bool PK>
 __device__ __forceinline__ uint32_t epi_dw_tile(const Params& p, const UpdateConsts& uc,
-                                                float* dw_out, int row0, int nbase, int nchunk,
-                                                uint32_t t_acc, float* xp, int lane) {
+                                                size_t e_off, float* dw_out, int row0, int nbase,
+                                                int nchunk, uint32_t t_acc, float* xp, int lane) {
   uint32_t n_changed = 0;
   DwLoads A, B;
   if (PIPE) dw_issue<PK>(p, row0, nbase, 0, lane, A);
@@ -471,14 +481,14 @@ __device__ __forceinline__ uint32_t epi_dw_tile(const Params& p, const UpdateCon
     __syncwarp();
     if (PIPE) {
       dw_issue<PK>(p, row0, gn0, 1, lane, B);
-      n_changed += dw_update<PK>(p, uc, dw_out, row0, gn0, 0, lane, xp, A);
+      n_changed += dw_update<PK>(p, uc, e_off, dw_out, row0, gn0, 0, lane, xp, A);
       if (cc + 1 < nchunk) dw_issue<PK>(p, row0, gn0 + 32, 0, lane, A);
-      n_changed += dw_update<PK>(p, uc, dw_out, row0, gn0, 1, lane, xp, B);
+      n_changed += dw_update<PK>(p, uc, e_off, dw_out, row0, gn0, 1, lane, xp, B);
     } else {
 #pragma unroll 1
       for (int h = 0; h < 2; ++h) {
         dw_issue<PK>(p, row0, gn0, h, lane, A);
-        n_changed += dw_update<PK>(p, uc, dw_out, row0, gn0, h, lane, xp, A);
+        n_changed += dw_update<PK>(p, uc, e_off, dw_out, row0, gn0, h, lane, xp, A);
       }
     }
     __syncwarp();  // the transpose buffer is rewritten for the next chunk
@@ -654,7 +664,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int nbase = (t % p.num_n) * BN + half * HALF;
       const bool row_ok = gm < p.M;
       float a_t = 0.0f;
-      if (EPI == GEMM_FWD && row_ok) a_t = __fdiv_rn(1.0f, __fmul_rn(p.s_x[gm], p.scale));
+      if (EPI == GEMM_FWD && row_ok) {
+        // the second of two stacked weights (whole tiles of columns): its scale
+        const float sw = p.split > 0 && (t % p.num_n) * BN >= p.split ? p.scale1 : p.scale;
+        a_t = __fdiv_rn(1.0f, __fmul_rn(p.s_x[gm], sw));
+      }
       for (int c = 0; c < nchunks; ++c, ++u) {
         const int b = u & 1;
         ok = warp_wait(&acc_full[b], (u >> 1) & 1u, p.wait_ns);
@@ -664,7 +678,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t t_run = tmem + lane_off + RUN_COL + static_cast<uint32_t>(half * HALF);
         const bool last = (c + 1 == nchunks);
         if (EPI == GEMM_DW) {
-          n_changed += epi_dw_tile<true, false>(p, uc, p.dW_out, gm - lane, nbase, HALF / 32, t_acc, xp, lane);
+          // the second of two stacked weights: its constants, its own element count
+          const bool second = p.split > 0 && (t / p.num_n) * BM >= p.split;
+          n_changed += epi_dw_tile<true, false>(p, second ? p.uc1 : uc,
+                                                second ? static_cast<size_t>(p.split) * p.N : 0,
+                                                p.dW_out, gm - lane, nbase, HALF / 32, t_acc, xp,
+                                                lane);
         } else
 #pragma unroll 1
         for (int cc = 0; cc < HALF / 32; ++cc) {
@@ -974,7 +993,11 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
       if (EPI == GEMM_DW && un.slice < 0 && !st_loaded)
         dw_load_first<PK>(p, gm - lane, nbase, lane, st);  // in flight during the wait below
       float a_t = 0.0f;
-      if ((EPI == GEMM_FWD || F8) && row_ok) a_t = __fdiv_rn(1.0f, __fmul_rn(p.s_x[gm], p.scale));
+      if ((EPI == GEMM_FWD || F8) && row_ok) {
+        // the second of two stacked weights (whole tiles of columns): its scale
+        const float sw = p.split > 0 && (tile % p.num_n) * BN >= p.split ? p.scale1 : p.scale;
+        a_t = __fdiv_rn(1.0f, __fmul_rn(p.s_x[gm], sw));
+      }
       if (DR) {
         static_assert(!DR || HALF == 64, "two 32-column chunks of running sums per lane");
         const int nchunks = (p.num_kb + p.chunk_kb - 1) / p.chunk_kb;
@@ -1118,8 +1141,14 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
             nbasen = (nu.tile % p.num_n) * BN + half * HALF;
           }
         }
-        n_changed += epi_dw_tile_roll<PK>(p, uc, dw_out, gm - lane, nbase, HALF / 32, t_acc, xp,
-                                          lane, st, row0n, nbasen);
+        // the second of two stacked weights: its constants, its own element count
+        if (p.split > 0 && (tile / p.num_n) * 256 >= p.split)
+          n_changed += epi_dw_tile_roll<PK>(p, p.uc1, static_cast<size_t>(p.split) * p.N, dw_out,
+                                            gm - lane, nbase, HALF / 32, t_acc, xp, lane, st,
+                                            row0n, nbasen);
+        else
+          n_changed += epi_dw_tile_roll<PK>(p, uc, 0, dw_out, gm - lane, nbase, HALF / 32, t_acc,
+                                            xp, lane, st, row0n, nbasen);
         st_loaded = row0n >= 0;
       } else
 #pragma unroll 1
@@ -1180,7 +1209,7 @@ EncodeTiledFn encode_fn() {
 // `inner` contiguous elements per row and `outer` rows; box of box_inner x
 // box_outer, 128-byte swizzle, zero fill.
 bool make_map(CUtensorMap* map, const void* ptr, uint64_t inner, uint64_t outer,
-              uint32_t box_inner, uint32_t box_outer, int elem_bytes = 2) {
+              uint32_t box_inner, uint32_t box_outer, int elem_bytes = 2, uint64_t row_elems = 0) {
   EncodeTiledFn enc = encode_fn();
   if (!enc) return false;
   // The encoder is a driver call and needs a context current in the calling
@@ -1193,7 +1222,8 @@ bool make_map(CUtensorMap* map, const void* ptr, uint64_t inner, uint64_t outer,
     bound = true;
   }
   const cuuint64_t dims[2] = {inner, outer};
-  const cuuint64_t strides[1] = {inner * static_cast<cuuint64_t>(elem_bytes)};
+  // rows `row_elems` elements apart (0: packed rows of `inner`)
+  const cuuint64_t strides[1] = {(row_elems ? row_elems : inner) * static_cast<cuuint64_t>(elem_bytes)};
   const cuuint32_t box[2] = {box_inner, box_outer};
   const cuuint32_t estr[2] = {1, 1};
   return enc(map, elem_bytes == 1 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
@@ -1423,6 +1453,15 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   p.changed = g.changed;
   p.uc = g.uc;
   p.uc_dev = g.uc_dev;
+  p.split = g.split;
+  p.scale1 = g.scale1;
+  p.uc1 = g.uc1;
+  // stacked weights: whole tiles (multiples of 256 of either tiling),
+  // constants in the parameter space
+  if (g.split > 0 && (g.split % 256 != 0 || g.uc_dev ||
+                      (g.kind != GEMM_FWD && g.kind != GEMM_DW) ||
+                      g.split >= (g.kind == GEMM_FWD ? g.N : g.M)))
+    return 1;
 
   CUtensorMap ta, tb;
   switch (g.kind) {
@@ -1448,7 +1487,7 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
       if (!make_map(&tb, g.B, g.Kred, g.N, 128, 128, 1)) return 3;
       return launch_pairs<false, false, GEMM_FWD8>(ta, tb, p, stream);
     case GEMM_DX:
-      if (!make_map(&ta, g.A, g.Kred, g.M, BK, BM)) return 3;
+      if (!make_map(&ta, g.A, g.Kred, g.M, BK, BM, 2, static_cast<uint64_t>(g.lda))) return 3;
       if (!make_map(&tb, g.B, g.N, g.Kred, 64, BK)) return 3;
       if (g2.pair) {
         TailPlan tp{0, 0, 0, 0, 0};
@@ -1477,7 +1516,8 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
         if (rc || tp.splits == 0) return rc;
         return launch_tail_update(tail_partials(g.ws, 0), tp.splits, tp.tail, tp.full,
                                   (g.N + 255) / 256, g.M, g.N, g.W, g.packed, g.m, g.v, g.uc,
-                                  g.uc_dev, g.changed, g.dW_out, stream);
+                                  g.uc_dev, g.changed, g.dW_out, stream,
+                                  g.split > 0 ? &g.uc1 : nullptr, g.split);
       }
       // split-T: fp32 partials of each token slice into the workspace slabs,
       // then one streaming pass sums the slabs in slice order and applies the
@@ -1495,6 +1535,16 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
         // gradient only: sum the slabs into dW_out
         return launch_slab_sum(static_cast<const float*>(g.ws), p.splits, p.slab, g.dW_out,
                                stream);
+      }
+      if (g.split > 0) {
+        // stacked weights: the rows of each with its own constants
+        const long long n0 = static_cast<long long>(g.split) * g.N;
+        const float* sl = static_cast<const float*>(g.ws);
+        return launch_sr_update_slabs(sl, p.splits, p.slab, g.W, g.m, g.v, n0, g.uc, nullptr,
+                                      g.changed, g.dW_out, stream, g.packed) ||
+               launch_sr_update_slabs(sl + n0, p.splits, p.slab, g.W + n0, g.m + n0, g.v + n0,
+                                      p.slab - n0, g.uc1, nullptr, g.changed,
+                                      g.dW_out ? g.dW_out + n0 : nullptr, stream, g.packed);
       }
       return launch_sr_update_slabs(static_cast<const float*>(g.ws), p.splits, p.slab, g.W, g.m,
                                     g.v, p.slab, g.uc, g.uc_dev, g.changed, g.dW_out, stream,

@@ -171,7 +171,7 @@ __global__ void __launch_bounds__(kThreads, 3)
                        int M, int N, int8_t* __restrict__ W, bool packed, float* __restrict__ m,
                        float* __restrict__ v, const UpdateConsts uc_arg,
                        const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed,
-                       float* __restrict__ dW_out) {
+                       float* __restrict__ dW_out, const UpdateConsts uc1, int split) {
   const UpdateConsts uc = DEV ? *uc_dev : uc_arg;
   uint8_t* Wp = reinterpret_cast<uint8_t*>(W);
   const int64_t ngroups = static_cast<int64_t>(tail) * 16384;  // 256 x 256 / 4 per tile
@@ -213,14 +213,19 @@ __global__ void __launch_bounds__(kThreads, 3)
                                              static_cast<signed char>((craw >> 16) & 0xFFu),
                                              static_cast<signed char>(craw >> 24));
         float4 m4 = cur.m, v4 = cur.v;
+        // rows from `split` on: the second of two stacked weights, its own
+        // constants and element count
+        const bool second = split > 0 && e >= static_cast<int64_t>(split) * N;
+        const UpdateConsts& u = second ? uc1 : uc;
+        const int64_t er = second ? e - static_cast<int64_t>(split) * N : e;
         uint4 w = make_uint4(0, 0, 0, 0);
-        if (uc.round_mode == 0)
-          w = sr_words(global_blk(uc, static_cast<uint64_t>(e >> 2)), uc.step_lo, uc.tensor_id,
-                       uc.key0, uc.key1);
-        const int32_t a = dqt_update_elem(uc, g4.x, c0.x, m4.x, v4.x, w.x);
-        const int32_t b = dqt_update_elem(uc, g4.y, c0.y, m4.y, v4.y, w.y);
-        const int32_t c = dqt_update_elem(uc, g4.z, c0.z, m4.z, v4.z, w.z);
-        const int32_t d = dqt_update_elem(uc, g4.w, c0.w, m4.w, v4.w, w.w);
+        if (u.round_mode == 0)
+          w = sr_words(global_blk(u, static_cast<uint64_t>(er >> 2)), u.step_lo, u.tensor_id,
+                       u.key0, u.key1);
+        const int32_t a = dqt_update_elem(u, g4.x, c0.x, m4.x, v4.x, w.x);
+        const int32_t b = dqt_update_elem(u, g4.y, c0.y, m4.y, v4.y, w.y);
+        const int32_t c = dqt_update_elem(u, g4.z, c0.z, m4.z, v4.z, w.z);
+        const int32_t d = dqt_update_elem(u, g4.w, c0.w, m4.w, v4.w, w.w);
         n_changed += (a != c0.x) + (b != c0.y) + (c != c0.z) + (d != c0.w);
         if (packed)
           Wp[e >> 2] = static_cast<uint8_t>(tern_pack4(a, b, c, d));
@@ -310,7 +315,8 @@ int launch_sr_update_slabs(const float* slabs, int splits, long long slab, int8_
 int launch_tail_update(const float* part, int splits, int tail, int full, int num_n, int M, int N,
                        int8_t* W, bool packed, float* m, float* v, const UpdateConsts& uc,
                        const UpdateConsts* uc_dev, unsigned long long* changed, float* dW_out,
-                       cudaStream_t stream) {
+                       cudaStream_t stream, const UpdateConsts* uc1, int split) {
+  const UpdateConsts u1 = uc1 ? *uc1 : uc;
   // the blocks that fit at once: each thread walks several groups, its next
   // group's loads in flight
   static int occ[2] = {0, 0};  // resident blocks per SM, per template instance
@@ -330,11 +336,12 @@ int launch_tail_update(const float* part, int splits, int tail, int full, int nu
   if (uc_dev)
     tail_update_kernel<true><<<blocks, kThreads, 0, stream>>>(part, splits, tail, full, num_n, M, N,
                                                               W, packed, m, v, uc, uc_dev, changed,
-                                                              dW_out);
+                                                              dW_out, u1, uc1 ? split : 0);
   else
     tail_update_kernel<false><<<blocks, kThreads, 0, stream>>>(part, splits, tail, full, num_n, M,
                                                                N, W, packed, m, v, uc, nullptr,
-                                                               changed, dW_out);
+                                                               changed, dW_out, u1,
+                                                               uc1 ? split : 0);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 

@@ -35,6 +35,8 @@ EXPORTED = [
     "dqt_bwd_dx_workspace_size", "dqt_bitlinear_bwd_dw_update_img",
     "dqt_bwd_dw_img_workspace_size", "dqt_codes_to_xdq", "dqt_fwd_workspace_size",
     "dqt_fwd_img_workspace_size", "dqt_bwd_dx_img_workspace_size",
+    "dqt_bitlinear_fwd_img_pair", "dqt_bitlinear_bwd_dw_update_img_pair",
+    "dqt_bitlinear_bwd_dx_img_ld",
 ]
 
 
@@ -98,11 +100,19 @@ def lib():
         L.dqt_fwd_workspace_size.restype = _sz
         L.dqt_bitlinear_fwd_img.argtypes = [_vp, _vp, _vp, _f32, dqt_grid_t, _i64, _i64, _i64,
                                             _vp, _vp, _vp, _sz, _vp]
+        L.dqt_bitlinear_fwd_img_pair.argtypes = [_vp, _vp, _vp, _i64, _f32, _f32, dqt_grid_t, _i64,
+                                                 _i64, _i64, _vp, _vp, _vp, _sz, _vp]
+        L.dqt_bitlinear_bwd_dw_update_img_pair.argtypes = [
+            _vp, _vp, _vp, _i64, _f32, _f32, _vp, _vp, C.POINTER(dqt_adamw_t),
+            C.POINTER(dqt_sr_t), C.POINTER(dqt_sr_t), dqt_grid_t, _i64, _i64, _i64, _vp, _vp,
+            _vp, _sz, _vp]
         L.dqt_fwd_img_workspace_size.argtypes = [_i64, _i64, _i64]
         L.dqt_fwd_img_workspace_size.restype = _sz
         L.dqt_bitlinear_bwd_dx.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp, _sz, _vp]
         L.dqt_bitlinear_bwd_dx_img.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp, _sz,
                                                _vp]
+        L.dqt_bitlinear_bwd_dx_img_ld.argtypes = [_vp, _i64, _vp, _f32, _i64, _i64, _i64, _vp, _vp,
+                                                  _sz, _vp]
         L.dqt_bwd_dx_workspace_size.argtypes = [_i64, _i64, _i64]
         L.dqt_bwd_dx_workspace_size.restype = _sz
         L.dqt_bwd_dx_img_workspace_size.argtypes = [_i64, _i64, _i64]
@@ -396,6 +406,29 @@ def dqt_bitlinear_fwd_img(Xq_img, s_x, W_img, s_w, bits_or_grid, Y=None, acc_out
     return Y
 
 
+def dqt_bitlinear_fwd_img_pair(Xq_img, s_x, W_img, N0, s_w0, s_w1, bits_or_grid, Y=None,
+                               acc_out=None, ws=None, stream=None):
+    """Two weights that read the same input, stacked along N (rows [0, N0)
+    of W_img the first's code image, scale s_w0; the rest the second's, s_w1):
+    Y [T, N] holds both outputs side by side.  `ws` as dqt_bitlinear_fwd_img."""
+    _need(Xq_img, "Xq_img", torch.bfloat16)
+    T, K = Xq_img.shape
+    _need(W_img, "W_img", torch.bfloat16)
+    N = W_img.shape[0]
+    _need(W_img, "W_img", torch.bfloat16, (N, K))
+    _need(s_x, "s_x", torch.float32, (T,))
+    if Y is None:
+        Y = torch.empty((T, N), dtype=torch.bfloat16, device=Xq_img.device)
+    _need(Y, "Y", torch.bfloat16, (T, N))
+    _opt(acc_out, "acc_out", torch.int32, (T, N))
+    ws, nws = _tail_workspace(lib().dqt_fwd_img_workspace_size(T, K, N), Xq_img.device, ws)
+    _check(lib().dqt_bitlinear_fwd_img_pair(_ptr(Xq_img), _ptr(s_x), _ptr(W_img), int(N0),
+                                            float(s_w0), float(s_w1), _grid(bits_or_grid), T, K, N,
+                                            _ptr(Y), _ptr(acc_out), _ptr(ws), nws, _stream(stream)),
+           "dqt_bitlinear_fwd_img_pair")
+    return Y
+
+
 def dqt_bwd_dx_workspace_size(T, N, K):
     return int(lib().dqt_bwd_dx_workspace_size(T, N, K))
 
@@ -428,8 +461,16 @@ def dqt_bitlinear_bwd_dx(dY, W, s_w, dX=None, ws=None, stream=None):
 
 def dqt_bitlinear_bwd_dx_img(dY, W_img, s_w, dX=None, ws=None, stream=None):
     """dX on the weight's bf16 image; `ws` as for dqt_bitlinear_fwd_img
-    (dqt_bwd_dx_img_workspace_size bytes)."""
-    _need(dY, "dY", torch.bfloat16)
+    (dqt_bwd_dx_img_workspace_size bytes).  dY may be a view of whole rows'
+    column range (e.g. one weight's half of a stacked output's gradient):
+    its rows are then read in place, dY.stride(0) elements apart."""
+    if dY is not None and dY.dim() == 2 and dY.stride(1) == 1 and dY.stride(0) > dY.shape[1]:
+        ldy = dY.stride(0)  # rows of a wider tensor
+        if not dY.is_cuda or dY.dtype != torch.bfloat16:
+            raise ValueError("dY must be a bf16 CUDA tensor")
+    else:
+        _need(dY, "dY", torch.bfloat16)
+        ldy = dY.shape[1]
     T, N = dY.shape
     _need(W_img, "W_img", torch.bfloat16)
     K = W_img.shape[1]
@@ -438,8 +479,8 @@ def dqt_bitlinear_bwd_dx_img(dY, W_img, s_w, dX=None, ws=None, stream=None):
         dX = torch.empty((T, K), dtype=torch.bfloat16, device=dY.device)
     _need(dX, "dX", torch.bfloat16, (T, K))
     ws, nws = _tail_workspace(lib().dqt_bwd_dx_img_workspace_size(T, N, K), dY.device, ws)
-    _check(lib().dqt_bitlinear_bwd_dx_img(_ptr(dY), _ptr(W_img), float(s_w), T, N, K,
-                                          _ptr(dX), _ptr(ws), nws, _stream(stream)),
+    _check(lib().dqt_bitlinear_bwd_dx_img_ld(_ptr(dY), ldy, _ptr(W_img), float(s_w), T, N, K,
+                                             _ptr(dX), _ptr(ws), nws, _stream(stream)),
            "dqt_bitlinear_bwd_dx_img")
     return dX
 
@@ -519,6 +560,30 @@ def dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, s_w, m, v, hp, sr, bits_or_grid,
         C.byref(hp) if hp is not None else None, C.byref(sr) if sr is not None else None,
         _grid(bits_or_grid), T, N, K, _ptr(dW_out), _ptr(changed_out), _ptr(ws), nws,
         _stream(stream)), "dqt_bitlinear_bwd_dw_update_img")
+    return W
+
+
+def dqt_bitlinear_bwd_dw_update_img_pair(dY, Xdq, W, N0, s_w0, s_w1, m, v, hp, sr0, sr1,
+                                         bits_or_grid, dW_out=None, changed_out=None, ws=None,
+                                         stream=None):
+    """The fused dW + update of two stacked weights (rows [0, N0) of W, m, v
+    and columns [0, N0) of dY the first's, with s_w0 and sr0; the rest the
+    second's, with s_w1 and sr1).  `ws` as dqt_bitlinear_bwd_dw_update_img."""
+    _need(dY, "dY", torch.bfloat16)
+    T, N = dY.shape
+    _need(Xdq, "Xdq", torch.bfloat16)
+    K = Xdq.shape[1]
+    _need(Xdq, "Xdq", torch.bfloat16, (T, K))
+    _need(W, "W", torch.int8, (N, K))
+    _need(m, "m", torch.float32, (N, K))
+    _need(v, "v", torch.float32, (N, K))
+    _opt(dW_out, "dW_out", torch.float32, (N, K))
+    _opt(changed_out, "changed_out", torch.int64, (1,))
+    ws, nws = _dw_workspace(T, N, K, dY.device, ws)
+    _check(lib().dqt_bitlinear_bwd_dw_update_img_pair(
+        _ptr(dY), _ptr(Xdq), _ptr(W), int(N0), float(s_w0), float(s_w1), _ptr(m), _ptr(v),
+        C.byref(hp), C.byref(sr0), C.byref(sr1), _grid(bits_or_grid), T, N, K, _ptr(dW_out),
+        _ptr(changed_out), _ptr(ws), nws, _stream(stream)), "dqt_bitlinear_bwd_dw_update_img_pair")
     return W
 
 

@@ -104,6 +104,16 @@ def test_argument_validation_without_launch(L):
     assert L.dqt_fwd_img_workspace_size(256, 512, 256) == 0
     assert L.dqt_fwd_img_workspace_size(8192, 2048, 5632) == 0
     assert L.dqt_bwd_dx_img_workspace_size(8192, 2048, 5632) == 0
+    # stacked weights: the split a positive multiple of 256 below N, both scales positive
+    assert L.dqt_bitlinear_fwd_img_pair(A, A, A, 200, 1.0, 1.0, g, 4, 8, 512, A, None, None, 0, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_fwd_img_pair(A, A, A, 512, 1.0, 1.0, g, 4, 8, 512, A, None, None, 0, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_fwd_img_pair(A, A, A, 256, 1.0, 0.0, g, 4, 8, 512, A, None, None, 0, None) == dqt.DQT_ERR_ARG
+    hp = dqt.adamw()
+    sr = dqt.sr_stream()
+    assert L.dqt_bitlinear_bwd_dw_update_img_pair(A, A, A, 100, 1.0, 1.0, A, A, hp, sr, sr, g, 4, 512, 8,
+                                                  None, None, None, 0, None) == dqt.DQT_ERR_ARG
+    assert L.dqt_bitlinear_bwd_dw_update_img_pair(A, A, None, 256, 1.0, 1.0, A, A, hp, sr, sr, g, 4, 512, 8,
+                                                  None, None, None, 0, None) == dqt.DQT_ERR_ARG
     # bad grid / scale
     assert L.dqt_bitlinear_fwd(A, A, A, 1.0, dqt.dqt_grid_t(2, 1), 4, 8, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ARG
     assert L.dqt_bitlinear_fwd(A, A, A, 1.0, dqt.dqt_grid_t(-129, 1), 4, 8, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ARG

@@ -1,0 +1,146 @@
+"""Two BitLinear weights that read the same input, stacked in one call (a
+LLaMA MLP's gate and up projections): dqt_bitlinear_fwd_img_pair and
+dqt_bitlinear_bwd_dw_update_img_pair.
+
+Each weight keeps its own per-tensor scale (Eq. 2-3) and its own
+stochastic-rounding stream (Philox elements counted from its own first
+element), so the stacked calls must give, bit for bit, what two separate
+calls give: the forward's Y and int32 accumulators, and the update's codes,
+moments and changed-code count.  Both GEMM tilings; the split at whole
+256-wide tiles.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from fused_rule import assert_fused_codes
+from paper_2412_04787_gb300 import dqt, inputs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2412_04787_gb300 import build
+    build.build()
+    dqt.lib()
+    yield
+    dqt.dqt_set_gemm_tiles(0)
+    torch.cuda.synchronize()
+
+
+def _weights(N0, N1, K, bits, seed):
+    qmin, qmax = oracle.grid(bits)
+    c0, s0, _ = oracle.absmean_init(inputs.normal((N0, K), 0.02, seed=seed).numpy(), qmin, qmax)
+    c1, s1, _ = oracle.absmean_init(inputs.normal((N1, K), 0.03, seed=seed + 1).numpy(), qmin, qmax)
+    assert s0 != s1  # two different per-tensor scales
+    return np.concatenate([c0, c1]), float(s0), float(s1), (qmin, qmax)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("T,K,N0,N1,bits", [(300, 264, 256, 264, 1.58), (1024, 2048, 5632, 5632, 1.58),
+                                            (256, 1088, 512, 256, 8)])
+def test_fwd_pair_equals_two_calls(mode, T, K, N0, N1, bits):
+    dqt.dqt_set_gemm_tiles(mode)
+    try:
+        X = inputs.normal((T, K), 1.0, seed=T + K, dtype=torch.bfloat16)
+        c, s0, s1, g = _weights(N0, N1, K, bits, seed=N0 + N1)
+        _, s_x, q_img, _ = dqt.dqt_act_quant_images(X.cuda(), want=("Xq_img",))
+        W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
+        N = N0 + N1
+        acc = torch.empty((T, N), dtype=torch.int32, device="cuda")
+        Y = dqt.dqt_bitlinear_fwd_img_pair(q_img, s_x, W_img, N0, s0, s1, g, acc_out=acc)
+        acc0 = torch.empty((T, N0), dtype=torch.int32, device="cuda")
+        acc1 = torch.empty((T, N1), dtype=torch.int32, device="cuda")
+        Y0 = dqt.dqt_bitlinear_fwd_img(q_img, s_x, W_img[:N0], s0, g, acc_out=acc0)
+        Y1 = dqt.dqt_bitlinear_fwd_img(q_img, s_x, W_img[N0:], s1, g, acc_out=acc1)
+        dqt.dqt_check_device_status()
+        assert torch.equal(acc[:, :N0], acc0) and torch.equal(acc[:, N0:], acc1)
+        assert torch.equal(Y[:, :N0].contiguous().view(torch.int16), Y0.view(torch.int16))
+        assert torch.equal(Y[:, N0:].contiguous().view(torch.int16), Y1.view(torch.int16))
+        # and the oracle on two rows, the second weight's scale included
+        rows = np.array([0, T - 1])
+        Xb = X[torch.from_numpy(rows)].contiguous().view(torch.int16).numpy().view(np.uint16)
+        q, s, _, _ = oracle.act_quant(Xb)
+        Yr, accr = oracle.fwd(q, s, c[N0:], np.float32(s1))
+        it = torch.from_numpy(rows).cuda()
+        assert np.array_equal(acc[it][:, N0:].cpu().numpy(), accr)
+        assert np.array_equal(Y[it][:, N0:].contiguous().view(torch.int16).cpu().numpy().view(np.uint16), Yr)
+    finally:
+        dqt.dqt_set_gemm_tiles(0)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("T,K,N0,N1,bits,step", [(256, 512, 256, 264, 1.58, 1),
+                                                 (1024, 2048, 5632, 5632, 1.58, 3),
+                                                 (512, 264, 512, 256, 8, 2)])
+def test_dw_update_pair_equals_two_calls(mode, T, K, N0, N1, bits, step):
+    dqt.dqt_set_gemm_tiles(mode)
+    try:
+        N = N0 + N1
+        X = inputs.normal((T, K), 1.0, seed=T, dtype=torch.bfloat16)
+        dY = inputs.normal((T, N), 1e-2, seed=T + 1, dtype=torch.bfloat16).cuda()
+        c, s0, s1, g = _weights(N0, N1, K, bits, seed=K)
+        _, s_x, _, Xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xdq",))
+        if step > 1:
+            m0 = inputs.normal((N, K), 1e-4, seed=7).cuda()
+            v0 = inputs.normal((N, K), 1e-4, seed=8).square().cuda()
+        else:
+            m0 = torch.zeros((N, K), device="cuda")
+            v0 = torch.zeros((N, K), device="cuda")
+        hp = dqt.adamw(lr=1e-3, weight_decay=0.01, step=step)
+        sr0 = dqt.sr_stream(seed=1234, tensor_id=4)
+        sr1 = dqt.sr_stream(seed=1234, tensor_id=5)
+        W = torch.from_numpy(c).cuda()
+        m, v = m0.clone(), v0.clone()
+        ch = torch.zeros(1, dtype=torch.int64, device="cuda")
+        dqt.dqt_bitlinear_bwd_dw_update_img_pair(dY, Xdq, W, N0, s0, s1, m, v, hp, sr0, sr1, g,
+                                                 changed_out=ch, ws=False)
+        # two separate calls on the halves (no token slicing on either side:
+        # the same tiles, the same fp32 sums)
+        Wa = torch.from_numpy(c[:N0]).cuda()
+        Wb = torch.from_numpy(c[N0:]).cuda()
+        ma, va = m0[:N0].clone(), v0[:N0].clone()
+        mb, vb = m0[N0:].clone(), v0[N0:].clone()
+        ch2 = torch.zeros(1, dtype=torch.int64, device="cuda")
+        dqt.dqt_bitlinear_bwd_dw_update_img(dY[:, :N0].contiguous(), Xdq, Wa, s0, ma, va, hp, sr0, g,
+                                            changed_out=ch2, ws=False)
+        dqt.dqt_bitlinear_bwd_dw_update_img(dY[:, N0:].contiguous(), Xdq, Wb, s1, mb, vb, hp, sr1, g,
+                                            changed_out=ch2, ws=False)
+        dqt.dqt_check_device_status()
+        assert torch.equal(W[:N0], Wa) and torch.equal(W[N0:], Wb)
+        assert torch.equal(m[:N0], ma) and torch.equal(m[N0:], mb)
+        assert torch.equal(v[:N0], va) and torch.equal(v[N0:], vb)
+        assert int(ch.item()) == int(ch2.item())
+        assert int(ch.item()) > 0
+    finally:
+        dqt.dqt_set_gemm_tiles(0)
+
+
+def test_dw_update_pair_with_token_slices():
+    """A stacked update whose output leaves the last wave short (token slices
+    and the streaming tail update): the second weight's rows in the tail take
+    its own constants and element count — equal to the slice-free call up to
+    the gradient's fp32 summation order (the fused-update rule)."""
+    T, K, N0, N1 = 4096, 2048, 2816 - 256, 2816 + 256  # 22 x 8 = 176 output tiles
+    N = N0 + N1
+    assert dqt.dqt_bwd_dw_img_workspace_size(T, N, K) > 0
+    X = inputs.normal((T, K), 1.0, seed=3, dtype=torch.bfloat16)
+    dY = inputs.normal((T, N), 1e-2, seed=4, dtype=torch.bfloat16).cuda()
+    c, s0, s1, g = _weights(N0, N1, K, 1.58, seed=9)
+    _, s_x, _, Xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xdq",))
+    hp = dqt.adamw(lr=1e-3, step=1)
+    sr0 = dqt.sr_stream(seed=77, tensor_id=0)
+    sr1 = dqt.sr_stream(seed=77, tensor_id=1)
+    outs = []
+    for ws in (None, False):
+        W = torch.from_numpy(c).cuda()
+        m = torch.zeros((N, K), device="cuda")
+        v = torch.zeros((N, K), device="cuda")
+        dqt.dqt_bitlinear_bwd_dw_update_img_pair(dY, Xdq, W, N0, s0, s1, m, v, hp, sr0, sr1, g, ws=ws)
+        outs.append(W)
+    dqt.dqt_check_device_status()
+    assert_fused_codes(outs[0].cpu().numpy(), outs[1].cpu().numpy(), "pair, sliced vs unsliced")
