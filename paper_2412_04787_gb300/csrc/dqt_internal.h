@@ -95,7 +95,8 @@ size_t gemm_tail_bytes(int M, int N, int Kred);
 int launch_tail_update(const float* part, int splits, int tail, int full, int num_n, int M, int N,
                        int8_t* W, bool packed, float* m, float* v, const UpdateConsts& uc,
                        const UpdateConsts* uc_dev, unsigned long long* changed, float* dW_out,
-                       cudaStream_t stream, const UpdateConsts* uc1 = nullptr, int split = 0);
+                       cudaStream_t stream, const UpdateConsts* uc1 = nullptr, int split = 0,
+                       bool col_major = false);
 
 // Sum `splits` fp32 slabs (stride `slab` elements) in slice order and apply
 // the update to W, m, v (numel elements); optionally write the sum to g_out.

@@ -107,7 +107,20 @@ struct Params {
   int split;
   float scale1;
   UpdateConsts uc1;
+  // 2-SM kernels: output tiles numbered down the columns (tile % num_m is
+  // the row tile) instead of along the rows: the A operand is then the one
+  // every wave re-reads (chosen when A's panels are the smaller set)
+  int num_m;
+  bool col_major;
 };
+
+// Row and column tile (256 x 256) of a 2-SM kernel's tile index.
+__device__ __forceinline__ int pair_tile_m(const Params& p, int tile) {
+  return p.col_major ? tile % p.num_m : tile / p.num_n;
+}
+__device__ __forceinline__ int pair_tile_n(const Params& p, int tile) {
+  return p.col_major ? tile / p.num_m : tile % p.num_n;
+}
 
 struct Unit {
   int tile, kb0, kb1;
@@ -853,8 +866,8 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
       for (int t = cid; t < p.num_tiles && ok; t += ncl) {
         const Unit un = decode_unit(p, t);
         const int tile = un.tile, kb0 = un.kb0, kb1 = un.kb1;
-        const int m0 = (tile / p.num_n) * 256 + static_cast<int>(rank) * 128;
-        const int n0 = (tile % p.num_n) * BN + static_cast<int>(rank) * 128;
+        const int m0 = pair_tile_m(p, tile) * 256 + static_cast<int>(rank) * 128;
+        const int n0 = pair_tile_n(p, tile) * BN + static_cast<int>(rank) * 128;
         for (int kb = kb0; kb < kb1; ++kb, ++it) {
           if (it >= ST && !mbar_wait_cl(&empty[s], ph ^ 1u, p.wait_ns)) {
             ok = false;
@@ -867,6 +880,11 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
           const int k0 = kb * KB;
           if (!A_MN) {
             tma_load_2d_pair(&tmA, bar, a, k0, m0);
+          } else if (EPI == GEMM_DW && p.col_major) {
+            // column-major tiles: dY's panels are re-read by every wave
+#pragma unroll
+            for (int j = 0; j < 2; ++j)
+              tma_load_2d_pair_hint(&tmA, bar, a + j * MN_CHUNK_BYTES, m0 + 64 * j, k0, pol_b);
           } else {
 #pragma unroll
             for (int j = 0; j < 2; ++j)
@@ -874,7 +892,7 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
           }
           if (!B_MN) {
             tma_load_2d_pair(&tmB, bar, b, k0, n0);
-          } else if (EPI == GEMM_DW) {
+          } else if (EPI == GEMM_DW && !p.col_major) {
             // X~ (all K columns) is re-read by every wave of output-row tiles,
             // while each dY column block is read by one wave: keep X~ in L2
 #pragma unroll
@@ -987,15 +1005,15 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
       const Unit un = decode_unit(p, t);
       const int tile = un.tile;
       float* dw_out = p.dW_out ? p.dW_out + un.slab * p.slab : nullptr;
-      const int gm = (tile / p.num_n) * 256 + static_cast<int>(rank) * 128 + row;
-      const int nbase = (tile % p.num_n) * BN + half * HALF;
+      const int gm = pair_tile_m(p, tile) * 256 + static_cast<int>(rank) * 128 + row;
+      const int nbase = pair_tile_n(p, tile) * BN + half * HALF;
       const bool row_ok = gm < p.M;
       if (EPI == GEMM_DW && un.slice < 0 && !st_loaded)
         dw_load_first<PK>(p, gm - lane, nbase, lane, st);  // in flight during the wait below
       float a_t = 0.0f;
       if ((EPI == GEMM_FWD || F8) && row_ok) {
         // the second of two stacked weights (whole tiles of columns): its scale
-        const float sw = p.split > 0 && (tile % p.num_n) * BN >= p.split ? p.scale1 : p.scale;
+        const float sw = p.split > 0 && pair_tile_n(p, tile) * BN >= p.split ? p.scale1 : p.scale;
         a_t = __fdiv_rn(1.0f, __fmul_rn(p.s_x[gm], sw));
       }
       if (DR) {
@@ -1137,12 +1155,12 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
         if (t + ncl < p.num_tiles) {
           const Unit nu = decode_unit(p, t + ncl);
           if (nu.slice < 0) {
-            row0n = (nu.tile / p.num_n) * 256 + static_cast<int>(rank) * 128 + quad * 32;
-            nbasen = (nu.tile % p.num_n) * BN + half * HALF;
+            row0n = pair_tile_m(p, nu.tile) * 256 + static_cast<int>(rank) * 128 + quad * 32;
+            nbasen = pair_tile_n(p, nu.tile) * BN + half * HALF;
           }
         }
         // the second of two stacked weights: its constants, its own element count
-        if (p.split > 0 && (tile / p.num_n) * 256 >= p.split)
+        if (p.split > 0 && pair_tile_m(p, tile) * 256 >= p.split)
           n_changed += epi_dw_tile_roll<PK>(p, p.uc1, static_cast<size_t>(p.split) * p.N, dw_out,
                                             gm - lane, nbase, HALF / 32, t_acc, xp, lane, st,
                                             row0n, nbasen);
@@ -1344,7 +1362,12 @@ int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStr
   constexpr int threads = PairCfg<EPI, DR>::THREADS;
   static int max_clusters = 0;  // per template instance
   p.num_n = (p.N + 255) / 256;
-  p.num_tiles = ((p.M + 255) / 256) * p.num_n * p.splits;
+  p.num_m = (p.M + 255) / 256;
+  p.num_tiles = p.num_m * p.num_n * p.splits;
+  // dW: the operand with fewer 256-wide panels is the one re-read by every
+  // wave (and kept in L2): X_tilde (along the rows) when the output has more
+  // row tiles, dY (down the columns) when it has more column tiles
+  p.col_major = EPI == GEMM_DW && p.num_n > p.num_m;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -1517,7 +1540,8 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
         return launch_tail_update(tail_partials(g.ws, 0), tp.splits, tp.tail, tp.full,
                                   (g.N + 255) / 256, g.M, g.N, g.W, g.packed, g.m, g.v, g.uc,
                                   g.uc_dev, g.changed, g.dW_out, stream,
-                                  g.split > 0 ? &g.uc1 : nullptr, g.split);
+                                  g.split > 0 ? &g.uc1 : nullptr, g.split,
+                                  (g.N + 255) / 256 > (g.M + 255) / 256);
       }
       // split-T: fp32 partials of each token slice into the workspace slabs,
       // then one streaming pass sums the slabs in slice order and applies the

@@ -142,13 +142,14 @@ __device__ __forceinline__ void tail_load(int64_t gi, const float* __restrict__ 
                                           int tail, int full, int num_n, int M, int N,
                                           const int8_t* __restrict__ W, bool packed,
                                           const float* __restrict__ m, const float* __restrict__ v,
-                                          TailGroup& g) {
+                                          bool col_major, TailGroup& g) {
   const int j = static_cast<int>(gi >> 14);
   const int r = static_cast<int>((gi >> 6) & 255);
   const int c4 = static_cast<int>(gi & 63) * 4;
   const int tile = full + j;
-  const int row = (tile / num_n) * 256 + r;
-  const int col = (tile % num_n) * 256 + c4;
+  const int num_m = (M + 255) / 256;  // the GEMM's tile numbering (see its col_major)
+  const int row = (col_major ? tile % num_m : tile / num_n) * 256 + r;
+  const int col = (col_major ? tile / num_m : tile % num_n) * 256 + c4;
   g.e = -1;
   if (row >= M || col >= N) return;  // N % 4 == 0: the whole group is in range
   g.e = static_cast<int64_t>(row) * N + col;
@@ -171,7 +172,8 @@ __global__ void __launch_bounds__(kThreads, 3)
                        int M, int N, int8_t* __restrict__ W, bool packed, float* __restrict__ m,
                        float* __restrict__ v, const UpdateConsts uc_arg,
                        const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed,
-                       float* __restrict__ dW_out, const UpdateConsts uc1, int split) {
+                       float* __restrict__ dW_out, const UpdateConsts uc1, int split,
+                       bool col_major) {
   const UpdateConsts uc = DEV ? *uc_dev : uc_arg;
   uint8_t* Wp = reinterpret_cast<uint8_t*>(W);
   const int64_t ngroups = static_cast<int64_t>(tail) * 16384;  // 256 x 256 / 4 per tile
@@ -180,12 +182,14 @@ __global__ void __launch_bounds__(kThreads, 3)
   uint32_t n_changed = 0;
   int64_t gi = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x;
   TailGroup cur;
-  if (gi < ngroups) tail_load(gi, part, splits, tail, full, num_n, M, N, W, packed, m, v, cur);
+  if (gi < ngroups)
+    tail_load(gi, part, splits, tail, full, num_n, M, N, W, packed, m, v, col_major, cur);
   for (; gi < ngroups; gi += stride) {
     TailGroup nxt;
     nxt.e = -1;
     if (gi + stride < ngroups)
-      tail_load(gi + stride, part, splits, tail, full, num_n, M, N, W, packed, m, v, nxt);
+      tail_load(gi + stride, part, splits, tail, full, num_n, M, N, W, packed, m, v, col_major,
+                nxt);
     if (cur.e >= 0) {
       const int64_t e = cur.e;
       float4 g4 = cur.p[0];
@@ -315,7 +319,7 @@ int launch_sr_update_slabs(const float* slabs, int splits, long long slab, int8_
 int launch_tail_update(const float* part, int splits, int tail, int full, int num_n, int M, int N,
                        int8_t* W, bool packed, float* m, float* v, const UpdateConsts& uc,
                        const UpdateConsts* uc_dev, unsigned long long* changed, float* dW_out,
-                       cudaStream_t stream, const UpdateConsts* uc1, int split) {
+                       cudaStream_t stream, const UpdateConsts* uc1, int split, bool col_major) {
   const UpdateConsts u1 = uc1 ? *uc1 : uc;
   // the blocks that fit at once: each thread walks several groups, its next
   // group's loads in flight
@@ -336,12 +340,13 @@ int launch_tail_update(const float* part, int splits, int tail, int full, int nu
   if (uc_dev)
     tail_update_kernel<true><<<blocks, kThreads, 0, stream>>>(part, splits, tail, full, num_n, M, N,
                                                               W, packed, m, v, uc, uc_dev, changed,
-                                                              dW_out, u1, uc1 ? split : 0);
+                                                              dW_out, u1, uc1 ? split : 0,
+                                                              col_major);
   else
     tail_update_kernel<false><<<blocks, kThreads, 0, stream>>>(part, splits, tail, full, num_n, M,
                                                                N, W, packed, m, v, uc, nullptr,
                                                                changed, dW_out, u1,
-                                                               uc1 ? split : 0);
+                                                               uc1 ? split : 0, col_major);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
