@@ -159,7 +159,7 @@ class MLPStep:
     """Device buffers and the launch sequence of one DQT MLP training step."""
 
     def __init__(self, dev, seed=1234, fp8=False, optimizer="adamw", packed=False, bits=1.58,
-                 operands="int8", tail_slices=True, stack_gate_up=False):
+                 operands="int8", tail_slices=True, stack_gate_up=False, next_image=True):
         from paper_2412_04787_gb300 import dqt, inputs
 
         self.dqt = dqt
@@ -238,6 +238,22 @@ class MLPStep:
                 self.W8[name] = torch.empty((N, K), dtype=torch.uint8, device=dev)
             self.Y[name] = torch.empty((T, N), dtype=torch.bfloat16, device=dev)
             self.dX[name] = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
+        # image operands with AdamW on int8 codes: each weight-gradient call
+        # writes the image of the codes it updates into the second of two
+        # image buffers (the next step's forward and dX operand), so that no
+        # step converts codes to images; the buffers swap after every step
+        self.nimg = next_image and not self.i8 and not fp8 and not packed and optimizer == "adamw"
+        if self.nimg:
+            self.W_img_next = {}
+            if self.stack:
+                self.W_img_gu_next = torch.empty_like(self.W_img_gu)
+            for name, K, N in PROJ:
+                if self.stack and name in ("gate", "up"):
+                    half = slice(0, INTER) if name == "gate" else slice(INTER, 2 * INTER)
+                    self.W_img_next[name] = self.W_img_gu_next[half]
+                else:
+                    self.W_img_next[name] = torch.empty((N, K), dtype=torch.bfloat16, device=dev)
+                dqt.dqt_codes_to_bf16(self.W[name], self.W_img[name])  # the first step's images
         # per activation: (scale, forward operand, dequantised bf16 image); the
         # forward operand is the int8 codes (no image), the bf16 code image,
         # or the E4M3 bytes with fp8
@@ -291,6 +307,8 @@ class MLPStep:
             # one weight image, one forward and one dW call for gate and up
             nbp = dqt.dqt_bwd_dw_img_workspace_size(T, 2 * INTER, HID)
             self.launches_per_step = (2 + 2 + 2 + 3 + (1 + (1 if nbp > 0 else 0)) + dw[2])
+        if self.nimg:  # the images come from the update: no conversion launches
+            self.launches_per_step -= 2 if self.stack else 3
             if nbp > max(nbw, 16):
                 self.dw_ws = [torch.empty(nbp, dtype=torch.uint8, device=dev) for _ in range(4)]
             nbt = max(nbt, dqt.dqt_fwd_img_workspace_size(T, HID, 2 * INTER))
@@ -316,6 +334,9 @@ class MLPStep:
         from paper_2412_04787_gb300 import dp
         if self.packed or self.optimizer != "adamw":
             raise SystemExit("the data-parallel exchange runs the AdamW step on int8 codes")
+        if self.nimg:  # the shard update writes codes only: images by conversion again
+            self.nimg = False
+            self.launches_per_step += 2 if self.stack else 3
         self.dp = {}
         for name, _, _ in PROJ:
             upd = dp.DataParallelUpdater(self.W[name])
@@ -455,7 +476,7 @@ class MLPStep:
                 timed(self.dw_kind, stream, lambda: dqt.dqt_bitlinear_bwd_dw_update_img_pair(
                     self.d["dY_gu"], xdq, self.W_gu, INTER, self.s_w["gate"], self.s_w["up"],
                     self.m_gu, self.v_gu, hp, self.sr["gate"], self.sr["up"], self.grid,
-                    changed_out=ch, ws=ws))
+                    changed_out=ch, ws=ws, W_img_next=self.W_img_gu_next if self.nimg else None))
                 return
             if self.dp and not self.i8:
                 upd = self.dp[name]
@@ -520,10 +541,13 @@ class MLPStep:
                 ws = self.dw_ws[s.index(stream)]
                 timed(self.dw_kind, stream, lambda: dqt.dqt_bitlinear_bwd_dw_update_img(
                     self.d["dY_" + name], xdq, self.W[name], self.s_w[name], self.m[name],
-                    self.v[name], hp, self.sr[name], self.grid, changed_out=ch, ws=ws))
+                    self.v[name], hp, self.sr[name], self.grid, changed_out=ch, ws=ws,
+                    W_img_next=self.W_img_next[name] if self.nimg else None))
 
         for st in s:
             after(st, main)
+        if self.nimg:  # this step's images were written by the last step's updates
+            codes = lambda name, stream: None  # noqa: E731
         # forward: the three weight images convert while X is quantised (one
         # pass writes both the forward's code image and the dequantised image
         # the weight gradient reads: splitting it into two passes, the second
@@ -570,6 +594,10 @@ class MLPStep:
             dx("up", s[2])
         for st in s:
             after(main, st)
+        if self.nimg:  # the images the updates wrote serve the next step
+            self.W_img, self.W_img_next = self.W_img_next, self.W_img
+            if self.stack:
+                self.W_img_gu, self.W_img_gu_next = self.W_img_gu_next, self.W_img_gu
 
     # algorithmic work per launch, per kernel kind
     def work(self):
@@ -693,7 +721,8 @@ def run_gpu(args):
     dqt_build.build()
     st = MLPStep(dev, fp8=args.act == "fp8", optimizer=args.optimizer, packed=args.packed,
                  bits=args.bits, operands=args.operands, tail_slices=not args.no_tail_slices,
-                 stack_gate_up=stacked_gate_up(args, dp_mode))
+                 stack_gate_up=stacked_gate_up(args, dp_mode),
+                 next_image=not args.convert_images)
     if dp_mode == "exchange":
         st.enable_dp()
     dqt = st.dqt
@@ -1616,6 +1645,9 @@ def main():
                          "operands and AdamW on int8 codes, they are two stacked weights of one "
                          "forward call and one dW + update call, each weight with its own scale "
                          "and SR stream; dX per weight)")
+    ap.add_argument("--convert-images", action="store_true",
+                    help="mlp, image operands: convert the codes to bf16 images at the start of "
+                         "every step instead of taking the images the last step's updates wrote")
     ap.add_argument("--no-tail-slices", action="store_true",
                     help="the forward and dX GEMMs without a workspace, so their last wave is "
                          "not cut into reduction slices (A/B of that schedule; image operands)")

@@ -299,12 +299,18 @@ int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const int8_t* Xq, const floa
 size_t dqt_bwd_dw_workspace_size(int64_t T, int64_t N, int64_t K);
 
 /* The same weight gradient + update on the X_tilde image Xdq bf16 [T, K]
- * (dqt_act_quant_images); ws: the token-slice workspace below, or NULL. */
+ * (dqt_act_quant_images); ws: the token-slice workspace below, or NULL.
+ * W_img_next: NULL, or bf16 [N, K] (16-byte aligned) that receives the exact
+ * bf16 image of the updated codes (the next forward's and dX's operand, as
+ * dqt_codes_to_bf16 would write it), written by the update itself; it must
+ * not be the image any kernel still in flight reads (this step's dX): keep
+ * two images and alternate them step by step.  Needs W, m, v. */
 int dqt_bitlinear_bwd_dw_update_img(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W,
                                     float s_w, float* m, float* v, const dqt_adamw_t* hp,
                                     const dqt_sr_t* sr, dqt_grid_t grid, int64_t T, int64_t N,
-                                    int64_t K, float* dW_out, unsigned long long* changed_out,
-                                    void* ws, size_t ws_bytes, void* stream);
+                                    int64_t K, float* dW_out, dqt_bf16* W_img_next,
+                                    unsigned long long* changed_out, void* ws, size_t ws_bytes,
+                                    void* stream);
 
 /* Workspace (bytes, 16-byte aligned device memory) that lets
  * dqt_bitlinear_bwd_dw_update_img (and the rest of dqt_bitlinear_bwd_dw_update's
@@ -333,14 +339,15 @@ size_t dqt_bwd_dw_img_workspace_size(int64_t T, int64_t N, int64_t K);
  * its own first element, so codes, m and v equal those of two
  * dqt_bitlinear_bwd_dw_update_img calls computing the same gradients.  N0 a
  * multiple of 256, 0 < N0 < N; ws of dqt_bwd_dw_img_workspace_size(T, N, K)
- * bytes or NULL; changed_out counts both weights' changed codes. */
+ * bytes or NULL; W_img_next as for dqt_bitlinear_bwd_dw_update_img (both
+ * weights' rows); changed_out counts both weights' changed codes. */
 int dqt_bitlinear_bwd_dw_update_img_pair(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W,
                                          int64_t N0, float s_w0, float s_w1, float* m, float* v,
                                          const dqt_adamw_t* hp, const dqt_sr_t* sr0,
                                          const dqt_sr_t* sr1, dqt_grid_t grid, int64_t T,
                                          int64_t N, int64_t K, float* dW_out,
-                                         unsigned long long* changed_out, void* ws,
-                                         size_t ws_bytes, void* stream);
+                                         dqt_bf16* W_img_next, unsigned long long* changed_out,
+                                         void* ws, size_t ws_bytes, void* stream);
 
 /* The AdamW + SR update of dqt_bitlinear_bwd_dw_update for a gradient already
  * in memory (Eq. 5 as a bandwidth-bound stream; 22 bytes per weight):

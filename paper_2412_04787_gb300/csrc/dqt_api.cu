@@ -558,7 +558,7 @@ int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const int8_t* Xq, const floa
   if (dqt::launch_codes_to_xdq(Xq, s_x, T, K, Xdq, as_stream(stream))) return DQT_ERR_CUDA;
   uint8_t* rest = static_cast<uint8_t*>(ws) + img;
   const size_t rest_bytes = ws_bytes - img;
-  return dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, s_w, m, v, hp, sr, grid, T, N, K, dW_out,
+  return dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, s_w, m, v, hp, sr, grid, T, N, K, dW_out, nullptr,
                                          changed_out, rest_bytes ? rest : nullptr, rest_bytes,
                                          stream);
 }
@@ -566,16 +566,17 @@ int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const int8_t* Xq, const floa
 int dqt_bitlinear_bwd_dw_update_img(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W,
                                     float s_w, float* m, float* v, const dqt_adamw_t* hp,
                                     const dqt_sr_t* sr, dqt_grid_t grid, int64_t T, int64_t N,
-                                    int64_t K, float* dW_out, unsigned long long* changed_out,
-                                    void* ws, size_t ws_bytes, void* stream) {
+                                    int64_t K, float* dW_out, dqt_bf16* W_img_next,
+                                    unsigned long long* changed_out, void* ws, size_t ws_bytes,
+                                    void* stream) {
   const bool upd = W || m || v;
   if (!dY || !Xdq || T <= 0 || N <= 0 || K <= 0) return DQT_ERR_ARG;
   if (upd && (!W || !m || !v)) return DQT_ERR_ARG;
-  if (!upd && !dW_out) return DQT_ERR_ARG;
+  if (!upd && (!dW_out || W_img_next)) return DQT_ERR_ARG;
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
   if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(Xdq) || (W && !aligned16(W)) ||
       (m && !aligned16(m)) || (v && !aligned16(v)) || (dW_out && !aligned16(dW_out)) ||
-      (ws && !aligned16(ws)))
+      (W_img_next && !aligned16(W_img_next)) || (ws && !aligned16(ws)))
     return DQT_ERR_ALIGN;
   dqt::GemmLaunch g{};
   g.ws = ws;
@@ -594,6 +595,7 @@ int dqt_bitlinear_bwd_dw_update_img(const dqt_bf16* dY, const dqt_bf16* Xdq, int
   g.m = m;
   g.v = v;
   g.dW_out = dW_out;
+  g.img_next = W_img_next;
   g.changed = upd ? changed_out : nullptr;
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
@@ -603,13 +605,14 @@ int dqt_bitlinear_bwd_dw_update_img_pair(const dqt_bf16* dY, const dqt_bf16* Xdq
                                          const dqt_adamw_t* hp, const dqt_sr_t* sr0,
                                          const dqt_sr_t* sr1, dqt_grid_t grid, int64_t T,
                                          int64_t N, int64_t K, float* dW_out,
-                                         unsigned long long* changed_out, void* ws,
-                                         size_t ws_bytes, void* stream) {
+                                         dqt_bf16* W_img_next, unsigned long long* changed_out,
+                                         void* ws, size_t ws_bytes, void* stream) {
   if (!dY || !Xdq || !W || !m || !v || T <= 0 || N <= 0 || K <= 0 || !pair_split_ok(N0, N))
     return DQT_ERR_ARG;
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
   if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(Xdq) || !aligned16(W) || !aligned16(m) ||
-      !aligned16(v) || (dW_out && !aligned16(dW_out)) || (ws && !aligned16(ws)))
+      !aligned16(v) || (dW_out && !aligned16(dW_out)) ||
+      (W_img_next && !aligned16(W_img_next)) || (ws && !aligned16(ws)))
     return DQT_ERR_ALIGN;
   dqt::GemmLaunch g{};
   g.ws = ws;
@@ -628,6 +631,7 @@ int dqt_bitlinear_bwd_dw_update_img_pair(const dqt_bf16* dY, const dqt_bf16* Xdq
   g.m = m;
   g.v = v;
   g.dW_out = dW_out;
+  g.img_next = W_img_next;
   g.changed = changed_out;
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }

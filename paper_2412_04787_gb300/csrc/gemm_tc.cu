@@ -112,7 +112,14 @@ struct Params {
   // every wave re-reads (chosen when A's panels are the smaller set)
   int num_m;
   bool col_major;
+  // dW: if set, the bf16 image of every updated code is written here too
+  // (the next forward's operand), at the code's element index
+  __nv_bfloat16* img_next;
 };
+
+// The bf16 image of four codes (exact: integers of magnitude <= 128).
+__device__ __forceinline__ void store_code_image4(__nv_bfloat16* img, size_t e, int32_t a, int32_t b,
+                                                  int32_t c, int32_t d);
 
 // Row and column tile (256 x 256) of a 2-SM kernel's tile index.
 __device__ __forceinline__ int pair_tile_m(const Params& p, int tile) {
@@ -178,6 +185,13 @@ __device__ __forceinline__ void l2_discard_line(const void* p) {
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+__device__ __forceinline__ void store_code_image4(__nv_bfloat16* img, size_t e, int32_t a, int32_t b,
+                                                  int32_t c, int32_t d) {
+  __stcs(reinterpret_cast<uint2*>(img + e),
+         make_uint2(pack_bf16x2(static_cast<float>(a), static_cast<float>(b)),
+                    pack_bf16x2(static_cast<float>(c), static_cast<float>(d))));
 }
 
 // Warp-uniform bounded wait: every lane waits, the warp fails if any lane did.
@@ -359,6 +373,7 @@ __device__ __forceinline__ uint32_t dw_update(const Params& p, const UpdateConst
       __stcs(reinterpret_cast<char4*>(p.W + e),
              make_char4(static_cast<signed char>(n0c), static_cast<signed char>(n1c),
                         static_cast<signed char>(n2c), static_cast<signed char>(n3c)));
+    if (p.img_next) store_code_image4(p.img_next, e, n0c, n1c, n2c, n3c);
     __stcs(reinterpret_cast<float4*>(p.m + e), L.m[j]);
     __stcs(reinterpret_cast<float4*>(p.v + e), L.v[j]);
   }
@@ -411,6 +426,7 @@ __device__ __forceinline__ uint32_t dw_update_row(const Params& p, const UpdateC
     __stcs(reinterpret_cast<char4*>(p.W + e),
            make_char4(static_cast<signed char>(n0c), static_cast<signed char>(n1c),
                       static_cast<signed char>(n2c), static_cast<signed char>(n3c)));
+  if (p.img_next) store_code_image4(p.img_next, e, n0c, n1c, n2c, n3c);
   __stcs(reinterpret_cast<float4*>(p.m + e), L.m);
   __stcs(reinterpret_cast<float4*>(p.v + e), L.v);
   return (n0c != c.x) + (n1c != c.y) + (n2c != c.z) + (n3c != c.w);
@@ -1479,6 +1495,8 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   p.split = g.split;
   p.scale1 = g.scale1;
   p.uc1 = g.uc1;
+  p.img_next = g.kind == GEMM_DW ? static_cast<__nv_bfloat16*>(g.img_next) : nullptr;
+  if (p.img_next && (g.packed || !g.W)) return 1;
   // stacked weights: whole tiles (multiples of 256 of either tiling),
   // constants in the parameter space
   if (g.split > 0 && (g.split % 256 != 0 || g.uc_dev ||
@@ -1541,7 +1559,8 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
                                   (g.N + 255) / 256, g.M, g.N, g.W, g.packed, g.m, g.v, g.uc,
                                   g.uc_dev, g.changed, g.dW_out, stream,
                                   g.split > 0 ? &g.uc1 : nullptr, g.split,
-                                  (g.N + 255) / 256 > (g.M + 255) / 256);
+                                  (g.N + 255) / 256 > (g.M + 255) / 256,
+                                  static_cast<uint16_t*>(g.img_next));
       }
       // split-T: fp32 partials of each token slice into the workspace slabs,
       // then one streaming pass sums the slabs in slice order and applies the
@@ -1559,6 +1578,15 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
         // gradient only: sum the slabs into dW_out
         return launch_slab_sum(static_cast<const float*>(g.ws), p.splits, p.slab, g.dW_out,
                                stream);
+      }
+      if (g.img_next) {
+        // the update, then the image of the updated codes
+        GemmLaunch g3 = g;
+        g3.img_next = nullptr;
+        const int rc3 = launch_gemm(g3, stream);
+        if (rc3) return rc3;
+        return launch_codes_to_bf16(g.W, static_cast<int64_t>(g.M) * g.N,
+                                    static_cast<uint16_t*>(g.img_next), stream);
       }
       if (g.split > 0) {
         // stacked weights: the rows of each with its own constants

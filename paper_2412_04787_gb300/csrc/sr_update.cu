@@ -173,7 +173,7 @@ __global__ void __launch_bounds__(kThreads, 3)
                        float* __restrict__ v, const UpdateConsts uc_arg,
                        const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed,
                        float* __restrict__ dW_out, const UpdateConsts uc1, int split,
-                       bool col_major) {
+                       bool col_major, uint16_t* __restrict__ img_next) {
   const UpdateConsts uc = DEV ? *uc_dev : uc_arg;
   uint8_t* Wp = reinterpret_cast<uint8_t*>(W);
   const int64_t ngroups = static_cast<int64_t>(tail) * 16384;  // 256 x 256 / 4 per tile
@@ -237,6 +237,13 @@ __global__ void __launch_bounds__(kThreads, 3)
           *reinterpret_cast<char4*>(W + e) =
               make_char4(static_cast<signed char>(a), static_cast<signed char>(b),
                          static_cast<signed char>(c), static_cast<signed char>(d));
+        if (img_next) {  // the bf16 image of the new codes (exact)
+          const __nv_bfloat162 lo = __floats2bfloat162_rn(static_cast<float>(a), static_cast<float>(b));
+          const __nv_bfloat162 hi = __floats2bfloat162_rn(static_cast<float>(c), static_cast<float>(d));
+          __stcs(reinterpret_cast<uint2*>(img_next + e),
+                 make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
+                            *reinterpret_cast<const uint32_t*>(&hi)));
+        }
         __stcs(reinterpret_cast<float4*>(m + e), m4);
         __stcs(reinterpret_cast<float4*>(v + e), v4);
       }
@@ -319,7 +326,8 @@ int launch_sr_update_slabs(const float* slabs, int splits, long long slab, int8_
 int launch_tail_update(const float* part, int splits, int tail, int full, int num_n, int M, int N,
                        int8_t* W, bool packed, float* m, float* v, const UpdateConsts& uc,
                        const UpdateConsts* uc_dev, unsigned long long* changed, float* dW_out,
-                       cudaStream_t stream, const UpdateConsts* uc1, int split, bool col_major) {
+                       cudaStream_t stream, const UpdateConsts* uc1, int split, bool col_major,
+                       uint16_t* img_next) {
   const UpdateConsts u1 = uc1 ? *uc1 : uc;
   // the blocks that fit at once: each thread walks several groups, its next
   // group's loads in flight
@@ -341,12 +349,13 @@ int launch_tail_update(const float* part, int splits, int tail, int full, int nu
     tail_update_kernel<true><<<blocks, kThreads, 0, stream>>>(part, splits, tail, full, num_n, M, N,
                                                               W, packed, m, v, uc, uc_dev, changed,
                                                               dW_out, u1, uc1 ? split : 0,
-                                                              col_major);
+                                                              col_major, img_next);
   else
     tail_update_kernel<false><<<blocks, kThreads, 0, stream>>>(part, splits, tail, full, num_n, M,
                                                                N, W, packed, m, v, uc, nullptr,
                                                                changed, dW_out, u1,
-                                                               uc1 ? split : 0, col_major);
+                                                               uc1 ? split : 0, col_major,
+                                                               img_next);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 

@@ -105,7 +105,7 @@ def lib():
         L.dqt_bitlinear_bwd_dw_update_img_pair.argtypes = [
             _vp, _vp, _vp, _i64, _f32, _f32, _vp, _vp, C.POINTER(dqt_adamw_t),
             C.POINTER(dqt_sr_t), C.POINTER(dqt_sr_t), dqt_grid_t, _i64, _i64, _i64, _vp, _vp,
-            _vp, _sz, _vp]
+            _vp, _vp, _sz, _vp]
         L.dqt_fwd_img_workspace_size.argtypes = [_i64, _i64, _i64]
         L.dqt_fwd_img_workspace_size.restype = _sz
         L.dqt_bitlinear_bwd_dx.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp, _sz, _vp]
@@ -124,7 +124,7 @@ def lib():
         L.dqt_bitlinear_bwd_dw_update_img.argtypes = [_vp, _vp, _vp, _f32, _vp, _vp,
                                                       C.POINTER(dqt_adamw_t),
                                                       C.POINTER(dqt_sr_t), dqt_grid_t, _i64,
-                                                      _i64, _i64, _vp, _vp, _vp, _sz, _vp]
+                                                      _i64, _i64, _vp, _vp, _vp, _vp, _sz, _vp]
         L.dqt_bwd_dw_workspace_size.argtypes = [_i64, _i64, _i64]
         L.dqt_bwd_dw_workspace_size.restype = _sz
         L.dqt_bwd_dw_img_workspace_size.argtypes = [_i64, _i64, _i64]
@@ -538,12 +538,13 @@ def dqt_bitlinear_bwd_dw_update(dY, Xq, s_x, W, s_w, m, v, hp, sr, bits_or_grid,
 
 
 def dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, s_w, m, v, hp, sr, bits_or_grid, dW_out=None,
-                                    changed_out=None, ws=None, stream=None):
+                                    changed_out=None, ws=None, stream=None, W_img_next=None):
     """Fused dW GEMM + AdamW + stochastic rounding on the X_tilde image Xdq;
     W, m, v updated in place.  With W = m = v = None only dW_out is computed.
     `ws`: split-T workspace (uint8 CUDA tensor of dqt_bwd_dw_img_workspace_size
     bytes); None allocates it when the shape benefits, False forces the single
-    fused kernel."""
+    fused kernel.  W_img_next (bf16 [N, K]): receives the image of the updated
+    codes (not the image this step's dX reads)."""
     _need(dY, "dY", torch.bfloat16)
     T, N = dY.shape
     _need(Xdq, "Xdq", torch.bfloat16)
@@ -553,19 +554,20 @@ def dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, s_w, m, v, hp, sr, bits_or_grid,
     _opt(m, "m", torch.float32, (N, K))
     _opt(v, "v", torch.float32, (N, K))
     _opt(dW_out, "dW_out", torch.float32, (N, K))
+    _opt(W_img_next, "W_img_next", torch.bfloat16, (N, K))
     _opt(changed_out, "changed_out", torch.int64, (1,))
     ws, nws = _dw_workspace(T, N, K, dY.device, ws)
     _check(lib().dqt_bitlinear_bwd_dw_update_img(
         _ptr(dY), _ptr(Xdq), _ptr(W), float(s_w), _ptr(m), _ptr(v),
         C.byref(hp) if hp is not None else None, C.byref(sr) if sr is not None else None,
-        _grid(bits_or_grid), T, N, K, _ptr(dW_out), _ptr(changed_out), _ptr(ws), nws,
-        _stream(stream)), "dqt_bitlinear_bwd_dw_update_img")
+        _grid(bits_or_grid), T, N, K, _ptr(dW_out), _ptr(W_img_next), _ptr(changed_out),
+        _ptr(ws), nws, _stream(stream)), "dqt_bitlinear_bwd_dw_update_img")
     return W
 
 
 def dqt_bitlinear_bwd_dw_update_img_pair(dY, Xdq, W, N0, s_w0, s_w1, m, v, hp, sr0, sr1,
                                          bits_or_grid, dW_out=None, changed_out=None, ws=None,
-                                         stream=None):
+                                         stream=None, W_img_next=None):
     """The fused dW + update of two stacked weights (rows [0, N0) of W, m, v
     and columns [0, N0) of dY the first's, with s_w0 and sr0; the rest the
     second's, with s_w1 and sr1).  `ws` as dqt_bitlinear_bwd_dw_update_img."""
@@ -578,12 +580,14 @@ def dqt_bitlinear_bwd_dw_update_img_pair(dY, Xdq, W, N0, s_w0, s_w1, m, v, hp, s
     _need(m, "m", torch.float32, (N, K))
     _need(v, "v", torch.float32, (N, K))
     _opt(dW_out, "dW_out", torch.float32, (N, K))
+    _opt(W_img_next, "W_img_next", torch.bfloat16, (N, K))
     _opt(changed_out, "changed_out", torch.int64, (1,))
     ws, nws = _dw_workspace(T, N, K, dY.device, ws)
     _check(lib().dqt_bitlinear_bwd_dw_update_img_pair(
         _ptr(dY), _ptr(Xdq), _ptr(W), int(N0), float(s_w0), float(s_w1), _ptr(m), _ptr(v),
         C.byref(hp), C.byref(sr0), C.byref(sr1), _grid(bits_or_grid), T, N, K, _ptr(dW_out),
-        _ptr(changed_out), _ptr(ws), nws, _stream(stream)), "dqt_bitlinear_bwd_dw_update_img_pair")
+        _ptr(W_img_next), _ptr(changed_out), _ptr(ws), nws, _stream(stream)),
+           "dqt_bitlinear_bwd_dw_update_img_pair")
     return W
 
 

@@ -1,6 +1,7 @@
 """Two BitLinear weights that read the same input, stacked in one call (a
 LLaMA MLP's gate and up projections): dqt_bitlinear_fwd_img_pair and
-dqt_bitlinear_bwd_dw_update_img_pair.
+dqt_bitlinear_bwd_dw_update_img_pair; and the next-step weight image the
+update writes (W_img_next).
 
 Each weight keeps its own per-tensor scale (Eq. 2-3) and its own
 stochastic-rounding stream (Philox elements counted from its own first
@@ -144,3 +145,48 @@ def test_dw_update_pair_with_token_slices():
         outs.append(W)
     dqt.dqt_check_device_status()
     assert_fused_codes(outs[0].cpu().numpy(), outs[1].cpu().numpy(), "pair, sliced vs unsliced")
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("T,K,N,bits", [(4096, 2048, 5632, 1.58),  # 176 tiles: token slices + tail kernel
+                                        (256, 512, 520, 8),        # one wave, ragged N
+                                        (4096, 512, 512, 1.58)])   # split-T path (few tiles)
+def test_dw_update_writes_next_image(mode, T, K, N, bits):
+    """W_img_next: the update also writes the bf16 image of the codes it
+    writes, byte for byte what dqt_codes_to_bf16 makes of them."""
+    dqt.dqt_set_gemm_tiles(mode)
+    try:
+        X = inputs.normal((T, K), 1.0, seed=T + N, dtype=torch.bfloat16)
+        dY = inputs.normal((T, N), 1e-2, seed=T + 7, dtype=torch.bfloat16).cuda()
+        qmin, qmax = oracle.grid(bits)
+        c, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=N).numpy(), qmin, qmax)
+        _, s_x, _, Xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xdq",))
+        W = torch.from_numpy(c).cuda()
+        m = torch.zeros((N, K), device="cuda")
+        v = torch.zeros((N, K), device="cuda")
+        img = torch.full((N, K), float("nan"), dtype=torch.bfloat16, device="cuda")
+        dqt.dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, float(s_w), m, v, dqt.adamw(lr=1e-2),
+                                            dqt.sr_stream(seed=3), (qmin, qmax), W_img_next=img)
+        dqt.dqt_check_device_status()
+        assert not torch.equal(W.cpu(), torch.from_numpy(c))  # the update moved codes
+        assert torch.equal(img.view(torch.int16), dqt.dqt_codes_to_bf16(W).view(torch.int16))
+    finally:
+        dqt.dqt_set_gemm_tiles(0)
+
+
+def test_dw_update_pair_writes_next_image():
+    T, K, N0, N1 = 1024, 2048, 5632, 5632
+    N = N0 + N1
+    X = inputs.normal((T, K), 1.0, seed=11, dtype=torch.bfloat16)
+    dY = inputs.normal((T, N), 1e-2, seed=12, dtype=torch.bfloat16).cuda()
+    c, s0, s1, g = _weights(N0, N1, K, 1.58, seed=13)
+    _, s_x, _, Xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xdq",))
+    W = torch.from_numpy(c).cuda()
+    m = torch.zeros((N, K), device="cuda")
+    v = torch.zeros((N, K), device="cuda")
+    img = torch.empty((N, K), dtype=torch.bfloat16, device="cuda")
+    dqt.dqt_bitlinear_bwd_dw_update_img_pair(dY, Xdq, W, N0, s0, s1, m, v, dqt.adamw(lr=1e-2),
+                                             dqt.sr_stream(seed=1), dqt.sr_stream(seed=1, tensor_id=1),
+                                             g, W_img_next=img)
+    dqt.dqt_check_device_status()
+    assert torch.equal(img.view(torch.int16), dqt.dqt_codes_to_bf16(W).view(torch.int16))
