@@ -82,7 +82,9 @@ def kernel_fingerprint(files=GEMM_SOURCES):
 # reports null.
 # With gate and up stacked, the mean over the step's two dW launches (the
 # stacked gate/up call and the down call, each its GEMM and streaming kernel).
-DW_TRAFFIC_STACKED = {"b62587c26333": ((563893248 + 158965760)
+DW_TRAFFIC_STACKED = {"769ac7621d63": ((563601152 + 158165760)
+                                         + (259388672 + 57002752 + 33059840 + 3328)) // 2,
+                      "b62587c26333": ((563893248 + 158965760)
                                          + (259276032 + 57066240 + 33059328 + 256)) // 2}
 DW_TRAFFIC_BYTES = {"ac36c0aa63c5": 261135360 + 57050112 + 33049600,
                     "82d12725fdfa": 262571008 + 61169152 + 33047808,
@@ -323,6 +325,8 @@ class MLPStep:
                           ["act_quant", "codes_to_bf16", "fwd"]) + ["bwd_dx", self.dw_kind]
         if optimizer == "adafactor":
             self.launches_per_step += 3 * 6
+        if self.nimg:  # no conversion launches: the updates write the images
+            self.kinds = [k for k in self.kinds if k != "codes_to_bf16"]
         self.streams = [torch.cuda.Stream(device=dev) for _ in range(4)]
         self.dp = None
 
