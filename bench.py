@@ -327,7 +327,11 @@ class MLPStep:
             self.launches_per_step += 3 * 6
         if self.nimg:  # no conversion launches: the updates write the images
             self.kinds = [k for k in self.kinds if k != "codes_to_bf16"]
-        self.streams = [torch.cuda.Stream(device=dev) for _ in range(4)]
+        # streams 0-2 carry the step's critical chain (act_quant X -> gate/up
+        # forward -> act_quant H -> down forward -> down dX -> gate/up
+        # backward); the down projection's dW (stream 3) is off it, so its
+        # blocks take the SMs only when the chain leaves some free
+        self.streams = [torch.cuda.Stream(device=dev, priority=-1 if i < 3 else 0) for i in range(4)]
         self.dp = None
 
     def enable_dp(self):

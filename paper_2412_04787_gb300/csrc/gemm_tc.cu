@@ -61,6 +61,17 @@ constexpr int kEpiWarps = 8;
 constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr uint64_t kDrainNs = 1000000000ull;  // wait for in-flight copies/MMAs on abort
 
+// Philox4x32-10 (the generator of sr_words) for the elements of one update
+// call: the round keys and, in the first round, the product of counter word
+// 2 (the step) and word 3 (the weight tensor) are the same for every
+// element, so the host computes them once (philox_call_consts).
+struct PhiloxCall {
+  uint32_t rk[20];  // rk[2r], rk[2r + 1]: round r's keys, key0 + r W0 and key1 + r W1
+  uint32_t c0x;     // hi(M1 * step) ^ rk[0]: round 0's first output word before ^ counter word 1
+  uint32_t c0y;     // lo(M1 * step): round 0's second output word
+  uint32_t x3k;     // tensor id ^ rk[1]
+};
+
 struct Params {
   int M, N, Kred, num_kb, chunk_kb;
   int num_n, num_tiles;
@@ -115,6 +126,10 @@ struct Params {
   // dW: if set, the bf16 image of every updated code is written here too
   // (the next forward's operand), at the code's element index
   __nv_bfloat16* img_next;
+  // dW with the constants in the parameter space: the parts of the
+  // stochastic-rounding generator that are the same for every element of
+  // the call, for uc and uc1
+  PhiloxCall pc, pc1;
 };
 
 // The bf16 image of four codes (exact: integers of magnitude <= 128).
@@ -388,6 +403,93 @@ struct DwRow {
   uint32_t c;
 };
 
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
+// The four Philox words of block `blk` (elements 4 blk .. 4 blk + 3), equal
+// to sr_words(blk, step, tensor id, key0, key1) of the call's constants.
+__device__ __forceinline__ uint4 philox_call(uint64_t blk, const PhiloxCall& k) {
+  const uint32_t x0 = static_cast<uint32_t>(blk), x1 = static_cast<uint32_t>(blk >> 32);
+  const uint64_t p0 = static_cast<uint64_t>(0xD2511F53u) * x0;
+  uint4 c = make_uint4(k.c0x ^ x1, k.c0y, static_cast<uint32_t>(p0 >> 32) ^ k.x3k,
+                       static_cast<uint32_t>(p0));
+#pragma unroll
+  for (int r = 1; r < 10; ++r) {
+    const uint64_t q0 = static_cast<uint64_t>(0xD2511F53u) * c.x;
+    const uint64_t q1 = static_cast<uint64_t>(0xCD9E8D57u) * c.z;
+    c = make_uint4(static_cast<uint32_t>(q1 >> 32) ^ c.y ^ k.rk[2 * r], static_cast<uint32_t>(q1),
+                   static_cast<uint32_t>(q0 >> 32) ^ c.w ^ k.rk[2 * r + 1], static_cast<uint32_t>(q0));
+  }
+  return c;
+}
+
+// Two fp32 values in one 64-bit register, and the packed IEEE operations on
+// them (each half rounded to nearest on its own, exactly as the scalar
+// __fmul_rn / __fadd_rn / __fsub_rn).
+__device__ __forceinline__ uint64_t f2_pack(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ float2 f2_unpack(uint64_t r) {
+  float2 f;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(f.x), "=f"(f.y) : "l"(r));
+  return f;
+}
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_sub(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+// dqt_update_elem (stochastic rounding, round_mode 0) on two elements at
+// once: the same IEEE operations in the same order, the multiplications,
+// additions and subtractions two at a time; square root, division, floor
+// and the conversions one at a time.  Returns the two new codes; m and v
+// (two elements each) are updated in place.
+__device__ __forceinline__ int2 dqt_update_pair_sr(const UpdateConsts& h, float ga, float gb,
+                                                   int32_t ca, int32_t cb, float& ma, float& mb,
+                                                   float& va, float& vb, uint32_t wa, uint32_t wb) {
+  const uint64_t g2 = f2_pack(ga, gb);
+  const uint64_t mn2 = f2_add(f2_mul(f2_pack(h.b1, h.b1), f2_pack(ma, mb)),
+                              f2_mul(f2_pack(h.omb1, h.omb1), g2));
+  const uint64_t vn2 = f2_add(f2_mul(f2_pack(h.b2, h.b2), f2_pack(va, vb)),
+                              f2_mul(f2_pack(h.omb2, h.omb2), f2_mul(g2, g2)));
+  const float2 mn = f2_unpack(mn2), vn = f2_unpack(vn2);
+  ma = mn.x;
+  mb = mn.y;
+  va = vn.x;
+  vb = vn.y;
+  const uint64_t den2 = f2_add(f2_mul(f2_pack(__fsqrt_rn(vn.x), __fsqrt_rn(vn.y)), f2_pack(h.k1, h.k1)),
+                               f2_pack(h.k2, h.k2));
+  const float2 den = f2_unpack(den2);
+  const uint64_t u2 = f2_pack(__fdiv_rn(mn.x, den.x), __fdiv_rn(mn.y, den.y));
+  const uint64_t x2 = f2_sub(f2_mul(f2_pack(static_cast<float>(ca), static_cast<float>(cb)),
+                                    f2_pack(h.decay, h.decay)),
+                             f2_mul(f2_pack(h.lrs, h.lrs), u2));
+  const float2 x = f2_unpack(x2);
+  const float fa = floorf(x.x), fb = floorf(x.y);
+  const float2 frac = f2_unpack(f2_sub(x2, f2_pack(fa, fb)));
+  const float2 U = f2_unpack(f2_mul(f2_pack(static_cast<float>(wa >> 8), static_cast<float>(wb >> 8)),
+                                    f2_pack(5.9604644775390625e-08f, 5.9604644775390625e-08f)));
+  const int32_t ra = static_cast<int32_t>(fa) + (U.x < frac.x ? 1 : 0);
+  const int32_t rb = static_cast<int32_t>(fb) + (U.y < frac.y ? 1 : 0);
+  return make_int2(min(max(ra, h.qmin), h.qmax), min(max(rb, h.qmin), h.qmax));
+}
+
 template <bool PK>
 __device__ __forceinline__ void dw_load_row(const Params& p, int gm, int gk, DwRow& L) {
   if (!p.W || gk >= p.N || gm >= p.M) return;
@@ -398,9 +500,10 @@ __device__ __forceinline__ void dw_load_row(const Params& p, int gm, int gk, DwR
   L.v = __ldcs(reinterpret_cast<const float4*>(p.v + e));
 }
 
-template <bool PK>
+template <bool PK, bool FAST>
 __device__ __forceinline__ uint32_t dw_update_row(const Params& p, const UpdateConsts& uc,
-                                                  size_t e_off, float* dw_out, int gm, int gk,
+                                                  const PhiloxCall& pc, size_t e_off,
+                                                  float* dw_out, int gm, int gk,
                                                   const float* src, DwRow& L) {
   if (gk >= p.N || gm >= p.M) return 0;
   const size_t e = static_cast<size_t>(gm) * p.N + gk;
@@ -412,13 +515,24 @@ __device__ __forceinline__ uint32_t dw_update_row(const Params& p, const UpdateC
                                   static_cast<signed char>((L.c >> 8) & 0xFFu),
                                   static_cast<signed char>((L.c >> 16) & 0xFFu),
                                   static_cast<signed char>(L.c >> 24));
-  uint4 w = make_uint4(0, 0, 0, 0);
-  if (uc.round_mode == 0)
-    w = sr_words(global_blk(uc, (e - e_off) >> 2), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
-  const int32_t n0c = dqt_update_elem(uc, g4.x, c.x, L.m.x, L.v.x, w.x);
-  const int32_t n1c = dqt_update_elem(uc, g4.y, c.y, L.m.y, L.v.y, w.y);
-  const int32_t n2c = dqt_update_elem(uc, g4.z, c.z, L.m.z, L.v.z, w.z);
-  const int32_t n3c = dqt_update_elem(uc, g4.w, c.w, L.m.w, L.v.w, w.w);
+  int32_t n0c, n1c, n2c, n3c;
+  if (FAST && uc.round_mode == 0) {
+    const uint4 w = philox_call(global_blk(uc, (e - e_off) >> 2), pc);
+    const int2 a = dqt_update_pair_sr(uc, g4.x, g4.y, c.x, c.y, L.m.x, L.m.y, L.v.x, L.v.y, w.x, w.y);
+    const int2 b = dqt_update_pair_sr(uc, g4.z, g4.w, c.z, c.w, L.m.z, L.m.w, L.v.z, L.v.w, w.z, w.w);
+    n0c = a.x;
+    n1c = a.y;
+    n2c = b.x;
+    n3c = b.y;
+  } else {
+    uint4 w = make_uint4(0, 0, 0, 0);
+    if (uc.round_mode == 0)
+      w = sr_words(global_blk(uc, (e - e_off) >> 2), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
+    n0c = dqt_update_elem(uc, g4.x, c.x, L.m.x, L.v.x, w.x);
+    n1c = dqt_update_elem(uc, g4.y, c.y, L.m.y, L.v.y, w.y);
+    n2c = dqt_update_elem(uc, g4.z, c.z, L.m.z, L.v.z, w.z);
+    n3c = dqt_update_elem(uc, g4.w, c.w, L.m.w, L.v.w, w.w);
+  }
   if (PK)
     __stcs(reinterpret_cast<uint8_t*>(p.W) + (e >> 2),
            static_cast<uint8_t>(tern_pack4(n0c, n1c, n2c, n3c)));
@@ -449,9 +563,10 @@ __device__ __forceinline__ void dw_load_first(const Params& p, int row0, int nba
 // arrive in.  On entry L holds the tile's first half-chunk.  Half-chunk q
 // covers chunk q / 2 (32 columns at nbase + 32 (q / 2)), rows
 // (lane >> 3) + 4 (4 (q % 2) + j), j = 0..3, and columns 4 (lane & 7) .. + 3.
-template <bool PK>
+template <bool PK, bool FAST>
 __device__ __forceinline__ uint32_t epi_dw_tile_roll(const Params& p, const UpdateConsts& uc,
-                                                     size_t e_off, float* dw_out, int row0, int nbase,
+                                                     const PhiloxCall& pc, size_t e_off,
+                                                     float* dw_out, int row0, int nbase,
                                                      int nchunk, uint32_t t_acc, float* xp,
                                                      int lane, DwRow (&L)[4], int row0n,
                                                      int nbasen) {
@@ -477,8 +592,8 @@ __device__ __forceinline__ uint32_t epi_dw_tile_roll(const Params& p, const Upda
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const int r = (lane >> 3) + 4 * (4 * h + j);
-      n_changed += dw_update_row<PK>(p, uc, e_off, dw_out, row0 + r, gn0 + cq,
-                                     xp + r * kStageLd + cq, L[j]);
+      n_changed += dw_update_row<PK, FAST>(p, uc, pc, e_off, dw_out, row0 + r, gn0 + cq,
+                                           xp + r * kStageLd + cq, L[j]);
       if (nrow0 >= 0) dw_load_row<PK>(p, nrow0 + (lane >> 3) + 4 * (4 * nh + j), ngk, L[j]);
     }
     if (h == 1) __syncwarp();  // the transpose buffer is rewritten for the next chunk
@@ -879,6 +994,7 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
       uint32_t ph = 0;    // phase (it / ST) & 1
       bool ok = true;
       const uint64_t pol_b = EPI == GEMM_DW ? l2_policy_evict_last() : 0ull;
+      const uint64_t pol_f = EPI == GEMM_DW ? l2_policy_evict_first() : 0ull;
       for (int t = cid; t < p.num_tiles && ok; t += ncl) {
         const Unit un = decode_unit(p, t);
         const int tile = un.tile, kb0 = un.kb0, kb1 = un.kb1;
@@ -901,6 +1017,12 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
 #pragma unroll
             for (int j = 0; j < 2; ++j)
               tma_load_2d_pair_hint(&tmA, bar, a + j * MN_CHUNK_BYTES, m0 + 64 * j, k0, pol_b);
+          } else if (EPI == GEMM_DW) {
+            // row-major tiles: each dY panel is read by the one wave of
+            // clusters that shares it, then never again
+#pragma unroll
+            for (int j = 0; j < 2; ++j)
+              tma_load_2d_pair_hint(&tmA, bar, a + j * MN_CHUNK_BYTES, m0 + 64 * j, k0, pol_f);
           } else {
 #pragma unroll
             for (int j = 0; j < 2; ++j)
@@ -1177,12 +1299,12 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
         }
         // the second of two stacked weights: its constants, its own element count
         if (p.split > 0 && pair_tile_m(p, tile) * 256 >= p.split)
-          n_changed += epi_dw_tile_roll<PK>(p, p.uc1, static_cast<size_t>(p.split) * p.N, dw_out,
-                                            gm - lane, nbase, HALF / 32, t_acc, xp, lane, st,
-                                            row0n, nbasen);
+          n_changed += epi_dw_tile_roll<PK, !UCD>(p, p.uc1, p.pc1, static_cast<size_t>(p.split) * p.N,
+                                                  dw_out, gm - lane, nbase, HALF / 32, t_acc, xp,
+                                                  lane, st, row0n, nbasen);
         else
-          n_changed += epi_dw_tile_roll<PK>(p, uc, 0, dw_out, gm - lane, nbase, HALF / 32, t_acc,
-                                            xp, lane, st, row0n, nbasen);
+          n_changed += epi_dw_tile_roll<PK, !UCD>(p, uc, p.pc, 0, dw_out, gm - lane, nbase,
+                                                  HALF / 32, t_acc, xp, lane, st, row0n, nbasen);
         st_loaded = row0n >= 0;
       } else
 #pragma unroll 1
@@ -1370,6 +1492,9 @@ int dw_splits(int M, int N, int Kred) {
 
 namespace {
 
+// Launches that cut their last wave with slice counters (all GEMM kinds).
+std::atomic<unsigned long long> g_tail_launches{0};
+
 template <bool A_MN, bool B_MN, int EPI, bool PK, bool DR, bool UCD>
 int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream,
                  void* tail_ws, size_t tail_ws_bytes, TailPlan* plan) {
@@ -1431,10 +1556,15 @@ int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStr
       p.part = part;
       p.num_tiles = tp.full + tp.tail * tp.splits;
       if (EPI != GEMM_DW) {
-        static std::atomic<unsigned long long> tag{0};
+        // The launch's tag: the process's count of such launches (one count
+        // for every GEMM kind, so a forward's counters never carry a later
+        // dX launch's tag), spread over 47 bits by an odd multiplier
+        // (distinct for distinct counts below 2^47), with bit 47 set, so
+        // that no word a workspace held before -- a small integer such as a
+        // count, or a positive float -- reads as this launch's tag.
+        const unsigned long long n = g_tail_launches.fetch_add(1) + 1;
         p.tail_ctr = static_cast<unsigned long long*>(tail_ws);
-        p.tail_tag = (tag.fetch_add(1) + 1) & 0xFFFFFFFFFFFFull;  // 48 bits, never 0
-        if (p.tail_tag == 0) p.tail_tag = 1;
+        p.tail_tag = ((n * 0x9E3779B97F4A7C15ull) & 0x7FFFFFFFFFFFull) | 0x800000000000ull;
       }
       *plan = tp;
     }
@@ -1446,6 +1576,20 @@ int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStr
 }
 
 }  // namespace
+
+// The per-call Philox constants of PhiloxCall from the update constants.
+static PhiloxCall philox_call_consts(const UpdateConsts& uc) {
+  PhiloxCall k{};
+  for (int r = 0; r < 10; ++r) {
+    k.rk[2 * r] = uc.key0 + static_cast<uint32_t>(r) * 0x9E3779B9u;
+    k.rk[2 * r + 1] = uc.key1 + static_cast<uint32_t>(r) * 0xBB67AE85u;
+  }
+  const uint64_t p1 = static_cast<uint64_t>(0xCD9E8D57u) * uc.step_lo;
+  k.c0x = static_cast<uint32_t>(p1 >> 32) ^ k.rk[0];
+  k.c0y = static_cast<uint32_t>(p1);
+  k.x3k = uc.tensor_id ^ k.rk[1];
+  return k;
+}
 
 int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   Params p{};
@@ -1491,10 +1635,12 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   p.dW_out = g.dW_out;
   p.changed = g.changed;
   p.uc = g.uc;
+  p.pc = philox_call_consts(g.uc);
   p.uc_dev = g.uc_dev;
   p.split = g.split;
   p.scale1 = g.scale1;
   p.uc1 = g.uc1;
+  p.pc1 = philox_call_consts(g.uc1);
   p.img_next = g.kind == GEMM_DW ? static_cast<__nv_bfloat16*>(g.img_next) : nullptr;
   if (p.img_next && (g.packed || !g.W)) return 1;
   // stacked weights: whole tiles (multiples of 256 of either tiling),

@@ -126,3 +126,56 @@ def test_dx_cut_reproducible_and_within_tolerance(T, N, K, cut):
     ref = oracle.bwd_dx(bits(dY[torch.from_numpy(rows)]), c, np.float32(s_w))
     got = dX1[torch.from_numpy(rows).cuda()].cpu().double().numpy()
     assert float(np.abs(got - ref).max() / np.abs(ref).max()) <= REL_TOL
+
+
+def test_stale_workspace_words_never_count_as_slices():
+    """The slice counters need no reset: each launch tags its counts, and the
+    tag is spread over 48 bits with its top bit set, so words the workspace
+    held before -- counts, small integers, other launches' counters -- never
+    read as this launch's slices.  Here the workspace is filled with every
+    small integer and with words whose tag field holds small launch numbers."""
+    T, N, K = 8192, 5632, 2048
+    need = dqt.dqt_bwd_dx_img_workspace_size(T, N, K)
+    assert need > 0
+    dY = inputs.normal((T, N), 1e-2, seed=31, dtype=torch.bfloat16).cuda()
+    qmin, qmax = oracle.grid(1.58)
+    c, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=32).numpy(), qmin, qmax)
+    W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
+    ref = dqt.dqt_bitlinear_bwd_dx_img(dY, W_img, float(s_w), ws=False)
+    words = need // 8
+    i = torch.arange(words, dtype=torch.int64, device="cuda")
+    for fill in (i + 65536,                 # counts 65536.. (tag field 1, 2, ...)
+                 ((i % 64) << 16) | 1,      # tag field 0..63, one slice done
+                 ((i % 64) << 16) | 2):     # tag field 0..63, two slices done
+        ws = torch.empty(need, dtype=torch.uint8, device="cuda")
+        ws.view(torch.int64)[:words] = fill
+        got = dqt.dqt_bitlinear_bwd_dx_img(dY, W_img, float(s_w), ws=ws)
+        dqt.dqt_check_device_status()
+        a, b = got.float(), ref.float()
+        floor = float(torch.abs(b).max()) * 2.0 ** -16
+        assert bool((torch.abs(a - b) <= torch.abs(b) * 2.0 ** -7 + floor).all())
+
+
+def test_forward_then_dx_on_one_workspace():
+    """A forward and a dX that cut their last waves on the same workspace,
+    one after the other: the dX launch's counters start from the forward's
+    leftovers, which carry another launch's tag and count as zero."""
+    T, N, K = 8192, 5632, 2048  # dX reduces over N = 5632; the forward below over 5632 too
+    need = max(dqt.dqt_bwd_dx_img_workspace_size(T, N, K), dqt.dqt_fwd_img_workspace_size(T, N, K))
+    ws = torch.zeros(need, dtype=torch.uint8, device="cuda")
+    qmin, qmax = oracle.grid(1.58)
+    X = inputs.normal((T, N), 1.0, seed=41, dtype=torch.bfloat16)
+    cf, sf, _ = oracle.absmean_init(inputs.normal((K, N), 0.02, seed=42).numpy(), qmin, qmax)
+    _, s_x, q_img, _ = dqt.dqt_act_quant_images(X.cuda(), want=("Xq_img",))
+    Wf = dqt.dqt_codes_to_bf16(torch.from_numpy(cf).cuda())
+    dY = inputs.normal((T, N), 1e-2, seed=43, dtype=torch.bfloat16).cuda()
+    c, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=44).numpy(), qmin, qmax)
+    W_img = dqt.dqt_codes_to_bf16(torch.from_numpy(c).cuda())
+    ref = dqt.dqt_bitlinear_bwd_dx_img(dY, W_img, float(s_w), ws=False)
+    for _ in range(3):
+        dqt.dqt_bitlinear_fwd_img(q_img, s_x, Wf, float(sf), (qmin, qmax), ws=ws)
+        got = dqt.dqt_bitlinear_bwd_dx_img(dY, W_img, float(s_w), ws=ws)
+        dqt.dqt_check_device_status()
+        a, b = got.float(), ref.float()
+        floor = float(torch.abs(b).max()) * 2.0 ** -16
+        assert bool((torch.abs(a - b) <= torch.abs(b) * 2.0 ** -7 + floor).all())
