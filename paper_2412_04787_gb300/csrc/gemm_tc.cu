@@ -426,70 +426,6 @@ __device__ __forceinline__ uint4 philox_call(uint64_t blk, const PhiloxCall& k) 
   return c;
 }
 
-// Two fp32 values in one 64-bit register, and the packed IEEE operations on
-// them (each half rounded to nearest on its own, exactly as the scalar
-// __fmul_rn / __fadd_rn / __fsub_rn).
-__device__ __forceinline__ uint64_t f2_pack(float a, float b) {
-  uint64_t r;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
-  return r;
-}
-__device__ __forceinline__ float2 f2_unpack(uint64_t r) {
-  float2 f;
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(f.x), "=f"(f.y) : "l"(r));
-  return f;
-}
-__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
-  uint64_t d;
-  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
-  uint64_t d;
-  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-__device__ __forceinline__ uint64_t f2_sub(uint64_t a, uint64_t b) {
-  uint64_t d;
-  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-
-// dqt_update_elem (stochastic rounding, round_mode 0) on two elements at
-// once: the same IEEE operations in the same order, the multiplications,
-// additions and subtractions two at a time; square root, division, floor
-// and the conversions one at a time.  Returns the two new codes; m and v
-// (two elements each) are updated in place.
-__device__ __forceinline__ int2 dqt_update_pair_sr(const UpdateConsts& h, float ga, float gb,
-                                                   int32_t ca, int32_t cb, float& ma, float& mb,
-                                                   float& va, float& vb, uint32_t wa, uint32_t wb) {
-  const uint64_t g2 = f2_pack(ga, gb);
-  const uint64_t mn2 = f2_add(f2_mul(f2_pack(h.b1, h.b1), f2_pack(ma, mb)),
-                              f2_mul(f2_pack(h.omb1, h.omb1), g2));
-  const uint64_t vn2 = f2_add(f2_mul(f2_pack(h.b2, h.b2), f2_pack(va, vb)),
-                              f2_mul(f2_pack(h.omb2, h.omb2), f2_mul(g2, g2)));
-  const float2 mn = f2_unpack(mn2), vn = f2_unpack(vn2);
-  ma = mn.x;
-  mb = mn.y;
-  va = vn.x;
-  vb = vn.y;
-  const uint64_t den2 = f2_add(f2_mul(f2_pack(__fsqrt_rn(vn.x), __fsqrt_rn(vn.y)), f2_pack(h.k1, h.k1)),
-                               f2_pack(h.k2, h.k2));
-  const float2 den = f2_unpack(den2);
-  const uint64_t u2 = f2_pack(__fdiv_rn(mn.x, den.x), __fdiv_rn(mn.y, den.y));
-  const uint64_t x2 = f2_sub(f2_mul(f2_pack(static_cast<float>(ca), static_cast<float>(cb)),
-                                    f2_pack(h.decay, h.decay)),
-                             f2_mul(f2_pack(h.lrs, h.lrs), u2));
-  const float2 x = f2_unpack(x2);
-  const float fa = floorf(x.x), fb = floorf(x.y);
-  const float2 frac = f2_unpack(f2_sub(x2, f2_pack(fa, fb)));
-  const float2 U = f2_unpack(f2_mul(f2_pack(static_cast<float>(wa >> 8), static_cast<float>(wb >> 8)),
-                                    f2_pack(5.9604644775390625e-08f, 5.9604644775390625e-08f)));
-  const int32_t ra = static_cast<int32_t>(fa) + (U.x < frac.x ? 1 : 0);
-  const int32_t rb = static_cast<int32_t>(fb) + (U.y < frac.y ? 1 : 0);
-  return make_int2(min(max(ra, h.qmin), h.qmax), min(max(rb, h.qmin), h.qmax));
-}
-
 template <bool PK>
 __device__ __forceinline__ void dw_load_row(const Params& p, int gm, int gk, DwRow& L) {
   if (!p.W || gk >= p.N || gm >= p.M) return;
@@ -515,24 +451,14 @@ __device__ __forceinline__ uint32_t dw_update_row(const Params& p, const UpdateC
                                   static_cast<signed char>((L.c >> 8) & 0xFFu),
                                   static_cast<signed char>((L.c >> 16) & 0xFFu),
                                   static_cast<signed char>(L.c >> 24));
-  int32_t n0c, n1c, n2c, n3c;
-  if (FAST && uc.round_mode == 0) {
-    const uint4 w = philox_call(global_blk(uc, (e - e_off) >> 2), pc);
-    const int2 a = dqt_update_pair_sr(uc, g4.x, g4.y, c.x, c.y, L.m.x, L.m.y, L.v.x, L.v.y, w.x, w.y);
-    const int2 b = dqt_update_pair_sr(uc, g4.z, g4.w, c.z, c.w, L.m.z, L.m.w, L.v.z, L.v.w, w.z, w.w);
-    n0c = a.x;
-    n1c = a.y;
-    n2c = b.x;
-    n3c = b.y;
-  } else {
-    uint4 w = make_uint4(0, 0, 0, 0);
-    if (uc.round_mode == 0)
-      w = sr_words(global_blk(uc, (e - e_off) >> 2), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
-    n0c = dqt_update_elem(uc, g4.x, c.x, L.m.x, L.v.x, w.x);
-    n1c = dqt_update_elem(uc, g4.y, c.y, L.m.y, L.v.y, w.y);
-    n2c = dqt_update_elem(uc, g4.z, c.z, L.m.z, L.v.z, w.z);
-    n3c = dqt_update_elem(uc, g4.w, c.w, L.m.w, L.v.w, w.w);
-  }
+  uint4 w = make_uint4(0, 0, 0, 0);
+  if (uc.round_mode == 0)
+    w = FAST ? philox_call(global_blk(uc, (e - e_off) >> 2), pc)
+             : sr_words(global_blk(uc, (e - e_off) >> 2), uc.step_lo, uc.tensor_id, uc.key0, uc.key1);
+  const int32_t n0c = dqt_update_elem(uc, g4.x, c.x, L.m.x, L.v.x, w.x);
+  const int32_t n1c = dqt_update_elem(uc, g4.y, c.y, L.m.y, L.v.y, w.y);
+  const int32_t n2c = dqt_update_elem(uc, g4.z, c.z, L.m.z, L.v.z, w.z);
+  const int32_t n3c = dqt_update_elem(uc, g4.w, c.w, L.m.w, L.v.w, w.w);
   if (PK)
     __stcs(reinterpret_cast<uint8_t*>(p.W) + (e >> 2),
            static_cast<uint8_t>(tern_pack4(n0c, n1c, n2c, n3c)));

@@ -397,7 +397,7 @@ def _fused(T, K, N, bits_w, step, seed, rows=None):
     vr = vg.cpu().numpy()[rows]
     assert np.abs(mr - m1).max() <= 1e-3 * np.abs(m1).max()
     assert np.abs(vr - v1).max() <= 1e-3 * np.abs(v1).max()
-    return Wg, dW, c, s_w, m, v, hp, sr, g, changed
+    return Wg, dW, c, s_w, m, v, hp, sr, g, changed, mg, vg
 
 
 @pytest.mark.parametrize("bits_w,step", [(1.58, 1), (8, 1), (8, 5), (1.58, 5)])
@@ -451,21 +451,26 @@ def test_fused_update_beyond_int32_sampled():
 
 def test_fused_equals_standalone_on_same_gradient():
     """Fused epilogue and standalone kernel draw the same uniforms for the same
-    element: given the fused kernel's own fp32 gradient, codes are identical."""
-    Wg, dW, c, s_w, m, v, hp, sr, g, changed = _fused(256, 512, 512, 8, 3, seed=61)
-    W2, m2, v2 = torch.from_numpy(c).cuda(), m.clone().cuda(), v.clone().cuda()
-    ch2 = torch.zeros(1, dtype=torch.int64, device="cuda")
-    dqt.dqt_sr_update(dW.reshape(-1), W2.reshape(-1), s_w, m2.reshape(-1), v2.reshape(-1), hp, sr,
-                      g, changed_out=ch2)
-    dqt.dqt_check_device_status()
-    assert torch.equal(W2, Wg)
-    assert int(ch2.item()) == int(changed.item())
+    element and evaluate the update in the same IEEE operations: given the
+    fused kernel's own fp32 gradient, codes, moments and the changed-code
+    count are identical, bit for bit (at one ragged shape as well)."""
+    for T, K, N, seed in ((256, 512, 512, 61), (256, 264, 520, 62)):
+        Wg, dW, c, s_w, m, v, hp, sr, g, changed, mg, vg = _fused(T, K, N, 8, 3, seed=seed)
+        W2, m2, v2 = torch.from_numpy(c).cuda(), m.clone().cuda(), v.clone().cuda()
+        ch2 = torch.zeros(1, dtype=torch.int64, device="cuda")
+        dqt.dqt_sr_update(dW.reshape(-1), W2.reshape(-1), s_w, m2.reshape(-1), v2.reshape(-1), hp,
+                          sr, g, changed_out=ch2)
+        dqt.dqt_check_device_status()
+        assert torch.equal(W2, Wg)
+        assert torch.equal(m2.view(torch.int32), mg.view(torch.int32))
+        assert torch.equal(v2.view(torch.int32), vg.view(torch.int32))
+        assert int(ch2.item()) == int(changed.item())
 
 
 def test_update_frequency_counter_ternary_step1():
     """Sec. 5.2 hook: the changed-code counter equals the number of codes that
     moved, and at step 1 the ternary rate is close to lr * s_w per movable code."""
-    Wg, dW, c, s_w, m, v, hp, sr, g, changed = _fused(256, 512, 512, 1.58, 1, seed=71)
+    Wg, dW, c, s_w, m, v, hp, sr, g, changed, _, _ = _fused(256, 512, 512, 1.58, 1, seed=71)
     moved = int((Wg.cpu().numpy() != c).sum())
     assert int(changed.item()) == moved
     rate = moved / c.size
