@@ -180,8 +180,7 @@ class MLPStep:
         # gate and up as two stacked weights of one call (the forward and the
         # fused dW + update; dX stays per weight): image operands, AdamW, int8
         # codes
-        self.stack = (stack_gate_up and not self.i8 and not fp8 and not packed
-                      and optimizer == "adamw")
+        self.stack = stack_gate_up and not self.i8 and not packed and optimizer == "adamw"
         self.grid = dqt.grid(bits)
         T = T_TOK
         # two seeded input sets, alternated step by step, so that the
@@ -214,6 +213,8 @@ class MLPStep:
             self.m_gu = torch.zeros((2 * INTER, HID), dtype=torch.float32, device=dev)
             self.v_gu = torch.zeros((2 * INTER, HID), dtype=torch.float32, device=dev)
             self.W_img_gu = torch.empty((2 * INTER, HID), dtype=torch.bfloat16, device=dev)
+            if fp8:
+                self.W8_gu = torch.empty((2 * INTER, HID), dtype=torch.uint8, device=dev)
             self.Y_gu = torch.empty((T, 2 * INTER), dtype=torch.bfloat16, device=dev)
         for i, (name, K, N) in enumerate(PROJ):
             W0 = inputs.normal((N, K), 0.02, seed=20 + i).to(dev)
@@ -225,6 +226,8 @@ class MLPStep:
                 self.W[name] = self.W_gu[half]
                 self.m[name], self.v[name] = self.m_gu[half], self.v_gu[half]
                 self.W_img[name] = self.W_img_gu[half]
+                if fp8:
+                    self.W8[name] = self.W8_gu[half]
                 self.Y[name] = self.Y_gu[:, half]
                 self.dX[name] = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
                 continue
@@ -246,18 +249,28 @@ class MLPStep:
         # writes the image of the codes it updates into the second of two
         # image buffers (the next step's forward and dX operand), so that no
         # step converts codes to images; the buffers swap after every step
-        self.nimg = next_image and not self.i8 and not fp8 and not packed and optimizer == "adamw"
+        # (with the FP8 forward, the E4M3 image of the forward beside the bf16
+        # image of dX, both written by the update)
+        self.nimg = next_image and not self.i8 and not packed and optimizer == "adamw"
         if self.nimg:
-            self.W_img_next = {}
+            self.W_img_next, self.W8_next = {}, {}
             if self.stack:
                 self.W_img_gu_next = torch.empty_like(self.W_img_gu)
+                if fp8:
+                    self.W8_gu_next = torch.empty_like(self.W8_gu)
             for name, K, N in PROJ:
                 if self.stack and name in ("gate", "up"):
                     half = slice(0, INTER) if name == "gate" else slice(INTER, 2 * INTER)
                     self.W_img_next[name] = self.W_img_gu_next[half]
+                    if fp8:
+                        self.W8_next[name] = self.W8_gu_next[half]
                 else:
                     self.W_img_next[name] = torch.empty((N, K), dtype=torch.bfloat16, device=dev)
+                    if fp8:
+                        self.W8_next[name] = torch.empty((N, K), dtype=torch.uint8, device=dev)
                 dqt.dqt_codes_to_bf16(self.W[name], self.W_img[name])  # the first step's images
+                if fp8:
+                    dqt.dqt_codes_to_fp8(self.W[name], self.grid, self.W8[name])
         # per activation: (scale, forward operand, dequantised bf16 image); the
         # forward operand is the int8 codes (no image), the bf16 code image,
         # or the E4M3 bytes with fp8
@@ -308,16 +321,18 @@ class MLPStep:
         # launch of its own)
         self.launches_per_step = 2 + 3 + 3 + 3 + sum(dw) + (3 if fp8 else 0) + (6 if self.i8 else 0)
         if self.stack:
-            # one weight image, one forward and one dW call for gate and up
+            # one weight image (two with FP8), one forward and one dW call for
+            # gate and up
             nbp = dqt.dqt_bwd_dw_img_workspace_size(T, 2 * INTER, HID)
-            self.launches_per_step = (2 + 2 + 2 + 3 + (1 + (1 if nbp > 0 else 0)) + dw[2])
-        if self.nimg:  # the images come from the update: no conversion launches
-            self.launches_per_step -= 2 if self.stack else 3
+            self.launches_per_step = (2 + self.conversions() + 2 + 3 + (1 + (1 if nbp > 0 else 0))
+                                      + dw[2])
             if nbp > max(nbw, 16):
                 self.dw_ws = [torch.empty(nbp, dtype=torch.uint8, device=dev) for _ in range(4)]
             nbt = max(nbt, dqt.dqt_fwd_img_workspace_size(T, HID, 2 * INTER))
             self.tail_ws = [torch.empty(max(nbt, 16), dtype=torch.uint8, device=dev)
                             if nbt and tail_slices else False for _ in range(4)]
+        if self.nimg:  # the images come from the update: no conversion launches
+            self.launches_per_step -= self.conversions()
         self.dw_kind = "bwd_dw_adafactor" if optimizer == "adafactor" else "bwd_dw_update"
         if self.i8:
             self.kinds = ["act_quant", "codes_to_bf16", "fwd", "bwd_dx", "codes_to_xdq",
@@ -328,13 +343,20 @@ class MLPStep:
         if optimizer == "adafactor":
             self.launches_per_step += 3 * 6
         if self.nimg:  # no conversion launches: the updates write the images
-            self.kinds = [k for k in self.kinds if k != "codes_to_bf16"]
+            self.kinds = [k for k in self.kinds if k not in ("codes_to_bf16", "codes_to_fp8")]
+
         # streams 0-2 carry the step's critical chain (act_quant X -> gate/up
         # forward -> act_quant H -> down forward -> down dX -> gate/up
         # backward); the down projection's dW (stream 3) is off it, so its
         # blocks take the SMs only when the chain leaves some free
         self.streams = [torch.cuda.Stream(device=dev, priority=-1 if i < 3 else 0) for i in range(4)]
         self.dp = None
+
+    def conversions(self):
+        """Weight-image conversion launches per step with image operands: one
+        per weight buffer (gate and up stacked: one buffer), twice with the
+        FP8 forward (E4M3 and bf16)."""
+        return (2 if self.stack else 3) * (2 if self.fp8 else 1)
 
     def enable_dp(self):
         """Data-parallel exchange per weight (one rank per GPU): the dW GEMM
@@ -345,8 +367,8 @@ class MLPStep:
         if self.packed or self.optimizer != "adamw":
             raise SystemExit("the data-parallel exchange runs the AdamW step on int8 codes")
         if self.nimg:  # the shard update writes codes only: images by conversion again
+            self.launches_per_step += self.conversions()
             self.nimg = False
-            self.launches_per_step += 2 if self.stack else 3
         self.dp = {}
         for name, _, _ in PROJ:
             upd = dp.DataParallelUpdater(self.W[name])
@@ -413,6 +435,9 @@ class MLPStep:
 
         def codes(name, stream):
             if name == "gate_up":  # both stacked weights' image in one launch
+                if self.fp8:
+                    timed("codes_to_fp8", stream,
+                          lambda: dqt.dqt_codes_to_fp8(self.W_gu, self.grid, self.W8_gu))
                 timed("codes_to_bf16", stream,
                       lambda: dqt.dqt_codes_to_bf16(self.W_gu, self.W_img_gu))
                 return
@@ -427,6 +452,11 @@ class MLPStep:
 
         def fwd(name, stream):
             s_x, q_img, _ = self.aq["H" if name == "down" else "X"]
+            if name == "gate_up" and self.fp8:  # the stacked E4M3 weights
+                timed("fwd_fp8", stream, lambda: dqt.dqt_bitlinear_fwd_fp8_pair(
+                    q_img, s_x, self.W8_gu, INTER, self.s_w["gate"], self.s_w["up"], self.grid,
+                    Y=self.Y_gu))
+                return
             if name == "gate_up":  # the stacked weights, [gate | up] in one output
                 timed("fwd", stream, lambda: dqt.dqt_bitlinear_fwd_img_pair(
                     q_img, s_x, self.W_img_gu, INTER, self.s_w["gate"], self.s_w["up"], self.grid,
@@ -486,7 +516,8 @@ class MLPStep:
                 timed(self.dw_kind, stream, lambda: dqt.dqt_bitlinear_bwd_dw_update_img_pair(
                     self.d["dY_gu"], xdq, self.W_gu, INTER, self.s_w["gate"], self.s_w["up"],
                     self.m_gu, self.v_gu, hp, self.sr["gate"], self.sr["up"], self.grid,
-                    changed_out=ch, ws=ws, W_img_next=self.W_img_gu_next if self.nimg else None))
+                    changed_out=ch, ws=ws, W_img_next=self.W_img_gu_next if self.nimg else None,
+                    W8_next=self.W8_gu_next if self.nimg and self.fp8 else None))
                 return
             if self.dp and not self.i8:
                 upd = self.dp[name]
@@ -552,7 +583,8 @@ class MLPStep:
                 timed(self.dw_kind, stream, lambda: dqt.dqt_bitlinear_bwd_dw_update_img(
                     self.d["dY_" + name], xdq, self.W[name], self.s_w[name], self.m[name],
                     self.v[name], hp, self.sr[name], self.grid, changed_out=ch, ws=ws,
-                    W_img_next=self.W_img_next[name] if self.nimg else None))
+                    W_img_next=self.W_img_next[name] if self.nimg else None,
+                    W8_next=self.W8_next[name] if self.nimg and self.fp8 else None))
 
         for st in s:
             after(st, main)
@@ -608,6 +640,10 @@ class MLPStep:
             self.W_img, self.W_img_next = self.W_img_next, self.W_img
             if self.stack:
                 self.W_img_gu, self.W_img_gu_next = self.W_img_gu_next, self.W_img_gu
+            if self.fp8:
+                self.W8, self.W8_next = self.W8_next, self.W8
+                if self.stack:
+                    self.W8_gu, self.W8_gu_next = self.W8_gu_next, self.W8_gu
 
     # algorithmic work per launch, per kernel kind
     def work(self):
@@ -644,7 +680,8 @@ class MLPStep:
                               [3.0 * T * K for _, K, N in PROJ]) if self.i8 else
                              [3.0 * HID * 2 * INTER, 3.0 * INTER * HID] if self.stack else
                              [(2.25 if self.packed else 3.0) * K * N for _, K, N in PROJ],
-            "codes_to_fp8": [(1.25 if self.packed else 2.0) * K * N for _, K, N in PROJ],
+            "codes_to_fp8": [2.0 * HID * 2 * INTER, 2.0 * INTER * HID] if self.stack else
+                            [(1.25 if self.packed else 2.0) * K * N for _, K, N in PROJ],
             # int8 codes read, bf16 image written, s_x read (gate, up: X; down: H)
             "codes_to_xdq": [3.0 * T * K + 4 * T for _, K, N in PROJ],
         }
@@ -1097,7 +1134,7 @@ def stacked_gate_up(args, dp_mode="replicas"):
     """Whether the MLP step runs gate and up as two stacked weights (one
     forward call, one dW + update call; MLPStep's condition; the data-parallel
     exchange keeps one weight per exchange)."""
-    return (not args.separate_gate_up and args.operands == "img" and args.act != "fp8"
+    return (not args.separate_gate_up and args.operands == "img"
             and not args.packed and args.optimizer == "adamw" and dp_mode != "exchange")
 
 

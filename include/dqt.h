@@ -304,13 +304,17 @@ size_t dqt_bwd_dw_workspace_size(int64_t T, int64_t N, int64_t K);
  * bf16 image of the updated codes (the next forward's and dX's operand, as
  * dqt_codes_to_bf16 would write it), written by the update itself; it must
  * not be the image any kernel still in flight reads (this step's dX): keep
- * two images and alternate them step by step.  Needs W, m, v. */
+ * two images and alternate them step by step.  W8_next: NULL, or uint8
+ * [N, K] (16-byte aligned) that receives the E4M3 image of the updated codes
+ * (the next FP8 forward's operand, as dqt_codes_to_fp8 would write it), under
+ * the same rule; only for grids whose codes stay within 16 in magnitude,
+ * else DQT_ERR_RANGE.  Each of the two images needs W, m, v. */
 int dqt_bitlinear_bwd_dw_update_img(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W,
                                     float s_w, float* m, float* v, const dqt_adamw_t* hp,
                                     const dqt_sr_t* sr, dqt_grid_t grid, int64_t T, int64_t N,
                                     int64_t K, float* dW_out, dqt_bf16* W_img_next,
-                                    unsigned long long* changed_out, void* ws, size_t ws_bytes,
-                                    void* stream);
+                                    uint8_t* W8_next, unsigned long long* changed_out, void* ws,
+                                    size_t ws_bytes, void* stream);
 
 /* Workspace (bytes, 16-byte aligned device memory) that lets
  * dqt_bitlinear_bwd_dw_update_img (and the rest of dqt_bitlinear_bwd_dw_update's
@@ -339,15 +343,16 @@ size_t dqt_bwd_dw_img_workspace_size(int64_t T, int64_t N, int64_t K);
  * its own first element, so codes, m and v equal those of two
  * dqt_bitlinear_bwd_dw_update_img calls computing the same gradients.  N0 a
  * multiple of 256, 0 < N0 < N; ws of dqt_bwd_dw_img_workspace_size(T, N, K)
- * bytes or NULL; W_img_next as for dqt_bitlinear_bwd_dw_update_img (both
- * weights' rows); changed_out counts both weights' changed codes. */
+ * bytes or NULL; W_img_next and W8_next as for dqt_bitlinear_bwd_dw_update_img
+ * (both weights' rows); changed_out counts both weights' changed codes. */
 int dqt_bitlinear_bwd_dw_update_img_pair(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W,
                                          int64_t N0, float s_w0, float s_w1, float* m, float* v,
                                          const dqt_adamw_t* hp, const dqt_sr_t* sr0,
                                          const dqt_sr_t* sr1, dqt_grid_t grid, int64_t T,
                                          int64_t N, int64_t K, float* dW_out,
-                                         dqt_bf16* W_img_next, unsigned long long* changed_out,
-                                         void* ws, size_t ws_bytes, void* stream);
+                                         dqt_bf16* W_img_next, uint8_t* W8_next,
+                                         unsigned long long* changed_out, void* ws,
+                                         size_t ws_bytes, void* stream);
 
 /* The AdamW + SR update of dqt_bitlinear_bwd_dw_update for a gradient already
  * in memory (Eq. 5 as a bandwidth-bound stream; 22 bytes per weight):
@@ -418,6 +423,16 @@ int dqt_codes_to_fp8(const int8_t* W, int64_t numel, dqt_grid_t grid, uint8_t* W
 int dqt_bitlinear_fwd_fp8(const uint8_t* Xq8, const float* s_x8, const uint8_t* W8, float s_w,
                           dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
                           float* acc_out, void* stream);
+
+/* dqt_bitlinear_fwd_fp8 for two stacked weights that read the same input (a
+ * LLaMA MLP's gate and up projections): W8 uint8 [N, K] holds both weights'
+ * E4M3 images (rows [0, N0) the first's), Y bf16 [T, N] both outputs side by
+ * side, the columns [0, N0) scaled with s_w0 and the rest with s_w1: Y and
+ * acc_out equal two dqt_bitlinear_fwd_fp8 calls', bit for bit.  N0 a multiple
+ * of 256, 0 < N0 < N; the rest as for dqt_bitlinear_fwd_fp8. */
+int dqt_bitlinear_fwd_fp8_pair(const uint8_t* Xq8, const float* s_x8, const uint8_t* W8, int64_t N0,
+                               float s_w0, float s_w1, dqt_grid_t grid, int64_t T, int64_t K,
+                               int64_t N, dqt_bf16* Y, float* acc_out, void* stream);
 
 /* ---- 2-bit packed ternary codes (Sec. 1: ternary weights need a fraction of
  * a byte each; 4 codes per byte here, 0.25 GB per 1B weights) ----------------

@@ -444,6 +444,35 @@ int dqt_bitlinear_fwd_fp8(const uint8_t* Xq8, const float* s_x8, const uint8_t* 
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
+int dqt_bitlinear_fwd_fp8_pair(const uint8_t* Xq8, const float* s_x8, const uint8_t* W8, int64_t N0,
+                               float s_w0, float s_w1, dqt_grid_t grid, int64_t T, int64_t K,
+                               int64_t N, dqt_bf16* Y, float* acc_out, void* stream) {
+  if (!Xq8 || !s_x8 || !W8 || !Y || T <= 0 || K <= 0 || N <= 0 || !grid_ok(grid) ||
+      !(s_w0 > 0.0f) || !isfinite(s_w0) || !(s_w1 > 0.0f) || !isfinite(s_w1) ||
+      !pair_split_ok(N0, N))
+    return DQT_ERR_ARG;
+  if (grid.qmin < -16 || grid.qmax > 16) return DQT_ERR_RANGE;
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
+  if (K % 16 || N % 8 || !aligned16(Xq8) || !aligned16(W8) || !aligned16(Y) ||
+      (acc_out && !aligned16(acc_out)))
+    return DQT_ERR_ALIGN;
+  dqt::GemmLaunch g{};
+  g.kind = dqt::GEMM_FWD8;
+  g.M = static_cast<int>(T);
+  g.N = static_cast<int>(N);
+  g.Kred = static_cast<int>(K);
+  g.A = Xq8;
+  g.B = W8;
+  g.pair = true;
+  g.s_x = s_x8;
+  g.scale = s_w0;
+  g.split = static_cast<int>(N0);
+  g.scale1 = s_w1;
+  g.out_bf16 = Y;
+  g.acc_f32 = acc_out;
+  return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
 static inline size_t ws_align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 size_t dqt_bwd_dx_workspace_size(int64_t T, int64_t N, int64_t K) {
@@ -559,7 +588,7 @@ int dqt_bitlinear_bwd_dw_update(const dqt_bf16* dY, const int8_t* Xq, const floa
   uint8_t* rest = static_cast<uint8_t*>(ws) + img;
   const size_t rest_bytes = ws_bytes - img;
   return dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, s_w, m, v, hp, sr, grid, T, N, K, dW_out, nullptr,
-                                         changed_out, rest_bytes ? rest : nullptr, rest_bytes,
+                                         nullptr, changed_out, rest_bytes ? rest : nullptr, rest_bytes,
                                          stream);
 }
 
@@ -567,16 +596,18 @@ int dqt_bitlinear_bwd_dw_update_img(const dqt_bf16* dY, const dqt_bf16* Xdq, int
                                     float s_w, float* m, float* v, const dqt_adamw_t* hp,
                                     const dqt_sr_t* sr, dqt_grid_t grid, int64_t T, int64_t N,
                                     int64_t K, float* dW_out, dqt_bf16* W_img_next,
-                                    unsigned long long* changed_out, void* ws, size_t ws_bytes,
-                                    void* stream) {
+                                    uint8_t* W8_next, unsigned long long* changed_out, void* ws,
+                                    size_t ws_bytes, void* stream) {
   const bool upd = W || m || v;
   if (!dY || !Xdq || T <= 0 || N <= 0 || K <= 0) return DQT_ERR_ARG;
   if (upd && (!W || !m || !v)) return DQT_ERR_ARG;
-  if (!upd && (!dW_out || W_img_next)) return DQT_ERR_ARG;
+  if (!upd && (!dW_out || W_img_next || W8_next)) return DQT_ERR_ARG;
+  if (W8_next && (grid.qmin < -16 || grid.qmax > 16)) return DQT_ERR_RANGE;
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
   if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(Xdq) || (W && !aligned16(W)) ||
       (m && !aligned16(m)) || (v && !aligned16(v)) || (dW_out && !aligned16(dW_out)) ||
-      (W_img_next && !aligned16(W_img_next)) || (ws && !aligned16(ws)))
+      (W_img_next && !aligned16(W_img_next)) || (W8_next && !aligned16(W8_next)) ||
+      (ws && !aligned16(ws)))
     return DQT_ERR_ALIGN;
   dqt::GemmLaunch g{};
   g.ws = ws;
@@ -596,6 +627,7 @@ int dqt_bitlinear_bwd_dw_update_img(const dqt_bf16* dY, const dqt_bf16* Xdq, int
   g.v = v;
   g.dW_out = dW_out;
   g.img_next = W_img_next;
+  g.img8_next = W8_next;
   g.changed = upd ? changed_out : nullptr;
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
@@ -605,14 +637,17 @@ int dqt_bitlinear_bwd_dw_update_img_pair(const dqt_bf16* dY, const dqt_bf16* Xdq
                                          const dqt_adamw_t* hp, const dqt_sr_t* sr0,
                                          const dqt_sr_t* sr1, dqt_grid_t grid, int64_t T,
                                          int64_t N, int64_t K, float* dW_out,
-                                         dqt_bf16* W_img_next, unsigned long long* changed_out,
-                                         void* ws, size_t ws_bytes, void* stream) {
+                                         dqt_bf16* W_img_next, uint8_t* W8_next,
+                                         unsigned long long* changed_out, void* ws,
+                                         size_t ws_bytes, void* stream) {
   if (!dY || !Xdq || !W || !m || !v || T <= 0 || N <= 0 || K <= 0 || !pair_split_ok(N0, N))
     return DQT_ERR_ARG;
+  if (W8_next && (grid.qmin < -16 || grid.qmax > 16)) return DQT_ERR_RANGE;
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
   if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(Xdq) || !aligned16(W) || !aligned16(m) ||
       !aligned16(v) || (dW_out && !aligned16(dW_out)) ||
-      (W_img_next && !aligned16(W_img_next)) || (ws && !aligned16(ws)))
+      (W_img_next && !aligned16(W_img_next)) || (W8_next && !aligned16(W8_next)) ||
+      (ws && !aligned16(ws)))
     return DQT_ERR_ALIGN;
   dqt::GemmLaunch g{};
   g.ws = ws;
@@ -632,6 +667,7 @@ int dqt_bitlinear_bwd_dw_update_img_pair(const dqt_bf16* dY, const dqt_bf16* Xdq
   g.v = v;
   g.dW_out = dW_out;
   g.img_next = W_img_next;
+  g.img8_next = W8_next;
   g.changed = changed_out;
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }

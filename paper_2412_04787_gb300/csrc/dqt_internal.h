@@ -65,7 +65,8 @@ struct GemmLaunch {
   float scale1;
   UpdateConsts uc1;
   int64_t lda;  // DX: elements between rows of A (dY); 0: packed rows
-  void* img_next;  // DW: bf16 image of the updated codes, or NULL
+  void* img_next;   // DW: bf16 image of the updated codes, or NULL
+  void* img8_next;  // DW: E4M3 image of the updated codes, or NULL
 };
 
 // Token slices the 2-SM dW GEMM of an M x N output reduced over Kred uses
@@ -97,7 +98,8 @@ int launch_tail_update(const float* part, int splits, int tail, int full, int nu
                        int8_t* W, bool packed, float* m, float* v, const UpdateConsts& uc,
                        const UpdateConsts* uc_dev, unsigned long long* changed, float* dW_out,
                        cudaStream_t stream, const UpdateConsts* uc1 = nullptr, int split = 0,
-                       bool col_major = false, uint16_t* img_next = nullptr);
+                       bool col_major = false, uint16_t* img_next = nullptr,
+                       uint8_t* img8_next = nullptr);
 
 // Sum `splits` fp32 slabs (stride `slab` elements) in slice order and apply
 // the update to W, m, v (numel elements); optionally write the sum to g_out.

@@ -43,6 +43,7 @@
 // third tensor-memory region (the 1-SM kernel, BN = 128).  Ternary weights
 // (max|c| = 1) need no drain for K <= 131072.
 #include <cuda.h>
+#include <cuda_fp8.h>
 
 #include <atomic>
 
@@ -126,6 +127,9 @@ struct Params {
   // dW: if set, the bf16 image of every updated code is written here too
   // (the next forward's operand), at the code's element index
   __nv_bfloat16* img_next;
+  // dW: if set, the E4M3 image of every updated code (the next FP8 forward's
+  // operand; exact for |code| <= 16)
+  uint8_t* img8_next;
   // dW with the constants in the parameter space: the parts of the
   // stochastic-rounding generator that are the same for every element of
   // the call, for uc and uc1
@@ -134,6 +138,10 @@ struct Params {
 
 // The bf16 image of four codes (exact: integers of magnitude <= 128).
 __device__ __forceinline__ void store_code_image4(__nv_bfloat16* img, size_t e, int32_t a, int32_t b,
+                                                  int32_t c, int32_t d);
+
+// The E4M3 image of four codes (exact for |code| <= 16).
+__device__ __forceinline__ void store_code_e4m3_4(uint8_t* img8, size_t e, int32_t a, int32_t b,
                                                   int32_t c, int32_t d);
 
 // Row and column tile (256 x 256) of a 2-SM kernel's tile index.
@@ -200,6 +208,15 @@ __device__ __forceinline__ void l2_discard_line(const void* p) {
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+__device__ __forceinline__ void store_code_e4m3_4(uint8_t* img8, size_t e, int32_t a, int32_t b,
+                                                  int32_t c, int32_t d) {
+  const uint32_t lo = __nv_cvt_float2_to_fp8x2(make_float2(static_cast<float>(a), static_cast<float>(b)),
+                                               __NV_SATFINITE, __NV_E4M3);
+  const uint32_t hi = __nv_cvt_float2_to_fp8x2(make_float2(static_cast<float>(c), static_cast<float>(d)),
+                                               __NV_SATFINITE, __NV_E4M3);
+  __stcs(reinterpret_cast<uint32_t*>(img8 + e), (lo & 0xFFFFu) | ((hi & 0xFFFFu) << 16));
 }
 
 __device__ __forceinline__ void store_code_image4(__nv_bfloat16* img, size_t e, int32_t a, int32_t b,
@@ -389,6 +406,7 @@ __device__ __forceinline__ uint32_t dw_update(const Params& p, const UpdateConst
              make_char4(static_cast<signed char>(n0c), static_cast<signed char>(n1c),
                         static_cast<signed char>(n2c), static_cast<signed char>(n3c)));
     if (p.img_next) store_code_image4(p.img_next, e, n0c, n1c, n2c, n3c);
+    if (p.img8_next) store_code_e4m3_4(p.img8_next, e, n0c, n1c, n2c, n3c);
     __stcs(reinterpret_cast<float4*>(p.m + e), L.m[j]);
     __stcs(reinterpret_cast<float4*>(p.v + e), L.v[j]);
   }
@@ -467,6 +485,7 @@ __device__ __forceinline__ uint32_t dw_update_row(const Params& p, const UpdateC
            make_char4(static_cast<signed char>(n0c), static_cast<signed char>(n1c),
                       static_cast<signed char>(n2c), static_cast<signed char>(n3c)));
   if (p.img_next) store_code_image4(p.img_next, e, n0c, n1c, n2c, n3c);
+  if (p.img8_next) store_code_e4m3_4(p.img8_next, e, n0c, n1c, n2c, n3c);
   __stcs(reinterpret_cast<float4*>(p.m + e), L.m);
   __stcs(reinterpret_cast<float4*>(p.v + e), L.v);
   return (n0c != c.x) + (n1c != c.y) + (n2c != c.z) + (n3c != c.w);
@@ -1568,12 +1587,13 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   p.uc1 = g.uc1;
   p.pc1 = philox_call_consts(g.uc1);
   p.img_next = g.kind == GEMM_DW ? static_cast<__nv_bfloat16*>(g.img_next) : nullptr;
-  if (p.img_next && (g.packed || !g.W)) return 1;
+  p.img8_next = g.kind == GEMM_DW ? static_cast<uint8_t*>(g.img8_next) : nullptr;
+  if ((p.img_next || p.img8_next) && (g.packed || !g.W)) return 1;
   // stacked weights: whole tiles (multiples of 256 of either tiling),
   // constants in the parameter space
   if (g.split > 0 && (g.split % 256 != 0 || g.uc_dev ||
-                      (g.kind != GEMM_FWD && g.kind != GEMM_DW) ||
-                      g.split >= (g.kind == GEMM_FWD ? g.N : g.M)))
+                      (g.kind != GEMM_FWD && g.kind != GEMM_FWD8 && g.kind != GEMM_DW) ||
+                      g.split >= (g.kind == GEMM_DW ? g.M : g.N)))
     return 1;
 
   CUtensorMap ta, tb;
@@ -1632,7 +1652,8 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
                                   g.uc_dev, g.changed, g.dW_out, stream,
                                   g.split > 0 ? &g.uc1 : nullptr, g.split,
                                   (g.N + 255) / 256 > (g.M + 255) / 256,
-                                  static_cast<uint16_t*>(g.img_next));
+                                  static_cast<uint16_t*>(g.img_next),
+                                  static_cast<uint8_t*>(g.img8_next));
       }
       // split-T: fp32 partials of each token slice into the workspace slabs,
       // then one streaming pass sums the slabs in slice order and applies the
@@ -1651,14 +1672,20 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
         return launch_slab_sum(static_cast<const float*>(g.ws), p.splits, p.slab, g.dW_out,
                                stream);
       }
-      if (g.img_next) {
-        // the update, then the image of the updated codes
+      if (g.img_next || g.img8_next) {
+        // the update, then the images of the updated codes
         GemmLaunch g3 = g;
         g3.img_next = nullptr;
+        g3.img8_next = nullptr;
         const int rc3 = launch_gemm(g3, stream);
         if (rc3) return rc3;
-        return launch_codes_to_bf16(g.W, static_cast<int64_t>(g.M) * g.N,
-                                    static_cast<uint16_t*>(g.img_next), stream);
+        const int64_t numel = static_cast<int64_t>(g.M) * g.N;
+        if (g.img_next &&
+            launch_codes_to_bf16(g.W, numel, static_cast<uint16_t*>(g.img_next), stream))
+          return 3;
+        return g.img8_next
+                   ? launch_codes_to_fp8(g.W, numel, static_cast<uint8_t*>(g.img8_next), stream)
+                   : 0;
       }
       if (g.split > 0) {
         // stacked weights: the rows of each with its own constants

@@ -6,6 +6,8 @@
 // exactly one Philox4x32-10 block (element e uses word e % 4 of block e / 4),
 // with 16-byte loads and stores of g, m, v and a 4-byte access to the codes
 // (one byte when the codes are 2-bit packed ternary: a group is one byte).
+#include <cuda_fp8.h>
+
 #include "dqt_internal.h"
 
 namespace dqt {
@@ -173,7 +175,8 @@ __global__ void __launch_bounds__(kThreads, 3)
                        float* __restrict__ v, const UpdateConsts uc_arg,
                        const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed,
                        float* __restrict__ dW_out, const UpdateConsts uc1, int split,
-                       bool col_major, uint16_t* __restrict__ img_next) {
+                       bool col_major, uint16_t* __restrict__ img_next,
+                       uint8_t* __restrict__ img8_next) {
   const UpdateConsts uc = DEV ? *uc_dev : uc_arg;
   uint8_t* Wp = reinterpret_cast<uint8_t*>(W);
   const int64_t ngroups = static_cast<int64_t>(tail) * 16384;  // 256 x 256 / 4 per tile
@@ -243,6 +246,13 @@ __global__ void __launch_bounds__(kThreads, 3)
           __stcs(reinterpret_cast<uint2*>(img_next + e),
                  make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
                             *reinterpret_cast<const uint32_t*>(&hi)));
+        }
+        if (img8_next) {  // the E4M3 image of the new codes (exact for |code| <= 16)
+          const uint32_t lo = __nv_cvt_float2_to_fp8x2(
+              make_float2(static_cast<float>(a), static_cast<float>(b)), __NV_SATFINITE, __NV_E4M3);
+          const uint32_t hi = __nv_cvt_float2_to_fp8x2(
+              make_float2(static_cast<float>(c), static_cast<float>(d)), __NV_SATFINITE, __NV_E4M3);
+          __stcs(reinterpret_cast<uint32_t*>(img8_next + e), (lo & 0xFFFFu) | ((hi & 0xFFFFu) << 16));
         }
         __stcs(reinterpret_cast<float4*>(m + e), m4);
         __stcs(reinterpret_cast<float4*>(v + e), v4);
@@ -327,7 +337,7 @@ int launch_tail_update(const float* part, int splits, int tail, int full, int nu
                        int8_t* W, bool packed, float* m, float* v, const UpdateConsts& uc,
                        const UpdateConsts* uc_dev, unsigned long long* changed, float* dW_out,
                        cudaStream_t stream, const UpdateConsts* uc1, int split, bool col_major,
-                       uint16_t* img_next) {
+                       uint16_t* img_next, uint8_t* img8_next) {
   const UpdateConsts u1 = uc1 ? *uc1 : uc;
   // the blocks that fit at once: each thread walks several groups, its next
   // group's loads in flight
@@ -349,13 +359,13 @@ int launch_tail_update(const float* part, int splits, int tail, int full, int nu
     tail_update_kernel<true><<<blocks, kThreads, 0, stream>>>(part, splits, tail, full, num_n, M, N,
                                                               W, packed, m, v, uc, uc_dev, changed,
                                                               dW_out, u1, uc1 ? split : 0,
-                                                              col_major, img_next);
+                                                              col_major, img_next, img8_next);
   else
     tail_update_kernel<false><<<blocks, kThreads, 0, stream>>>(part, splits, tail, full, num_n, M,
                                                                N, W, packed, m, v, uc, nullptr,
                                                                changed, dW_out, u1,
                                                                uc1 ? split : 0, col_major,
-                                                               img_next);
+                                                               img_next, img8_next);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 

@@ -23,7 +23,7 @@ EXPORTED = [
     "dqt_bitlinear_bwd_dw_update", "dqt_sr_update", "dqt_absmean_init_noalloc",
     "dqt_set_gemm_tiles", "dqt_update_consts_size", "dqt_update_consts",
     "dqt_bitlinear_bwd_dw_update_dev", "dqt_sr_update_dev", "dqt_bwd_dw_workspace_size",
-    "dqt_act_quant_fp8", "dqt_codes_to_fp8", "dqt_bitlinear_fwd_fp8",
+    "dqt_act_quant_fp8", "dqt_codes_to_fp8", "dqt_bitlinear_fwd_fp8", "dqt_bitlinear_fwd_fp8_pair",
     "dqt_pack_ternary", "dqt_unpack_ternary", "dqt_packed_to_bf16", "dqt_packed_to_fp8",
     "dqt_sr_update_packed", "dqt_bitlinear_bwd_dw_update_packed",
     "dqt_adafactor_workspace_size", "dqt_adafactor_stats", "dqt_adafactor_apply",
@@ -105,7 +105,7 @@ def lib():
         L.dqt_bitlinear_bwd_dw_update_img_pair.argtypes = [
             _vp, _vp, _vp, _i64, _f32, _f32, _vp, _vp, C.POINTER(dqt_adamw_t),
             C.POINTER(dqt_sr_t), C.POINTER(dqt_sr_t), dqt_grid_t, _i64, _i64, _i64, _vp, _vp,
-            _vp, _vp, _sz, _vp]
+            _vp, _vp, _vp, _sz, _vp]
         L.dqt_fwd_img_workspace_size.argtypes = [_i64, _i64, _i64]
         L.dqt_fwd_img_workspace_size.restype = _sz
         L.dqt_bitlinear_bwd_dx.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp, _sz, _vp]
@@ -124,7 +124,8 @@ def lib():
         L.dqt_bitlinear_bwd_dw_update_img.argtypes = [_vp, _vp, _vp, _f32, _vp, _vp,
                                                       C.POINTER(dqt_adamw_t),
                                                       C.POINTER(dqt_sr_t), dqt_grid_t, _i64,
-                                                      _i64, _i64, _vp, _vp, _vp, _vp, _sz, _vp]
+                                                      _i64, _i64, _vp, _vp, _vp, _vp, _vp, _sz,
+                                                      _vp]
         L.dqt_bwd_dw_workspace_size.argtypes = [_i64, _i64, _i64]
         L.dqt_bwd_dw_workspace_size.restype = _sz
         L.dqt_bwd_dw_img_workspace_size.argtypes = [_i64, _i64, _i64]
@@ -142,6 +143,8 @@ def lib():
         L.dqt_codes_to_fp8.argtypes = [_vp, _i64, dqt_grid_t, _vp, _vp]
         L.dqt_bitlinear_fwd_fp8.argtypes = [_vp, _vp, _vp, _f32, dqt_grid_t, _i64, _i64, _i64,
                                             _vp, _vp, _vp]
+        L.dqt_bitlinear_fwd_fp8_pair.argtypes = [_vp, _vp, _vp, _i64, _f32, _f32, dqt_grid_t, _i64,
+                                                 _i64, _i64, _vp, _vp, _vp]
         for name in ("dqt_pack_ternary", "dqt_unpack_ternary", "dqt_packed_to_bf16",
                      "dqt_packed_to_fp8"):
             getattr(L, name).argtypes = [_vp, _i64, _vp, _vp]
@@ -538,13 +541,15 @@ def dqt_bitlinear_bwd_dw_update(dY, Xq, s_x, W, s_w, m, v, hp, sr, bits_or_grid,
 
 
 def dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, s_w, m, v, hp, sr, bits_or_grid, dW_out=None,
-                                    changed_out=None, ws=None, stream=None, W_img_next=None):
+                                    changed_out=None, ws=None, stream=None, W_img_next=None,
+                                    W8_next=None):
     """Fused dW GEMM + AdamW + stochastic rounding on the X_tilde image Xdq;
     W, m, v updated in place.  With W = m = v = None only dW_out is computed.
     `ws`: split-T workspace (uint8 CUDA tensor of dqt_bwd_dw_img_workspace_size
     bytes); None allocates it when the shape benefits, False forces the single
-    fused kernel.  W_img_next (bf16 [N, K]): receives the image of the updated
-    codes (not the image this step's dX reads)."""
+    fused kernel.  W_img_next (bf16 [N, K]) and W8_next (uint8 [N, K], E4M3):
+    receive the images of the updated codes (not images this step still
+    reads)."""
     _need(dY, "dY", torch.bfloat16)
     T, N = dY.shape
     _need(Xdq, "Xdq", torch.bfloat16)
@@ -555,19 +560,20 @@ def dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, s_w, m, v, hp, sr, bits_or_grid,
     _opt(v, "v", torch.float32, (N, K))
     _opt(dW_out, "dW_out", torch.float32, (N, K))
     _opt(W_img_next, "W_img_next", torch.bfloat16, (N, K))
+    _opt(W8_next, "W8_next", torch.uint8, (N, K))
     _opt(changed_out, "changed_out", torch.int64, (1,))
     ws, nws = _dw_workspace(T, N, K, dY.device, ws)
     _check(lib().dqt_bitlinear_bwd_dw_update_img(
         _ptr(dY), _ptr(Xdq), _ptr(W), float(s_w), _ptr(m), _ptr(v),
         C.byref(hp) if hp is not None else None, C.byref(sr) if sr is not None else None,
-        _grid(bits_or_grid), T, N, K, _ptr(dW_out), _ptr(W_img_next), _ptr(changed_out),
-        _ptr(ws), nws, _stream(stream)), "dqt_bitlinear_bwd_dw_update_img")
+        _grid(bits_or_grid), T, N, K, _ptr(dW_out), _ptr(W_img_next), _ptr(W8_next),
+        _ptr(changed_out), _ptr(ws), nws, _stream(stream)), "dqt_bitlinear_bwd_dw_update_img")
     return W
 
 
 def dqt_bitlinear_bwd_dw_update_img_pair(dY, Xdq, W, N0, s_w0, s_w1, m, v, hp, sr0, sr1,
                                          bits_or_grid, dW_out=None, changed_out=None, ws=None,
-                                         stream=None, W_img_next=None):
+                                         stream=None, W_img_next=None, W8_next=None):
     """The fused dW + update of two stacked weights (rows [0, N0) of W, m, v
     and columns [0, N0) of dY the first's, with s_w0 and sr0; the rest the
     second's, with s_w1 and sr1).  `ws` as dqt_bitlinear_bwd_dw_update_img."""
@@ -581,12 +587,13 @@ def dqt_bitlinear_bwd_dw_update_img_pair(dY, Xdq, W, N0, s_w0, s_w1, m, v, hp, s
     _need(v, "v", torch.float32, (N, K))
     _opt(dW_out, "dW_out", torch.float32, (N, K))
     _opt(W_img_next, "W_img_next", torch.bfloat16, (N, K))
+    _opt(W8_next, "W8_next", torch.uint8, (N, K))
     _opt(changed_out, "changed_out", torch.int64, (1,))
     ws, nws = _dw_workspace(T, N, K, dY.device, ws)
     _check(lib().dqt_bitlinear_bwd_dw_update_img_pair(
         _ptr(dY), _ptr(Xdq), _ptr(W), int(N0), float(s_w0), float(s_w1), _ptr(m), _ptr(v),
         C.byref(hp), C.byref(sr0), C.byref(sr1), _grid(bits_or_grid), T, N, K, _ptr(dW_out),
-        _ptr(W_img_next), _ptr(changed_out), _ptr(ws), nws, _stream(stream)),
+        _ptr(W_img_next), _ptr(W8_next), _ptr(changed_out), _ptr(ws), nws, _stream(stream)),
            "dqt_bitlinear_bwd_dw_update_img_pair")
     return W
 
@@ -704,6 +711,27 @@ def dqt_bitlinear_fwd_fp8(Xq8, s_x8, W8, s_w, bits_or_grid, Y=None, acc_out=None
     _check(lib().dqt_bitlinear_fwd_fp8(_ptr(Xq8), _ptr(s_x8), _ptr(W8), float(s_w),
                                        _grid(bits_or_grid), T, K, N, _ptr(Y), _ptr(acc_out),
                                        _stream(stream)), "dqt_bitlinear_fwd_fp8")
+    return Y
+
+
+def dqt_bitlinear_fwd_fp8_pair(Xq8, s_x8, W8, N0, s_w0, s_w1, bits_or_grid, Y=None, acc_out=None,
+                               stream=None):
+    """The FP8 forward of two stacked weights: rows [0, N0) of W8 and columns
+    [0, N0) of Y the first weight's (scale s_w0), the rest the second's."""
+    _need(Xq8, "Xq8", torch.uint8)
+    T, K = Xq8.shape
+    _need(W8, "W8", torch.uint8)
+    N = W8.shape[0]
+    _need(W8, "W8", torch.uint8, (N, K))
+    _need(s_x8, "s_x8", torch.float32, (T,))
+    if Y is None:
+        Y = torch.empty((T, N), dtype=torch.bfloat16, device=Xq8.device)
+    _need(Y, "Y", torch.bfloat16, (T, N))
+    _opt(acc_out, "acc_out", torch.float32, (T, N))
+    _check(lib().dqt_bitlinear_fwd_fp8_pair(_ptr(Xq8), _ptr(s_x8), _ptr(W8), int(N0), float(s_w0),
+                                            float(s_w1), _grid(bits_or_grid), T, K, N, _ptr(Y),
+                                            _ptr(acc_out), _stream(stream)),
+           "dqt_bitlinear_fwd_fp8_pair")
     return Y
 
 

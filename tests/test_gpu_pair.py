@@ -190,3 +190,74 @@ def test_dw_update_pair_writes_next_image():
                                              g, W_img_next=img)
     dqt.dqt_check_device_status()
     assert torch.equal(img.view(torch.int16), dqt.dqt_codes_to_bf16(W).view(torch.int16))
+
+
+@pytest.mark.parametrize("T,K,N0,N1", [(300, 272, 256, 264), (1024, 2048, 5632, 5632)])
+def test_fwd_fp8_pair_equals_two_calls(T, K, N0, N1):
+    """The stacked FP8 forward: each half of the output with its own scale,
+    equal to two dqt_bitlinear_fwd_fp8 calls (the same fp32 sums per tile)."""
+    X = inputs.normal((T, K), 1.0, seed=T + 3, dtype=torch.bfloat16).cuda()
+    c, s0, s1, g = _weights(N0, N1, K, 1.58, seed=N0 + 7)
+    q8, s8, _ = dqt.dqt_act_quant_fp8(X, want_xdq=False)
+    W8 = dqt.dqt_codes_to_fp8(torch.from_numpy(c).cuda(), g)
+    N = N0 + N1
+    acc = torch.empty((T, N), dtype=torch.float32, device="cuda")
+    Y = dqt.dqt_bitlinear_fwd_fp8_pair(q8, s8, W8, N0, s0, s1, g, acc_out=acc)
+    acc0 = torch.empty((T, N0), dtype=torch.float32, device="cuda")
+    acc1 = torch.empty((T, N1), dtype=torch.float32, device="cuda")
+    Y0 = dqt.dqt_bitlinear_fwd_fp8(q8, s8, W8[:N0], s0, g, acc_out=acc0)
+    Y1 = dqt.dqt_bitlinear_fwd_fp8(q8, s8, W8[N0:], s1, g, acc_out=acc1)
+    dqt.dqt_check_device_status()
+    assert torch.equal(acc[:, :N0].view(torch.int32), acc0.view(torch.int32))
+    assert torch.equal(acc[:, N0:].view(torch.int32), acc1.view(torch.int32))
+    assert torch.equal(Y[:, :N0].contiguous().view(torch.int16), Y0.view(torch.int16))
+    assert torch.equal(Y[:, N0:].contiguous().view(torch.int16), Y1.view(torch.int16))
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("T,K,N", [(4096, 2048, 5632),   # token slices + tail kernel
+                                   (256, 512, 520),      # one wave, ragged N
+                                   (4096, 512, 512)])    # split-T path
+def test_dw_update_writes_next_e4m3_image(mode, T, K, N):
+    """W8_next: the update also writes the E4M3 image of the codes it writes,
+    byte for byte what dqt_codes_to_fp8 makes of them (with the bf16 image
+    beside it)."""
+    dqt.dqt_set_gemm_tiles(mode)
+    try:
+        X = inputs.normal((T, K), 1.0, seed=T + N + 1, dtype=torch.bfloat16)
+        dY = inputs.normal((T, N), 1e-2, seed=T + 9, dtype=torch.bfloat16).cuda()
+        qmin, qmax = oracle.grid(1.58)
+        c, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=N + 1).numpy(), qmin, qmax)
+        _, s_x, _, Xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xdq",))
+        W = torch.from_numpy(c).cuda()
+        m = torch.zeros((N, K), device="cuda")
+        v = torch.zeros((N, K), device="cuda")
+        img = torch.full((N, K), float("nan"), dtype=torch.bfloat16, device="cuda")
+        img8 = torch.full((N, K), 0x7F, dtype=torch.uint8, device="cuda")
+        dqt.dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, float(s_w), m, v, dqt.adamw(lr=1e-2),
+                                            dqt.sr_stream(seed=5), (qmin, qmax), W_img_next=img,
+                                            W8_next=img8)
+        dqt.dqt_check_device_status()
+        assert not torch.equal(W.cpu(), torch.from_numpy(c))
+        assert torch.equal(img8, dqt.dqt_codes_to_fp8(W, (qmin, qmax)))
+        assert torch.equal(img.view(torch.int16), dqt.dqt_codes_to_bf16(W).view(torch.int16))
+    finally:
+        dqt.dqt_set_gemm_tiles(0)
+
+
+def test_dw_update_pair_writes_next_e4m3_image():
+    T, K, N0, N1 = 1024, 2048, 5632, 5632
+    N = N0 + N1
+    X = inputs.normal((T, K), 1.0, seed=21, dtype=torch.bfloat16)
+    dY = inputs.normal((T, N), 1e-2, seed=22, dtype=torch.bfloat16).cuda()
+    c, s0, s1, g = _weights(N0, N1, K, 1.58, seed=23)
+    _, s_x, _, Xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xdq",))
+    W = torch.from_numpy(c).cuda()
+    m = torch.zeros((N, K), device="cuda")
+    v = torch.zeros((N, K), device="cuda")
+    img8 = torch.empty((N, K), dtype=torch.uint8, device="cuda")
+    dqt.dqt_bitlinear_bwd_dw_update_img_pair(dY, Xdq, W, N0, s0, s1, m, v, dqt.adamw(lr=1e-2),
+                                             dqt.sr_stream(seed=2), dqt.sr_stream(seed=2, tensor_id=1),
+                                             g, W8_next=img8)
+    dqt.dqt_check_device_status()
+    assert torch.equal(img8, dqt.dqt_codes_to_fp8(W, g))
