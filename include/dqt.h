@@ -376,15 +376,18 @@ int dqt_sr_update(const float* grad, int8_t* W, float s_w, float* m, float* v,
  * The _dev entry points are dqt_bitlinear_bwd_dw_update_img and dqt_sr_update
  * with (hp, sr, grid, s_w) replaced by that device block; results are
  * identical for identical constants.  W, m, v are required; the weight
- * gradient takes the X_tilde image Xdq and the token-slice workspace of
- * dqt_bitlinear_bwd_dw_update_img. */
+ * gradient takes the X_tilde image Xdq, the token-slice workspace and the
+ * next-step images W_img_next / W8_next of dqt_bitlinear_bwd_dw_update_img
+ * (W8_next only for grids within 16 in magnitude: the grid is in the device
+ * block, so this call cannot check it). */
 size_t dqt_update_consts_size(void);
 int dqt_update_consts(const dqt_adamw_t* hp, const dqt_sr_t* sr, dqt_grid_t grid, float s_w,
                       void* out, size_t out_bytes);
 int dqt_bitlinear_bwd_dw_update_dev(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W, float* m,
                                     float* v, const void* consts_dev, int64_t T, int64_t N,
-                                    int64_t K, float* dW_out, unsigned long long* changed_out,
-                                    void* ws, size_t ws_bytes, void* stream);
+                                    int64_t K, float* dW_out, dqt_bf16* W_img_next,
+                                    uint8_t* W8_next, unsigned long long* changed_out, void* ws,
+                                    size_t ws_bytes, void* stream);
 int dqt_sr_update_dev(const float* grad, int8_t* W, float* m, float* v, const void* consts_dev,
                       int64_t numel, unsigned long long* changed_out, void* stream);
 

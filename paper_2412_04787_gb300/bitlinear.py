@@ -81,14 +81,14 @@ class _BitLinearFn(torch.autograd.Function):
         x2 = x2.contiguous()
         if layer.act == "fp8":
             q8, s_x, xdq = _quantised(x, x2, "fp8")
-            y = dqt.dqt_bitlinear_fwd_fp8(q8, s_x, layer.weight_fp8(), float(layer.s_w),
+            y = dqt.dqt_bitlinear_fwd_fp8(q8, s_x, layer.image_fp8(), float(layer.s_w),
                                           layer.grid_tuple)
-            w_img = None  # dX needs the bf16 image: built in backward
+            w_img = None  # dX needs the bf16 image: taken in backward
         else:
             _, s_x, q_img, xdq = _quantised(x, x2, "int8")
             # the weight's code image serves the forward and, kept until the
             # backward, dX (the codes change only after dX, in the update)
-            w_img = layer.weight_bf16()
+            w_img = layer.image_bf16()
             y = dqt.dqt_bitlinear_fwd_img(q_img, s_x, w_img, float(layer.s_w), layer.grid_tuple)
         ctx.save_for_backward(xdq, w_img)
         ctx.layer = layer
@@ -107,7 +107,7 @@ class _BitLinearFn(torch.autograd.Function):
         dy2 = dy2.contiguous()
         # the codes have not changed since the forward
         if w_img is None:
-            w_img = layer.weight_bf16()
+            w_img = layer.image_bf16()
         dx = dqt.dqt_bitlinear_bwd_dx_img(dy2, w_img, float(layer.s_w))
         if layer.update_in_backward:
             layer._dqt_update(dy2, xdq)
@@ -180,6 +180,14 @@ class DQTBitLinear(torch.nn.Module):
         self.tensor_id = int(tensor_id)
         # device-resident update constants (CUDA-graph replay), see prepare_step
         self.uc_dev = None
+        # the codes' bf16 (and, with act="fp8", E4M3) operand images, kept
+        # from step to step: the AdamW update on int8 codes rewrites them with
+        # the codes it writes, after this step's dX has read them (one stream:
+        # the update is ordered after dX), so no step converts the codes;
+        # they are rebuilt when the codes' version counter says the codes
+        # were changed from outside (copy_, load_state_dict)
+        self._img = self._img8 = None
+        self._img_version = self._img8_version = -1
         # anchor: a 0-element tensor that requires grad, so the layer's
         # backward (and with it the DQT update) runs even if x does not
         self._anchor = torch.nn.Parameter(torch.zeros(0, device=device), requires_grad=True)
@@ -215,6 +223,47 @@ class DQTBitLinear(torch.nn.Module):
         if self.packed:
             return dqt.dqt_packed_to_fp8(self.codes, shape)
         return dqt.dqt_codes_to_fp8(self.codes, self.grid_tuple)
+
+    def _images_kept(self):
+        # the updates that write the images: AdamW on int8 codes
+        return self.optimizer == "adamw" and not self.packed
+
+    def image_bf16(self):
+        """The bf16 image of the current codes (the forward's and dX's
+        operand); kept from step to step where the update rewrites it."""
+        if not self._images_kept():
+            return self.weight_bf16()
+        if self._img is None:
+            self._img = torch.empty((self.out_features, self.in_features), dtype=torch.bfloat16,
+                                    device=self.codes.device)
+            self._img_version = -1
+        if self._img_version != self.codes._version:
+            dqt.dqt_codes_to_bf16(self.codes, self._img)
+            self._img_version = self.codes._version
+        return self._img
+
+    def image_fp8(self):
+        """The E4M3 image of the current codes (the FP8 forward's operand),
+        kept like image_bf16."""
+        if not self._images_kept():
+            return self.weight_fp8()
+        if self._img8 is None:
+            self._img8 = torch.empty((self.out_features, self.in_features), dtype=torch.uint8,
+                                     device=self.codes.device)
+            self._img8_version = -1
+        if self._img8_version != self.codes._version:
+            dqt.dqt_codes_to_fp8(self.codes, self.grid_tuple, self._img8)
+            self._img8_version = self.codes._version
+        return self._img8
+
+    def _next_images(self):
+        # the kept images that are current: the update writes the images of
+        # the codes it writes into them (an image not current stays stale and
+        # is rebuilt when next used)
+        v = self.codes._version
+        img = self._img if self._img is not None and self._img_version == v else None
+        img8 = self._img8 if self._img8 is not None and self._img8_version == v else None
+        return img, img8
 
     def _hyper(self, step):
         hp = dqt.adamw(lr=self.lr, beta1=self.betas[0], beta2=self.betas[1], eps=self.eps,
@@ -254,14 +303,17 @@ class DQTBitLinear(torch.nn.Module):
             dqt.dqt_bitlinear_bwd_dw_update_packed(dy2, xdq, self.codes, self.s_w, self.m, self.v,
                                                    hp, sr, changed_out=self.changed)
             return
+        img, img8 = self._next_images()
         if self.uc_dev is not None:
             dqt.dqt_bitlinear_bwd_dw_update_dev(dy2, xdq, self.codes, self.m, self.v, self.uc_dev,
-                                                changed_out=self.changed)
+                                                changed_out=self.changed, W_img_next=img,
+                                                W8_next=img8)
             return
         self.step += 1
         hp, sr = self._hyper(self.step)
         dqt.dqt_bitlinear_bwd_dw_update_img(dy2, xdq, self.codes, self.s_w, self.m, self.v, hp, sr,
-                                            self.grid_tuple, changed_out=self.changed)
+                                            self.grid_tuple, changed_out=self.changed,
+                                            W_img_next=img, W8_next=img8)
 
     def extra_repr(self):
         return "in_features=%d, out_features=%d, grid=%s, act=%s, optimizer=%s, packed=%s" % (

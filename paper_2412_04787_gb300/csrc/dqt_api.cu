@@ -699,13 +699,15 @@ int dqt_update_consts(const dqt_adamw_t* hp, const dqt_sr_t* sr, dqt_grid_t grid
 
 int dqt_bitlinear_bwd_dw_update_dev(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W, float* m,
                                     float* v, const void* consts_dev, int64_t T, int64_t N,
-                                    int64_t K, float* dW_out, unsigned long long* changed_out,
-                                    void* ws, size_t ws_bytes, void* stream) {
+                                    int64_t K, float* dW_out, dqt_bf16* W_img_next,
+                                    uint8_t* W8_next, unsigned long long* changed_out, void* ws,
+                                    size_t ws_bytes, void* stream) {
   if (!dY || !Xdq || !W || !m || !v || !consts_dev || T <= 0 || N <= 0 || K <= 0)
     return DQT_ERR_ARG;
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
   if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(Xdq) || !aligned16(W) || !aligned16(m) ||
       !aligned16(v) || !aligned16(consts_dev) || (dW_out && !aligned16(dW_out)) ||
+      (W_img_next && !aligned16(W_img_next)) || (W8_next && !aligned16(W8_next)) ||
       (ws && !aligned16(ws)))
     return DQT_ERR_ALIGN;
   dqt::GemmLaunch g{};
@@ -721,6 +723,8 @@ int dqt_bitlinear_bwd_dw_update_dev(const dqt_bf16* dY, const dqt_bf16* Xdq, int
   g.m = m;
   g.v = v;
   g.dW_out = dW_out;
+  g.img_next = W_img_next;
+  g.img8_next = W8_next;
   g.changed = changed_out;
   g.uc_dev = static_cast<const dqt::UpdateConsts*>(consts_dev);
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;

@@ -102,11 +102,13 @@ int launch_tail_update(const float* part, int splits, int tail, int full, int nu
                        uint8_t* img8_next = nullptr);
 
 // Sum `splits` fp32 slabs (stride `slab` elements) in slice order and apply
-// the update to W, m, v (numel elements); optionally write the sum to g_out.
+// the update to W, m, v (numel elements); optionally write the sum to g_out
+// and the bf16 / E4M3 images of the new codes to img / img8 (int8 codes).
 int launch_sr_update_slabs(const float* slabs, int splits, long long slab, int8_t* W, float* m,
                            float* v, int64_t numel, const UpdateConsts& uc,
                            const UpdateConsts* uc_dev, unsigned long long* changed, float* g_out,
-                           cudaStream_t stream, bool packed = false);
+                           cudaStream_t stream, bool packed = false, uint16_t* img = nullptr,
+                           uint8_t* img8 = nullptr);
 // Sum the slabs into out (gradient only).
 int launch_slab_sum(const float* slabs, int splits, long long slab, float* out,
                     cudaStream_t stream);

@@ -1672,34 +1672,23 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
         return launch_slab_sum(static_cast<const float*>(g.ws), p.splits, p.slab, g.dW_out,
                                stream);
       }
-      if (g.img_next || g.img8_next) {
-        // the update, then the images of the updated codes
-        GemmLaunch g3 = g;
-        g3.img_next = nullptr;
-        g3.img8_next = nullptr;
-        const int rc3 = launch_gemm(g3, stream);
-        if (rc3) return rc3;
-        const int64_t numel = static_cast<int64_t>(g.M) * g.N;
-        if (g.img_next &&
-            launch_codes_to_bf16(g.W, numel, static_cast<uint16_t*>(g.img_next), stream))
-          return 3;
-        return g.img8_next
-                   ? launch_codes_to_fp8(g.W, numel, static_cast<uint8_t*>(g.img8_next), stream)
-                   : 0;
-      }
+      // (the images of the updated codes are written by the same pass)
+      uint16_t* img = static_cast<uint16_t*>(g.img_next);
+      uint8_t* img8 = static_cast<uint8_t*>(g.img8_next);
       if (g.split > 0) {
         // stacked weights: the rows of each with its own constants
         const long long n0 = static_cast<long long>(g.split) * g.N;
         const float* sl = static_cast<const float*>(g.ws);
         return launch_sr_update_slabs(sl, p.splits, p.slab, g.W, g.m, g.v, n0, g.uc, nullptr,
-                                      g.changed, g.dW_out, stream, g.packed) ||
+                                      g.changed, g.dW_out, stream, g.packed, img, img8) ||
                launch_sr_update_slabs(sl + n0, p.splits, p.slab, g.W + n0, g.m + n0, g.v + n0,
                                       p.slab - n0, g.uc1, nullptr, g.changed,
-                                      g.dW_out ? g.dW_out + n0 : nullptr, stream, g.packed);
+                                      g.dW_out ? g.dW_out + n0 : nullptr, stream, g.packed,
+                                      img ? img + n0 : nullptr, img8 ? img8 + n0 : nullptr);
       }
       return launch_sr_update_slabs(static_cast<const float*>(g.ws), p.splits, p.slab, g.W, g.m,
                                     g.v, p.slab, g.uc, g.uc_dev, g.changed, g.dW_out, stream,
-                                    g.packed);
+                                    g.packed, img, img8);
     }
   }
   return 1;

@@ -39,15 +39,36 @@ __device__ __forceinline__ float slab_grad1(const float* __restrict__ grad, int 
   return g;
 }
 
+// The bf16 and E4M3 images of four new codes (either pointer may be NULL).
+__device__ __forceinline__ void store_images4(uint16_t* img, uint8_t* img8, int64_t e, int32_t a,
+                                              int32_t b, int32_t c, int32_t d) {
+  if (img) {
+    const __nv_bfloat162 lo = __floats2bfloat162_rn(static_cast<float>(a), static_cast<float>(b));
+    const __nv_bfloat162 hi = __floats2bfloat162_rn(static_cast<float>(c), static_cast<float>(d));
+    __stcs(reinterpret_cast<uint2*>(img + e),
+           make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi)));
+  }
+  if (img8) {
+    const uint32_t lo = __nv_cvt_float2_to_fp8x2(
+        make_float2(static_cast<float>(a), static_cast<float>(b)), __NV_SATFINITE, __NV_E4M3);
+    const uint32_t hi = __nv_cvt_float2_to_fp8x2(
+        make_float2(static_cast<float>(c), static_cast<float>(d)), __NV_SATFINITE, __NV_E4M3);
+    __stcs(reinterpret_cast<uint32_t*>(img8 + e), (lo & 0xFFFFu) | ((hi & 0xFFFFu) << 16));
+  }
+}
+
 // DEV: the constants are read from device memory (else the kernel's
 // parameter space); SLABS: the gradient may be split into slabs and the
-// summed gradient written out.  The plain instance is the leanest stream.
+// summed gradient written out, and the images of the new codes (img bf16,
+// img8 E4M3, int8 codes only) written beside them.  The plain instance is the
+// leanest stream.
 template <bool packed, bool DEV, bool SLABS>
 __global__ void __launch_bounds__(kThreads)
     sr_update_kernel(const float* __restrict__ grad, int nsplit, long long slab,
                      float* __restrict__ g_out, int8_t* __restrict__ W, float* __restrict__ m,
                      float* __restrict__ v, int64_t numel, const UpdateConsts uc_arg,
-                     const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed) {
+                     const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed,
+                     uint16_t* __restrict__ img, uint8_t* __restrict__ img8) {
   uint8_t* Wp = reinterpret_cast<uint8_t*>(W);
   const UpdateConsts uc = DEV ? *uc_dev : uc_arg;
   const int64_t ngroups = numel >> 2;
@@ -77,6 +98,7 @@ __global__ void __launch_bounds__(kThreads)
       *reinterpret_cast<char4*>(W + e) =
           make_char4(static_cast<signed char>(a), static_cast<signed char>(b),
                      static_cast<signed char>(c), static_cast<signed char>(d));
+    if (SLABS && !packed) store_images4(img, img8, e, a, b, c, d);
     __stcs(reinterpret_cast<float4*>(m + e), m4);
     __stcs(reinterpret_cast<float4*>(v + e), v4);
   }
@@ -100,6 +122,10 @@ __global__ void __launch_bounds__(kThreads)
       n_changed += (r != c0);
       if (packed) pr[j] = r;
       else W[e] = static_cast<int8_t>(r);
+      if (SLABS && !packed && img) img[e] = __bfloat16_as_ushort(__float2bfloat16_rn(static_cast<float>(r)));
+      if (SLABS && !packed && img8)
+        img8[e] = static_cast<uint8_t>(
+            __nv_cvt_float_to_fp8(static_cast<float>(r), __NV_SATFINITE, __NV_E4M3));
       m[e] = mm;
       v[e] = vv;
     }
@@ -293,27 +319,30 @@ namespace {
 template <bool packed, bool DEV, bool SLABS>
 void sr_launch(const float* grad, int splits, long long slab, float* g_out, int8_t* W, float* m,
                float* v, int64_t numel, const UpdateConsts& uc, const UpdateConsts* uc_dev,
-               unsigned long long* changed, cudaStream_t stream) {
+               unsigned long long* changed, cudaStream_t stream, uint16_t* img = nullptr,
+               uint8_t* img8 = nullptr) {
   sr_update_kernel<packed, DEV, SLABS><<<stream_blocks(numel), kThreads, 0, stream>>>(
-      grad, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed);
+      grad, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed, img, img8);
 }
 
 template <bool packed>
 void sr_dispatch(const float* grad, int splits, long long slab, float* g_out, int8_t* W, float* m,
                  float* v, int64_t numel, const UpdateConsts& uc, const UpdateConsts* uc_dev,
-                 unsigned long long* changed, cudaStream_t stream) {
-  const bool slabs = splits > 1 || g_out;
+                 unsigned long long* changed, cudaStream_t stream, uint16_t* img = nullptr,
+                 uint8_t* img8 = nullptr) {
+  // the image outputs are those of the slab instance
+  const bool slabs = splits > 1 || g_out || img || img8;
   if (uc_dev) {
     if (slabs)
       sr_launch<packed, true, true>(grad, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed,
-                                    stream);
+                                    stream, img, img8);
     else
       sr_launch<packed, true, false>(grad, 1, 0, nullptr, W, m, v, numel, uc, uc_dev, changed,
                                      stream);
   } else {
     if (slabs)
       sr_launch<packed, false, true>(grad, splits, slab, g_out, W, m, v, numel, uc, nullptr,
-                                     changed, stream);
+                                     changed, stream, img, img8);
     else
       sr_launch<packed, false, false>(grad, 1, 0, nullptr, W, m, v, numel, uc, nullptr, changed,
                                       stream);
@@ -325,11 +354,12 @@ void sr_dispatch(const float* grad, int splits, long long slab, float* g_out, in
 int launch_sr_update_slabs(const float* slabs, int splits, long long slab, int8_t* W, float* m,
                            float* v, int64_t numel, const UpdateConsts& uc,
                            const UpdateConsts* uc_dev, unsigned long long* changed, float* g_out,
-                           cudaStream_t stream, bool packed) {
+                           cudaStream_t stream, bool packed, uint16_t* img, uint8_t* img8) {
   if (packed)
     sr_dispatch<true>(slabs, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed, stream);
   else
-    sr_dispatch<false>(slabs, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed, stream);
+    sr_dispatch<false>(slabs, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed, stream,
+                       img, img8);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 

@@ -137,7 +137,7 @@ def lib():
         L.dqt_update_consts.argtypes = [C.POINTER(dqt_adamw_t), C.POINTER(dqt_sr_t), dqt_grid_t,
                                         _f32, _vp, _sz]
         L.dqt_bitlinear_bwd_dw_update_dev.argtypes = [_vp, _vp, _vp, _vp, _vp, _vp, _i64, _i64,
-                                                      _i64, _vp, _vp, _vp, _sz, _vp]
+                                                      _i64, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
         L.dqt_sr_update_dev.argtypes = [_vp, _vp, _vp, _vp, _vp, _i64, _vp, _vp]
         L.dqt_act_quant_fp8.argtypes = [_vp, _i64, _i64, _vp, _vp, _vp, _vp]
         L.dqt_codes_to_fp8.argtypes = [_vp, _i64, dqt_grid_t, _vp, _vp]
@@ -626,9 +626,9 @@ def dqt_update_consts(hp, sr, bits_or_grid, s_w, out=None):
 
 
 def dqt_bitlinear_bwd_dw_update_dev(dY, Xdq, W, m, v, consts_dev, dW_out=None, changed_out=None,
-                                    ws=None, stream=None):
-    """As dqt_bitlinear_bwd_dw_update with the update constants read from the
-    device block `consts_dev` (uint8 CUDA tensor) when the kernel runs."""
+                                    ws=None, stream=None, W_img_next=None, W8_next=None):
+    """As dqt_bitlinear_bwd_dw_update_img with the update constants read from
+    the device block `consts_dev` (uint8 CUDA tensor) when the kernel runs."""
     _need(dY, "dY", torch.bfloat16)
     T, N = dY.shape
     _need(Xdq, "Xdq", torch.bfloat16)
@@ -639,11 +639,14 @@ def dqt_bitlinear_bwd_dw_update_dev(dY, Xdq, W, m, v, consts_dev, dW_out=None, c
     _need(v, "v", torch.float32, (N, K))
     _need(consts_dev, "consts_dev", torch.uint8)
     _opt(dW_out, "dW_out", torch.float32, (N, K))
+    _opt(W_img_next, "W_img_next", torch.bfloat16, (N, K))
+    _opt(W8_next, "W8_next", torch.uint8, (N, K))
     _opt(changed_out, "changed_out", torch.int64, (1,))
     ws, nws = _dw_workspace(T, N, K, dY.device, ws)
     _check(lib().dqt_bitlinear_bwd_dw_update_dev(
         _ptr(dY), _ptr(Xdq), _ptr(W), _ptr(m), _ptr(v), _ptr(consts_dev), T, N, K, _ptr(dW_out),
-        _ptr(changed_out), _ptr(ws), nws, _stream(stream)), "dqt_bitlinear_bwd_dw_update_dev")
+        _ptr(W_img_next), _ptr(W8_next), _ptr(changed_out), _ptr(ws), nws, _stream(stream)),
+           "dqt_bitlinear_bwd_dw_update_dev")
     return W
 
 
