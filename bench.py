@@ -1549,10 +1549,11 @@ def run_layer(args):
 def layer_step(bits=1.58, steps=200, warmup=10):
     """One BitLinear layer's training step at T=256, K=512, N=512 (X ~N(0,1),
     dY ~N(0,1e-2), ternary codes by AbsMean of N(0,0.02), AdamW lr 1e-3, Philox
-    seed 1234): act_quant, forward, dX and the fused dW + AdamW + SR update,
-    which also writes the weight's code image for the next step.  dX needs
-    neither act_quant nor the forward, so it runs beside them on a second
-    stream; the update waits for both.  At this size every kernel is latency-bound, so the
+    seed 1234): act_quant, forward, then dX and the fused dW + AdamW + SR
+    update side by side on two streams (the backward after the forward, as in
+    a network, where dY follows from Y); the update writes the weight's code
+    image for the next step into the second of two image buffers, so it never
+    touches the image dX reads.  At this size every kernel is latency-bound, so the
     K timed steps are captured as one CUDA graph (step i reads its update
     constants from row i of a device block, uploaded in one copy at the start
     of the timed region) and the time is the GPU's, not the Python launch
@@ -1565,7 +1566,7 @@ def layer_step(bits=1.58, steps=200, warmup=10):
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     T, K, N = LAYER_SHAPE
-    KS = steps
+    KS = steps + steps % 2  # even: each replay starts on the image its predecessor left in imgs[0]
     grid = dqt.grid(bits)
     host = [(inputs.normal((T, K), 1.0, seed=1 + 100 * r, dtype=torch.bfloat16).pin_memory(),
              inputs.normal((T, N), 1e-2, seed=2 + 100 * r, dtype=torch.bfloat16).pin_memory())
@@ -1596,24 +1597,26 @@ def layer_step(bits=1.58, steps=200, warmup=10):
     state = {"step": 0}
     ch_host = torch.empty(KS, dtype=torch.int64).pin_memory()
 
-    dqt.dqt_codes_to_bf16(W, W_img)  # the first step's image; each update writes the next
+    # two image buffers: step i reads imgs[i % 2], its update writes imgs[(i + 1) % 2]
+    imgs = [W_img, torch.empty_like(W_img)]
+    dqt.dqt_codes_to_bf16(W, imgs[0])  # the first step's image
     branch = torch.cuda.Stream()
 
     def kernels(i):
         main = torch.cuda.current_stream()
+        img, img_next = imgs[i % 2], imgs[(i + 1) % 2]
+        dqt.dqt_act_quant_images(X, None, s_x, q_img, xdq, want=())
+        dqt.dqt_bitlinear_fwd_img(q_img, s_x, img, s_w, grid, Y=Y)
         fork = torch.cuda.Event()
         fork.record(main)
         branch.wait_event(fork)
-        with torch.cuda.stream(branch):  # dX reads dY and the image only
-            dqt.dqt_bitlinear_bwd_dx_img(dY, W_img, s_w, dX=dX)
-        dqt.dqt_act_quant_images(X, None, s_x, q_img, xdq, want=())
-        dqt.dqt_bitlinear_fwd_img(q_img, s_x, W_img, s_w, grid, Y=Y)
+        with torch.cuda.stream(branch):
+            dqt.dqt_bitlinear_bwd_dx_img(dY, img, s_w, dX=dX)
+        dqt.dqt_bitlinear_bwd_dw_update_dev(dY, xdq, W, m, v, uc_dev[i % KS], changed_out=changed,
+                                            ws=ws, W_img_next=img_next)
         join = torch.cuda.Event()
         join.record(branch)
         main.wait_event(join)
-        # the update rewrites the codes and their image after both read them
-        dqt.dqt_bitlinear_bwd_dw_update_dev(dY, xdq, W, m, v, uc_dev[i], changed_out=changed,
-                                            ws=ws, W_img_next=W_img)
 
     def fill(block):
         for i in range(block.shape[0]):
@@ -1621,7 +1624,9 @@ def layer_step(bits=1.58, steps=200, warmup=10):
             dqt.dqt_update_consts(dqt.adamw(lr=1e-3, step=state["step"]), sr, grid, s_w,
                                   out=block[i])
 
-    # warm-up: eager steps, each with its own constants row
+    # warm-up: eager steps, each with its own constants row; an even number,
+    # so that the graph's first step finds its image in imgs[0]
+    warmup += warmup % 2
     side = torch.cuda.Stream()
     side.wait_stream(torch.cuda.current_stream())
     warm = torch.zeros((warmup, row), dtype=torch.uint8).pin_memory()
@@ -1631,7 +1636,7 @@ def layer_step(bits=1.58, steps=200, warmup=10):
             dqt.dqt_update_consts(dqt.adamw(lr=1e-3, step=state["step"]), sr, grid, s_w,
                                   out=warm[i])
             uc_dev[i % KS].copy_(warm[i], non_blocking=True)
-            kernels(i % KS)
+            kernels(i)
     torch.cuda.current_stream().wait_stream(side)
     torch.cuda.synchronize()
     graph = torch.cuda.CUDAGraph()
