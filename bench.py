@@ -82,7 +82,9 @@ def kernel_fingerprint(files=GEMM_SOURCES):
 # reports null.
 # With gate and up stacked, the mean over the step's two dW launches (the
 # stacked gate/up call and the down call, each its GEMM and streaming kernel).
-DW_TRAFFIC_STACKED = {"58ba5df98181": ((464767488 + 147933696)
+DW_TRAFFIC_STACKED = {"e8a6edbac357": ((499344640 + 147830784)
+                                         + (258470912 + 57011456 + 33059840 + 256)) // 2,
+                      "58ba5df98181": ((464767488 + 147933696)
                                          + (258423552 + 57020416 + 33059584 + 256)) // 2,
                       "769ac7621d63": ((563601152 + 158165760)
                                          + (259388672 + 57002752 + 33059840 + 3328)) // 2,
