@@ -184,6 +184,9 @@ class MLPStep:
         # codes
         self.stack = stack_gate_up and not self.i8 and not packed and optimizer == "adamw"
         self.grid = dqt.grid(bits)
+        # FP8 forward on codes beyond 16 in magnitude: the split E4M3 image
+        # [N, 2K] (dqt_codes_to_fp8_split), converted every step
+        self.w8_split = fp8 and dqt.fp8_split_grid(self.grid)
         T = T_TOK
         # two seeded input sets, alternated step by step, so that the
         # optimiser sees changing gradients as in training
@@ -216,7 +219,8 @@ class MLPStep:
             self.v_gu = torch.zeros((2 * INTER, HID), dtype=torch.float32, device=dev)
             self.W_img_gu = torch.empty((2 * INTER, HID), dtype=torch.bfloat16, device=dev)
             if fp8:
-                self.W8_gu = torch.empty((2 * INTER, HID), dtype=torch.uint8, device=dev)
+                self.W8_gu = torch.empty((2 * INTER, HID * (2 if self.w8_split else 1)),
+                                         dtype=torch.uint8, device=dev)
             self.Y_gu = torch.empty((T, 2 * INTER), dtype=torch.bfloat16, device=dev)
         for i, (name, K, N) in enumerate(PROJ):
             W0 = inputs.normal((N, K), 0.02, seed=20 + i).to(dev)
@@ -244,7 +248,8 @@ class MLPStep:
             if not self.i8:  # the int8-operand calls make their images in workspaces
                 self.W_img[name] = torch.empty((N, K), dtype=torch.bfloat16, device=dev)
             if fp8:
-                self.W8[name] = torch.empty((N, K), dtype=torch.uint8, device=dev)
+                self.W8[name] = torch.empty((N, K * (2 if self.w8_split else 1)), dtype=torch.uint8,
+                                            device=dev)
             self.Y[name] = torch.empty((T, N), dtype=torch.bfloat16, device=dev)
             self.dX[name] = torch.empty((T, K), dtype=torch.bfloat16, device=dev)
         # image operands with AdamW on int8 codes: each weight-gradient call
@@ -253,7 +258,8 @@ class MLPStep:
         # step converts codes to images; the buffers swap after every step
         # (with the FP8 forward, the E4M3 image of the forward beside the bf16
         # image of dX, both written by the update)
-        self.nimg = next_image and not self.i8 and not packed and optimizer == "adamw"
+        self.nimg = (next_image and not self.i8 and not packed and optimizer == "adamw"
+                     and not self.w8_split)
         if self.nimg:
             self.W_img_next, self.W8_next = {}, {}
             if self.stack:
@@ -439,7 +445,8 @@ class MLPStep:
             if name == "gate_up":  # both stacked weights' image in one launch
                 if self.fp8:
                     timed("codes_to_fp8", stream,
-                          lambda: dqt.dqt_codes_to_fp8(self.W_gu, self.grid, self.W8_gu))
+                          lambda: dqt.dqt_codes_to_fp8_split(self.W_gu, self.W8_gu) if self.w8_split
+                          else dqt.dqt_codes_to_fp8(self.W_gu, self.grid, self.W8_gu))
                 timed("codes_to_bf16", stream,
                       lambda: dqt.dqt_codes_to_bf16(self.W_gu, self.W_img_gu))
                 return
@@ -447,6 +454,7 @@ class MLPStep:
             if self.fp8:
                 timed("codes_to_fp8", stream,
                       lambda: dqt.dqt_packed_to_fp8(self.W[name], shape, self.W8[name]) if self.packed
+                      else dqt.dqt_codes_to_fp8_split(self.W[name], self.W8[name]) if self.w8_split
                       else dqt.dqt_codes_to_fp8(self.W[name], self.grid, self.W8[name]))
             timed("codes_to_bf16", stream,
                   lambda: dqt.dqt_packed_to_bf16(self.W[name], shape, self.W_img[name]) if self.packed

@@ -411,9 +411,16 @@ int dqt_act_quant_fp8(const dqt_bf16* X, int64_t T, int64_t K, uint8_t* Xq8, flo
 
 /* E4M3 image of weight codes: W8[i] = E4M3(W[i]), exact because every integer
  * of magnitude <= 16 is an E4M3 value.  The grid bounds the codes: grids
- * with a code beyond 16 in magnitude (6- to 8-bit) return DQT_ERR_RANGE (use
- * the integer path, dqt_bitlinear_fwd).  numel >= 1. */
+ * with a code beyond 16 in magnitude (6- to 8-bit) return DQT_ERR_RANGE (their
+ * E4M3 form is dqt_codes_to_fp8_split).  numel >= 1. */
 int dqt_codes_to_fp8(const int8_t* W, int64_t numel, dqt_grid_t grid, uint8_t* W8, void* stream);
+
+/* E4M3 split image of codes of any width, for the FP8 forward of 6- to 8-bit
+ * grids: each code c = 16 h + l with h = c >> 4 (floor(c / 16), in [-8, 7])
+ * and l = c & 15 (in [0, 15]); 16 h and l are E4M3 values, so both halves
+ * are exact.  W int8 [N, K] -> W8 uint8 [N, 2K]: row n holds E4M3(16 h) of
+ * its K codes, then E4M3(l).  K a multiple of 16. */
+int dqt_codes_to_fp8_split(const int8_t* W, int64_t N, int64_t K, uint8_t* W8, void* stream);
 
 /* Forward on E4M3 operands (tcgen05 kind::f8f6f4, fp32 accumulation):
  *   acc[t,n] = sum_k value(Xq8[t,k]) * c[n,k]       fp32 accumulator
@@ -421,8 +428,12 @@ int dqt_codes_to_fp8(const int8_t* W, int64_t numel, dqt_grid_t grid, uint8_t* W
  * Each product is exact; the sum is rounded by the fp32 accumulation (in an
  * order the hardware chooses), so Y equals the exact-sum formula up to that
  * rounding.  Xq8 uint8 [T, K], s_x8 fp32 [T] (dqt_act_quant_fp8); W8 uint8
- * [N, K] (dqt_codes_to_fp8); grid as for dqt_codes_to_fp8; Y bf16 [T, N] out;
- * acc_out fp32 [T, N] out, or NULL.  K a multiple of 16, N of 8. */
+ * [N, K] (dqt_codes_to_fp8) for grids within 16 in magnitude; Y bf16 [T, N]
+ * out; acc_out fp32 [T, N] out, or NULL.  K a multiple of 16, N of 8.
+ * Grids beyond 16 (6- to 8-bit): W8 is the split image uint8 [N, 2K]
+ * (dqt_codes_to_fp8_split) and the sum runs over both halves, the activation
+ * row read for each: acc = sum_k value(Xq8[t,k]) 16 h[n,k] + value(Xq8[t,k])
+ * l[n,k], 2K exact products accumulated in fp32; K a multiple of 128. */
 int dqt_bitlinear_fwd_fp8(const uint8_t* Xq8, const float* s_x8, const uint8_t* W8, float s_w,
                           dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
                           float* acc_out, void* stream);
@@ -432,7 +443,8 @@ int dqt_bitlinear_fwd_fp8(const uint8_t* Xq8, const float* s_x8, const uint8_t* 
  * E4M3 images (rows [0, N0) the first's), Y bf16 [T, N] both outputs side by
  * side, the columns [0, N0) scaled with s_w0 and the rest with s_w1: Y and
  * acc_out equal two dqt_bitlinear_fwd_fp8 calls', bit for bit.  N0 a multiple
- * of 256, 0 < N0 < N; the rest as for dqt_bitlinear_fwd_fp8. */
+ * of 256, 0 < N0 < N; the rest (the split image of wide grids included) as
+ * for dqt_bitlinear_fwd_fp8. */
 int dqt_bitlinear_fwd_fp8_pair(const uint8_t* Xq8, const float* s_x8, const uint8_t* W8, int64_t N0,
                                float s_w0, float s_w1, dqt_grid_t grid, int64_t T, int64_t K,
                                int64_t N, dqt_bf16* Y, float* acc_out, void* stream);

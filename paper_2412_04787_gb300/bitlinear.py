@@ -150,8 +150,12 @@ class DQTBitLinear(torch.nn.Module):
         self.out_features = out_features
         g = dqt.grid(bits)
         self.grid_tuple = (g.qmin, g.qmax)
-        if act == "fp8" and (g.qmin < -16 or g.qmax > 16):
-            raise ValueError("the E4M3 weight image holds codes up to 16 in magnitude (<= 5 bits)")
+        # E4M3 weight image: the codes themselves up to 16 in magnitude (<= 5
+        # bits), else the split image [N, 2K] of 16 (c >> 4) and c & 15
+        self.w8_split = act == "fp8" and (g.qmin < -16 or g.qmax > 16)
+        if self.w8_split and in_features % 128:
+            raise ValueError("the split E4M3 forward (6- to 8-bit codes) needs in_features a "
+                             "multiple of 128")
         if self.packed and (g.qmin, g.qmax) != (-1, 1):
             raise ValueError("packed storage holds ternary codes only")
         self.lr, self.betas, self.eps, self.weight_decay = lr, tuple(betas), eps, weight_decay
@@ -222,6 +226,8 @@ class DQTBitLinear(torch.nn.Module):
         shape = (self.out_features, self.in_features)
         if self.packed:
             return dqt.dqt_packed_to_fp8(self.codes, shape)
+        if self.w8_split:
+            return dqt.dqt_codes_to_fp8_split(self.codes)
         return dqt.dqt_codes_to_fp8(self.codes, self.grid_tuple)
 
     def _images_kept(self):
@@ -248,11 +254,15 @@ class DQTBitLinear(torch.nn.Module):
         if not self._images_kept():
             return self.weight_fp8()
         if self._img8 is None:
-            self._img8 = torch.empty((self.out_features, self.in_features), dtype=torch.uint8,
-                                     device=self.codes.device)
+            self._img8 = torch.empty((self.out_features,
+                                      self.in_features * (2 if self.w8_split else 1)),
+                                     dtype=torch.uint8, device=self.codes.device)
             self._img8_version = -1
         if self._img8_version != self.codes._version:
-            dqt.dqt_codes_to_fp8(self.codes, self.grid_tuple, self._img8)
+            if self.w8_split:
+                dqt.dqt_codes_to_fp8_split(self.codes, self._img8)
+            else:
+                dqt.dqt_codes_to_fp8(self.codes, self.grid_tuple, self._img8)
             self._img8_version = self.codes._version
         return self._img8
 
@@ -263,6 +273,11 @@ class DQTBitLinear(torch.nn.Module):
         v = self.codes._version
         img = self._img if self._img is not None and self._img_version == v else None
         img8 = self._img8 if self._img8 is not None and self._img8_version == v else None
+        if img8 is not None and self.w8_split:
+            # the update writes the plain E4M3 image only: the split one is
+            # rebuilt from the new codes at the next forward
+            img8 = None
+            self._img8_version = -1
         return img, img8
 
     def _hyper(self, step):

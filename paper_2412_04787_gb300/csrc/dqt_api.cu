@@ -418,22 +418,35 @@ int dqt_codes_to_fp8(const int8_t* W, int64_t numel, dqt_grid_t grid, uint8_t* W
   return dqt::launch_codes_to_fp8(W, numel, W8, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
+int dqt_codes_to_fp8_split(const int8_t* W, int64_t N, int64_t K, uint8_t* W8, void* stream) {
+  if (!W || !W8 || N <= 0 || K <= 0) return DQT_ERR_ARG;
+  if (N > kMaxDim || K > kMaxDim) return DQT_ERR_RANGE;
+  if (K % 16 || !aligned16(W) || !aligned16(W8)) return DQT_ERR_ALIGN;
+  return dqt::launch_codes_to_fp8_split(W, N, K, W8, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
+// The E4M3 forward's weight form for a grid: codes within 16 in magnitude are
+// E4M3 values (W8 [N, K]); wider codes take the split image (W8 [N, 2K], the
+// activation row read for both halves; K a multiple of 128).
+static bool fp8_split(dqt_grid_t grid) { return grid.qmin < -16 || grid.qmax > 16; }
+
 int dqt_bitlinear_fwd_fp8(const uint8_t* Xq8, const float* s_x8, const uint8_t* W8, float s_w,
                           dqt_grid_t grid, int64_t T, int64_t K, int64_t N, dqt_bf16* Y,
                           float* acc_out, void* stream) {
   if (!Xq8 || !s_x8 || !W8 || !Y || T <= 0 || K <= 0 || N <= 0 || !grid_ok(grid) ||
       !(s_w > 0.0f) || !isfinite(s_w))
     return DQT_ERR_ARG;
-  if (grid.qmin < -16 || grid.qmax > 16) return DQT_ERR_RANGE;
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
-  if (K % 16 || N % 8 || !aligned16(Xq8) || !aligned16(W8) || !aligned16(Y) ||
+  const bool split = fp8_split(grid);
+  if (K % (split ? 128 : 16) || N % 8 || !aligned16(Xq8) || !aligned16(W8) || !aligned16(Y) ||
       (acc_out && !aligned16(acc_out)))
     return DQT_ERR_ALIGN;
   dqt::GemmLaunch g{};
   g.kind = dqt::GEMM_FWD8;
   g.M = static_cast<int>(T);
   g.N = static_cast<int>(N);
-  g.Kred = static_cast<int>(K);
+  g.Kred = static_cast<int>(split ? 2 * K : K);
+  g.a_wrap = split ? static_cast<int>(K) : 0;
   g.A = Xq8;
   g.B = W8;
   g.pair = true;
@@ -451,16 +464,17 @@ int dqt_bitlinear_fwd_fp8_pair(const uint8_t* Xq8, const float* s_x8, const uint
       !(s_w0 > 0.0f) || !isfinite(s_w0) || !(s_w1 > 0.0f) || !isfinite(s_w1) ||
       !pair_split_ok(N0, N))
     return DQT_ERR_ARG;
-  if (grid.qmin < -16 || grid.qmax > 16) return DQT_ERR_RANGE;
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim) return DQT_ERR_RANGE;
-  if (K % 16 || N % 8 || !aligned16(Xq8) || !aligned16(W8) || !aligned16(Y) ||
+  const bool split = fp8_split(grid);
+  if (K % (split ? 128 : 16) || N % 8 || !aligned16(Xq8) || !aligned16(W8) || !aligned16(Y) ||
       (acc_out && !aligned16(acc_out)))
     return DQT_ERR_ALIGN;
   dqt::GemmLaunch g{};
   g.kind = dqt::GEMM_FWD8;
   g.M = static_cast<int>(T);
   g.N = static_cast<int>(N);
-  g.Kred = static_cast<int>(K);
+  g.Kred = static_cast<int>(split ? 2 * K : K);
+  g.a_wrap = split ? static_cast<int>(K) : 0;
   g.A = Xq8;
   g.B = W8;
   g.pair = true;

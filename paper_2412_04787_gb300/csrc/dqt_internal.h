@@ -67,6 +67,10 @@ struct GemmLaunch {
   int64_t lda;  // DX: elements between rows of A (dY); 0: packed rows
   void* img_next;   // DW: bf16 image of the updated codes, or NULL
   void* img8_next;  // DW: E4M3 image of the updated codes, or NULL
+  // FWD8 on split codes: B is [N, Kred = 2 a_wrap] (each code c as 16 (c >> 4)
+  // in the first half of its row and c & 15 in the second) and A [M, a_wrap]
+  // is read twice, k-block kb from column (kb * 128) mod a_wrap; 0: no split
+  int a_wrap;
 };
 
 // Token slices the 2-SM dW GEMM of an M x N output reduced over Kred uses
@@ -126,6 +130,10 @@ int launch_codes_to_xdq(const int8_t* Xq, const float* s_x, int64_t T, int64_t K
 int launch_act_quant_fp8(const uint16_t* X, int64_t T, int64_t K, uint8_t* Xq8, float* s8,
                          uint16_t* Xdq, cudaStream_t stream);
 int launch_codes_to_fp8(const int8_t* W, int64_t numel, uint8_t* W8, cudaStream_t stream);
+// E4M3 split image of codes [N, K] (K % 16 == 0): W8 [N, 2K], row n holds
+// 16 (c >> 4) for every code of row n, then c & 15 (both exact in E4M3).
+int launch_codes_to_fp8_split(const int8_t* W, int64_t N, int64_t K, uint8_t* W8,
+                              cudaStream_t stream);
 int launch_absmean_partial(const float* W0, int64_t numel, double* ws, cudaStream_t stream);
 int launch_absmean_codes(const float* W0, int64_t numel, float s_w, int32_t qmin, int32_t qmax,
                          int8_t* codes, cudaStream_t stream);

@@ -134,6 +134,9 @@ struct Params {
   // stochastic-rounding generator that are the same for every element of
   // the call, for uc and uc1
   PhiloxCall pc, pc1;
+  // FWD8 on split codes: A's k-block kb is read from column (kb * 128) mod
+  // a_wrap (the activation row serves both halves of the split weight row)
+  int a_wrap;
 };
 
 // The bf16 image of four codes (exact: integers of magnitude <= 128).
@@ -956,7 +959,7 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
           uint8_t* b = sB + s * S::B_BYTES;
           const int k0 = kb * KB;
           if (!A_MN) {
-            tma_load_2d_pair(&tmA, bar, a, k0, m0);
+            tma_load_2d_pair(&tmA, bar, a, F8 && p.a_wrap ? k0 % p.a_wrap : k0, m0);
           } else if (EPI == GEMM_DW && p.col_major) {
             // column-major tiles: dY's panels are re-read by every wave
 #pragma unroll
@@ -1588,6 +1591,7 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   p.pc1 = philox_call_consts(g.uc1);
   p.img_next = g.kind == GEMM_DW ? static_cast<__nv_bfloat16*>(g.img_next) : nullptr;
   p.img8_next = g.kind == GEMM_DW ? static_cast<uint8_t*>(g.img8_next) : nullptr;
+  p.a_wrap = g.kind == GEMM_FWD8 ? g.a_wrap : 0;
   if ((p.img_next || p.img8_next) && (g.packed || !g.W)) return 1;
   // stacked weights: whole tiles (multiples of 256 of either tiling),
   // constants in the parameter space
@@ -1616,7 +1620,8 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
       return launch_tiles<256, false, false, GEMM_FWD, false>(ta, tb, p, stream);
     case GEMM_FWD8:
       // 2-SM tiles whatever the tiling mode: E4M3 rows of 128 elements
-      if (!make_map(&ta, g.A, g.Kred, g.M, 128, BM, 1)) return 3;
+      if (g.a_wrap && (g.a_wrap % 128 != 0 || g.Kred != 2 * g.a_wrap)) return 1;
+      if (!make_map(&ta, g.A, g.a_wrap ? g.a_wrap : g.Kred, g.M, 128, BM, 1)) return 3;
       if (!make_map(&tb, g.B, g.Kred, g.N, 128, 128, 1)) return 3;
       return launch_pairs<false, false, GEMM_FWD8>(ta, tb, p, stream);
     case GEMM_DX:

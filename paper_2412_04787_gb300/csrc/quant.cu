@@ -529,6 +529,44 @@ __global__ void codes_to_fp8_kernel(const int8_t* __restrict__ W, int64_t numel,
       out[e] = static_cast<uint8_t>(codes4_to_e4m3(static_cast<uint8_t>(W[e])) & 0xFFu);
 }
 
+// E4M3 split image of codes wider than 16 in magnitude: c = 16 h + l with
+// h = c >> 4 (floor(c / 16), in [-8, 7]) and l = c & 15 (in [0, 15]); 16 h
+// (a multiple of 16 of magnitude <= 128, at most three significant bits)
+// and l are E4M3 values, so each half is exact.  Row n of the [N, 2K] image:
+// 16 h of its K codes, then their l.  One thread step: 16 codes of a row.
+__global__ void codes_to_fp8_split_kernel(const int8_t* __restrict__ W, int64_t N, int64_t K,
+                                          uint8_t* __restrict__ out) {
+  const int64_t vpr = K >> 4;  // 16-code vectors per row
+  const int64_t nvec = N * vpr;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
+       i += stride) {
+    const int64_t n = i / vpr, k = (i - n * vpr) << 4;
+    const uint4 u = __ldcs(reinterpret_cast<const uint4*>(W + n * K + k));
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+    uint32_t hi[4], lo[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      float h[4], l[4];
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        const int32_t c = static_cast<int8_t>((w[j] >> (8 * b)) & 0xFFu);
+        h[b] = static_cast<float>(16 * (c >> 4));
+        l[b] = static_cast<float>(c & 15);
+      }
+      const uint32_t h01 = __nv_cvt_float2_to_fp8x2(make_float2(h[0], h[1]), __NV_SATFINITE, __NV_E4M3);
+      const uint32_t h23 = __nv_cvt_float2_to_fp8x2(make_float2(h[2], h[3]), __NV_SATFINITE, __NV_E4M3);
+      const uint32_t l01 = __nv_cvt_float2_to_fp8x2(make_float2(l[0], l[1]), __NV_SATFINITE, __NV_E4M3);
+      const uint32_t l23 = __nv_cvt_float2_to_fp8x2(make_float2(l[2], l[3]), __NV_SATFINITE, __NV_E4M3);
+      hi[j] = (h01 & 0xFFFFu) | ((h23 & 0xFFFFu) << 16);
+      lo[j] = (l01 & 0xFFFFu) | ((l23 & 0xFFFFu) << 16);
+    }
+    uint8_t* row = out + n * 2 * K;
+    __stcs(reinterpret_cast<uint4*>(row + k), make_uint4(hi[0], hi[1], hi[2], hi[3]));
+    __stcs(reinterpret_cast<uint4*>(row + K + k), make_uint4(lo[0], lo[1], lo[2], lo[3]));
+  }
+}
+
 // Eq. 2, stage 1: each of kAbsmeanBlocks blocks sums |w| in fp64 over a fixed
 // strided subset and reduces in a fixed tree: the result does not depend on
 // scheduling.
@@ -687,6 +725,13 @@ int launch_act_quant_fp8(const uint16_t* X, int64_t T, int64_t K, uint8_t* Xq8, 
 int launch_codes_to_fp8(const int8_t* W, int64_t numel, uint8_t* W8, cudaStream_t stream) {
   const int threads = 256;
   codes_to_fp8_kernel<<<grid_for((numel >> 4) + 1, threads), threads, 0, stream>>>(W, numel, W8);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
+}
+
+int launch_codes_to_fp8_split(const int8_t* W, int64_t N, int64_t K, uint8_t* W8,
+                              cudaStream_t stream) {
+  const int threads = 256;
+  codes_to_fp8_split_kernel<<<grid_for(N * (K >> 4), threads), threads, 0, stream>>>(W, N, K, W8);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 

@@ -23,7 +23,8 @@ EXPORTED = [
     "dqt_bitlinear_bwd_dw_update", "dqt_sr_update", "dqt_absmean_init_noalloc",
     "dqt_set_gemm_tiles", "dqt_update_consts_size", "dqt_update_consts",
     "dqt_bitlinear_bwd_dw_update_dev", "dqt_sr_update_dev", "dqt_bwd_dw_workspace_size",
-    "dqt_act_quant_fp8", "dqt_codes_to_fp8", "dqt_bitlinear_fwd_fp8", "dqt_bitlinear_fwd_fp8_pair",
+    "dqt_act_quant_fp8", "dqt_codes_to_fp8", "dqt_codes_to_fp8_split", "dqt_bitlinear_fwd_fp8",
+    "dqt_bitlinear_fwd_fp8_pair",
     "dqt_pack_ternary", "dqt_unpack_ternary", "dqt_packed_to_bf16", "dqt_packed_to_fp8",
     "dqt_sr_update_packed", "dqt_bitlinear_bwd_dw_update_packed",
     "dqt_adafactor_workspace_size", "dqt_adafactor_stats", "dqt_adafactor_apply",
@@ -141,6 +142,7 @@ def lib():
         L.dqt_sr_update_dev.argtypes = [_vp, _vp, _vp, _vp, _vp, _i64, _vp, _vp]
         L.dqt_act_quant_fp8.argtypes = [_vp, _i64, _i64, _vp, _vp, _vp, _vp]
         L.dqt_codes_to_fp8.argtypes = [_vp, _i64, dqt_grid_t, _vp, _vp]
+        L.dqt_codes_to_fp8_split.argtypes = [_vp, _i64, _i64, _vp, _vp]
         L.dqt_bitlinear_fwd_fp8.argtypes = [_vp, _vp, _vp, _f32, dqt_grid_t, _i64, _i64, _i64,
                                             _vp, _vp, _vp]
         L.dqt_bitlinear_fwd_fp8_pair.argtypes = [_vp, _vp, _vp, _i64, _f32, _f32, dqt_grid_t, _i64,
@@ -700,12 +702,36 @@ def dqt_codes_to_fp8(W, bits_or_grid, W8=None, stream=None):
     return W8
 
 
+def dqt_codes_to_fp8_split(W, W8=None, stream=None):
+    """E4M3 split image [N, 2K] of int8 codes [N, K] of any width: 16 (c >> 4)
+    in the first half of each row, c & 15 in the second."""
+    _need(W, "W", torch.int8)
+    if W.dim() != 2:
+        raise ValueError("W must be [N, K]")
+    N, K = W.shape
+    if W8 is None:
+        W8 = torch.empty((N, 2 * K), dtype=torch.uint8, device=W.device)
+    _need(W8, "W8", torch.uint8, (N, 2 * K))
+    _check(lib().dqt_codes_to_fp8_split(_ptr(W), N, K, _ptr(W8), _stream(stream)),
+           "dqt_codes_to_fp8_split")
+    return W8
+
+
+def fp8_split_grid(bits_or_grid):
+    """Whether the E4M3 forward takes the split weight image [N, 2K] for this
+    grid (codes beyond 16 in magnitude)."""
+    g = _grid(bits_or_grid)
+    return g.qmin < -16 or g.qmax > 16
+
+
 def dqt_bitlinear_fwd_fp8(Xq8, s_x8, W8, s_w, bits_or_grid, Y=None, acc_out=None, stream=None):
+    """The E4M3 forward; W8 [N, K] (dqt_codes_to_fp8), or [N, 2K]
+    (dqt_codes_to_fp8_split) for grids beyond 16 in magnitude."""
     _need(Xq8, "Xq8", torch.uint8)
     T, K = Xq8.shape
     _need(W8, "W8", torch.uint8)
     N = W8.shape[0]
-    _need(W8, "W8", torch.uint8, (N, K))
+    _need(W8, "W8", torch.uint8, (N, 2 * K if fp8_split_grid(bits_or_grid) else K))
     _need(s_x8, "s_x8", torch.float32, (T,))
     if Y is None:
         Y = torch.empty((T, N), dtype=torch.bfloat16, device=Xq8.device)
@@ -725,7 +751,7 @@ def dqt_bitlinear_fwd_fp8_pair(Xq8, s_x8, W8, N0, s_w0, s_w1, bits_or_grid, Y=No
     T, K = Xq8.shape
     _need(W8, "W8", torch.uint8)
     N = W8.shape[0]
-    _need(W8, "W8", torch.uint8, (N, K))
+    _need(W8, "W8", torch.uint8, (N, 2 * K if fp8_split_grid(bits_or_grid) else K))
     _need(s_x8, "s_x8", torch.float32, (T,))
     if Y is None:
         Y = torch.empty((T, N), dtype=torch.bfloat16, device=Xq8.device)

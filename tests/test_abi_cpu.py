@@ -121,7 +121,8 @@ def test_argument_validation_without_launch(L):
     # the stacked FP8 forward: the same split rule, and the E4M3-exact grid
     assert L.dqt_bitlinear_fwd_fp8_pair(A, A, A, 200, 1.0, 1.0, g, 4, 16, 512, A, None, None) == dqt.DQT_ERR_ARG
     assert L.dqt_bitlinear_fwd_fp8_pair(A, A, A, 256, 1.0, 0.0, g, 4, 16, 512, A, None, None) == dqt.DQT_ERR_ARG
-    assert L.dqt_bitlinear_fwd_fp8_pair(A, A, A, 256, 1.0, 1.0, g8, 4, 16, 512, A, None, None) == dqt.DQT_ERR_RANGE
+    # wide grids take the split image: the reduction a multiple of 128
+    assert L.dqt_bitlinear_fwd_fp8_pair(A, A, A, 256, 1.0, 1.0, g8, 4, 16, 512, A, None, None) == dqt.DQT_ERR_ALIGN
     # bad grid / scale
     assert L.dqt_bitlinear_fwd(A, A, A, 1.0, dqt.dqt_grid_t(2, 1), 4, 8, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ARG
     assert L.dqt_bitlinear_fwd(A, A, A, 1.0, dqt.dqt_grid_t(-129, 1), 4, 8, 8, A, None, A, 1 << 24, None) == dqt.DQT_ERR_ARG
@@ -182,7 +183,10 @@ def test_fp8_argument_validation(L):
     assert L.dqt_codes_to_fp8(A, 64, dqt.dqt_grid_t(-32, 31), A, None) == dqt.DQT_ERR_RANGE
     assert L.dqt_codes_to_fp8(A, 0, t, A, None) == dqt.DQT_ERR_ARG
     # forward
-    assert L.dqt_bitlinear_fwd_fp8(A, A, A, 1.0, g8, 4, 32, 8, A, None, None) == dqt.DQT_ERR_RANGE
+    assert L.dqt_bitlinear_fwd_fp8(A, A, A, 1.0, g8, 4, 32, 8, A, None, None) == dqt.DQT_ERR_ALIGN
+    # the split image: K a multiple of 16
+    assert L.dqt_codes_to_fp8_split(A, 4, 24, A, None) == dqt.DQT_ERR_ALIGN
+    assert L.dqt_codes_to_fp8_split(A, 0, 32, A, None) == dqt.DQT_ERR_ARG
     assert L.dqt_bitlinear_fwd_fp8(A, A, A, 1.0, t, 4, 24, 8, A, None, None) == dqt.DQT_ERR_ALIGN
     assert L.dqt_bitlinear_fwd_fp8(A, A, A, 1.0, t, 4, 32, 12, A, None, None) == dqt.DQT_ERR_ALIGN
     assert L.dqt_bitlinear_fwd_fp8(A, A, A, 0.0, t, 4, 32, 8, A, None, None) == dqt.DQT_ERR_ARG

@@ -155,3 +155,91 @@ def test_fwd_fp8_matches_integer_path_on_integer_values():
     Y_int, acc_int = oracle.fwd(q.numpy(), s, c, s_w)
     assert (acc.cpu().numpy() == acc_int.astype(np.float32)).all()
     assert (bits(Y8) == Y_int).all()
+
+
+def _split_halves(c):
+    """The split of codes c = 16 h + l (h = c >> 4, l = c & 15)."""
+    c = c.astype(np.int32)
+    return 16 * (c >> 4), c & 15
+
+
+@pytest.mark.parametrize("N,K", [(64, 16), (520, 256), (1000, 2048)])
+def test_codes_to_fp8_split_exact(N, K):
+    g = torch.Generator().manual_seed(N + K)
+    c = torch.randint(-128, 128, (N, K), generator=g, dtype=torch.int8)
+    h16, l = _split_halves(c.numpy())
+    ref = np.concatenate([oracle.codes_to_e4m3(h16.astype(np.int16)),
+                          oracle.codes_to_e4m3(l.astype(np.int16))], axis=1)
+    got = dqt.dqt_codes_to_fp8_split(c.cuda()).cpu().numpy()
+    assert (got == ref).all()
+    # both halves are exact: their values add back to the codes
+    v = np.vectorize(oracle.e4m3_value)(got).astype(np.float64)
+    assert (v[:, :K] + v[:, K:] == c.numpy().astype(np.float64)).all()
+
+
+def _check_fwd_split(q8, s8, c, s_w, Y_gpu, acc_gpu, rows=None):
+    """The split forward: 2K exact products in fp32, so the accumulators are
+    held to (2K - 1) 2^-24 sum_k |value(Xq8)| (|16 h| + |l|) of the exact sum
+    (the oracle's, over value(Xq8) c) and Y to one bf16 ulp plus that bound
+    scaled by 1 / (s_x8 s_w)."""
+    q8r = q8 if rows is None else q8[rows]
+    s8r = s8 if rows is None else s8[rows]
+    Y_ref, acc_ref = oracle.fwd_fp8(q8r, s8r, c, s_w)
+    xv = np.vectorize(oracle.e4m3_value)(q8r)
+    h16, l = _split_halves(c)
+    mag = np.abs(xv) @ (np.abs(h16) + np.abs(l)).astype(np.float64).T
+    K = q8.shape[1]
+    bound = (2 * K - 1) * 2.0 ** -24 * mag
+    acc_g = acc_gpu if rows is None else acc_gpu[rows]
+    err = np.abs(acc_g.astype(np.float64) - acc_ref)
+    assert (err <= bound).all(), float((err / np.maximum(bound, 1e-300)).max())
+    a_t = (np.float32(1.0) / (s8r.astype(np.float32) * np.float32(s_w))).astype(np.float64)
+    y_ref = torch.from_numpy(Y_ref.view(np.int16)).view(torch.bfloat16).double().numpy()
+    Yg = Y_gpu if rows is None else Y_gpu[rows]
+    y_gpu = torch.from_numpy(Yg.view(np.int16)).view(torch.bfloat16).double().numpy()
+    ulp = np.exp2(np.floor(np.log2(np.maximum(np.abs(y_ref), 1e-38))) - 7)
+    assert (np.abs(y_gpu - y_ref) <= ulp + a_t[:, None] * bound * 1.01).all()
+    return float((Y_ref == Yg).mean())
+
+
+@pytest.mark.parametrize("T,K,N,bits_w", [(256, 512, 512, 8), (300, 256, 520, 8), (129, 384, 264, 6)])
+def test_fwd_fp8_split_codes(T, K, N, bits_w):
+    """6- to 8-bit codes through the FP8 forward: the split image, the
+    activation row read for both halves."""
+    X = _x(T, K, seed=5 * T + K)
+    W0 = inputs.normal((N, K), 0.02, seed=N + 11)
+    qmin, qmax = oracle.grid(bits_w)
+    c, s_w, _ = oracle.absmean_init(W0.numpy(), qmin, qmax)
+    q8, s8, _ = oracle.act_quant_fp8(bits(X))
+    W8 = dqt.dqt_codes_to_fp8_split(torch.from_numpy(c).cuda())
+    acc = torch.empty((T, N), dtype=torch.float32, device="cuda")
+    Y = dqt.dqt_bitlinear_fwd_fp8(torch.from_numpy(q8).cuda(), torch.from_numpy(s8).cuda(), W8,
+                                  float(s_w), (qmin, qmax), acc_out=acc)
+    dqt.dqt_check_device_status()
+    same = _check_fwd_split(q8, s8, c, float(s_w), bits(Y), acc.cpu().numpy())
+    assert same > 0.8, same
+
+
+def test_fwd_fp8_split_llama_mlp_sampled_rows_and_pair():
+    """8-bit codes at the MLP's gate/up shape (T = 8192, K = 2048, N = 2 x
+    5632 stacked, one scale per weight), on sampled rows; the stacked call
+    equals two calls bit for bit."""
+    T, K, N0 = 8192, 2048, 5632
+    X = inputs.normal((T, K), 1.0, seed=111, dtype=torch.bfloat16)
+    qmin, qmax = oracle.grid(8)
+    c0, s0, _ = oracle.absmean_init(inputs.normal((N0, K), 0.02, seed=113).numpy(), qmin, qmax)
+    c1, s1, _ = oracle.absmean_init(inputs.normal((N0, K), 0.03, seed=114).numpy(), qmin, qmax)
+    c = np.concatenate([c0, c1])
+    g8, gs, _ = dqt.dqt_act_quant_fp8(X.cuda(), want_xdq=False)
+    W8 = dqt.dqt_codes_to_fp8_split(torch.from_numpy(c).cuda())
+    acc = torch.empty((T, 2 * N0), dtype=torch.float32, device="cuda")
+    Y = dqt.dqt_bitlinear_fwd_fp8_pair(g8, gs, W8, N0, float(s0), float(s1), (qmin, qmax), acc_out=acc)
+    acc1 = torch.empty((T, N0), dtype=torch.float32, device="cuda")
+    Y1 = dqt.dqt_bitlinear_fwd_fp8(g8, gs, W8[N0:], float(s1), (qmin, qmax), acc_out=acc1)
+    dqt.dqt_check_device_status()
+    assert torch.equal(acc[:, N0:].view(torch.int32), acc1.view(torch.int32))
+    assert torch.equal(Y[:, N0:].contiguous().view(torch.int16), Y1.view(torch.int16))
+    rows = np.array([0, 1, 255, 256, 4097, 8191])
+    q8, s8, _ = oracle.act_quant_fp8(bits(X[rows]))
+    assert (g8.cpu().numpy()[rows] == q8).all()
+    _check_fwd_split(q8, s8, c0, float(s0), bits(Y[:, :N0].contiguous())[rows], acc.cpu().numpy()[rows, :N0])

@@ -128,7 +128,7 @@ def test_fwd_fp8_matches_fp64_matmul():
     Xb = inputs.normal((T, K), 1.0, seed=21, dtype=torch.bfloat16)
     q8, s8, _ = oracle.act_quant_fp8(inputs.bf16_bits(Xb))
     W0 = inputs.normal((N, K), 0.02, seed=22).numpy()
-    for qmin, qmax in [(-1, 1), (-16, 15)]:
+    for qmin, qmax in [(-1, 1), (-16, 15), (-128, 127)]:
         c, s_w, _ = oracle.absmean_init(W0, qmin, qmax)
         Y, acc = oracle.fwd_fp8(q8, s8, c, s_w)
         xv = np.vectorize(oracle.e4m3_value)(q8)  # decoded by the format definition
@@ -139,9 +139,13 @@ def test_fwd_fp8_matches_fp64_matmul():
         assert (inputs.bf16_bits(torch.from_numpy(yf).to(torch.bfloat16)) == Y).all()
 
 
-def test_fwd_fp8_rejects_codes_beyond_16():
-    q8 = np.zeros((2, 16), np.uint8)
-    c = np.zeros((8, 16), np.int8)
-    c[3, 4] = 17
-    with pytest.raises(ValueError):
-        oracle.fwd_fp8(q8, np.ones(2, np.float32), c, 1.0)
+def test_fwd_fp8_wide_codes_split_exactly():
+    """Codes beyond 16 in magnitude reach the E4M3 forward as 16 (c >> 4) and
+    c & 15: both are E4M3 values (decoded by the format definition) and they
+    add back to c for every int8 code, so the exact sum over value(q8) c is
+    the sum over the two halves."""
+    c = np.arange(-128, 128, dtype=np.int32)
+    h16, l = 16 * (c >> 4), c & 15
+    vh = np.vectorize(oracle.e4m3_value)(oracle.codes_to_e4m3(h16.astype(np.int8)))
+    vl = np.vectorize(oracle.e4m3_value)(oracle.codes_to_e4m3(l.astype(np.int8)))
+    assert (vh == h16).all() and (vl == l).all() and (vh + vl == c).all()
