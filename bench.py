@@ -185,7 +185,8 @@ class MLPStep:
         self.stack = stack_gate_up and not self.i8 and not packed and optimizer == "adamw"
         self.grid = dqt.grid(bits)
         # FP8 forward on codes beyond 16 in magnitude: the split E4M3 image
-        # [N, 2K] (dqt_codes_to_fp8_split), converted every step
+        # [N, 2K] (dqt_codes_to_fp8_split's layout, written by the update like
+        # the other images)
         self.w8_split = fp8 and dqt.fp8_split_grid(self.grid)
         T = T_TOK
         # two seeded input sets, alternated step by step, so that the
@@ -258,8 +259,7 @@ class MLPStep:
         # step converts codes to images; the buffers swap after every step
         # (with the FP8 forward, the E4M3 image of the forward beside the bf16
         # image of dX, both written by the update)
-        self.nimg = (next_image and not self.i8 and not packed and optimizer == "adamw"
-                     and not self.w8_split)
+        self.nimg = next_image and not self.i8 and not packed and optimizer == "adamw"
         if self.nimg:
             self.W_img_next, self.W8_next = {}, {}
             if self.stack:
@@ -275,9 +275,11 @@ class MLPStep:
                 else:
                     self.W_img_next[name] = torch.empty((N, K), dtype=torch.bfloat16, device=dev)
                     if fp8:
-                        self.W8_next[name] = torch.empty((N, K), dtype=torch.uint8, device=dev)
+                        self.W8_next[name] = torch.empty_like(self.W8[name])
                 dqt.dqt_codes_to_bf16(self.W[name], self.W_img[name])  # the first step's images
-                if fp8:
+                if fp8 and self.w8_split:
+                    dqt.dqt_codes_to_fp8_split(self.W[name], self.W8[name])
+                elif fp8:
                     dqt.dqt_codes_to_fp8(self.W[name], self.grid, self.W8[name])
         # per activation: (scale, forward operand, dequantised bf16 image); the
         # forward operand is the int8 codes (no image), the bf16 code image,

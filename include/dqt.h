@@ -305,10 +305,12 @@ size_t dqt_bwd_dw_workspace_size(int64_t T, int64_t N, int64_t K);
  * dqt_codes_to_bf16 would write it), written by the update itself; it must
  * not be the image any kernel still in flight reads (this step's dX): keep
  * two images and alternate them step by step.  W8_next: NULL, or uint8
- * [N, K] (16-byte aligned) that receives the E4M3 image of the updated codes
- * (the next FP8 forward's operand, as dqt_codes_to_fp8 would write it), under
- * the same rule; only for grids whose codes stay within 16 in magnitude,
- * else DQT_ERR_RANGE.  Each of the two images needs W, m, v. */
+ * (16-byte aligned) that receives the E4M3 image of the updated codes (the
+ * next FP8 forward's operand), under the same rule: for grids whose codes
+ * stay within 16 in magnitude [N, K] as dqt_codes_to_fp8 would write it, for
+ * wider grids (6- to 8-bit) the split image [N, 2K] as dqt_codes_to_fp8_split
+ * would write it (K a multiple of 16, else DQT_ERR_ALIGN).  Each of the two
+ * images needs W, m, v. */
 int dqt_bitlinear_bwd_dw_update_img(const dqt_bf16* dY, const dqt_bf16* Xdq, int8_t* W,
                                     float s_w, float* m, float* v, const dqt_adamw_t* hp,
                                     const dqt_sr_t* sr, dqt_grid_t grid, int64_t T, int64_t N,
@@ -378,8 +380,9 @@ int dqt_sr_update(const float* grad, int8_t* W, float s_w, float* m, float* v,
  * identical for identical constants.  W, m, v are required; the weight
  * gradient takes the X_tilde image Xdq, the token-slice workspace and the
  * next-step images W_img_next / W8_next of dqt_bitlinear_bwd_dw_update_img
- * (W8_next only for grids within 16 in magnitude: the grid is in the device
- * block, so this call cannot check it). */
+ * (W8_next the direct image [N, K] only, for grids within 16 in magnitude:
+ * the grid is in the device block, so this call can neither check it nor
+ * choose the split image). */
 size_t dqt_update_consts_size(void);
 int dqt_update_consts(const dqt_adamw_t* hp, const dqt_sr_t* sr, dqt_grid_t grid, float s_w,
                       void* out, size_t out_bytes);

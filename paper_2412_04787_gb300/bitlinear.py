@@ -273,8 +273,9 @@ class DQTBitLinear(torch.nn.Module):
         v = self.codes._version
         img = self._img if self._img is not None and self._img_version == v else None
         img8 = self._img8 if self._img8 is not None and self._img8_version == v else None
-        if img8 is not None and self.w8_split:
-            # the update writes the plain E4M3 image only: the split one is
+        if img8 is not None and self.w8_split and self.uc_dev is not None:
+            # with the constants in device memory the update cannot tell the
+            # grid, and writes the plain E4M3 image only: the split one is
             # rebuilt from the new codes at the next forward
             img8 = None
             self._img8_version = -1

@@ -616,9 +616,11 @@ int dqt_bitlinear_bwd_dw_update_img(const dqt_bf16* dY, const dqt_bf16* Xdq, int
   if (!dY || !Xdq || T <= 0 || N <= 0 || K <= 0) return DQT_ERR_ARG;
   if (upd && (!W || !m || !v)) return DQT_ERR_ARG;
   if (!upd && (!dW_out || W_img_next || W8_next)) return DQT_ERR_ARG;
-  if (W8_next && (grid.qmin < -16 || grid.qmax > 16)) return DQT_ERR_RANGE;
+  // codes wider than E4M3's exact integers: W8_next receives the split image
+  const bool w8_split = W8_next && fp8_split(grid);
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
-  if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(Xdq) || (W && !aligned16(W)) ||
+  if (K % 8 || N % 8 || (w8_split && K % 16) || !aligned16(dY) || !aligned16(Xdq) ||
+      (W && !aligned16(W)) ||
       (m && !aligned16(m)) || (v && !aligned16(v)) || (dW_out && !aligned16(dW_out)) ||
       (W_img_next && !aligned16(W_img_next)) || (W8_next && !aligned16(W8_next)) ||
       (ws && !aligned16(ws)))
@@ -642,6 +644,7 @@ int dqt_bitlinear_bwd_dw_update_img(const dqt_bf16* dY, const dqt_bf16* Xdq, int
   g.dW_out = dW_out;
   g.img_next = W_img_next;
   g.img8_next = W8_next;
+  g.img8_split = w8_split;
   g.changed = upd ? changed_out : nullptr;
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
@@ -656,9 +659,10 @@ int dqt_bitlinear_bwd_dw_update_img_pair(const dqt_bf16* dY, const dqt_bf16* Xdq
                                          size_t ws_bytes, void* stream) {
   if (!dY || !Xdq || !W || !m || !v || T <= 0 || N <= 0 || K <= 0 || !pair_split_ok(N0, N))
     return DQT_ERR_ARG;
-  if (W8_next && (grid.qmin < -16 || grid.qmax > 16)) return DQT_ERR_RANGE;
+  const bool w8_split = W8_next && fp8_split(grid);
   if (T > kMaxDim || K > kMaxDim || N > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
-  if (K % 8 || N % 8 || !aligned16(dY) || !aligned16(Xdq) || !aligned16(W) || !aligned16(m) ||
+  if (K % 8 || N % 8 || (w8_split && K % 16) || !aligned16(dY) || !aligned16(Xdq) ||
+      !aligned16(W) || !aligned16(m) ||
       !aligned16(v) || (dW_out && !aligned16(dW_out)) ||
       (W_img_next && !aligned16(W_img_next)) || (W8_next && !aligned16(W8_next)) ||
       (ws && !aligned16(ws)))
@@ -682,6 +686,7 @@ int dqt_bitlinear_bwd_dw_update_img_pair(const dqt_bf16* dY, const dqt_bf16* Xdq
   g.dW_out = dW_out;
   g.img_next = W_img_next;
   g.img8_next = W8_next;
+  g.img8_split = w8_split;
   g.changed = changed_out;
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }

@@ -67,6 +67,9 @@ struct GemmLaunch {
   int64_t lda;  // DX: elements between rows of A (dY); 0: packed rows
   void* img_next;   // DW: bf16 image of the updated codes, or NULL
   void* img8_next;  // DW: E4M3 image of the updated codes, or NULL
+  // DW: img8_next is the split image [M, 2 N] (16 (c >> 4), then c & 15 in
+  // each row) of codes wider than E4M3's exact integers
+  bool img8_split;
   // FWD8 on split codes: B is [N, Kred = 2 a_wrap] (each code c as 16 (c >> 4)
   // in the first half of its row and c & 15 in the second) and A [M, a_wrap]
   // is read twice, k-block kb from column (kb * 128) mod a_wrap; 0: no split
@@ -97,22 +100,25 @@ size_t gemm_tail_bytes(int M, int N, int Kred);
 // 65536 floats, tile-local row-major 256 x 256; tile full + j of an M x N
 // output with num_n tiles per row) in slice order and applies the update of
 // sr_update_kernel to W, m, v (if W) at the global element indices, and/or
-// writes the summed gradient to dW_out.
+// writes the summed gradient to dW_out.  img8_split: img8_next is the split
+// E4M3 image, rows of 2 N bytes.
 int launch_tail_update(const float* part, int splits, int tail, int full, int num_n, int M, int N,
                        int8_t* W, bool packed, float* m, float* v, const UpdateConsts& uc,
                        const UpdateConsts* uc_dev, unsigned long long* changed, float* dW_out,
                        cudaStream_t stream, const UpdateConsts* uc1 = nullptr, int split = 0,
                        bool col_major = false, uint16_t* img_next = nullptr,
-                       uint8_t* img8_next = nullptr);
+                       uint8_t* img8_next = nullptr, bool img8_split = false);
 
 // Sum `splits` fp32 slabs (stride `slab` elements) in slice order and apply
 // the update to W, m, v (numel elements); optionally write the sum to g_out
-// and the bf16 / E4M3 images of the new codes to img / img8 (int8 codes).
+// and the bf16 / E4M3 images of the new codes to img / img8 (int8 codes);
+// img8_k > 0: img8 is the split E4M3 image of rows of img8_k codes (2 img8_k
+// bytes each: 16 (c >> 4), then c & 15), numel a multiple of img8_k.
 int launch_sr_update_slabs(const float* slabs, int splits, long long slab, int8_t* W, float* m,
                            float* v, int64_t numel, const UpdateConsts& uc,
                            const UpdateConsts* uc_dev, unsigned long long* changed, float* g_out,
                            cudaStream_t stream, bool packed = false, uint16_t* img = nullptr,
-                           uint8_t* img8 = nullptr);
+                           uint8_t* img8 = nullptr, int64_t img8_k = 0);
 // Sum the slabs into out (gradient only).
 int launch_slab_sum(const float* slabs, int splits, long long slab, float* out,
                     cudaStream_t stream);

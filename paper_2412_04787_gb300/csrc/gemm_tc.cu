@@ -128,8 +128,10 @@ struct Params {
   // (the next forward's operand), at the code's element index
   __nv_bfloat16* img_next;
   // dW: if set, the E4M3 image of every updated code (the next FP8 forward's
-  // operand; exact for |code| <= 16)
+  // operand; exact for |code| <= 16), or with img8_split the split image
+  // [M, 2N] of wider codes: 16 (c >> 4) at column gk of row gm, c & 15 at N + gk
   uint8_t* img8_next;
+  int img8_split;
   // dW with the constants in the parameter space: the parts of the
   // stochastic-rounding generator that are the same for every element of
   // the call, for uc and uc1
@@ -146,6 +148,10 @@ __device__ __forceinline__ void store_code_image4(__nv_bfloat16* img, size_t e, 
 // The E4M3 image of four codes (exact for |code| <= 16).
 __device__ __forceinline__ void store_code_e4m3_4(uint8_t* img8, size_t e, int32_t a, int32_t b,
                                                   int32_t c, int32_t d);
+
+// The E4M3 image of four updated codes at element e = gm N + gk, direct or split.
+__device__ __forceinline__ void store_img8(const Params& p, size_t e, int gm, int32_t a, int32_t b,
+                                           int32_t c, int32_t d);
 
 // Row and column tile (256 x 256) of a 2-SM kernel's tile index.
 __device__ __forceinline__ int pair_tile_m(const Params& p, int tile) {
@@ -220,6 +226,18 @@ __device__ __forceinline__ void store_code_e4m3_4(uint8_t* img8, size_t e, int32
   const uint32_t hi = __nv_cvt_float2_to_fp8x2(make_float2(static_cast<float>(c), static_cast<float>(d)),
                                                __NV_SATFINITE, __NV_E4M3);
   __stcs(reinterpret_cast<uint32_t*>(img8 + e), (lo & 0xFFFFu) | ((hi & 0xFFFFu) << 16));
+}
+
+__device__ __forceinline__ void store_img8(const Params& p, size_t e, int gm, int32_t a, int32_t b,
+                                           int32_t c, int32_t d) {
+  if (!p.img8_split) {
+    store_code_e4m3_4(p.img8_next, e, a, b, c, d);
+    return;
+  }
+  // split row gm of 2N bytes: the high halves at gm 2N + gk = e + gm N, the low N later
+  const size_t h = e + static_cast<size_t>(gm) * p.N;
+  store_code_e4m3_4(p.img8_next, h, 16 * (a >> 4), 16 * (b >> 4), 16 * (c >> 4), 16 * (d >> 4));
+  store_code_e4m3_4(p.img8_next, h + p.N, a & 15, b & 15, c & 15, d & 15);
 }
 
 __device__ __forceinline__ void store_code_image4(__nv_bfloat16* img, size_t e, int32_t a, int32_t b,
@@ -409,7 +427,7 @@ __device__ __forceinline__ uint32_t dw_update(const Params& p, const UpdateConst
              make_char4(static_cast<signed char>(n0c), static_cast<signed char>(n1c),
                         static_cast<signed char>(n2c), static_cast<signed char>(n3c)));
     if (p.img_next) store_code_image4(p.img_next, e, n0c, n1c, n2c, n3c);
-    if (p.img8_next) store_code_e4m3_4(p.img8_next, e, n0c, n1c, n2c, n3c);
+    if (p.img8_next) store_img8(p, e, gm, n0c, n1c, n2c, n3c);
     __stcs(reinterpret_cast<float4*>(p.m + e), L.m[j]);
     __stcs(reinterpret_cast<float4*>(p.v + e), L.v[j]);
   }
@@ -488,7 +506,7 @@ __device__ __forceinline__ uint32_t dw_update_row(const Params& p, const UpdateC
            make_char4(static_cast<signed char>(n0c), static_cast<signed char>(n1c),
                       static_cast<signed char>(n2c), static_cast<signed char>(n3c)));
   if (p.img_next) store_code_image4(p.img_next, e, n0c, n1c, n2c, n3c);
-  if (p.img8_next) store_code_e4m3_4(p.img8_next, e, n0c, n1c, n2c, n3c);
+  if (p.img8_next) store_img8(p, e, gm, n0c, n1c, n2c, n3c);
   __stcs(reinterpret_cast<float4*>(p.m + e), L.m);
   __stcs(reinterpret_cast<float4*>(p.v + e), L.v);
   return (n0c != c.x) + (n1c != c.y) + (n2c != c.z) + (n3c != c.w);
@@ -1591,6 +1609,7 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   p.pc1 = philox_call_consts(g.uc1);
   p.img_next = g.kind == GEMM_DW ? static_cast<__nv_bfloat16*>(g.img_next) : nullptr;
   p.img8_next = g.kind == GEMM_DW ? static_cast<uint8_t*>(g.img8_next) : nullptr;
+  p.img8_split = p.img8_next && g.img8_split ? 1 : 0;
   p.a_wrap = g.kind == GEMM_FWD8 ? g.a_wrap : 0;
   if ((p.img_next || p.img8_next) && (g.packed || !g.W)) return 1;
   // stacked weights: whole tiles (multiples of 256 of either tiling),
@@ -1658,7 +1677,7 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
                                   g.split > 0 ? &g.uc1 : nullptr, g.split,
                                   (g.N + 255) / 256 > (g.M + 255) / 256,
                                   static_cast<uint16_t*>(g.img_next),
-                                  static_cast<uint8_t*>(g.img8_next));
+                                  static_cast<uint8_t*>(g.img8_next), p.img8_split != 0);
       }
       // split-T: fp32 partials of each token slice into the workspace slabs,
       // then one streaming pass sums the slabs in slice order and applies the
@@ -1680,20 +1699,22 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
       // (the images of the updated codes are written by the same pass)
       uint16_t* img = static_cast<uint16_t*>(g.img_next);
       uint8_t* img8 = static_cast<uint8_t*>(g.img8_next);
+      const int64_t img8_k = p.img8_split ? g.N : 0;  // split image rows: 2 N bytes
       if (g.split > 0) {
         // stacked weights: the rows of each with its own constants
         const long long n0 = static_cast<long long>(g.split) * g.N;
         const float* sl = static_cast<const float*>(g.ws);
         return launch_sr_update_slabs(sl, p.splits, p.slab, g.W, g.m, g.v, n0, g.uc, nullptr,
-                                      g.changed, g.dW_out, stream, g.packed, img, img8) ||
+                                      g.changed, g.dW_out, stream, g.packed, img, img8, img8_k) ||
                launch_sr_update_slabs(sl + n0, p.splits, p.slab, g.W + n0, g.m + n0, g.v + n0,
                                       p.slab - n0, g.uc1, nullptr, g.changed,
                                       g.dW_out ? g.dW_out + n0 : nullptr, stream, g.packed,
-                                      img ? img + n0 : nullptr, img8 ? img8 + n0 : nullptr);
+                                      img ? img + n0 : nullptr,
+                                      img8 ? img8 + (img8_k ? 2 * n0 : n0) : nullptr, img8_k);
       }
       return launch_sr_update_slabs(static_cast<const float*>(g.ws), p.splits, p.slab, g.W, g.m,
                                     g.v, p.slab, g.uc, g.uc_dev, g.changed, g.dW_out, stream,
-                                    g.packed, img, img8);
+                                    g.packed, img, img8, img8_k);
     }
   }
   return 1;

@@ -39,36 +39,55 @@ __device__ __forceinline__ float slab_grad1(const float* __restrict__ grad, int 
   return g;
 }
 
+__device__ __forceinline__ uint32_t e4m3x4(int32_t a, int32_t b, int32_t c, int32_t d) {
+  const uint32_t lo = __nv_cvt_float2_to_fp8x2(
+      make_float2(static_cast<float>(a), static_cast<float>(b)), __NV_SATFINITE, __NV_E4M3);
+  const uint32_t hi = __nv_cvt_float2_to_fp8x2(
+      make_float2(static_cast<float>(c), static_cast<float>(d)), __NV_SATFINITE, __NV_E4M3);
+  return (lo & 0xFFFFu) | ((hi & 0xFFFFu) << 16);
+}
+
+// The E4M3 image of four new codes at element e: direct (img8_k == 0), or
+// split into rows of img8_k codes, each row 2 img8_k bytes with 16 (c >> 4)
+// at the code's column and c & 15 img8_k bytes later (e % 4 == 0 and img8_k
+// % 4 == 0, so the four codes share a row).
+__device__ __forceinline__ void store_e4m3_4(uint8_t* img8, int64_t img8_k, int64_t e, int32_t a,
+                                             int32_t b, int32_t c, int32_t d) {
+  if (!img8_k) {
+    __stcs(reinterpret_cast<uint32_t*>(img8 + e), e4m3x4(a, b, c, d));
+    return;
+  }
+  const int64_t h = e + (e / img8_k) * img8_k;
+  __stcs(reinterpret_cast<uint32_t*>(img8 + h),
+         e4m3x4(16 * (a >> 4), 16 * (b >> 4), 16 * (c >> 4), 16 * (d >> 4)));
+  __stcs(reinterpret_cast<uint32_t*>(img8 + h + img8_k), e4m3x4(a & 15, b & 15, c & 15, d & 15));
+}
+
 // The bf16 and E4M3 images of four new codes (either pointer may be NULL).
-__device__ __forceinline__ void store_images4(uint16_t* img, uint8_t* img8, int64_t e, int32_t a,
-                                              int32_t b, int32_t c, int32_t d) {
+__device__ __forceinline__ void store_images4(uint16_t* img, uint8_t* img8, int64_t img8_k,
+                                              int64_t e, int32_t a, int32_t b, int32_t c,
+                                              int32_t d) {
   if (img) {
     const __nv_bfloat162 lo = __floats2bfloat162_rn(static_cast<float>(a), static_cast<float>(b));
     const __nv_bfloat162 hi = __floats2bfloat162_rn(static_cast<float>(c), static_cast<float>(d));
     __stcs(reinterpret_cast<uint2*>(img + e),
            make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi)));
   }
-  if (img8) {
-    const uint32_t lo = __nv_cvt_float2_to_fp8x2(
-        make_float2(static_cast<float>(a), static_cast<float>(b)), __NV_SATFINITE, __NV_E4M3);
-    const uint32_t hi = __nv_cvt_float2_to_fp8x2(
-        make_float2(static_cast<float>(c), static_cast<float>(d)), __NV_SATFINITE, __NV_E4M3);
-    __stcs(reinterpret_cast<uint32_t*>(img8 + e), (lo & 0xFFFFu) | ((hi & 0xFFFFu) << 16));
-  }
+  if (img8) store_e4m3_4(img8, img8_k, e, a, b, c, d);
 }
 
 // DEV: the constants are read from device memory (else the kernel's
 // parameter space); SLABS: the gradient may be split into slabs and the
 // summed gradient written out, and the images of the new codes (img bf16,
-// img8 E4M3, int8 codes only) written beside them.  The plain instance is the
-// leanest stream.
+// img8 E4M3, direct or split as in store_e4m3_4; int8 codes only) written
+// beside them.  The plain instance is the leanest stream.
 template <bool packed, bool DEV, bool SLABS>
 __global__ void __launch_bounds__(kThreads)
     sr_update_kernel(const float* __restrict__ grad, int nsplit, long long slab,
                      float* __restrict__ g_out, int8_t* __restrict__ W, float* __restrict__ m,
                      float* __restrict__ v, int64_t numel, const UpdateConsts uc_arg,
                      const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed,
-                     uint16_t* __restrict__ img, uint8_t* __restrict__ img8) {
+                     uint16_t* __restrict__ img, uint8_t* __restrict__ img8, int64_t img8_k) {
   uint8_t* Wp = reinterpret_cast<uint8_t*>(W);
   const UpdateConsts uc = DEV ? *uc_dev : uc_arg;
   const int64_t ngroups = numel >> 2;
@@ -98,7 +117,7 @@ __global__ void __launch_bounds__(kThreads)
       *reinterpret_cast<char4*>(W + e) =
           make_char4(static_cast<signed char>(a), static_cast<signed char>(b),
                      static_cast<signed char>(c), static_cast<signed char>(d));
-    if (SLABS && !packed) store_images4(img, img8, e, a, b, c, d);
+    if (SLABS && !packed) store_images4(img, img8, img8_k, e, a, b, c, d);
     __stcs(reinterpret_cast<float4*>(m + e), m4);
     __stcs(reinterpret_cast<float4*>(v + e), v4);
   }
@@ -123,9 +142,10 @@ __global__ void __launch_bounds__(kThreads)
       if (packed) pr[j] = r;
       else W[e] = static_cast<int8_t>(r);
       if (SLABS && !packed && img) img[e] = __bfloat16_as_ushort(__float2bfloat16_rn(static_cast<float>(r)));
-      if (SLABS && !packed && img8)
+      if (SLABS && !packed && img8) {  // (a split image has no ragged tail: numel % 4 == 0)
         img8[e] = static_cast<uint8_t>(
             __nv_cvt_float_to_fp8(static_cast<float>(r), __NV_SATFINITE, __NV_E4M3));
+      }
       m[e] = mm;
       v[e] = vv;
     }
@@ -202,7 +222,7 @@ __global__ void __launch_bounds__(kThreads, 3)
                        const UpdateConsts* __restrict__ uc_dev, unsigned long long* changed,
                        float* __restrict__ dW_out, const UpdateConsts uc1, int split,
                        bool col_major, uint16_t* __restrict__ img_next,
-                       uint8_t* __restrict__ img8_next) {
+                       uint8_t* __restrict__ img8_next, bool img8_split) {
   const UpdateConsts uc = DEV ? *uc_dev : uc_arg;
   uint8_t* Wp = reinterpret_cast<uint8_t*>(W);
   const int64_t ngroups = static_cast<int64_t>(tail) * 16384;  // 256 x 256 / 4 per tile
@@ -273,13 +293,9 @@ __global__ void __launch_bounds__(kThreads, 3)
                  make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
                             *reinterpret_cast<const uint32_t*>(&hi)));
         }
-        if (img8_next) {  // the E4M3 image of the new codes (exact for |code| <= 16)
-          const uint32_t lo = __nv_cvt_float2_to_fp8x2(
-              make_float2(static_cast<float>(a), static_cast<float>(b)), __NV_SATFINITE, __NV_E4M3);
-          const uint32_t hi = __nv_cvt_float2_to_fp8x2(
-              make_float2(static_cast<float>(c), static_cast<float>(d)), __NV_SATFINITE, __NV_E4M3);
-          __stcs(reinterpret_cast<uint32_t*>(img8_next + e), (lo & 0xFFFFu) | ((hi & 0xFFFFu) << 16));
-        }
+        // the E4M3 image of the new codes (exact for |code| <= 16), or their
+        // split image (rows of N codes)
+        if (img8_next) store_e4m3_4(img8_next, img8_split ? N : 0, e, a, b, c, d);
         __stcs(reinterpret_cast<float4*>(m + e), m4);
         __stcs(reinterpret_cast<float4*>(v + e), v4);
       }
@@ -320,29 +336,29 @@ template <bool packed, bool DEV, bool SLABS>
 void sr_launch(const float* grad, int splits, long long slab, float* g_out, int8_t* W, float* m,
                float* v, int64_t numel, const UpdateConsts& uc, const UpdateConsts* uc_dev,
                unsigned long long* changed, cudaStream_t stream, uint16_t* img = nullptr,
-               uint8_t* img8 = nullptr) {
+               uint8_t* img8 = nullptr, int64_t img8_k = 0) {
   sr_update_kernel<packed, DEV, SLABS><<<stream_blocks(numel), kThreads, 0, stream>>>(
-      grad, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed, img, img8);
+      grad, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed, img, img8, img8_k);
 }
 
 template <bool packed>
 void sr_dispatch(const float* grad, int splits, long long slab, float* g_out, int8_t* W, float* m,
                  float* v, int64_t numel, const UpdateConsts& uc, const UpdateConsts* uc_dev,
                  unsigned long long* changed, cudaStream_t stream, uint16_t* img = nullptr,
-                 uint8_t* img8 = nullptr) {
+                 uint8_t* img8 = nullptr, int64_t img8_k = 0) {
   // the image outputs are those of the slab instance
   const bool slabs = splits > 1 || g_out || img || img8;
   if (uc_dev) {
     if (slabs)
       sr_launch<packed, true, true>(grad, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed,
-                                    stream, img, img8);
+                                    stream, img, img8, img8_k);
     else
       sr_launch<packed, true, false>(grad, 1, 0, nullptr, W, m, v, numel, uc, uc_dev, changed,
                                      stream);
   } else {
     if (slabs)
       sr_launch<packed, false, true>(grad, splits, slab, g_out, W, m, v, numel, uc, nullptr,
-                                     changed, stream, img, img8);
+                                     changed, stream, img, img8, img8_k);
     else
       sr_launch<packed, false, false>(grad, 1, 0, nullptr, W, m, v, numel, uc, nullptr, changed,
                                       stream);
@@ -354,12 +370,13 @@ void sr_dispatch(const float* grad, int splits, long long slab, float* g_out, in
 int launch_sr_update_slabs(const float* slabs, int splits, long long slab, int8_t* W, float* m,
                            float* v, int64_t numel, const UpdateConsts& uc,
                            const UpdateConsts* uc_dev, unsigned long long* changed, float* g_out,
-                           cudaStream_t stream, bool packed, uint16_t* img, uint8_t* img8) {
+                           cudaStream_t stream, bool packed, uint16_t* img, uint8_t* img8,
+                           int64_t img8_k) {
   if (packed)
     sr_dispatch<true>(slabs, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed, stream);
   else
     sr_dispatch<false>(slabs, splits, slab, g_out, W, m, v, numel, uc, uc_dev, changed, stream,
-                       img, img8);
+                       img, img8, img8_k);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
@@ -367,7 +384,7 @@ int launch_tail_update(const float* part, int splits, int tail, int full, int nu
                        int8_t* W, bool packed, float* m, float* v, const UpdateConsts& uc,
                        const UpdateConsts* uc_dev, unsigned long long* changed, float* dW_out,
                        cudaStream_t stream, const UpdateConsts* uc1, int split, bool col_major,
-                       uint16_t* img_next, uint8_t* img8_next) {
+                       uint16_t* img_next, uint8_t* img8_next, bool img8_split) {
   const UpdateConsts u1 = uc1 ? *uc1 : uc;
   // the blocks that fit at once: each thread walks several groups, its next
   // group's loads in flight
@@ -389,13 +406,14 @@ int launch_tail_update(const float* part, int splits, int tail, int full, int nu
     tail_update_kernel<true><<<blocks, kThreads, 0, stream>>>(part, splits, tail, full, num_n, M, N,
                                                               W, packed, m, v, uc, uc_dev, changed,
                                                               dW_out, u1, uc1 ? split : 0,
-                                                              col_major, img_next, img8_next);
+                                                              col_major, img_next, img8_next,
+                                                              img8_split);
   else
     tail_update_kernel<false><<<blocks, kThreads, 0, stream>>>(part, splits, tail, full, num_n, M,
                                                                N, W, packed, m, v, uc, nullptr,
                                                                changed, dW_out, u1,
                                                                uc1 ? split : 0, col_major,
-                                                               img_next, img8_next);
+                                                               img_next, img8_next, img8_split);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 

@@ -549,9 +549,9 @@ def dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, s_w, m, v, hp, sr, bits_or_grid,
     W, m, v updated in place.  With W = m = v = None only dW_out is computed.
     `ws`: split-T workspace (uint8 CUDA tensor of dqt_bwd_dw_img_workspace_size
     bytes); None allocates it when the shape benefits, False forces the single
-    fused kernel.  W_img_next (bf16 [N, K]) and W8_next (uint8 [N, K], E4M3):
-    receive the images of the updated codes (not images this step still
-    reads)."""
+    fused kernel.  W_img_next (bf16 [N, K]) and W8_next (uint8, E4M3: [N, K],
+    or the split image [N, 2K] for grids beyond 16 in magnitude) receive the
+    images of the updated codes (not images this step still reads)."""
     _need(dY, "dY", torch.bfloat16)
     T, N = dY.shape
     _need(Xdq, "Xdq", torch.bfloat16)
@@ -562,7 +562,7 @@ def dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, s_w, m, v, hp, sr, bits_or_grid,
     _opt(v, "v", torch.float32, (N, K))
     _opt(dW_out, "dW_out", torch.float32, (N, K))
     _opt(W_img_next, "W_img_next", torch.bfloat16, (N, K))
-    _opt(W8_next, "W8_next", torch.uint8, (N, K))
+    _opt(W8_next, "W8_next", torch.uint8, (N, 2 * K if fp8_split_grid(bits_or_grid) else K))
     _opt(changed_out, "changed_out", torch.int64, (1,))
     ws, nws = _dw_workspace(T, N, K, dY.device, ws)
     _check(lib().dqt_bitlinear_bwd_dw_update_img(
@@ -589,7 +589,7 @@ def dqt_bitlinear_bwd_dw_update_img_pair(dY, Xdq, W, N0, s_w0, s_w1, m, v, hp, s
     _need(v, "v", torch.float32, (N, K))
     _opt(dW_out, "dW_out", torch.float32, (N, K))
     _opt(W_img_next, "W_img_next", torch.bfloat16, (N, K))
-    _opt(W8_next, "W8_next", torch.uint8, (N, K))
+    _opt(W8_next, "W8_next", torch.uint8, (N, 2 * K if fp8_split_grid(bits_or_grid) else K))
     _opt(changed_out, "changed_out", torch.int64, (1,))
     ws, nws = _dw_workspace(T, N, K, dY.device, ws)
     _check(lib().dqt_bitlinear_bwd_dw_update_img_pair(

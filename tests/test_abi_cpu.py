@@ -114,10 +114,11 @@ def test_argument_validation_without_launch(L):
                                                   None, None, None, None, None, 0, None) == dqt.DQT_ERR_ARG
     assert L.dqt_bitlinear_bwd_dw_update_img_pair(A, A, None, 256, 1.0, 1.0, A, A, hp, sr, sr, g, 4, 512, 8,
                                                   None, None, None, None, None, 0, None) == dqt.DQT_ERR_ARG
-    # an E4M3 image of the updated codes only for grids within 16 in magnitude
+    # the E4M3 image of wider codes is the split image: rows of K codes, K a
+    # multiple of 16
     g8 = dqt.dqt_grid_t(-128, 127)
     assert L.dqt_bitlinear_bwd_dw_update_img_pair(A, A, A, 256, 1.0, 1.0, A, A, hp, sr, sr, g8, 4, 512, 8,
-                                                  None, None, A, None, None, 0, None) == dqt.DQT_ERR_RANGE
+                                                  None, None, A, None, None, 0, None) == dqt.DQT_ERR_ALIGN
     # the stacked FP8 forward: the same split rule, and the E4M3-exact grid
     assert L.dqt_bitlinear_fwd_fp8_pair(A, A, A, 200, 1.0, 1.0, g, 4, 16, 512, A, None, None) == dqt.DQT_ERR_ARG
     assert L.dqt_bitlinear_fwd_fp8_pair(A, A, A, 256, 1.0, 0.0, g, 4, 16, 512, A, None, None) == dqt.DQT_ERR_ARG
@@ -146,8 +147,8 @@ def test_update_argument_validation(L):
     # an image of the updated codes needs the update
     assert L.dqt_bitlinear_bwd_dw_update_img(A, A, None, 1.0, None, None, *ok, g, 4, 8, 8, A, A, None, None, None, 0, None) == dqt.DQT_ERR_ARG
     assert L.dqt_bitlinear_bwd_dw_update_img(A, A, None, 1.0, None, None, *ok, g, 4, 8, 8, A, None, A, None, None, 0, None) == dqt.DQT_ERR_ARG
-    # an E4M3 image only for grids within 16 in magnitude
-    assert L.dqt_bitlinear_bwd_dw_update_img(A, A, A, 1.0, A, A, *ok, dqt.dqt_grid_t(-128, 127), 4, 8, 8, None, None, A, None, None, 0, None) == dqt.DQT_ERR_RANGE
+    # the split E4M3 image of wider codes needs K a multiple of 16
+    assert L.dqt_bitlinear_bwd_dw_update_img(A, A, A, 1.0, A, A, *ok, dqt.dqt_grid_t(-128, 127), 4, 8, 8, None, None, A, None, None, 0, None) == dqt.DQT_ERR_ALIGN
     assert L.dqt_bitlinear_bwd_dw_update(A, A, A, None, 1.0, None, None, *ok, g, 4, 8, 16, None, None, A, 1 << 20, None) == dqt.DQT_ERR_ARG
     # the int8 call needs the X_tilde image in its workspace, 16-byte int8 rows
     assert L.dqt_bwd_dw_workspace_size(4, 8, 16) >= 4 * 16 * 2

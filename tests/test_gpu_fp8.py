@@ -243,3 +243,30 @@ def test_fwd_fp8_split_llama_mlp_sampled_rows_and_pair():
     q8, s8, _ = oracle.act_quant_fp8(bits(X[rows]))
     assert (g8.cpu().numpy()[rows] == q8).all()
     _check_fwd_split(q8, s8, c0, float(s0), bits(Y[:, :N0].contiguous())[rows], acc.cpu().numpy()[rows, :N0])
+
+
+def test_layer_keeps_split_image_across_steps():
+    """A DQTBitLinear on 8-bit codes with the E4M3 forward: its update writes
+    the split image of the new codes into the layer's cached operand, so the
+    next forward converts nothing and reads exactly the image of the new
+    codes (and gives the forward of a freshly converted image, bit for bit)."""
+    from paper_2412_04787_gb300.bitlinear import DQTBitLinear
+    T, K, N = 384, 256, 520
+    layer = DQTBitLinear(K, N, bits=8, lr=1e-2, seed=5, tensor_id=1, init_seed=9, act="fp8")
+    assert layer.w8_split
+    X = inputs.normal((T, K), 1.0, seed=12, dtype=torch.bfloat16).cuda()
+    dY = inputs.normal((T, N), 1e-2, seed=13, dtype=torch.bfloat16).cuda()
+    c0 = layer.codes.clone()
+    for _ in range(2):
+        layer(X.requires_grad_(True)).backward(dY)
+    torch.cuda.synchronize()
+    assert not torch.equal(layer.codes, c0)
+    assert layer._img8_version == layer.codes._version  # kept current by the update
+    img8 = layer.image_fp8()
+    assert torch.equal(img8, dqt.dqt_codes_to_fp8_split(layer.codes))
+    q8, s8, _ = dqt.dqt_act_quant_fp8(X.detach(), want_xdq=False)
+    y = layer(X.detach())
+    y_ref = dqt.dqt_bitlinear_fwd_fp8(q8, s8, dqt.dqt_codes_to_fp8_split(layer.codes),
+                                      float(layer.s_w), layer.grid_tuple)
+    dqt.dqt_check_device_status()
+    assert torch.equal(y.view(torch.int16), y_ref.view(torch.int16))

@@ -261,3 +261,52 @@ def test_dw_update_pair_writes_next_e4m3_image():
                                              g, W8_next=img8)
     dqt.dqt_check_device_status()
     assert torch.equal(img8, dqt.dqt_codes_to_fp8(W, g))
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("T,K,N,bits", [(4096, 2048, 5632, 8),   # token slices + tail kernel
+                                        (256, 512, 520, 6),      # one wave, ragged N
+                                        (4096, 512, 512, 8)])    # split-T path
+def test_dw_update_writes_next_split_e4m3_image(mode, T, K, N, bits):
+    """W8_next for codes wider than 16 in magnitude: the update writes the
+    split E4M3 image [N, 2K] of the codes it writes, byte for byte what
+    dqt_codes_to_fp8_split makes of them."""
+    dqt.dqt_set_gemm_tiles(mode)
+    try:
+        X = inputs.normal((T, K), 1.0, seed=T + N + 2, dtype=torch.bfloat16)
+        dY = inputs.normal((T, N), 1e-2, seed=T + 10, dtype=torch.bfloat16).cuda()
+        qmin, qmax = oracle.grid(bits)
+        c, s_w, _ = oracle.absmean_init(inputs.normal((N, K), 0.02, seed=N + 2).numpy(), qmin, qmax)
+        _, s_x, _, Xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xdq",))
+        W = torch.from_numpy(c).cuda()
+        m = torch.zeros((N, K), device="cuda")
+        v = torch.zeros((N, K), device="cuda")
+        img8 = torch.full((N, 2 * K), 0x7F, dtype=torch.uint8, device="cuda")
+        dqt.dqt_bitlinear_bwd_dw_update_img(dY, Xdq, W, float(s_w), m, v, dqt.adamw(lr=1e-2),
+                                            dqt.sr_stream(seed=6), (qmin, qmax), W8_next=img8)
+        dqt.dqt_check_device_status()
+        assert not torch.equal(W.cpu(), torch.from_numpy(c))
+        assert torch.equal(img8, dqt.dqt_codes_to_fp8_split(W))
+    finally:
+        dqt.dqt_set_gemm_tiles(0)
+
+
+@pytest.mark.parametrize("T,K,N0,N1", [(1024, 2048, 5632, 5632),  # token slices + tail kernel
+                                       (4096, 512, 256, 256)])    # split-T path, one slab pass each
+def test_dw_update_pair_writes_next_split_e4m3_image(T, K, N0, N1):
+    N = N0 + N1
+    X = inputs.normal((T, K), 1.0, seed=31, dtype=torch.bfloat16)
+    dY = inputs.normal((T, N), 1e-2, seed=32, dtype=torch.bfloat16).cuda()
+    c, s0, s1, g = _weights(N0, N1, K, 8, seed=33)
+    _, s_x, _, Xdq = dqt.dqt_act_quant_images(X.cuda(), want=("Xdq",))
+    W = torch.from_numpy(c).cuda()
+    m = torch.zeros((N, K), device="cuda")
+    v = torch.zeros((N, K), device="cuda")
+    img = torch.empty((N, K), dtype=torch.bfloat16, device="cuda")
+    img8 = torch.full((N, 2 * K), 0x7F, dtype=torch.uint8, device="cuda")
+    dqt.dqt_bitlinear_bwd_dw_update_img_pair(dY, Xdq, W, N0, s0, s1, m, v, dqt.adamw(lr=1e-2),
+                                             dqt.sr_stream(seed=4), dqt.sr_stream(seed=4, tensor_id=1),
+                                             g, W_img_next=img, W8_next=img8)
+    dqt.dqt_check_device_status()
+    assert torch.equal(img8, dqt.dqt_codes_to_fp8_split(W))
+    assert torch.equal(img.view(torch.int16), dqt.dqt_codes_to_bf16(W).view(torch.int16))
