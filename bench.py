@@ -89,7 +89,9 @@ DW_TRAFFIC_STACKED = {"e8a6edbac357": ((499344640 + 147830784)
                       "769ac7621d63": ((563601152 + 158165760)
                                          + (259388672 + 57002752 + 33059840 + 3328)) // 2,
                       "b62587c26333": ((563893248 + 158965760)
-                                         + (259276032 + 57066240 + 33059328 + 256)) // 2}
+                                         + (259276032 + 57066240 + 33059328 + 256)) // 2,
+                      "e40fd6702992": ((516993536 + 147382272)
+                                         + (259118848 + 57005568 + 33063680 + 768)) // 2}
 DW_TRAFFIC_BYTES = {"ac36c0aa63c5": 261135360 + 57050112 + 33049600,
                     "82d12725fdfa": 262571008 + 61169152 + 33047808,
                     "a25cf8632190": 261430272 + 59386112 + 33048064}
