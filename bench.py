@@ -996,7 +996,8 @@ def run_gpu(args):
             "roofline": roofline, "kernels": kern, "e2e": e2e,
             "gpu_launches": st.launches_per_step * args.steps,
             "clocks": clk.summary(), "cpu_baseline": cpu,
-            "changed_codes_last_step": [int(x) for x in res_host[(e_steps - 1) % 2].tolist()],
+            "changed_codes_last_step": changed_by_projection(
+                [int(x) for x in res_host[(e_steps - 1) % 2].tolist()], st.stack),
         }
         line.update(extra)
         print(json.dumps(line))
@@ -1150,6 +1151,14 @@ def stacked_gate_up(args, dp_mode="replicas"):
     exchange keeps one weight per exchange)."""
     return (not args.separate_gate_up and args.operands == "img"
             and not args.packed and args.optimizer == "adamw" and dp_mode != "exchange")
+
+
+def changed_by_projection(counts, stacked):
+    """Codes the last e2e step changed, per weight-gradient call: with gate and
+    up stacked their one call counts both (slot 1 is then unused)."""
+    if stacked:
+        return {"gate+up": counts[0], "down": counts[2]}
+    return dict(zip(("gate", "up", "down"), counts))
 
 
 def mlp_config(bits=1.58, fp8=False, optimizer="adamw", packed=False, i8=True, parallelism=None,

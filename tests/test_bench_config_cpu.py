@@ -26,3 +26,11 @@ def test_decoder_sizes():
     for sz, tflop in ((small, 8.35), (large, 111.0)):
         tokens = sz["batch"] * sz["seq"]
         assert abs(6.0 * tokens * _bitlinear_weights(sz) / 1e12 - tflop) / tflop < 0.01
+
+
+def test_changed_counts_are_labelled_by_call():
+    """The bench line's changed-code counts name the weight-gradient call they
+    come from: one count for gate and up when they are stacked."""
+    import bench
+    assert bench.changed_by_projection([5, 0, 7], True) == {"gate+up": 5, "down": 7}
+    assert bench.changed_by_projection([5, 6, 7], False) == {"gate": 5, "up": 6, "down": 7}
