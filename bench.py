@@ -92,6 +92,8 @@ DW_TRAFFIC_STACKED = {"e8a6edbac357": ((499344640 + 147830784)
                                          + (259276032 + 57066240 + 33059328 + 256)) // 2,
                       "e40fd6702992": ((516993536 + 147382272)
                                          + (259118848 + 57005568 + 33063680 + 768)) // 2}
+# DRAM bytes (read + write, ncu) of the grouped launch of both dW problems
+DW_TRAFFIC_GROUP = {"7eaccd5d9509": 873590272 + 328523520}
 DW_TRAFFIC_BYTES = {"ac36c0aa63c5": 261135360 + 57050112 + 33049600,
                     "82d12725fdfa": 262571008 + 61169152 + 33047808,
                     "a25cf8632190": 261430272 + 59386112 + 33048064}
@@ -167,7 +169,8 @@ class MLPStep:
     """Device buffers and the launch sequence of one DQT MLP training step."""
 
     def __init__(self, dev, seed=1234, fp8=False, optimizer="adamw", packed=False, bits=1.58,
-                 operands="int8", tail_slices=True, stack_gate_up=False, next_image=True):
+                 operands="int8", tail_slices=True, stack_gate_up=False, next_image=True,
+                 dw_group=False):
         from paper_2412_04787_gb300 import dqt, inputs
 
         self.dqt = dqt
@@ -185,6 +188,9 @@ class MLPStep:
         # fused dW + update; dX stays per weight): image operands, AdamW, int8
         # codes
         self.stack = stack_gate_up and not self.i8 and not packed and optimizer == "adamw"
+        # the step's two weight-gradient problems (gate and up stacked, and
+        # down) in one persistent launch (dqt_bitlinear_bwd_dw_update_group)
+        self.group = dw_group and self.stack
         self.grid = dqt.grid(bits)
         # FP8 forward on codes beyond 16 in magnitude: the split E4M3 image
         # [N, 2K] (dqt_codes_to_fp8_split's layout, written by the update like
@@ -336,8 +342,8 @@ class MLPStep:
             # one weight image (two with FP8), one forward and one dW call for
             # gate and up
             nbp = dqt.dqt_bwd_dw_img_workspace_size(T, 2 * INTER, HID)
-            self.launches_per_step = (2 + self.conversions() + 2 + 3 + (1 + (1 if nbp > 0 else 0))
-                                      + dw[2])
+            self.launches_per_step = (2 + self.conversions() + 2 + 3 +
+                                      (1 if self.group else (1 + (1 if nbp > 0 else 0)) + dw[2]))
             if nbp > max(nbw, 16):
                 self.dw_ws = [torch.empty(nbp, dtype=torch.uint8, device=dev) for _ in range(4)]
             nbt = max(nbt, dqt.dqt_fwd_img_workspace_size(T, HID, 2 * INTER))
@@ -381,6 +387,7 @@ class MLPStep:
         if self.nimg:  # the shard update writes codes only: images by conversion again
             self.launches_per_step += self.conversions()
             self.nimg = False
+        self.group = False
         self.dp = {}
         for name, _, _ in PROJ:
             upd = dp.DataParallelUpdater(self.W[name])
@@ -522,6 +529,20 @@ class MLPStep:
                 self.d["dY_" + name], self.W_img[name], self.s_w[name], dX=self.dX[name],
                 ws=self.tail_ws[s.index(stream)]))
 
+        def dw_group(stream):
+            nimg = self.nimg
+            timed(self.dw_kind, stream, lambda: dqt.dqt_bitlinear_bwd_dw_update_group([
+                dict(dY=self.d["dY_gu"], Xdq=self.aq["X"][2], W=self.W_gu, m=self.m_gu, v=self.v_gu,
+                     N0=INTER, s_w0=self.s_w["gate"], s_w1=self.s_w["up"], sr0=self.sr["gate"],
+                     sr1=self.sr["up"], W_img_next=self.W_img_gu_next if nimg else None,
+                     W8_next=self.W8_gu_next if nimg and self.fp8 else None,
+                     changed_out=self.changed[0:1]),
+                dict(dY=self.d["dY_down"], Xdq=self.aq["H"][2], W=self.W["down"], m=self.m["down"],
+                     v=self.v["down"], s_w0=self.s_w["down"], sr0=self.sr["down"],
+                     W_img_next=self.W_img_next["down"] if nimg else None,
+                     W8_next=self.W8_next["down"] if nimg and self.fp8 else None,
+                     changed_out=self.changed[2:3])], hp, self.grid))
+
         def dw(i, name, stream):
             xdq = self.aq["H" if name == "down" else "X"][2]
             ch = self.changed[i:i + 1]
@@ -630,7 +651,8 @@ class MLPStep:
         # backward: down projection (dX and dW independent)
         after(s[3], s[2])
         dx("down", s[2])
-        dw(2, "down", s[3])
+        if not self.group:  # (grouped: with the gate and up update below)
+            dw(2, "down", s[3])
         # backward: gate and up, after the down projection's dX
         dx_down = torch.cuda.Event()
         dx_down.record(s[2])
@@ -639,7 +661,11 @@ class MLPStep:
                 st.wait_event(dx_down)
         # each weight-gradient GEMM is enqueued ahead of its dX: the longer
         # kernel then takes the SMs first and the dX kernels fill its last wave
-        if self.stack:
+        if self.group:
+            dw_group(s[1])
+            dx("gate", s[0])
+            dx("up", s[2])
+        elif self.stack:
             dw(0, "gate_up", s[1])
             dx("gate", s[0])
             dx("up", s[2])
@@ -668,6 +694,8 @@ class MLPStep:
         if self.stack:  # gate and up in one forward and one dW call
             flops["fwd"] = [2.0 * T * HID * 2 * INTER, 2.0 * T * INTER * HID]
             flops["bwd_dw_update"] = list(flops["fwd"])
+        if self.group:  # and both dW problems in one launch
+            flops["bwd_dw_update"] = [sum(flops["fwd"])]
         flops["bwd_dw_adafactor"] = list(flops["fwd"])
         flops["bwd_dw"] = list(flops["fwd"])  # gradient only (data-parallel exchange)
         flops["fwd_fp8"] = list(flops["fwd"])
@@ -783,7 +811,7 @@ def run_gpu(args):
     st = MLPStep(dev, fp8=args.act == "fp8", optimizer=args.optimizer, packed=args.packed,
                  bits=args.bits, operands=args.operands, tail_slices=not args.no_tail_slices,
                  stack_gate_up=stacked_gate_up(args, dp_mode),
-                 next_image=not args.convert_images)
+                 next_image=not args.convert_images, dw_group=args.dw_group == "on")
     if dp_mode == "exchange":
         st.enable_dp()
     dqt = st.dqt
@@ -864,11 +892,15 @@ def run_gpu(args):
                               % (which, pk_kind, serial_ms_total)),
                 "timing": "mean CUDA-event duration of its launches over a second timed region "
                           "of the same K steps run serially on one stream (%.4f ms/step)" % serial_ms_step,
-                "traffic": ((DW_TRAFFIC_STACKED if st.stack else DW_TRAFFIC_BYTES)
+                "traffic": ((DW_TRAFFIC_GROUP if st.group else
+                             DW_TRAFFIC_STACKED if st.stack else DW_TRAFFIC_BYTES)
                             .get(kernel_fingerprint())
                             if dom == "bwd_dw_update" and not st.packed else None),
                 "kernel_fingerprint": kernel_fingerprint(),
-                "algorithmic_per_launch": ("2*T*K*N FLOP (T=8192; gate and up stacked: K,N = "
+                "algorithmic_per_launch": ("sum of 2*T*K*N FLOP over both problems of the one "
+                                           "grouped launch (T=8192; gate and up stacked: K,N = "
+                                           "2048,11264; down: 5632,2048)" if st.group else
+                                           "2*T*K*N FLOP (T=8192; gate and up stacked: K,N = "
                                            "2048,11264; down: 5632,2048)" if st.stack else
                                            "2*T*K*N FLOP (T=8192; K,N = 2048,5632 / 5632,2048)")}
     kern = {}
@@ -1733,6 +1765,9 @@ def main():
                          "operands and AdamW on int8 codes, they are two stacked weights of one "
                          "forward call and one dW + update call, each weight with its own scale "
                          "and SR stream; dX per weight)")
+    ap.add_argument("--dw-group", choices=("on", "off"), default="on",
+                    help="MLP step with gate and up stacked: both weight-gradient problems in one "
+                         "persistent launch (on) or in two calls (off)")
     ap.add_argument("--convert-images", action="store_true",
                     help="mlp, image operands: convert the codes to bf16 images at the start of "
                          "every step instead of taking the images the last step's updates wrote")

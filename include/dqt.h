@@ -356,6 +356,39 @@ int dqt_bitlinear_bwd_dw_update_img_pair(const dqt_bf16* dY, const dqt_bf16* Xdq
                                          unsigned long long* changed_out, void* ws,
                                          size_t ws_bytes, void* stream);
 
+/* One weight-gradient + update problem of a grouped call: dY bf16 [T, N],
+ * Xdq bf16 [T, K]; W int8, m, v fp32 [N, K] updated in place; N0 = 0 for one
+ * weight (s_w0, sr0), or the split of two stacked weights as for
+ * dqt_bitlinear_bwd_dw_update_img_pair (rows [0, N0) with s_w0 and sr0, the
+ * rest with s_w1 and sr1); W_img_next, W8_next and changed_out as for
+ * dqt_bitlinear_bwd_dw_update_img (NULL for none). */
+typedef struct {
+  const dqt_bf16* dY;
+  const dqt_bf16* Xdq;
+  int8_t* W;
+  float* m;
+  float* v;
+  int64_t N, K, N0;
+  float s_w0, s_w1;
+  const dqt_sr_t* sr0;
+  const dqt_sr_t* sr1;
+  dqt_bf16* W_img_next;
+  uint8_t* W8_next;
+  unsigned long long* changed_out;
+} dqt_dw_problem_t;
+
+/* Two weight-gradient + update problems over the same T tokens (a LLaMA
+ * MLP's stacked gate and up, and its down projection) in one persistent
+ * launch (Eq. 5 per weight, as dqt_bitlinear_bwd_dw_update_img): the 2-SM
+ * CTA pairs walk both problems' 256 x 256 tiles, so together they fill the
+ * waves (no token slices, no streaming tail).  Codes, moments, images and
+ * counts equal those of the two calls made with ws = NULL, bit for bit.
+ * nprob must be 2; hp and grid are the problems' common AdamW constants and
+ * grid.  Checks and status codes as for the single calls. */
+int dqt_bitlinear_bwd_dw_update_group(const dqt_dw_problem_t* probs, int nprob,
+                                      const dqt_adamw_t* hp, dqt_grid_t grid, int64_t T,
+                                      void* stream);
+
 /* The AdamW + SR update of dqt_bitlinear_bwd_dw_update for a gradient already
  * in memory (Eq. 5 as a bandwidth-bound stream; 22 bytes per weight):
  *   grad fp32 [numel];  W int8 [numel] in place;  m, v fp32 [numel] in place.

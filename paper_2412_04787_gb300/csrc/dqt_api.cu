@@ -691,6 +691,53 @@ int dqt_bitlinear_bwd_dw_update_img_pair(const dqt_bf16* dY, const dqt_bf16* Xdq
   return dqt::launch_gemm(g, as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
 }
 
+// One problem of a grouped call into a launch record (the checks of the
+// single and stacked calls).
+static int dw_problem(const dqt_dw_problem_t& q, const dqt_adamw_t* hp, dqt_grid_t grid,
+                      int64_t T, dqt::GemmLaunch& g) {
+  const int64_t N = q.N, K = q.K;
+  if (!q.dY || !q.Xdq || !q.W || !q.m || !q.v || !q.sr0 || T <= 0 || N <= 0 || K <= 0)
+    return DQT_ERR_ARG;
+  if (q.N0 != 0 && (!pair_split_ok(q.N0, N) || !q.sr1)) return DQT_ERR_ARG;
+  const bool w8_split = q.W8_next && fp8_split(grid);
+  if (T > kMaxDim || K > kMaxDim || N > kMaxDim || N * K > (int64_t(1) << 62)) return DQT_ERR_RANGE;
+  if (K % 8 || N % 8 || (w8_split && K % 16) || !aligned16(q.dY) || !aligned16(q.Xdq) ||
+      !aligned16(q.W) || !aligned16(q.m) || !aligned16(q.v) ||
+      (q.W_img_next && !aligned16(q.W_img_next)) || (q.W8_next && !aligned16(q.W8_next)))
+    return DQT_ERR_ALIGN;
+  g = dqt::GemmLaunch{};
+  int rc = make_update_consts(hp, q.sr0, grid, q.s_w0, &g.uc);
+  if (rc == DQT_OK && q.N0 != 0) rc = make_update_consts(hp, q.sr1, grid, q.s_w1, &g.uc1);
+  if (rc != DQT_OK) return rc;
+  g.split = static_cast<int>(q.N0);
+  g.kind = dqt::GEMM_DW;
+  g.M = static_cast<int>(N);
+  g.N = static_cast<int>(K);
+  g.Kred = static_cast<int>(T);
+  g.A = q.dY;
+  g.B = q.Xdq;
+  g.W = q.W;
+  g.m = q.m;
+  g.v = q.v;
+  g.img_next = q.W_img_next;
+  g.img8_next = q.W8_next;
+  g.img8_split = w8_split;
+  g.changed = q.changed_out;
+  return DQT_OK;
+}
+
+int dqt_bitlinear_bwd_dw_update_group(const dqt_dw_problem_t* probs, int nprob,
+                                      const dqt_adamw_t* hp, dqt_grid_t grid, int64_t T,
+                                      void* stream) {
+  if (!probs || nprob != 2) return DQT_ERR_ARG;
+  dqt::GemmLaunch g[2];
+  for (int i = 0; i < 2; ++i) {
+    const int rc = dw_problem(probs[i], hp, grid, T, g[i]);
+    if (rc != DQT_OK) return rc;
+  }
+  return dqt::launch_dw_group(g[0], g[1], as_stream(stream)) ? DQT_ERR_CUDA : DQT_OK;
+}
+
 int dqt_sr_update(const float* grad, int8_t* W, float s_w, float* m, float* v,
                   const dqt_adamw_t* hp, const dqt_sr_t* sr, dqt_grid_t grid, int64_t numel,
                   unsigned long long* changed_out, void* stream) {

@@ -124,6 +124,12 @@ int launch_slab_sum(const float* slabs, int splits, long long slab, float* out,
                     cudaStream_t stream);
 
 int launch_gemm(const GemmLaunch& g, cudaStream_t stream);
+// Two 2-SM dW + update launches (kind GEMM_DW, int8 codes with W, m, v,
+// constants by value, the same reduction length Kred) as one persistent
+// launch over both problems' whole tiles; dW_out, stacked weights (split)
+// and the next-step images as for launch_gemm.  Nonzero on an unsupported
+// launch record (1) or a CUDA error (3).
+int launch_dw_group(const GemmLaunch& g0, const GemmLaunch& g1, cudaStream_t stream);
 
 int launch_act_quant(const uint16_t* X, int64_t T, int64_t K, int8_t* Xq, float* s_x,
                      uint16_t* Xq_img, uint16_t* Xdq, cudaStream_t stream);

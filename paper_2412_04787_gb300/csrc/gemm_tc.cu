@@ -886,12 +886,16 @@ struct SmemPair {
 // UCD: the dW update constants come from device memory (p.uc_dev, copied to
 // shared memory once); otherwise the epilogue reads them straight from the
 // kernel's parameter space, where they take no registers.
-template <bool A_MN, bool B_MN, int EPI, bool PK = false, bool DR = false, bool UCD = false>
-__global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
-    gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA,
-                     const __grid_constant__ CUtensorMap tmB, const __grid_constant__ Params p) {
+// GRP: one launch for two dW problems over the same reduction length: p's
+// units, then p2's (tensor maps tmA2, tmB2), each with its own shape,
+// optimiser state, images, constants and tile order; whole tiles only.
+template <bool A_MN, bool B_MN, int EPI, bool PK, bool DR, bool UCD, bool GRP>
+__device__ __forceinline__ void gemm_pair_body(const CUtensorMap& tmA, const CUtensorMap& tmB,
+                                               const Params& p, const CUtensorMap& tmA2,
+                                               const CUtensorMap& tmB2, const Params& p2) {
   using S = SmemPair<EPI, DR>;
   static_assert(!DR || EPI == GEMM_FWD, "drained chunks: exact integer forward only");
+  static_assert(!GRP || (EPI == GEMM_DW && !DR && !UCD), "grouped launches: dW, constants by value");
   constexpr int ST = S::STAGES;
   constexpr int EW = S::EW;
   constexpr int BN = 256;           // pair tile width; each CTA holds all 256 columns of its rows
@@ -943,6 +947,10 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
     fence_mbarrier_init();
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
+    if (GRP) {
+      tma_prefetch_desc(&tmA2);
+      tma_prefetch_desc(&tmB2);
+    }
   }
   if (warp == 1) tmem_alloc_pair(tmem_slot, TMEM_COLS);
   tc_fence_before();
@@ -961,58 +969,63 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
       bool ok = true;
       const uint64_t pol_b = EPI == GEMM_DW ? l2_policy_evict_last() : 0ull;
       const uint64_t pol_f = EPI == GEMM_DW ? l2_policy_evict_first() : 0ull;
-      for (int t = cid; t < p.num_tiles && ok; t += ncl) {
-        const Unit un = decode_unit(p, t);
+      // one unit of problem q (tensor maps A, B), its unit index tl; false:
+      // a wait ran out
+      auto produce = [&](const CUtensorMap& A, const CUtensorMap& B, const Params& q,
+                         int tl) -> bool {
+        const Unit un = decode_unit(q, tl);
         const int tile = un.tile, kb0 = un.kb0, kb1 = un.kb1;
-        const int m0 = pair_tile_m(p, tile) * 256 + static_cast<int>(rank) * 128;
-        const int n0 = pair_tile_n(p, tile) * BN + static_cast<int>(rank) * 128;
+        const int m0 = pair_tile_m(q, tile) * 256 + static_cast<int>(rank) * 128;
+        const int n0 = pair_tile_n(q, tile) * BN + static_cast<int>(rank) * 128;
         for (int kb = kb0; kb < kb1; ++kb, ++it) {
-          if (it >= ST && !mbar_wait_cl(&empty[s], ph ^ 1u, p.wait_ns)) {
-            ok = false;
-            break;
-          }
+          if (it >= ST && !mbar_wait_cl(&empty[s], ph ^ 1u, q.wait_ns)) return false;
           if (leader) mbar_arrive_expect_tx(&full[s], 2 * S::STAGE_BYTES);
           const uint32_t bar = full_lead + 8u * s;
           uint8_t* a = sA + s * S::A_BYTES;
           uint8_t* b = sB + s * S::B_BYTES;
           const int k0 = kb * KB;
           if (!A_MN) {
-            tma_load_2d_pair(&tmA, bar, a, F8 && p.a_wrap ? k0 % p.a_wrap : k0, m0);
-          } else if (EPI == GEMM_DW && p.col_major) {
+            tma_load_2d_pair(&A, bar, a, F8 && q.a_wrap ? k0 % q.a_wrap : k0, m0);
+          } else if (EPI == GEMM_DW && q.col_major) {
             // column-major tiles: dY's panels are re-read by every wave
 #pragma unroll
             for (int j = 0; j < 2; ++j)
-              tma_load_2d_pair_hint(&tmA, bar, a + j * MN_CHUNK_BYTES, m0 + 64 * j, k0, pol_b);
+              tma_load_2d_pair_hint(&A, bar, a + j * MN_CHUNK_BYTES, m0 + 64 * j, k0, pol_b);
           } else if (EPI == GEMM_DW) {
             // row-major tiles: each dY panel is read by the one wave of
             // clusters that shares it, then never again
 #pragma unroll
             for (int j = 0; j < 2; ++j)
-              tma_load_2d_pair_hint(&tmA, bar, a + j * MN_CHUNK_BYTES, m0 + 64 * j, k0, pol_f);
+              tma_load_2d_pair_hint(&A, bar, a + j * MN_CHUNK_BYTES, m0 + 64 * j, k0, pol_f);
           } else {
 #pragma unroll
             for (int j = 0; j < 2; ++j)
-              tma_load_2d_pair(&tmA, bar, a + j * MN_CHUNK_BYTES, m0 + 64 * j, k0);
+              tma_load_2d_pair(&A, bar, a + j * MN_CHUNK_BYTES, m0 + 64 * j, k0);
           }
           if (!B_MN) {
-            tma_load_2d_pair(&tmB, bar, b, k0, n0);
-          } else if (EPI == GEMM_DW && !p.col_major) {
+            tma_load_2d_pair(&B, bar, b, k0, n0);
+          } else if (EPI == GEMM_DW && !q.col_major) {
             // X~ (all K columns) is re-read by every wave of output-row tiles,
             // while each dY column block is read by one wave: keep X~ in L2
 #pragma unroll
             for (int j = 0; j < 2; ++j)
-              tma_load_2d_pair_hint(&tmB, bar, b + j * MN_CHUNK_BYTES, n0 + 64 * j, k0, pol_b);
+              tma_load_2d_pair_hint(&B, bar, b + j * MN_CHUNK_BYTES, n0 + 64 * j, k0, pol_b);
           } else {
 #pragma unroll
             for (int j = 0; j < 2; ++j)
-              tma_load_2d_pair(&tmB, bar, b + j * MN_CHUNK_BYTES, n0 + 64 * j, k0);
+              tma_load_2d_pair(&B, bar, b + j * MN_CHUNK_BYTES, n0 + 64 * j, k0);
           }
           if (++s == ST) {
             s = 0;
             ph ^= 1u;
           }
         }
-      }
+        return true;
+      };
+      const int total = GRP ? p.num_tiles + p2.num_tiles : p.num_tiles;
+      for (int t = cid; t < total && ok; t += ncl)
+        ok = (GRP && t >= p.num_tiles) ? produce(tmA2, tmB2, p2, t - p.num_tiles)
+                                       : produce(tmA, tmB, p, t);
       if (!ok) record_timeout(p.status);
       // The leader sees every stage's completion (both CTAs' copies land on
       // its barriers): let the last stages land before the pair exits.
@@ -1043,8 +1056,10 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
       constexpr uint32_t kAStage = S::A_BYTES >> 4, kBStage = S::B_BYTES >> 4;
       constexpr uint32_t kAStep = A_MN ? (2048 >> 4) : (32 >> 4);  // per 16-element k step
       constexpr uint32_t kBStep = B_MN ? (2048 >> 4) : (32 >> 4);
-      for (int t = cid; t < p.num_tiles && ok; t += ncl) {
-        const Unit un = decode_unit(p, t);
+      const int total = GRP ? p.num_tiles + p2.num_tiles : p.num_tiles;
+      for (int t = cid; t < total && ok; t += ncl) {
+        const Unit un =
+            (GRP && t >= p.num_tiles) ? decode_unit(p2, t - p.num_tiles) : decode_unit(p, t);
         const int kb0 = un.kb0, kb1 = un.kb1;
         int left = 0;  // DR: k-blocks left in the current chunk
         for (int kb = kb0; kb < kb1; ++kb) {
@@ -1099,34 +1114,36 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
     const int row = quad * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     float* xp = reinterpret_cast<float*>(smem + S::XPOSE_OFF) + (warp - 2) * 32 * kStageLd;
-    const UpdateConsts& uc = UCD ? *uc_s : p.uc;
-    uint32_t n_changed = 0;
+    uint32_t n_changed = 0, n_changed2 = 0;  // changed codes of p's and p2's units
     int u = 0;
     bool ok = true;
     DwRow st[4];            // dW: optimiser state of the half-chunk being updated
     bool st_loaded = false;  // st already holds this unit's first half-chunk
-    for (int t = cid; t < p.num_tiles && ok; t += ncl, ++u) {
-      const Unit un = decode_unit(p, t);
+    // one unit (tile or slice) of problem q, its unit index tl; false: a wait
+    // ran out
+    auto epi_unit = [&](const Params& q, int tl, uint32_t& n_changed) -> bool {
+      const UpdateConsts& uc = UCD ? *uc_s : q.uc;
+      const Unit un = decode_unit(q, tl);
       const int tile = un.tile;
-      float* dw_out = p.dW_out ? p.dW_out + un.slab * p.slab : nullptr;
-      const int gm = pair_tile_m(p, tile) * 256 + static_cast<int>(rank) * 128 + row;
-      const int nbase = pair_tile_n(p, tile) * BN + half * HALF;
-      const bool row_ok = gm < p.M;
+      float* dw_out = q.dW_out ? q.dW_out + un.slab * q.slab : nullptr;
+      const int gm = pair_tile_m(q, tile) * 256 + static_cast<int>(rank) * 128 + row;
+      const int nbase = pair_tile_n(q, tile) * BN + half * HALF;
+      const bool row_ok = gm < q.M;
       if (EPI == GEMM_DW && un.slice < 0 && !st_loaded)
-        dw_load_first<PK>(p, gm - lane, nbase, lane, st);  // in flight during the wait below
+        dw_load_first<PK>(q, gm - lane, nbase, lane, st);  // in flight during the wait below
       float a_t = 0.0f;
       if ((EPI == GEMM_FWD || F8) && row_ok) {
         // the second of two stacked weights (whole tiles of columns): its scale
-        const float sw = p.split > 0 && pair_tile_n(p, tile) * BN >= p.split ? p.scale1 : p.scale;
-        a_t = __fdiv_rn(1.0f, __fmul_rn(p.s_x[gm], sw));
+        const float sw = q.split > 0 && pair_tile_n(q, tile) * BN >= q.split ? q.scale1 : q.scale;
+        a_t = __fdiv_rn(1.0f, __fmul_rn(q.s_x[gm], sw));
       }
       if (DR) {
         static_assert(!DR || HALF == 64, "two 32-column chunks of running sums per lane");
-        const int nchunks = (p.num_kb + p.chunk_kb - 1) / p.chunk_kb;
+        const int nchunks = (q.num_kb + q.chunk_kb - 1) / q.chunk_kb;
         int32_t run0[32], run1[32];
         for (int c = 0; c < nchunks; ++c, ++u) {
           const int b = u & 1;
-          ok = __all_sync(0xffffffffu, mbar_wait_cl(&acc_full[b], (u >> 1) & 1u, p.wait_ns));
+          ok = __all_sync(0xffffffffu, mbar_wait_cl(&acc_full[b], (u >> 1) & 1u, q.wait_ns));
           if (!ok) break;
           tc_fence_after();
           const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(b * BN + half * HALF);
@@ -1146,17 +1163,17 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive_cluster(acc_empty_lead + 8u * b);
         }
-        if (!ok) break;
+        if (!ok) return false;
         if (row_ok) {
-          if (nbase < p.N) epi_fwd_int(p, gm, nbase, a_t, run0);
-          if (nbase + 32 < p.N) epi_fwd_int(p, gm, nbase + 32, a_t, run1);
+          if (nbase < q.N) epi_fwd_int(q, gm, nbase, a_t, run0);
+          if (nbase + 32 < q.N) epi_fwd_int(q, gm, nbase + 32, a_t, run1);
         }
         --u;  // the loop header counts one unit per tile
-        continue;
+        return true;
       }
       const int b = u & 1;
-      ok = __all_sync(0xffffffffu, mbar_wait_cl(&acc_full[b], (u >> 1) & 1u, p.wait_ns));
-      if (!ok) break;
+      ok = __all_sync(0xffffffffu, mbar_wait_cl(&acc_full[b], (u >> 1) & 1u, q.wait_ns));
+      if (!ok) return false;
       tc_fence_after();
       const uint32_t t_acc = tmem + lane_off + static_cast<uint32_t>(b * BN + half * HALF);
       if ((EPI == GEMM_DW || EPI == GEMM_FWD || EPI == GEMM_DX) && un.slice >= 0) {
@@ -1168,9 +1185,9 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
         // 1024 (8 (row / 32) + column / 32) floats), each stored as [column
         // quad][row][4]: a warp's store of one column quad of its 32 rows is
         // 512 contiguous bytes, and so is the fix-up's load below.
-        const int jt = tile - p.full_tiles;
+        const int jt = tile - q.full_tiles;
         const long long roff = (static_cast<long long>(rank) * 128 + row) * 256 + half * HALF;
-        const long long tile_off = (static_cast<long long>(un.slice) * p.tail_tiles + jt) * 65536LL;
+        const long long tile_off = (static_cast<long long>(un.slice) * q.tail_tiles + jt) * 65536LL;
         const int blk0 = ((static_cast<int>(rank) * 4 + quad) * 8 + half * (HALF / 32)) * 1024;
 #pragma unroll 1
         for (int cc = 0; cc < HALF / 32; ++cc) {
@@ -1178,8 +1195,8 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
           tmem_ld_32x32b_x32(t_acc + cc * 32, a);
           tmem_ld_wait();
           float4* dst = EPI == GEMM_DW
-                            ? reinterpret_cast<float4*>(p.part + tile_off + roff + cc * 32)
-                            : reinterpret_cast<float4*>(p.part + tile_off + blk0 + cc * 1024) + lane;
+                            ? reinterpret_cast<float4*>(q.part + tile_off + roff + cc * 32)
+                            : reinterpret_cast<float4*>(q.part + tile_off + blk0 + cc * 1024) + lane;
 #pragma unroll
           for (int j = 0; j < 8; ++j)
             __stcg(dst + (EPI == GEMM_DW ? j : 32 * j),
@@ -1197,10 +1214,10 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
           unsigned long long done = 0;
           if (lane == 0) {
             unsigned long long* ctr =
-                p.tail_ctr + (static_cast<long long>(jt) * 2 + rank) * EW + (warp - 2);
+                q.tail_ctr + (static_cast<long long>(jt) * 2 + rank) * EW + (warp - 2);
             unsigned long long assumed = 0ull, nv;
             while (true) {  // at most tail_splits + 1 tries: each failure sees another slice's count
-              nv = (assumed >> 16) == p.tail_tag ? assumed + 1ull : ((p.tail_tag << 16) | 1ull);
+              nv = (assumed >> 16) == q.tail_tag ? assumed + 1ull : ((q.tail_tag << 16) | 1ull);
               const unsigned long long prev = atomicCAS(ctr, assumed, nv);
               if (prev == assumed) break;
               assumed = prev;
@@ -1208,10 +1225,10 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
             done = nv & 0xFFFFull;
           }
           done = __shfl_sync(0xffffffffu, done, 0);
-          if (done == static_cast<unsigned long long>(p.tail_splits)) {
+          if (done == static_cast<unsigned long long>(q.tail_splits)) {
             __threadfence();
-            const float* src0 = p.part + static_cast<long long>(jt) * 65536LL + blk0;
-            const long long sstride = static_cast<long long>(p.tail_tiles) * 65536LL;
+            const float* src0 = q.part + static_cast<long long>(jt) * 65536LL + blk0;
+            const long long sstride = static_cast<long long>(q.tail_tiles) * 65536LL;
 #pragma unroll 1
             for (int cc = 0; cc < HALF / 32; ++cc) {
               const int gn0 = nbase + cc * 32;
@@ -1225,7 +1242,7 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
                 f[4 * j + 3] = v.w;
               }
 #pragma unroll 1
-              for (int sl = 1; sl < p.tail_splits; ++sl) {
+              for (int sl = 1; sl < q.tail_splits; ++sl) {
 #pragma unroll
                 for (int j = 0; j < 8; ++j) {
                   const float4 v = __ldcg(
@@ -1240,36 +1257,36 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
               // from L2 so that they are never written back
               __syncwarp();
 #pragma unroll 1
-              for (int sl = 0; sl < p.tail_splits; ++sl)
+              for (int sl = 0; sl < q.tail_splits; ++sl)
                 l2_discard_line(src0 + sl * sstride + cc * 1024 + lane * 32);
-              if (gn0 >= p.N || !row_ok) continue;
+              if (gn0 >= q.N || !row_ok) continue;
               uint32_t a[32];
 #pragma unroll
               for (int i = 0; i < 32; ++i) a[i] = __float_as_uint(f[i]);
-              if (EPI == GEMM_FWD) epi_fwd(p, gm, gn0, a_t, a, a, false);  // no running sums
-              else epi_dx(p, gm, gn0, a);
+              if (EPI == GEMM_FWD) epi_fwd(q, gm, gn0, a_t, a, a, false);  // no running sums
+              else epi_dx(q, gm, gn0, a);
             }
           }
-          continue;  // the accumulator is already released
+          return true;  // the accumulator is already released
         }
       } else if (EPI == GEMM_DW) {
         // the first half-chunk of this warp's next unit, if a whole tile,
         // is loaded during this tile's last half-chunk
         int row0n = -1, nbasen = 0;
-        if (t + ncl < p.num_tiles) {
-          const Unit nu = decode_unit(p, t + ncl);
+        if (tl + ncl < q.num_tiles) {
+          const Unit nu = decode_unit(q, tl + ncl);
           if (nu.slice < 0) {
-            row0n = pair_tile_m(p, nu.tile) * 256 + static_cast<int>(rank) * 128 + quad * 32;
-            nbasen = pair_tile_n(p, nu.tile) * BN + half * HALF;
+            row0n = pair_tile_m(q, nu.tile) * 256 + static_cast<int>(rank) * 128 + quad * 32;
+            nbasen = pair_tile_n(q, nu.tile) * BN + half * HALF;
           }
         }
         // the second of two stacked weights: its constants, its own element count
-        if (p.split > 0 && pair_tile_m(p, tile) * 256 >= p.split)
-          n_changed += epi_dw_tile_roll<PK, !UCD>(p, p.uc1, p.pc1, static_cast<size_t>(p.split) * p.N,
+        if (q.split > 0 && pair_tile_m(q, tile) * 256 >= q.split)
+          n_changed += epi_dw_tile_roll<PK, !UCD>(q, q.uc1, q.pc1, static_cast<size_t>(q.split) * q.N,
                                                   dw_out, gm - lane, nbase, HALF / 32, t_acc, xp,
                                                   lane, st, row0n, nbasen);
         else
-          n_changed += epi_dw_tile_roll<PK, !UCD>(p, uc, p.pc, 0, dw_out, gm - lane, nbase,
+          n_changed += epi_dw_tile_roll<PK, !UCD>(q, uc, q.pc, 0, dw_out, gm - lane, nbase,
                                                   HALF / 32, t_acc, xp, lane, st, row0n, nbasen);
         st_loaded = row0n >= 0;
       } else
@@ -1279,21 +1296,32 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
         tmem_ld_32x32b_x32(t_acc + cc * 32, a);
         tmem_ld_wait();
         const int gn0 = nbase + cc * 32;
-        if (gn0 >= p.N) continue;  // warp-uniform
+        if (gn0 >= q.N) continue;  // warp-uniform
         if (!row_ok) continue;
-        if (EPI == GEMM_FWD) epi_fwd(p, gm, gn0, a_t, a, r, false);
-        else if (F8) epi_fwd8(p, gm, gn0, a_t, a);
-        else epi_dx(p, gm, gn0, a);
+        if (EPI == GEMM_FWD) epi_fwd(q, gm, gn0, a_t, a, r, false);
+        else if (F8) epi_fwd8(q, gm, gn0, a_t, a);
+        else epi_dx(q, gm, gn0, a);
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(acc_empty_lead + 8u * b);
-    }
+      return true;
+    };
+    const int total = GRP ? p.num_tiles + p2.num_tiles : p.num_tiles;
+    for (int t = cid; t < total && ok; t += ncl, ++u)
+      ok = (GRP && t >= p.num_tiles) ? epi_unit(p2, t - p.num_tiles, n_changed2)
+                                     : epi_unit(p, t, n_changed);
     if (!ok && lane == 0) record_timeout(p.status);
     if (EPI == GEMM_DW && p.changed) {
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) n_changed += __shfl_xor_sync(0xffffffffu, n_changed, off);
       if (lane == 0 && n_changed) atomicAdd(p.changed, static_cast<unsigned long long>(n_changed));
+    }
+    if (GRP && p2.changed) {
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1)
+        n_changed2 += __shfl_xor_sync(0xffffffffu, n_changed2, off);
+      if (lane == 0 && n_changed2) atomicAdd(p2.changed, static_cast<unsigned long long>(n_changed2));
     }
   }
 
@@ -1304,6 +1332,24 @@ __global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
     tc_fence_after();
     tmem_dealloc_pair(tmem, TMEM_COLS);
   }
+}
+
+template <bool A_MN, bool B_MN, int EPI, bool PK = false, bool DR = false, bool UCD = false>
+__global__ void __launch_bounds__(PairCfg<EPI, DR>::THREADS, 1)
+    gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA,
+                     const __grid_constant__ CUtensorMap tmB, const __grid_constant__ Params p) {
+  gemm_pair_body<A_MN, B_MN, EPI, PK, DR, UCD, false>(tmA, tmB, p, tmA, tmB, p);
+}
+
+// Two dW + update problems in one persistent launch (both operands MN-major,
+// int8 codes, constants by value).
+__global__ void __launch_bounds__(PairCfg<GEMM_DW, false>::THREADS, 1)
+    gemm_dw_group_kernel(const __grid_constant__ CUtensorMap tmA,
+                         const __grid_constant__ CUtensorMap tmB, const __grid_constant__ Params p,
+                         const __grid_constant__ CUtensorMap tmA2,
+                         const __grid_constant__ CUtensorMap tmB2,
+                         const __grid_constant__ Params p2) {
+  gemm_pair_body<true, true, GEMM_DW, false, false, false, true>(tmA, tmB, p, tmA2, tmB2, p2);
 }
 
 // ---------------------------------------------------------------------------
@@ -1461,6 +1507,17 @@ namespace {
 // Launches that cut their last wave with slice counters (all GEMM kinds).
 std::atomic<unsigned long long> g_tail_launches{0};
 
+// 256 x 256 pair tiles of a 2-SM launch.  dW: the operand with fewer
+// 256-wide panels is the one re-read by every wave (and kept in L2): X_tilde
+// (along the rows) when the output has more row tiles, dY (down the columns)
+// when it has more column tiles.
+void pair_tiling(Params& p, bool dw) {
+  p.num_n = (p.N + 255) / 256;
+  p.num_m = (p.M + 255) / 256;
+  p.num_tiles = p.num_m * p.num_n * p.splits;
+  p.col_major = dw && p.num_n > p.num_m;
+}
+
 template <bool A_MN, bool B_MN, int EPI, bool PK, bool DR, bool UCD>
 int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStream_t stream,
                  void* tail_ws, size_t tail_ws_bytes, TailPlan* plan) {
@@ -1468,13 +1525,7 @@ int launch_pairs(const CUtensorMap& ta, const CUtensorMap& tb, Params p, cudaStr
   const int smem = SmemPair<EPI, DR>::BYTES;
   constexpr int threads = PairCfg<EPI, DR>::THREADS;
   static int max_clusters = 0;  // per template instance
-  p.num_n = (p.N + 255) / 256;
-  p.num_m = (p.M + 255) / 256;
-  p.num_tiles = p.num_m * p.num_n * p.splits;
-  // dW: the operand with fewer 256-wide panels is the one re-read by every
-  // wave (and kept in L2): X_tilde (along the rows) when the output has more
-  // row tiles, dY (down the columns) when it has more column tiles
-  p.col_major = EPI == GEMM_DW && p.num_n > p.num_m;
+  pair_tiling(p, EPI == GEMM_DW);
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -1557,6 +1608,38 @@ static PhiloxCall philox_call_consts(const UpdateConsts& uc) {
   return k;
 }
 
+// The arguments every GEMM kind takes from its launch record (the watchdog,
+// pointers, scales, update constants and images).
+static int fill_common(const GemmLaunch& g, Params& p) {
+  p.wait_ns = wait_limit_ns();
+  p.status = status_word();
+  if (!p.status) return 3;
+  p.s_x = g.s_x;
+  p.scale = g.scale;
+  p.out_bf16 = static_cast<__nv_bfloat16*>(g.out_bf16);
+  p.acc_out = g.acc_out;
+  p.acc_f32 = g.acc_f32;
+  p.W = g.W;
+  p.packed = g.packed;
+  p.m = g.m;
+  p.v = g.v;
+  p.dW_out = g.dW_out;
+  p.changed = g.changed;
+  p.uc = g.uc;
+  p.pc = philox_call_consts(g.uc);
+  p.uc_dev = g.uc_dev;
+  p.split = g.split;
+  p.scale1 = g.scale1;
+  p.uc1 = g.uc1;
+  p.pc1 = philox_call_consts(g.uc1);
+  p.img_next = g.kind == GEMM_DW ? static_cast<__nv_bfloat16*>(g.img_next) : nullptr;
+  p.img8_next = g.kind == GEMM_DW ? static_cast<uint8_t*>(g.img8_next) : nullptr;
+  p.img8_split = p.img8_next && g.img8_split ? 1 : 0;
+  p.a_wrap = g.kind == GEMM_FWD8 ? g.a_wrap : 0;
+  if ((p.img_next || p.img8_next) && (g.packed || !g.W)) return 1;
+  return 0;
+}
+
 int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
   Params p{};
   p.M = g.M;
@@ -1586,32 +1669,8 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
     p.splits = (p.num_kb + p.kb_per_split - 1) / p.kb_per_split;
     p.slab = static_cast<long long>(g.M) * g.N;
   }
-  p.wait_ns = wait_limit_ns();
-  p.status = status_word();
-  if (!p.status) return 3;
-  p.s_x = g.s_x;
-  p.scale = g.scale;
-  p.out_bf16 = static_cast<__nv_bfloat16*>(g.out_bf16);
-  p.acc_out = g.acc_out;
-  p.acc_f32 = g.acc_f32;
-  p.W = g.W;
-  p.packed = g.packed;
-  p.m = g.m;
-  p.v = g.v;
-  p.dW_out = g.dW_out;
-  p.changed = g.changed;
-  p.uc = g.uc;
-  p.pc = philox_call_consts(g.uc);
-  p.uc_dev = g.uc_dev;
-  p.split = g.split;
-  p.scale1 = g.scale1;
-  p.uc1 = g.uc1;
-  p.pc1 = philox_call_consts(g.uc1);
-  p.img_next = g.kind == GEMM_DW ? static_cast<__nv_bfloat16*>(g.img_next) : nullptr;
-  p.img8_next = g.kind == GEMM_DW ? static_cast<uint8_t*>(g.img8_next) : nullptr;
-  p.img8_split = p.img8_next && g.img8_split ? 1 : 0;
-  p.a_wrap = g.kind == GEMM_FWD8 ? g.a_wrap : 0;
-  if ((p.img_next || p.img8_next) && (g.packed || !g.W)) return 1;
+  const int rc = fill_common(g, p);
+  if (rc) return rc;
   // stacked weights: whole tiles (multiples of 256 of either tiling),
   // constants in the parameter space
   if (g.split > 0 && (g.split % 256 != 0 || g.uc_dev ||
@@ -1718,6 +1777,72 @@ int launch_gemm(const GemmLaunch& g, cudaStream_t stream) {
     }
   }
   return 1;
+}
+
+int launch_dw_group(const GemmLaunch& g0, const GemmLaunch& g1, cudaStream_t stream) {
+  if (g0.kind != GEMM_DW || g1.kind != GEMM_DW || g0.Kred != g1.Kred) return 1;
+  Params p[2];
+  CUtensorMap ta[2], tb[2];
+  for (int i = 0; i < 2; ++i) {
+    const GemmLaunch& g = i ? g1 : g0;
+    if (g.packed || !g.W || !g.m || !g.v || g.uc_dev) return 1;
+    if (g.split > 0 && (g.split % 256 != 0 || g.split >= g.M)) return 1;
+    Params& q = p[i];
+    q = Params{};
+    q.M = g.M;
+    q.N = g.N;
+    q.Kred = g.Kred;
+    q.num_kb = (g.Kred + BK - 1) / BK;
+    q.chunk_kb = q.num_kb;
+    q.splits = 1;
+    q.kb_per_split = q.num_kb;
+    q.slab = 0;
+    const int rc = fill_common(g, q);
+    if (rc) return rc;
+    pair_tiling(q, true);
+    // whole tiles only: the two problems' tiles fill the waves together
+    q.full_units = q.num_tiles;
+    q.full_tiles = q.num_tiles;
+    q.tail_tiles = 0;
+    q.tail_splits = 1;
+    q.tail_kbps = q.num_kb;
+    q.part = nullptr;
+    if (!make_map(&ta[i], g.A, g.M, g.Kred, 64, BK)) return 3;
+    if (!make_map(&tb[i], g.B, g.N, g.Kred, 64, BK)) return 3;
+  }
+  auto kern = gemm_dw_group_kernel;
+  const int smem = SmemPair<GEMM_DW, false>::BYTES;
+  constexpr int threads = PairCfg<GEMM_DW, false>::THREADS;
+  static int max_clusters = 0;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(threads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (max_clusters == 0) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+        cudaSuccess)
+      return 3;
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    cfg.gridDim = dim3(sms, 1, 1);
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n < 1) return 3;
+    max_clusters = n;
+  }
+  const int total = p[0].num_tiles + p[1].num_tiles;
+  const int clusters = total < max_clusters ? total : max_clusters;
+  cfg.gridDim = dim3(2 * clusters, 1, 1);
+  if (cudaLaunchKernelEx(&cfg, kern, ta[0], tb[0], p[0], ta[1], tb[1], p[1]) != cudaSuccess)
+    return 3;
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : 3;
 }
 
 }  // namespace dqt

@@ -37,7 +37,7 @@ EXPORTED = [
     "dqt_bwd_dw_img_workspace_size", "dqt_codes_to_xdq", "dqt_fwd_workspace_size",
     "dqt_fwd_img_workspace_size", "dqt_bwd_dx_img_workspace_size",
     "dqt_bitlinear_fwd_img_pair", "dqt_bitlinear_bwd_dw_update_img_pair",
-    "dqt_bitlinear_bwd_dx_img_ld",
+    "dqt_bitlinear_bwd_dx_img_ld", "dqt_bitlinear_bwd_dw_update_group",
 ]
 
 
@@ -59,6 +59,14 @@ class dqt_adamw_t(C.Structure):
 class dqt_sr_t(C.Structure):
     _fields_ = [("seed", C.c_uint64), ("tensor_id", C.c_uint32), ("round_mode", C.c_int32),
                 ("elem0", C.c_int64)]
+
+
+class dqt_dw_problem_t(C.Structure):
+    _fields_ = [("dY", C.c_void_p), ("Xdq", C.c_void_p), ("W", C.c_void_p), ("m", C.c_void_p),
+                ("v", C.c_void_p), ("N", C.c_int64), ("K", C.c_int64), ("N0", C.c_int64),
+                ("s_w0", C.c_float), ("s_w1", C.c_float), ("sr0", C.POINTER(dqt_sr_t)),
+                ("sr1", C.POINTER(dqt_sr_t)), ("W_img_next", C.c_void_p), ("W8_next", C.c_void_p),
+                ("changed_out", C.c_void_p)]
 
 
 class dqt_adafactor_t(C.Structure):
@@ -107,6 +115,8 @@ def lib():
             _vp, _vp, _vp, _i64, _f32, _f32, _vp, _vp, C.POINTER(dqt_adamw_t),
             C.POINTER(dqt_sr_t), C.POINTER(dqt_sr_t), dqt_grid_t, _i64, _i64, _i64, _vp, _vp,
             _vp, _vp, _vp, _sz, _vp]
+        L.dqt_bitlinear_bwd_dw_update_group.argtypes = [
+            C.POINTER(dqt_dw_problem_t), C.c_int, C.POINTER(dqt_adamw_t), dqt_grid_t, _i64, _vp]
         L.dqt_fwd_img_workspace_size.argtypes = [_i64, _i64, _i64]
         L.dqt_fwd_img_workspace_size.restype = _sz
         L.dqt_bitlinear_bwd_dx.argtypes = [_vp, _vp, _f32, _i64, _i64, _i64, _vp, _vp, _sz, _vp]
@@ -598,6 +608,52 @@ def dqt_bitlinear_bwd_dw_update_img_pair(dY, Xdq, W, N0, s_w0, s_w1, m, v, hp, s
         _ptr(W_img_next), _ptr(W8_next), _ptr(changed_out), _ptr(ws), nws, _stream(stream)),
            "dqt_bitlinear_bwd_dw_update_img_pair")
     return W
+
+
+def dqt_bitlinear_bwd_dw_update_group(problems, hp, bits_or_grid, stream=None):
+    """Two weight-gradient + update problems over the same tokens in one
+    persistent launch.  `problems`: two dicts with dY, Xdq, W, m, v, s_w0 and
+    sr0, and optionally N0 (two stacked weights, with s_w1 and sr1),
+    W_img_next, W8_next and changed_out, as for
+    dqt_bitlinear_bwd_dw_update_img(_pair).  Results equal the two calls
+    made with ws=False."""
+    if len(problems) != 2:
+        raise ValueError("two problems")
+    arr = (dqt_dw_problem_t * 2)()
+    keep = []
+    T0 = None
+    split = fp8_split_grid(bits_or_grid)
+    for i, pr in enumerate(problems):
+        dY = _need(pr["dY"], "dY", torch.bfloat16)
+        T, N = dY.shape
+        Xdq = _need(pr["Xdq"], "Xdq", torch.bfloat16)
+        K = Xdq.shape[1]
+        _need(Xdq, "Xdq", torch.bfloat16, (T, K))
+        if T0 is not None and T != T0:
+            raise ValueError("the problems must share T")
+        T0 = T
+        _need(pr["W"], "W", torch.int8, (N, K))
+        _need(pr["m"], "m", torch.float32, (N, K))
+        _need(pr["v"], "v", torch.float32, (N, K))
+        _opt(pr.get("W_img_next"), "W_img_next", torch.bfloat16, (N, K))
+        _opt(pr.get("W8_next"), "W8_next", torch.uint8, (N, 2 * K if split else K))
+        _opt(pr.get("changed_out"), "changed_out", torch.int64, (1,))
+        sr0, sr1 = pr["sr0"], pr.get("sr1")
+        keep += [sr0, sr1]
+        a = arr[i]
+        a.dY, a.Xdq = dY.data_ptr(), Xdq.data_ptr()
+        a.W, a.m, a.v = pr["W"].data_ptr(), pr["m"].data_ptr(), pr["v"].data_ptr()
+        a.N, a.K, a.N0 = N, K, int(pr.get("N0", 0))
+        a.s_w0, a.s_w1 = float(pr["s_w0"]), float(pr.get("s_w1", 0.0))
+        a.sr0 = C.pointer(sr0)
+        a.sr1 = C.pointer(sr1) if sr1 is not None else None
+        for f in ("W_img_next", "W8_next", "changed_out"):
+            t = pr.get(f)
+            setattr(a, f, t.data_ptr() if t is not None else None)
+    _check(lib().dqt_bitlinear_bwd_dw_update_group(arr, 2, C.byref(hp), _grid(bits_or_grid), T0,
+                                                   _stream(stream)),
+           "dqt_bitlinear_bwd_dw_update_group")
+    del keep
 
 
 def dqt_sr_update(grad, W, s_w, m, v, hp, sr, bits_or_grid, changed_out=None, stream=None):

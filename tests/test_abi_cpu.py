@@ -282,3 +282,41 @@ def test_sr_stream_offset_validation(L):
     A = _p(0x10000)
     assert L.dqt_adafactor_apply(A, A, 0, A, A, A, 1, C.byref(sr), g, 8, 8, None,
                                  None) == dqt.DQT_ERR_ARG
+
+
+def test_dw_group_argument_validation(L):
+    """The grouped weight-gradient call checks both problems on the host
+    before it launches anything."""
+    g = dqt.dqt_grid_t(-1, 1)
+    hp = dqt.adamw()
+    sr = dqt.sr_stream()
+    a = 0x10000
+
+    def prob(N=512, K=256, N0=0, W=a, sr1=None, W8=None):
+        pr = dqt.dqt_dw_problem_t()
+        pr.dY, pr.Xdq, pr.W, pr.m, pr.v = a, a, W, a, a
+        pr.N, pr.K, pr.N0 = N, K, N0
+        pr.s_w0, pr.s_w1 = 1.0, 1.0
+        pr.sr0 = C.pointer(sr)
+        pr.sr1 = C.pointer(sr1) if sr1 is not None else None
+        pr.W8_next = W8
+        return pr
+
+    def call(p0, p1, n=2):
+        arr = (dqt.dqt_dw_problem_t * 2)(p0, p1)
+        return L.dqt_bitlinear_bwd_dw_update_group(arr, n, C.byref(hp), g, 4, None)
+
+    assert L.dqt_bitlinear_bwd_dw_update_group(None, 2, C.byref(hp), g, 4, None) == dqt.DQT_ERR_ARG
+    assert call(prob(), prob(), n=1) == dqt.DQT_ERR_ARG
+    assert call(prob(), prob(W=None)) == dqt.DQT_ERR_ARG             # no codes
+    assert call(prob(N0=256), prob()) == dqt.DQT_ERR_ARG             # stacked without sr1
+    assert call(prob(N0=200, sr1=sr), prob()) == dqt.DQT_ERR_ARG     # split not on a tile
+    assert call(prob(), prob(K=260)) == dqt.DQT_ERR_ALIGN            # K % 8
+    assert call(prob(), prob(W=a + 4)) == dqt.DQT_ERR_ALIGN          # 16-byte alignment
+    g8 = dqt.dqt_grid_t(-128, 127)
+    arr = (dqt.dqt_dw_problem_t * 2)(prob(K=264, W8=a), prob())
+    # the split E4M3 image of wide codes needs K % 16
+    assert L.dqt_bitlinear_bwd_dw_update_group(arr, 2, C.byref(hp), g8, 4, None) == dqt.DQT_ERR_ALIGN
+    bad = dqt.adamw(step=0)
+    arr = (dqt.dqt_dw_problem_t * 2)(prob(), prob())
+    assert L.dqt_bitlinear_bwd_dw_update_group(arr, 2, C.byref(bad), g, 4, None) == dqt.DQT_ERR_ARG

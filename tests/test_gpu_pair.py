@@ -310,3 +310,71 @@ def test_dw_update_pair_writes_next_split_e4m3_image(T, K, N0, N1):
     dqt.dqt_check_device_status()
     assert torch.equal(img8, dqt.dqt_codes_to_fp8_split(W))
     assert torch.equal(img.view(torch.int16), dqt.dqt_codes_to_bf16(W).view(torch.int16))
+
+
+def _state(N, K, seed):
+    m = inputs.normal((N, K), 1e-4, seed=seed).cuda()
+    v = inputs.normal((N, K), 1e-4, seed=seed + 1).abs().square().cuda()
+    return m, v
+
+
+# (T, K0, N0 split, N1 rest of the stacked problem, K1, N of the second
+# problem, bits): the LLaMA-MLP pair (gate + up stacked, and down) at 2048
+# tokens, and a ragged one (partial tiles in rows, columns and tokens)
+GROUP_CASES = [(2048, 2048, 5632, 5632, 5632, 2048, 1.58),
+               (2048, 2048, 5632, 5632, 5632, 2048, 8),
+               (300, 272, 256, 264, 264, 520, 1.58)]
+
+
+@pytest.mark.parametrize("T,K0,Na,Nb,K1,N1,bits", GROUP_CASES)
+def test_dw_update_group_equals_separate_calls(T, K0, Na, Nb, K1, N1, bits):
+    """One launch over both problems' tiles: codes, moments, next-step images
+    and changed counts equal the stacked call and the single call made
+    separately with whole tiles (ws=False), bit for bit."""
+    N0 = Na + Nb
+    c0, s0, s1, g = _weights(Na, Nb, K0, bits, seed=T + 1)
+    qmin, qmax = g
+    c1, s2, _ = oracle.absmean_init(inputs.normal((N1, K1), 0.02, seed=T + 5).numpy(), qmin, qmax)
+    s2 = float(s2)
+    X0 = inputs.normal((T, K0), 1.0, seed=T + 2, dtype=torch.bfloat16).cuda()
+    X1 = inputs.normal((T, K1), 1.0, seed=T + 3, dtype=torch.bfloat16).cuda()
+    dY0 = inputs.normal((T, N0), 1e-2, seed=T + 4, dtype=torch.bfloat16).cuda()
+    dY1 = inputs.normal((T, N1), 1e-2, seed=T + 6, dtype=torch.bfloat16).cuda()
+    _, _, _, Xd0 = dqt.dqt_act_quant_images(X0, want=("Xdq",))
+    _, _, _, Xd1 = dqt.dqt_act_quant_images(X1, want=("Xdq",))
+    m0, v0 = _state(N0, K0, T + 7)
+    m1, v1 = _state(N1, K1, T + 9)
+    hp = dqt.adamw(lr=1e-2, weight_decay=0.01, step=3)
+    sra, srb, src = dqt.sr_stream(seed=8), dqt.sr_stream(seed=8, tensor_id=1), dqt.sr_stream(seed=8, tensor_id=2)
+    w8 = 2 if dqt.fp8_split_grid(g) else 1
+    out = []
+    for grouped in (True, False):
+        W0, W1 = torch.from_numpy(c0).cuda(), torch.from_numpy(c1).cuda()
+        M0, V0, M1, V1 = m0.clone(), v0.clone(), m1.clone(), v1.clone()
+        i0 = torch.empty((N0, K0), dtype=torch.bfloat16, device="cuda")
+        i1 = torch.empty((N1, K1), dtype=torch.bfloat16, device="cuda")
+        e0 = torch.empty((N0, K0 * w8), dtype=torch.uint8, device="cuda")
+        e1 = torch.empty((N1, K1 * w8), dtype=torch.uint8, device="cuda")
+        ch = torch.zeros(2, dtype=torch.int64, device="cuda")
+        if grouped:
+            dqt.dqt_bitlinear_bwd_dw_update_group(
+                [dict(dY=dY0, Xdq=Xd0, W=W0, m=M0, v=V0, N0=Na, s_w0=s0, s_w1=s1, sr0=sra, sr1=srb,
+                      W_img_next=i0, W8_next=e0, changed_out=ch[0:1]),
+                 dict(dY=dY1, Xdq=Xd1, W=W1, m=M1, v=V1, s_w0=s2, sr0=src, W_img_next=i1,
+                      W8_next=e1, changed_out=ch[1:2])], hp, g)
+        else:
+            dqt.dqt_bitlinear_bwd_dw_update_img_pair(dY0, Xd0, W0, Na, s0, s1, M0, V0, hp, sra, srb, g,
+                                                     changed_out=ch[0:1], ws=False, W_img_next=i0,
+                                                     W8_next=e0)
+            dqt.dqt_bitlinear_bwd_dw_update_img(dY1, Xd1, W1, s2, M1, V1, hp, src, g,
+                                                changed_out=ch[1:2], ws=False, W_img_next=i1,
+                                                W8_next=e1)
+        dqt.dqt_check_device_status()
+        out.append([W0, W1, M0, V0, M1, V1, i0, i1, e0, e1, ch])
+    names = ["W0", "W1", "m0", "v0", "m1", "v1", "img0", "img1", "e4m3_0", "e4m3_1", "changed"]
+    for n, a, b in zip(names, out[0], out[1]):
+        a = a.view(torch.int16) if a.dtype == torch.bfloat16 else a
+        b = b.view(torch.int16) if b.dtype == torch.bfloat16 else b
+        assert torch.equal(a, b), n
+    assert int(out[0][-1][0]) > 0 and int(out[0][-1][1]) > 0
+    assert not torch.equal(out[0][0].cpu(), torch.from_numpy(c0))
