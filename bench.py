@@ -895,7 +895,9 @@ def run_gpu(args):
                 "traffic": ((DW_TRAFFIC_GROUP if st.group else
                              DW_TRAFFIC_STACKED if st.stack else DW_TRAFFIC_BYTES)
                             .get(kernel_fingerprint())
-                            if dom == "bwd_dw_update" and not st.packed else None),
+                            # (the FP8 step's update also writes E4M3 images:
+                            # not the captured traffic)
+                            if dom == "bwd_dw_update" and not st.packed and not st.fp8 else None),
                 "kernel_fingerprint": kernel_fingerprint(),
                 "algorithmic_per_launch": ("sum of 2*T*K*N FLOP over both problems of the one "
                                            "grouped launch (T=8192; gate and up stacked: K,N = "
